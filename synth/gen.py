@@ -1,0 +1,112 @@
+"""Seeded generators for synthetic weights and inputs.
+
+Both the CUDA path and the CPU oracle consume the tensors made here; this
+module only draws random numbers and stores them in the storage dtype.
+
+Reproducibility rules:
+  * one PCG64 stream per tensor, keyed (seed, model_id, layer, tensor slot);
+  * values are drawn in float64 and rounded once, round-to-nearest-even,
+    to the storage dtype (fp32, fp16, or bf16 kept as uint16 bit patterns);
+  * weights use seed 0, inputs seed 1 (request r of a stream: seed 1000*r+1).
+
+Initialisation per workload:
+  mlp6      W ~ N(0, 1/fan_in), b = 0
+  resnet50  conv W ~ N(0, 2/fan_in) with an inference BatchNorm folded in:
+            gamma ~ U(0.5, 1.5), beta ~ N(0, 0.1), mean ~ N(0, 0.1),
+            var ~ U(0.5, 1.5), eps = 1e-5; W' = W*g/sqrt(var+eps),
+            b' = beta - mean*g/sqrt(var+eps) (folded in float64, rounded once);
+            FC W ~ N(0, 1/fan_in), b ~ N(0, 0.01)
+  vgg16     W ~ N(0, 2/fan_in) (He) for ReLU layers, N(0, 1/fan_in) for the
+            last FC, b = 0
+  yolov3    W ~ N(0, 1/fan_in), b ~ N(0, 0.01)
+  inputs    N(0, 1)
+"""
+import numpy as np
+
+_NP_DTYPE = {"f32": np.float32, "f16": np.float16, "bf16": np.uint16}
+
+
+def _rng(*key):
+    return np.random.Generator(np.random.PCG64(np.random.SeedSequence(list(key))))
+
+
+def round_to_storage(x64, dtype):
+    """float64 array -> storage array (RNE, one rounding)."""
+    x64 = np.ascontiguousarray(x64, dtype=np.float64)
+    if dtype == "f32":
+        return x64.astype(np.float32)
+    if dtype == "f16":
+        return x64.astype(np.float16)
+    if dtype == "bf16":
+        # Round the float64 significand to 8 bits (RNE) by integer arithmetic
+        # on the bit pattern, then the value is exact in float32 and its top
+        # 16 bits are the bf16 pattern.
+        b = x64.view(np.uint64)
+        lsb = (b >> np.uint64(45)) & np.uint64(1)
+        b = (b + np.uint64((1 << 44) - 1) + lsb) & ~np.uint64((1 << 45) - 1)
+        f32 = b.view(np.float64).astype(np.float32)
+        return (f32.view(np.uint32) >> np.uint32(16)).astype(np.uint16)
+    raise ValueError(dtype)
+
+
+def _fan_in(layer):
+    if layer["op"] == "conv":
+        return layer["cin"] * layer["kh"] * layer["kw"]
+    return layer["k"]
+
+
+def layer_weights(model, li, seed=0):
+    """Parameter tensors of layer li as storage arrays ([] for weightless ops)."""
+    layer = model["layers"][li]
+    if layer["op"] not in ("conv", "linear"):
+        return []
+    dt, mid, name = model["dtype"], model["model_id"], model["name"]
+    fan = _fan_in(layer)
+    if layer["op"] == "conv":
+        wshape = (layer["cout"], layer["kh"], layer["kw"], layer["cin"])
+        nout = layer["cout"]
+    else:
+        wshape = (layer["n"], layer["k"])
+        nout = layer["n"]
+    rw, rb = _rng(seed, mid, li, 0), _rng(seed, mid, li, 1)
+    if name == "mlp6":
+        w = rw.normal(0.0, np.sqrt(1.0 / fan), wshape)
+        b = np.zeros(nout)
+    elif name == "resnet50":
+        if layer["op"] == "conv":
+            w = rw.normal(0.0, np.sqrt(2.0 / fan), wshape)
+            gamma = rb.uniform(0.5, 1.5, nout)
+            beta = rb.normal(0.0, 0.1, nout)
+            mean = rb.normal(0.0, 0.1, nout)
+            var = rb.uniform(0.5, 1.5, nout)
+            scale = gamma / np.sqrt(var + 1e-5)
+            w = w * scale[:, None, None, None]
+            b = beta - mean * scale
+        else:
+            w = rw.normal(0.0, np.sqrt(1.0 / fan), wshape)
+            b = rb.normal(0.0, 0.01, nout)
+    elif name == "vgg16":
+        gain = 2.0 if layer["act"] == "relu" else 1.0
+        w = rw.normal(0.0, np.sqrt(gain / fan), wshape)
+        b = np.zeros(nout)
+    elif name == "yolov3":
+        w = rw.normal(0.0, np.sqrt(1.0 / fan), wshape)
+        b = rb.normal(0.0, 0.01, nout)
+    else:
+        raise ValueError(name)
+    return [round_to_storage(w, dt), round_to_storage(b, dt)]
+
+
+def model_weights(model, seed=0):
+    """List (per layer) of lists of storage arrays."""
+    return [layer_weights(model, li, seed) for li in range(len(model["layers"]))]
+
+
+def model_input(model, seed=1, request=0):
+    """Model input, NHWC storage array, N(0, 1)."""
+    r = _rng(seed + 1000 * request, model["model_id"], 0xFFFF, 0)
+    return round_to_storage(r.normal(0.0, 1.0, model["input"]), model["dtype"])
+
+
+def storage_nbytes(dtype):
+    return np.dtype(_NP_DTYPE[dtype]).itemsize

@@ -1,0 +1,207 @@
+"""Pins of the partitioning oracle: the paper's printed block counts and
+Eq. 1 example, closed forms of the pipeline recurrence, an independent
+event simulation, and invariants of the workspace and unit splitting."""
+import itertools
+import os
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+from oracle import plan as P
+import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _golden_lines(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        return [l.split("#")[0].strip() for l in f if l.split("#")[0].strip()]
+
+
+def test_block_count_rule_matches_paper():
+    for line in _golden_lines("block_count.txt"):
+        s, b, m, n = (int(v) for v in line.split())
+        assert P.block_count_rule(s, b, m) == n
+
+
+def test_eq1_worked_example():
+    kv = dict(t.split("=") for t in _golden_lines("eq1_examples.txt")[0].split())
+    sumM, M = Fraction(kv["sumM"]), Fraction(kv["M"])
+    # proportional share of model i = M_i / sum M * M = (2/3) M_i
+    assert M / sumM == Fraction(kv["proportional_fraction"])
+    # With equal performance scores the second term is M/n each; the first
+    # term is (1 - 1/n) of the proportional share.
+    demands = [Fraction(1, 2), Fraction(1, 2), Fraction(1, 2)]
+    A = P.eq1_split(demands, [1, 1, 1], M)
+    assert sum(A) == M
+    assert A[0] == Fraction(2, 3) * demands[0] * Fraction(2, 3) + M / 9
+
+
+def test_eq1_selfdriving_budgets_consistent():
+    kv = dict(t.split("=") for t in _golden_lines("eq1_examples.txt")[1].split())
+    M = int(kv["M"])
+    sizes = [int(v) for v in kv["sizes"].split(",")]
+    budgets = [int(v) for v in kv["budgets"].split(",")]
+    assert sum(budgets) == M
+    n, S = len(sizes), sum(sizes)
+    first = [Fraction(s, S) * (1 - Fraction(1, n)) * M for s in sizes]
+    # every printed budget is at least its proportional term; the rest is the
+    # performance-score term, whose shares must sum to one
+    shares = [(b - f) / (Fraction(M) / n) for b, f in zip(budgets, first)]
+    assert all(0 <= s <= 1 for s in shares)
+    assert abs(float(sum(shares)) - 1.0) < 0.01
+    # Eq. 1 with those shares as performance scores gives the printed budgets
+    A = P.eq1_split(sizes, shares, M)
+    assert all(abs(float(a) - b) < 1.0 for a, b in zip(A, budgets))
+
+
+def test_eq1_within_budget_returns_demands():
+    assert P.eq1_split([3, 4], [1, 1], 10) == [3, 4]
+
+
+def _blocks(t_in, t_ex, t_out, n):
+    return [(0, t_in, t_ex, t_out)] * n
+
+
+@pytest.mark.parametrize("t_in,t_ex", [(5, 9), (9, 5), (7, 7), (1, 100), (100, 1)])
+@pytest.mark.parametrize("n", [1, 2, 3, 7])
+def test_pipeline_closed_forms(t_in, t_ex, n):
+    # two slots, free release: one copy ahead of execution
+    two = P.pipeline_time(_blocks(t_in, t_ex, 0, n), 2)
+    assert two == (t_in + n * t_ex if t_ex >= t_in else n * t_in + t_ex)
+    # one slot: strictly serial
+    assert P.pipeline_time(_blocks(t_in, t_ex, 0, n), 1) == n * (t_in + t_ex)
+
+
+def _simulate(blocks, slots):
+    """Event simulation with explicit resources: a copy engine, a compute
+    engine and `slots` arena slots, each with the time it becomes free."""
+    copy_free = comp_free = 0
+    slot_free = [0] * slots
+    prev_exec_end = 0
+    for k, (_, t_in, t_ex, t_out) in enumerate(blocks):
+        s = k % slots
+        start_copy = max(copy_free, slot_free[s])
+        copy_free = start_copy + t_in
+        start_exec = max(comp_free, copy_free, prev_exec_end)
+        comp_free = prev_exec_end = start_exec + t_ex
+        slot_free[s] = comp_free + t_out
+    return comp_free
+
+
+def test_pipeline_matches_event_simulation():
+    r = np.random.default_rng(0)
+    for _ in range(2000):
+        n = int(r.integers(1, 9))
+        blocks = [(0, int(r.integers(0, 50)), int(r.integers(0, 50)), int(r.integers(0, 20)))
+                  for _ in range(n)]
+        for slots in (1, 2):
+            assert P.pipeline_time(blocks, slots) == _simulate(blocks, slots)
+
+
+def test_eq4_hand_example():
+    # three blocks (t_in, t_ex, t_out): (4,3,1), (6,2,1), (5,8,2)
+    blocks = [(0, 4, 3, 1), (0, 6, 2, 1), (0, 5, 8, 2)]
+    # i=2: ov = (1 + 5) - (2 + 0) = 4 ; i=3: ov = (1 + 0) - (8 + 4) = -11
+    assert P.eq4_objective(blocks) == 4
+    assert P.eq4_objective(blocks[:1]) == 0
+
+
+def _uniform_model(nl, width, dtype="f16"):
+    layers = [dict(op="linear", src=[i - 1], k=width, n=width, act="relu", res=None, res_post=False)
+              for i in range(nl)]
+    return dict(name="u", model_id=50, dtype=dtype, input=(4, 1, 1, width), layers=layers,
+                outputs=[nl - 1])
+
+
+def test_workspace_mlp_is_two_buffers():
+    # the 6-layer MLP needs exactly two activation buffers (ping-pong)
+    m = synth.arch.mlp6()
+    ws, offs, ob, oo = P.workspace(m)
+    assert ws == 2 * 8 * 1024 * 4
+    assert sorted(set(offs.values())) == [0, 8 * 1024 * 4]
+    assert ob == 8 * 1024 * 4 and oo == {5: 0}
+
+
+@pytest.mark.parametrize("name", ["resnet50", "yolov3", "vgg16"])
+def test_workspace_no_live_overlap_and_first_fit(name):
+    m = synth.arch.MODELS[name]()
+    ws, offs, _, _ = P.workspace(m)
+    shapes = P.out_shapes(m)
+    es = P.ES[m["dtype"]]
+    nl = len(m["layers"])
+    last = list(range(nl))
+    for j, L in enumerate(m["layers"]):
+        for i in list(L["src"]) + ([L["res"]] if L.get("res") is not None else []):
+            if i >= 0:
+                last[i] = max(last[i], j)
+    size = {i: P.align(int(np.prod(shapes[i])) * es) for i in offs}
+    items = sorted(offs)
+    for a, b in itertools.combinations(items, 2):
+        live = a <= last[b] and b <= last[a]
+        if live:
+            assert offs[a] + size[a] <= offs[b] or offs[b] + size[b] <= offs[a]
+    assert ws == max(offs[i] + size[i] for i in items)
+    # first fit: no lower aligned offset was free when the tensor was placed
+    for i in items:
+        earlier = [j for j in items if j < i and j <= last[i] and i <= last[j]]
+        for o in range(0, offs[i], 256 * max(1, offs[i] // 256 // 64)):
+            clash = any(not (o + size[i] <= offs[j] or offs[j] + size[j] <= o) for j in earlier)
+            assert clash
+
+
+def test_units_split_vgg_fc1():
+    m = synth.arch.vgg16()
+    wb = P.weight_bytes(m)
+    budget = wb // 4 // 256 * 256
+    arena, slot, _ = P.arena_and_slot(m, budget, 2, False)
+    us = P.units(m, slot)
+    fc1 = [u for u in us if u["layer"] == 18]
+    assert len(fc1) > 1
+    assert sum(u["rows"] for u in fc1) == 4096
+    assert all(u["rows"] % 128 == 0 for u in fc1)
+    assert all(u["bytes"] <= slot for u in us)
+    assert [u["row0"] for u in fc1] == list(np.cumsum([0] + [u["rows"] for u in fc1[:-1]]))
+    assert sum(u["flops"] for u in fc1) == 2 * 25088 * 4096
+
+
+def test_units_infeasible_when_conv_too_large():
+    m = synth.arch.resnet50()
+    assert P.units(m, 1 << 20) is None
+
+
+def test_exhaustive_respects_rules():
+    r = np.random.default_rng(1)
+    coef = P.Coef(alpha_as=2_000_000, beta_ns=500, gamma_as=3000, eta_ns=50)
+    for _ in range(20):
+        nl = int(r.integers(2, 8))
+        m = _uniform_model(nl, 256)
+        s = P.weight_bytes(m)
+        budget = int(r.integers(s // nl * 2, s * 2 + 1))
+        res = P.exhaustive_partition(m, budget, coef)
+        if res is None:
+            assert P.units(m, budget // 2 // 256 * 256) is None or \
+                max(u["bytes"] for u in P.units(m, budget // 2 // 256 * 256)) > budget // 2
+            continue
+        # two blocks co-resident within the budget: n >= ceil(2 s / b)
+        assert res["n"] >= P.block_count_rule(s, budget)
+        # the optimum is no worse than every feasible alternative
+        for cuts in itertools.combinations(range(1, nl), res["n"] - 1):
+            v = P.evaluate_cuts(m, budget, coef, list(cuts))
+            assert v is None or v >= res["predicted_ns"]
+
+
+def test_rule_count_is_fewest_feasible_blocks():
+    # balanced layers: the fewest blocks of any feasible partition equals the
+    # paper's n = ceil(2 s / b); the exact objective may pick more blocks
+    # (a smaller first block shortens the pipeline fill)
+    coef = P.Coef(alpha_as=1000, beta_ns=100, gamma_as=100_000, eta_ns=0)
+    m = _uniform_model(6, 512)
+    s = P.weight_bytes(m)
+    for per_block in (1, 2, 3, 6):
+        budget = 2 * per_block * (s // 6)
+        fewest = min(len(c) + 1 for k in range(6) for c in itertools.combinations(range(1, 6), k)
+                     if P.evaluate_cuts(m, budget, coef, list(c)) is not None)
+        assert fewest == P.block_count_rule(s, budget) == 6 // per_block
+        assert P.exhaustive_partition(m, budget, coef)["n"] >= fewest
