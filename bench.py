@@ -1,0 +1,368 @@
+"""Benchmark of block-swapped inference on one GB300 (or N replicas).
+
+A step is one swapped inference of the workload: every block's weights are
+swapped from pinned host memory into the two-slot device arena and every
+layer runs from the arena.  Default workload: the ResNet-50-shaped CNN at
+batch 1 with a device budget of 40 % of its weight bytes.
+
+Reported (one JSON line, rank 0):
+  value        whole-job inferences/s (device-timed, inputs resident in HBM)
+  ms_per_step  swapped latency; dinf_ms the all-resident latency with the
+               same kernels; ratio = swapped / DInf
+  e2e          the same metric through swapnet_infer_host (host input and
+               output buffers, copies inside the timed region)
+  link         host-to-device bytes per swap-in over the swap time, against
+               the measured pinned cudaMemcpy peak
+  roofline     the dominant kernel's algorithmic FLOPs (or bytes) per launch
+               over its CUDA-event launch duration, against MEASURED_PEAKS.json
+  cpu_baseline the float64 CPU oracle on a bounded sample of the workload
+L2 is flushed (a 512 MiB write) before every timed step; the flush is not
+timed.  Replicas only: with torchrun each rank runs its own engine on its own
+GPU with no collective on the data path.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "swapped/DInf latency ratio and ms/inference at budget; host-link GB/s vs peak (1 GB300)"
+
+CONFIGS = {
+    # name: (builder, budget fraction of weight bytes, slots, activations in budget, workload text)
+    "resnet50": ("resnet50", dict(batch=1), 0.40,
+                 "ResNet-50-shaped CNN, fp16, batch 1, 1x3x224x224, budget 40% of weight bytes"),
+    "mlp6": ("mlp6", dict(batch=8), None,
+             "6-layer MLP width 1024 fp32 batch 8, budget = 2 layers of weights + 2 activation buffers"),
+    "vgg16_b1": ("vgg16", dict(batch=1), 0.25, "VGG-16-shaped CNN, fp16, batch 1, budget 25% of weight bytes"),
+    "vgg16_b16": ("vgg16", dict(batch=16), 0.25, "VGG-16-shaped CNN, fp16, batch 16, budget 25% of weight bytes"),
+}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return d["hbm_gbs"], d["bf16_tflops"], d.get("bf16_tflops_sustained"), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[4:8]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def cpu_oracle_baseline(model, weights, x, budget_s=12.0, max_runs=5):
+    """The float64 oracle as it stands, timed on the host cores on a bounded
+    sample (whole inferences until budget_s seconds of CPU work)."""
+    from oracle import forward as F
+    t0 = time.perf_counter()
+    runs = 0
+    while runs < max_runs:
+        F.forward(model, weights, x)
+        runs += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    dt = time.perf_counter() - t0
+    cores = len(os.sched_getaffinity(0))
+    return {"value": runs / dt, "unit": "inferences/s", "cores": cores, "kind": "oracle",
+            "sample": "%d whole float64 inference(s) of the same workload (numpy, BLAS threads = %d cores)"
+                      % (runs, cores)}
+
+
+def build_workload(name):
+    import synth
+    from oracle import plan as OP
+    arch, kw, frac, text = CONFIGS[name]
+    m = synth.arch.MODELS[arch](**kw)
+    w = synth.gen.model_weights(m)
+    x = synth.gen.model_input(m)
+    wb = OP.weight_bytes(m)
+    if frac is None:
+        budget = 8_462_336
+    else:
+        budget = int(wb * frac) // 256 * 256
+    return m, w, x, wb, budget, text
+
+
+def run_reference(args, rank, world):
+    """The reference arm: the CPU oracle, timed as it stands on the host cores."""
+    if rank != 0:
+        return
+    m, w, x, wb, budget, text = build_workload(args.config)
+    from oracle import forward as F
+    for _ in range(max(0, min(args.warmup, 1))):
+        F.forward(m, w, x)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        F.forward(m, w, x)
+        times.append(time.perf_counter() - t0)
+    ms = 1000.0 * sum(times) / len(times)
+    cores = len(os.sched_getaffinity(0))
+    val = 1000.0 / ms
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": val, "unit": "inferences/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": text, "budget_bytes": budget, "weight_bytes": wb, "l2": "n/a (CPU)"},
+        "cpu_baseline": {"value": val, "unit": "inferences/s", "cores": cores, "kind": "oracle",
+                         "sample": "one whole float64 inference per step"},
+        "e2e": {"value": val, "unit": "inferences/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="swapnet", choices=["swapnet", "reference"])
+    ap.add_argument("--config", default="resnet50", choices=sorted(CONFIGS))
+    ap.add_argument("--variant", default="auto", choices=["auto", "memcpy", "zerocopy"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+
+    import torch
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2401_16757_gb300 import capi
+
+    m, w, x, wb, budget, text = build_workload(args.config)
+    d = capi.Desc(m)
+    variant = {"auto": capi.SWAP_AUTO, "memcpy": capi.SWAP_MEMCPY, "zerocopy": capi.SWAP_ZEROCOPY}[args.variant]
+    if args.config == "mlp6":
+        opt = capi.options(slots=2, activations_in_budget=1, swap_variant=variant)
+    else:
+        opt = capi.options(swap_variant=variant)
+    plan = capi.Plan.partition(d, budget, opt)
+    rplan = capi.Plan.resident(d)
+    info = plan.info()
+    host = capi.HostWeights(w)
+    eng = capi.Engine(plan, host)
+    reng = capi.Engine(rplan, host)
+    stream = torch.cuda.current_stream()
+    sp = stream.cuda_stream
+    d_in = torch.empty(max(16, info["input_bytes"]), dtype=torch.uint8, device="cuda")
+    d_in[:info["input_bytes"]].copy_(torch.from_numpy(x.view(np.uint8).reshape(-1)))
+    d_out = torch.empty(info["output_bytes"], dtype=torch.uint8, device="cuda")
+    flush = torch.empty(512 << 20, dtype=torch.uint8, device="cuda")
+
+    def timed(engine, steps, flush_l2=True):
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+        for a, b in evs:
+            if flush_l2:
+                flush.zero_()
+            a.record(stream)
+            engine.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
+            b.record(stream)
+        torch.cuda.synchronize()
+        return [a.elapsed_time(b) for a, b in evs]
+
+    for _ in range(args.warmup):
+        eng.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
+        reng.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
+    eng.sync()
+    reng.sync()
+
+    # ---- timed region: swapped inference
+    clocks = ClockSampler(local)
+    clocks.start()
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    launches0 = eng.stats()["kernel_launches"]
+    t_wall0 = time.perf_counter()
+    ms_list = timed(eng, args.steps)
+    t_wall = time.perf_counter() - t_wall0
+    launches = eng.stats()["kernel_launches"] - launches0
+    if dist:
+        dist.barrier()
+    clk = clocks.stop()
+    eng.sync()
+    ms_swapped = sum(ms_list) / len(ms_list)
+    total_ms = sum(ms_list)
+    if dist:
+        t = torch.tensor([total_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    value = world * args.steps / (total_ms / 1000.0)
+
+    # ---- DInf: same kernels, weights resident
+    ms_dinf_list = timed(reng, args.steps)
+    ms_dinf = sum(ms_dinf_list) / len(ms_dinf_list)
+
+    # ---- e2e: host buffers through swapnet_infer_host
+    h_in = torch.empty(info["input_bytes"], dtype=torch.uint8, pin_memory=True)
+    h_in.copy_(torch.from_numpy(x.view(np.uint8).reshape(-1)))
+    h_out = torch.empty(info["output_bytes"], dtype=torch.uint8, pin_memory=True)
+    for _ in range(3):
+        eng.infer_host(h_in.data_ptr(), h_out.data_ptr(), sp)
+    torch.cuda.synchronize()
+    e2e_ms = []
+    for _ in range(args.steps):
+        flush.zero_()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        eng.infer_host(h_in.data_ptr(), h_out.data_ptr(), sp)
+        b.record(stream)
+        b.synchronize()
+        e2e_ms.append(a.elapsed_time(b))
+    e2e_val = 1000.0 / (sum(e2e_ms) / len(e2e_ms))
+
+    # ---- profiled pass: per-unit kernel and per-block swap times
+    units = plan.units()
+    blocks = plan.blocks()
+    kinds = eng.unit_kernels()
+    eng.set_profiling(True)
+    prof_steps = min(20, args.steps)
+    acc_u = np.zeros(len(units))
+    acc_s = np.zeros(len(blocks))
+    for _ in range(prof_steps):
+        flush.zero_()
+        eng.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
+        u_us, s_us = eng.last_times(len(units), len(blocks))
+        acc_u += np.array(u_us)
+        acc_s += np.array(s_us)
+    eng.set_profiling(False)
+    acc_u /= prof_steps
+    acc_s /= prof_steps
+    share = {}
+    for k, t in zip(kinds, acc_u):
+        share[k] = share.get(k, 0.0) + t
+    dom = max(share, key=share.get)
+    dom_idx = [i for i, k in enumerate(kinds) if k == dom]
+    dom_flops = sum(units[i]["flops"] for i in dom_idx)
+    dom_us = sum(acc_u[i] for i in dom_idx)
+    hbm, tf_burst, tf_sust, peak_src = load_peaks()
+    achieved_tf = dom_flops / (dom_us * 1e-6) / 1e12 if dom_us > 0 else 0.0
+    roofline = {"bound": "tensor", "kernel": dom, "launches_per_step": len(dom_idx),
+                "achieved": achieved_tf, "peak": tf_burst, "unit": "TFLOP/s",
+                "frac": achieved_tf / tf_burst, "peak_source": peak_src + " bf16 burst",
+                "traffic": None, "share_of_kernel_time": dom_us / max(1e-9, acc_u.sum()),
+                "kernel_time_share": {k: round(v / max(1e-9, acc_u.sum()), 4) for k, v in share.items()}}
+    if dom in ("skinny_linear", "maxpool", "gap", "upsample2x", "concat"):
+        roofline.update(bound="hbm", unit="GB/s", peak=hbm, peak_source=peak_src + " copy")
+
+    # ---- host link: bytes per swap over swap time, against pinned memcpy peak
+    swap_bytes = sum(b["bytes"] for b in blocks)
+    swap_us = float(acc_s.sum())
+    pk = torch.empty(256 << 20, dtype=torch.uint8, pin_memory=True)
+    dv = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    best = 1e9
+    for _ in range(5):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        dv.copy_(pk, non_blocking=True)
+        b.record(stream)
+        b.synchronize()
+        best = min(best, a.elapsed_time(b))
+    link_peak = (256 << 20) / (best / 1000.0) / 1e9
+    link_gbs = swap_bytes / (swap_us * 1e-6) / 1e9 if swap_us > 0 else None
+    # roofline of the whole step (slower of tensor FLOPs and swapped bytes over the link)
+    flops = sum(u["flops"] for u in units)
+    step_bound_ms = max(flops / (tf_burst * 1e12), swap_bytes / (link_peak * 1e9)) * 1e3
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        cpu = cpu_oracle_baseline(m, w, x)
+
+    if rank == 0:
+        eb = eng.blocks()
+        line = {
+            "metric": METRIC, "value": value, "unit": "inferences/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_swapped, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32" if m["dtype"] == "f32" else m["dtype"], "data": "synthetic",
+            "config": {"workload": text, "budget_bytes": budget, "weight_bytes": wb,
+                       "n_blocks": info["n_blocks"], "cuts": plan.cuts(), "slot_bytes": info["slot_bytes"],
+                       "workspace_bytes": info["workspace_bytes"], "l2": "flushed (512 MiB write) before each step",
+                       "swap_variants": [b["variant"] for b in eb], "parallelism": "replicas" if world > 1 else "1 GPU"},
+            "dinf_ms": ms_dinf, "ratio": ms_swapped / ms_dinf,
+            "p50_ms": statistics.median(ms_list), "p99_ms": float(np.percentile(ms_list, 99)),
+            "e2e": {"value": e2e_val, "unit": "inferences/s", "h2d_bytes_per_step": info["input_bytes"],
+                    "d2h_bytes_per_step": info["output_bytes"]},
+            "link": {"achieved_gbs": link_gbs, "peak_gbs": link_peak, "peak_source": "pinned cudaMemcpy H2D 256 MiB",
+                     "frac": (link_gbs / link_peak) if link_gbs else None, "bytes_per_step": swap_bytes},
+            "step_roofline": {"bound_ms": step_bound_ms, "frac": step_bound_ms / ms_swapped},
+            "roofline": roofline,
+            "gpu_launches": launches,
+            "clocks": clk,
+            "cpu_baseline": cpu,
+            "wall_s_timed": t_wall,
+        }
+        print(json.dumps(line))
+    if dist:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,303 @@
+/*
+ * swapnet.h — C ABI of libswapnet: block-swapped DNN inference under a
+ * device-memory budget on one GPU (SwapNet, arXiv 2401.16757).
+ *
+ * The problem the calls solve is the paper's (Sec. 3 "Basic Idea", Sec.
+ * 6.2.2 "Partition Blocks within DNN"): given a memory budget b for a model
+ * of size s > b, cut the layer sequence into n blocks and execute them in
+ * order, swapping each block's parameters into device memory before it runs
+ * and releasing them after.  Sec. 6.2.2 ("Allocate Memory Budget across
+ * DNNs", Eq. 1) shares one budget among several models.
+ *
+ * Conventions for every call:
+ *   - Status: int, SWAPNET_OK (0) on success, a negative swapnet_status
+ *     otherwise.  No C++ exception crosses this boundary.  Output handles
+ *     and output arrays are written only on success.  swapnet_last_error()
+ *     returns a message for the calling thread's most recent failure.
+ *   - Ownership: plans and engines are opaque, library-owned and freed with
+ *     swapnet_plan_free / swapnet_engine_free.  Host weight buffers, model
+ *     descriptors, and caller-provided device buffers stay caller-owned.
+ *   - Layout: activations are NHWC in the model's storage dtype; conv
+ *     weights are [cout][kh][kw][cin]; linear weights are [out][in]; a
+ *     linear layer flattens its input per batch item in (h, w, c) order.
+ *   - Threads: a plan is immutable after creation and may be shared; an
+ *     engine is used by one host thread at a time.
+ */
+#ifndef SWAPNET_H
+#define SWAPNET_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ------------------------------------------------------------------ status */
+typedef enum swapnet_status {
+  SWAPNET_OK = 0,
+  SWAPNET_ERR_INVALID_ARG = -1, /* malformed descriptor, option or argument */
+  SWAPNET_ERR_INFEASIBLE = -2,  /* no partition fits the budget            */
+  SWAPNET_ERR_OOM = -3,         /* host or device allocation failed        */
+  SWAPNET_ERR_CUDA = -4,        /* a CUDA runtime/driver call failed       */
+  SWAPNET_ERR_TIMEOUT = -5,     /* a bounded device-side wait gave up      */
+  SWAPNET_ERR_MISALIGNED = -6,  /* a pointer or size breaks an alignment rule */
+  SWAPNET_ERR_UNSUPPORTED = -7  /* shape/dtype combination not implemented */
+} swapnet_status;
+
+/* ------------------------------------------------------------ descriptors */
+typedef enum swapnet_dtype { SWAPNET_F32 = 0, SWAPNET_F16 = 1, SWAPNET_BF16 = 2 } swapnet_dtype;
+
+typedef enum swapnet_op {
+  SWAPNET_OP_LINEAR = 1,     /* y[m,o] = act(sum_i x[m,i] W[o,i] + b[o] (+res)) */
+  SWAPNET_OP_CONV2D = 2,     /* zero-padded 2-D convolution, + bias (+res), act  */
+  SWAPNET_OP_MAXPOOL = 3,    /* window max; padding never wins                  */
+  SWAPNET_OP_GAP = 4,        /* global average over H and W                     */
+  SWAPNET_OP_UPSAMPLE2X = 5, /* nearest neighbour, factor 2 in H and W          */
+  SWAPNET_OP_CONCAT = 6      /* channels of src0 followed by channels of src1   */
+} swapnet_op;
+
+typedef enum swapnet_act { SWAPNET_ACT_NONE = 0, SWAPNET_ACT_RELU = 1, SWAPNET_ACT_LEAKY = 2 } swapnet_act;
+
+#define SWAPNET_SRC_INPUT (-1) /* the model input                       */
+#define SWAPNET_SRC_NONE (-2)  /* unused producer / no residual operand */
+
+/* One layer of the model information table (Sec. 6.1, Table 2: per layer
+ * size, parameter depth and FLOPs — derived here from the shapes).  Layers
+ * are listed in execution order; producers precede consumers. */
+typedef struct swapnet_layer {
+  int32_t op;       /* swapnet_op                                             */
+  int32_t src0;     /* producer of the input (layer index or SWAPNET_SRC_INPUT) */
+  int32_t src1;     /* second input of CONCAT, else SWAPNET_SRC_NONE           */
+  int32_t res;      /* residual operand (layer index) or SWAPNET_SRC_NONE      */
+  int32_t act;      /* swapnet_act                                             */
+  int32_t res_post; /* 0: act(acc + b + res); 1: act(acc + b) + res            */
+  int32_t cin;      /* conv: input channels;  linear: input features            */
+  int32_t cout;     /* conv: output channels; linear: output features           */
+  int32_t kh, kw, stride, pad; /* conv and maxpool window                      */
+  int32_t is_output;/* nonzero: a model output, written to the output buffer   */
+  int32_t reserved;
+  int64_t t_ex_ns;  /* measured execution delay; 0 = gamma * FLOPs (Sec. 6.1)  */
+} swapnet_layer;
+
+/* Parameter tensors of a layer, in this order, are what swapnet_load's
+ * host_weights lists: CONV2D and LINEAR have two (weights, bias); the other
+ * ops none.  Model outputs are written to the output buffer in increasing
+ * layer order, each at a 256-byte aligned offset. */
+typedef struct swapnet_model_desc {
+  int32_t dtype;    /* swapnet_dtype of weights and activations          */
+  int32_t n_layers;
+  const swapnet_layer* layers;
+  int32_t in_n, in_h, in_w, in_c; /* model input, NHWC (a matrix is n x 1 x 1 x c) */
+} swapnet_model_desc;
+
+typedef enum swapnet_swap_variant {
+  SWAPNET_SWAP_AUTO = 0,     /* pick per block by measured time at load        */
+  SWAPNET_SWAP_MEMCPY = 1,   /* copy engine: cudaMemcpyAsync from pinned memory */
+  SWAPNET_SWAP_ZEROCOPY = 2  /* SM kernel reading mapped host memory           */
+} swapnet_swap_variant;
+
+/* Options.  Delay coefficients follow Sec. 6.1: t_in = alpha*s + beta*d,
+ * t_ex = gamma*f, t_out = eta*d, in integer units (attoseconds per byte or
+ * FLOP; nanoseconds per tensor). */
+typedef struct swapnet_options {
+  int32_t slots;                 /* arena slots: 2 (swap overlaps compute) or 1 */
+  int32_t activations_in_budget; /* 1: the budget also covers the activation workspace */
+  int32_t swap_variant;          /* swapnet_swap_variant                         */
+  int32_t objective;             /* 0: m-slot pipeline completion; 1: Eq. 4 sum  */
+  uint64_t alpha_as_per_byte;
+  uint64_t beta_ns_per_tensor;
+  uint64_t gamma_as_per_flop;
+  uint64_t eta_ns_per_tensor;
+  int32_t zc_ctas;               /* CTAs of the zero-copy swap kernel, 0 = default */
+  int32_t reserved[7];
+} swapnet_options;
+
+/* Fills the defaults: 2 slots, activations outside the budget, AUTO swap,
+ * pipeline objective, alpha = 2.5e6 as/B (400 GB/s), beta = 2000 ns,
+ * gamma = 2000 as/FLOP (500 TFLOP/s), eta = 0. */
+void swapnet_default_options(swapnet_options* opt);
+
+/* ------------------------------------------------------------------ plans */
+typedef struct swapnet_plan swapnet_plan;
+
+typedef struct swapnet_plan_info {
+  uint32_t n_blocks;
+  uint32_t n_units;        /* layers, with oversize linear layers split      */
+  uint32_t slots;          /* 0 for a resident (all weights in HBM) plan     */
+  uint32_t n_layers;
+  uint64_t budget_bytes;
+  uint64_t arena_bytes;    /* device bytes for weights                       */
+  uint64_t slot_bytes;     /* capacity of one slot                           */
+  uint64_t workspace_bytes;/* intermediate activations (liveness-planned)    */
+  uint64_t input_bytes;    /* model input                                    */
+  uint64_t output_bytes;   /* all model outputs, 256-byte aligned each       */
+  uint64_t weight_bytes;   /* sum of 256-aligned parameter tensor sizes      */
+  uint64_t plan_bytes;     /* host bytes of the plan (the resident skeleton) */
+  int64_t predicted_ns;    /* objective value of the chosen partition        */
+} swapnet_plan_info;
+
+typedef struct swapnet_unit_info {
+  int32_t layer;   /* layer index                                            */
+  int32_t row0;    /* first output feature (linear pieces), else 0           */
+  int32_t rows;    /* output features in this unit (linear), else 0          */
+  int32_t depth;   /* parameter tensors                                      */
+  uint64_t bytes;  /* 256-aligned parameter bytes                            */
+  uint64_t flops;
+  int64_t t_ex_ns;
+} swapnet_unit_info;
+
+typedef struct swapnet_block_info {
+  uint32_t unit0, unit1; /* units [unit0, unit1)                             */
+  uint32_t slot;         /* arena slot the block is swapped into             */
+  uint32_t depth;
+  uint64_t bytes;
+  int64_t t_in_ns, t_ex_ns, t_out_ns;
+} swapnet_block_info;
+
+/* Partition the model for a budget (Sec. 6.2.2, Eq. 2-3; objective per
+ * opt->objective).  Every block must fit one slot of floor(arena/slots)
+ * bytes (arena = budget, minus the workspace when activations_in_budget).
+ * A linear layer larger than a slot is split along output features into
+ * pieces of a multiple of 128 features.  Ties: fewer blocks, then the
+ * lexicographically smallest cut vector.  Host only; no device work.
+ * Errors: INVALID_ARG (descriptor/options), INFEASIBLE (no partition). */
+int swapnet_partition(const swapnet_model_desc* desc, uint64_t budget_bytes,
+                      const swapnet_options* opt /* nullable: defaults */,
+                      swapnet_plan** out_plan);
+
+/* Build a plan from explicit cut points (Sec. 6.2.2 "create_blocks"): cut c
+ * places a block boundary before unit c; cuts strictly increasing in
+ * [1, n_units).  Units are computed for the budget as in swapnet_partition.
+ * Errors: INVALID_ARG (bad cuts), INFEASIBLE (a block exceeds a slot). */
+int swapnet_plan_from_cuts(const swapnet_model_desc* desc, const uint32_t* cuts, uint32_t n_cuts,
+                           uint64_t budget_bytes, const swapnet_options* opt,
+                           swapnet_plan** out_plan);
+
+/* The sufficient-memory reference (DInf): one block holding every weight,
+ * loaded once and kept resident; the same kernels run the same units. */
+int swapnet_plan_resident(const swapnet_model_desc* desc, const swapnet_options* opt,
+                          swapnet_plan** out_plan);
+
+int swapnet_plan_info_get(const swapnet_plan* plan, swapnet_plan_info* info);
+/* Copy up to `cap` entries; return the number available in *n (nullable). */
+int swapnet_plan_cuts(const swapnet_plan* plan, uint32_t* cuts, uint32_t cap, uint32_t* n);
+int swapnet_plan_units(const swapnet_plan* plan, swapnet_unit_info* units, uint32_t cap, uint32_t* n);
+int swapnet_plan_blocks(const swapnet_plan* plan, swapnet_block_info* blocks, uint32_t cap, uint32_t* n);
+/* Byte offset of each model output inside the output buffer (in layer order). */
+int swapnet_plan_output_offsets(const swapnet_plan* plan, uint64_t* offs, uint32_t cap, uint32_t* n);
+void swapnet_plan_free(swapnet_plan* plan);
+
+/* Multi-DNN budget split (Sec. 6.2.2, Eq. 1): with demands M_i (weight
+ * bytes) and performance scores PS_i = u_i * latency_i / M_i (latency_i =
+ * predicted all-resident latency), model i receives
+ *   A_i = M_i/sum(M) (1 - 1/n) M + PS_i/sum(PS) (1/n) M,
+ * floored to 256 bytes, when sum(M) > M (else A_i = M_i); each model is
+ * then partitioned for A_i.  budgets_out[n] and plans_out[n] are written on
+ * success only; the caller frees each plan. */
+int swapnet_schedule(const swapnet_model_desc* const* models, const float* urgency, uint32_t n,
+                     uint64_t arena_bytes, const swapnet_options* opt,
+                     uint64_t* budgets_out, swapnet_plan** plans_out);
+
+/* ---------------------------------------------------------------- engines */
+typedef struct swapnet_engine swapnet_engine;
+typedef struct CUstream_st* swapnet_stream; /* a cudaStream_t; NULL = legacy default stream */
+
+/* Bind a plan to host weights and device memory (Sec. 4.2 zero-copy
+ * swap-in, Sec. 5.2 assembly by reference).
+ *   host_weights: n_tensors pointers, one per parameter tensor in layer
+ *     order; caller-owned, must outlive the engine and must not change.
+ *     They are page-locked and mapped in place (cudaHostRegister), never
+ *     copied on the host; memory already pinned by CUDA is used as is.
+ *   d_arena: device buffer of >= arena_bytes for the weight slots, 256-byte
+ *     aligned; NULL = the library allocates it.  d_workspace likewise for
+ *     the activation workspace.
+ * The plan is copied; it may be freed after this call.  Creates a copy
+ * stream and per-slot events; resolves every layer's parameter address to
+ * slot base + offset and builds its TMA descriptors once (the skeleton).
+ * With SWAPNET_SWAP_AUTO it times both swap variants per block and keeps
+ * the faster.  A resident plan copies all weights to the arena here.
+ * Errors: INVALID_ARG, MISALIGNED, OOM, CUDA, UNSUPPORTED. */
+int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint32_t n_tensors,
+                 void* d_arena, uint64_t arena_bytes, void* d_workspace, uint64_t workspace_bytes,
+                 swapnet_engine** out_engine);
+
+/* One inference, asynchronous on `stream` (Sec. 4.3, Sec. 6.2.2 with m
+ * slots): block k is swapped into slot k mod m on the engine's copy stream
+ * once the slot's previous block has finished executing, and its layers run
+ * on `stream` once the swap is done; block k+1's swap overlaps block k's
+ * execution.  d_input / d_output are device pointers of input_bytes and
+ * output_bytes (plan info), 16-byte aligned.  Device faults surface at the
+ * next synchronising call; bounded device waits report through
+ * swapnet_engine_sync.  Errors: INVALID_ARG, MISALIGNED, CUDA. */
+int swapnet_infer(swapnet_engine* eng, const void* d_input, void* d_output, swapnet_stream stream);
+
+/* As swapnet_infer, from and to host buffers: the input is copied to an
+ * engine-owned device buffer and the outputs back, all on `stream` (copies
+ * are asynchronous when the host buffers are pinned).  The host output is
+ * valid after the stream has been synchronised. */
+int swapnet_infer_host(swapnet_engine* eng, const void* h_input, void* h_output, swapnet_stream stream);
+
+/* Waits for the engine's streams; returns TIMEOUT if a kernel's bounded
+ * wait gave up since the last call (the error word is then cleared), CUDA
+ * on a device error. */
+int swapnet_engine_sync(swapnet_engine* eng);
+
+typedef struct swapnet_engine_block {
+  int32_t variant;       /* swapnet_swap_variant chosen for the block     */
+  int32_t n_segments;    /* contiguous host->arena copies per swap-in     */
+  float memcpy_us;       /* measured at load (AUTO), else 0               */
+  float zerocopy_us;
+} swapnet_engine_block;
+
+int swapnet_engine_blocks(const swapnet_engine* eng, swapnet_engine_block* blocks, uint32_t cap,
+                          uint32_t* n);
+/* Counters since load (kernel launches include the layer kernels and the
+ * zero-copy swap kernels the engine launched; memcpy_calls counts copy-engine
+ * transfers). */
+typedef struct swapnet_engine_stats {
+  uint64_t infer_calls;
+  uint64_t kernel_launches;
+  uint64_t memcpy_calls;
+  uint64_t bytes_swapped;
+} swapnet_engine_stats;
+int swapnet_engine_stats_get(const swapnet_engine* eng, swapnet_engine_stats* stats);
+
+/* Kernel family that runs each unit. */
+typedef enum swapnet_kernel_kind {
+  SWAPNET_KERNEL_TC_GEMM = 1,     /* tcgen05 GEMM, A and B by TMA             */
+  SWAPNET_KERNEL_TC_CONV = 2,     /* tcgen05 implicit-GEMM conv (A gathered)  */
+  SWAPNET_KERNEL_SKINNY = 3,      /* SIMT linear, <= 16 rows                  */
+  SWAPNET_KERNEL_DIRECT_CONV = 4, /* SIMT direct convolution                  */
+  SWAPNET_KERNEL_MAXPOOL = 5,
+  SWAPNET_KERNEL_GAP = 6,
+  SWAPNET_KERNEL_UPSAMPLE = 7,
+  SWAPNET_KERNEL_CONCAT = 8
+} swapnet_kernel_kind;
+int swapnet_engine_unit_kernels(const swapnet_engine* eng, int32_t* kinds, uint32_t cap, uint32_t* n);
+
+/* Device timing for measurement: while enabled, every swapnet_infer records
+ * a CUDA event pair around each unit's kernel (on the inference stream) and
+ * around each block's swap-in (on the copy stream).  The events add a small
+ * gap between launches; leave profiling off for latency measurements.
+ * swapnet_engine_last_times synchronises and returns, for the most recent
+ * profiled inference, microseconds per unit and per block swap-in. */
+int swapnet_engine_set_profiling(swapnet_engine* eng, int enable);
+int swapnet_engine_last_times(swapnet_engine* eng, float* unit_us, uint32_t n_units, float* swap_us,
+                              uint32_t n_blocks);
+
+void swapnet_engine_free(swapnet_engine* eng);
+
+/* ------------------------------------------------------------------- misc */
+const char* swapnet_strerror(int status);
+const char* swapnet_last_error(void);
+
+/* Host-side fault injection for tests: the next `count` calls of the named
+ * step fail as if the CUDA call had failed.  what: 1 = cudaHostRegister,
+ * 2 = device allocation, 3 = event/stream creation.  count 0 disarms. */
+int swapnet_debug_fail_next(int what, int count);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SWAPNET_H */

@@ -1,0 +1,350 @@
+"""ctypes binding of libswapnet (include/swapnet.h): argument marshalling only.
+
+Every step of the inference path runs in the library's CUDA kernels; this
+module converts Python descriptions to the C structs, calls the C entry
+points and raises SwapnetError on a non-zero status.  It fails loudly when
+the shared library is missing.
+"""
+import ctypes as C
+import os
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libswapnet.so")
+
+OK, ERR_INVALID_ARG, ERR_INFEASIBLE, ERR_OOM, ERR_CUDA, ERR_TIMEOUT, ERR_MISALIGNED, ERR_UNSUPPORTED = \
+    0, -1, -2, -3, -4, -5, -6, -7
+F32, F16, BF16 = 0, 1, 2
+OP = {"linear": 1, "conv": 2, "maxpool": 3, "gap": 4, "upsample2x": 5, "concat": 6}
+ACT = {"none": 0, "relu": 1, "leaky": 2}
+DTYPE = {"f32": F32, "f16": F16, "bf16": BF16}
+SWAP_AUTO, SWAP_MEMCPY, SWAP_ZEROCOPY = 0, 1, 2
+SRC_INPUT, SRC_NONE = -1, -2
+
+
+class Layer(C.Structure):
+    _fields_ = [("op", C.c_int32), ("src0", C.c_int32), ("src1", C.c_int32), ("res", C.c_int32),
+                ("act", C.c_int32), ("res_post", C.c_int32), ("cin", C.c_int32), ("cout", C.c_int32),
+                ("kh", C.c_int32), ("kw", C.c_int32), ("stride", C.c_int32), ("pad", C.c_int32),
+                ("is_output", C.c_int32), ("reserved", C.c_int32), ("t_ex_ns", C.c_int64)]
+
+
+class ModelDesc(C.Structure):
+    _fields_ = [("dtype", C.c_int32), ("n_layers", C.c_int32), ("layers", C.POINTER(Layer)),
+                ("in_n", C.c_int32), ("in_h", C.c_int32), ("in_w", C.c_int32), ("in_c", C.c_int32)]
+
+
+class Options(C.Structure):
+    _fields_ = [("slots", C.c_int32), ("activations_in_budget", C.c_int32), ("swap_variant", C.c_int32),
+                ("objective", C.c_int32), ("alpha_as_per_byte", C.c_uint64), ("beta_ns_per_tensor", C.c_uint64),
+                ("gamma_as_per_flop", C.c_uint64), ("eta_ns_per_tensor", C.c_uint64), ("zc_ctas", C.c_int32),
+                ("reserved", C.c_int32 * 7)]
+
+
+class PlanInfo(C.Structure):
+    _fields_ = [("n_blocks", C.c_uint32), ("n_units", C.c_uint32), ("slots", C.c_uint32),
+                ("n_layers", C.c_uint32), ("budget_bytes", C.c_uint64), ("arena_bytes", C.c_uint64),
+                ("slot_bytes", C.c_uint64), ("workspace_bytes", C.c_uint64), ("input_bytes", C.c_uint64),
+                ("output_bytes", C.c_uint64), ("weight_bytes", C.c_uint64), ("plan_bytes", C.c_uint64),
+                ("predicted_ns", C.c_int64)]
+
+
+class UnitInfo(C.Structure):
+    _fields_ = [("layer", C.c_int32), ("row0", C.c_int32), ("rows", C.c_int32), ("depth", C.c_int32),
+                ("bytes", C.c_uint64), ("flops", C.c_uint64), ("t_ex_ns", C.c_int64)]
+
+
+class BlockInfo(C.Structure):
+    _fields_ = [("unit0", C.c_uint32), ("unit1", C.c_uint32), ("slot", C.c_uint32), ("depth", C.c_uint32),
+                ("bytes", C.c_uint64), ("t_in_ns", C.c_int64), ("t_ex_ns", C.c_int64), ("t_out_ns", C.c_int64)]
+
+
+class EngineStats(C.Structure):
+    _fields_ = [("infer_calls", C.c_uint64), ("kernel_launches", C.c_uint64), ("memcpy_calls", C.c_uint64),
+                ("bytes_swapped", C.c_uint64)]
+
+
+KERNEL_KIND = {1: "tc_gemm", 2: "tc_conv", 3: "skinny_linear", 4: "direct_conv", 5: "maxpool", 6: "gap",
+               7: "upsample2x", 8: "concat"}
+
+
+class EngineBlock(C.Structure):
+    _fields_ = [("variant", C.c_int32), ("n_segments", C.c_int32), ("memcpy_us", C.c_float),
+                ("zerocopy_us", C.c_float)]
+
+
+EXPORTS = ["swapnet_default_options", "swapnet_partition", "swapnet_plan_from_cuts", "swapnet_plan_resident",
+           "swapnet_plan_info_get", "swapnet_plan_cuts", "swapnet_plan_units", "swapnet_plan_blocks",
+           "swapnet_plan_output_offsets", "swapnet_plan_free", "swapnet_schedule", "swapnet_load",
+           "swapnet_infer", "swapnet_infer_host", "swapnet_engine_sync", "swapnet_engine_blocks",
+           "swapnet_engine_free", "swapnet_engine_stats_get", "swapnet_engine_unit_kernels",
+           "swapnet_engine_set_profiling", "swapnet_engine_last_times", "swapnet_strerror", "swapnet_last_error", "swapnet_debug_fail_next"]
+
+_lib = None
+
+
+class SwapnetError(RuntimeError):
+    def __init__(self, code, what):
+        self.code = code
+        super().__init__("%s: %s (%d): %s" % (what, lib().swapnet_strerror(code).decode(), code,
+                                               lib().swapnet_last_error().decode()))
+
+
+def lib():
+    """The loaded libswapnet (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise ImportError("libswapnet.so is not built: run __graft_entry__.build() or "
+                          "python paper_2401_16757_gb300/build.py")
+    L = C.CDLL(LIB_PATH)
+    P = C.c_void_p
+    sig = {
+        "swapnet_default_options": (None, [C.POINTER(Options)]),
+        "swapnet_partition": (C.c_int, [C.POINTER(ModelDesc), C.c_uint64, C.POINTER(Options), C.POINTER(P)]),
+        "swapnet_plan_from_cuts": (C.c_int, [C.POINTER(ModelDesc), C.POINTER(C.c_uint32), C.c_uint32, C.c_uint64,
+                                             C.POINTER(Options), C.POINTER(P)]),
+        "swapnet_plan_resident": (C.c_int, [C.POINTER(ModelDesc), C.POINTER(Options), C.POINTER(P)]),
+        "swapnet_plan_info_get": (C.c_int, [P, C.POINTER(PlanInfo)]),
+        "swapnet_plan_cuts": (C.c_int, [P, C.POINTER(C.c_uint32), C.c_uint32, C.POINTER(C.c_uint32)]),
+        "swapnet_plan_units": (C.c_int, [P, C.POINTER(UnitInfo), C.c_uint32, C.POINTER(C.c_uint32)]),
+        "swapnet_plan_blocks": (C.c_int, [P, C.POINTER(BlockInfo), C.c_uint32, C.POINTER(C.c_uint32)]),
+        "swapnet_plan_output_offsets": (C.c_int, [P, C.POINTER(C.c_uint64), C.c_uint32, C.POINTER(C.c_uint32)]),
+        "swapnet_plan_free": (None, [P]),
+        "swapnet_schedule": (C.c_int, [C.POINTER(C.POINTER(ModelDesc)), C.POINTER(C.c_float), C.c_uint32,
+                                       C.c_uint64, C.POINTER(Options), C.POINTER(C.c_uint64), C.POINTER(P)]),
+        "swapnet_load": (C.c_int, [P, C.POINTER(P), C.c_uint32, P, C.c_uint64, P, C.c_uint64, C.POINTER(P)]),
+        "swapnet_infer": (C.c_int, [P, P, P, P]),
+        "swapnet_infer_host": (C.c_int, [P, P, P, P]),
+        "swapnet_engine_sync": (C.c_int, [P]),
+        "swapnet_engine_blocks": (C.c_int, [P, C.POINTER(EngineBlock), C.c_uint32, C.POINTER(C.c_uint32)]),
+        "swapnet_engine_free": (None, [P]),
+        "swapnet_engine_stats_get": (C.c_int, [P, C.POINTER(EngineStats)]),
+        "swapnet_engine_unit_kernels": (C.c_int, [P, C.POINTER(C.c_int32), C.c_uint32, C.POINTER(C.c_uint32)]),
+        "swapnet_engine_set_profiling": (C.c_int, [P, C.c_int]),
+        "swapnet_engine_last_times": (C.c_int, [P, C.POINTER(C.c_float), C.c_uint32, C.POINTER(C.c_float),
+                                                C.c_uint32]),
+        "swapnet_strerror": (C.c_char_p, [C.c_int]),
+        "swapnet_last_error": (C.c_char_p, []),
+        "swapnet_debug_fail_next": (C.c_int, [C.c_int, C.c_int]),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(L, name)
+        f.restype, f.argtypes = res, args
+    _lib = L
+    return L
+
+
+def check(rc, what):
+    if rc != OK:
+        raise SwapnetError(rc, what)
+
+
+# ------------------------------------------------------------------ options
+def options(**kw):
+    o = Options()
+    lib().swapnet_default_options(C.byref(o))
+    for k, v in kw.items():
+        if not hasattr(o, k):
+            raise KeyError(k)
+        setattr(o, k, v)
+    return o
+
+
+# ------------------------------------------------------------ descriptors
+class Desc:
+    """A C model descriptor built from a layer-sequence dict (see synth.arch)."""
+
+    def __init__(self, model, t_ex_ns=None):
+        layers = model["layers"]
+        arr = (Layer * len(layers))()
+        outs = set(model["outputs"])
+        for i, L in enumerate(layers):
+            c = arr[i]
+            c.op = OP[L["op"]]
+            c.src0 = L["src"][0]
+            c.src1 = L["src"][1] if len(L["src"]) > 1 else SRC_NONE
+            c.res = SRC_NONE if L.get("res") is None else L["res"]
+            c.act = ACT[L.get("act", "none")]
+            c.res_post = 1 if L.get("res_post") else 0
+            if L["op"] == "conv":
+                c.cin, c.cout, c.kh, c.kw, c.stride, c.pad = L["cin"], L["cout"], L["kh"], L["kw"], L["stride"], L["pad"]
+            elif L["op"] == "linear":
+                c.cin, c.cout = L["k"], L["n"]
+            elif L["op"] == "maxpool":
+                c.kh, c.kw, c.stride, c.pad = L["kh"], L["kw"], L["stride"], L["pad"]
+            c.is_output = 1 if i in outs else 0
+            c.t_ex_ns = 0 if t_ex_ns is None else int(t_ex_ns[i])
+        n, h, w, ch = model["input"]
+        self.layers = arr
+        self.c = ModelDesc(DTYPE[model["dtype"]], len(layers), arr, n, h, w, ch)
+        self.model = model
+
+
+class Plan:
+    def __init__(self, handle):
+        self.h = C.c_void_p(handle)
+
+    @staticmethod
+    def partition(desc, budget, opt=None):
+        h = C.c_void_p()
+        check(lib().swapnet_partition(C.byref(desc.c), budget, C.byref(opt) if opt else None, C.byref(h)),
+              "swapnet_partition")
+        return Plan(h.value)
+
+    @staticmethod
+    def from_cuts(desc, cuts, budget, opt=None):
+        h = C.c_void_p()
+        arr = (C.c_uint32 * max(1, len(cuts)))(*cuts)
+        check(lib().swapnet_plan_from_cuts(C.byref(desc.c), arr, len(cuts), budget,
+                                           C.byref(opt) if opt else None, C.byref(h)), "swapnet_plan_from_cuts")
+        return Plan(h.value)
+
+    @staticmethod
+    def resident(desc, opt=None):
+        h = C.c_void_p()
+        check(lib().swapnet_plan_resident(C.byref(desc.c), C.byref(opt) if opt else None, C.byref(h)),
+              "swapnet_plan_resident")
+        return Plan(h.value)
+
+    def info(self):
+        i = PlanInfo()
+        check(lib().swapnet_plan_info_get(self.h, C.byref(i)), "swapnet_plan_info_get")
+        return {f: getattr(i, f) for f, _ in PlanInfo._fields_}
+
+    def cuts(self):
+        n = C.c_uint32()
+        check(lib().swapnet_plan_cuts(self.h, None, 0, C.byref(n)), "swapnet_plan_cuts")
+        arr = (C.c_uint32 * max(1, n.value))()
+        check(lib().swapnet_plan_cuts(self.h, arr, n.value, None), "swapnet_plan_cuts")
+        return list(arr[:n.value])
+
+    def units(self):
+        n = C.c_uint32()
+        check(lib().swapnet_plan_units(self.h, None, 0, C.byref(n)), "swapnet_plan_units")
+        arr = (UnitInfo * max(1, n.value))()
+        check(lib().swapnet_plan_units(self.h, arr, n.value, None), "swapnet_plan_units")
+        return [{f: getattr(u, f) for f, _ in UnitInfo._fields_} for u in arr[:n.value]]
+
+    def blocks(self):
+        n = C.c_uint32()
+        check(lib().swapnet_plan_blocks(self.h, None, 0, C.byref(n)), "swapnet_plan_blocks")
+        arr = (BlockInfo * max(1, n.value))()
+        check(lib().swapnet_plan_blocks(self.h, arr, n.value, None), "swapnet_plan_blocks")
+        return [{f: getattr(b, f) for f, _ in BlockInfo._fields_} for b in arr[:n.value]]
+
+    def output_offsets(self):
+        n = C.c_uint32()
+        check(lib().swapnet_plan_output_offsets(self.h, None, 0, C.byref(n)), "swapnet_plan_output_offsets")
+        arr = (C.c_uint64 * max(1, n.value))()
+        check(lib().swapnet_plan_output_offsets(self.h, arr, n.value, None), "swapnet_plan_output_offsets")
+        return list(arr[:n.value])
+
+    def free(self):
+        if self.h and self.h.value:
+            lib().swapnet_plan_free(self.h)
+            self.h = C.c_void_p()
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+
+def schedule(descs, urgency, arena_bytes, opt=None):
+    n = len(descs)
+    ptrs = (C.POINTER(ModelDesc) * n)(*[C.pointer(d.c) for d in descs])
+    urg = (C.c_float * n)(*urgency)
+    budgets = (C.c_uint64 * n)()
+    plans = (C.c_void_p * n)()
+    check(lib().swapnet_schedule(ptrs, urg, n, arena_bytes, C.byref(opt) if opt else None, budgets, plans),
+          "swapnet_schedule")
+    return list(budgets), [Plan(p) for p in plans]
+
+
+# ------------------------------------------------------------ host weights
+class HostWeights:
+    """All parameter tensors of a model packed in one page-aligned host
+    buffer, each tensor at a 256-byte aligned offset in layer order (the
+    layout of the arena slots, so a block's tensors are one contiguous
+    range)."""
+
+    def __init__(self, weights):
+        flat = [np.ascontiguousarray(t) for lw in weights for t in lw]
+        offs, cur = [], 0
+        for t in flat:
+            offs.append(cur)
+            cur += (t.nbytes + 255) // 256 * 256
+        page = os.sysconf("SC_PAGE_SIZE")
+        raw = np.empty(cur + 2 * page, dtype=np.uint8)
+        start = (-raw.ctypes.data) % page
+        self.buf = raw[start:start + cur]
+        self._raw = raw
+        for t, o in zip(flat, offs):
+            self.buf[o:o + t.nbytes] = t.view(np.uint8).reshape(-1)
+        base = self.buf.ctypes.data
+        self.ptrs = (C.c_void_p * max(1, len(flat)))(*[base + o for o in offs])
+        self.n = len(flat)
+        self.nbytes = cur
+
+
+class Engine:
+    def __init__(self, plan, host, d_arena=0, arena_bytes=0, d_ws=0, ws_bytes=0):
+        self.host = host  # keep the host buffer alive
+        h = C.c_void_p()
+        check(lib().swapnet_load(plan.h, host.ptrs, host.n, C.c_void_p(d_arena or None), arena_bytes,
+                                 C.c_void_p(d_ws or None), ws_bytes, C.byref(h)), "swapnet_load")
+        self.h = h
+
+    def infer(self, d_in, d_out, stream=0):
+        check(lib().swapnet_infer(self.h, C.c_void_p(d_in), C.c_void_p(d_out), C.c_void_p(stream or None)),
+              "swapnet_infer")
+
+    def infer_host(self, h_in, h_out, stream=0):
+        check(lib().swapnet_infer_host(self.h, C.c_void_p(h_in), C.c_void_p(h_out), C.c_void_p(stream or None)),
+              "swapnet_infer_host")
+
+    def sync(self):
+        check(lib().swapnet_engine_sync(self.h), "swapnet_engine_sync")
+
+    def blocks(self):
+        n = C.c_uint32()
+        check(lib().swapnet_engine_blocks(self.h, None, 0, C.byref(n)), "swapnet_engine_blocks")
+        arr = (EngineBlock * max(1, n.value))()
+        check(lib().swapnet_engine_blocks(self.h, arr, n.value, None), "swapnet_engine_blocks")
+        return [{f: getattr(b, f) for f, _ in EngineBlock._fields_} for b in arr[:n.value]]
+
+    def stats(self):
+        st = EngineStats()
+        check(lib().swapnet_engine_stats_get(self.h, C.byref(st)), "swapnet_engine_stats_get")
+        return {f: getattr(st, f) for f, _ in EngineStats._fields_}
+
+    def unit_kernels(self):
+        n = C.c_uint32()
+        check(lib().swapnet_engine_unit_kernels(self.h, None, 0, C.byref(n)), "swapnet_engine_unit_kernels")
+        arr = (C.c_int32 * max(1, n.value))()
+        check(lib().swapnet_engine_unit_kernels(self.h, arr, n.value, None), "swapnet_engine_unit_kernels")
+        return [KERNEL_KIND.get(k, str(k)) for k in arr[:n.value]]
+
+    def set_profiling(self, enable):
+        check(lib().swapnet_engine_set_profiling(self.h, 1 if enable else 0), "swapnet_engine_set_profiling")
+
+    def last_times(self, n_units, n_blocks):
+        u = (C.c_float * max(1, n_units))()
+        b = (C.c_float * max(1, n_blocks))()
+        check(lib().swapnet_engine_last_times(self.h, u, n_units, b, n_blocks), "swapnet_engine_last_times")
+        return list(u[:n_units]), list(b[:n_blocks])
+
+    def free(self):
+        if self.h and self.h.value:
+            lib().swapnet_engine_free(self.h)
+            self.h = C.c_void_p()
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass

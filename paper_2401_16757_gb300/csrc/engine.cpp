@@ -1,0 +1,636 @@
+// Engine: binds a plan to host weights and device memory, and runs the
+// block pipeline (Sec. 4 swapping, Sec. 5 assembly by reference, Sec. 6.2.2
+// with m = slots blocks co-resident).
+#include <cuda_runtime.h>
+#include <unistd.h>
+
+#include <algorithm>
+#include <cstring>
+#include <map>
+#include <memory>
+#include <mutex>
+#include <new>
+#include <utility>
+
+#include "internal.h"
+#include "kernels.h"
+
+namespace swapnet {
+
+int g_fail_next[4] = {0, 0, 0, 0};
+
+// Host ranges this library page-locked, shared by every engine that uses
+// them: (base, length) -> number of engines.  A range is unregistered when
+// its last engine is freed.
+static std::mutex g_reg_mu;
+static std::map<std::pair<uintptr_t, size_t>, int> g_reg;
+
+static void unregister_range(uintptr_t base, size_t len) {
+  std::lock_guard<std::mutex> lk(g_reg_mu);
+  auto it = g_reg.find({base, len});
+  if (it == g_reg.end()) return;
+  if (--it->second == 0) {
+    cudaHostUnregister(reinterpret_cast<void*>(base));
+    g_reg.erase(it);
+  }
+}
+
+static bool injected(int what) {
+  if (what < 1 || what > 3 || g_fail_next[what] <= 0) return false;
+  --g_fail_next[what];
+  return true;
+}
+
+#define CU(call, what)                                                                         \
+  do {                                                                                         \
+    cudaError_t e_ = (call);                                                                   \
+    if (e_ != cudaSuccess) {                                                                   \
+      set_error(std::string(what) + ": " + cudaGetErrorString(e_));                          \
+      return SWAPNET_ERR_CUDA;                                                                 \
+    }                                                                                          \
+  } while (0)
+
+struct Segment {
+  const char* src;  // device alias of host memory
+  char* dst;
+  uint64_t bytes;
+};
+
+struct EngBlock {
+  std::vector<Segment> segs;
+  int variant = SWAPNET_SWAP_MEMCPY;
+  float memcpy_us = 0.f, zerocopy_us = 0.f;
+};
+
+struct UnitExec {
+  const void* w = nullptr;
+  const void* b = nullptr;
+  bool use_tc = false;
+  TcGemm g{};
+  TcPlan tc{};
+  const void* tmA_for = nullptr;  // A pointer the TMA map was encoded for
+};
+
+struct HostRange {
+  uintptr_t base;
+  size_t len;
+  bool registered_by_us;
+  char* dev;
+};
+
+}  // namespace swapnet
+
+using namespace swapnet;
+
+struct swapnet_engine {
+  swapnet_plan plan;
+  int device = 0;
+  int num_sms = 0;
+  char* d_arena = nullptr;
+  bool own_arena = false;
+  char* d_ws = nullptr;
+  bool own_ws = false;
+  char* d_in_stage = nullptr;
+  char* d_out_stage = nullptr;
+  std::vector<HostRange> ranges;
+  std::vector<const char*> tensor_dev;  // device alias per tensor
+  cudaStream_t copy = nullptr;
+  cudaEvent_t slot_free[2] = {nullptr, nullptr};
+  cudaEvent_t ready[2] = {nullptr, nullptr};
+  std::vector<EngBlock> blocks;
+  std::vector<UnitExec> ux;
+  int* err_word = nullptr;
+  int zc_ctas = 32;
+  bool weights_loaded = false;  // resident plan: copied once at load
+  std::vector<int> unit_kind;   // swapnet_kernel_kind per unit
+  swapnet_engine_stats stats{};
+  bool profiling = false;
+  std::vector<cudaEvent_t> ev_unit;  // 2 per unit
+  std::vector<cudaEvent_t> ev_swap;  // 2 per block
+};
+
+namespace swapnet {
+
+static int release(swapnet_engine* e) {
+  if (!e) return SWAPNET_OK;
+  cudaSetDevice(e->device);
+  if (e->copy) cudaStreamSynchronize(e->copy);
+  for (cudaEvent_t ev : {e->slot_free[0], e->slot_free[1], e->ready[0], e->ready[1]})
+    if (ev) cudaEventDestroy(ev);
+  for (cudaEvent_t ev : e->ev_unit) cudaEventDestroy(ev);
+  for (cudaEvent_t ev : e->ev_swap) cudaEventDestroy(ev);
+  if (e->copy) cudaStreamDestroy(e->copy);
+  if (e->own_arena && e->d_arena) cudaFree(e->d_arena);
+  if (e->own_ws && e->d_ws) cudaFree(e->d_ws);
+  if (e->d_in_stage) cudaFree(e->d_in_stage);
+  if (e->d_out_stage) cudaFree(e->d_out_stage);
+  for (const HostRange& r : e->ranges)
+    if (r.registered_by_us) unregister_range(r.base, r.len);
+  delete e;
+  return SWAPNET_OK;
+}
+
+// Page-lock and map the caller's weight buffers in place; record the device
+// alias of every tensor.
+static int register_host(swapnet_engine* e, const void* const* hw, uint32_t nt) {
+  const Model& m = e->plan.model;
+  const uintptr_t page = (uintptr_t)sysconf(_SC_PAGESIZE);
+  struct R { uintptr_t lo, hi; };
+  std::vector<R> rs;
+  for (uint32_t t = 0; t < nt; ++t) {
+    if (!hw[t]) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null host weight pointer");
+    const uintptr_t p = reinterpret_cast<uintptr_t>(hw[t]);
+    if (m.tensor_raw[t] == 0) continue;
+    rs.push_back(R{p / page * page, (p + m.tensor_raw[t] + page - 1) / page * page});
+  }
+  std::sort(rs.begin(), rs.end(), [](const R& a, const R& b) { return a.lo < b.lo; });
+  std::vector<R> merged;
+  for (const R& r : rs) {
+    if (!merged.empty() && r.lo <= merged.back().hi) merged.back().hi = std::max(merged.back().hi, r.hi);
+    else merged.push_back(r);
+  }
+  for (const R& r : merged) {
+    HostRange hr{r.lo, (size_t)(r.hi - r.lo), false, nullptr};
+    void* base = reinterpret_cast<void*>(r.lo);
+    std::lock_guard<std::mutex> lk(g_reg_mu);
+    auto it = g_reg.find({hr.base, hr.len});
+    if (it != g_reg.end()) {
+      ++it->second;
+      hr.registered_by_us = true;
+      e->ranges.push_back(hr);
+      continue;
+    }
+    cudaError_t err = injected(1) ? cudaErrorMemoryAllocation
+                                  : cudaHostRegister(base, hr.len, cudaHostRegisterMapped | cudaHostRegisterReadOnly);
+    if (err == cudaErrorNotSupported || err == cudaErrorInvalidValue) {
+      cudaGetLastError();
+      err = cudaHostRegister(base, hr.len, cudaHostRegisterMapped);
+    }
+    if (err == cudaSuccess) {
+      hr.registered_by_us = true;
+      g_reg[{hr.base, hr.len}] = 1;
+    } else if (err == cudaErrorHostMemoryAlreadyRegistered) {
+      cudaGetLastError();  // pinned by its owner (e.g. cudaHostAlloc): used as is
+    } else {
+      cudaGetLastError();
+      set_error(std::string("cudaHostRegister: ") + cudaGetErrorString(err));
+      return SWAPNET_ERR_CUDA;  // ranges registered so far are released with the engine
+    }
+    e->ranges.push_back(hr);
+  }
+  e->tensor_dev.assign(nt, nullptr);
+  for (uint32_t t = 0; t < nt; ++t) {
+    if (m.tensor_raw[t] == 0) continue;
+    void* dptr = nullptr;
+    cudaError_t err = cudaHostGetDevicePointer(&dptr, const_cast<void*>(hw[t]), 0);
+    if (err != cudaSuccess || !dptr) {
+      cudaGetLastError();
+      SN_FAIL(SWAPNET_ERR_CUDA, std::string("cudaHostGetDevicePointer: ") + cudaGetErrorString(err));
+    }
+    e->tensor_dev[t] = static_cast<const char*>(dptr);
+  }
+  return SWAPNET_OK;
+}
+
+static char* slot_base(swapnet_engine* e, int slot) { return e->d_arena + (uint64_t)slot * e->plan.slot; }
+
+static void build_segments(swapnet_engine* e) {
+  const swapnet_plan& p = e->plan;
+  e->blocks.assign(p.blocks.size(), EngBlock{});
+  for (size_t k = 0; k < p.blocks.size(); ++k) {
+    const Block& B = p.blocks[k];
+    std::vector<Segment>& segs = e->blocks[k].segs;
+    char* base = slot_base(e, B.slot);
+    for (int u = B.u0; u < B.u1; ++u) {
+      const Unit& U = p.units[u];
+      for (int t = 0; t < U.nt; ++t) {
+        if (U.tlen[t] == 0) continue;
+        Segment s{e->tensor_dev[U.tidx[t]] + U.toff[t], base + U.slot_off[t], U.tlen[t]};
+        if (!segs.empty()) {
+          Segment& q = segs.back();
+          // coalesce when host and slot offsets advance together
+          if (s.src > q.src && s.dst > q.dst && (uint64_t)(s.src - q.src) == (uint64_t)(s.dst - q.dst) &&
+              (uint64_t)(s.dst - q.dst) <= align_up(q.bytes)) {
+            q.bytes = (uint64_t)(s.dst - q.dst) + s.bytes;
+            continue;
+          }
+        }
+        segs.push_back(s);
+      }
+    }
+  }
+}
+
+static int swap_block(swapnet_engine* e, size_t k, int variant, cudaStream_t s) {
+  const EngBlock& b = e->blocks[k];
+  if (variant == SWAPNET_SWAP_ZEROCOPY) {
+    std::vector<ZcSeg> z;
+    z.reserve(b.segs.size());
+    for (const Segment& g : b.segs) {
+      z.push_back(ZcSeg{g.src, g.dst, g.bytes});
+      e->stats.bytes_swapped += g.bytes;
+    }
+    e->stats.kernel_launches += (z.size() + 47) / 48;
+    return launch_zerocopy(z.data(), (int)z.size(), e->zc_ctas, s);
+  }
+  for (const Segment& g : b.segs) {
+    CU(cudaMemcpyAsync(g.dst, g.src, g.bytes, cudaMemcpyDefault, s), "swap-in copy");
+    e->stats.bytes_swapped += g.bytes;
+    e->stats.memcpy_calls += 1;
+  }
+  return SWAPNET_OK;
+}
+
+static bool zerocopy_ok(const EngBlock& b) {
+  for (const Segment& g : b.segs)
+    if (((uintptr_t)g.src | (uintptr_t)g.dst) & 15) return false;
+  return true;
+}
+
+// Time both swap variants per block (best of 3 each) and keep the faster.
+static int calibrate(swapnet_engine* e) {
+  cudaEvent_t a, b;
+  CU(cudaEventCreate(&a), "event");
+  CU(cudaEventCreate(&b), "event");
+  int rc = SWAPNET_OK;
+  for (size_t k = 0; k < e->blocks.size() && rc == SWAPNET_OK; ++k) {
+    EngBlock& B = e->blocks[k];
+    float best[3] = {1e30f, 1e30f, 1e30f};
+    for (int v : {SWAPNET_SWAP_MEMCPY, SWAPNET_SWAP_ZEROCOPY}) {
+      if (v == SWAPNET_SWAP_ZEROCOPY && !zerocopy_ok(B)) continue;
+      for (int rep = 0; rep < 3 && rc == SWAPNET_OK; ++rep) {
+        cudaEventRecord(a, e->copy);
+        rc = swap_block(e, k, v, e->copy);
+        cudaEventRecord(b, e->copy);
+        if (cudaEventSynchronize(b) != cudaSuccess) { rc = SWAPNET_ERR_CUDA; break; }
+        float ms = 0;
+        cudaEventElapsedTime(&ms, a, b);
+        best[v] = std::min(best[v], ms * 1000.f);
+      }
+    }
+    B.memcpy_us = best[SWAPNET_SWAP_MEMCPY];
+    B.zerocopy_us = best[SWAPNET_SWAP_ZEROCOPY] < 1e29f ? best[SWAPNET_SWAP_ZEROCOPY] : 0.f;
+    B.variant = (B.zerocopy_us > 0.f && B.zerocopy_us < B.memcpy_us) ? SWAPNET_SWAP_ZEROCOPY : SWAPNET_SWAP_MEMCPY;
+  }
+  cudaEventDestroy(a);
+  cudaEventDestroy(b);
+  return rc;
+}
+
+static const char* act_ptr(const swapnet_engine* e, int src, const void* din, const void* dout) {
+  if (src == SWAPNET_SRC_INPUT) return static_cast<const char*>(din);
+  const Layer& L = e->plan.model.L[src];
+  if (L.out_off >= 0) return static_cast<const char*>(dout) + L.out_off;
+  return e->d_ws + L.ws_off;
+}
+
+static char* out_ptr(const swapnet_engine* e, int li, void* dout) {
+  const Layer& L = e->plan.model.L[li];
+  if (L.out_off >= 0) return static_cast<char*>(dout) + L.out_off;
+  return e->d_ws + L.ws_off;
+}
+
+// Fill the GEMM description of a unit for the given activation pointers.
+static bool unit_gemm(const swapnet_engine* e, const Unit& U, const UnitExec& X, const char* x, const char* r,
+                      char* y, TcGemm* g) {
+  const Model& m = e->plan.model;
+  const Layer& L = m.L[U.layer];
+  const int es = m.es;
+  std::memset(g, 0, sizeof(*g));
+  g->dtype = m.dtype;
+  g->W = X.w;
+  g->e.bias = X.b;
+  g->e.act = L.d.act;
+  g->e.res_post = L.d.res_post;
+  if (L.d.op == SWAPNET_OP_LINEAR) {
+    g->M = L.n; g->N = U.rows; g->K = L.d.cin;
+    g->A = x; g->lda = L.d.cin; g->conv = 0;
+    g->y = y + (int64_t)U.row0 * es; g->ldy = L.d.cout;
+    g->e.res = r ? r + (int64_t)U.row0 * es : nullptr; g->e.ldr = L.d.cout;
+    return true;
+  }
+  // conv
+  g->N = L.d.cout;
+  g->K = L.d.kh * L.d.kw * L.d.cin;
+  g->M = L.on * L.oh * L.ow;
+  g->y = y; g->ldy = L.d.cout;
+  g->e.res = r; g->e.ldr = L.d.cout;
+  g->A = x;
+  const bool pointwise = L.d.kh == 1 && L.d.kw == 1 && L.d.stride == 1 && L.d.pad == 0;
+  g->conv = pointwise ? 0 : 1;
+  g->lda = L.d.cin;
+  g->H = L.h; g->Wd = L.w; g->C = L.d.cin; g->Ho = L.oh; g->Wo = L.ow;
+  g->kh = L.d.kh; g->kw = L.d.kw; g->stride = L.d.stride; g->pad = L.d.pad;
+  return true;
+}
+
+static bool wants_tc(const Model& m, const Layer& L) {
+  if (m.dtype == SWAPNET_F32) return false;
+  if (L.d.op == SWAPNET_OP_LINEAR) return L.n > 16 && L.d.cin % 8 == 0;
+  if (L.d.op == SWAPNET_OP_CONV2D) return L.d.cin % 8 == 0;
+  return false;
+}
+
+static int prepare_units(swapnet_engine* e) {
+  const swapnet_plan& p = e->plan;
+  const Model& m = p.model;
+  e->ux.assign(p.units.size(), UnitExec{});
+  e->unit_kind.assign(p.units.size(), 0);
+  for (size_t u = 0; u < p.units.size(); ++u) {
+    const Layer& L = m.L[p.units[u].layer];
+    int k = 0;
+    switch (L.d.op) {
+      case SWAPNET_OP_LINEAR: k = wants_tc(m, L) ? SWAPNET_KERNEL_TC_GEMM : SWAPNET_KERNEL_SKINNY; break;
+      case SWAPNET_OP_CONV2D:
+        if (!wants_tc(m, L)) k = SWAPNET_KERNEL_DIRECT_CONV;
+        else if (L.d.kh == 1 && L.d.kw == 1 && L.d.stride == 1 && L.d.pad == 0) k = SWAPNET_KERNEL_TC_GEMM;
+        else k = SWAPNET_KERNEL_TC_CONV;
+        break;
+      case SWAPNET_OP_MAXPOOL: k = SWAPNET_KERNEL_MAXPOOL; break;
+      case SWAPNET_OP_GAP: k = SWAPNET_KERNEL_GAP; break;
+      case SWAPNET_OP_UPSAMPLE2X: k = SWAPNET_KERNEL_UPSAMPLE; break;
+      case SWAPNET_OP_CONCAT: k = SWAPNET_KERNEL_CONCAT; break;
+    }
+    e->unit_kind[u] = k;
+  }
+  for (const Block& B : p.blocks) {
+    char* base = slot_base(e, B.slot);
+    for (int u = B.u0; u < B.u1; ++u) {
+      const Unit& U = p.units[u];
+      UnitExec& X = e->ux[u];
+      if (U.nt == 2) { X.w = base + U.slot_off[0]; X.b = base + U.slot_off[1]; }
+      const Layer& L = m.L[U.layer];
+      if (!wants_tc(m, L)) continue;
+      X.use_tc = true;
+      // A pointers in the workspace are fixed; the model input and outputs
+      // are bound per call (the map is re-encoded when they change).
+      const char* x = (L.d.src0 == SWAPNET_SRC_INPUT || m.L[L.d.src0].out_off >= 0)
+                          ? nullptr
+                          : act_ptr(e, L.d.src0, nullptr, nullptr);
+      TcGemm g;
+      unit_gemm(e, U, X, x, nullptr, nullptr, &g);
+      if (!g.conv && !x) g.A = nullptr;
+      int rc = tc_prepare(g, &X.tc);
+      if (rc) return rc;
+      X.tmA_for = g.A;
+    }
+  }
+  return SWAPNET_OK;
+}
+
+static int run_unit(swapnet_engine* e, int u, const void* din, void* dout, cudaStream_t s) {
+  const swapnet_plan& p = e->plan;
+  const Model& m = p.model;
+  const Unit& U = p.units[u];
+  UnitExec& X = e->ux[u];
+  const Layer& L = m.L[U.layer];
+  const char* x = act_ptr(e, L.d.src0, din, dout);
+  const char* r = L.d.res == SWAPNET_SRC_NONE ? nullptr : act_ptr(e, L.d.res, din, dout);
+  char* y = out_ptr(e, U.layer, dout);
+  const int es = m.es;
+  switch (L.d.op) {
+    case SWAPNET_OP_LINEAR:
+    case SWAPNET_OP_CONV2D: {
+      if (X.use_tc) {
+        TcGemm g;
+        unit_gemm(e, U, X, x, r, y, &g);
+        if (!g.conv && g.A != X.tmA_for) {
+          int rc = tc_prepare(g, &X.tc);
+          if (rc) return rc;
+          X.tmA_for = g.A;
+        }
+        return launch_tc_gemm(g, X.tc, e->err_word, s);
+      }
+      Epi ep{X.b, nullptr, L.d.cout, L.d.act, L.d.res_post};
+      if (L.d.op == SWAPNET_OP_LINEAR) {
+        ep.res = r ? r + (int64_t)U.row0 * es : nullptr;
+        return launch_linear_skinny(m.dtype, x, L.n, L.d.cin, X.w, U.rows, ep, y + (int64_t)U.row0 * es,
+                                    L.d.cout, s);
+      }
+      ep.res = r;
+      return launch_conv_direct(m.dtype, x, L.n, L.h, L.w, L.d.cin, X.w, L.d.cout, L.d.kh, L.d.kw, L.d.stride,
+                                L.d.pad, L.oh, L.ow, ep, y, s);
+    }
+    case SWAPNET_OP_MAXPOOL:
+      return launch_maxpool(m.dtype, x, L.n, L.h, L.w, L.c, L.d.kh, L.d.kw, L.d.stride, L.d.pad, L.oh, L.ow, y, s);
+    case SWAPNET_OP_GAP:
+      return launch_gap(m.dtype, x, L.n, L.h, L.w, L.c, y, s);
+    case SWAPNET_OP_UPSAMPLE2X:
+      return launch_upsample2x(m.dtype, x, L.n, L.h, L.w, L.c, y, s);
+    case SWAPNET_OP_CONCAT:
+      return launch_concat(m.dtype, x, L.c, act_ptr(e, L.d.src1, din, dout), L.c1, (int64_t)L.n * L.h * L.w, y, s);
+    default:
+      SN_FAIL(SWAPNET_ERR_INVALID_ARG, "unknown op");
+  }
+}
+
+}  // namespace swapnet
+
+extern "C" {
+
+int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint32_t n_tensors, void* d_arena,
+                 uint64_t arena_bytes, void* d_workspace, uint64_t workspace_bytes, swapnet_engine** out) {
+  if (!plan || !out || (n_tensors && !host_weights)) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+  if ((int)n_tensors != plan->model.n_tensors)
+    SN_FAIL(SWAPNET_ERR_INVALID_ARG, "expected " + std::to_string(plan->model.n_tensors) + " host tensors");
+  if (((uintptr_t)d_arena | (uintptr_t)d_workspace) % kAlign)
+    SN_FAIL(SWAPNET_ERR_MISALIGNED, "device buffers must be 256-byte aligned");
+  const uint64_t arena_need = plan->resident ? plan->arena : plan->slot * (uint64_t)plan->opt.slots;
+  if (d_arena && arena_bytes < arena_need) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "arena buffer too small");
+  if (d_workspace && workspace_bytes < plan->model.ws_bytes)
+    SN_FAIL(SWAPNET_ERR_INVALID_ARG, "workspace buffer too small");
+  swapnet_engine* e = new (std::nothrow) swapnet_engine();
+  if (!e) SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
+  std::unique_ptr<swapnet_engine, int (*)(swapnet_engine*)> guard(e, release);
+  try {
+    e->plan = *plan;
+  } catch (const std::bad_alloc&) {
+    SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
+  }
+  CU(cudaGetDevice(&e->device), "cudaGetDevice");
+  CU(cudaDeviceGetAttribute(&e->num_sms, cudaDevAttrMultiProcessorCount, e->device), "device attribute");
+  e->zc_ctas = plan->opt.zc_ctas > 0 ? plan->opt.zc_ctas : 32;
+  int rc = tc_error_word(&e->err_word);
+  if (rc) return rc;
+  // device memory
+  if (d_arena) {
+    e->d_arena = static_cast<char*>(d_arena);
+  } else {
+    if (injected(2)) SN_FAIL(SWAPNET_ERR_OOM, "arena allocation failed (injected)");
+    if (cudaMalloc(&e->d_arena, std::max<uint64_t>(arena_need, kAlign)) != cudaSuccess) {
+      cudaGetLastError();
+      SN_FAIL(SWAPNET_ERR_OOM, "arena allocation failed");
+    }
+    e->own_arena = true;
+  }
+  if (d_workspace || plan->model.ws_bytes == 0) {
+    e->d_ws = static_cast<char*>(d_workspace);
+  } else {
+    if (injected(2)) SN_FAIL(SWAPNET_ERR_OOM, "workspace allocation failed (injected)");
+    if (cudaMalloc(&e->d_ws, plan->model.ws_bytes) != cudaSuccess) {
+      cudaGetLastError();
+      SN_FAIL(SWAPNET_ERR_OOM, "workspace allocation failed");
+    }
+    e->own_ws = true;
+  }
+  if (injected(3)) SN_FAIL(SWAPNET_ERR_CUDA, "stream creation failed (injected)");
+  int lo = 0, hi = 0;
+  CU(cudaDeviceGetStreamPriorityRange(&lo, &hi), "stream priority range");
+  CU(cudaStreamCreateWithPriority(&e->copy, cudaStreamNonBlocking, hi), "copy stream");
+  for (int s = 0; s < 2; ++s) {
+    CU(cudaEventCreateWithFlags(&e->slot_free[s], cudaEventDisableTiming), "event");
+    CU(cudaEventCreateWithFlags(&e->ready[s], cudaEventDisableTiming), "event");
+  }
+  rc = register_host(e, host_weights, n_tensors);
+  if (rc) return rc;
+  build_segments(e);
+  rc = prepare_units(e);
+  if (rc) return rc;
+  const int variant = plan->opt.swap_variant;
+  if (plan->resident) {
+    for (size_t k = 0; k < e->blocks.size() && !rc; ++k) rc = swap_block(e, k, SWAPNET_SWAP_MEMCPY, e->copy);
+    if (rc) return rc;
+    CU(cudaStreamSynchronize(e->copy), "resident upload");
+    e->weights_loaded = true;
+  } else if (variant == SWAPNET_SWAP_AUTO) {
+    rc = calibrate(e);
+    if (rc) return rc;
+  } else {
+    for (EngBlock& b : e->blocks) {
+      b.variant = variant;
+      if (variant == SWAPNET_SWAP_ZEROCOPY && !zerocopy_ok(b)) SN_FAIL(SWAPNET_ERR_MISALIGNED, "zero-copy needs 16-byte aligned host tensors");
+    }
+  }
+  e->stats = swapnet_engine_stats{};
+  *out = guard.release();
+  return SWAPNET_OK;
+}
+
+int swapnet_infer(swapnet_engine* e, const void* din, void* dout, swapnet_stream stream) {
+  if (!e || !din || !dout) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+  if (((uintptr_t)din | (uintptr_t)dout) & 15) SN_FAIL(SWAPNET_ERR_MISALIGNED, "input/output must be 16-byte aligned");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  CU(cudaSetDevice(e->device), "cudaSetDevice");
+  const swapnet_plan& p = e->plan;
+  const bool prof = e->profiling;
+  for (size_t k = 0; k < p.blocks.size(); ++k) {
+    const Block& B = p.blocks[k];
+    if (!p.resident) {
+      CU(cudaStreamWaitEvent(e->copy, e->slot_free[B.slot], 0), "wait slot");
+      if (prof) CU(cudaEventRecord(e->ev_swap[2 * k], e->copy), "profile event");
+      int rc = swap_block(e, k, e->blocks[k].variant, e->copy);
+      if (rc) return rc;
+      if (prof) CU(cudaEventRecord(e->ev_swap[2 * k + 1], e->copy), "profile event");
+      CU(cudaEventRecord(e->ready[B.slot], e->copy), "record ready");
+      CU(cudaStreamWaitEvent(s, e->ready[B.slot], 0), "wait ready");
+    }
+    for (int u = B.u0; u < B.u1; ++u) {
+      if (prof) CU(cudaEventRecord(e->ev_unit[2 * u], s), "profile event");
+      int rc = run_unit(e, u, din, dout, s);
+      if (rc) return rc;
+      if (prof) CU(cudaEventRecord(e->ev_unit[2 * u + 1], s), "profile event");
+      e->stats.kernel_launches += 1;
+    }
+    if (!p.resident) CU(cudaEventRecord(e->slot_free[B.slot], s), "record slot free");
+  }
+  e->stats.infer_calls += 1;
+  return SWAPNET_OK;
+}
+
+int swapnet_infer_host(swapnet_engine* e, const void* hin, void* hout, swapnet_stream stream) {
+  if (!e || !hin || !hout) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  CU(cudaSetDevice(e->device), "cudaSetDevice");
+  const Model& m = e->plan.model;
+  if (!e->d_in_stage) {
+    if (cudaMalloc(&e->d_in_stage, align_up(m.in_bytes)) != cudaSuccess ||
+        cudaMalloc(&e->d_out_stage, align_up(m.out_bytes)) != cudaSuccess) {
+      cudaGetLastError();
+      SN_FAIL(SWAPNET_ERR_OOM, "staging allocation failed");
+    }
+  }
+  CU(cudaMemcpyAsync(e->d_in_stage, hin, m.in_bytes, cudaMemcpyHostToDevice, s), "input copy");
+  int rc = swapnet_infer(e, e->d_in_stage, e->d_out_stage, stream);
+  if (rc) return rc;
+  CU(cudaMemcpyAsync(hout, e->d_out_stage, m.out_bytes, cudaMemcpyDeviceToHost, s), "output copy");
+  return SWAPNET_OK;
+}
+
+int swapnet_engine_sync(swapnet_engine* e) {
+  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+  CU(cudaSetDevice(e->device), "cudaSetDevice");
+  CU(cudaStreamSynchronize(e->copy), "copy stream");
+  CU(cudaDeviceSynchronize(), "device synchronize");
+  int w = 0;
+  CU(cudaMemcpy(&w, e->err_word, sizeof(int), cudaMemcpyDeviceToHost), "error word");
+  if (w) {
+    const int zero = 0;
+    cudaMemcpy(e->err_word, &zero, sizeof(int), cudaMemcpyHostToDevice);
+    SN_FAIL(SWAPNET_ERR_TIMEOUT, "a device-side wait gave up");
+  }
+  return SWAPNET_OK;
+}
+
+int swapnet_engine_blocks(const swapnet_engine* e, swapnet_engine_block* b, uint32_t cap, uint32_t* n) {
+  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+  if (n) *n = (uint32_t)e->blocks.size();
+  for (uint32_t i = 0; b && i < cap && i < e->blocks.size(); ++i) {
+    const EngBlock& B = e->blocks[i];
+    b[i] = swapnet_engine_block{B.variant, (int32_t)B.segs.size(), B.memcpy_us, B.zerocopy_us};
+  }
+  return SWAPNET_OK;
+}
+
+int swapnet_engine_stats_get(const swapnet_engine* e, swapnet_engine_stats* st) {
+  if (!e || !st) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+  *st = e->stats;
+  return SWAPNET_OK;
+}
+
+int swapnet_engine_unit_kernels(const swapnet_engine* e, int32_t* kinds, uint32_t cap, uint32_t* n) {
+  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+  if (n) *n = (uint32_t)e->unit_kind.size();
+  for (uint32_t i = 0; kinds && i < cap && i < e->unit_kind.size(); ++i) kinds[i] = e->unit_kind[i];
+  return SWAPNET_OK;
+}
+
+int swapnet_engine_set_profiling(swapnet_engine* e, int enable) {
+  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+  CU(cudaSetDevice(e->device), "cudaSetDevice");
+  if (enable && e->ev_unit.empty()) {
+    e->ev_unit.assign(2 * e->plan.units.size(), nullptr);
+    e->ev_swap.assign(2 * e->plan.blocks.size(), nullptr);
+    for (cudaEvent_t& ev : e->ev_unit) CU(cudaEventCreate(&ev), "event");
+    for (cudaEvent_t& ev : e->ev_swap) CU(cudaEventCreate(&ev), "event");
+  }
+  e->profiling = enable != 0;
+  return SWAPNET_OK;
+}
+
+int swapnet_engine_last_times(swapnet_engine* e, float* unit_us, uint32_t nu, float* swap_us, uint32_t nb) {
+  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+  if (e->ev_unit.empty()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "profiling was never enabled");
+  CU(cudaSetDevice(e->device), "cudaSetDevice");
+  CU(cudaDeviceSynchronize(), "device synchronize");
+  for (uint32_t u = 0; unit_us && u < nu && u < e->plan.units.size(); ++u) {
+    float ms = 0.f;
+    CU(cudaEventElapsedTime(&ms, e->ev_unit[2 * u], e->ev_unit[2 * u + 1]), "elapsed");
+    unit_us[u] = ms * 1000.f;
+  }
+  for (uint32_t k = 0; swap_us && k < nb && k < e->plan.blocks.size(); ++k) {
+    float ms = 0.f;
+    if (!e->plan.resident) CU(cudaEventElapsedTime(&ms, e->ev_swap[2 * k], e->ev_swap[2 * k + 1]), "elapsed");
+    swap_us[k] = ms * 1000.f;
+  }
+  return SWAPNET_OK;
+}
+
+void swapnet_engine_free(swapnet_engine* e) { release(e); }
+
+int swapnet_debug_fail_next(int what, int count) {
+  if (what < 1 || what > 3 || count < 0) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad fault-injection request");
+  g_fail_next[what] = count;
+  return SWAPNET_OK;
+}
+
+}  // extern "C"

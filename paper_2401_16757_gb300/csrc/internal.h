@@ -1,0 +1,94 @@
+// Internal structures shared by the host-side translation units of libswapnet.
+#pragma once
+#include <cstdint>
+#include <string>
+#include <vector>
+
+#include "../../include/swapnet.h"
+
+namespace swapnet {
+
+constexpr uint64_t kAlign = 256;
+inline uint64_t align_up(uint64_t x, uint64_t a = kAlign) { return (x + a - 1) / a * a; }
+inline uint64_t ceil_div_u(uint64_t a, uint64_t b) { return (a + b - 1) / b; }
+
+// Thread-local error message for swapnet_last_error().
+void set_error(const std::string& msg);
+
+struct Status {
+  int code = SWAPNET_OK;
+  static Status ok() { return Status{}; }
+};
+
+#define SN_FAIL(code, msg)   \
+  do {                       \
+    ::swapnet::set_error(msg); \
+    return (code);           \
+  } while (0)
+
+int dtype_size(int dtype);
+
+// One analysed layer: descriptor plus derived shapes, sizes and liveness.
+struct Layer {
+  swapnet_layer d;
+  int n, h, w, c;        // dims of src0 (the main input)
+  int on, oh, ow, oc;    // output dims
+  int c1;                // channels of src1 (concat)
+  int n_tensors;
+  uint64_t tbytes[2];    // raw bytes of each parameter tensor
+  int first_tensor;      // global index of the first parameter tensor
+  uint64_t flops;
+  int last_use;          // last layer reading this output (inclusive)
+  int64_t ws_off;        // workspace offset, -1 when the output is a model output
+  int64_t out_off;       // offset in the output buffer, -1 if not an output
+  uint64_t out_bytes;    // raw bytes of the output tensor
+};
+
+struct Model {
+  int dtype = 0, es = 0;
+  int in_n = 0, in_h = 0, in_w = 0, in_c = 0;
+  std::vector<Layer> L;
+  int n_tensors = 0;
+  uint64_t ws_bytes = 0, out_bytes = 0, in_bytes = 0, weight_bytes = 0;
+  std::vector<uint64_t> tensor_raw;  // raw bytes per global tensor
+};
+
+// Partition unit: a layer, or a piece of an oversize linear layer.
+struct Unit {
+  int layer, row0, rows, depth;
+  uint64_t bytes, flops;
+  int64_t t_ex;
+  // parameter tensors of the unit: global tensor index, byte offset in that
+  // tensor, bytes to copy, offset inside the block's slot
+  int nt;
+  int tidx[2];
+  uint64_t toff[2], tlen[2], slot_off[2];
+};
+
+struct Block {
+  int u0, u1, slot, depth;
+  uint64_t bytes;
+  int64_t t_in, t_ex, t_out;
+};
+
+}  // namespace swapnet
+
+struct swapnet_plan {
+  swapnet::Model model;
+  swapnet_options opt;
+  bool resident = false;
+  uint64_t budget = 0, arena = 0, slot = 0;
+  std::vector<swapnet::Unit> units;
+  std::vector<swapnet::Block> blocks;
+  std::vector<uint32_t> cuts;
+  int64_t predicted = 0;
+};
+
+namespace swapnet {
+int analyse_model(const swapnet_model_desc* desc, Model* m);
+int make_units(const Model& m, const swapnet_options& opt, uint64_t slot, std::vector<Unit>* out);
+void finalize_blocks(swapnet_plan* p, const std::vector<uint32_t>& cuts);
+int64_t pipeline_ns(const std::vector<Block>& b, int slots);
+int64_t eq4_ns(const std::vector<Block>& b);
+uint64_t resident_latency_ns(const Model& m, const swapnet_options& opt);
+}  // namespace swapnet

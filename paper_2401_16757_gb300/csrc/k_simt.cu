@@ -1,0 +1,305 @@
+// SIMT layer kernels: skinny linear (M <= 16, HBM-bound GEMV family),
+// direct convolution for channel counts the tensor-core path cannot tile,
+// pooling, upsampling and channel concatenation.  NHWC everywhere.
+#include <cstdio>
+
+#include "device.cuh"
+#include "internal.h"
+#include "kernels.h"
+
+namespace swapnet {
+
+namespace {
+
+template <typename T> struct Vec16 { static constexpr int N = 16 / sizeof(T); };
+
+__device__ __forceinline__ uint4 ld_stream16(const void* p) {
+  uint4 r;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(p));
+  return r;
+}
+
+template <typename T> __device__ __forceinline__ void unpack16(const uint4& v, float* f) {
+  const T* e = reinterpret_cast<const T*>(&v);
+#pragma unroll
+  for (int i = 0; i < Vec16<T>::N; ++i) f[i] = to_f<T>(e[i]);
+}
+
+// ------------------------------------------------------------ skinny linear
+// One CTA (8 warps) computes COLS output features for all M rows.  Warp w
+// reduces the K range [w*Kw, (w+1)*Kw); inside a warp lane l takes the
+// 16-byte chunks l, l+32, ...; partial sums are combined by a butterfly and
+// then across warps in index order, so the result does not depend on
+// scheduling.
+constexpr int kSkCols = 2;
+constexpr int kSkWarps = 8;
+
+template <typename T, int MT>
+__global__ void __launch_bounds__(kSkWarps * 32) linear_skinny_kernel(const T* __restrict__ x, int M, int K,
+                                                                      const T* __restrict__ W, int N, Epi e,
+                                                                      T* __restrict__ y, int64_t ldy) {
+  constexpr int V = Vec16<T>::N;
+  __shared__ float red[kSkWarps][kSkCols][MT];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int o0 = blockIdx.x * kSkCols;
+  const int kchunks = K / V;                       // K % V == 0 (checked on the host)
+  const int per_warp = (kchunks + kSkWarps - 1) / kSkWarps;
+  const int c_begin = warp * per_warp;
+  const int c_end = min(kchunks, c_begin + per_warp);
+  float acc[kSkCols][MT];
+#pragma unroll
+  for (int c = 0; c < kSkCols; ++c)
+#pragma unroll
+    for (int m = 0; m < MT; ++m) acc[c][m] = 0.f;
+
+  for (int ch = c_begin + lane; ch < c_end; ch += 32) {
+    const int k = ch * V;
+    float wv[kSkCols][V];
+#pragma unroll
+    for (int c = 0; c < kSkCols; ++c) {
+      if (o0 + c < N) {
+        unpack16<T>(ld_stream16(W + (int64_t)(o0 + c) * K + k), wv[c]);
+      } else {
+#pragma unroll
+        for (int i = 0; i < V; ++i) wv[c][i] = 0.f;
+      }
+    }
+#pragma unroll
+    for (int m = 0; m < MT; ++m) {
+      if (m < M) {
+        float xv[V];
+        unpack16<T>(__ldg(reinterpret_cast<const uint4*>(x + (int64_t)m * K + k)), xv);
+#pragma unroll
+        for (int c = 0; c < kSkCols; ++c)
+#pragma unroll
+          for (int i = 0; i < V; ++i) acc[c][m] = fmaf(wv[c][i], xv[i], acc[c][m]);
+      }
+    }
+  }
+#pragma unroll
+  for (int c = 0; c < kSkCols; ++c)
+#pragma unroll
+    for (int m = 0; m < MT; ++m) {
+      float v = acc[c][m];
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+      if (lane == 0) red[warp][c][m] = v;
+    }
+  __syncthreads();
+  const int t = threadIdx.x;
+  if (t < kSkCols * MT) {
+    const int c = t / MT, m = t % MT;
+    const int o = o0 + c;
+    if (m < M && o < N) {
+      float s = 0.f;
+#pragma unroll
+      for (int w = 0; w < kSkWarps; ++w) s += red[w][c][m];
+      const float b = to_f<T>(reinterpret_cast<const T*>(e.bias)[o]);
+      float r = 0.f;
+      if (e.res) r = to_f<T>(reinterpret_cast<const T*>(e.res)[(int64_t)m * e.ldr + o]);
+      y[(int64_t)m * ldy + o] = from_f<T>(epilogue(s, b, r, e.res != nullptr, e.act, e.res_post));
+    }
+  }
+}
+
+template <typename T>
+int skinny_dispatch(const void* x, int M, int K, const void* W, int N, const Epi& e, void* y, int64_t ldy,
+                    cudaStream_t s) {
+  const dim3 grid((N + kSkCols - 1) / kSkCols), block(kSkWarps * 32);
+  const T* xp = static_cast<const T*>(x);
+  const T* wp = static_cast<const T*>(W);
+  T* yp = static_cast<T*>(y);
+  if (M <= 1) linear_skinny_kernel<T, 1><<<grid, block, 0, s>>>(xp, M, K, wp, N, e, yp, ldy);
+  else if (M <= 2) linear_skinny_kernel<T, 2><<<grid, block, 0, s>>>(xp, M, K, wp, N, e, yp, ldy);
+  else if (M <= 4) linear_skinny_kernel<T, 4><<<grid, block, 0, s>>>(xp, M, K, wp, N, e, yp, ldy);
+  else if (M <= 8) linear_skinny_kernel<T, 8><<<grid, block, 0, s>>>(xp, M, K, wp, N, e, yp, ldy);
+  else linear_skinny_kernel<T, 16><<<grid, block, 0, s>>>(xp, M, K, wp, N, e, yp, ldy);
+  return cudaGetLastError() == cudaSuccess ? SWAPNET_OK : SWAPNET_ERR_CUDA;
+}
+
+// ------------------------------------------------------------ direct conv
+// Thread = one output pixel x 8 output channels; the lanes of a warp share
+// the channel group, so weight loads are warp-uniform (broadcast).
+constexpr int kDcCo = 8;
+
+template <typename T>
+__global__ void conv_direct_kernel(const T* __restrict__ x, int n, int h, int w, int cin,
+                                   const T* __restrict__ W, int cout, int kh, int kw, int stride, int pad, int oh,
+                                   int ow, Epi e, T* __restrict__ y) {
+  const int64_t pix = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t npix = (int64_t)n * oh * ow;
+  const int co0 = blockIdx.y * kDcCo;
+  if (pix >= npix) return;
+  const int img = (int)(pix / ((int64_t)oh * ow));
+  const int rem = (int)(pix % ((int64_t)oh * ow));
+  const int oy = rem / ow, ox = rem % ow;
+  float acc[kDcCo];
+#pragma unroll
+  for (int j = 0; j < kDcCo; ++j) acc[j] = 0.f;
+  for (int r = 0; r < kh; ++r) {
+    const int iy = oy * stride + r - pad;
+    if (iy < 0 || iy >= h) continue;
+    for (int s = 0; s < kw; ++s) {
+      const int ix = ox * stride + s - pad;
+      if (ix < 0 || ix >= w) continue;
+      const T* xp = x + (((int64_t)img * h + iy) * w + ix) * cin;
+      for (int c = 0; c < cin; ++c) {
+        const float xv = to_f<T>(xp[c]);
+#pragma unroll
+        for (int j = 0; j < kDcCo; ++j) {
+          const int co = co0 + j;
+          if (co < cout) acc[j] = fmaf(xv, to_f<T>(__ldg(W + (((int64_t)co * kh + r) * kw + s) * cin + c)), acc[j]);
+        }
+      }
+    }
+  }
+  const T* bias = reinterpret_cast<const T*>(e.bias);
+  const T* res = reinterpret_cast<const T*>(e.res);
+#pragma unroll
+  for (int j = 0; j < kDcCo; ++j) {
+    const int co = co0 + j;
+    if (co >= cout) break;
+    const float rv = res ? to_f<T>(res[pix * e.ldr + co]) : 0.f;
+    y[pix * cout + co] = from_f<T>(epilogue(acc[j], to_f<T>(bias[co]), rv, res != nullptr, e.act, e.res_post));
+  }
+}
+
+// ------------------------------------------------------------ pooling etc.
+template <typename T>
+__global__ void maxpool_kernel(const T* __restrict__ x, int n, int h, int w, int c, int kh, int kw, int stride,
+                               int pad, int oh, int ow, T* __restrict__ y) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t total = (int64_t)n * oh * ow * c;
+  if (idx >= total) return;
+  const int ch = (int)(idx % c);
+  const int64_t p = idx / c;
+  const int ox = (int)(p % ow);
+  const int oy = (int)((p / ow) % oh);
+  const int img = (int)(p / ((int64_t)ow * oh));
+  float m = -INFINITY;
+  for (int r = 0; r < kh; ++r) {
+    const int iy = oy * stride + r - pad;
+    if (iy < 0 || iy >= h) continue;
+    for (int s = 0; s < kw; ++s) {
+      const int ix = ox * stride + s - pad;
+      if (ix < 0 || ix >= w) continue;
+      m = fmaxf(m, to_f<T>(x[(((int64_t)img * h + iy) * w + ix) * c + ch]));
+    }
+  }
+  y[idx] = from_f<T>(m);
+}
+
+template <typename T>
+__global__ void gap_kernel(const T* __restrict__ x, int n, int hw, int c, T* __restrict__ y) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (int64_t)n * c) return;
+  const int img = (int)(idx / c), ch = (int)(idx % c);
+  const T* p = x + (int64_t)img * hw * c + ch;
+  float s = 0.f;
+  for (int i = 0; i < hw; ++i) s += to_f<T>(p[(int64_t)i * c]);
+  y[idx] = from_f<T>(s / (float)hw);
+}
+
+template <typename T>
+__global__ void upsample2x_kernel(const T* __restrict__ x, int n, int h, int w, int c, T* __restrict__ y) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t total = (int64_t)n * 2 * h * 2 * w * c;
+  if (idx >= total) return;
+  const int ch = (int)(idx % c);
+  const int64_t p = idx / c;
+  const int ox = (int)(p % (2 * w));
+  const int oy = (int)((p / (2 * w)) % (2 * h));
+  const int img = (int)(p / ((int64_t)4 * w * h));
+  y[idx] = x[(((int64_t)img * h + oy / 2) * w + ox / 2) * c + ch];
+}
+
+template <typename T>
+__global__ void concat_kernel(const T* __restrict__ a, int ca, const T* __restrict__ b, int cb, int64_t pixels,
+                              T* __restrict__ y) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int c = ca + cb;
+  if (idx >= pixels * c) return;
+  const int64_t p = idx / c;
+  const int ch = (int)(idx % c);
+  y[idx] = ch < ca ? a[p * ca + ch] : b[p * cb + (ch - ca)];
+}
+
+inline int grid1d(int64_t total, int block) { return (int)((total + block - 1) / block); }
+
+}  // namespace
+
+#define SN_DISPATCH(dtype, T, ...)                    \
+  switch (dtype) {                                    \
+    case SWAPNET_F32: { using T = float; __VA_ARGS__; break; }          \
+    case SWAPNET_F16: { using T = __half; __VA_ARGS__; break; }         \
+    case SWAPNET_BF16: { using T = __nv_bfloat16; __VA_ARGS__; break; } \
+    default: return SWAPNET_ERR_INVALID_ARG;          \
+  }
+
+static int last_launch() {
+  const cudaError_t err = cudaGetLastError();
+  if (err != cudaSuccess) {
+    set_error(std::string("kernel launch: ") + cudaGetErrorString(err));
+    return SWAPNET_ERR_CUDA;
+  }
+  return SWAPNET_OK;
+}
+
+int launch_linear_skinny(int dtype, const void* x, int M, int K, const void* W, int N, const Epi& e, void* y,
+                         int64_t ldy, cudaStream_t s) {
+  const int es = dtype_size(dtype);
+  if (M < 1 || M > 16 || K < 1 || N < 1) SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "skinny linear: M must be in [1, 16]");
+  if ((K * es) % 16 || ((uintptr_t)x | (uintptr_t)W) % 16)
+    SN_FAIL(SWAPNET_ERR_MISALIGNED, "skinny linear: rows must be 16-byte aligned");
+  SN_DISPATCH(dtype, T, return skinny_dispatch<T>(x, M, K, W, N, e, y, ldy, s));
+  return SWAPNET_OK;
+}
+
+int launch_conv_direct(int dtype, const void* x, int n, int h, int w, int cin, const void* W, int cout, int kh,
+                       int kw, int stride, int pad, int oh, int ow, const Epi& e, void* y, cudaStream_t s) {
+  const int64_t npix = (int64_t)n * oh * ow;
+  const dim3 grid(grid1d(npix, 128), (cout + kDcCo - 1) / kDcCo);
+  SN_DISPATCH(dtype, T,
+              conv_direct_kernel<T><<<grid, 128, 0, s>>>(static_cast<const T*>(x), n, h, w, cin,
+                                                         static_cast<const T*>(W), cout, kh, kw, stride, pad, oh,
+                                                         ow, e, static_cast<T*>(y)));
+  return last_launch();
+}
+
+int launch_maxpool(int dtype, const void* x, int n, int h, int w, int c, int kh, int kw, int stride, int pad,
+                   int oh, int ow, void* y, cudaStream_t s) {
+  const int64_t total = (int64_t)n * oh * ow * c;
+  SN_DISPATCH(dtype, T,
+              maxpool_kernel<T><<<grid1d(total, 256), 256, 0, s>>>(static_cast<const T*>(x), n, h, w, c, kh, kw,
+                                                                    stride, pad, oh, ow, static_cast<T*>(y)));
+  return last_launch();
+}
+
+int launch_gap(int dtype, const void* x, int n, int h, int w, int c, void* y, cudaStream_t s) {
+  SN_DISPATCH(dtype, T,
+              gap_kernel<T><<<grid1d((int64_t)n * c, 256), 256, 0, s>>>(static_cast<const T*>(x), n, h * w, c,
+                                                                         static_cast<T*>(y)));
+  return last_launch();
+}
+
+int launch_upsample2x(int dtype, const void* x, int n, int h, int w, int c, void* y, cudaStream_t s) {
+  const int64_t total = (int64_t)n * 4 * h * w * c;
+  SN_DISPATCH(dtype, T,
+              upsample2x_kernel<T><<<grid1d(total, 256), 256, 0, s>>>(static_cast<const T*>(x), n, h, w, c,
+                                                                       static_cast<T*>(y)));
+  return last_launch();
+}
+
+int launch_concat(int dtype, const void* a, int ca, const void* b, int cb, int64_t pixels, void* y,
+                  cudaStream_t s) {
+  const int64_t total = pixels * (ca + cb);
+  SN_DISPATCH(dtype, T,
+              concat_kernel<T><<<grid1d(total, 256), 256, 0, s>>>(static_cast<const T*>(a), ca,
+                                                                   static_cast<const T*>(b), cb, pixels,
+                                                                   static_cast<T*>(y)));
+  return last_launch();
+}
+
+}  // namespace swapnet

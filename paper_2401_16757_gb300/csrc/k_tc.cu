@@ -1,0 +1,347 @@
+// tcgen05 tensor-core GEMM and implicit-GEMM convolution for sm_103a.
+//
+//   C[m, n] = sum_k A[m, k] * B[n, k],  fp16/bf16 operands, fp32 accumulate
+//   in TMEM, fused epilogue (bias, residual, activation) on the way out.
+//
+// B is a weight matrix [N][K] (K contiguous) that lives in the arena slot of
+// the block being executed; it is staged by TMA (128-byte swizzle).  A is
+// either a row-major activation matrix (linear layers, 1x1 stride-1 convs),
+// also staged by TMA, or the implicit im2col of an NHWC input for general
+// convolutions, gathered by four warps with cp.async (zero fill for padding)
+// into the same swizzled layout.  One CTA computes one 128 x BN tile:
+//   warp 0      TMA producer (one elected lane)
+//   warp 1      TMEM allocation and MMA issue (one elected lane)
+//   warps 2..5  im2col gather (conv) and the epilogue (TMEM -> registers ->
+//               global), warp w reading TMEM lanes 32*(w % 4) .. +31.
+// Every wait is bounded; on timeout the kernel records kDevErrTimeout in
+// the error word, drains what it started, frees TMEM and returns.
+#include <cudaTypedefs.h>
+
+#include <cstring>
+#include <mutex>
+#include <type_traits>
+
+#include "device.cuh"
+#include "internal.h"
+#include "kernels.h"
+
+namespace swapnet {
+
+__device__ int g_tc_err;
+
+namespace {
+
+constexpr int kBM = 128;
+constexpr int kBK = 64;  // 64 x 2 bytes = one 128-byte swizzle row
+constexpr int kStages = 4;
+constexpr int kThreads = 192;
+constexpr int kLag = 2;  // gather: stages of cp.async in flight per thread
+constexpr int kABytes = kBM * kBK * 2;
+
+template <int BN> struct Cfg {
+  static constexpr int kBBytes = BN * kBK * 2;
+  static constexpr int kSmem = kStages * (kABytes + kBBytes) + 1024 + 256;
+};
+
+struct TcArgs {
+  int M, N, K;
+  const void* x;  // conv input (gather)
+  int H, Wd, C, Ho, Wo, kh, kw, stride, pad;
+  Epi e;
+  void* y;
+  int64_t ldy;
+  int* err;
+};
+
+template <typename T>
+__device__ __forceinline__ void store_row32(T* dst, const float* v) {
+  // 32 consecutive outputs, 16-byte stores
+  uint4 pk[4];
+  T* e = reinterpret_cast<T*>(pk);
+#pragma unroll
+  for (int j = 0; j < 32; ++j) e[j] = from_f<T>(v[j]);
+  uint4* d = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+  for (int q = 0; q < 4; ++q) d[q] = pk[q];
+}
+
+template <typename T, int BN, bool GATHER>
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const TcArgs p) {
+  constexpr int kBBytes = Cfg<BN>::kBBytes;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + kStages * kABytes;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sB + kStages * kBBytes);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kStages + 2);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + kStages);
+  const uint32_t accum_bar = smem_u32(bars + 2 * kStages), drain_bar = smem_u32(bars + 2 * kStages + 1);
+  auto full_bar = [&](int s) { return full0 + 8u * s; };
+  auto empty_bar = [&](int s) { return empty0 + 8u * s; };
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int m0 = blockIdx.x * kBM, n0 = blockIdx.y * BN;
+  const int KB = (p.K + kBK - 1) / kBK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(full_bar(s), GATHER ? 1 + 128 : 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    mbar_init(accum_bar, 1);
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+    fence_proxy_async_smem();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), BN);
+    tmem_relinquish();
+  }
+  if (threadIdx.x == 0) {
+    prefetch_tmap(&tmB);
+    if (!GATHER) prefetch_tmap(&tmA);
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer
+      int kb = 0;
+      for (; kb < KB; ++kb) {
+        const int s = kb % kStages, r = kb / kStages;
+        if (!mbar_wait_bounded(empty_bar(s), (r & 1) ^ 1, abort_flag, p.err)) break;
+        mbar_arrive_expect_tx(full_bar(s), kBBytes + (GATHER ? 0 : kABytes));
+        tma_load_2d(smem_u32(sB + s * kBBytes), &tmB, full_bar(s), kb * kBK, n0);
+        if (!GATHER) tma_load_2d(smem_u32(sA + s * kABytes), &tmA, full_bar(s), kb * kBK, m0);
+      }
+      if (kb < KB) {
+        // aborted: let the loads already issued land before the CTA exits
+        volatile int no_abort = 0;
+        for (int j = (kb > kStages ? kb - kStages : 0); j < kb; ++j)
+          mbar_wait_bounded(full_bar(j % kStages), (j / kStages) & 1, &no_abort, nullptr);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer
+      constexpr uint32_t idesc = idesc_f16(sizeof(T) == 2 && !std::is_same<T, __half>::value ? 1 : 0, kBM, BN);
+      for (int kb = 0; kb < KB; ++kb) {
+        const int s = kb % kStages, r = kb / kStages;
+        if (!mbar_wait_bounded(full_bar(s), r & 1, abort_flag, p.err)) break;
+        tc_fence_after();
+        const uint64_t ad = smem_desc_sw128(smem_u32(sA + s * kABytes));
+        const uint64_t bd = smem_desc_sw128(smem_u32(sB + s * kBBytes));
+#pragma unroll
+        for (int k = 0; k < kBK / 16; ++k)
+          tc_mma_f16(tmem, ad + 2ull * k, bd + 2ull * k, idesc, (kb | k) != 0);
+        tc_commit(empty_bar(s));
+      }
+      tc_commit(accum_bar);  // fires once every MMA issued above has completed
+    }
+  } else {
+    const int t = threadIdx.x - 64;  // 0..127
+    if (GATHER) {
+      // ---------------- implicit im2col gather of A (row t of the tile)
+      const int m = m0 + t;
+      const bool mvalid = m < p.M;
+      int img = 0, oy = 0, ox = 0;
+      if (mvalid) {
+        const int hw = p.Ho * p.Wo;
+        img = m / hw;
+        const int rem = m - img * hw;
+        oy = rem / p.Wo;
+        ox = rem - oy * p.Wo;
+      }
+      const int iy0 = oy * p.stride - p.pad, ix0 = ox * p.stride - p.pad;
+      const T* xb = static_cast<const T*>(p.x) + (int64_t)img * p.H * p.Wd * p.C;
+      const uint32_t row_off = (uint32_t)((t >> 3) * 1024 + (t & 7) * 128);
+      int kb = 0;
+      for (; kb < KB; ++kb) {
+        const int s = kb % kStages, r = kb / kStages;
+        if (!mbar_wait_bounded(empty_bar(s), (r & 1) ^ 1, abort_flag, p.err)) break;
+        const uint32_t dst_row = smem_u32(sA + s * kABytes) + row_off;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int k = kb * kBK + j * 8;
+          bool valid = mvalid && k < p.K;
+          const T* src = static_cast<const T*>(p.x);
+          if (valid) {
+            const int tap = k / p.C;
+            const int c = k - tap * p.C;
+            const int ry = tap / p.kw;
+            const int rx = tap - ry * p.kw;
+            const int iy = iy0 + ry, ix = ix0 + rx;
+            valid = (unsigned)iy < (unsigned)p.H && (unsigned)ix < (unsigned)p.Wd;
+            if (valid) src = xb + ((int64_t)iy * p.Wd + ix) * p.C + c;
+          }
+          cp_async_16(dst_row + (uint32_t)((j ^ (t & 7)) << 4), src, valid);
+        }
+        cp_async_commit();
+        if (kb >= kLag) {
+          cp_async_wait<kLag>();
+          fence_proxy_async_smem();
+          mbar_arrive(full_bar((kb - kLag) % kStages));
+        }
+      }
+      cp_async_wait<0>();
+      fence_proxy_async_smem();
+      for (int j = (kb > kLag ? kb - kLag : 0); j < kb; ++j) mbar_arrive(full_bar(j % kStages));
+    }
+    // ---------------- epilogue
+    const int q = warp & 3;
+    const int row = q * 32 + lane;
+    const int m = m0 + row;
+    const bool ok = mbar_wait_bounded(accum_bar, 0, abort_flag, p.err);
+    tc_fence_after();
+    if (ok) {
+      const T* bias = static_cast<const T*>(p.e.bias);
+      const T* res = static_cast<const T*>(p.e.res);
+      T* y = static_cast<T*>(p.y);
+      const bool vec_ok = ((p.ldy | n0) % 8 == 0) && (!res || ((p.e.ldr | n0) % 8 == 0));
+#pragma unroll 1
+      for (int c0 = 0; c0 < BN; c0 += 32) {
+        uint32_t r[32];
+        tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)c0, r);
+        tmem_ld_wait();
+        const int n = n0 + c0;
+        if (m >= p.M || n >= p.N) continue;
+        float v[32];
+        if (vec_ok && n + 32 <= p.N) {
+          float rv[32];
+          if (res) {
+            uint4 pk[4];
+            const uint4* rp = reinterpret_cast<const uint4*>(res + (int64_t)m * p.e.ldr + n);
+#pragma unroll
+            for (int qq = 0; qq < 4; ++qq) pk[qq] = rp[qq];
+            const T* re = reinterpret_cast<const T*>(pk);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) rv[j] = to_f<T>(re[j]);
+          }
+#pragma unroll
+          for (int j = 0; j < 32; ++j)
+            v[j] = epilogue(__uint_as_float(r[j]), to_f<T>(bias[n + j]), res ? rv[j] : 0.f, res != nullptr,
+                            p.e.act, p.e.res_post);
+          store_row32<T>(y + (int64_t)m * p.ldy + n, v);
+        } else {
+          for (int j = 0; j < 32 && n + j < p.N; ++j) {
+            const float rv = res ? to_f<T>(res[(int64_t)m * p.e.ldr + n + j]) : 0.f;
+            y[(int64_t)m * p.ldy + n + j] = from_f<T>(
+                epilogue(__uint_as_float(r[j]), to_f<T>(bias[n + j]), rv, res != nullptr, p.e.act, p.e.res_post));
+          }
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, BN);
+  }
+}
+
+// ------------------------------------------------------------ host side
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  });
+  return fn;
+}
+
+int make_tmap(CUtensorMap* m, int dtype, const void* base, uint64_t inner, uint64_t rows, uint64_t row_stride_bytes,
+              uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (!fn) SN_FAIL(SWAPNET_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+  if (((uintptr_t)base & 15) || (row_stride_bytes & 15))
+    SN_FAIL(SWAPNET_ERR_MISALIGNED, "TMA operand must be 16-byte aligned with a 16-byte multiple row stride");
+  const cuuint64_t dims[2] = {inner, rows};
+  const cuuint64_t strides[1] = {row_stride_bytes};
+  const cuuint32_t box[2] = {(cuuint32_t)kBK, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  const CUresult r = fn(m, dtype == SWAPNET_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16,
+                        2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) SN_FAIL(SWAPNET_ERR_CUDA, "cuTensorMapEncodeTiled failed (" + std::to_string((int)r) + ")");
+  return SWAPNET_OK;
+}
+
+template <typename T, int BN, bool GATHER>
+int launch_inst(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) {
+  static bool attr_done = false;  // per instantiation
+  auto kern = tc_gemm_kernel<T, BN, GATHER>;
+  if (!attr_done) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<BN>::kSmem) != cudaSuccess)
+      SN_FAIL(SWAPNET_ERR_CUDA, "cudaFuncSetAttribute failed");
+    attr_done = true;
+  }
+  TcArgs a;
+  std::memset(&a, 0, sizeof(a));
+  a.M = g.M; a.N = g.N; a.K = g.K;
+  a.x = g.A;
+  a.H = g.H; a.Wd = g.Wd; a.C = g.C; a.Ho = g.Ho; a.Wo = g.Wo;
+  a.kh = g.kh; a.kw = g.kw; a.stride = g.stride; a.pad = g.pad;
+  a.e = g.e; a.y = g.y; a.ldy = g.ldy; a.err = err;
+  const dim3 grid((g.M + kBM - 1) / kBM, (g.N + BN - 1) / BN);
+  kern<<<grid, kThreads, Cfg<BN>::kSmem, s>>>(pl.tmA, pl.tmB, a);
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) SN_FAIL(SWAPNET_ERR_CUDA, std::string("tcgen05 GEMM launch: ") + cudaGetErrorString(e));
+  return SWAPNET_OK;
+}
+
+}  // namespace
+
+int tc_prepare(const TcGemm& g, TcPlan* p) {
+  std::memset(p, 0, sizeof(*p));
+  if (g.dtype != SWAPNET_F16 && g.dtype != SWAPNET_BF16) SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "tcgen05 path: fp16/bf16 only");
+  if (g.K % 8) SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "tcgen05 path: K must be a multiple of 8");
+  if (g.conv && g.C % 8) SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "tcgen05 conv: channels must be a multiple of 8");
+  if ((uintptr_t)g.y % 2) SN_FAIL(SWAPNET_ERR_MISALIGNED, "unaligned output");
+  if (g.N <= 64) {
+    p->bn = 64;
+  } else {
+    const int64_t tiles128 = (int64_t)((g.M + kBM - 1) / kBM) * ((g.N + 127) / 128);
+    p->bn = tiles128 < 148 ? 64 : 128;
+  }
+  int rc = make_tmap(&p->tmB, g.dtype, g.W, (uint64_t)g.K, (uint64_t)g.N, (uint64_t)g.K * 2, (uint32_t)p->bn);
+  if (rc) return rc;
+  if (!g.conv && g.A) {
+    rc = make_tmap(&p->tmA, g.dtype, g.A, (uint64_t)g.K, (uint64_t)g.M, (uint64_t)g.lda * 2, (uint32_t)kBM);
+    if (rc) return rc;
+  }
+  p->ready = 1;
+  return SWAPNET_OK;
+}
+
+int launch_tc_gemm(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) {
+  if (!pl.ready) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "tcgen05 GEMM not prepared");
+  const bool bf = g.dtype == SWAPNET_BF16;
+  if (g.conv) {
+    if (pl.bn == 64) return bf ? launch_inst<__nv_bfloat16, 64, true>(g, pl, err, s) : launch_inst<__half, 64, true>(g, pl, err, s);
+    return bf ? launch_inst<__nv_bfloat16, 128, true>(g, pl, err, s) : launch_inst<__half, 128, true>(g, pl, err, s);
+  }
+  if (pl.bn == 64) return bf ? launch_inst<__nv_bfloat16, 64, false>(g, pl, err, s) : launch_inst<__half, 64, false>(g, pl, err, s);
+  return bf ? launch_inst<__nv_bfloat16, 128, false>(g, pl, err, s) : launch_inst<__half, 128, false>(g, pl, err, s);
+}
+
+int tc_error_word(int** ptr) {
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_tc_err) != cudaSuccess) SN_FAIL(SWAPNET_ERR_CUDA, "cudaGetSymbolAddress failed");
+  *ptr = static_cast<int*>(p);
+  return SWAPNET_OK;
+}
+
+}  // namespace swapnet

@@ -1,0 +1,74 @@
+// Host-side launchers of the layer and swap kernels (internal interface).
+// Every launcher validates what its kernel assumes (alignment, sizes) and
+// returns a swapnet_status; it never synchronises.
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cstdint>
+
+namespace swapnet {
+
+// Epilogue operands shared by linear and conv layers.
+struct Epi {
+  const void* bias;  // [n] (a piece's own slice for split linear layers)
+  const void* res;   // residual, row stride ldr elements, or nullptr
+  int64_t ldr;
+  int act;
+  int res_post;
+};
+
+// y[m, col0 + o] (row stride ldy) = epi(sum_k x[m,k] W[o,k]) for o < N,
+// M <= 16.  fp32 / fp16 / bf16; fixed-order reduction (deterministic).
+int launch_linear_skinny(int dtype, const void* x, int M, int K, const void* W, int N, const Epi& e, void* y,
+                         int64_t ldy, cudaStream_t s);
+
+// Direct convolution (SIMT) for any channel count; NHWC in, NHWC out.
+int launch_conv_direct(int dtype, const void* x, int n, int h, int w, int cin, const void* W, int cout, int kh,
+                       int kw, int stride, int pad, int oh, int ow, const Epi& e, void* y, cudaStream_t s);
+
+int launch_maxpool(int dtype, const void* x, int n, int h, int w, int c, int kh, int kw, int stride, int pad,
+                   int oh, int ow, void* y, cudaStream_t s);
+int launch_gap(int dtype, const void* x, int n, int h, int w, int c, void* y, cudaStream_t s);
+int launch_upsample2x(int dtype, const void* x, int n, int h, int w, int c, void* y, cudaStream_t s);
+int launch_concat(int dtype, const void* a, int ca, const void* b, int cb, int64_t pixels, void* y,
+                  cudaStream_t s);
+
+// Zero-copy swap: copy segments from mapped host memory (device aliases)
+// into the arena with 16-byte vector loads/stores.
+struct ZcSeg {
+  const void* src;  // device alias of page-locked host memory, 16-byte aligned
+  void* dst;        // arena, 16-byte aligned
+  uint64_t bytes;
+};
+int launch_zerocopy(const ZcSeg* segs, int nseg, int ctas, cudaStream_t s);
+
+// tcgen05 GEMM / implicit-GEMM convolution (fp16 or bf16, fp32 accumulate).
+struct TcGemm {
+  int dtype;          // SWAPNET_F16 or SWAPNET_BF16
+  int M, N, K;
+  // B operand: weights [N][K] row-major (K contiguous)
+  const void* W;
+  // A operand: either a row-major [M][K] matrix (conv == 0) ...
+  const void* A;
+  int64_t lda;
+  // ... or the implicit im2col of an NHWC input (conv == 1)
+  int conv;
+  int H, Wd, C, Ho, Wo, kh, kw, stride, pad;
+  Epi e;
+  void* y;
+  int64_t ldy;
+};
+// Pre-encoded descriptors of one GEMM (built once per layer at load time).
+struct TcPlan {
+  CUtensorMap tmA;  // valid when conv == 0
+  CUtensorMap tmB;
+  int bn;           // N tile
+  int ready;
+};
+int tc_prepare(const TcGemm& g, TcPlan* p);
+int launch_tc_gemm(const TcGemm& g, const TcPlan& p, int* dev_err, cudaStream_t s);
+
+// Device error word of the tcgen05 kernels (bounded waits).
+int tc_error_word(int** ptr);
+
+}  // namespace swapnet

@@ -1,0 +1,668 @@
+// Host-side planning: model analysis (Sec. 6.1 model information table),
+// activation workspace, partition units, the delay model (Sec. 6.1), the
+// partition search (Sec. 6.2.2, Eq. 2-4) and the multi-DNN split (Eq. 1).
+// No device work happens here.
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <memory>
+#include <new>
+
+#include "internal.h"
+
+namespace swapnet {
+
+int dtype_size(int dtype) {
+  switch (dtype) {
+    case SWAPNET_F32: return 4;
+    case SWAPNET_F16: return 2;
+    case SWAPNET_BF16: return 2;
+    default: return 0;
+  }
+}
+
+static uint64_t mul_div_ceil(uint64_t a, uint64_t b, uint64_t d) {
+  unsigned __int128 p = (unsigned __int128)a * b;
+  return (uint64_t)((p + d - 1) / d);
+}
+
+// ------------------------------------------------------------ model analysis
+int analyse_model(const swapnet_model_desc* desc, Model* m) {
+  if (!desc || !desc->layers || desc->n_layers <= 0) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "empty model descriptor");
+  m->dtype = desc->dtype;
+  m->es = dtype_size(desc->dtype);
+  if (!m->es) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "unknown dtype");
+  if (desc->in_n <= 0 || desc->in_h <= 0 || desc->in_w <= 0 || desc->in_c <= 0)
+    SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad input shape");
+  m->in_n = desc->in_n; m->in_h = desc->in_h; m->in_w = desc->in_w; m->in_c = desc->in_c;
+  m->in_bytes = (uint64_t)m->in_n * m->in_h * m->in_w * m->in_c * m->es;
+  const int nl = desc->n_layers;
+  m->L.assign(nl, Layer{});
+  m->n_tensors = 0;
+  m->tensor_raw.clear();
+  m->weight_bytes = 0;
+  for (int i = 0; i < nl; ++i) {
+    Layer& L = m->L[i];
+    L.d = desc->layers[i];
+    const swapnet_layer& d = L.d;
+    auto dims_of = [&](int src, int* n, int* h, int* w, int* c) -> bool {
+      if (src == SWAPNET_SRC_INPUT) { *n = m->in_n; *h = m->in_h; *w = m->in_w; *c = m->in_c; return true; }
+      if (src < 0 || src >= i) return false;
+      const Layer& P = m->L[src];
+      *n = P.on; *h = P.oh; *w = P.ow; *c = P.oc;
+      return true;
+    };
+    if (!dims_of(d.src0, &L.n, &L.h, &L.w, &L.c))
+      SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": bad src0");
+    L.c1 = 0;
+    L.n_tensors = 0;
+    L.tbytes[0] = L.tbytes[1] = 0;
+    L.flops = 0;
+    const uint64_t es = m->es;
+    switch (d.op) {
+      case SWAPNET_OP_CONV2D: {
+        if (d.cin != L.c || d.cout <= 0 || d.kh <= 0 || d.kw <= 0 || d.stride <= 0 || d.pad < 0)
+          SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": bad conv parameters");
+        L.on = L.n;
+        L.oh = (L.h + 2 * d.pad - d.kh) / d.stride + 1;
+        L.ow = (L.w + 2 * d.pad - d.kw) / d.stride + 1;
+        L.oc = d.cout;
+        if (L.oh <= 0 || L.ow <= 0) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": empty output");
+        L.n_tensors = 2;
+        L.tbytes[0] = (uint64_t)d.cout * d.kh * d.kw * d.cin * es;
+        L.tbytes[1] = (uint64_t)d.cout * es;
+        L.flops = 2ull * L.on * L.oh * L.ow * (uint64_t)d.cout * d.cin * d.kh * d.kw;
+        break;
+      }
+      case SWAPNET_OP_LINEAR: {
+        if ((int64_t)d.cin != (int64_t)L.h * L.w * L.c || d.cout <= 0)
+          SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": linear in-features mismatch");
+        L.on = L.n; L.oh = 1; L.ow = 1; L.oc = d.cout;
+        L.n_tensors = 2;
+        L.tbytes[0] = (uint64_t)d.cout * d.cin * es;
+        L.tbytes[1] = (uint64_t)d.cout * es;
+        L.flops = 2ull * L.n * (uint64_t)d.cin * d.cout;
+        break;
+      }
+      case SWAPNET_OP_MAXPOOL: {
+        if (d.kh <= 0 || d.kw <= 0 || d.stride <= 0 || d.pad < 0 || 2 * d.pad >= d.kh + 1 + d.kh || d.pad >= d.kh || d.pad >= d.kw)
+          SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": bad pool window");
+        L.on = L.n;
+        L.oh = (L.h + 2 * d.pad - d.kh) / d.stride + 1;
+        L.ow = (L.w + 2 * d.pad - d.kw) / d.stride + 1;
+        L.oc = L.c;
+        if (L.oh <= 0 || L.ow <= 0) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": empty output");
+        break;
+      }
+      case SWAPNET_OP_GAP:
+        L.on = L.n; L.oh = 1; L.ow = 1; L.oc = L.c;
+        break;
+      case SWAPNET_OP_UPSAMPLE2X:
+        L.on = L.n; L.oh = 2 * L.h; L.ow = 2 * L.w; L.oc = L.c;
+        break;
+      case SWAPNET_OP_CONCAT: {
+        int n1, h1, w1, c1;
+        if (!dims_of(d.src1, &n1, &h1, &w1, &c1) || n1 != L.n || h1 != L.h || w1 != L.w)
+          SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": concat operands mismatch");
+        L.c1 = c1;
+        L.on = L.n; L.oh = L.h; L.ow = L.w; L.oc = L.c + c1;
+        break;
+      }
+      default:
+        SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": unknown op");
+    }
+    if (d.op != SWAPNET_OP_CONCAT && d.src1 != SWAPNET_SRC_NONE)
+      SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": src1 only for concat");
+    if (d.res != SWAPNET_SRC_NONE) {
+      if (d.op != SWAPNET_OP_CONV2D && d.op != SWAPNET_OP_LINEAR)
+        SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": residual only on conv/linear");
+      if (d.res < 0 || d.res >= i) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": bad residual");
+      const Layer& R = m->L[d.res];
+      if (R.on != L.on || R.oh != L.oh || R.ow != L.ow || R.oc != L.oc)
+        SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": residual shape mismatch");
+    }
+    if (d.act < SWAPNET_ACT_NONE || d.act > SWAPNET_ACT_LEAKY)
+      SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": bad activation");
+    if (d.t_ex_ns < 0) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "negative t_ex_ns");
+    L.first_tensor = m->n_tensors;
+    for (int t = 0; t < L.n_tensors; ++t) {
+      m->tensor_raw.push_back(L.tbytes[t]);
+      m->weight_bytes += align_up(L.tbytes[t]);
+    }
+    m->n_tensors += L.n_tensors;
+    L.out_bytes = (uint64_t)L.on * L.oh * L.ow * L.oc * es;
+  }
+  // liveness: last reader of every output
+  for (int i = 0; i < nl; ++i) m->L[i].last_use = i;
+  for (int j = 0; j < nl; ++j) {
+    const swapnet_layer& d = m->L[j].d;
+    for (int s : {d.src0, d.src1, d.res})
+      if (s >= 0) m->L[s].last_use = std::max(m->L[s].last_use, j);
+  }
+  // outputs go to the output buffer, in layer order
+  uint64_t cur = 0;
+  for (int i = 0; i < nl; ++i) {
+    Layer& L = m->L[i];
+    L.out_off = -1;
+    if (L.d.is_output) { L.out_off = (int64_t)cur; cur += align_up(L.out_bytes); }
+  }
+  if (cur == 0) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "model has no output layer");
+  m->out_bytes = cur;
+  // workspace: first fit over live intervals
+  struct Placed { int lo, hi; uint64_t off, size; };
+  std::vector<Placed> placed;
+  uint64_t ws = 0;
+  for (int i = 0; i < nl; ++i) {
+    Layer& L = m->L[i];
+    L.ws_off = -1;
+    if (L.d.is_output) continue;
+    const uint64_t size = align_up(L.out_bytes);
+    std::vector<const Placed*> conf;
+    for (const Placed& p : placed)
+      if (p.lo <= L.last_use && i <= p.hi) conf.push_back(&p);
+    std::vector<uint64_t> cand{0};
+    for (const Placed* p : conf) cand.push_back(p->off + p->size);
+    std::sort(cand.begin(), cand.end());
+    uint64_t chosen = 0;
+    for (uint64_t o : cand) {
+      bool ok = true;
+      for (const Placed* p : conf)
+        if (!(o + size <= p->off || p->off + p->size <= o)) { ok = false; break; }
+      if (ok) { chosen = o; break; }
+    }
+    L.ws_off = (int64_t)chosen;
+    placed.push_back(Placed{i, L.last_use, chosen, size});
+    ws = std::max(ws, chosen + size);
+  }
+  m->ws_bytes = ws;
+  return SWAPNET_OK;
+}
+
+static int64_t unit_tex(const Model& m, const swapnet_options& opt, const Layer& L, uint64_t flops, int rows) {
+  if (L.d.t_ex_ns > 0) {
+    if (L.d.op == SWAPNET_OP_LINEAR && rows != L.d.cout)
+      return (int64_t)ceil_div_u((uint64_t)L.d.t_ex_ns * rows, (uint64_t)L.d.cout);
+    return L.d.t_ex_ns;
+  }
+  (void)m;
+  return (int64_t)mul_div_ceil(opt.gamma_as_per_flop, flops, 1000000000ull);
+}
+
+int make_units(const Model& m, const swapnet_options& opt, uint64_t slot, std::vector<Unit>* out) {
+  out->clear();
+  const uint64_t es = m.es;
+  for (int li = 0; li < (int)m.L.size(); ++li) {
+    const Layer& L = m.L[li];
+    uint64_t size = 0;
+    for (int t = 0; t < L.n_tensors; ++t) size += align_up(L.tbytes[t]);
+    if (size <= slot) {
+      Unit u{};
+      u.layer = li; u.row0 = 0; u.rows = (L.d.op == SWAPNET_OP_LINEAR) ? L.d.cout : 0;
+      u.depth = L.n_tensors; u.bytes = size; u.flops = L.flops;
+      u.t_ex = unit_tex(m, opt, L, L.flops, u.rows);
+      u.nt = L.n_tensors;
+      for (int t = 0; t < L.n_tensors; ++t) {
+        u.tidx[t] = L.first_tensor + t; u.toff[t] = 0; u.tlen[t] = L.tbytes[t];
+      }
+      out->push_back(u);
+      continue;
+    }
+    if (L.d.op != SWAPNET_OP_LINEAR)
+      SN_FAIL(SWAPNET_ERR_INFEASIBLE, "layer " + std::to_string(li) + " (" + std::to_string(size) +
+                                          " B) does not fit a slot of " + std::to_string(slot) + " B");
+    const uint64_t K = L.d.cin, N = L.d.cout;
+    auto piece_bytes = [&](uint64_t r) { return align_up(r * K * es) + align_up(r * es); };
+    uint64_t rmax = 0;
+    for (uint64_t r = 128; r <= N + 127 && piece_bytes(r) <= slot; r += 128) rmax = r;
+    if (rmax == 0)
+      SN_FAIL(SWAPNET_ERR_INFEASIBLE, "layer " + std::to_string(li) + ": 128 output features exceed a slot");
+    const uint64_t np = ceil_div_u(N, rmax);
+    const uint64_t rr = ceil_div_u(ceil_div_u(N, np), 128) * 128;
+    for (uint64_t r0 = 0; r0 < N; r0 += rr) {
+      const uint64_t rows = std::min(rr, N - r0);
+      Unit u{};
+      u.layer = li; u.row0 = (int)r0; u.rows = (int)rows; u.depth = 2;
+      u.bytes = piece_bytes(rows);
+      u.flops = 2ull * L.n * K * rows;
+      u.t_ex = unit_tex(m, opt, L, u.flops, (int)rows);
+      u.nt = 2;
+      u.tidx[0] = L.first_tensor; u.toff[0] = r0 * K * es; u.tlen[0] = rows * K * es;
+      u.tidx[1] = L.first_tensor + 1; u.toff[1] = r0 * es; u.tlen[1] = rows * es;
+      out->push_back(u);
+    }
+  }
+  return SWAPNET_OK;
+}
+
+static Block make_block(const std::vector<Unit>& us, int a, int b, const swapnet_options& opt) {
+  Block B{};
+  B.u0 = a; B.u1 = b;
+  for (int u = a; u < b; ++u) { B.bytes += us[u].bytes; B.depth += us[u].depth; B.t_ex += us[u].t_ex; }
+  B.t_in = (int64_t)mul_div_ceil(opt.alpha_as_per_byte, B.bytes, 1000000000ull) +
+           (int64_t)(opt.beta_ns_per_tensor * B.depth);
+  B.t_out = (int64_t)(opt.eta_ns_per_tensor * B.depth);
+  return B;
+}
+
+int64_t pipeline_ns(const std::vector<Block>& b, int slots) {
+  int64_t C = 0, E = 0;
+  std::vector<int64_t> R;
+  for (size_t k = 0; k < b.size(); ++k) {
+    const int64_t gate = ((int64_t)k - slots >= 0) ? R[k - slots] : 0;
+    C = std::max(C, gate) + b[k].t_in;
+    E = std::max(E, C) + b[k].t_ex;
+    R.push_back(E + b[k].t_out);
+  }
+  return E;
+}
+
+int64_t eq4_ns(const std::vector<Block>& b) {
+  const size_t n = b.size();
+  int64_t total = 0, ov_prev = 0;
+  for (size_t i = 1; i < n; ++i) {
+    const int64_t tin_next = (i + 1 < n) ? b[i + 1].t_in : 0;
+    const int64_t ov = (b[i - 1].t_out + tin_next) - (b[i].t_ex + ov_prev);
+    total += std::max<int64_t>(ov, 0);
+    ov_prev = ov;
+  }
+  return total;
+}
+
+uint64_t resident_latency_ns(const Model& m, const swapnet_options& opt) {
+  uint64_t t = 0;
+  for (const Layer& L : m.L)
+    t += (uint64_t)unit_tex(m, opt, L, L.flops, L.d.op == SWAPNET_OP_LINEAR ? L.d.cout : 0);
+  return t;
+}
+
+void finalize_blocks(swapnet_plan* p, const std::vector<uint32_t>& cuts) {
+  p->cuts = cuts;
+  p->blocks.clear();
+  std::vector<uint32_t> b{0};
+  b.insert(b.end(), cuts.begin(), cuts.end());
+  b.push_back((uint32_t)p->units.size());
+  const int slots = p->resident ? 1 : p->opt.slots;
+  for (size_t k = 0; k + 1 < b.size(); ++k) {
+    Block B = make_block(p->units, (int)b[k], (int)b[k + 1], p->opt);
+    B.slot = (int)(k % slots);
+    // slot layout: tensors in unit order, 256-byte aligned
+    uint64_t off = 0;
+    for (int u = B.u0; u < B.u1; ++u) {
+      Unit& U = p->units[u];
+      for (int t = 0; t < U.nt; ++t) { U.slot_off[t] = off; off += align_up(U.tlen[t]); }
+    }
+    p->blocks.push_back(B);
+  }
+  if (p->resident) {
+    int64_t t = 0;
+    for (const Unit& u : p->units) t += u.t_ex;
+    p->predicted = t;
+  } else {
+    p->predicted = p->opt.objective == 0 ? pipeline_ns(p->blocks, p->opt.slots) : eq4_ns(p->blocks);
+  }
+}
+
+// ----------------------------------------------------------- partition search
+namespace {
+
+struct State {
+  int64_t v[4];     // C, E, R_{k-1}, R_k (m = 2) or C, E, R_k, 0 (m = 1)
+  int nblocks;
+  int prev_j;       // boundary of the previous state
+  int prev_idx;     // index in the previous frontier
+};
+
+struct Search {
+  const std::vector<Unit>& us;
+  const swapnet_options& opt;
+  uint64_t slot;
+  int slots;
+  std::vector<std::vector<State>> front;
+
+  Search(const std::vector<Unit>& u, const swapnet_options& o, uint64_t s)
+      : us(u), opt(o), slot(s), slots(o.slots) {}
+
+  std::vector<uint32_t> cuts_of(int j, int idx) const {
+    std::vector<uint32_t> c;
+    while (j > 0) {
+      const State& s = front[j][idx];
+      if (s.prev_j > 0) c.push_back((uint32_t)s.prev_j);
+      const int pj = s.prev_j, pi = s.prev_idx;
+      j = pj; idx = pi;
+    }
+    std::reverse(c.begin(), c.end());
+    return c;
+  }
+
+  // a is preferred-or-equal to b on ties (fewer blocks, then lexicographic cuts)
+  bool tie_le(int j, int ia, int ib) const {
+    const State& a = front[j][ia];
+    const State& b = front[j][ib];
+    if (a.nblocks != b.nblocks) return a.nblocks < b.nblocks;
+    return cuts_of(j, ia) <= cuts_of(j, ib);
+  }
+
+  static bool le_all(const State& a, const State& b) {
+    for (int t = 0; t < 4; ++t)
+      if (a.v[t] > b.v[t]) return false;
+    return true;
+  }
+
+  void insert(int j, const State& s) {
+    std::vector<State>& F = front[j];
+    F.push_back(s);
+    const int is = (int)F.size() - 1;
+    for (int t = 0; t < is; ++t)
+      if (le_all(F[t], F[is]) && tie_le(j, t, is)) { F.pop_back(); return; }
+    std::vector<State> keep;
+    keep.reserve(F.size());
+    for (int t = 0; t < is; ++t)
+      if (!(le_all(F[is], F[t]) && tie_le(j, is, t))) keep.push_back(F[t]);
+    keep.push_back(F[is]);
+    F.swap(keep);
+  }
+
+  State step(const State& s, const Block& B) const {
+    State r{};
+    if (slots == 2) {
+      const int64_t C = std::max(s.v[0], s.v[2]) + B.t_in;
+      const int64_t E = std::max(s.v[1], C) + B.t_ex;
+      r.v[0] = C; r.v[1] = E; r.v[2] = s.v[3]; r.v[3] = E + B.t_out;
+    } else {
+      const int64_t C = std::max(s.v[0], s.v[2]) + B.t_in;
+      const int64_t E = std::max(s.v[1], C) + B.t_ex;
+      r.v[0] = C; r.v[1] = E; r.v[2] = E + B.t_out; r.v[3] = 0;
+    }
+    r.nblocks = s.nblocks + 1;
+    return r;
+  }
+};
+
+}  // namespace
+
+static int search_pipeline(swapnet_plan* p, std::vector<uint32_t>* best_cuts) {
+  const int U = (int)p->units.size();
+  Search S(p->units, p->opt, p->slot);
+  S.front.assign(U + 1, {});
+  State s0{};
+  s0.prev_j = -1; s0.prev_idx = -1; s0.nblocks = 0;
+  S.front[0].push_back(s0);
+  // frontier states of boundary j only get children once j is final
+  for (int j = 0; j < U; ++j) {
+    // rebuild the frontier list copy, since insert() on j' > j does not touch it
+    for (int idx = 0; idx < (int)S.front[j].size(); ++idx) {
+      uint64_t bytes = 0;
+      for (int j2 = j + 1; j2 <= U; ++j2) {
+        bytes += p->units[j2 - 1].bytes;
+        if (bytes > p->slot) break;
+        Block B = make_block(p->units, j, j2, p->opt);
+        State c = S.step(S.front[j][idx], B);
+        c.prev_j = j; c.prev_idx = idx;
+        S.insert(j2, c);
+      }
+    }
+  }
+  const std::vector<State>& F = S.front[U];
+  if (F.empty()) SN_FAIL(SWAPNET_ERR_INFEASIBLE, "no feasible partition");
+  int best = 0;
+  for (int i = 1; i < (int)F.size(); ++i) {
+    if (F[i].v[1] < F[best].v[1] || (F[i].v[1] == F[best].v[1] && S.tie_le(U, i, best) &&
+                                     !S.tie_le(U, best, i)))
+      best = i;
+  }
+  *best_cuts = S.cuts_of(U, best);
+  return SWAPNET_OK;
+}
+
+static int search_exhaustive_eq4(swapnet_plan* p, std::vector<uint32_t>* best_cuts) {
+  const int U = (int)p->units.size();
+  if (U > 24) SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "objective 1 (Eq. 4) search is exhaustive: at most 24 units");
+  bool found = false;
+  int64_t bo = 0;
+  std::vector<uint32_t> bc;
+  for (uint64_t mask = 0; mask < (1ull << (U - 1)); ++mask) {
+    std::vector<uint32_t> cuts;
+    for (int c = 1; c < U; ++c)
+      if ((mask >> (c - 1)) & 1) cuts.push_back((uint32_t)c);
+    std::vector<uint32_t> b{0};
+    b.insert(b.end(), cuts.begin(), cuts.end());
+    b.push_back((uint32_t)U);
+    std::vector<Block> blocks;
+    bool ok = true;
+    for (size_t k = 0; k + 1 < b.size(); ++k) {
+      Block B = make_block(p->units, (int)b[k], (int)b[k + 1], p->opt);
+      if (B.bytes > p->slot) { ok = false; break; }
+      blocks.push_back(B);
+    }
+    if (!ok) continue;
+    const int64_t o = eq4_ns(blocks);
+    if (!found || o < bo || (o == bo && (cuts.size() < bc.size() || (cuts.size() == bc.size() && cuts < bc)))) {
+      found = true; bo = o; bc = cuts;
+    }
+  }
+  if (!found) SN_FAIL(SWAPNET_ERR_INFEASIBLE, "no feasible partition");
+  *best_cuts = bc;
+  return SWAPNET_OK;
+}
+
+static int check_options(const swapnet_options& o) {
+  if (o.slots != 1 && o.slots != 2) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "slots must be 1 or 2");
+  if (o.objective != 0 && o.objective != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "objective must be 0 or 1");
+  if (o.swap_variant < 0 || o.swap_variant > 2) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad swap_variant");
+  if (o.zc_ctas < 0 || o.zc_ctas > 4096) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad zc_ctas");
+  return SWAPNET_OK;
+}
+
+static int prepare(const swapnet_model_desc* desc, uint64_t budget, const swapnet_options* opt,
+                   std::unique_ptr<swapnet_plan>* out) {
+  std::unique_ptr<swapnet_plan> p(new (std::nothrow) swapnet_plan());
+  if (!p) SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
+  if (opt) p->opt = *opt; else swapnet_default_options(&p->opt);
+  int rc = check_options(p->opt);
+  if (rc) return rc;
+  rc = analyse_model(desc, &p->model);
+  if (rc) return rc;
+  p->budget = budget;
+  const uint64_t ws = p->model.ws_bytes;
+  if (p->opt.activations_in_budget && budget <= ws)
+    SN_FAIL(SWAPNET_ERR_INFEASIBLE, "budget does not cover the activation workspace");
+  p->arena = p->opt.activations_in_budget ? budget - ws : budget;
+  p->slot = (p->arena / (uint64_t)p->opt.slots) / kAlign * kAlign;
+  rc = make_units(p->model, p->opt, p->slot, &p->units);
+  if (rc) return rc;
+  *out = std::move(p);
+  return SWAPNET_OK;
+}
+
+}  // namespace swapnet
+
+using namespace swapnet;
+
+extern "C" {
+
+void swapnet_default_options(swapnet_options* o) {
+  if (!o) return;
+  std::memset(o, 0, sizeof(*o));
+  o->slots = 2;
+  o->activations_in_budget = 0;
+  o->swap_variant = SWAPNET_SWAP_AUTO;
+  o->objective = 0;
+  o->alpha_as_per_byte = 2500000;  // 400 GB/s
+  o->beta_ns_per_tensor = 2000;
+  o->gamma_as_per_flop = 2000;     // 500 TFLOP/s
+  o->eta_ns_per_tensor = 0;
+  o->zc_ctas = 0;
+}
+
+int swapnet_partition(const swapnet_model_desc* desc, uint64_t budget, const swapnet_options* opt,
+                      swapnet_plan** out) {
+  if (!out) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null out_plan");
+  try {
+    std::unique_ptr<swapnet_plan> p;
+    int rc = prepare(desc, budget, opt, &p);
+    if (rc) return rc;
+    std::vector<uint32_t> cuts;
+    rc = p->opt.objective == 0 ? search_pipeline(p.get(), &cuts) : search_exhaustive_eq4(p.get(), &cuts);
+    if (rc) return rc;
+    finalize_blocks(p.get(), cuts);
+    *out = p.release();
+    return SWAPNET_OK;
+  } catch (const std::bad_alloc&) {
+    SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
+  }
+}
+
+int swapnet_plan_from_cuts(const swapnet_model_desc* desc, const uint32_t* cuts, uint32_t n_cuts,
+                           uint64_t budget, const swapnet_options* opt, swapnet_plan** out) {
+  if (!out || (n_cuts && !cuts)) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+  try {
+    std::unique_ptr<swapnet_plan> p;
+    int rc = prepare(desc, budget, opt, &p);
+    if (rc) return rc;
+    std::vector<uint32_t> c(cuts, cuts + n_cuts);
+    uint32_t prev = 0;
+    for (uint32_t v : c) {
+      if (v <= prev || v >= p->units.size()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "cuts must increase within [1, n_units)");
+      prev = v;
+    }
+    finalize_blocks(p.get(), c);
+    for (const Block& B : p->blocks)
+      if (B.bytes > p->slot) SN_FAIL(SWAPNET_ERR_INFEASIBLE, "a block exceeds the slot");
+    *out = p.release();
+    return SWAPNET_OK;
+  } catch (const std::bad_alloc&) {
+    SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
+  }
+}
+
+int swapnet_plan_resident(const swapnet_model_desc* desc, const swapnet_options* opt, swapnet_plan** out) {
+  if (!out) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null out_plan");
+  try {
+    std::unique_ptr<swapnet_plan> p(new swapnet_plan());
+    if (opt) p->opt = *opt; else swapnet_default_options(&p->opt);
+    int rc = check_options(p->opt);
+    if (rc) return rc;
+    rc = analyse_model(desc, &p->model);
+    if (rc) return rc;
+    p->resident = true;
+    p->arena = p->model.weight_bytes;
+    p->slot = p->arena;
+    p->budget = p->arena;
+    rc = make_units(p->model, p->opt, ~0ull, &p->units);
+    if (rc) return rc;
+    finalize_blocks(p.get(), {});
+    *out = p.release();
+    return SWAPNET_OK;
+  } catch (const std::bad_alloc&) {
+    SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
+  }
+}
+
+int swapnet_plan_info_get(const swapnet_plan* p, swapnet_plan_info* info) {
+  if (!p || !info) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+  swapnet_plan_info r{};
+  r.n_blocks = (uint32_t)p->blocks.size();
+  r.n_units = (uint32_t)p->units.size();
+  r.slots = p->resident ? 0 : (uint32_t)p->opt.slots;
+  r.n_layers = (uint32_t)p->model.L.size();
+  r.budget_bytes = p->budget;
+  r.arena_bytes = p->arena;
+  r.slot_bytes = p->slot;
+  r.workspace_bytes = p->model.ws_bytes;
+  r.input_bytes = p->model.in_bytes;
+  r.output_bytes = p->model.out_bytes;
+  r.weight_bytes = p->model.weight_bytes;
+  r.plan_bytes = sizeof(swapnet_plan) + p->units.size() * sizeof(Unit) + p->blocks.size() * sizeof(Block) +
+                 p->model.L.size() * sizeof(Layer) + p->cuts.size() * sizeof(uint32_t);
+  r.predicted_ns = p->predicted;
+  *info = r;
+  return SWAPNET_OK;
+}
+
+int swapnet_plan_cuts(const swapnet_plan* p, uint32_t* cuts, uint32_t cap, uint32_t* n) {
+  if (!p) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null plan");
+  if (n) *n = (uint32_t)p->cuts.size();
+  for (uint32_t i = 0; cuts && i < cap && i < p->cuts.size(); ++i) cuts[i] = p->cuts[i];
+  return SWAPNET_OK;
+}
+
+int swapnet_plan_units(const swapnet_plan* p, swapnet_unit_info* u, uint32_t cap, uint32_t* n) {
+  if (!p) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null plan");
+  if (n) *n = (uint32_t)p->units.size();
+  for (uint32_t i = 0; u && i < cap && i < p->units.size(); ++i) {
+    const Unit& U = p->units[i];
+    u[i] = swapnet_unit_info{U.layer, U.row0, U.rows, U.depth, U.bytes, U.flops, U.t_ex};
+  }
+  return SWAPNET_OK;
+}
+
+int swapnet_plan_blocks(const swapnet_plan* p, swapnet_block_info* b, uint32_t cap, uint32_t* n) {
+  if (!p) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null plan");
+  if (n) *n = (uint32_t)p->blocks.size();
+  for (uint32_t i = 0; b && i < cap && i < p->blocks.size(); ++i) {
+    const Block& B = p->blocks[i];
+    b[i] = swapnet_block_info{(uint32_t)B.u0, (uint32_t)B.u1, (uint32_t)B.slot, (uint32_t)B.depth, B.bytes,
+                              B.t_in, B.t_ex, B.t_out};
+  }
+  return SWAPNET_OK;
+}
+
+int swapnet_plan_output_offsets(const swapnet_plan* p, uint64_t* offs, uint32_t cap, uint32_t* n) {
+  if (!p) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null plan");
+  uint32_t k = 0;
+  for (const Layer& L : p->model.L) {
+    if (L.out_off < 0) continue;
+    if (offs && k < cap) offs[k] = (uint64_t)L.out_off;
+    ++k;
+  }
+  if (n) *n = k;
+  return SWAPNET_OK;
+}
+
+void swapnet_plan_free(swapnet_plan* p) { delete p; }
+
+int swapnet_schedule(const swapnet_model_desc* const* models, const float* urgency, uint32_t n,
+                     uint64_t M, const swapnet_options* opt, uint64_t* budgets_out, swapnet_plan** plans_out) {
+  if (!models || !urgency || n == 0 || !plans_out) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+  try {
+    swapnet_options o;
+    if (opt) o = *opt; else swapnet_default_options(&o);
+    std::vector<Model> ms(n);
+    std::vector<long double> demand(n), ps(n);
+    long double sumM = 0, sumPS = 0;
+    for (uint32_t i = 0; i < n; ++i) {
+      int rc = analyse_model(models[i], &ms[i]);
+      if (rc) return rc;
+      if (!(urgency[i] >= 0.0f) || !std::isfinite(urgency[i])) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad urgency");
+      demand[i] = (long double)ms[i].weight_bytes;
+      const long double lat = (long double)resident_latency_ns(ms[i], o);
+      ps[i] = (long double)urgency[i] * lat / demand[i];
+      sumM += demand[i];
+      sumPS += ps[i];
+    }
+    std::vector<uint64_t> budgets(n);
+    for (uint32_t i = 0; i < n; ++i) {
+      if (sumM <= (long double)M) { budgets[i] = ms[i].weight_bytes; continue; }
+      long double a = demand[i] / sumM * (1.0L - 1.0L / n) * (long double)M;
+      if (sumPS > 0) a += ps[i] / sumPS * (1.0L / n) * (long double)M;
+      budgets[i] = (uint64_t)floorl(a) / kAlign * kAlign;
+    }
+    std::vector<swapnet_plan*> plans(n, nullptr);
+    for (uint32_t i = 0; i < n; ++i) {
+      int rc = swapnet_partition(models[i], budgets[i], &o, &plans[i]);
+      if (rc) {
+        for (swapnet_plan* q : plans) delete q;
+        return rc;
+      }
+    }
+    for (uint32_t i = 0; i < n; ++i) {
+      plans_out[i] = plans[i];
+      if (budgets_out) budgets_out[i] = budgets[i];
+    }
+    return SWAPNET_OK;
+  } catch (const std::bad_alloc&) {
+    SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
+  }
+}
+
+}  // extern "C"

@@ -12,7 +12,9 @@ Reproducibility rules:
 Initialisation per workload:
   mlp6      W ~ N(0, 1/fan_in), b = 0
   resnet50  conv W ~ N(0, 2/fan_in) with an inference BatchNorm folded in:
-            gamma ~ U(0.5, 1.5), beta ~ N(0, 0.1), mean ~ N(0, 0.1),
+            gamma ~ U(0.5, 1.5) (U(0, 0.2) for the last BN of each residual
+            branch, which keeps fp16 activations finite through 16
+            unnormalised residual adds), beta ~ N(0, 0.1), mean ~ N(0, 0.1),
             var ~ U(0.5, 1.5), eps = 1e-5; W' = W*g/sqrt(var+eps),
             b' = beta - mean*g/sqrt(var+eps) (folded in float64, rounded once);
             FC W ~ N(0, 1/fan_in), b ~ N(0, 0.01)
@@ -75,7 +77,10 @@ def layer_weights(model, li, seed=0):
     elif name == "resnet50":
         if layer["op"] == "conv":
             w = rw.normal(0.0, np.sqrt(2.0 / fan), wshape)
-            gamma = rb.uniform(0.5, 1.5, nout)
+            # the last BN of a residual branch: small gamma (zero-gamma style
+            # residual init); elsewhere U(0.5, 1.5)
+            last = layer.get("res") is not None
+            gamma = rb.uniform(0.0, 0.2, nout) if last else rb.uniform(0.5, 1.5, nout)
             beta = rb.normal(0.0, 0.1, nout)
             mean = rb.normal(0.0, 0.1, nout)
             var = rb.uniform(0.5, 1.5, nout)

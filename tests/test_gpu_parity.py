@@ -1,0 +1,174 @@
+"""GPU parity through the C ABI: every kernel and whole workloads against
+the CPU oracle, and swapped against all-resident (bit-exact)."""
+import numpy as np
+import pytest
+
+from oracle import plan as OP
+import synth
+from paper_2401_16757_gb300 import capi
+from helpers import Runner, check_close, oracle_outputs, rel_l2
+
+pytestmark = pytest.mark.gpu
+
+
+def _conv(src, cin, cout, k, stride=1, pad=None, act="relu", res=None, res_post=False):
+    return dict(op="conv", src=[src], cin=cin, cout=cout, kh=k, kw=k, stride=stride,
+                pad=k // 2 if pad is None else pad, act=act, res=res, res_post=res_post)
+
+
+def _model(layers, inp, dtype="f16", outputs=None, mid=40):
+    return dict(name="yolov3", model_id=mid, dtype=dtype, input=inp, layers=layers,
+                outputs=outputs or [len(layers) - 1])
+
+
+def _swap_and_resident(m, budget_frac=0.5, slots=2, variant=capi.SWAP_AUTO):
+    w = synth.gen.model_weights(m)
+    x = synth.gen.model_input(m)
+    d = capi.Desc(m)
+    wb = OP.weight_bytes(m)
+    opt = capi.options(slots=slots, swap_variant=variant)
+    biggest = max(sum(OP.align(b) for b in OP.layer_tensor_bytes(m, i)) for i in range(len(m["layers"])))
+    budget = max(int(wb * budget_frac), 2 * biggest + 512) // 256 * 256
+    host = capi.HostWeights(w)
+    sw = Runner(m, w, capi.Plan.partition(d, budget, opt), host)
+    rs = Runner(m, w, capi.Plan.resident(d), host)
+    return w, x, sw, rs
+
+
+def _check_model(m, budget_frac=0.5, slots=2, variant=capi.SWAP_AUTO):
+    w, x, sw, rs = _swap_and_resident(m, budget_frac, slots, variant)
+    ref = oracle_outputs(m, w, x)
+    got_sw = sw.run(x)
+    got_rs = rs.run(x)
+    for a, b in zip(got_sw, got_rs):
+        assert a.tobytes() == b.tobytes(), "swapped and resident differ"
+    check_close(m, sw.decode(got_sw), ref)
+    return sw
+
+
+# ----------------------------------------------------------------- kernels
+@pytest.mark.parametrize("dtype", ["f16", "bf16"])
+@pytest.mark.parametrize("k,stride,cin,cout,hw", [
+    (3, 1, 64, 64, 19),     # gather path, ragged M tile
+    (3, 2, 32, 96, 23),     # Cin=32: K=288 not a multiple of 64; stride 2
+    (1, 1, 64, 200, 17),    # pointwise: TMA A path, N not a multiple of 64
+    (1, 2, 128, 256, 14),   # strided pointwise: gather path
+    (7, 2, 3, 64, 40),      # stem: direct conv (Cin=3)
+    (3, 1, 3, 16, 12),      # direct conv
+])
+def test_conv_layer(dtype, k, stride, cin, cout, hw):
+    m = _model([_conv(-1, cin, cout, k, stride)], (2, hw, hw, cin), dtype)
+    _check_model(m)
+
+
+@pytest.mark.parametrize("res_post,act", [(False, "relu"), (True, "leaky"), (False, "none")])
+def test_conv_residual_epilogue(res_post, act):
+    layers = [_conv(-1, 64, 128, 1, act="none"),
+              _conv(-1, 64, 64, 3),
+              _conv(1, 64, 128, 3, act=act, res=0, res_post=res_post)]
+    _check_model(_model(layers, (1, 30, 30, 64)))
+
+
+@pytest.mark.parametrize("dtype", ["f16", "bf16", "f32"])
+@pytest.mark.parametrize("rows,k,n", [(1, 2048, 1000), (16, 4096, 640), (8, 1024, 1024), (200, 512, 384),
+                                      (300, 256, 64), (129, 1024, 136)])
+def test_linear_layer(dtype, rows, k, n):
+    if dtype == "f32" and rows > 16:
+        pytest.skip("fp32 linear is the skinny kernel (rows <= 16)")
+    layers = [dict(op="linear", src=[-1], k=k, n=n, act="relu", res=None, res_post=False),
+              dict(op="linear", src=[0], k=n, n=n, act="none", res=0, res_post=False)]
+    _check_model(_model(layers, (rows, 1, 1, k), dtype))
+
+
+@pytest.mark.parametrize("dtype", ["f16", "f32"])
+def test_pool_upsample_concat(dtype):
+    layers = [dict(op="maxpool", src=[-1], kh=3, kw=3, stride=2, pad=1),
+              dict(op="maxpool", src=[0], kh=2, kw=2, stride=2, pad=0),
+              dict(op="upsample2x", src=[1]),
+              dict(op="concat", src=[2, 0]),
+              dict(op="gap", src=[3])]
+    m = _model(layers, (2, 32, 32, 24), dtype, outputs=[3, 4])
+    # no weights: swapped plan has nothing to swap; compare to the oracle
+    w = synth.gen.model_weights(m)
+    x = synth.gen.model_input(m)
+    r = Runner(m, w, capi.Plan.resident(capi.Desc(m)))
+    got = r.decode(r.run(x))
+    ref = oracle_outputs(m, w, x)
+    np.testing.assert_array_equal(got[0], ref[0])      # max / copy ops are exact
+    check_close(m, got[1:], ref[1:])
+
+
+# ----------------------------------------------------------------- workloads
+@pytest.mark.parametrize("variant", [capi.SWAP_MEMCPY, capi.SWAP_ZEROCOPY, capi.SWAP_AUTO])
+def test_mlp_config(variant):
+    """6-layer fp32 MLP: explicit 3 x 2 plan in one slot (budget = one block
+    of weights + two activation buffers), the planner's 2-slot plan, and the
+    resident reference; all equal bit for bit and within 1e-4 of the oracle."""
+    m = synth.arch.mlp6()
+    w = synth.gen.model_weights(m)
+    x = synth.gen.model_input(m)
+    d = capi.Desc(m)
+    budget = 8_462_336
+    host = capi.HostWeights(w)
+    p1 = capi.Plan.from_cuts(d, [2, 4], budget, capi.options(slots=1, activations_in_budget=1,
+                                                               swap_variant=variant))
+    p2 = capi.Plan.partition(d, budget, capi.options(slots=2, activations_in_budget=1, swap_variant=variant))
+    assert p2.cuts() == [1, 2, 3, 4, 5]
+    outs = [Runner(m, w, p, host).run(x) for p in (p1, p2, capi.Plan.resident(d))]
+    for o in outs[1:]:
+        assert o[0].tobytes() == outs[0][0].tobytes()
+    ref = oracle_outputs(m, w, x)
+    check_close(m, [o.astype(np.float64) for o in outs[0]], ref)
+
+
+def test_mlp_repeated_calls_stable():
+    m = synth.arch.mlp6()
+    w = synth.gen.model_weights(m)
+    d = capi.Desc(m)
+    r = Runner(m, w, capi.Plan.partition(d, 8_462_336, capi.options(activations_in_budget=1)))
+    first = None
+    for req in range(5):
+        x = synth.gen.model_input(m, request=req % 2)
+        o = r.run(x)[0].tobytes()
+        if req == 0:
+            first = o
+        if req % 2 == 0:
+            assert o == first
+
+
+def test_every_partition_bit_exact_tiny():
+    layers = [_conv(-1, 16, 32, 3), _conv(0, 32, 32, 3, stride=2), _conv(1, 32, 64, 1),
+              dict(op="maxpool", src=[2], kh=2, kw=2, stride=2, pad=0),
+              dict(op="gap", src=[3]),
+              dict(op="linear", src=[4], k=64, n=40, act="none", res=None, res_post=False)]
+    m = _model(layers, (1, 24, 24, 16))
+    w = synth.gen.model_weights(m)
+    x = synth.gen.model_input(m)
+    d = capi.Desc(m)
+    host = capi.HostWeights(w)
+    base = Runner(m, w, capi.Plan.resident(d), host).run(x)[0].tobytes()
+    budget = 2 * OP.weight_bytes(m)
+    import itertools
+    for k in range(0, 6):
+        for cuts in itertools.combinations(range(1, 6), k):
+            p = capi.Plan.from_cuts(d, list(cuts), budget, capi.options())
+            assert Runner(m, w, p, host).run(x)[0].tobytes() == base, cuts
+
+
+def test_resnet50_config():
+    """ResNet-50 (BN folded), batch 1, budget 40 % of the weight bytes."""
+    m = synth.arch.resnet50()
+    sw = _check_model(m, budget_frac=0.4)
+    assert sw.info["n_blocks"] >= OP.block_count_rule(sw.info["weight_bytes"], sw.info["budget_bytes"])
+
+
+def test_swap_variants_bit_exact_resnet():
+    m = synth.arch.resnet50()
+    w = synth.gen.model_weights(m)
+    x = synth.gen.model_input(m)
+    d = capi.Desc(m)
+    host = capi.HostWeights(w)
+    budget = int(OP.weight_bytes(m) * 0.4) // 256 * 256
+    outs = [Runner(m, w, capi.Plan.partition(d, budget, capi.options(swap_variant=v)), host).run(x)[0].tobytes()
+            for v in (capi.SWAP_MEMCPY, capi.SWAP_ZEROCOPY)]
+    assert outs[0] == outs[1]

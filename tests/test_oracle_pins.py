@@ -177,3 +177,17 @@ def test_outputs_are_representable():
     m = _tiny_resnet()
     out = F.forward(m, synth.gen.model_weights(m), synth.gen.model_input(m))[0]
     np.testing.assert_array_equal(out.astype(np.float16).astype(np.float64), out)
+
+
+@pytest.mark.parametrize("name", ["resnet50", "vgg16", "yolov3"])
+def test_workload_activations_stay_in_fp16_range(name):
+    # every layer output of the full-size workload is finite and well inside
+    # the fp16 range (no overflow, no collapse to zero)
+    m = synth.arch.MODELS[name]()
+    w = synth.gen.model_weights(m)
+    x = synth.gen.model_input(m)
+    x_in = F.nhwc_to_nchw(F.decode(x, m["dtype"]))
+    acts = F.forward_range(m, w, {}, x_in, 0, len(m["layers"]))
+    for a in acts.values():
+        assert np.all(np.isfinite(a)) and np.max(np.abs(a)) < 6e4
+        assert np.sqrt(np.mean(a ** 2)) > 1e-2
