@@ -110,12 +110,15 @@ typedef struct swapnet_options {
   uint64_t gamma_as_per_flop;
   uint64_t eta_ns_per_tensor;
   int32_t zc_ctas;               /* CTAs of the zero-copy swap kernel, 0 = default */
-  int32_t reserved[7];
+  int32_t graphs;                /* 1 (default): each (input, output) binding of an
+                                    engine is captured once as a CUDA graph and
+                                    replayed; 0: launch eagerly every call      */
+  int32_t reserved[6];
 } swapnet_options;
 
 /* Fills the defaults: 2 slots, activations outside the budget, AUTO swap,
  * pipeline objective, alpha = 2.5e6 as/B (400 GB/s), beta = 2000 ns,
- * gamma = 2000 as/FLOP (500 TFLOP/s), eta = 0. */
+ * gamma = 2000 as/FLOP (500 TFLOP/s), eta = 0, CUDA graphs on. */
 void swapnet_default_options(swapnet_options* opt);
 
 /* ------------------------------------------------------------------ plans */
@@ -272,7 +275,8 @@ typedef enum swapnet_kernel_kind {
   SWAPNET_KERNEL_MAXPOOL = 5,
   SWAPNET_KERNEL_GAP = 6,
   SWAPNET_KERNEL_UPSAMPLE = 7,
-  SWAPNET_KERNEL_CONCAT = 8
+  SWAPNET_KERNEL_CONCAT = 8,
+  SWAPNET_KERNEL_TILED = 9        /* SIMT tiled linear (general fallback)     */
 } swapnet_kernel_kind;
 int swapnet_engine_unit_kernels(const swapnet_engine* eng, int32_t* kinds, uint32_t cap, uint32_t* n);
 

@@ -39,7 +39,7 @@ class Options(C.Structure):
     _fields_ = [("slots", C.c_int32), ("activations_in_budget", C.c_int32), ("swap_variant", C.c_int32),
                 ("objective", C.c_int32), ("alpha_as_per_byte", C.c_uint64), ("beta_ns_per_tensor", C.c_uint64),
                 ("gamma_as_per_flop", C.c_uint64), ("eta_ns_per_tensor", C.c_uint64), ("zc_ctas", C.c_int32),
-                ("reserved", C.c_int32 * 7)]
+                ("graphs", C.c_int32), ("reserved", C.c_int32 * 6)]
 
 
 class PlanInfo(C.Structure):
@@ -66,7 +66,7 @@ class EngineStats(C.Structure):
 
 
 KERNEL_KIND = {1: "tc_gemm", 2: "tc_conv", 3: "skinny_linear", 4: "direct_conv", 5: "maxpool", 6: "gap",
-               7: "upsample2x", 8: "concat"}
+               7: "upsample2x", 8: "concat", 9: "tiled_linear"}
 
 
 class EngineBlock(C.Structure):

@@ -107,6 +107,13 @@ struct swapnet_engine {
   bool profiling = false;
   std::vector<cudaEvent_t> ev_unit;  // 2 per unit
   std::vector<cudaEvent_t> ev_swap;  // 2 per block
+  cudaStream_t cap = nullptr;        // capture origin stream
+  cudaEvent_t fork = nullptr, join = nullptr;
+  // per (input, output, profiling) binding
+  std::map<std::pair<std::pair<const void*, void*>, bool>, cudaGraphExec_t> graphs;
+  char* d_splitk = nullptr;          // split-K scratch: tile counters, then fp32 partials
+  uint64_t splitk_bytes = 0;
+  uint64_t splitk_counter_bytes = 0;
 };
 
 namespace swapnet {
@@ -117,11 +124,16 @@ static int release(swapnet_engine* e) {
   if (e->copy) cudaStreamSynchronize(e->copy);
   for (cudaEvent_t ev : {e->slot_free[0], e->slot_free[1], e->ready[0], e->ready[1]})
     if (ev) cudaEventDestroy(ev);
+  for (auto& kv : e->graphs) cudaGraphExecDestroy(kv.second);
+  if (e->fork) cudaEventDestroy(e->fork);
+  if (e->join) cudaEventDestroy(e->join);
+  if (e->cap) cudaStreamDestroy(e->cap);
   for (cudaEvent_t ev : e->ev_unit) cudaEventDestroy(ev);
   for (cudaEvent_t ev : e->ev_swap) cudaEventDestroy(ev);
   if (e->copy) cudaStreamDestroy(e->copy);
   if (e->own_arena && e->d_arena) cudaFree(e->d_arena);
   if (e->own_ws && e->d_ws) cudaFree(e->d_ws);
+  if (e->d_splitk) cudaFree(e->d_splitk);
   if (e->d_in_stage) cudaFree(e->d_in_stage);
   if (e->d_out_stage) cudaFree(e->d_out_stage);
   for (const HostRange& r : e->ranges)
@@ -230,7 +242,6 @@ static int swap_block(swapnet_engine* e, size_t k, int variant, cudaStream_t s) 
       z.push_back(ZcSeg{g.src, g.dst, g.bytes});
       e->stats.bytes_swapped += g.bytes;
     }
-    e->stats.kernel_launches += (z.size() + 47) / 48;
     return launch_zerocopy(z.data(), (int)z.size(), e->zc_ctas, s);
   }
   for (const Segment& g : b.segs) {
@@ -298,6 +309,7 @@ static bool unit_gemm(const swapnet_engine* e, const Unit& U, const UnitExec& X,
   const int es = m.es;
   std::memset(g, 0, sizeof(*g));
   g->dtype = m.dtype;
+  g->num_sms = e->num_sms;
   g->W = X.w;
   g->e.bias = X.b;
   g->e.act = L.d.act;
@@ -324,6 +336,10 @@ static bool unit_gemm(const swapnet_engine* e, const Unit& U, const UnitExec& X,
   return true;
 }
 
+static bool skinny_ok(const Model& m, const Layer& L) {
+  return L.n <= 16 && ((uint64_t)L.d.cin * m.es) % 16 == 0;
+}
+
 static bool wants_tc(const Model& m, const Layer& L) {
   if (m.dtype == SWAPNET_F32) return false;
   if (L.d.op == SWAPNET_OP_LINEAR) return L.n > 16 && L.d.cin % 8 == 0;
@@ -340,7 +356,9 @@ static int prepare_units(swapnet_engine* e) {
     const Layer& L = m.L[p.units[u].layer];
     int k = 0;
     switch (L.d.op) {
-      case SWAPNET_OP_LINEAR: k = wants_tc(m, L) ? SWAPNET_KERNEL_TC_GEMM : SWAPNET_KERNEL_SKINNY; break;
+      case SWAPNET_OP_LINEAR:
+        k = wants_tc(m, L) ? SWAPNET_KERNEL_TC_GEMM : skinny_ok(m, L) ? SWAPNET_KERNEL_SKINNY : SWAPNET_KERNEL_TILED;
+        break;
       case SWAPNET_OP_CONV2D:
         if (!wants_tc(m, L)) k = SWAPNET_KERNEL_DIRECT_CONV;
         else if (L.d.kh == 1 && L.d.kw == 1 && L.d.stride == 1 && L.d.pad == 0) k = SWAPNET_KERNEL_TC_GEMM;
@@ -399,13 +417,20 @@ static int run_unit(swapnet_engine* e, int u, const void* din, void* dout, cudaS
           if (rc) return rc;
           X.tmA_for = g.A;
         }
+        if (X.tc.splits > 1) {
+          g.counters = reinterpret_cast<int*>(e->d_splitk);
+          g.partial = reinterpret_cast<float*>(e->d_splitk + e->splitk_counter_bytes);
+        }
         return launch_tc_gemm(g, X.tc, e->err_word, s);
       }
       Epi ep{X.b, nullptr, L.d.cout, L.d.act, L.d.res_post};
       if (L.d.op == SWAPNET_OP_LINEAR) {
         ep.res = r ? r + (int64_t)U.row0 * es : nullptr;
-        return launch_linear_skinny(m.dtype, x, L.n, L.d.cin, X.w, U.rows, ep, y + (int64_t)U.row0 * es,
-                                    L.d.cout, s);
+        if (skinny_ok(m, L))
+          return launch_linear_skinny(m.dtype, x, L.n, L.d.cin, X.w, U.rows, ep, y + (int64_t)U.row0 * es,
+                                      L.d.cout, s);
+        return launch_linear_tiled(m.dtype, x, L.n, L.d.cin, X.w, U.rows, ep, y + (int64_t)U.row0 * es, L.d.cout,
+                                   s);
       }
       ep.res = r;
       return launch_conv_direct(m.dtype, x, L.n, L.h, L.w, L.d.cin, X.w, L.d.cout, L.d.kh, L.d.kw, L.d.stride,
@@ -481,11 +506,32 @@ int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint
     CU(cudaEventCreateWithFlags(&e->slot_free[s], cudaEventDisableTiming), "event");
     CU(cudaEventCreateWithFlags(&e->ready[s], cudaEventDisableTiming), "event");
   }
+  CU(cudaStreamCreateWithFlags(&e->cap, cudaStreamNonBlocking), "capture stream");
+  CU(cudaEventCreateWithFlags(&e->fork, cudaEventDisableTiming), "event");
+  CU(cudaEventCreateWithFlags(&e->join, cudaEventDisableTiming), "event");
   rc = register_host(e, host_weights, n_tensors);
   if (rc) return rc;
   build_segments(e);
   rc = prepare_units(e);
   if (rc) return rc;
+  {
+    uint64_t part = 0;
+    int64_t tiles = 0;
+    for (const UnitExec& X : e->ux)
+      if (X.use_tc && X.tc.splits > 1) {
+        part = std::max(part, X.tc.scratch_bytes);
+        tiles = std::max(tiles, X.tc.tiles);
+      }
+    if (part) {
+      e->splitk_counter_bytes = align_up((uint64_t)tiles * sizeof(int));
+      e->splitk_bytes = e->splitk_counter_bytes + part;
+      if (injected(2) || cudaMalloc(&e->d_splitk, e->splitk_bytes) != cudaSuccess) {
+        cudaGetLastError();
+        SN_FAIL(SWAPNET_ERR_OOM, "split-K scratch allocation failed");
+      }
+      CU(cudaMemset(e->d_splitk, 0, e->splitk_counter_bytes), "split-K counters");
+    }
+  }
   const int variant = plan->opt.swap_variant;
   if (plan->resident) {
     for (size_t k = 0; k < e->blocks.size() && !rc; ++k) rc = swap_block(e, k, SWAPNET_SWAP_MEMCPY, e->copy);
@@ -506,17 +552,23 @@ int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint
   return SWAPNET_OK;
 }
 
-int swapnet_infer(swapnet_engine* e, const void* din, void* dout, swapnet_stream stream) {
-  if (!e || !din || !dout) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
-  if (((uintptr_t)din | (uintptr_t)dout) & 15) SN_FAIL(SWAPNET_ERR_MISALIGNED, "input/output must be 16-byte aligned");
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  CU(cudaSetDevice(e->device), "cudaSetDevice");
+}  // extern "C"
+
+namespace swapnet {
+
+// Enqueue one inference: swaps on the copy stream, layers on `s`.
+// Inside a graph capture a slot's first use in the inference has no
+// in-graph predecessor to wait for (the graph as a whole is ordered after
+// earlier work on the launch stream), so that wait is omitted.
+static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t s, bool capturing = false) {
   const swapnet_plan& p = e->plan;
-  const bool prof = e->profiling;
+  const bool prof = e->profiling && !capturing;
+  bool used[2] = {false, false};
   for (size_t k = 0; k < p.blocks.size(); ++k) {
     const Block& B = p.blocks[k];
     if (!p.resident) {
-      CU(cudaStreamWaitEvent(e->copy, e->slot_free[B.slot], 0), "wait slot");
+      if (!capturing || used[B.slot]) CU(cudaStreamWaitEvent(e->copy, e->slot_free[B.slot], 0), "wait slot");
+      used[B.slot] = true;
       if (prof) CU(cudaEventRecord(e->ev_swap[2 * k], e->copy), "profile event");
       int rc = swap_block(e, k, e->blocks[k].variant, e->copy);
       if (rc) return rc;
@@ -529,10 +581,86 @@ int swapnet_infer(swapnet_engine* e, const void* din, void* dout, swapnet_stream
       int rc = run_unit(e, u, din, dout, s);
       if (rc) return rc;
       if (prof) CU(cudaEventRecord(e->ev_unit[2 * u + 1], s), "profile event");
-      e->stats.kernel_launches += 1;
     }
     if (!p.resident) CU(cudaEventRecord(e->slot_free[B.slot], s), "record slot free");
   }
+  return SWAPNET_OK;
+}
+
+static uint64_t launches_per_infer(const swapnet_engine* e) {
+  uint64_t n = e->plan.units.size();
+  if (!e->plan.resident)
+    for (const EngBlock& b : e->blocks)
+      if (b.variant == SWAPNET_SWAP_ZEROCOPY) n += (b.segs.size() + 47) / 48;
+  return n;
+}
+
+// Capture one inference for this binding as a graph: the capture starts on
+// the engine's own stream, the copy stream joins through an event (fork) and
+// rejoins at the end, so slot gating becomes graph edges.
+static int capture(swapnet_engine* e, const void* din, void* dout, cudaGraphExec_t* out) {
+  const swapnet_engine_stats saved = e->stats;
+  CU(cudaStreamBeginCapture(e->cap, cudaStreamCaptureModeThreadLocal), "begin capture");
+  int rc = SWAPNET_OK;
+  cudaGraph_t g = nullptr;
+  do {
+    if (!e->plan.resident) {
+      if (cudaEventRecord(e->fork, e->cap) != cudaSuccess || cudaStreamWaitEvent(e->copy, e->fork, 0) != cudaSuccess) {
+        rc = SWAPNET_ERR_CUDA;
+        break;
+      }
+    }
+    rc = enqueue(e, din, dout, e->cap, true);
+    if (rc) break;
+    if (!e->plan.resident) {
+      if (cudaEventRecord(e->join, e->copy) != cudaSuccess || cudaStreamWaitEvent(e->cap, e->join, 0) != cudaSuccess)
+        rc = SWAPNET_ERR_CUDA;
+    }
+  } while (0);
+  const cudaError_t ee = cudaStreamEndCapture(e->cap, &g);
+  e->stats = saved;
+  if (rc || ee != cudaSuccess || !g) {
+    if (g) cudaGraphDestroy(g);
+    cudaGetLastError();
+    SN_FAIL(rc ? rc : SWAPNET_ERR_CUDA, "graph capture failed");
+  }
+  const cudaError_t ie = cudaGraphInstantiate(out, g, 0);
+  cudaGraphDestroy(g);
+  if (ie != cudaSuccess) {
+    cudaGetLastError();
+    SN_FAIL(SWAPNET_ERR_CUDA, std::string("graph instantiate: ") + cudaGetErrorString(ie));
+  }
+  return SWAPNET_OK;
+}
+
+}  // namespace swapnet
+
+extern "C" {
+
+int swapnet_infer(swapnet_engine* e, const void* din, void* dout, swapnet_stream stream) {
+  if (!e || !din || !dout) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+  if (((uintptr_t)din | (uintptr_t)dout) & 15) SN_FAIL(SWAPNET_ERR_MISALIGNED, "input/output must be 16-byte aligned");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  CU(cudaSetDevice(e->device), "cudaSetDevice");
+  if (e->plan.opt.graphs && !e->profiling) {  // event timing needs eager launches
+    const auto key = std::make_pair(std::make_pair(din, dout), false);
+    auto it = e->graphs.find(key);
+    if (it == e->graphs.end()) {
+      if (e->graphs.size() >= 8) {
+        for (auto& kv : e->graphs) cudaGraphExecDestroy(kv.second);
+        e->graphs.clear();
+      }
+      cudaGraphExec_t ge = nullptr;
+      int rc = capture(e, din, dout, &ge);
+      if (rc) return rc;
+      it = e->graphs.emplace(key, ge).first;
+    }
+    CU(cudaGraphLaunch(it->second, s), "graph launch");
+  } else {
+    int rc = enqueue(e, din, dout, s);
+    if (rc) return rc;
+  }
+  e->stats.kernel_launches += launches_per_infer(e);
   e->stats.infer_calls += 1;
   return SWAPNET_OK;
 }
@@ -566,6 +694,7 @@ int swapnet_engine_sync(swapnet_engine* e) {
   if (w) {
     const int zero = 0;
     cudaMemcpy(e->err_word, &zero, sizeof(int), cudaMemcpyHostToDevice);
+    if (e->d_splitk) cudaMemset(e->d_splitk, 0, e->splitk_counter_bytes);  // an aborted kernel may leave counts
     SN_FAIL(SWAPNET_ERR_TIMEOUT, "a device-side wait gave up");
   }
   return SWAPNET_OK;

@@ -119,18 +119,78 @@ int skinny_dispatch(const void* x, int M, int K, const void* W, int N, const Epi
   return cudaGetLastError() == cudaSuccess ? SWAPNET_OK : SWAPNET_ERR_CUDA;
 }
 
+// ------------------------------------------------------------ tiled linear
+// General fallback for any M, K, N and dtype: 64 x 64 output tile per CTA,
+// 16 x 16 threads with 4 x 4 outputs each, K staged through shared memory
+// in steps of 16, fp32 accumulation in a fixed order.
+template <typename T>
+__global__ void __launch_bounds__(256) linear_tiled_kernel(const T* __restrict__ x, int M, int K,
+                                                           const T* __restrict__ W, int N, Epi e,
+                                                           T* __restrict__ y, int64_t ldy) {
+  __shared__ float xs[16][64 + 1];
+  __shared__ float ws[16][64 + 1];
+  const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
+  const int m0 = blockIdx.y * 64, n0 = blockIdx.x * 64;
+  float acc[4][4] = {};
+  for (int k0 = 0; k0 < K; k0 += 16) {
+    for (int i = threadIdx.x; i < 16 * 64; i += 256) {
+      const int kk = i % 16, r = i / 16;
+      const int m = m0 + r, n = n0 + r, k = k0 + kk;
+      xs[kk][r] = (m < M && k < K) ? to_f<T>(x[(int64_t)m * K + k]) : 0.f;
+      ws[kk][r] = (n < N && k < K) ? to_f<T>(W[(int64_t)n * K + k]) : 0.f;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < 16; ++kk) {
+      float a[4], b[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) { a[i] = xs[kk][ty + 16 * i]; b[i] = ws[kk][tx + 16 * i]; }
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+  const T* bias = reinterpret_cast<const T*>(e.bias);
+  const T* res = reinterpret_cast<const T*>(e.res);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int m = m0 + ty + 16 * i;
+    if (m >= M) continue;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int n = n0 + tx + 16 * j;
+      if (n >= N) continue;
+      const float rv = res ? to_f<T>(res[(int64_t)m * e.ldr + n]) : 0.f;
+      y[(int64_t)m * ldy + n] = from_f<T>(epilogue(acc[i][j], to_f<T>(bias[n]), rv, res != nullptr, e.act, e.res_post));
+    }
+  }
+}
+
 // ------------------------------------------------------------ direct conv
-// Thread = one output pixel x 8 output channels; the lanes of a warp share
-// the channel group, so weight loads are warp-uniform (broadcast).
-constexpr int kDcCo = 8;
+// Thread = one output pixel x 16 output channels.  The CTA's 16 filters are
+// staged in shared memory as fp32, laid out [tap][cin][16] so each input
+// value meets 16 weights read as four broadcast float4 loads.  Used for
+// channel counts the tensor-core path cannot tile (e.g. a 3-channel image).
+constexpr int kDcCo = 16;
 
 template <typename T>
-__global__ void conv_direct_kernel(const T* __restrict__ x, int n, int h, int w, int cin,
-                                   const T* __restrict__ W, int cout, int kh, int kw, int stride, int pad, int oh,
-                                   int ow, Epi e, T* __restrict__ y) {
+__global__ void __launch_bounds__(128) conv_direct_kernel(const T* __restrict__ x, int n, int h, int w, int cin,
+                                                          const T* __restrict__ W, int cout, int kh, int kw,
+                                                          int stride, int pad, int oh, int ow, Epi e,
+                                                          T* __restrict__ y) {
+  extern __shared__ float ws[];  // [kh*kw*cin][kDcCo]
+  const int co0 = blockIdx.y * kDcCo;
+  const int taps = kh * kw * cin;
+  for (int i = threadIdx.x; i < taps * kDcCo; i += blockDim.x) {
+    const int j = i % kDcCo, tc = i / kDcCo;  // tc = (r*kw + s)*cin + c
+    const int co = co0 + j;
+    ws[i] = co < cout ? to_f<T>(W[(int64_t)co * taps + tc]) : 0.f;
+  }
+  __syncthreads();
   const int64_t pix = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t npix = (int64_t)n * oh * ow;
-  const int co0 = blockIdx.y * kDcCo;
   if (pix >= npix) return;
   const int img = (int)(pix / ((int64_t)oh * ow));
   const int rem = (int)(pix % ((int64_t)oh * ow));
@@ -145,12 +205,16 @@ __global__ void conv_direct_kernel(const T* __restrict__ x, int n, int h, int w,
       const int ix = ox * stride + s - pad;
       if (ix < 0 || ix >= w) continue;
       const T* xp = x + (((int64_t)img * h + iy) * w + ix) * cin;
+      const float4* wp = reinterpret_cast<const float4*>(ws + (int64_t)((r * kw + s) * cin) * kDcCo);
       for (int c = 0; c < cin; ++c) {
         const float xv = to_f<T>(xp[c]);
 #pragma unroll
-        for (int j = 0; j < kDcCo; ++j) {
-          const int co = co0 + j;
-          if (co < cout) acc[j] = fmaf(xv, to_f<T>(__ldg(W + (((int64_t)co * kh + r) * kw + s) * cin + c)), acc[j]);
+        for (int q = 0; q < kDcCo / 4; ++q) {
+          const float4 wv = wp[c * (kDcCo / 4) + q];
+          acc[4 * q + 0] = fmaf(xv, wv.x, acc[4 * q + 0]);
+          acc[4 * q + 1] = fmaf(xv, wv.y, acc[4 * q + 1]);
+          acc[4 * q + 2] = fmaf(xv, wv.z, acc[4 * q + 2]);
+          acc[4 * q + 3] = fmaf(xv, wv.w, acc[4 * q + 3]);
         }
       }
     }
@@ -160,9 +224,10 @@ __global__ void conv_direct_kernel(const T* __restrict__ x, int n, int h, int w,
 #pragma unroll
   for (int j = 0; j < kDcCo; ++j) {
     const int co = co0 + j;
-    if (co >= cout) break;
-    const float rv = res ? to_f<T>(res[pix * e.ldr + co]) : 0.f;
-    y[pix * cout + co] = from_f<T>(epilogue(acc[j], to_f<T>(bias[co]), rv, res != nullptr, e.act, e.res_post));
+    if (co < cout) {
+      const float rv = res ? to_f<T>(res[pix * e.ldr + co]) : 0.f;
+      y[pix * cout + co] = from_f<T>(epilogue(acc[j], to_f<T>(bias[co]), rv, res != nullptr, e.act, e.res_post));
+    }
   }
 }
 
@@ -257,14 +322,30 @@ int launch_linear_skinny(int dtype, const void* x, int M, int K, const void* W, 
   return SWAPNET_OK;
 }
 
+int launch_linear_tiled(int dtype, const void* x, int M, int K, const void* W, int N, const Epi& e, void* y,
+                        int64_t ldy, cudaStream_t s) {
+  if (M < 1 || K < 1 || N < 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "tiled linear: empty shape");
+  const dim3 grid((N + 63) / 64, (M + 63) / 64);
+  SN_DISPATCH(dtype, T,
+              linear_tiled_kernel<T><<<grid, 256, 0, s>>>(static_cast<const T*>(x), M, K, static_cast<const T*>(W), N,
+                                                           e, static_cast<T*>(y), ldy));
+  return last_launch();
+}
+
 int launch_conv_direct(int dtype, const void* x, int n, int h, int w, int cin, const void* W, int cout, int kh,
                        int kw, int stride, int pad, int oh, int ow, const Epi& e, void* y, cudaStream_t s) {
   const int64_t npix = (int64_t)n * oh * ow;
+  const size_t smem = (size_t)kh * kw * cin * kDcCo * sizeof(float);
+  if (smem > 200 * 1024) SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "direct conv: filter too large for shared memory");
   const dim3 grid(grid1d(npix, 128), (cout + kDcCo - 1) / kDcCo);
-  SN_DISPATCH(dtype, T,
-              conv_direct_kernel<T><<<grid, 128, 0, s>>>(static_cast<const T*>(x), n, h, w, cin,
-                                                         static_cast<const T*>(W), cout, kh, kw, stride, pad, oh,
-                                                         ow, e, static_cast<T*>(y)));
+  SN_DISPATCH(dtype, T, {
+    auto kern = conv_direct_kernel<T>;
+    if (smem > 48 * 1024 &&
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+      SN_FAIL(SWAPNET_ERR_CUDA, "cudaFuncSetAttribute failed");
+    kern<<<grid, 128, smem, s>>>(static_cast<const T*>(x), n, h, w, cin, static_cast<const T*>(W), cout, kh, kw,
+                                 stride, pad, oh, ow, e, static_cast<T*>(y));
+  });
   return last_launch();
 }
 

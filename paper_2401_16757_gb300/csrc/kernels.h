@@ -22,6 +22,11 @@ struct Epi {
 int launch_linear_skinny(int dtype, const void* x, int M, int K, const void* W, int N, const Epi& e, void* y,
                          int64_t ldy, cudaStream_t s);
 
+// General tiled SIMT linear (any M, K, N): the fallback when neither the
+// tensor-core nor the skinny kernel applies.
+int launch_linear_tiled(int dtype, const void* x, int M, int K, const void* W, int N, const Epi& e, void* y,
+                        int64_t ldy, cudaStream_t s);
+
 // Direct convolution (SIMT) for any channel count; NHWC in, NHWC out.
 int launch_conv_direct(int dtype, const void* x, int n, int h, int w, int cin, const void* W, int cout, int kh,
                        int kw, int stride, int pad, int oh, int ow, const Epi& e, void* y, cudaStream_t s);
@@ -57,12 +62,19 @@ struct TcGemm {
   Epi e;
   void* y;
   int64_t ldy;
+  int num_sms;          // used by tc_prepare to size the grid
+  float* partial;       // split-K scratch (TcPlan::scratch_bytes), set per launch
+  int* counters;        // split-K tile counters (TcPlan::tiles ints, zeroed once)
 };
 // Pre-encoded descriptors of one GEMM (built once per layer at load time).
 struct TcPlan {
   CUtensorMap tmA;  // valid when conv == 0
   CUtensorMap tmB;
   int bn;           // N tile
+  int splits;       // K splits (grid z); 1 = no split
+  int kb_per_split; // 64-wide k-blocks per split
+  int64_t tiles;    // output tiles (split-K counters needed)
+  uint64_t scratch_bytes;  // fp32 partials of all splits
   int ready;
 };
 int tc_prepare(const TcGemm& g, TcPlan* p);

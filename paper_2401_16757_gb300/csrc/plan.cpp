@@ -450,6 +450,7 @@ static int check_options(const swapnet_options& o) {
   if (o.objective != 0 && o.objective != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "objective must be 0 or 1");
   if (o.swap_variant < 0 || o.swap_variant > 2) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad swap_variant");
   if (o.zc_ctas < 0 || o.zc_ctas > 4096) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad zc_ctas");
+  if (o.graphs != 0 && o.graphs != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "graphs must be 0 or 1");
   return SWAPNET_OK;
 }
 
@@ -492,6 +493,7 @@ void swapnet_default_options(swapnet_options* o) {
   o->gamma_as_per_flop = 2000;     // 500 TFLOP/s
   o->eta_ns_per_tensor = 0;
   o->zc_ctas = 0;
+  o->graphs = 1;
 }
 
 int swapnet_partition(const swapnet_model_desc* desc, uint64_t budget, const swapnet_options* opt,

@@ -55,6 +55,8 @@ def _check_model(m, budget_frac=0.5, slots=2, variant=capi.SWAP_AUTO):
     (1, 2, 128, 256, 14),   # strided pointwise: gather path
     (7, 2, 3, 64, 40),      # stem: direct conv (Cin=3)
     (3, 1, 3, 16, 12),      # direct conv
+    (3, 1, 256, 256, 7),    # deep K, one M tile: split-K with last-CTA reduction
+    (3, 1, 64, 24, 9),      # N below one 32-column chunk
 ])
 def test_conv_layer(dtype, k, stride, cin, cout, hw):
     m = _model([_conv(-1, cin, cout, k, stride)], (2, hw, hw, cin), dtype)
@@ -71,10 +73,8 @@ def test_conv_residual_epilogue(res_post, act):
 
 @pytest.mark.parametrize("dtype", ["f16", "bf16", "f32"])
 @pytest.mark.parametrize("rows,k,n", [(1, 2048, 1000), (16, 4096, 640), (8, 1024, 1024), (200, 512, 384),
-                                      (300, 256, 64), (129, 1024, 136)])
+                                      (300, 256, 64), (129, 1024, 136), (40, 512, 130)])
 def test_linear_layer(dtype, rows, k, n):
-    if dtype == "f32" and rows > 16:
-        pytest.skip("fp32 linear is the skinny kernel (rows <= 16)")
     layers = [dict(op="linear", src=[-1], k=k, n=n, act="relu", res=None, res_post=False),
               dict(op="linear", src=[0], k=n, n=n, act="none", res=0, res_post=False)]
     _check_model(_model(layers, (rows, 1, 1, k), dtype))
