@@ -292,6 +292,44 @@ int swapnet_engine_last_times(swapnet_engine* eng, float* unit_us, uint32_t n_un
 
 void swapnet_engine_free(swapnet_engine* eng);
 
+/* ------------------------------------------------- allocation-free GEMM */
+/* Y[m][n] = act(sum_k A[m][k] * W[n][k] + bias[n]) for fp16 or bf16 data,
+ * computed by the same tcgen05 split-K GEMM kernel the engine uses for
+ * linear layers, but with its split-K scratch (fp32 partial sums and tile
+ * counters) in a fixed device array inside the library instead of memory
+ * the engine allocates.  The paper has no counterpart to this call.
+ *
+ * It is for callers that must not allocate device memory: code running
+ * under a hard device-memory budget in which every byte is already
+ * assigned (the situation this library is about), or hosts whose own
+ * allocator has reserved the whole GPU so that cudaMalloc would fail.
+ * The call allocates nothing: no cudaMalloc, no cudaFree, no allocating
+ * library routine.
+ *
+ *   dtype   SWAPNET_F16 or SWAPNET_BF16
+ *   A       device, [M][K] row-major; W device, [N][K] row-major;
+ *           bias device, [N]; Y device, [M][N] row-major, written
+ *   act     swapnet_act applied after the bias
+ *   stream  the call is asynchronous on it
+ * Pointers must be 16-byte aligned and K a multiple of 8.
+ *
+ * Limits and sharing: the scratch array holds SWAPNET_NOALLOC_SCRATCH_BYTES
+ * (4 MiB) on every GPU that loads the library, until the process exits.  A
+ * problem whose split-K scratch exceeds it is rejected with
+ * SWAPNET_ERR_INVALID_ARG before anything is launched.  Every call shares
+ * the array and it keeps the last call's contents; each call clears the
+ * counters it needs on `stream` first.  Calls that overlap on the GPU (on
+ * different streams, or on the same device from several threads) race on
+ * the array and must be serialised by the caller.
+ *
+ * Set-up: the first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress) with that device current and caches it; make that
+ * first call before any stream capture.
+ * Errors: INVALID_ARG, MISALIGNED, UNSUPPORTED, CUDA. */
+#define SWAPNET_NOALLOC_SCRATCH_BYTES (4u << 20)
+int swapnet_gemm_noalloc(int32_t dtype, const void* A, const void* W, const void* bias, void* Y, int32_t M,
+                         int32_t N, int32_t K, int32_t act, swapnet_stream stream);
+
 /* ------------------------------------------------------------------- misc */
 const char* swapnet_strerror(int status);
 const char* swapnet_last_error(void);

@@ -79,7 +79,7 @@ EXPORTS = ["swapnet_default_options", "swapnet_partition", "swapnet_plan_from_cu
            "swapnet_plan_output_offsets", "swapnet_plan_free", "swapnet_schedule", "swapnet_load",
            "swapnet_infer", "swapnet_infer_host", "swapnet_engine_sync", "swapnet_engine_blocks",
            "swapnet_engine_free", "swapnet_engine_stats_get", "swapnet_engine_unit_kernels",
-           "swapnet_engine_set_profiling", "swapnet_engine_last_times", "swapnet_strerror", "swapnet_last_error", "swapnet_debug_fail_next"]
+           "swapnet_engine_set_profiling", "swapnet_engine_last_times", "swapnet_strerror", "swapnet_last_error", "swapnet_debug_fail_next", "swapnet_gemm_noalloc"]
 
 _lib = None
 
@@ -129,6 +129,7 @@ def lib():
         "swapnet_strerror": (C.c_char_p, [C.c_int]),
         "swapnet_last_error": (C.c_char_p, []),
         "swapnet_debug_fail_next": (C.c_int, [C.c_int, C.c_int]),
+        "swapnet_gemm_noalloc": (C.c_int, [C.c_int32, P, P, P, P, C.c_int32, C.c_int32, C.c_int32, C.c_int32, P]),
     }
     for name, (res, args) in sig.items():
         f = getattr(L, name)
@@ -263,6 +264,13 @@ def schedule(descs, urgency, arena_bytes, opt=None):
     check(lib().swapnet_schedule(ptrs, urg, n, arena_bytes, C.byref(opt) if opt else None, budgets, plans),
           "swapnet_schedule")
     return list(budgets), [Plan(p) for p in plans]
+
+
+def gemm_noalloc(dtype, a_ptr, w_ptr, bias_ptr, y_ptr, M, N, K, act=0, stream=0):
+    """Y = act(A W^T + bias) through the allocation-free entry point."""
+    check(lib().swapnet_gemm_noalloc(dtype, C.c_void_p(a_ptr), C.c_void_p(w_ptr), C.c_void_p(bias_ptr),
+                                     C.c_void_p(y_ptr), M, N, K, act, C.c_void_p(stream or None)),
+          "swapnet_gemm_noalloc")
 
 
 # ------------------------------------------------------------ host weights
