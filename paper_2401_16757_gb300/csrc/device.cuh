@@ -80,11 +80,27 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Wait for the phase with the given parity to complete.  Gives up after
-// kWaitLimitNs (or at once when *abort is set by another thread), setting
-// *abort and the global error word; returns false then.
+__device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Wait for the phase with the given parity to complete.  Polls without
+// suspending for the first iterations (short, latency-critical waits), then
+// with the suspending try_wait.  Gives up after kWaitLimitNs (or at once
+// when *abort is set by another thread), setting *abort and the global
+// error word; returns false then.
 __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort,
                                                   int* err) {
+  for (int it = 0; it < 4096; ++it)
+    if (mbar_test_wait(bar, parity)) return true;
   uint64_t t0 = 0;
   for (uint32_t it = 0;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
@@ -100,6 +116,16 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
       }
     }
   }
+}
+
+// ------------------------------------------------- programmatic launch
+// Kernels launched with programmatic stream serialization may start while
+// the previous kernel in the stream is still running; they must wait here
+// before touching anything that kernel writes.  Every CTA calls it, so a
+// grid never completes before the grids it depends on.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
 // ---------------------------------------------------------------- TMA

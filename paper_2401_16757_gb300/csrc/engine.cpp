@@ -310,6 +310,7 @@ static bool unit_gemm(const swapnet_engine* e, const Unit& U, const UnitExec& X,
   std::memset(g, 0, sizeof(*g));
   g->dtype = m.dtype;
   g->num_sms = e->num_sms;
+  g->cluster_max = 16;
   g->W = X.w;
   g->e.bias = X.b;
   g->e.act = L.d.act;
@@ -557,17 +558,25 @@ int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint
 namespace swapnet {
 
 // Enqueue one inference: swaps on the copy stream, layers on `s`.
-// Inside a graph capture a slot's first use in the inference has no
-// in-graph predecessor to wait for (the graph as a whole is ordered after
-// earlier work on the launch stream), so that wait is omitted.
+// Enqueue one inference: swaps on the copy stream, layers on `s`.  Each
+// inference is self-contained: the copy stream forks from `s` (so swaps
+// start after everything already queued on `s`, which also orders them
+// after the previous inference's use of the slots), a slot's later reuse
+// waits for the block that last used it in this inference, and the copy
+// stream joins `s` again at the end.  The same sequence is captured as a
+// graph, where the fork, the slot gating and the join become graph edges.
 static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t s, bool capturing = false) {
   const swapnet_plan& p = e->plan;
   const bool prof = e->profiling && !capturing;
   bool used[2] = {false, false};
+  if (!p.resident) {
+    CU(cudaEventRecord(e->fork, s), "record fork");
+    CU(cudaStreamWaitEvent(e->copy, e->fork, 0), "wait fork");
+  }
   for (size_t k = 0; k < p.blocks.size(); ++k) {
     const Block& B = p.blocks[k];
     if (!p.resident) {
-      if (!capturing || used[B.slot]) CU(cudaStreamWaitEvent(e->copy, e->slot_free[B.slot], 0), "wait slot");
+      if (used[B.slot]) CU(cudaStreamWaitEvent(e->copy, e->slot_free[B.slot], 0), "wait slot");
       used[B.slot] = true;
       if (prof) CU(cudaEventRecord(e->ev_swap[2 * k], e->copy), "profile event");
       int rc = swap_block(e, k, e->blocks[k].variant, e->copy);
@@ -583,6 +592,10 @@ static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t 
       if (prof) CU(cudaEventRecord(e->ev_unit[2 * u + 1], s), "profile event");
     }
     if (!p.resident) CU(cudaEventRecord(e->slot_free[B.slot], s), "record slot free");
+  }
+  if (!p.resident) {
+    CU(cudaEventRecord(e->join, e->copy), "record join");
+    CU(cudaStreamWaitEvent(s, e->join, 0), "wait join");
   }
   return SWAPNET_OK;
 }
@@ -601,22 +614,8 @@ static uint64_t launches_per_infer(const swapnet_engine* e) {
 static int capture(swapnet_engine* e, const void* din, void* dout, cudaGraphExec_t* out) {
   const swapnet_engine_stats saved = e->stats;
   CU(cudaStreamBeginCapture(e->cap, cudaStreamCaptureModeThreadLocal), "begin capture");
-  int rc = SWAPNET_OK;
   cudaGraph_t g = nullptr;
-  do {
-    if (!e->plan.resident) {
-      if (cudaEventRecord(e->fork, e->cap) != cudaSuccess || cudaStreamWaitEvent(e->copy, e->fork, 0) != cudaSuccess) {
-        rc = SWAPNET_ERR_CUDA;
-        break;
-      }
-    }
-    rc = enqueue(e, din, dout, e->cap, true);
-    if (rc) break;
-    if (!e->plan.resident) {
-      if (cudaEventRecord(e->join, e->copy) != cudaSuccess || cudaStreamWaitEvent(e->cap, e->join, 0) != cudaSuccess)
-        rc = SWAPNET_ERR_CUDA;
-    }
-  } while (0);
+  const int rc = enqueue(e, din, dout, e->cap, true);
   const cudaError_t ee = cudaStreamEndCapture(e->cap, &g);
   e->stats = saved;
   if (rc || ee != cudaSuccess || !g) {

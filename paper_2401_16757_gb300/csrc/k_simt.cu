@@ -2,6 +2,7 @@
 // direct convolution for channel counts the tensor-core path cannot tile,
 // pooling, upsampling and channel concatenation.  NHWC everywhere.
 #include <cstdio>
+#include <cstring>
 
 #include "device.cuh"
 #include "internal.h"
@@ -12,6 +13,25 @@ namespace swapnet {
 namespace {
 
 template <typename T> struct Vec16 { static constexpr int N = 16 / sizeof(T); };
+
+// Launch with programmatic stream serialization: the kernel may start while
+// the previous kernel on the stream drains; it waits (pdl_wait) before
+// reading that kernel's output.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg;
+  std::memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
 
 __device__ __forceinline__ uint4 ld_stream16(const void* p) {
   uint4 r;
@@ -42,6 +62,8 @@ __global__ void __launch_bounds__(kSkWarps * 32) linear_skinny_kernel(const T* _
                                                                       T* __restrict__ y, int64_t ldy) {
   constexpr int V = Vec16<T>::N;
   __shared__ float red[kSkWarps][kSkCols][MT];
+  pdl_wait();
+  pdl_launch_dependents();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int o0 = blockIdx.x * kSkCols;
   const int kchunks = K / V;                       // K % V == 0 (checked on the host)
@@ -111,11 +133,11 @@ int skinny_dispatch(const void* x, int M, int K, const void* W, int N, const Epi
   const T* xp = static_cast<const T*>(x);
   const T* wp = static_cast<const T*>(W);
   T* yp = static_cast<T*>(y);
-  if (M <= 1) linear_skinny_kernel<T, 1><<<grid, block, 0, s>>>(xp, M, K, wp, N, e, yp, ldy);
-  else if (M <= 2) linear_skinny_kernel<T, 2><<<grid, block, 0, s>>>(xp, M, K, wp, N, e, yp, ldy);
-  else if (M <= 4) linear_skinny_kernel<T, 4><<<grid, block, 0, s>>>(xp, M, K, wp, N, e, yp, ldy);
-  else if (M <= 8) linear_skinny_kernel<T, 8><<<grid, block, 0, s>>>(xp, M, K, wp, N, e, yp, ldy);
-  else linear_skinny_kernel<T, 16><<<grid, block, 0, s>>>(xp, M, K, wp, N, e, yp, ldy);
+  if (M <= 1) launch_pdl(linear_skinny_kernel<T, 1>, grid, block, 0, s, xp, M, K, wp, N, e, yp, ldy);
+  else if (M <= 2) launch_pdl(linear_skinny_kernel<T, 2>, grid, block, 0, s, xp, M, K, wp, N, e, yp, ldy);
+  else if (M <= 4) launch_pdl(linear_skinny_kernel<T, 4>, grid, block, 0, s, xp, M, K, wp, N, e, yp, ldy);
+  else if (M <= 8) launch_pdl(linear_skinny_kernel<T, 8>, grid, block, 0, s, xp, M, K, wp, N, e, yp, ldy);
+  else launch_pdl(linear_skinny_kernel<T, 16>, grid, block, 0, s, xp, M, K, wp, N, e, yp, ldy);
   return cudaGetLastError() == cudaSuccess ? SWAPNET_OK : SWAPNET_ERR_CUDA;
 }
 
@@ -129,6 +151,8 @@ __global__ void __launch_bounds__(256) linear_tiled_kernel(const T* __restrict__
                                                            T* __restrict__ y, int64_t ldy) {
   __shared__ float xs[16][64 + 1];
   __shared__ float ws[16][64 + 1];
+  pdl_wait();
+  pdl_launch_dependents();
   const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
   const int m0 = blockIdx.y * 64, n0 = blockIdx.x * 64;
   float acc[4][4] = {};
@@ -188,6 +212,8 @@ __global__ void __launch_bounds__(128) conv_direct_kernel(const T* __restrict__ 
     const int co = co0 + j;
     ws[i] = co < cout ? to_f<T>(W[(int64_t)co * taps + tc]) : 0.f;
   }
+  pdl_wait();  // the filters come from the arena; the input from the previous kernel
+  pdl_launch_dependents();
   __syncthreads();
   const int64_t pix = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t npix = (int64_t)n * oh * ow;
@@ -235,6 +261,8 @@ __global__ void __launch_bounds__(128) conv_direct_kernel(const T* __restrict__ 
 template <typename T>
 __global__ void maxpool_kernel(const T* __restrict__ x, int n, int h, int w, int c, int kh, int kw, int stride,
                                int pad, int oh, int ow, T* __restrict__ y) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t total = (int64_t)n * oh * ow * c;
   if (idx >= total) return;
@@ -258,6 +286,8 @@ __global__ void maxpool_kernel(const T* __restrict__ x, int n, int h, int w, int
 
 template <typename T>
 __global__ void gap_kernel(const T* __restrict__ x, int n, int hw, int c, T* __restrict__ y) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (int64_t)n * c) return;
   const int img = (int)(idx / c), ch = (int)(idx % c);
@@ -269,6 +299,8 @@ __global__ void gap_kernel(const T* __restrict__ x, int n, int hw, int c, T* __r
 
 template <typename T>
 __global__ void upsample2x_kernel(const T* __restrict__ x, int n, int h, int w, int c, T* __restrict__ y) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t total = (int64_t)n * 2 * h * 2 * w * c;
   if (idx >= total) return;
@@ -283,6 +315,8 @@ __global__ void upsample2x_kernel(const T* __restrict__ x, int n, int h, int w, 
 template <typename T>
 __global__ void concat_kernel(const T* __restrict__ a, int ca, const T* __restrict__ b, int cb, int64_t pixels,
                               T* __restrict__ y) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int c = ca + cb;
   if (idx >= pixels * c) return;
@@ -292,6 +326,8 @@ __global__ void concat_kernel(const T* __restrict__ a, int ca, const T* __restri
 }
 
 inline int grid1d(int64_t total, int block) { return (int)((total + block - 1) / block); }
+
+
 
 }  // namespace
 
@@ -327,8 +363,8 @@ int launch_linear_tiled(int dtype, const void* x, int M, int K, const void* W, i
   if (M < 1 || K < 1 || N < 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "tiled linear: empty shape");
   const dim3 grid((N + 63) / 64, (M + 63) / 64);
   SN_DISPATCH(dtype, T,
-              linear_tiled_kernel<T><<<grid, 256, 0, s>>>(static_cast<const T*>(x), M, K, static_cast<const T*>(W), N,
-                                                           e, static_cast<T*>(y), ldy));
+              launch_pdl(linear_tiled_kernel<T>, grid, dim3(256), 0, s, static_cast<const T*>(x), M, K,
+                         static_cast<const T*>(W), N, e, static_cast<T*>(y), ldy));
   return last_launch();
 }
 
@@ -343,8 +379,8 @@ int launch_conv_direct(int dtype, const void* x, int n, int h, int w, int cin, c
     if (smem > 48 * 1024 &&
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
       SN_FAIL(SWAPNET_ERR_CUDA, "cudaFuncSetAttribute failed");
-    kern<<<grid, 128, smem, s>>>(static_cast<const T*>(x), n, h, w, cin, static_cast<const T*>(W), cout, kh, kw,
-                                 stride, pad, oh, ow, e, static_cast<T*>(y));
+    launch_pdl(kern, grid, dim3(128), smem, s, static_cast<const T*>(x), n, h, w, cin, static_cast<const T*>(W), cout,
+               kh, kw, stride, pad, oh, ow, e, static_cast<T*>(y));
   });
   return last_launch();
 }
@@ -353,23 +389,23 @@ int launch_maxpool(int dtype, const void* x, int n, int h, int w, int c, int kh,
                    int oh, int ow, void* y, cudaStream_t s) {
   const int64_t total = (int64_t)n * oh * ow * c;
   SN_DISPATCH(dtype, T,
-              maxpool_kernel<T><<<grid1d(total, 256), 256, 0, s>>>(static_cast<const T*>(x), n, h, w, c, kh, kw,
-                                                                    stride, pad, oh, ow, static_cast<T*>(y)));
+              launch_pdl(maxpool_kernel<T>, dim3(grid1d(total, 256)), dim3(256), 0, s, static_cast<const T*>(x), n, h,
+                         w, c, kh, kw, stride, pad, oh, ow, static_cast<T*>(y)));
   return last_launch();
 }
 
 int launch_gap(int dtype, const void* x, int n, int h, int w, int c, void* y, cudaStream_t s) {
   SN_DISPATCH(dtype, T,
-              gap_kernel<T><<<grid1d((int64_t)n * c, 256), 256, 0, s>>>(static_cast<const T*>(x), n, h * w, c,
-                                                                         static_cast<T*>(y)));
+              launch_pdl(gap_kernel<T>, dim3(grid1d((int64_t)n * c, 256)), dim3(256), 0, s, static_cast<const T*>(x),
+                         n, h * w, c, static_cast<T*>(y)));
   return last_launch();
 }
 
 int launch_upsample2x(int dtype, const void* x, int n, int h, int w, int c, void* y, cudaStream_t s) {
   const int64_t total = (int64_t)n * 4 * h * w * c;
   SN_DISPATCH(dtype, T,
-              upsample2x_kernel<T><<<grid1d(total, 256), 256, 0, s>>>(static_cast<const T*>(x), n, h, w, c,
-                                                                       static_cast<T*>(y)));
+              launch_pdl(upsample2x_kernel<T>, dim3(grid1d(total, 256)), dim3(256), 0, s, static_cast<const T*>(x), n,
+                         h, w, c, static_cast<T*>(y)));
   return last_launch();
 }
 
@@ -377,9 +413,8 @@ int launch_concat(int dtype, const void* a, int ca, const void* b, int cb, int64
                   cudaStream_t s) {
   const int64_t total = pixels * (ca + cb);
   SN_DISPATCH(dtype, T,
-              concat_kernel<T><<<grid1d(total, 256), 256, 0, s>>>(static_cast<const T*>(a), ca,
-                                                                   static_cast<const T*>(b), cb, pixels,
-                                                                   static_cast<T*>(y)));
+              launch_pdl(concat_kernel<T>, dim3(grid1d(total, 256)), dim3(256), 0, s, static_cast<const T*>(a), ca,
+                         static_cast<const T*>(b), cb, pixels, static_cast<T*>(y)));
   return last_launch();
 }
 

@@ -41,7 +41,11 @@ template <int BN> struct Cfg {
   static constexpr int kStages = BN == 64 ? 6 : 4;
   static constexpr int kLag = kStages - 2;  // gather: cp.async groups in flight per thread
   static constexpr int kBBytes = BN * kBK * 2;
-  static constexpr int kSmem = kStages * (kABytes + kBBytes) + 1024 + 256;
+  static constexpr int kStageBytes = kStages * (kABytes + kBBytes);
+  // cluster split-K receive buffer: up to 16 splits x ceil(128/splits) rows
+  static constexpr int kRecvBytes = (kBM + 15) * (BN + 4) * 4;
+  static constexpr int kBiasBytes = BN * 4;
+  static constexpr int kSmem = kStageBytes + kRecvBytes + kBiasBytes + 256 + 1024;
 };
 
 struct TcArgs {
@@ -53,8 +57,9 @@ struct TcArgs {
   int64_t ldy;
   int* err;
   int kb_per_split;  // k-blocks per split; gridDim.z splits
-  float* partial;    // [splits][M][N] fp32 partial sums (split-K only)
-  int* counters;     // per output tile, zero between launches (split-K only)
+  float* partial;    // [splits][M][N] fp32 partial sums (global split-K only)
+  int* counters;     // per output tile, zero between launches (global split-K only)
+  int cluster;       // 1: the splits of a tile form a cluster and reduce through DSMEM
 };
 
 // ---- register-only epilogue helpers
@@ -82,18 +87,19 @@ template <> __device__ __forceinline__ float hi_f<__nv_bfloat16>(uint32_t u) { r
 
 // 8 consecutive outputs (16 bytes): acc -> bias, residual, activation -> T.
 template <typename T>
-__device__ __forceinline__ void epi8(const float (&a)[8], const T* bias, const T* res, T* out, int act,
+__device__ __forceinline__ void epi8(const float (&a)[8], const float* sb, const T* res, T* out, int act,
                                      int res_post) {
-  const uint4 b = *reinterpret_cast<const uint4*>(bias);
+  const float4 b0 = *reinterpret_cast<const float4*>(sb);
+  const float4 b1 = *reinterpret_cast<const float4*>(sb + 4);
+  const float bf[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
   uint4 r = make_uint4(0, 0, 0, 0);
   if (res) r = *reinterpret_cast<const uint4*>(res);
-  const uint32_t bw[4] = {b.x, b.y, b.z, b.w};
   const uint32_t rw[4] = {r.x, r.y, r.z, r.w};
   uint32_t o[4];
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    const float v0 = epilogue(a[2 * i], lo_f<T>(bw[i]), lo_f<T>(rw[i]), res != nullptr, act, res_post);
-    const float v1 = epilogue(a[2 * i + 1], hi_f<T>(bw[i]), hi_f<T>(rw[i]), res != nullptr, act, res_post);
+    const float v0 = epilogue(a[2 * i], bf[2 * i], lo_f<T>(rw[i]), res != nullptr, act, res_post);
+    const float v1 = epilogue(a[2 * i + 1], bf[2 * i + 1], hi_f<T>(rw[i]), res != nullptr, act, res_post);
     o[i] = pack2<T>(v0, v1);
   }
   *reinterpret_cast<uint4*>(out) = make_uint4(o[0], o[1], o[2], o[3]);
@@ -101,8 +107,8 @@ __device__ __forceinline__ void epi8(const float (&a)[8], const T* bias, const T
 
 // Final epilogue of 32 columns [n, n+32) of row m from fp32 values v.
 template <typename T>
-__device__ __forceinline__ void finish32(const float (&v)[32], const TcArgs& p, int m, int n, bool vec_ok) {
-  const T* bias = static_cast<const T*>(p.e.bias);
+__device__ __forceinline__ void finish32(const float (&v)[32], const float* sb, const TcArgs& p, int m, int n,
+                                         bool vec_ok) {
   const T* res = static_cast<const T*>(p.e.res);
   T* y = static_cast<T*>(p.y) + (int64_t)m * p.ldy;
   const T* rrow = res ? res + (int64_t)m * p.e.ldr : nullptr;
@@ -112,20 +118,50 @@ __device__ __forceinline__ void finish32(const float (&v)[32], const TcArgs& p, 
       float a[8];
 #pragma unroll
       for (int j = 0; j < 8; ++j) a[j] = v[8 * q + j];
-      epi8<T>(a, bias + n + 8 * q, rrow ? rrow + n + 8 * q : nullptr, y + n + 8 * q, p.e.act, p.e.res_post);
+      epi8<T>(a, sb + 8 * q, rrow ? rrow + n + 8 * q : nullptr, y + n + 8 * q, p.e.act, p.e.res_post);
     }
   } else {
 #pragma unroll
     for (int j = 0; j < 32; ++j) {
       if (n + j < p.N) {
         const float rv = rrow ? to_f<T>(rrow[n + j]) : 0.f;
-        y[n + j] = from_f<T>(epilogue(v[j], to_f<T>(bias[n + j]), rv, rrow != nullptr, p.e.act, p.e.res_post));
+        y[n + j] = from_f<T>(epilogue(v[j], sb[j], rv, rrow != nullptr, p.e.act, p.e.res_post));
       }
     }
   }
 }
 
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+// Final epilogue of 4 columns [n, n+4) of row m.
+template <typename T>
+__device__ __forceinline__ void finish4(const float4& v, const float* sb, const TcArgs& p, int m, int n) {
+  const T* res = static_cast<const T*>(p.e.res);
+  T* y = static_cast<T*>(p.y) + (int64_t)m * p.ldy;
+  const T* rrow = res ? res + (int64_t)m * p.e.ldr : nullptr;
+  const float a[4] = {v.x, v.y, v.z, v.w};
+  const bool vec = n + 4 <= p.N && ((p.ldy | n) % 4 == 0) && (!rrow || (p.e.ldr % 4 == 0));
+  if (vec) {
+    uint2 rr = make_uint2(0, 0);
+    if (rrow) rr = *reinterpret_cast<const uint2*>(rrow + n);
+    const float b0 = sb[0], b1 = sb[1], b2 = sb[2], b3 = sb[3];
+    const float r0 = lo_f<T>(rr.x), r1 = hi_f<T>(rr.x), r2 = lo_f<T>(rr.y), r3 = hi_f<T>(rr.y);
+    const int hr = rrow != nullptr;
+    const uint32_t w0 = pack2<T>(epilogue(a[0], b0, r0, hr, p.e.act, p.e.res_post),
+                                 epilogue(a[1], b1, r1, hr, p.e.act, p.e.res_post));
+    const uint32_t w1 = pack2<T>(epilogue(a[2], b2, r2, hr, p.e.act, p.e.res_post),
+                                 epilogue(a[3], b3, r3, hr, p.e.act, p.e.res_post));
+    *reinterpret_cast<uint2*>(y + n) = make_uint2(w0, w1);
+  } else {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      if (n + j < p.N) {
+        const float rv = rrow ? to_f<T>(rrow[n + j]) : 0.f;
+        y[n + j] = from_f<T>(epilogue(a[j], sb[j], rv, rrow != nullptr, p.e.act, p.e.res_post));
+      }
+    }
+  }
+}
 
 template <typename T, int BN, bool GATHER>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -137,7 +173,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + kStages * kABytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sB + kStages * kBBytes);
+  float* recv = reinterpret_cast<float*>(smem + Cfg<BN>::kStageBytes);
+  float* sbias = reinterpret_cast<float*>(smem + Cfg<BN>::kStageBytes + Cfg<BN>::kRecvBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Cfg<BN>::kStageBytes + Cfg<BN>::kRecvBytes + Cfg<BN>::kBiasBytes);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kStages + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   volatile int* last_flag = reinterpret_cast<volatile int*>(tmem_slot + 2);
@@ -152,6 +190,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int kb0 = blockIdx.z * p.kb_per_split;
   const int nk = min(KB, kb0 + p.kb_per_split) - kb0;  // >= 1 by construction
   const int splits = gridDim.z;
+  const bool csplit = splits > 1 && p.cluster;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -172,15 +211,32 @@ __global__ void __launch_bounds__(kThreads, 1)
     prefetch_tmap(&tmB);
     if (!GATHER) prefetch_tmap(&tmA);
   }
+  // bias of this tile to shared memory (weights: ready before the kernel)
+  if (threadIdx.x >= 64) {
+    const T* bias = static_cast<const T*>(p.e.bias);
+    for (int j = threadIdx.x - 64; j < BN; j += 128) sbias[j] = (n0 + j < p.N) ? to_f<T>(bias[n0 + j]) : 0.f;
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  pdl_launch_dependents();
+  if (csplit) asm volatile("barrier.cluster.arrive.relaxed;" ::: "memory");  // peers started (waited before DSMEM use)
 
   if (warp == 0) {
     if (lane == 0) {
-      // ---------------- TMA producer
-      int i = 0;
+      // ---------------- TMA producer: weight tiles of the first stages go
+      // out before waiting for the previous kernel (they do not depend on it)
+      const int early = min(nk, kStages);
+      for (int i = 0; i < early; ++i) {
+        mbar_arrive_expect_tx(full_bar(i), kBBytes + (GATHER ? 0 : kABytes));
+        tma_load_2d(smem_u32(sB + i * kBBytes), &tmB, full_bar(i), (kb0 + i) * kBK, n0);
+      }
+      pdl_wait();
+      if (!GATHER)
+        for (int i = 0; i < early; ++i)
+          tma_load_2d(smem_u32(sA + i * kABytes), &tmA, full_bar(i), (kb0 + i) * kBK, m0);
+      int i = early;
       for (; i < nk; ++i) {
         const int s = i % kStages, r = i / kStages, kb = kb0 + i;
         if (!mbar_wait_bounded(empty_bar(s), (r & 1) ^ 1, abort_flag, p.err)) break;
@@ -194,8 +250,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int j = (i > kStages ? i - kStages : 0); j < i; ++j)
           mbar_wait_bounded(full_bar(j % kStages), (j / kStages) & 1, &no_abort, nullptr);
       }
+    } else {
+      pdl_wait();
     }
   } else if (warp == 1) {
+    pdl_wait();
     if (lane == 0) {
       // ---------------- MMA issuer
       constexpr uint32_t idesc = idesc_f16(std::is_same<T, __nv_bfloat16>::value ? 1 : 0, kBM, BN);
@@ -213,6 +272,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     const int t = threadIdx.x - 64;  // 0..127
+    pdl_wait();
     if (GATHER) {
       // ---------------- implicit im2col gather of A (row t of the tile)
       const int m = m0 + t;
@@ -228,30 +288,45 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int iy0 = oy * p.stride - p.pad, ix0 = ox * p.stride - p.pad;
       const T* xb = static_cast<const T*>(p.x) + (int64_t)img * p.H * p.Wd * p.C;
       const uint32_t row_off = (uint32_t)((t >> 3) * 1024 + (t & 7) * 128);
+      const uint32_t sw = (uint32_t)(t & 7);
+      // position of the first K element of this split: tap (ry, rx), channel c
+      int k = kb0 * kBK;
+      int tap = k / p.C;
+      int c = k - tap * p.C;
+      int ry = tap / p.kw, rx = tap - (tap / p.kw) * p.kw;
+      const bool whole_tap = (p.C % kBK) == 0;  // a 64-wide K block never straddles taps
       int i = 0;
       for (; i < nk; ++i) {
-        const int s = i % kStages, r = i / kStages, kb = kb0 + i;
+        const int s = i % kStages, r = i / kStages;
         if (!mbar_wait_bounded(empty_bar(s), (r & 1) ^ 1, abort_flag, p.err)) break;
         const uint32_t dst_row = smem_u32(sA + s * kABytes) + row_off;
-        // the 64-wide K block starts at tap kb*64 / C (C is a multiple of 8)
-        int k = kb * kBK;
-        int tap = k / p.C;
-        int c = k - tap * p.C;
+        if (whole_tap) {
+          const int iy = iy0 + ry, ix = ix0 + rx;
+          const bool valid = mvalid && k < p.K && (unsigned)iy < (unsigned)p.H && (unsigned)ix < (unsigned)p.Wd;
+          const T* src = valid ? xb + ((int64_t)iy * p.Wd + ix) * p.C + c : static_cast<const T*>(p.x);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          bool valid = mvalid && k < p.K;
-          const T* src = static_cast<const T*>(p.x);
-          if (valid) {
-            const int ry = tap / p.kw;
-            const int rx = tap - ry * p.kw;
-            const int iy = iy0 + ry, ix = ix0 + rx;
-            valid = (unsigned)iy < (unsigned)p.H && (unsigned)ix < (unsigned)p.Wd;
-            if (valid) src = xb + ((int64_t)iy * p.Wd + ix) * p.C + c;
+          for (int j = 0; j < 8; ++j) cp_async_16(dst_row + (((uint32_t)j ^ sw) << 4), src + (valid ? 8 * j : 0), valid);
+          k += kBK;
+          c += kBK;
+          if (c == p.C) {
+            c = 0;
+            if (++rx == p.kw) { rx = 0; ++ry; }
           }
-          cp_async_16(dst_row + (uint32_t)((j ^ (t & 7)) << 4), src, valid);
-          k += 8;
-          c += 8;
-          if (c == p.C) { c = 0; ++tap; }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int iy = iy0 + ry, ix = ix0 + rx;
+            const bool valid =
+                mvalid && k < p.K && (unsigned)iy < (unsigned)p.H && (unsigned)ix < (unsigned)p.Wd;
+            const T* src = valid ? xb + ((int64_t)iy * p.Wd + ix) * p.C + c : static_cast<const T*>(p.x);
+            cp_async_16(dst_row + (((uint32_t)j ^ sw) << 4), src, valid);
+            k += 8;
+            c += 8;
+            if (c == p.C) {
+              c = 0;
+              if (++rx == p.kw) { rx = 0; ++ry; }
+            }
+          }
         }
         cp_async_commit();
         if (i >= kLag) {
@@ -266,7 +341,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     // ---------------- epilogue
     const int q = warp & 3;
-    const int m = m0 + q * 32 + lane;
+    const int row = q * 32 + lane;
+    const int m = m0 + row;
     const bool ok = mbar_wait_bounded(accum_bar, 0, abort_flag, p.err);
     tc_fence_after();
     const bool vec_ok = ((p.ldy | n0) % 8 == 0) && (!p.e.res || ((p.e.ldr | n0) % 8 == 0));
@@ -280,12 +356,37 @@ __global__ void __launch_bounds__(kThreads, 1)
           float v[32];
 #pragma unroll
           for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-          finish32<T>(v, p, m, n0 + c0, vec_ok);
+          finish32<T>(v, sbias + c0, p, m, n0 + c0, vec_ok);
+        }
+      }
+    } else if (csplit) {
+      // cluster split-K: push this split's rows to the CTA that owns them
+      // (owner of row w = w / rows_per_owner), slot = this split's index
+      const int rpo = (kBM + splits - 1) / splits;
+      const uint32_t owner = (uint32_t)(row / rpo);
+      const int rr = row - (int)owner * rpo;
+      const uint32_t base = smem_u32(recv) + (uint32_t)(((blockIdx.z * rpo + rr) * (BN + 4)) * 4);
+      asm volatile("barrier.cluster.wait;" ::: "memory");  // every peer is running
+#pragma unroll 1
+      for (int c0 = 0; c0 < BN; c0 += 32) {
+        uint32_t r[32];
+        tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)c0, r);
+        tmem_ld_wait();
+        if (ok && m < p.M) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            uint32_t ra;
+            asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(base + (uint32_t)((c0 + 4 * j) * 4)), "r"(owner));
+            asm volatile("st.shared::cluster.v4.f32 [%0], {%1,%2,%3,%4};" ::"r"(ra), "f"(__uint_as_float(r[4 * j])),
+                         "f"(__uint_as_float(r[4 * j + 1])), "f"(__uint_as_float(r[4 * j + 2])),
+                         "f"(__uint_as_float(r[4 * j + 3]))
+                         : "memory");
+          }
         }
       }
     } else if (ok) {
-      // split-K: publish the fp32 partial tile, then the last CTA of this
-      // tile sums all partials in split order and applies the epilogue.
+      // global split-K: publish the fp32 partial tile, then the last CTA of
+      // this tile sums all partials in split order and applies the epilogue.
       float* part = p.partial + ((int64_t)blockIdx.z * p.M) * p.N;
       const bool pvec = (p.N % 4 == 0);
 #pragma unroll 1
@@ -342,9 +443,30 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (n + j < p.N) v[j] += __ldcg(src + j);
             }
           }
-          finish32<T>(v, p, m, n, vec_ok);
+          finish32<T>(v, sbias + c0, p, m, n, vec_ok);
         }
       }
+    }
+  }
+  if (csplit) {
+    if (threadIdx.x < 64) asm volatile("barrier.cluster.wait;" ::: "memory");  // pairs the early arrive
+    // all pushes are visible after this barrier; each CTA reduces the rows
+    // it owns from its own receive buffer, in split order 0..S-1
+    asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+    const int rpo = (kBM + splits - 1) / splits;
+    const int r0 = (int)blockIdx.z * rpo;
+    const int rows = max(0, min(min(rpo, kBM - r0), p.M - m0 - r0));
+    const int groups = rows * (BN / 4);
+    for (int g = threadIdx.x; g < groups; g += kThreads) {
+      const int rr = g / (BN / 4), c4 = g % (BN / 4);
+      const int n = n0 + 4 * c4;
+      const float* src = recv + rr * (BN + 4) + 4 * c4;
+      float4 acc = *reinterpret_cast<const float4*>(src);
+      for (int z = 1; z < splits; ++z) {
+        const float4 v = *reinterpret_cast<const float4*>(src + z * rpo * (BN + 4));
+        acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+      }
+      if (n < p.N) finish4<T>(acc, sbias + 4 * c4, p, m0 + r0 + rr, n);
     }
   }
   tc_fence_before();
@@ -407,12 +529,86 @@ int launch_inst(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) {
   a.kb_per_split = pl.kb_per_split;
   a.partial = g.partial;
   a.counters = g.counters;
-  if (pl.splits > 1 && (!g.partial || !g.counters)) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "split-K needs scratch");
+  if (pl.splits > 1 && !pl.cluster && (!g.partial || !g.counters))
+    SN_FAIL(SWAPNET_ERR_INVALID_ARG, "split-K needs scratch");
   const dim3 grid((g.M + kBM - 1) / kBM, (g.N + BN - 1) / BN, pl.splits);
-  kern<<<grid, kThreads, Cfg<BN>::kSmem, s>>>(pl.tmA, pl.tmB, a);
-  const cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) SN_FAIL(SWAPNET_ERR_CUDA, std::string("tcgen05 GEMM launch: ") + cudaGetErrorString(e));
+  a.cluster = pl.cluster;
+  const bool csplit = pl.splits > 1 && pl.cluster;
+  if (csplit) {
+    static bool np_done = false;  // per instantiation
+    if (!np_done) {
+      if (cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)
+        SN_FAIL(SWAPNET_ERR_CUDA, "non-portable cluster attribute failed");
+      np_done = true;
+    }
+  }
+  cudaLaunchConfig_t cfg;
+  std::memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = Cfg<BN>::kSmem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  int na = 0;
+  attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[na].val.programmaticStreamSerializationAllowed = 1;
+  ++na;
+  if (csplit) {
+    attr[na].id = cudaLaunchAttributeClusterDimension;
+    attr[na].val.clusterDim.x = 1;
+    attr[na].val.clusterDim.y = 1;
+    attr[na].val.clusterDim.z = pl.splits;
+    ++na;
+  }
+  cfg.attrs = attr;
+  cfg.numAttrs = na;
+  const cudaError_t le = cudaLaunchKernelEx(&cfg, kern, pl.tmA, pl.tmB, a);
+  if (le != cudaSuccess) SN_FAIL(SWAPNET_ERR_CUDA, std::string("tcgen05 GEMM launch: ") + cudaGetErrorString(le));
   return SWAPNET_OK;
+}
+
+
+// Largest cluster (along the split dimension) that the device can co-schedule
+// for this kernel instance: 16, 8, 4 or 2 (cached per instance).
+template <typename T, int BN, bool GATHER>
+int max_cluster_inst() {
+  static int cached = -1;
+  if (cached >= 0) return cached;
+  auto kern = tc_gemm_kernel<T, BN, GATHER>;
+  cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<BN>::kSmem);
+  cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  int best = 1;
+  for (int c : {16, 8, 4, 2}) {
+    cudaLaunchConfig_t cfg;
+    std::memset(&cfg, 0, sizeof(cfg));
+    cfg.gridDim = dim3(1, 1, c);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = Cfg<BN>::kSmem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = c;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) == cudaSuccess && n > 0) {
+      best = c;
+      break;
+    }
+    cudaGetLastError();
+  }
+  cached = best;
+  return best;
+}
+
+int max_cluster(int dtype, int bn, bool gather) {
+  const bool bf = dtype == SWAPNET_BF16;
+  if (bn == 64)
+    return gather ? (bf ? max_cluster_inst<__nv_bfloat16, 64, true>() : max_cluster_inst<__half, 64, true>())
+                  : (bf ? max_cluster_inst<__nv_bfloat16, 64, false>() : max_cluster_inst<__half, 64, false>());
+  return gather ? (bf ? max_cluster_inst<__nv_bfloat16, 128, true>() : max_cluster_inst<__half, 128, true>())
+                : (bf ? max_cluster_inst<__nv_bfloat16, 128, false>() : max_cluster_inst<__half, 128, false>());
 }
 
 }  // namespace
@@ -434,11 +630,13 @@ int tc_prepare(const TcGemm& g, TcPlan* p) {
   const int64_t tiles = (int64_t)((g.M + kBM - 1) / kBM) * ((g.N + p->bn - 1) / p->bn);
   const int KB = (g.K + kBK - 1) / kBK;
   int64_t splits = tiles >= sms ? 1 : std::min<int64_t>(sms / tiles, std::max(1, KB / 2));
-  splits = std::max<int64_t>(1, std::min<int64_t>(splits, 32));
+  const int cap = g.cluster_max > 0 ? std::min(g.cluster_max, max_cluster(g.dtype, p->bn, g.conv != 0)) : 32;
+  splits = std::max<int64_t>(1, std::min<int64_t>(splits, cap));
+  p->cluster = g.cluster_max > 0 ? 1 : 0;
   p->kb_per_split = (KB + (int)splits - 1) / (int)splits;
   p->splits = (KB + p->kb_per_split - 1) / p->kb_per_split;
   p->tiles = tiles;
-  p->scratch_bytes = p->splits > 1 ? (uint64_t)p->splits * g.M * g.N * sizeof(float) : 0;
+  p->scratch_bytes = (p->splits > 1 && !p->cluster) ? (uint64_t)p->splits * g.M * g.N * sizeof(float) : 0;
   int rc = make_tmap(&p->tmB, g.dtype, g.W, (uint64_t)g.K, (uint64_t)g.N, (uint64_t)g.K * 2, (uint32_t)p->bn);
   if (rc) return rc;
   if (!g.conv && g.A) {
@@ -540,7 +738,7 @@ extern "C" int swapnet_gemm_noalloc(int32_t dtype, const void* A, const void* W,
   TcPlan pl;
   int rc = tc_prepare(g, &pl);
   if (rc) return rc;
-  if (pl.splits > 1) {
+  if (pl.splits > 1) {  // cluster_max == 0: global split-K scratch
     const uint64_t counters = (uint64_t)pl.tiles * sizeof(int);
     if (counters > kNoAllocCounterBytes || kNoAllocCounterBytes + pl.scratch_bytes > kNoAllocBytes)
       SN_FAIL(SWAPNET_ERR_INVALID_ARG, "problem needs " + std::to_string(kNoAllocCounterBytes + pl.scratch_bytes) +

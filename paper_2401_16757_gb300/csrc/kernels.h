@@ -63,6 +63,8 @@ struct TcGemm {
   void* y;
   int64_t ldy;
   int num_sms;          // used by tc_prepare to size the grid
+  int cluster_max;      // > 0: split K across a thread-block cluster of at most
+                        // this many CTAs (DSMEM reduction); 0: global scratch
   float* partial;       // split-K scratch (TcPlan::scratch_bytes), set per launch
   int* counters;        // split-K tile counters (TcPlan::tiles ints, zeroed once)
 };
@@ -72,6 +74,7 @@ struct TcPlan {
   CUtensorMap tmB;
   int bn;           // N tile
   int splits;       // K splits (grid z); 1 = no split
+  int cluster;      // splits reduce through a cluster (no global scratch)
   int kb_per_split; // 64-wide k-blocks per split
   int64_t tiles;    // output tiles (split-K counters needed)
   uint64_t scratch_bytes;  // fp32 partials of all splits
