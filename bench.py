@@ -47,6 +47,25 @@ CONFIGS = {
 }
 
 
+# DRAM traffic per launch of a kernel family, from ncu (dram__bytes_read.sum
+# + dram__bytes_write.sum averaged over the launches of one swapped step of
+# the named workload), valid only for the kernel sources it was taken on.
+TRAFFIC = {
+    # (workload, kernel family): (sha1 prefix of the kernel sources, bytes per launch)
+    ("resnet50", "tc_gemm"): ("2b29561bcde9", 1419277),
+    ("resnet50", "tc_conv"): ("2b29561bcde9", 1804400),
+}
+
+
+def kernel_sources_sha():
+    import hashlib
+    h = hashlib.sha1()
+    for f in ("k_tc.cu", "k_simt.cu", "device.cuh"):
+        with open(os.path.join(ROOT, "paper_2401_16757_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:12]
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -70,7 +89,7 @@ class ClockSampler:
     def start(self):
         try:
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
-                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
@@ -200,14 +219,20 @@ def main():
     m, w, x, wb, budget, text = build_workload(args.config)
     d = capi.Desc(m)
     variant = {"auto": capi.SWAP_AUTO, "memcpy": capi.SWAP_MEMCPY, "zerocopy": capi.SWAP_ZEROCOPY}[args.variant]
-    if args.config == "mlp6":
-        opt = capi.options(slots=2, activations_in_budget=1, swap_variant=variant)
-    else:
-        opt = capi.options(swap_variant=variant)
-    plan = capi.Plan.partition(d, budget, opt)
+    act_in = 1 if args.config == "mlp6" else 0
+    opt0 = capi.options(slots=2, activations_in_budget=act_in, swap_variant=variant)
+    host = capi.HostWeights(w)
+    # offline profiling (Sec. 6.1): plan with default coefficients, measure
+    # every layer's execution delay and the link on this GPU, then plan again
+    plan0 = capi.Plan.partition(d, budget, opt0)
+    eng0 = capi.Engine(plan0, host)
+    t_ex, alpha = capi.calibrate(m, plan0, eng0)
+    dc = capi.Desc(m, t_ex_ns=t_ex)
+    opt = capi.options(slots=2, activations_in_budget=act_in, swap_variant=variant,
+                       alpha_as_per_byte=alpha or 4_750_000, beta_ns_per_tensor=0, eta_ns_per_tensor=0)
+    plan = capi.Plan.partition(dc, budget, opt)
     rplan = capi.Plan.resident(d)
     info = plan.info()
-    host = capi.HostWeights(w)
     eng = capi.Engine(plan, host)
     reng = capi.Engine(rplan, host)
     stream = torch.cuda.current_stream()
@@ -242,7 +267,9 @@ def main():
     torch.cuda.synchronize()
     launches0 = eng.stats()["kernel_launches"]
     t_wall0 = time.perf_counter()
+    torch.cuda.nvtx.range_push("swapped_steps")  # ncu --nvtx --nvtx-include swapped_steps/
     ms_list = timed(eng, args.steps)
+    torch.cuda.nvtx.range_pop()
     t_wall = time.perf_counter() - t_wall0
     launches = eng.stats()["kernel_launches"] - launches0
     if dist:
@@ -260,6 +287,11 @@ def main():
     # ---- DInf: same kernels, weights resident
     ms_dinf_list = timed(reng, args.steps)
     ms_dinf = sum(ms_dinf_list) / len(ms_dinf_list)
+    # ---- the plan made with the default (uncalibrated) coefficients
+    for _ in range(3):
+        eng0.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
+    ms_uncal_list = timed(eng0, min(args.steps, 50))
+    ms_uncal = sum(ms_uncal_list) / len(ms_uncal_list)
 
     # ---- e2e: host buffers through swapnet_infer_host
     h_in = torch.empty(info["input_bytes"], dtype=torch.uint8, pin_memory=True)
@@ -308,8 +340,11 @@ def main():
     roofline = {"bound": "tensor", "kernel": dom, "launches_per_step": len(dom_idx),
                 "achieved": achieved_tf, "peak": tf_burst, "unit": "TFLOP/s",
                 "frac": achieved_tf / tf_burst, "peak_source": peak_src + " bf16 burst",
-                "traffic": None, "share_of_kernel_time": dom_us / max(1e-9, acc_u.sum()),
+                "traffic": None, "kernel_sources_sha": kernel_sources_sha(), "share_of_kernel_time": dom_us / max(1e-9, acc_u.sum()),
                 "kernel_time_share": {k: round(v / max(1e-9, acc_u.sum()), 4) for k, v in share.items()}}
+    tr = TRAFFIC.get((args.config, dom))
+    if tr and tr[0] == roofline["kernel_sources_sha"]:
+        roofline["traffic"] = tr[1]
     if dom in ("skinny_linear", "maxpool", "gap", "upsample2x", "concat"):
         roofline.update(bound="hbm", unit="GB/s", peak=hbm, peak_source=peak_src + " copy")
 
@@ -347,6 +382,8 @@ def main():
                        "workspace_bytes": info["workspace_bytes"], "l2": "flushed (512 MiB write) before each step",
                        "swap_variants": [b["variant"] for b in eb], "parallelism": "replicas" if world > 1 else "1 GPU"},
             "dinf_ms": ms_dinf, "ratio": ms_swapped / ms_dinf,
+            "predicted_ms": info["predicted_ns"] / 1e6,
+            "uncalibrated_plan": {"cuts": plan0.cuts(), "ms": ms_uncal},
             "p50_ms": statistics.median(ms_list), "p99_ms": float(np.percentile(ms_list, 99)),
             "e2e": {"value": e2e_val, "unit": "inferences/s", "h2d_bytes_per_step": info["input_bytes"],
                     "d2h_bytes_per_step": info["output_bytes"]},

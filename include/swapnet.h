@@ -131,7 +131,7 @@ typedef struct swapnet_plan_info {
   uint32_t n_layers;
   uint64_t budget_bytes;
   uint64_t arena_bytes;    /* device bytes for weights                       */
-  uint64_t slot_bytes;     /* capacity of one slot                           */
+  uint64_t slot_bytes;     /* largest piece of a split linear layer          */
   uint64_t workspace_bytes;/* intermediate activations (liveness-planned)    */
   uint64_t input_bytes;    /* model input                                    */
   uint64_t output_bytes;   /* all model outputs, 256-byte aligned each       */
@@ -152,17 +152,22 @@ typedef struct swapnet_unit_info {
 
 typedef struct swapnet_block_info {
   uint32_t unit0, unit1; /* units [unit0, unit1)                             */
-  uint32_t slot;         /* arena slot the block is swapped into             */
+  uint32_t slot;         /* block parity: which co-resident position it takes */
   uint32_t depth;
   uint64_t bytes;
   int64_t t_in_ns, t_ex_ns, t_out_ns;
+  uint64_t offset;       /* byte offset of the block in the arena            */
 } swapnet_block_info;
 
 /* Partition the model for a budget (Sec. 6.2.2, Eq. 2-3; objective per
- * opt->objective).  Every block must fit one slot of floor(arena/slots)
- * bytes (arena = budget, minus the workspace when activations_in_budget).
- * A linear layer larger than a slot is split along output features into
- * pieces of a multiple of 128 features.  Ties: fewer blocks, then the
+ * opt->objective).  The arena is the budget (minus the workspace when
+ * activations_in_budget), rounded down to 256 bytes.  With two co-resident
+ * blocks every pair of consecutive blocks must fit the arena together
+ * (Eq. 3: s_i + s_{i+1} <= b): even blocks are placed at the bottom of the
+ * arena and odd blocks against its top.  With one slot each block must fit
+ * the arena alone.  A linear layer larger than slot_bytes (half the arena
+ * with two blocks) is split along output features into pieces of a
+ * multiple of 128 features.  Ties: fewer blocks, then the
  * lexicographically smallest cut vector.  Host only; no device work.
  * Errors: INVALID_ARG (descriptor/options), INFEASIBLE (no partition). */
 int swapnet_partition(const swapnet_model_desc* desc, uint64_t budget_bytes,
@@ -287,6 +292,15 @@ int swapnet_engine_unit_kernels(const swapnet_engine* eng, int32_t* kinds, uint3
  * swapnet_engine_last_times synchronises and returns, for the most recent
  * profiled inference, microseconds per unit and per block swap-in. */
 int swapnet_engine_set_profiling(swapnet_engine* eng, int enable);
+
+/* Offline profiling of the execution delays (Sec. 6.1: the paper fits its
+ * coefficients once per device).  Times every unit's kernel on the engine's
+ * device as a graph of `reps` back-to-back launches (so consecutive launches
+ * overlap as they do inside an inference) and writes microseconds per launch
+ * to unit_us[0..n_units).  The values a unit reads are whatever its buffers
+ * hold; the kernels' timing does not depend on them.  Synchronous.
+ * Errors: INVALID_ARG, OOM (staging buffers), CUDA. */
+int swapnet_engine_measure_units(swapnet_engine* eng, int32_t reps, float* unit_us, uint32_t n_units);
 int swapnet_engine_last_times(swapnet_engine* eng, float* unit_us, uint32_t n_units, float* swap_us,
                               uint32_t n_blocks);
 

@@ -12,9 +12,11 @@ per block (t_in) or per layer (t_ex).  A layer may carry a measured t_ex that
 replaces gamma * f.
 
 Sec. 6.2.2 partitions the layer sequence into n blocks, p = (p_1..p_{n-1}),
-minimising t(p) (Eq. 2) subject to the block-size constraint (Eq. 3).  With
-the arena cut into `slots` equal slots, every block must fit one slot.  The
-objective is either
+minimising t(p) (Eq. 2) subject to the block-size constraint (Eq. 3): with
+m = 2 blocks co-resident, every two consecutive blocks fit the arena together,
+s_i + s_{i+1} <= arena (the arena is the budget less the workspace when that
+is counted, rounded down to 256 bytes); with one slot, every block fits the
+arena alone.  The objective is either
   0: the completion time of the m-slot swap/execute pipeline,
        C_k = max(C_{k-1}, R_{k-m}) + t_in_k       (copy of block k ends)
        E_k = max(E_{k-1}, C_k) + t_ex_k           (execution of block k ends)
@@ -151,12 +153,15 @@ class Coef:
         self.alpha_as, self.beta_ns, self.gamma_as, self.eta_ns = alpha_as, beta_ns, gamma_as, eta_ns
 
 
-def units(model, slot, t_ex_override=None):
+def units(model, slot, t_ex_override=None, region=None):
     """Partition units: layers in order, except that a linear layer larger
-    than one slot becomes pieces of whole output features (a multiple of 128
-    per piece, as equal as that allows).  Returns a list of dicts
-    {layer, row0, rows, bytes, depth, flops, t_ex_ns} or None when some layer
-    cannot fit a slot."""
+    than `slot` (half the arena when two blocks are co-resident) becomes
+    pieces of whole output features (a multiple of 128 per piece, as equal
+    as that allows).  Other layers may be as large as `region` (the whole
+    arena).  Returns a list of dicts {layer, row0, rows, bytes, depth, flops,
+    t_ex_ovr} or None when some layer cannot fit."""
+    if region is None:
+        region = slot
     shapes = out_shapes(model)
     es = ES[model["dtype"]]
     out = []
@@ -165,7 +170,7 @@ def units(model, slot, t_ex_override=None):
         size = sum(align(b) for b in tb)
         f = layer_flops(model, li, shapes)
         ovr = 0 if t_ex_override is None else t_ex_override[li]
-        if size <= slot:
+        if size <= slot or (L["op"] != "linear" and size <= region):
             out.append(dict(layer=li, row0=0, rows=L.get("n", 0), bytes=size, depth=len(tb),
                             flops=f, t_ex_ovr=ovr))
             continue
@@ -242,12 +247,24 @@ def eq4_objective(blocks):
 
 
 def arena_and_slot(model, budget, slots, activations_in_budget):
+    """(arena, slot, workspace): slot bounds a piece of a split linear layer."""
     ws = workspace(model)[0]
     arena = budget - ws if activations_in_budget else budget
     if arena <= 0:
         return None
     slot = (arena // slots) // ALIGN * ALIGN
     return arena, slot, ws
+
+
+def feasible(blocks, region, slots):
+    """Eq. 3: consecutive blocks fit the arena together (two co-resident
+    blocks); every block fits it alone."""
+    for k, b in enumerate(blocks):
+        if b[0] > region:
+            return False
+        if slots == 2 and k > 0 and blocks[k - 1][0] + b[0] > region:
+            return False
+    return True
 
 
 def exhaustive_partition(model, budget, coef, slots=2, activations_in_budget=False,
@@ -260,7 +277,8 @@ def exhaustive_partition(model, budget, coef, slots=2, activations_in_budget=Fal
     if a is None:
         return None
     arena, slot, ws = a
-    us = units(model, slot, t_ex_override)
+    region = arena // ALIGN * ALIGN
+    us = units(model, slot, t_ex_override, region)
     if us is None:
         return None
     U = len(us)
@@ -268,7 +286,7 @@ def exhaustive_partition(model, budget, coef, slots=2, activations_in_budget=Fal
     for mask in range(1 << (U - 1)):
         cuts = tuple(c for c in range(1, U) if mask >> (c - 1) & 1)
         blocks = block_costs(us, cuts, coef)
-        if any(b[0] > slot for b in blocks):
+        if not feasible(blocks, region, slots):
             continue
         obj = pipeline_time(blocks, slots) if objective == 0 else eq4_objective(blocks)
         key = (obj, len(blocks), cuts)
@@ -287,11 +305,12 @@ def evaluate_cuts(model, budget, coef, cuts, slots=2, activations_in_budget=Fals
     if a is None:
         return None
     arena, slot, ws = a
-    us = units(model, slot, t_ex_override)
+    region = arena // ALIGN * ALIGN
+    us = units(model, slot, t_ex_override, region)
     if us is None:
         return None
     blocks = block_costs(us, cuts, coef)
-    if any(b[0] > slot for b in blocks):
+    if not feasible(blocks, region, slots):
         return None
     return pipeline_time(blocks, slots) if objective == 0 else eq4_objective(blocks)
 

@@ -57,7 +57,8 @@ class UnitInfo(C.Structure):
 
 class BlockInfo(C.Structure):
     _fields_ = [("unit0", C.c_uint32), ("unit1", C.c_uint32), ("slot", C.c_uint32), ("depth", C.c_uint32),
-                ("bytes", C.c_uint64), ("t_in_ns", C.c_int64), ("t_ex_ns", C.c_int64), ("t_out_ns", C.c_int64)]
+                ("bytes", C.c_uint64), ("t_in_ns", C.c_int64), ("t_ex_ns", C.c_int64), ("t_out_ns", C.c_int64),
+                ("offset", C.c_uint64)]
 
 
 class EngineStats(C.Structure):
@@ -79,7 +80,7 @@ EXPORTS = ["swapnet_default_options", "swapnet_partition", "swapnet_plan_from_cu
            "swapnet_plan_output_offsets", "swapnet_plan_free", "swapnet_schedule", "swapnet_load",
            "swapnet_infer", "swapnet_infer_host", "swapnet_engine_sync", "swapnet_engine_blocks",
            "swapnet_engine_free", "swapnet_engine_stats_get", "swapnet_engine_unit_kernels",
-           "swapnet_engine_set_profiling", "swapnet_engine_last_times", "swapnet_strerror", "swapnet_last_error", "swapnet_debug_fail_next", "swapnet_gemm_noalloc"]
+           "swapnet_engine_set_profiling", "swapnet_engine_last_times", "swapnet_engine_measure_units", "swapnet_strerror", "swapnet_last_error", "swapnet_debug_fail_next", "swapnet_gemm_noalloc"]
 
 _lib = None
 
@@ -124,6 +125,7 @@ def lib():
         "swapnet_engine_stats_get": (C.c_int, [P, C.POINTER(EngineStats)]),
         "swapnet_engine_unit_kernels": (C.c_int, [P, C.POINTER(C.c_int32), C.c_uint32, C.POINTER(C.c_uint32)]),
         "swapnet_engine_set_profiling": (C.c_int, [P, C.c_int]),
+        "swapnet_engine_measure_units": (C.c_int, [P, C.c_int32, C.POINTER(C.c_float), C.c_uint32]),
         "swapnet_engine_last_times": (C.c_int, [P, C.POINTER(C.c_float), C.c_uint32, C.POINTER(C.c_float),
                                                 C.c_uint32]),
         "swapnet_strerror": (C.c_char_p, [C.c_int]),
@@ -266,6 +268,27 @@ def schedule(descs, urgency, arena_bytes, opt=None):
     return list(budgets), [Plan(p) for p in plans]
 
 
+def calibrate(model, plan, engine, reps=20):
+    """Measured delay model (Sec. 6.1) from a loaded engine: per-layer t_ex
+    in ns (sum of the layer's units) and alpha in attoseconds per byte from
+    the per-block copy times measured at load.  Returns (t_ex_ns list,
+    alpha_as_per_byte or None)."""
+    units = plan.units()
+    us = engine.measure_units(len(units), reps)
+    t_ex = [0] * len(model["layers"])
+    for u, t in zip(units, us):
+        t_ex[u["layer"]] += int(round(t * 1000.0))
+    t_ex = [max(1, v) for v in t_ex]
+    alpha = None
+    blocks = plan.blocks()
+    eb = engine.blocks()
+    tot_b = sum(b["bytes"] for b, e in zip(blocks, eb) if e["memcpy_us"] > 0)
+    tot_us = sum(e["memcpy_us"] for e in eb if e["memcpy_us"] > 0)
+    if tot_b > 0 and tot_us > 0:
+        alpha = int(round(tot_us * 1e12 / tot_b))
+    return t_ex, alpha
+
+
 def gemm_noalloc(dtype, a_ptr, w_ptr, bias_ptr, y_ptr, M, N, K, act=0, stream=0):
     """Y = act(A W^T + bias) through the allocation-free entry point."""
     check(lib().swapnet_gemm_noalloc(dtype, C.c_void_p(a_ptr), C.c_void_p(w_ptr), C.c_void_p(bias_ptr),
@@ -339,6 +362,11 @@ class Engine:
 
     def set_profiling(self, enable):
         check(lib().swapnet_engine_set_profiling(self.h, 1 if enable else 0), "swapnet_engine_set_profiling")
+
+    def measure_units(self, n_units, reps=20):
+        u = (C.c_float * max(1, n_units))()
+        check(lib().swapnet_engine_measure_units(self.h, reps, u, n_units), "swapnet_engine_measure_units")
+        return list(u[:n_units])
 
     def last_times(self, n_units, n_blocks):
         u = (C.c_float * max(1, n_units))()

@@ -204,7 +204,7 @@ static int register_host(swapnet_engine* e, const void* const* hw, uint32_t nt) 
   return SWAPNET_OK;
 }
 
-static char* slot_base(swapnet_engine* e, int slot) { return e->d_arena + (uint64_t)slot * e->plan.slot; }
+static char* block_base(swapnet_engine* e, const Block& B) { return e->d_arena + B.base; }
 
 static void build_segments(swapnet_engine* e) {
   const swapnet_plan& p = e->plan;
@@ -212,7 +212,7 @@ static void build_segments(swapnet_engine* e) {
   for (size_t k = 0; k < p.blocks.size(); ++k) {
     const Block& B = p.blocks[k];
     std::vector<Segment>& segs = e->blocks[k].segs;
-    char* base = slot_base(e, B.slot);
+    char* base = block_base(e, B);
     for (int u = B.u0; u < B.u1; ++u) {
       const Unit& U = p.units[u];
       for (int t = 0; t < U.nt; ++t) {
@@ -373,7 +373,7 @@ static int prepare_units(swapnet_engine* e) {
     e->unit_kind[u] = k;
   }
   for (const Block& B : p.blocks) {
-    char* base = slot_base(e, B.slot);
+    char* base = block_base(e, B);
     for (int u = B.u0; u < B.u1; ++u) {
       const Unit& U = p.units[u];
       UnitExec& X = e->ux[u];
@@ -461,7 +461,7 @@ int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint
     SN_FAIL(SWAPNET_ERR_INVALID_ARG, "expected " + std::to_string(plan->model.n_tensors) + " host tensors");
   if (((uintptr_t)d_arena | (uintptr_t)d_workspace) % kAlign)
     SN_FAIL(SWAPNET_ERR_MISALIGNED, "device buffers must be 256-byte aligned");
-  const uint64_t arena_need = plan->resident ? plan->arena : plan->slot * (uint64_t)plan->opt.slots;
+  const uint64_t arena_need = plan->region;
   if (d_arena && arena_bytes < arena_need) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "arena buffer too small");
   if (d_workspace && workspace_bytes < plan->model.ws_bytes)
     SN_FAIL(SWAPNET_ERR_INVALID_ARG, "workspace buffer too small");
@@ -706,6 +706,57 @@ int swapnet_engine_blocks(const swapnet_engine* e, swapnet_engine_block* b, uint
     const EngBlock& B = e->blocks[i];
     b[i] = swapnet_engine_block{B.variant, (int32_t)B.segs.size(), B.memcpy_us, B.zerocopy_us};
   }
+  return SWAPNET_OK;
+}
+
+int swapnet_engine_measure_units(swapnet_engine* e, int32_t reps, float* unit_us, uint32_t n_units) {
+  if (!e || !unit_us || reps < 1 || reps > 10000) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad argument");
+  CU(cudaSetDevice(e->device), "cudaSetDevice");
+  const Model& m = e->plan.model;
+  if (!e->d_in_stage) {
+    if (cudaMalloc(&e->d_in_stage, align_up(m.in_bytes)) != cudaSuccess ||
+        cudaMalloc(&e->d_out_stage, align_up(m.out_bytes)) != cudaSuccess) {
+      cudaGetLastError();
+      SN_FAIL(SWAPNET_ERR_OOM, "staging allocation failed");
+    }
+    CU(cudaMemset(e->d_in_stage, 0, align_up(m.in_bytes)), "clear staging");
+  }
+  cudaEvent_t a, b;
+  CU(cudaEventCreate(&a), "event");
+  CU(cudaEventCreate(&b), "event");
+  int rc = SWAPNET_OK;
+  const bool prof = e->profiling;
+  e->profiling = false;
+  for (uint32_t u = 0; u < n_units && u < e->plan.units.size() && rc == SWAPNET_OK; ++u) {
+    cudaGraph_t g = nullptr;
+    cudaGraphExec_t ge = nullptr;
+    if (cudaStreamBeginCapture(e->cap, cudaStreamCaptureModeThreadLocal) != cudaSuccess) { rc = SWAPNET_ERR_CUDA; break; }
+    for (int r = 0; r < reps && rc == SWAPNET_OK; ++r) rc = run_unit(e, (int)u, e->d_in_stage, e->d_out_stage, e->cap);
+    const cudaError_t ce = cudaStreamEndCapture(e->cap, &g);
+    if (rc || ce != cudaSuccess || cudaGraphInstantiate(&ge, g, 0) != cudaSuccess) {
+      if (g) cudaGraphDestroy(g);
+      cudaGetLastError();
+      rc = rc ? rc : SWAPNET_ERR_CUDA;
+      break;
+    }
+    cudaGraphDestroy(g);
+    float best = 1e30f;
+    for (int t = 0; t < 3; ++t) {
+      cudaEventRecord(a, e->cap);
+      cudaGraphLaunch(ge, e->cap);
+      cudaEventRecord(b, e->cap);
+      if (cudaEventSynchronize(b) != cudaSuccess) { rc = SWAPNET_ERR_CUDA; break; }
+      float ms = 0.f;
+      cudaEventElapsedTime(&ms, a, b);
+      if (t > 0) best = std::min(best, ms);  // the first replay warms caches
+    }
+    cudaGraphExecDestroy(ge);
+    unit_us[u] = best * 1000.f / (float)reps;
+  }
+  e->profiling = prof;
+  cudaEventDestroy(a);
+  cudaEventDestroy(b);
+  if (rc) SN_FAIL(rc, "unit measurement failed");
   return SWAPNET_OK;
 }
 

@@ -68,6 +68,7 @@ struct Unit {
 struct Block {
   int u0, u1, slot, depth;
   uint64_t bytes;
+  uint64_t base;  // offset of the block in the arena
   int64_t t_in, t_ex, t_out;
 };
 
@@ -77,7 +78,10 @@ struct swapnet_plan {
   swapnet::Model model;
   swapnet_options opt;
   bool resident = false;
-  uint64_t budget = 0, arena = 0, slot = 0;
+  // arena: bytes the blocks share; region: the 256-aligned part blocks use;
+  // slot: largest piece of a split linear layer (half the region for two
+  // co-resident blocks), also the bound for one block with one slot
+  uint64_t budget = 0, arena = 0, region = 0, slot = 0;
   std::vector<swapnet::Unit> units;
   std::vector<swapnet::Block> blocks;
   std::vector<uint32_t> cuts;
@@ -86,7 +90,7 @@ struct swapnet_plan {
 
 namespace swapnet {
 int analyse_model(const swapnet_model_desc* desc, Model* m);
-int make_units(const Model& m, const swapnet_options& opt, uint64_t slot, std::vector<Unit>* out);
+int make_units(const Model& m, const swapnet_options& opt, uint64_t slot, uint64_t region, std::vector<Unit>* out);
 void finalize_blocks(swapnet_plan* p, const std::vector<uint32_t>& cuts);
 int64_t pipeline_ns(const std::vector<Block>& b, int slots);
 int64_t eq4_ns(const std::vector<Block>& b);

@@ -188,14 +188,14 @@ static int64_t unit_tex(const Model& m, const swapnet_options& opt, const Layer&
   return (int64_t)mul_div_ceil(opt.gamma_as_per_flop, flops, 1000000000ull);
 }
 
-int make_units(const Model& m, const swapnet_options& opt, uint64_t slot, std::vector<Unit>* out) {
+int make_units(const Model& m, const swapnet_options& opt, uint64_t slot, uint64_t region, std::vector<Unit>* out) {
   out->clear();
   const uint64_t es = m.es;
   for (int li = 0; li < (int)m.L.size(); ++li) {
     const Layer& L = m.L[li];
     uint64_t size = 0;
     for (int t = 0; t < L.n_tensors; ++t) size += align_up(L.tbytes[t]);
-    if (size <= slot) {
+    if (size <= slot || (L.d.op != SWAPNET_OP_LINEAR && size <= region)) {
       Unit u{};
       u.layer = li; u.row0 = 0; u.rows = (L.d.op == SWAPNET_OP_LINEAR) ? L.d.cout : 0;
       u.depth = L.n_tensors; u.bytes = size; u.flops = L.flops;
@@ -209,7 +209,7 @@ int make_units(const Model& m, const swapnet_options& opt, uint64_t slot, std::v
     }
     if (L.d.op != SWAPNET_OP_LINEAR)
       SN_FAIL(SWAPNET_ERR_INFEASIBLE, "layer " + std::to_string(li) + " (" + std::to_string(size) +
-                                          " B) does not fit a slot of " + std::to_string(slot) + " B");
+                                          " B) does not fit the arena of " + std::to_string(region) + " B");
     const uint64_t K = L.d.cin, N = L.d.cout;
     auto piece_bytes = [&](uint64_t r) { return align_up(r * K * es) + align_up(r * es); };
     uint64_t rmax = 0;
@@ -285,6 +285,10 @@ void finalize_blocks(swapnet_plan* p, const std::vector<uint32_t>& cuts) {
   for (size_t k = 0; k + 1 < b.size(); ++k) {
     Block B = make_block(p->units, (int)b[k], (int)b[k + 1], p->opt);
     B.slot = (int)(k % slots);
+    // two co-resident blocks (Eq. 3): even blocks from the bottom of the
+    // region, odd blocks against its top, so s_k + s_{k+1} <= region keeps
+    // consecutive blocks apart
+    B.base = (slots == 2 && (k % 2) == 1) ? p->region - B.bytes : 0;
     // slot layout: tensors in unit order, 256-byte aligned
     uint64_t off = 0;
     for (int u = B.u0; u < B.u1; ++u) {
@@ -303,10 +307,17 @@ void finalize_blocks(swapnet_plan* p, const std::vector<uint32_t>& cuts) {
 }
 
 // ----------------------------------------------------------- partition search
+// Feasibility of consecutive blocks: each fits the region; with two
+// co-resident blocks every adjacent pair fits it together (Eq. 3).
+static bool pair_ok(const swapnet_plan* p, uint64_t prev_bytes, uint64_t bytes) {
+  if (bytes > p->region) return false;
+  return p->opt.slots != 2 || prev_bytes + bytes <= p->region;
+}
+
 namespace {
 
 struct State {
-  int64_t v[4];     // C, E, R_{k-1}, R_k (m = 2) or C, E, R_k, 0 (m = 1)
+  int64_t v[5];     // C, E, R_{k-1}, R_k (m = 2) or C, E, R_k, 0 (m = 1); bytes of the last block
   int nblocks;
   int prev_j;       // boundary of the previous state
   int prev_idx;     // index in the previous frontier
@@ -343,7 +354,7 @@ struct Search {
   }
 
   static bool le_all(const State& a, const State& b) {
-    for (int t = 0; t < 4; ++t)
+    for (int t = 0; t < 5; ++t)
       if (a.v[t] > b.v[t]) return false;
     return true;
   }
@@ -373,6 +384,7 @@ struct Search {
       const int64_t E = std::max(s.v[1], C) + B.t_ex;
       r.v[0] = C; r.v[1] = E; r.v[2] = E + B.t_out; r.v[3] = 0;
     }
+    r.v[4] = slots == 2 ? (int64_t)B.bytes : 0;
     r.nblocks = s.nblocks + 1;
     return r;
   }
@@ -392,9 +404,10 @@ static int search_pipeline(swapnet_plan* p, std::vector<uint32_t>* best_cuts) {
     // rebuild the frontier list copy, since insert() on j' > j does not touch it
     for (int idx = 0; idx < (int)S.front[j].size(); ++idx) {
       uint64_t bytes = 0;
+      const uint64_t prev = (uint64_t)S.front[j][idx].v[4];
       for (int j2 = j + 1; j2 <= U; ++j2) {
         bytes += p->units[j2 - 1].bytes;
-        if (bytes > p->slot) break;
+        if (!pair_ok(p, prev, bytes)) break;
         Block B = make_block(p->units, j, j2, p->opt);
         State c = S.step(S.front[j][idx], B);
         c.prev_j = j; c.prev_idx = idx;
@@ -431,7 +444,7 @@ static int search_exhaustive_eq4(swapnet_plan* p, std::vector<uint32_t>* best_cu
     bool ok = true;
     for (size_t k = 0; k + 1 < b.size(); ++k) {
       Block B = make_block(p->units, (int)b[k], (int)b[k + 1], p->opt);
-      if (B.bytes > p->slot) { ok = false; break; }
+      if (!pair_ok(p, blocks.empty() ? 0 : blocks.back().bytes, B.bytes)) { ok = false; break; }
       blocks.push_back(B);
     }
     if (!ok) continue;
@@ -468,8 +481,9 @@ static int prepare(const swapnet_model_desc* desc, uint64_t budget, const swapne
   if (p->opt.activations_in_budget && budget <= ws)
     SN_FAIL(SWAPNET_ERR_INFEASIBLE, "budget does not cover the activation workspace");
   p->arena = p->opt.activations_in_budget ? budget - ws : budget;
+  p->region = p->arena / kAlign * kAlign;
   p->slot = (p->arena / (uint64_t)p->opt.slots) / kAlign * kAlign;
-  rc = make_units(p->model, p->opt, p->slot, &p->units);
+  rc = make_units(p->model, p->opt, p->slot, p->region, &p->units);
   if (rc) return rc;
   *out = std::move(p);
   return SWAPNET_OK;
@@ -528,8 +542,9 @@ int swapnet_plan_from_cuts(const swapnet_model_desc* desc, const uint32_t* cuts,
       prev = v;
     }
     finalize_blocks(p.get(), c);
-    for (const Block& B : p->blocks)
-      if (B.bytes > p->slot) SN_FAIL(SWAPNET_ERR_INFEASIBLE, "a block exceeds the slot");
+    for (size_t k = 0; k < p->blocks.size(); ++k)
+      if (!pair_ok(p.get(), k ? p->blocks[k - 1].bytes : 0, p->blocks[k].bytes))
+        SN_FAIL(SWAPNET_ERR_INFEASIBLE, "a block (or two adjacent blocks) exceeds the arena");
     *out = p.release();
     return SWAPNET_OK;
   } catch (const std::bad_alloc&) {
@@ -548,9 +563,10 @@ int swapnet_plan_resident(const swapnet_model_desc* desc, const swapnet_options*
     if (rc) return rc;
     p->resident = true;
     p->arena = p->model.weight_bytes;
+    p->region = p->arena;
     p->slot = p->arena;
     p->budget = p->arena;
-    rc = make_units(p->model, p->opt, ~0ull, &p->units);
+    rc = make_units(p->model, p->opt, ~0ull, ~0ull, &p->units);
     if (rc) return rc;
     finalize_blocks(p.get(), {});
     *out = p.release();
@@ -604,7 +620,7 @@ int swapnet_plan_blocks(const swapnet_plan* p, swapnet_block_info* b, uint32_t c
   for (uint32_t i = 0; b && i < cap && i < p->blocks.size(); ++i) {
     const Block& B = p->blocks[i];
     b[i] = swapnet_block_info{(uint32_t)B.u0, (uint32_t)B.u1, (uint32_t)B.slot, (uint32_t)B.depth, B.bytes,
-                              B.t_in, B.t_ex, B.t_out};
+                              B.t_in, B.t_ex, B.t_out, B.base};
   }
   return SWAPNET_OK;
 }

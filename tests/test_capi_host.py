@@ -119,7 +119,8 @@ def test_units_workspace_match_oracle(name):
     opt = capi.options()
     budget = wb * 3 // 10 // 256 * 256
     a = P.arena_and_slot(m, budget, 2, False)
-    ref_units = P.units(m, a[1])
+    region = a[0] // 256 * 256
+    ref_units = P.units(m, a[1], None, region)
     plan = capi.Plan.partition(capi.Desc(m), budget, opt)
     info = plan.info()
     ws, offs, ob, oo = P.workspace(m)
@@ -131,9 +132,14 @@ def test_units_workspace_match_oracle(name):
     for g, u in zip(got, ref_units):
         assert (g["layer"], g["bytes"], g["depth"], g["flops"]) == (u["layer"], u["bytes"], u["depth"], u["flops"])
         assert g["t_ex_ns"] == P.unit_t_ex(u, _coef(opt))
-    # every block fits its slot; blocks alternate slots
-    for k, b in enumerate(plan.blocks()):
-        assert b["bytes"] <= info["slot_bytes"] and b["slot"] == k % 2
+    # Eq. 3: consecutive blocks fit the arena together; even blocks at the
+    # bottom, odd blocks against the top, so neighbours never overlap
+    blocks = plan.blocks()
+    for k, b in enumerate(blocks):
+        assert b["bytes"] <= region and b["slot"] == k % 2
+        assert b["offset"] == (0 if k % 2 == 0 else region - b["bytes"])
+        if k:
+            assert blocks[k - 1]["bytes"] + b["bytes"] <= region
 
 
 def test_plan_from_cuts_and_predicted():

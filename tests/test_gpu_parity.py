@@ -172,3 +172,27 @@ def test_swap_variants_bit_exact_resnet():
     outs = [Runner(m, w, capi.Plan.partition(d, budget, capi.options(swap_variant=v)), host).run(x)[0].tobytes()
             for v in (capi.SWAP_MEMCPY, capi.SWAP_ZEROCOPY)]
     assert outs[0] == outs[1]
+
+
+def test_calibrated_plan_is_exact_and_feasible():
+    """Offline profiling (measured per-layer t_ex and link alpha) changes the
+    partition, never the result."""
+    m = synth.arch.resnet50()
+    w = synth.gen.model_weights(m)
+    x = synth.gen.model_input(m)
+    d = capi.Desc(m)
+    host = capi.HostWeights(w)
+    budget = int(OP.weight_bytes(m) * 0.4) // 256 * 256
+    p0 = capi.Plan.partition(d, budget, capi.options())
+    r0 = Runner(m, w, p0, host)
+    t_ex, alpha = capi.calibrate(m, p0, r0.engine)
+    assert all(t > 0 for t in t_ex) and alpha and alpha > 0
+    p1 = capi.Plan.partition(capi.Desc(m, t_ex_ns=t_ex), budget,
+                             capi.options(alpha_as_per_byte=alpha, beta_ns_per_tensor=0))
+    region = p1.info()["arena_bytes"] // 256 * 256
+    bl = p1.blocks()
+    assert all(b["bytes"] <= region for b in bl)
+    assert all(bl[k - 1]["bytes"] + bl[k]["bytes"] <= region for k in range(1, len(bl)))
+    base = Runner(m, w, capi.Plan.resident(d), host).run(x)[0].tobytes()
+    assert r0.run(x)[0].tobytes() == base
+    assert Runner(m, w, p1, host).run(x)[0].tobytes() == base

@@ -156,7 +156,7 @@ def test_units_split_vgg_fc1():
     wb = P.weight_bytes(m)
     budget = wb // 4 // 256 * 256
     arena, slot, _ = P.arena_and_slot(m, budget, 2, False)
-    us = P.units(m, slot)
+    us = P.units(m, slot, None, arena // 256 * 256)
     fc1 = [u for u in us if u["layer"] == 18]
     assert len(fc1) > 1
     assert sum(u["rows"] for u in fc1) == 4096
@@ -181,11 +181,13 @@ def test_exhaustive_respects_rules():
         budget = int(r.integers(s // nl * 2, s * 2 + 1))
         res = P.exhaustive_partition(m, budget, coef)
         if res is None:
-            assert P.units(m, budget // 2 // 256 * 256) is None or \
-                max(u["bytes"] for u in P.units(m, budget // 2 // 256 * 256)) > budget // 2
+            us = P.units(m, budget // 2 // 256 * 256, None, budget // 256 * 256)
+            assert us is None or max(u["bytes"] for u in us) > budget // 2
             continue
-        # two blocks co-resident within the budget: n >= ceil(2 s / b)
-        assert res["n"] >= P.block_count_rule(s, budget)
+        # two co-resident blocks within the budget: summing s_i + s_{i+1} <= b
+        # over the n-1 neighbour pairs gives 2s - s_1 - s_n <= (n-1) b, so
+        # n >= ceil(2 s / b) - 1 (the paper's rule, less the two end blocks)
+        assert res["n"] >= P.block_count_rule(s, budget) - 1
         # the optimum is no worse than every feasible alternative
         for cuts in itertools.combinations(range(1, nl), res["n"] - 1):
             v = P.evaluate_cuts(m, budget, coef, list(cuts))
@@ -199,9 +201,12 @@ def test_rule_count_is_fewest_feasible_blocks():
     coef = P.Coef(alpha_as=1000, beta_ns=100, gamma_as=100_000, eta_ns=0)
     m = _uniform_model(6, 512)
     s = P.weight_bytes(m)
-    for per_block in (1, 2, 3, 6):
+    # the rule is for models larger than the budget (s > b); when the model
+    # fits, one block suffices
+    for per_block in (1, 2):
         budget = 2 * per_block * (s // 6)
         fewest = min(len(c) + 1 for k in range(6) for c in itertools.combinations(range(1, 6), k)
                      if P.evaluate_cuts(m, budget, coef, list(c)) is not None)
         assert fewest == P.block_count_rule(s, budget) == 6 // per_block
         assert P.exhaustive_partition(m, budget, coef)["n"] >= fewest
+    assert P.evaluate_cuts(m, s, coef, []) is not None   # one block fits when s <= b
