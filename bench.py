@@ -274,7 +274,6 @@ def main():
     launches = eng.stats()["kernel_launches"] - launches0
     if dist:
         dist.barrier()
-    clk = clocks.stop()
     eng.sync()
     ms_swapped = sum(ms_list) / len(ms_list)
     total_ms = sum(ms_list)
@@ -310,6 +309,7 @@ def main():
         b.synchronize()
         e2e_ms.append(a.elapsed_time(b))
     e2e_val = 1000.0 / (sum(e2e_ms) / len(e2e_ms))
+    clk = clocks.stop()
 
     # ---- profiled pass: per-unit kernel and per-block swap times
     units = plan.units()

@@ -303,6 +303,12 @@ int swapnet_engine_set_profiling(swapnet_engine* eng, int enable);
 int swapnet_engine_measure_units(swapnet_engine* eng, int32_t reps, float* unit_us, uint32_t n_units);
 int swapnet_engine_last_times(swapnet_engine* eng, float* unit_us, uint32_t n_units, float* swap_us,
                               uint32_t n_blocks);
+/* Start and end of every unit kernel and block swap-in of the most recent
+ * profiled inference, in microseconds after the first of those events
+ * (arrays of n_units and n_blocks entries; swap entries are 0 for a
+ * resident plan).  Synchronises. */
+int swapnet_engine_last_timeline(swapnet_engine* eng, float* unit_start, float* unit_end, uint32_t n_units,
+                                 float* swap_start, float* swap_end, uint32_t n_blocks);
 
 void swapnet_engine_free(swapnet_engine* eng);
 

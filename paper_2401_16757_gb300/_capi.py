@@ -80,7 +80,8 @@ EXPORTS = ["swapnet_default_options", "swapnet_partition", "swapnet_plan_from_cu
            "swapnet_plan_output_offsets", "swapnet_plan_free", "swapnet_schedule", "swapnet_load",
            "swapnet_infer", "swapnet_infer_host", "swapnet_engine_sync", "swapnet_engine_blocks",
            "swapnet_engine_free", "swapnet_engine_stats_get", "swapnet_engine_unit_kernels",
-           "swapnet_engine_set_profiling", "swapnet_engine_last_times", "swapnet_engine_measure_units", "swapnet_strerror", "swapnet_last_error", "swapnet_debug_fail_next", "swapnet_gemm_noalloc"]
+           "swapnet_engine_set_profiling", "swapnet_engine_last_times", "swapnet_engine_measure_units",
+           "swapnet_engine_last_timeline", "swapnet_strerror", "swapnet_last_error", "swapnet_debug_fail_next", "swapnet_gemm_noalloc"]
 
 _lib = None
 
@@ -126,6 +127,8 @@ def lib():
         "swapnet_engine_unit_kernels": (C.c_int, [P, C.POINTER(C.c_int32), C.c_uint32, C.POINTER(C.c_uint32)]),
         "swapnet_engine_set_profiling": (C.c_int, [P, C.c_int]),
         "swapnet_engine_measure_units": (C.c_int, [P, C.c_int32, C.POINTER(C.c_float), C.c_uint32]),
+        "swapnet_engine_last_timeline": (C.c_int, [P, C.POINTER(C.c_float), C.POINTER(C.c_float), C.c_uint32,
+                                                   C.POINTER(C.c_float), C.POINTER(C.c_float), C.c_uint32]),
         "swapnet_engine_last_times": (C.c_int, [P, C.POINTER(C.c_float), C.c_uint32, C.POINTER(C.c_float),
                                                 C.c_uint32]),
         "swapnet_strerror": (C.c_char_p, [C.c_int]),
@@ -303,17 +306,25 @@ class HostWeights:
     layout of the arena slots, so a block's tensors are one contiguous
     range)."""
 
-    def __init__(self, weights):
+    def __init__(self, weights, buffer=None):
+        """buffer: optional caller-provided uint8 array (e.g. already pinned)
+        of at least the packed size; default: pageable memory the library
+        page-locks in place."""
         flat = [np.ascontiguousarray(t) for lw in weights for t in lw]
         offs, cur = [], 0
         for t in flat:
             offs.append(cur)
             cur += (t.nbytes + 255) // 256 * 256
-        page = os.sysconf("SC_PAGE_SIZE")
-        raw = np.empty(cur + 2 * page, dtype=np.uint8)
-        start = (-raw.ctypes.data) % page
-        self.buf = raw[start:start + cur]
-        self._raw = raw
+        if buffer is not None:
+            assert buffer.nbytes >= cur and buffer.ctypes.data % 256 == 0
+            self.buf = buffer[:cur]
+            self._raw = buffer
+        else:
+            page = os.sysconf("SC_PAGE_SIZE")
+            raw = np.empty(cur + 2 * page, dtype=np.uint8)
+            start = (-raw.ctypes.data) % page
+            self.buf = raw[start:start + cur]
+            self._raw = raw
         for t, o in zip(flat, offs):
             self.buf[o:o + t.nbytes] = t.view(np.uint8).reshape(-1)
         base = self.buf.ctypes.data
@@ -367,6 +378,14 @@ class Engine:
         u = (C.c_float * max(1, n_units))()
         check(lib().swapnet_engine_measure_units(self.h, reps, u, n_units), "swapnet_engine_measure_units")
         return list(u[:n_units])
+
+    def last_timeline(self, n_units, n_blocks):
+        """(unit start, unit end, swap start, swap end) lists in microseconds."""
+        a, b = (C.c_float * max(1, n_units))(), (C.c_float * max(1, n_units))()
+        c, d = (C.c_float * max(1, n_blocks))(), (C.c_float * max(1, n_blocks))()
+        check(lib().swapnet_engine_last_timeline(self.h, a, b, n_units, c, d, n_blocks),
+              "swapnet_engine_last_timeline")
+        return list(a[:n_units]), list(b[:n_units]), list(c[:n_blocks]), list(d[:n_blocks])
 
     def last_times(self, n_units, n_blocks):
         u = (C.c_float * max(1, n_units))()

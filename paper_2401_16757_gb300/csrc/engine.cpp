@@ -164,6 +164,20 @@ static int register_host(swapnet_engine* e, const void* const* hw, uint32_t nt) 
   for (const R& r : merged) {
     HostRange hr{r.lo, (size_t)(r.hi - r.lo), false, nullptr};
     void* base = reinterpret_cast<void*>(r.lo);
+    {  // memory CUDA already page-locked (cudaHostAlloc / cudaMallocHost) is used as is
+      uintptr_t probe = r.hi - 1;
+      for (uint32_t t = 0; t < nt; ++t) {
+        const uintptr_t p = reinterpret_cast<uintptr_t>(hw[t]);
+        if (m.tensor_raw[t] && p >= r.lo && p < r.hi) { probe = p; break; }
+      }
+      cudaPointerAttributes pa;
+      if (cudaPointerGetAttributes(&pa, reinterpret_cast<void*>(probe)) == cudaSuccess &&
+          pa.type == cudaMemoryTypeHost && g_reg.find({hr.base, hr.len}) == g_reg.end()) {
+        e->ranges.push_back(hr);
+        continue;
+      }
+      cudaGetLastError();
+    }
     std::lock_guard<std::mutex> lk(g_reg_mu);
     auto it = g_reg.find({hr.base, hr.len});
     if (it != g_reg.end()) {
@@ -800,6 +814,42 @@ int swapnet_engine_last_times(swapnet_engine* e, float* unit_us, uint32_t nu, fl
     float ms = 0.f;
     if (!e->plan.resident) CU(cudaEventElapsedTime(&ms, e->ev_swap[2 * k], e->ev_swap[2 * k + 1]), "elapsed");
     swap_us[k] = ms * 1000.f;
+  }
+  return SWAPNET_OK;
+}
+
+int swapnet_engine_last_timeline(swapnet_engine* e, float* us0, float* us1, uint32_t nu, float* ss0, float* ss1,
+                                 uint32_t nb) {
+  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+  if (e->ev_unit.empty()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "profiling was never enabled");
+  CU(cudaSetDevice(e->device), "cudaSetDevice");
+  CU(cudaDeviceSynchronize(), "device synchronize");
+  const bool sw = !e->plan.resident && !e->ev_swap.empty();
+  cudaEvent_t origin = sw ? e->ev_swap[0] : e->ev_unit[0];
+  float first = 0.f;
+  if (sw) {  // the first kernel may start before the first swap event on another stream
+    float d = 0.f;
+    CU(cudaEventElapsedTime(&d, e->ev_swap[0], e->ev_unit[0]), "elapsed");
+    first = std::min(0.f, d);
+  }
+  auto rel = [&](cudaEvent_t ev, float* out) -> int {
+    float ms = 0.f;
+    CU(cudaEventElapsedTime(&ms, origin, ev), "elapsed");
+    *out = (ms - first) * 1000.f;
+    return SWAPNET_OK;
+  };
+  for (uint32_t u = 0; u < nu && u < e->plan.units.size(); ++u) {
+    if (us0 && rel(e->ev_unit[2 * u], &us0[u])) return SWAPNET_ERR_CUDA;
+    if (us1 && rel(e->ev_unit[2 * u + 1], &us1[u])) return SWAPNET_ERR_CUDA;
+  }
+  for (uint32_t k = 0; k < nb && k < e->plan.blocks.size(); ++k) {
+    if (!sw) {
+      if (ss0) ss0[k] = 0.f;
+      if (ss1) ss1[k] = 0.f;
+      continue;
+    }
+    if (ss0 && rel(e->ev_swap[2 * k], &ss0[k])) return SWAPNET_ERR_CUDA;
+    if (ss1 && rel(e->ev_swap[2 * k + 1], &ss1[k])) return SWAPNET_ERR_CUDA;
   }
   return SWAPNET_OK;
 }

@@ -196,3 +196,78 @@ def test_calibrated_plan_is_exact_and_feasible():
     base = Runner(m, w, capi.Plan.resident(d), host).run(x)[0].tobytes()
     assert r0.run(x)[0].tobytes() == base
     assert Runner(m, w, p1, host).run(x)[0].tobytes() == base
+
+
+def test_vgg16_b1_config():
+    """VGG-16, batch 1, budget 25 % of the weight bytes: FC1 (205 MB) is cut
+    into output-feature pieces; swapped equals resident bit for bit."""
+    m = synth.arch.vgg16(batch=1)
+    w = synth.gen.model_weights(m)
+    x = synth.gen.model_input(m)
+    d = capi.Desc(m)
+    budget = int(OP.weight_bytes(m) * 0.25) // 256 * 256
+    host = capi.HostWeights(w)
+    sw = Runner(m, w, capi.Plan.partition(d, budget, capi.options()), host)
+    assert sum(1 for u in sw.plan.units() if u["layer"] == 18) > 1   # FC1 split
+    got = sw.run(x)
+    assert got[0].tobytes() == Runner(m, w, capi.Plan.resident(d), host).run(x)[0].tobytes()
+    check_close(m, sw.decode(got), oracle_outputs(m, w, x))
+
+
+def test_vgg16_b16_sampled_images():
+    """VGG-16 at batch 16 (the bench launch configuration): images 0 and 15 of
+    the GPU batch against the oracle run on those two images alone (the
+    network treats images independently)."""
+    m = synth.arch.vgg16(batch=16)
+    w = synth.gen.model_weights(m)
+    x = synth.gen.model_input(m)
+    d = capi.Desc(m)
+    budget = int(OP.weight_bytes(m) * 0.25) // 256 * 256
+    host = capi.HostWeights(w)
+    sw = Runner(m, w, capi.Plan.partition(d, budget, capi.options()), host)
+    got = sw.run(x)[0]
+    rs = Runner(m, w, capi.Plan.resident(d), host).run(x)[0]
+    assert got.tobytes() == rs.tobytes()
+    m2 = synth.arch.vgg16(batch=2)
+    ref = oracle_outputs(m2, w, np.ascontiguousarray(x[[0, 15]]))[0]
+    check_close(m2, [sw.decode([got[[0, 15]]])[0]], [ref])
+
+
+def test_yolov3_config():
+    """Darknet-53 + three YOLOv3 heads at 416x416: routes, upsample, concat,
+    LeakyReLU and post-activation shortcuts; three output tensors."""
+    m = synth.arch.yolov3()
+    sw = _check_model(m, budget_frac=0.3)
+    assert len(sw.offs) == 3
+
+
+def test_multi_dnn_schedule_concurrent():
+    """Eq. 1 split of one arena (30 % of the summed weight bytes) over
+    ResNet-50, VGG-16 and YOLOv3; the three engines run concurrently on their
+    own streams and each output equals its resident run bit for bit."""
+    import torch
+    ms = [synth.arch.resnet50(), synth.arch.vgg16(), synth.arch.yolov3()]
+    total = sum(OP.weight_bytes(m) for m in ms)
+    M = int(total * 0.3) // 256 * 256
+    descs = [capi.Desc(m) for m in ms]
+    budgets, plans = capi.schedule(descs, [1.0, 1.0, 1.0], M, capi.options())
+    assert sum(budgets) <= M
+    runners, xs, refs = [], [], []
+    for m, d, p in zip(ms, descs, plans):
+        w = synth.gen.model_weights(m)
+        host = capi.HostWeights(w)
+        runners.append(Runner(m, w, p, host))
+        xs.append(synth.gen.model_input(m))
+        refs.append(Runner(m, w, capi.Plan.resident(d), host).run(xs[-1]))
+    streams = [torch.cuda.Stream() for _ in ms]
+    for r, x in zip(runners, xs):
+        r.d_in[:x.nbytes].copy_(torch.from_numpy(np.ascontiguousarray(x).view(np.uint8).reshape(-1)))
+    torch.cuda.synchronize()
+    for _ in range(3):
+        for r, s in zip(runners, streams):
+            r.engine.infer(r.d_in.data_ptr(), r.d_out.data_ptr(), s.cuda_stream)
+    torch.cuda.synchronize()
+    for r, ref in zip(runners, refs):
+        r.engine.sync()
+        got = r.outputs_raw()
+        assert all(a.tobytes() == b.tobytes() for a, b in zip(got, ref))
