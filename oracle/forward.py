@@ -13,8 +13,17 @@ from the textbook definition of each layer:
   gap      mean over H and W
   upsample nearest neighbour, factor 2
   concat   channels of src[0] followed by channels of src[1]
-  act      relu(x) = max(x, 0); leaky(x) = x if x > 0 else 0.1 x
+  act      relu(x) = max(x, 0); leaky(x) = x if x > 0 else 0.1 x;
+           swiglu: silu(r) * (acc + b) with silu(z) = z / (1 + e^-z), r the
+           gate layer's output
   residual res_post False: act(acc + b + r); True: act(acc + b) + r
+  embed    rows of the table picked by the token ids
+  rmsnorm  x / sqrt(mean(x^2) + eps) * g
+  attention  RoPE (adjacent pairs, angle = position * theta^(-2i/Dh)) on q
+           and k, both rounded to the storage dtype; k and v appended to the
+           layer's cache at positions pos0..; query t attends to positions
+           0..pos0+t: softmax(q k^T / sqrt(Dh)) v per head
+  argmax   first index of the row maximum (int32 on the GPU)
 
 Precision.  Arithmetic is float64.  The GPU path stores every layer output in
 the model's storage dtype; the oracle rounds each layer output to that dtype
@@ -56,6 +65,45 @@ def round_as(x, dtype):
 
 
 # ----------------------------------------------------------------- layers
+def silu(z):
+    return z / (1.0 + np.exp(-z))
+
+
+def rmsnorm(x2d, g, eps):
+    """x / sqrt(mean(x^2) + eps) * g over the last axis."""
+    return x2d / np.sqrt(np.mean(x2d * x2d, axis=-1, keepdims=True) + eps) * g[None, :]
+
+
+def rope(x2d, positions, heads, theta):
+    """Rotate adjacent pairs (2i, 2i+1) of every head by position * theta^(-2i/Dh)."""
+    t, width = x2d.shape
+    dh = width // heads
+    x = x2d.reshape(t, heads, dh // 2, 2)
+    inv = theta ** (-np.arange(0, dh, 2, dtype=np.float64) / dh)     # [Dh/2]
+    ang = np.asarray(positions, dtype=np.float64)[:, None] * inv[None, :]   # [T, Dh/2]
+    c, s = np.cos(ang)[:, None, :], np.sin(ang)[:, None, :]
+    x0, x1 = x[..., 0], x[..., 1]
+    out = np.stack([x0 * c - x1 * s, x0 * s + x1 * c], axis=-1)
+    return out.reshape(t, width)
+
+
+def causal_attention(q2d, keys, values, pos0, heads):
+    """Query t (position pos0 + t) attends to cache positions 0..pos0+t:
+    softmax(q k^T / sqrt(Dh)) v, per head."""
+    t, width = q2d.shape
+    dh = width // heads
+    out = np.zeros((t, width))
+    for h in range(heads):
+        sl = slice(h * dh, (h + 1) * dh)
+        for i in range(t):
+            n = pos0 + i + 1
+            sc = keys[:n, sl] @ q2d[i, sl] / np.sqrt(dh)
+            p = np.exp(sc - sc.max())
+            p /= p.sum()
+            out[i, sl] = p @ values[:n, sl]
+    return out
+
+
 def act_fn(y, act):
     if act == "none":
         return y
@@ -129,20 +177,48 @@ def nchw_to_nhwc(a):
     return np.ascontiguousarray(np.asarray(a).transpose(0, 2, 3, 1))
 
 
-def run_layer(layer, dtype, tensors, acts, x_in):
+def _as2d(a):
+    return a.reshape(a.shape[0], -1)
+
+
+def run_layer(layer, dtype, tensors, acts, x_in, state=None, li=None):
     """Compute one layer (float64 in, rounded float64 out).
 
     tensors: the layer's storage arrays; acts: dict layer index -> NCHW
-    float64 output; x_in: NCHW float64 model input.
+    float64 output; x_in: NCHW float64 model input (token ids for a token
+    model); state: KV caches and position for attention layers.
     """
     def get(i):
         return x_in if i == -1 else acts[i]
 
     op = layer["op"]
     src = get(layer["src"][0])
+    if op == "embed":
+        table = decode(tensors[0], dtype)
+        ids = np.asarray(src).reshape(-1).astype(np.int64)
+        return table[ids].reshape(len(ids), -1, 1, 1)          # a copy: no rounding needed
+    if op == "rmsnorm":
+        y = rmsnorm(_as2d(src), decode(tensors[0], dtype), layer["eps"])
+        return round_as(y, dtype).reshape(src.shape)
+    if op == "attention":
+        q, k, v = (_as2d(get(i)) for i in layer["src"])
+        t = q.shape[0]
+        pos0 = state["pos"]
+        pos = np.arange(pos0, pos0 + t)
+        qr = round_as(rope(q, pos, layer["heads"], layer["theta"]), dtype)
+        kr = round_as(rope(k, pos, layer["heads"], layer["theta"]), dtype)
+        cache = state["kv"].setdefault(li, (np.zeros((layer["max_seq"], q.shape[1])),
+                                            np.zeros((layer["max_seq"], q.shape[1]))))
+        cache[0][pos0:pos0 + t] = kr
+        cache[1][pos0:pos0 + t] = v
+        y = causal_attention(qr, cache[0], cache[1], pos0, layer["heads"])
+        return round_as(y, dtype).reshape(t, -1, 1, 1)
+    if op == "argmax":
+        a = _as2d(src)
+        return np.argmax(a, axis=1).astype(np.float64).reshape(-1, 1, 1, 1)
     if op in ("conv", "linear"):
         w = decode(tensors[0], dtype)
-        b = decode(tensors[1], dtype)
+        b = decode(tensors[1], dtype) if len(tensors) > 1 else np.zeros(w.shape[0])
         if op == "conv":
             y = conv2d(src, w, b, layer["stride"], layer["pad"])
         else:
@@ -151,7 +227,9 @@ def run_layer(layer, dtype, tensors, acts, x_in):
             assert flat.shape[1] == layer["k"], (flat.shape, layer["k"])
             y = linear(flat, w, b).reshape(n, layer["n"], 1, 1)
         r = None if layer.get("res") is None else get(layer["res"])
-        if r is not None and not layer["res_post"]:
+        if layer.get("act") == "swiglu":
+            y = silu(r) * y
+        elif r is not None and not layer["res_post"]:
             y = act_fn(y + r, layer["act"])
         elif r is not None:
             y = act_fn(y, layer["act"]) + r
@@ -170,19 +248,35 @@ def run_layer(layer, dtype, tensors, acts, x_in):
     return round_as(y, dtype)
 
 
-def forward_range(model, weights, acts, x_in, lo, hi):
+def forward_range(model, weights, acts, x_in, lo, hi, state=None):
     """Run layers [lo, hi) in order, adding their outputs to `acts`."""
     dt = model["dtype"]
     for li in range(lo, hi):
-        acts[li] = run_layer(model["layers"][li], dt, weights[li], acts, x_in)
+        acts[li] = run_layer(model["layers"][li], dt, weights[li], acts, x_in, state, li)
     return acts
 
 
-def forward(model, weights, x_nhwc, check_range=True):
+def new_state():
+    """KV caches and the number of positions already cached."""
+    return {"pos": 0, "kv": {}}
+
+
+def _model_input(model, x_nhwc):
+    if model.get("input_dtype") == "i32":
+        return np.asarray(x_nhwc)
+    return nhwc_to_nchw(decode(x_nhwc, model["dtype"]))
+
+
+def forward(model, weights, x_nhwc, check_range=True, state=None):
     """Plain forward pass; returns the model outputs as NHWC float64 arrays
-    (values exactly representable in the storage dtype)."""
-    x_in = nhwc_to_nchw(decode(x_nhwc, model["dtype"]))
-    acts = forward_range(model, weights, {}, x_in, 0, len(model["layers"]))
+    (values exactly representable in the storage dtype).  Token models keep
+    their KV caches and position in `state`, advanced by the tokens read."""
+    x_in = _model_input(model, x_nhwc)
+    if state is None:
+        state = new_state()
+    acts = forward_range(model, weights, {}, x_in, 0, len(model["layers"]), state)
+    if model.get("input_dtype") == "i32":
+        state["pos"] += int(np.asarray(x_nhwc).shape[0])
     outs = [nchw_to_nhwc(acts[i]) for i in model["outputs"]]
     if check_range:
         for o in outs:
@@ -190,8 +284,8 @@ def forward(model, weights, x_nhwc, check_range=True):
     return outs
 
 
-def forward_all(model, weights, x_nhwc):
+def forward_all(model, weights, x_nhwc, state=None):
     """Every layer output, NHWC float64 (for per-layer parity checks)."""
-    x_in = nhwc_to_nchw(decode(x_nhwc, model["dtype"]))
-    acts = forward_range(model, weights, {}, x_in, 0, len(model["layers"]))
+    x_in = _model_input(model, x_nhwc)
+    acts = forward_range(model, weights, {}, x_in, 0, len(model["layers"]), state or new_state())
     return {i: nchw_to_nhwc(a) for i, a in acts.items()}

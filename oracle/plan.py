@@ -76,9 +76,20 @@ def out_shapes(model):
             shapes.append((n, 2 * h, 2 * w, c))
         elif op == "concat":
             shapes.append((n, h, w, c + shp(L["src"][1])[3]))
+        elif op == "embed":
+            shapes.append((n * h * w, 1, 1, L["d"]))
+        elif op in ("rmsnorm", "attention"):
+            shapes.append((n, h, w, c))
+        elif op == "argmax":
+            shapes.append((n, 1, 1, 1))
         else:
             raise ValueError(op)
     return shapes
+
+
+def out_elem_bytes(model, li):
+    """Element size of a layer output (argmax writes int32 indices)."""
+    return 4 if model["layers"][li]["op"] == "argmax" else ES[model["dtype"]]
 
 
 def layer_tensor_bytes(model, li):
@@ -86,8 +97,19 @@ def layer_tensor_bytes(model, li):
     if L["op"] == "conv":
         return [L["cout"] * L["kh"] * L["kw"] * L["cin"] * es, L["cout"] * es]
     if L["op"] == "linear":
-        return [L["n"] * L["k"] * es, L["n"] * es]
+        w = [L["n"] * L["k"] * es]
+        return w if L.get("bias") is False else w + [L["n"] * es]
+    if L["op"] == "embed":
+        return [L["vocab"] * L["d"] * es]
+    if L["op"] == "rmsnorm":
+        return [L["d"] * es]
     return []
+
+
+def host_resident(model, li):
+    """The embedding table stays in host memory: its rows are gathered
+    (zero-copy) by the lookup, never swapped into the arena."""
+    return model["layers"][li]["op"] == "embed"
 
 
 def layer_flops(model, li, shapes):
@@ -97,6 +119,8 @@ def layer_flops(model, li, shapes):
         return 2 * n * ho * wo * co * L["cin"] * L["kh"] * L["kw"]
     if L["op"] == "linear":
         return 2 * n * L["k"] * L["n"]
+    if L["op"] == "attention":
+        return 4 * n * L["max_seq"] * co
     return 0
 
 
@@ -122,13 +146,13 @@ def workspace(model):
         for i in refs:
             if i >= 0:
                 last[i] = max(last[i], j)
-    outs = list(model["outputs"])
+    outs = sorted(model["outputs"])
     placed = []  # (lo, hi, off, size)
     offs = {}
     for i in range(nl):
         if i in outs:
             continue
-        size = align(math.prod(shapes[i]) * es)
+        size = align(math.prod(shapes[i]) * out_elem_bytes(model, i))
         conflict = [p for p in placed if p[0] <= last[i] and i <= p[1]]
         cands = sorted({0} | {p[2] + p[3] for p in conflict})
         for o in cands:
@@ -140,7 +164,7 @@ def workspace(model):
     out_off, cur = {}, 0
     for i in outs:
         out_off[i] = cur
-        cur += align(math.prod(shapes[i]) * es)
+        cur += align(math.prod(shapes[i]) * out_elem_bytes(model, i))
     return ws, offs, cur, out_off
 
 
@@ -167,7 +191,7 @@ def units(model, slot, t_ex_override=None, region=None):
     out = []
     for li, L in enumerate(model["layers"]):
         tb = layer_tensor_bytes(model, li)
-        size = sum(align(b) for b in tb)
+        size = 0 if host_resident(model, li) else sum(align(b) for b in tb)
         f = layer_flops(model, li, shapes)
         ovr = 0 if t_ex_override is None else t_ex_override[li]
         if size <= slot or (L["op"] != "linear" and size <= region):
@@ -179,7 +203,7 @@ def units(model, slot, t_ex_override=None, region=None):
         K, N = L["k"], L["n"]
 
         def piece_bytes(r):
-            return align(r * K * es) + align(r * es)
+            return align(r * K * es) + (0 if L.get("bias") is False else align(r * es))
 
         rmax = 0
         r = 128
@@ -193,7 +217,7 @@ def units(model, slot, t_ex_override=None, region=None):
         row0 = 0
         while row0 < N:
             rows = min(rr, N - row0)
-            out.append(dict(layer=li, row0=row0, rows=rows, bytes=piece_bytes(rows), depth=2,
+            out.append(dict(layer=li, row0=row0, rows=rows, bytes=piece_bytes(rows), depth=len(tb),
                             flops=2 * shapes[li][0] * K * rows,
                             t_ex_ovr=(ceil_div(ovr * rows, N) if ovr else 0)))
             row0 += rows

@@ -11,6 +11,7 @@ A model is a dict:
 
 Layer dict keys (all integers unless noted):
   op        'linear' | 'conv' | 'maxpool' | 'gap' | 'upsample2x' | 'concat'
+            | 'embed' | 'rmsnorm' | 'attention' | 'argmax'
   src       list of producer layer indices; -1 is the model input
   linear:   k (input features = H*W*C of the input, flattened in (h, w, c)
             order), n (output features), act, res, res_post
@@ -20,7 +21,12 @@ Layer dict keys (all integers unless noted):
   gap:      global average over H and W
   upsample2x: nearest-neighbour x2 in H and W
   concat:   channel concatenation of src[0] then src[1]
-  act       'none' | 'relu' | 'leaky' (slope 0.1)
+  embed:    vocab, d (rows of the table picked by int32 token ids)
+  rmsnorm:  d, eps: x / sqrt(mean(x^2) + eps) * g
+  attention: src = [q, k, v]; heads, max_seq, theta (RoPE base)
+  argmax:   index of the largest value of each row (ties: lowest index)
+  act       'none' | 'relu' | 'leaky' (slope 0.1) | 'swiglu' (silu(res) * y)
+  bias      False: the linear layer has no bias tensor
   res       index of a layer whose output is added element-wise, or None
   res_post  False: out = act(acc + bias + res)   (ResNet bottleneck)
             True:  out = act(acc + bias) + res   (Darknet shortcut)
@@ -147,14 +153,61 @@ def yolov3(batch=1, res=416, classes=80):
                 layers=L, outputs=outs)
 
 
+
+
+def llm(layers=32, d=4096, heads=32, ffn=11008, vocab=32000, tokens=512, max_seq=544):
+    """LLaMA-7B-shaped decoder (pre-norm, RMSNorm eps 1e-6 with gains, RoPE
+    theta 10000 on adjacent pairs, causal attention with a KV cache of
+    max_seq positions, SwiGLU FFN, untied LM head, no biases), bf16.
+
+    The input is `tokens` int32 token ids; outputs are the logits of every
+    position and their argmax (ties -> lowest index).  Decoder layer i:
+      rmsnorm -> q, k, v -> attention -> o (+x) -> rmsnorm -> gate, up
+      (silu(gate) * up) -> down (+h)
+    """
+    L = [dict(op="embed", src=[-1], vocab=vocab, d=d)]
+    x = 0
+    for _ in range(layers):
+        L.append(dict(op="rmsnorm", src=[x], d=d, eps=1e-6))
+        xn = len(L) - 1
+        q = len(L); L.append(_linear(xn, d, d))
+        k = len(L); L.append(_linear(xn, d, d))
+        v = len(L); L.append(_linear(xn, d, d))
+        L.append(dict(op="attention", src=[q, k, v], heads=heads, max_seq=max_seq, theta=10000.0))
+        a = len(L) - 1
+        L.append(_linear(a, d, d, res=x))
+        h = len(L) - 1
+        L.append(dict(op="rmsnorm", src=[h], d=d, eps=1e-6))
+        hn = len(L) - 1
+        g = len(L); L.append(_linear(hn, d, ffn))
+        L.append(dict(_linear(hn, d, ffn), act="swiglu", res=g))
+        u = len(L) - 1
+        L.append(_linear(u, ffn, d, res=h))
+        x = len(L) - 1
+    L.append(dict(op="rmsnorm", src=[x], d=d, eps=1e-6))
+    L.append(_linear(len(L) - 1, d, vocab))
+    head = len(L) - 1
+    L.append(dict(op="argmax", src=[head]))
+    for l in L:
+        if l["op"] == "linear":
+            l["bias"] = False
+    return dict(name="llm", model_id=5, dtype="bf16", input=(tokens, 1, 1, 1), input_dtype="i32",
+                layers=L, outputs=[head, len(L) - 1])
+
+
 def tensor_shapes(layer):
     """Names and shapes of a layer's parameter tensors, in storage order."""
     if layer["op"] == "conv":
         return [("w", (layer["cout"], layer["kh"], layer["kw"], layer["cin"])),
                 ("b", (layer["cout"],))]
     if layer["op"] == "linear":
-        return [("w", (layer["n"], layer["k"])), ("b", (layer["n"],))]
+        t = [("w", (layer["n"], layer["k"]))]
+        return t if layer.get("bias") is False else t + [("b", (layer["n"],))]
+    if layer["op"] == "embed":
+        return [("table", (layer["vocab"], layer["d"]))]
+    if layer["op"] == "rmsnorm":
+        return [("g", (layer["d"],))]
     return []
 
 
-MODELS = {"mlp6": mlp6, "resnet50": resnet50, "vgg16": vgg16, "yolov3": yolov3}
+MODELS = {"mlp6": mlp6, "resnet50": resnet50, "vgg16": vgg16, "yolov3": yolov3, "llm": llm}

@@ -21,7 +21,9 @@ Initialisation per workload:
   vgg16     W ~ N(0, 2/fan_in) (He) for ReLU layers, N(0, 1/fan_in) for the
             last FC, b = 0
   yolov3    W ~ N(0, 1/fan_in), b ~ N(0, 0.01)
-  inputs    N(0, 1)
+  llm       every matrix and the embedding N(0, 0.02) (drawn in float32,
+            rounded to bf16), RMSNorm gains 1, no biases
+  inputs    N(0, 1); token ids U[0, vocab) with seed 2
 """
 import numpy as np
 
@@ -57,9 +59,36 @@ def _fan_in(layer):
     return layer["k"]
 
 
+def _bf16_from_f32(f):
+    """float32 -> bf16 bit patterns, round-to-nearest-even."""
+    u = f.view(np.uint32)
+    lsb = (u >> np.uint32(16)) & np.uint32(1)
+    return ((u + np.uint32(0x7FFF) + lsb) >> np.uint32(16)).astype(np.uint16)
+
+
+def llm_tensor(model, li, ti, shape, seed=0):
+    """LLM parameters: N(0, 0.02) drawn in float32 (the 7B tables are large),
+    rounded once to bf16; RMSNorm gains are 1."""
+    layer = model["layers"][li]
+    if layer["op"] == "rmsnorm":
+        return np.full(shape, 0x3F80, dtype=np.uint16)   # 1.0
+    r = _rng(seed, model["model_id"], li, ti)
+    f = r.standard_normal(int(np.prod(shape)), dtype=np.float32)
+    f *= np.float32(0.02)
+    return _bf16_from_f32(f).reshape(shape)
+
+
 def layer_weights(model, li, seed=0):
     """Parameter tensors of layer li as storage arrays ([] for weightless ops)."""
     layer = model["layers"][li]
+    if model["name"] == "llm":
+        from .arch import tensor_shapes
+        return [llm_tensor(model, li, ti, shp, seed) for ti, (_, shp) in enumerate(tensor_shapes(layer))]
+    if layer["op"] == "rmsnorm":   # gains of a non-LLM test model: U(0.5, 1.5)
+        return [round_to_storage(_rng(seed, model["model_id"], li, 0).uniform(0.5, 1.5, layer["d"]), model["dtype"])]
+    if layer["op"] == "embed":
+        return [round_to_storage(_rng(seed, model["model_id"], li, 0).normal(0.0, 1.0, (layer["vocab"], layer["d"])),
+                                 model["dtype"])]
     if layer["op"] not in ("conv", "linear"):
         return []
     dt, mid, name = model["dtype"], model["model_id"], model["name"]
@@ -71,6 +100,8 @@ def layer_weights(model, li, seed=0):
         wshape = (layer["n"], layer["k"])
         nout = layer["n"]
     rw, rb = _rng(seed, mid, li, 0), _rng(seed, mid, li, 1)
+    if layer.get("bias") is False:
+        return [round_to_storage(rw.normal(0.0, np.sqrt(1.0 / fan), wshape), dt)]
     if name == "mlp6":
         w = rw.normal(0.0, np.sqrt(1.0 / fan), wshape)
         b = np.zeros(nout)
@@ -108,7 +139,12 @@ def model_weights(model, seed=0):
 
 
 def model_input(model, seed=1, request=0):
-    """Model input, NHWC storage array, N(0, 1)."""
+    """Model input, NHWC storage array, N(0, 1); for token models, int32 ids
+    U[0, vocab) with seed 2."""
+    if model.get("input_dtype") == "i32":
+        vocab = model["layers"][0]["vocab"]
+        r = _rng(2 + 1000 * request, model["model_id"], 0xFFFF, 0)
+        return r.integers(0, vocab, size=model["input"], dtype=np.int32)
     r = _rng(seed + 1000 * request, model["model_id"], 0xFFFF, 0)
     return round_to_storage(r.normal(0.0, 1.0, model["input"]), model["dtype"])
 

@@ -191,3 +191,90 @@ def test_workload_activations_stay_in_fp16_range(name):
     for a in acts.values():
         assert np.all(np.isfinite(a)) and np.max(np.abs(a)) < 6e4
         assert np.sqrt(np.mean(a ** 2)) > 1e-2
+
+
+# ----------------------------------------------------------------- decoder ops
+def test_rmsnorm_closed_forms():
+    g = np.array([0.5, 2.0, -1.0, 3.0])
+    y = F.rmsnorm(np.full((1, 4), -7.0), g, 1e-12)          # constant row -> sign * g
+    np.testing.assert_allclose(y[0], -g, rtol=1e-9)
+    r = np.random.default_rng(3).normal(size=(3, 64))
+    np.testing.assert_allclose(F.rmsnorm(5.0 * r, np.ones(64), 0.0), F.rmsnorm(r, np.ones(64), 0.0), rtol=1e-12)
+    y = F.rmsnorm(r, np.ones(64), 0.0)
+    np.testing.assert_allclose(np.mean(y * y, axis=1), 1.0, rtol=1e-12)   # unit mean square
+
+
+def test_rope_identity_norm_composition():
+    r = np.random.default_rng(4).normal(size=(3, 32))          # 2 heads x 16
+    np.testing.assert_allclose(F.rope(r, [0, 0, 0], 2, 10000.0), r, rtol=0, atol=0)
+    y = F.rope(r, [5, 17, 300], 2, 10000.0)
+    pn = lambda a: np.hypot(a.reshape(3, 16, 2)[..., 0], a.reshape(3, 16, 2)[..., 1])
+    np.testing.assert_allclose(pn(y), pn(r), rtol=1e-12)
+    # one pair by hand: dims (2, 3) of head 1 use i = 1 -> angle = p * theta^(-2/16)
+    p, ang = 17, 17 * 10000.0 ** (-2.0 / 16)
+    x0, x1 = r[1, 16 + 2], r[1, 16 + 3]
+    np.testing.assert_allclose(y[1, 16 + 2:16 + 4], [x0 * np.cos(ang) - x1 * np.sin(ang),
+                                                     x0 * np.sin(ang) + x1 * np.cos(ang)], rtol=1e-12)
+    # rotations compose: rope(rope(x, a), b) = rope(x, a + b)
+    np.testing.assert_allclose(F.rope(F.rope(r, [3, 4, 5], 2, 10000.0), [7, 8, 9], 2, 10000.0),
+                               F.rope(r, [10, 12, 14], 2, 10000.0), rtol=1e-10, atol=1e-12)
+
+
+def test_attention_special_cases_and_brute_force():
+    r = np.random.default_rng(5)
+    v = r.normal(size=(6, 8))
+    k = r.normal(size=(6, 8))
+    # a single query at position 0 sees only itself: output = v[0]
+    np.testing.assert_allclose(F.causal_attention(r.normal(size=(1, 8)), k, v, 0, 2), v[:1], rtol=1e-12)
+    # zero query: uniform weights over the visible positions
+    out = F.causal_attention(np.zeros((2, 8)), k, v, 3, 2)
+    np.testing.assert_allclose(out[0], v[:4].mean(axis=0), rtol=1e-12)
+    np.testing.assert_allclose(out[1], v[:5].mean(axis=0), rtol=1e-12)
+    # brute force: explicit loops over heads, queries and keys
+    q = r.normal(size=(3, 8))
+    got = F.causal_attention(q, k, v, 2, 2)
+    for h in range(2):
+        for i in range(3):
+            n = 2 + i + 1
+            s = [sum(q[i, h * 4 + d] * k[j, h * 4 + d] for d in range(4)) / 2.0 for j in range(n)]
+            e = [np.exp(x - max(s)) for x in s]
+            for d in range(4):
+                ref = sum(e[j] * v[j, h * 4 + d] for j in range(n)) / sum(e)
+                assert abs(got[i, h * 4 + d] - ref) < 1e-12
+
+
+def test_silu_and_argmax():
+    assert F.silu(0.0) == 0.0
+    np.testing.assert_allclose(F.silu(1.0), 1.0 / (1.0 + np.exp(-1.0)), rtol=1e-15)
+    np.testing.assert_allclose(F.silu(40.0), 40.0, rtol=1e-15)
+    assert abs(F.silu(-40.0)) < 1e-15
+    layer = dict(op="argmax", src=[-1])
+    x = np.array([[1.0, 3.0, 3.0, 2.0], [5.0, 5.0, 5.0, 5.0]]).reshape(2, 4, 1, 1)
+    out = F.run_layer(layer, "bf16", [], {}, x)
+    assert out.ravel().tolist() == [1.0, 0.0]      # ties -> lowest index
+
+
+def _tiny_llm(tokens):
+    return synth.arch.llm(layers=2, d=64, heads=2, ffn=160, vocab=300, tokens=tokens, max_seq=24)
+
+
+def test_embedding_gathers_rows():
+    m = _tiny_llm(5)
+    w = synth.gen.model_weights(m)
+    ids = np.array([3, 299, 0, 3, 17], dtype=np.int32).reshape(5, 1, 1, 1)
+    out = F.run_layer(m["layers"][0], "bf16", w[0], {}, ids)
+    np.testing.assert_array_equal(out.reshape(5, -1), F.decode(w[0][0], "bf16")[[3, 299, 0, 3, 17]])
+
+
+def test_kv_cache_prefill_then_decode_equals_longer_prefill():
+    # logits of token T from prefill(T) + one decode step equal the last row
+    # of prefill(T + 1): the cache carries exactly the keys and values
+    w = synth.gen.model_weights(_tiny_llm(9))
+    ids = synth.gen.model_input(_tiny_llm(9))
+    st = F.new_state()
+    F.forward(_tiny_llm(8), w, ids[:8], state=st)
+    step = F.forward(_tiny_llm(1), w, ids[8:9], state=st)[0]
+    assert st["pos"] == 9
+    full = F.forward(_tiny_llm(9), w, ids)[0]
+    got, ref = step.ravel(), full[8].ravel()
+    assert np.linalg.norm(got - ref) <= 1e-3 * np.linalg.norm(ref)
