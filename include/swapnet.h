@@ -46,7 +46,12 @@ typedef enum swapnet_status {
 } swapnet_status;
 
 /* ------------------------------------------------------------ descriptors */
-typedef enum swapnet_dtype { SWAPNET_F32 = 0, SWAPNET_F16 = 1, SWAPNET_BF16 = 2 } swapnet_dtype;
+typedef enum swapnet_dtype {
+  SWAPNET_F32 = 0,
+  SWAPNET_F16 = 1,
+  SWAPNET_BF16 = 2,
+  SWAPNET_I32 = 3 /* model input only: token ids */
+} swapnet_dtype;
 
 typedef enum swapnet_op {
   SWAPNET_OP_LINEAR = 1,     /* y[m,o] = act(sum_i x[m,i] W[o,i] + b[o] (+res)) */
@@ -54,10 +59,27 @@ typedef enum swapnet_op {
   SWAPNET_OP_MAXPOOL = 3,    /* window max; padding never wins                  */
   SWAPNET_OP_GAP = 4,        /* global average over H and W                     */
   SWAPNET_OP_UPSAMPLE2X = 5, /* nearest neighbour, factor 2 in H and W          */
-  SWAPNET_OP_CONCAT = 6      /* channels of src0 followed by channels of src1   */
+  SWAPNET_OP_CONCAT = 6,     /* channels of src0 followed by channels of src1   */
+  SWAPNET_OP_EMBED = 7,      /* rows of a [cin = vocab][cout = d] table picked by the
+                                int32 token ids of the model input; the table
+                                stays in host memory and its rows are read there
+                                (never swapped)                                  */
+  SWAPNET_OP_RMSNORM = 8,    /* x / sqrt(mean(x^2) + eps) * g over cout = d      */
+  SWAPNET_OP_ATTENTION = 9,  /* RoPE on q = src0 and k = src1, both stored rounded;
+                                k and v = src2 appended to this layer's cache at
+                                the state position; query t attends causally to
+                                positions 0..pos+t: softmax(q k^T / sqrt(Dh)) v  */
+  SWAPNET_OP_ARGMAX = 10     /* int32 index of each row's maximum (ties: lowest) */
 } swapnet_op;
 
-typedef enum swapnet_act { SWAPNET_ACT_NONE = 0, SWAPNET_ACT_RELU = 1, SWAPNET_ACT_LEAKY = 2 } swapnet_act;
+typedef enum swapnet_act {
+  SWAPNET_ACT_NONE = 0,
+  SWAPNET_ACT_RELU = 1,
+  SWAPNET_ACT_LEAKY = 2,  /* slope 0.1 */
+  SWAPNET_ACT_SWIGLU = 3  /* silu(res) * (acc + b), res = the gate layer */
+} swapnet_act;
+
+#define SWAPNET_LAYER_NO_BIAS 1 /* flags: a linear layer without bias tensor */
 
 #define SWAPNET_SRC_INPUT (-1) /* the model input                       */
 #define SWAPNET_SRC_NONE (-2)  /* unused producer / no residual operand */
@@ -76,19 +98,30 @@ typedef struct swapnet_layer {
   int32_t cout;     /* conv: output channels; linear: output features           */
   int32_t kh, kw, stride, pad; /* conv and maxpool window                      */
   int32_t is_output;/* nonzero: a model output, written to the output buffer   */
-  int32_t reserved;
+  int32_t flags;    /* SWAPNET_LAYER_NO_BIAS                                   */
   int64_t t_ex_ns;  /* measured execution delay; 0 = gamma * FLOPs (Sec. 6.1)  */
+  int32_t src2;     /* ATTENTION: the values layer                             */
+  int32_t heads;    /* ATTENTION: heads (head width = cout / heads)            */
+  int32_t max_seq;  /* ATTENTION: positions the KV cache holds                 */
+  float eps;        /* RMSNORM epsilon                                         */
+  float theta;      /* ATTENTION: RoPE base (angle = pos * theta^(-2i/Dh))     */
+  int32_t reserved;
 } swapnet_layer;
 
 /* Parameter tensors of a layer, in this order, are what swapnet_load's
- * host_weights lists: CONV2D and LINEAR have two (weights, bias); the other
- * ops none.  Model outputs are written to the output buffer in increasing
- * layer order, each at a 256-byte aligned offset. */
+ * host_weights lists: CONV2D and LINEAR have two (weights, bias; one with
+ * SWAPNET_LAYER_NO_BIAS), EMBED one (the table), RMSNORM one (the gains);
+ * the other ops none.  Model outputs are written to the output buffer in
+ * increasing layer order, each at a 256-byte aligned offset (ARGMAX outputs
+ * are int32, everything else the model dtype).  ATTENTION uses cout = the
+ * width of q, k and v (heads x head width, head width 128). */
 typedef struct swapnet_model_desc {
   int32_t dtype;    /* swapnet_dtype of weights and activations          */
   int32_t n_layers;
   const swapnet_layer* layers;
   int32_t in_n, in_h, in_w, in_c; /* model input, NHWC (a matrix is n x 1 x 1 x c) */
+  int32_t in_dtype; /* dtype of the model input: the model dtype or SWAPNET_I32 (token ids) */
+  int32_t reserved;
 } swapnet_model_desc;
 
 typedef enum swapnet_swap_variant {
@@ -138,6 +171,10 @@ typedef struct swapnet_plan_info {
   uint64_t weight_bytes;   /* sum of 256-aligned parameter tensor sizes      */
   uint64_t plan_bytes;     /* host bytes of the plan (the resident skeleton) */
   int64_t predicted_ns;    /* objective value of the chosen partition        */
+  uint64_t state_bytes;    /* decoder state (position + KV caches), 0 if none */
+  int32_t exact;           /* 1: the search proved the plan optimal; 0: its
+                              frontier was capped and the plan is the best found */
+  int32_t reserved;
 } swapnet_plan_info;
 
 typedef struct swapnet_unit_info {
@@ -251,6 +288,20 @@ int swapnet_infer_host(swapnet_engine* eng, const void* h_input, void* h_output,
  * on a device error. */
 int swapnet_engine_sync(swapnet_engine* eng);
 
+/* Decoder state of a model with ATTENTION layers: a device buffer of
+ * state_bytes (plan info), caller-owned, 256-byte aligned.  Layout: an int32
+ * position (tokens already cached) in the first 256 bytes, then for every
+ * ATTENTION layer in layer order its key cache and value cache
+ * [max_seq][cout] in the model dtype, each 256-byte aligned.  Zero the
+ * buffer to start a new sequence.  Each inference reads the position on the
+ * device, appends its tokens at that position and advances it by the number
+ * of input tokens, so a prefill engine and a decode engine built from the
+ * same layers can share one state buffer, and a decode step replays the same
+ * CUDA graph every time.  A position that would pass max_seq is not written;
+ * swapnet_engine_sync then reports SWAPNET_ERR_INVALID_ARG.
+ * Must be bound before the first swapnet_infer of such a model. */
+int swapnet_engine_bind_state(swapnet_engine* eng, void* d_state, uint64_t state_bytes);
+
 typedef struct swapnet_engine_block {
   int32_t variant;       /* swapnet_swap_variant chosen for the block     */
   int32_t n_segments;    /* contiguous host->arena copies per swap-in     */
@@ -281,7 +332,11 @@ typedef enum swapnet_kernel_kind {
   SWAPNET_KERNEL_GAP = 6,
   SWAPNET_KERNEL_UPSAMPLE = 7,
   SWAPNET_KERNEL_CONCAT = 8,
-  SWAPNET_KERNEL_TILED = 9        /* SIMT tiled linear (general fallback)     */
+  SWAPNET_KERNEL_TILED = 9,       /* SIMT tiled linear (general fallback)     */
+  SWAPNET_KERNEL_EMBED = 10,      /* zero-copy embedding gather               */
+  SWAPNET_KERNEL_RMSNORM = 11,
+  SWAPNET_KERNEL_ATTENTION = 12,  /* two launches: RoPE + cache append, attention */
+  SWAPNET_KERNEL_ARGMAX = 13
 } swapnet_kernel_kind;
 int swapnet_engine_unit_kernels(const swapnet_engine* eng, int32_t* kinds, uint32_t cap, uint32_t* n);
 

@@ -77,7 +77,7 @@ def out_shapes(model):
         elif op == "concat":
             shapes.append((n, h, w, c + shp(L["src"][1])[3]))
         elif op == "embed":
-            shapes.append((n * h * w, 1, 1, L["d"]))
+            shapes.append((n * h * w * c, 1, 1, L["d"]))
         elif op in ("rmsnorm", "attention"):
             shapes.append((n, h, w, c))
         elif op == "argmax":

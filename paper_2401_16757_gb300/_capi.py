@@ -16,9 +16,12 @@ LIB_PATH = os.path.join(_PKG, "libswapnet.so")
 OK, ERR_INVALID_ARG, ERR_INFEASIBLE, ERR_OOM, ERR_CUDA, ERR_TIMEOUT, ERR_MISALIGNED, ERR_UNSUPPORTED = \
     0, -1, -2, -3, -4, -5, -6, -7
 F32, F16, BF16 = 0, 1, 2
-OP = {"linear": 1, "conv": 2, "maxpool": 3, "gap": 4, "upsample2x": 5, "concat": 6}
-ACT = {"none": 0, "relu": 1, "leaky": 2}
-DTYPE = {"f32": F32, "f16": F16, "bf16": BF16}
+I32 = 3
+OP = {"linear": 1, "conv": 2, "maxpool": 3, "gap": 4, "upsample2x": 5, "concat": 6, "embed": 7, "rmsnorm": 8,
+      "attention": 9, "argmax": 10}
+ACT = {"none": 0, "relu": 1, "leaky": 2, "swiglu": 3}
+DTYPE = {"f32": F32, "f16": F16, "bf16": BF16, "i32": I32}
+LAYER_NO_BIAS = 1
 SWAP_AUTO, SWAP_MEMCPY, SWAP_ZEROCOPY = 0, 1, 2
 SRC_INPUT, SRC_NONE = -1, -2
 
@@ -27,12 +30,15 @@ class Layer(C.Structure):
     _fields_ = [("op", C.c_int32), ("src0", C.c_int32), ("src1", C.c_int32), ("res", C.c_int32),
                 ("act", C.c_int32), ("res_post", C.c_int32), ("cin", C.c_int32), ("cout", C.c_int32),
                 ("kh", C.c_int32), ("kw", C.c_int32), ("stride", C.c_int32), ("pad", C.c_int32),
-                ("is_output", C.c_int32), ("reserved", C.c_int32), ("t_ex_ns", C.c_int64)]
+                ("is_output", C.c_int32), ("flags", C.c_int32), ("t_ex_ns", C.c_int64), ("src2", C.c_int32),
+                ("heads", C.c_int32), ("max_seq", C.c_int32), ("eps", C.c_float), ("theta", C.c_float),
+                ("reserved", C.c_int32)]
 
 
 class ModelDesc(C.Structure):
     _fields_ = [("dtype", C.c_int32), ("n_layers", C.c_int32), ("layers", C.POINTER(Layer)),
-                ("in_n", C.c_int32), ("in_h", C.c_int32), ("in_w", C.c_int32), ("in_c", C.c_int32)]
+                ("in_n", C.c_int32), ("in_h", C.c_int32), ("in_w", C.c_int32), ("in_c", C.c_int32),
+                ("in_dtype", C.c_int32), ("reserved", C.c_int32)]
 
 
 class Options(C.Structure):
@@ -47,7 +53,8 @@ class PlanInfo(C.Structure):
                 ("n_layers", C.c_uint32), ("budget_bytes", C.c_uint64), ("arena_bytes", C.c_uint64),
                 ("slot_bytes", C.c_uint64), ("workspace_bytes", C.c_uint64), ("input_bytes", C.c_uint64),
                 ("output_bytes", C.c_uint64), ("weight_bytes", C.c_uint64), ("plan_bytes", C.c_uint64),
-                ("predicted_ns", C.c_int64)]
+                ("predicted_ns", C.c_int64), ("state_bytes", C.c_uint64), ("exact", C.c_int32),
+                ("reserved", C.c_int32)]
 
 
 class UnitInfo(C.Structure):
@@ -67,7 +74,8 @@ class EngineStats(C.Structure):
 
 
 KERNEL_KIND = {1: "tc_gemm", 2: "tc_conv", 3: "skinny_linear", 4: "direct_conv", 5: "maxpool", 6: "gap",
-               7: "upsample2x", 8: "concat", 9: "tiled_linear"}
+               7: "upsample2x", 8: "concat", 9: "tiled_linear", 10: "embed", 11: "rmsnorm", 12: "attention",
+               13: "argmax"}
 
 
 class EngineBlock(C.Structure):
@@ -81,7 +89,8 @@ EXPORTS = ["swapnet_default_options", "swapnet_partition", "swapnet_plan_from_cu
            "swapnet_infer", "swapnet_infer_host", "swapnet_engine_sync", "swapnet_engine_blocks",
            "swapnet_engine_free", "swapnet_engine_stats_get", "swapnet_engine_unit_kernels",
            "swapnet_engine_set_profiling", "swapnet_engine_last_times", "swapnet_engine_measure_units",
-           "swapnet_engine_last_timeline", "swapnet_strerror", "swapnet_last_error", "swapnet_debug_fail_next", "swapnet_gemm_noalloc"]
+           "swapnet_engine_last_timeline",
+           "swapnet_engine_bind_state", "swapnet_strerror", "swapnet_last_error", "swapnet_debug_fail_next", "swapnet_gemm_noalloc"]
 
 _lib = None
 
@@ -121,6 +130,7 @@ def lib():
         "swapnet_infer": (C.c_int, [P, P, P, P]),
         "swapnet_infer_host": (C.c_int, [P, P, P, P]),
         "swapnet_engine_sync": (C.c_int, [P]),
+        "swapnet_engine_bind_state": (C.c_int, [P, P, C.c_uint64]),
         "swapnet_engine_blocks": (C.c_int, [P, C.POINTER(EngineBlock), C.c_uint32, C.POINTER(C.c_uint32)]),
         "swapnet_engine_free": (None, [P]),
         "swapnet_engine_stats_get": (C.c_int, [P, C.POINTER(EngineStats)]),
@@ -181,11 +191,29 @@ class Desc:
                 c.cin, c.cout = L["k"], L["n"]
             elif L["op"] == "maxpool":
                 c.kh, c.kw, c.stride, c.pad = L["kh"], L["kw"], L["stride"], L["pad"]
+            elif L["op"] == "embed":
+                c.cin, c.cout = L["vocab"], L["d"]
+            elif L["op"] == "rmsnorm":
+                c.cout, c.eps = L["d"], L["eps"]
+            elif L["op"] == "attention":
+                c.src0, c.src1, c.src2 = L["src"]
+                c.heads, c.max_seq, c.theta = L["heads"], L["max_seq"], L["theta"]
+            if L["op"] == "attention":
+                c.cout = 0  # filled below from the q width
+            if L["op"] != "attention":
+                c.src2 = SRC_NONE
+            if L.get("bias") is False:
+                c.flags |= LAYER_NO_BIAS
             c.is_output = 1 if i in outs else 0
             c.t_ex_ns = 0 if t_ex_ns is None else int(t_ex_ns[i])
+        # attention width = width of its q input
+        for i, L in enumerate(layers):
+            if L["op"] == "attention":
+                arr[i].cout = arr[L["src"][0]].cout
         n, h, w, ch = model["input"]
         self.layers = arr
-        self.c = ModelDesc(DTYPE[model["dtype"]], len(layers), arr, n, h, w, ch)
+        in_dt = DTYPE[model.get("input_dtype", model["dtype"])]
+        self.c = ModelDesc(DTYPE[model["dtype"]], len(layers), arr, n, h, w, ch, in_dt, 0)
         self.model = model
 
 
@@ -340,6 +368,9 @@ class Engine:
         check(lib().swapnet_load(plan.h, host.ptrs, host.n, C.c_void_p(d_arena or None), arena_bytes,
                                  C.c_void_p(d_ws or None), ws_bytes, C.byref(h)), "swapnet_load")
         self.h = h
+
+    def bind_state(self, d_state, nbytes):
+        check(lib().swapnet_engine_bind_state(self.h, C.c_void_p(d_state), nbytes), "swapnet_engine_bind_state")
 
     def infer(self, d_in, d_out, stream=0):
         check(lib().swapnet_infer(self.h, C.c_void_p(d_in), C.c_void_p(d_out), C.c_void_p(stream or None)),

@@ -10,7 +10,7 @@
 namespace swapnet {
 
 // Error codes written to the device error word by bounded waits.
-enum DevErr : int { kDevErrNone = 0, kDevErrTimeout = 1 };
+enum DevErr : int { kDevErrNone = 0, kDevErrTimeout = 1, kDevErrBounds = 2 };
 
 // ---------------------------------------------------------------- elements
 template <typename T> __device__ __forceinline__ float to_f(T v);
@@ -32,6 +32,7 @@ __device__ __forceinline__ float apply_act(float v, int act) {
 // Fused epilogue of one output element: bias, residual and activation in
 // fp32, in the order the layer defines.
 __device__ __forceinline__ float epilogue(float acc, float bias, float res, int has_res, int act, int res_post) {
+  if (act == SWAPNET_ACT_SWIGLU) return res / (1.0f + expf(-res)) * (acc + bias);  // silu(gate) * (acc + b)
   float v = acc + bias;
   if (has_res && !res_post) v += res;
   v = apply_act(v, act);

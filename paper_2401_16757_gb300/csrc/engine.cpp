@@ -111,6 +111,7 @@ struct swapnet_engine {
   cudaEvent_t fork = nullptr, join = nullptr;
   // per (input, output, profiling) binding
   std::map<std::pair<std::pair<const void*, void*>, bool>, cudaGraphExec_t> graphs;
+  char* d_state = nullptr;           // decoder state (position + KV caches), caller-owned
   char* d_splitk = nullptr;          // split-K scratch: tile counters, then fp32 partials
   uint64_t splitk_bytes = 0;
   uint64_t splitk_counter_bytes = 0;
@@ -229,6 +230,7 @@ static void build_segments(swapnet_engine* e) {
     char* base = block_base(e, B);
     for (int u = B.u0; u < B.u1; ++u) {
       const Unit& U = p.units[u];
+      if (U.host) continue;  // host-resident parameters are never swapped
       for (int t = 0; t < U.nt; ++t) {
         if (U.tlen[t] == 0) continue;
         Segment s{e->tensor_dev[U.tidx[t]] + U.toff[t], base + U.slot_off[t], U.tlen[t]};
@@ -383,6 +385,10 @@ static int prepare_units(swapnet_engine* e) {
       case SWAPNET_OP_GAP: k = SWAPNET_KERNEL_GAP; break;
       case SWAPNET_OP_UPSAMPLE2X: k = SWAPNET_KERNEL_UPSAMPLE; break;
       case SWAPNET_OP_CONCAT: k = SWAPNET_KERNEL_CONCAT; break;
+      case SWAPNET_OP_EMBED: k = SWAPNET_KERNEL_EMBED; break;
+      case SWAPNET_OP_RMSNORM: k = SWAPNET_KERNEL_RMSNORM; break;
+      case SWAPNET_OP_ATTENTION: k = SWAPNET_KERNEL_ATTENTION; break;
+      case SWAPNET_OP_ARGMAX: k = SWAPNET_KERNEL_ARGMAX; break;
     }
     e->unit_kind[u] = k;
   }
@@ -391,7 +397,12 @@ static int prepare_units(swapnet_engine* e) {
     for (int u = B.u0; u < B.u1; ++u) {
       const Unit& U = p.units[u];
       UnitExec& X = e->ux[u];
-      if (U.nt == 2) { X.w = base + U.slot_off[0]; X.b = base + U.slot_off[1]; }
+      if (U.host) {
+        X.w = e->tensor_dev[U.tidx[0]];  // device alias of the page-locked host table
+      } else {
+        if (U.nt >= 1) X.w = base + U.slot_off[0];
+        if (U.nt == 2) X.b = base + U.slot_off[1];
+      }
       const Layer& L = m.L[U.layer];
       if (!wants_tc(m, L)) continue;
       X.use_tc = true;
@@ -459,6 +470,20 @@ static int run_unit(swapnet_engine* e, int u, const void* din, void* dout, cudaS
       return launch_upsample2x(m.dtype, x, L.n, L.h, L.w, L.c, y, s);
     case SWAPNET_OP_CONCAT:
       return launch_concat(m.dtype, x, L.c, act_ptr(e, L.d.src1, din, dout), L.c1, (int64_t)L.n * L.h * L.w, y, s);
+    case SWAPNET_OP_EMBED:
+      return launch_embed(m.dtype, X.w, reinterpret_cast<const int*>(x), L.on, L.d.cin, L.d.cout, y, e->err_word, s);
+    case SWAPNET_OP_RMSNORM:
+      return launch_rmsnorm(m.dtype, x, X.w, L.n, L.c, L.d.eps, y, s);
+    case SWAPNET_OP_ATTENTION: {
+      if (!e->d_state) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "decoder state not bound (swapnet_engine_bind_state)");
+      char* kc = e->d_state + L.state_off;
+      char* vc = kc + align_up((uint64_t)L.d.max_seq * L.c * es);
+      return launch_attention(m.dtype, const_cast<char*>(x), act_ptr(e, L.d.src1, din, dout),
+                              act_ptr(e, L.d.src2, din, dout), kc, vc, reinterpret_cast<const int*>(e->d_state),
+                              L.n, L.d.heads, L.c, L.d.theta, L.d.max_seq, y, e->err_word, s);
+    }
+    case SWAPNET_OP_ARGMAX:
+      return launch_argmax(m.dtype, x, L.n, L.c1, reinterpret_cast<int*>(y), s);
     default:
       SN_FAIL(SWAPNET_ERR_INVALID_ARG, "unknown op");
   }
@@ -607,6 +632,12 @@ static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t 
     }
     if (!p.resident) CU(cudaEventRecord(e->slot_free[B.slot], s), "record slot free");
   }
+  if (p.model.has_attention) {
+    if (!e->d_state) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "decoder state not bound (swapnet_engine_bind_state)");
+    const Model& m = p.model;
+    int rc = launch_advance(reinterpret_cast<int*>(e->d_state), m.in_n * m.in_h * m.in_w * m.in_c, s);
+    if (rc) return rc;
+  }
   if (!p.resident) {
     CU(cudaEventRecord(e->join, e->copy), "record join");
     CU(cudaStreamWaitEvent(s, e->join, 0), "wait join");
@@ -615,7 +646,8 @@ static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t 
 }
 
 static uint64_t launches_per_infer(const swapnet_engine* e) {
-  uint64_t n = e->plan.units.size();
+  uint64_t n = e->plan.units.size() + (e->plan.model.has_attention ? 1 : 0);
+  for (int k : e->unit_kind) n += (k == SWAPNET_KERNEL_ATTENTION) ? 1 : 0;
   if (!e->plan.resident)
     for (const EngBlock& b : e->blocks)
       if (b.variant == SWAPNET_SWAP_ZEROCOPY) n += (b.segs.size() + 47) / 48;
@@ -708,6 +740,7 @@ int swapnet_engine_sync(swapnet_engine* e) {
     const int zero = 0;
     cudaMemcpy(e->err_word, &zero, sizeof(int), cudaMemcpyHostToDevice);
     if (e->d_splitk) cudaMemset(e->d_splitk, 0, e->splitk_counter_bytes);  // an aborted kernel may leave counts
+    if (w == 2) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "a token id or a cache position was out of range");
     SN_FAIL(SWAPNET_ERR_TIMEOUT, "a device-side wait gave up");
   }
   return SWAPNET_OK;
@@ -771,6 +804,17 @@ int swapnet_engine_measure_units(swapnet_engine* e, int32_t reps, float* unit_us
   cudaEventDestroy(a);
   cudaEventDestroy(b);
   if (rc) SN_FAIL(rc, "unit measurement failed");
+  return SWAPNET_OK;
+}
+
+int swapnet_engine_bind_state(swapnet_engine* e, void* d_state, uint64_t bytes) {
+  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+  if (!e->plan.model.has_attention) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "the model has no decoder state");
+  if (!d_state || bytes < e->plan.model.state_bytes) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "state buffer too small");
+  if ((uintptr_t)d_state % kAlign) SN_FAIL(SWAPNET_ERR_MISALIGNED, "state buffer must be 256-byte aligned");
+  e->d_state = static_cast<char*>(d_state);
+  for (auto& kv : e->graphs) cudaGraphExecDestroy(kv.second);  // captured with the old state
+  e->graphs.clear();
   return SWAPNET_OK;
 }
 

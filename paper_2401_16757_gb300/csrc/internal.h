@@ -42,10 +42,14 @@ struct Layer {
   int64_t ws_off;        // workspace offset, -1 when the output is a model output
   int64_t out_off;       // offset in the output buffer, -1 if not an output
   uint64_t out_bytes;    // raw bytes of the output tensor
+  bool host_resident;    // parameters read in host memory, never swapped (EMBED)
+  int64_t state_off;     // ATTENTION: offset of its key cache in the decoder state
 };
 
 struct Model {
-  int dtype = 0, es = 0;
+  int dtype = 0, es = 0, in_dtype = 0;
+  uint64_t state_bytes = 0;  // decoder state: 256-byte position header + KV caches
+  bool has_attention = false;
   int in_n = 0, in_h = 0, in_w = 0, in_c = 0;
   std::vector<Layer> L;
   int n_tensors = 0;
@@ -63,6 +67,7 @@ struct Unit {
   int nt;
   int tidx[2];
   uint64_t toff[2], tlen[2], slot_off[2];
+  bool host;  // host-resident parameters: not swapped, read through the mapped alias
 };
 
 struct Block {
@@ -86,6 +91,7 @@ struct swapnet_plan {
   std::vector<swapnet::Block> blocks;
   std::vector<uint32_t> cuts;
   int64_t predicted = 0;
+  bool exact = true;  // the search proved the plan optimal for its objective
 };
 
 namespace swapnet {

@@ -1,0 +1,268 @@
+// Decoder-layer kernels: embedding gather (zero-copy from the host-resident
+// table), RMSNorm, RoPE + KV-cache append, causal attention with an online
+// softmax, row argmax, and the device-side advance of the cache position.
+// bf16 / fp16 storage, fp32 arithmetic, fixed reduction orders.
+#include <cstring>
+
+#include "device.cuh"
+#include "internal.h"
+#include "kernels.h"
+
+namespace swapnet {
+
+namespace {
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg;
+  std::memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
+int done(cudaError_t e, const char* what) {
+  if (e == cudaSuccess) e = cudaGetLastError();
+  if (e != cudaSuccess) SN_FAIL(SWAPNET_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+  return SWAPNET_OK;
+}
+
+// ------------------------------------------------------------ embedding
+// Row t of the output is row ids[t] of the table, read straight from the
+// page-locked host table (device alias) with 16-byte loads.
+template <typename T>
+__global__ void __launch_bounds__(256) embed_kernel(const T* __restrict__ table, const int* __restrict__ ids,
+                                                    int vocab, int d, T* __restrict__ out, int* err) {
+  pdl_wait();
+  pdl_launch_dependents();
+  const int t = blockIdx.x;
+  const int id = ids[t];
+  const bool ok = id >= 0 && id < vocab;
+  if (!ok && threadIdx.x == 0) atomicExch(err, kDevErrBounds);
+  const uint4* src = reinterpret_cast<const uint4*>(table + (int64_t)(ok ? id : 0) * d);
+  uint4* dst = reinterpret_cast<uint4*>(out + (int64_t)t * d);
+  const int n16 = d * (int)sizeof(T) / 16;
+  for (int i = threadIdx.x; i < n16; i += blockDim.x) dst[i] = ok ? src[i] : make_uint4(0, 0, 0, 0);
+}
+
+// ------------------------------------------------------------ RMSNorm
+// One CTA per row; the sum of squares is reduced in a fixed order (lane
+// partials, warp butterfly, warps in index order).
+template <typename T>
+__global__ void __launch_bounds__(256) rmsnorm_kernel(const T* __restrict__ x, const T* __restrict__ g, int d,
+                                                      float eps, T* __restrict__ y) {
+  __shared__ float wsum[8];
+  pdl_wait();
+  pdl_launch_dependents();
+  const T* xr = x + (int64_t)blockIdx.x * d;
+  float s = 0.f;
+  for (int i = threadIdx.x; i < d; i += blockDim.x) {
+    const float v = to_f<T>(xr[i]);
+    s = fmaf(v, v, s);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+  if ((threadIdx.x & 31) == 0) wsum[threadIdx.x >> 5] = s;
+  __syncthreads();
+  float tot = 0.f;
+  for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += wsum[w];
+  const float r = 1.0f / sqrtf(tot / (float)d + eps);
+  T* yr = y + (int64_t)blockIdx.x * d;
+  for (int i = threadIdx.x; i < d; i += blockDim.x) yr[i] = from_f<T>(to_f<T>(xr[i]) * r * to_f<T>(g[i]));
+}
+
+// ------------------------------------------------------------ RoPE + cache
+// Thread = one adjacent pair (2i, 2i+1) of one head of one token: rotates
+// q in place and k into the key cache at the state position, copies v into
+// the value cache.  Angles: position * theta^(-2i/Dh), computed in fp32.
+template <typename T>
+__global__ void __launch_bounds__(256) rope_append_kernel(T* __restrict__ q, const T* __restrict__ k,
+                                                          const T* __restrict__ v, T* __restrict__ kc,
+                                                          T* __restrict__ vc, const int* __restrict__ pos_ptr,
+                                                          int width, int dh, float theta, int max_seq, int* err) {
+  pdl_wait();
+  pdl_launch_dependents();
+  const int t = blockIdx.y;
+  const int pair = blockIdx.x * blockDim.x + threadIdx.x;  // over width / 2
+  if (pair >= width / 2) return;
+  const int pos = *pos_ptr + t;
+  if (pos >= max_seq) {
+    if (pair == 0) atomicExch(err, kDevErrBounds);
+    return;
+  }
+  const int col = 2 * pair;
+  const int i = (col % dh) / 2;
+  const float inv = powf(theta, -2.0f * (float)i / (float)dh);
+  float sn, cs;
+  sincosf((float)pos * inv, &sn, &cs);
+  T* qp = q + (int64_t)t * width + col;
+  const float q0 = to_f<T>(qp[0]), q1 = to_f<T>(qp[1]);
+  qp[0] = from_f<T>(q0 * cs - q1 * sn);
+  qp[1] = from_f<T>(q0 * sn + q1 * cs);
+  const T* kp = k + (int64_t)t * width + col;
+  const float k0 = to_f<T>(kp[0]), k1 = to_f<T>(kp[1]);
+  T* kd = kc + (int64_t)pos * width + col;
+  kd[0] = from_f<T>(k0 * cs - k1 * sn);
+  kd[1] = from_f<T>(k0 * sn + k1 * cs);
+  const T* vp = v + (int64_t)t * width + col;
+  T* vd = vc + (int64_t)pos * width + col;
+  vd[0] = vp[0];
+  vd[1] = vp[1];
+}
+
+// ------------------------------------------------------------ attention
+// Warp = one (query, head); each lane holds 4 of the 128 head dimensions.
+// Keys are visited in position order with an online softmax in fp32:
+// m (running max), l (running denominator), acc (running numerator).
+constexpr int kDh = 128;
+
+template <typename T>
+__device__ __forceinline__ void load4(const T* p, float* f) {
+  const uint2 u = *reinterpret_cast<const uint2*>(p);
+  const T* e = reinterpret_cast<const T*>(&u);
+#pragma unroll
+  for (int j = 0; j < 4; ++j) f[j] = to_f<T>(e[j]);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) attention_kernel(const T* __restrict__ q, const T* __restrict__ kc,
+                                                        const T* __restrict__ vc, const int* __restrict__ pos_ptr,
+                                                        int T_, int heads, int width, int max_seq,
+                                                        T* __restrict__ out) {
+  pdl_wait();
+  pdl_launch_dependents();
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (warp >= T_ * heads) return;
+  const int t = warp / heads, h = warp % heads;
+  const int pos = *pos_ptr + t;
+  const int n = min(pos + 1, max_seq);
+  const int c0 = h * kDh + lane * 4;
+  float qv[4];
+  load4<T>(q + (int64_t)t * width + c0, qv);
+  const float scale = rsqrtf((float)kDh);
+  float m = -INFINITY, l = 0.f, acc[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int j = 0; j < n; ++j) {
+    float kv[4];
+    load4<T>(kc + (int64_t)j * width + c0, kv);
+    float s = qv[0] * kv[0] + qv[1] * kv[1] + qv[2] * kv[2] + qv[3] * kv[3];
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+    s *= scale;
+    const float mn = fmaxf(m, s);
+    const float a = expf(m - mn);   // 0 on the first key (m = -inf)
+    const float p = expf(s - mn);
+    float vv[4];
+    load4<T>(vc + (int64_t)j * width + c0, vv);
+    l = l * a + p;
+#pragma unroll
+    for (int d = 0; d < 4; ++d) acc[d] = acc[d] * a + p * vv[d];
+    m = mn;
+  }
+  const float inv = 1.0f / l;
+  T* o = out + (int64_t)t * width + c0;
+#pragma unroll
+  for (int d = 0; d < 4; ++d) o[d] = from_f<T>(acc[d] * inv);
+}
+
+// ------------------------------------------------------------ argmax
+template <typename T>
+__global__ void __launch_bounds__(256) argmax_kernel(const T* __restrict__ x, int n, int* __restrict__ out) {
+  __shared__ float sv[256];
+  __shared__ int si[256];
+  pdl_wait();
+  pdl_launch_dependents();
+  const T* row = x + (int64_t)blockIdx.x * n;
+  float best = -INFINITY;
+  int bi = 0x7fffffff;
+  for (int j = threadIdx.x; j < n; j += blockDim.x) {
+    const float v = to_f<T>(row[j]);
+    if (v > best) { best = v; bi = j; }  // strictly greater: first index wins
+  }
+  sv[threadIdx.x] = best;
+  si[threadIdx.x] = bi;
+  __syncthreads();
+  for (int stride = blockDim.x / 2; stride > 0; stride >>= 1) {
+    if ((int)threadIdx.x < stride) {
+      const float ov = sv[threadIdx.x + stride];
+      const int oi = si[threadIdx.x + stride];
+      if (ov > sv[threadIdx.x] || (ov == sv[threadIdx.x] && oi < si[threadIdx.x])) {
+        sv[threadIdx.x] = ov;
+        si[threadIdx.x] = oi;
+      }
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) out[blockIdx.x] = si[0] == 0x7fffffff ? 0 : si[0];
+}
+
+__global__ void advance_kernel(int* pos_ptr, int n) {
+  pdl_wait();
+  pdl_launch_dependents();
+  *pos_ptr += n;
+}
+
+}  // namespace
+
+#define SN_DISPATCH16(dtype, T, ...)                                     \
+  switch (dtype) {                                                       \
+    case SWAPNET_F16: { using T = __half; __VA_ARGS__; break; }          \
+    case SWAPNET_BF16: { using T = __nv_bfloat16; __VA_ARGS__; break; }  \
+    default: SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "decoder kernels: fp16 / bf16 only"); \
+  }
+
+int launch_embed(int dtype, const void* table, const int* ids, int tokens, int vocab, int d, void* out, int* err,
+                 cudaStream_t s) {
+  if ((d * 2) % 16 || ((uintptr_t)table | (uintptr_t)out) % 16)
+    SN_FAIL(SWAPNET_ERR_MISALIGNED, "embedding rows must be 16-byte aligned");
+  SN_DISPATCH16(dtype, T, return done(launch_pdl(embed_kernel<T>, dim3(tokens), dim3(256), 0, s,
+                                                 static_cast<const T*>(table), ids, vocab, d,
+                                                 static_cast<T*>(out), err), "embedding launch"));
+  return SWAPNET_OK;
+}
+
+int launch_rmsnorm(int dtype, const void* x, const void* g, int rows, int d, float eps, void* y, cudaStream_t s) {
+  SN_DISPATCH16(dtype, T, return done(launch_pdl(rmsnorm_kernel<T>, dim3(rows), dim3(256), 0, s,
+                                                 static_cast<const T*>(x), static_cast<const T*>(g), d, eps,
+                                                 static_cast<T*>(y)), "rmsnorm launch"));
+  return SWAPNET_OK;
+}
+
+int launch_attention(int dtype, void* q, const void* k, const void* v, void* kc, void* vc, const int* pos_ptr,
+                     int tokens, int heads, int width, float theta, int max_seq, void* out, int* err,
+                     cudaStream_t s) {
+  if (width % heads || width / heads != kDh) SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "attention: head width must be 128");
+  SN_DISPATCH16(dtype, T, {
+    const dim3 g1((width / 2 + 255) / 256, tokens);
+    int rc = done(launch_pdl(rope_append_kernel<T>, g1, dim3(256), 0, s, static_cast<T*>(q),
+                             static_cast<const T*>(k), static_cast<const T*>(v), static_cast<T*>(kc),
+                             static_cast<T*>(vc), pos_ptr, width, kDh, theta, max_seq, err),
+                  "rope launch");
+    if (rc) return rc;
+    const int warps = tokens * heads;
+    return done(launch_pdl(attention_kernel<T>, dim3((warps * 32 + 255) / 256), dim3(256), 0, s,
+                           static_cast<const T*>(q), static_cast<const T*>(kc), static_cast<const T*>(vc),
+                           pos_ptr, tokens, heads, width, max_seq, static_cast<T*>(out)),
+                "attention launch");
+  });
+  return SWAPNET_OK;
+}
+
+int launch_argmax(int dtype, const void* x, int rows, int n, int* out, cudaStream_t s) {
+  SN_DISPATCH16(dtype, T, return done(launch_pdl(argmax_kernel<T>, dim3(rows), dim3(256), 0, s,
+                                                 static_cast<const T*>(x), n, out), "argmax launch"));
+  return SWAPNET_OK;
+}
+
+int launch_advance(int* pos_ptr, int n, cudaStream_t s) {
+  return done(launch_pdl(advance_kernel, dim3(1), dim3(1), 0, s, pos_ptr, n), "position advance launch");
+}
+
+}  // namespace swapnet

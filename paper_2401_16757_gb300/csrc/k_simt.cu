@@ -118,7 +118,7 @@ __global__ void __launch_bounds__(kSkWarps * 32) linear_skinny_kernel(const T* _
       float s = 0.f;
 #pragma unroll
       for (int w = 0; w < kSkWarps; ++w) s += red[w][c][m];
-      const float b = to_f<T>(reinterpret_cast<const T*>(e.bias)[o]);
+      const float b = e.bias ? to_f<T>(reinterpret_cast<const T*>(e.bias)[o]) : 0.f;
       float r = 0.f;
       if (e.res) r = to_f<T>(reinterpret_cast<const T*>(e.res)[(int64_t)m * e.ldr + o]);
       y[(int64_t)m * ldy + o] = from_f<T>(epilogue(s, b, r, e.res != nullptr, e.act, e.res_post));
@@ -187,7 +187,8 @@ __global__ void __launch_bounds__(256) linear_tiled_kernel(const T* __restrict__
       const int n = n0 + tx + 16 * j;
       if (n >= N) continue;
       const float rv = res ? to_f<T>(res[(int64_t)m * e.ldr + n]) : 0.f;
-      y[(int64_t)m * ldy + n] = from_f<T>(epilogue(acc[i][j], to_f<T>(bias[n]), rv, res != nullptr, e.act, e.res_post));
+      y[(int64_t)m * ldy + n] =
+          from_f<T>(epilogue(acc[i][j], bias ? to_f<T>(bias[n]) : 0.f, rv, res != nullptr, e.act, e.res_post));
     }
   }
 }
@@ -252,7 +253,8 @@ __global__ void __launch_bounds__(128) conv_direct_kernel(const T* __restrict__ 
     const int co = co0 + j;
     if (co < cout) {
       const float rv = res ? to_f<T>(res[pix * e.ldr + co]) : 0.f;
-      y[pix * cout + co] = from_f<T>(epilogue(acc[j], to_f<T>(bias[co]), rv, res != nullptr, e.act, e.res_post));
+      y[pix * cout + co] =
+        from_f<T>(epilogue(acc[j], bias ? to_f<T>(bias[co]) : 0.f, rv, res != nullptr, e.act, e.res_post));
     }
   }
 }

@@ -214,7 +214,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   // bias of this tile to shared memory (weights: ready before the kernel)
   if (threadIdx.x >= 64) {
     const T* bias = static_cast<const T*>(p.e.bias);
-    for (int j = threadIdx.x - 64; j < BN; j += 128) sbias[j] = (n0 + j < p.N) ? to_f<T>(bias[n0 + j]) : 0.f;
+    for (int j = threadIdx.x - 64; j < BN; j += 128) sbias[j] = (bias && n0 + j < p.N) ? to_f<T>(bias[n0 + j]) : 0.f;
   }
   tc_fence_before();
   __syncthreads();

@@ -38,6 +38,19 @@ int launch_upsample2x(int dtype, const void* x, int n, int h, int w, int c, void
 int launch_concat(int dtype, const void* a, int ca, const void* b, int cb, int64_t pixels, void* y,
                   cudaStream_t s);
 
+// Decoder kernels (fp16 / bf16).  The embedding table pointer is the device
+// alias of the page-locked host table.  The attention launcher runs the RoPE
+// + cache-append kernel (q rotated in place) and then the attention kernel;
+// pos_ptr is the device-side position of the decoder state.
+int launch_embed(int dtype, const void* table, const int* ids, int tokens, int vocab, int d, void* out, int* err,
+                 cudaStream_t s);
+int launch_rmsnorm(int dtype, const void* x, const void* g, int rows, int d, float eps, void* y, cudaStream_t s);
+int launch_attention(int dtype, void* q, const void* k, const void* v, void* kc, void* vc, const int* pos_ptr,
+                     int tokens, int heads, int width, float theta, int max_seq, void* out, int* err,
+                     cudaStream_t s);
+int launch_argmax(int dtype, const void* x, int rows, int n, int* out, cudaStream_t s);
+int launch_advance(int* pos_ptr, int n, cudaStream_t s);
+
 // Zero-copy swap: copy segments from mapped host memory (device aliases)
 // into the arena with 16-byte vector loads/stores.
 struct ZcSeg {

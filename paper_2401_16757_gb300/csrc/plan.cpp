@@ -31,11 +31,18 @@ int analyse_model(const swapnet_model_desc* desc, Model* m) {
   if (!desc || !desc->layers || desc->n_layers <= 0) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "empty model descriptor");
   m->dtype = desc->dtype;
   m->es = dtype_size(desc->dtype);
-  if (!m->es) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "unknown dtype");
+  if (!m->es || desc->dtype == SWAPNET_I32) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "unknown dtype");
+  m->in_dtype = desc->in_dtype;
+  if (m->in_dtype != m->dtype && m->in_dtype != SWAPNET_I32)
+    SN_FAIL(SWAPNET_ERR_INVALID_ARG, "input dtype must be the model dtype or int32 token ids");
   if (desc->in_n <= 0 || desc->in_h <= 0 || desc->in_w <= 0 || desc->in_c <= 0)
     SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad input shape");
   m->in_n = desc->in_n; m->in_h = desc->in_h; m->in_w = desc->in_w; m->in_c = desc->in_c;
-  m->in_bytes = (uint64_t)m->in_n * m->in_h * m->in_w * m->in_c * m->es;
+  m->in_bytes = (uint64_t)m->in_n * m->in_h * m->in_w * m->in_c *
+                (m->in_dtype == SWAPNET_I32 ? 4 : m->es);
+  m->state_bytes = 0;
+  m->has_attention = false;
+  uint64_t state_cur = kAlign;  // position header
   const int nl = desc->n_layers;
   m->L.assign(nl, Layer{});
   m->n_tensors = 0;
@@ -58,7 +65,16 @@ int analyse_model(const swapnet_model_desc* desc, Model* m) {
     L.n_tensors = 0;
     L.tbytes[0] = L.tbytes[1] = 0;
     L.flops = 0;
+    L.host_resident = false;
+    L.state_off = -1;
     const uint64_t es = m->es;
+    const bool token_input = d.src0 == SWAPNET_SRC_INPUT && m->in_dtype == SWAPNET_I32;
+    if (token_input && d.op != SWAPNET_OP_EMBED)
+      SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": only EMBED reads token ids");
+    auto same_dims = [&](int src) -> bool {
+      int n, h, w, c;
+      return dims_of(src, &n, &h, &w, &c) && n == L.n && h == L.h && w == L.w && c == L.c;
+    };
     switch (d.op) {
       case SWAPNET_OP_CONV2D: {
         if (d.cin != L.c || d.cout <= 0 || d.kh <= 0 || d.kw <= 0 || d.stride <= 0 || d.pad < 0)
@@ -78,9 +94,9 @@ int analyse_model(const swapnet_model_desc* desc, Model* m) {
         if ((int64_t)d.cin != (int64_t)L.h * L.w * L.c || d.cout <= 0)
           SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": linear in-features mismatch");
         L.on = L.n; L.oh = 1; L.ow = 1; L.oc = d.cout;
-        L.n_tensors = 2;
+        L.n_tensors = (d.flags & SWAPNET_LAYER_NO_BIAS) ? 1 : 2;
         L.tbytes[0] = (uint64_t)d.cout * d.cin * es;
-        L.tbytes[1] = (uint64_t)d.cout * es;
+        L.tbytes[1] = L.n_tensors == 2 ? (uint64_t)d.cout * es : 0;
         L.flops = 2ull * L.n * (uint64_t)d.cin * d.cout;
         break;
       }
@@ -108,11 +124,44 @@ int analyse_model(const swapnet_model_desc* desc, Model* m) {
         L.on = L.n; L.oh = L.h; L.ow = L.w; L.oc = L.c + c1;
         break;
       }
+      case SWAPNET_OP_EMBED: {
+        if (!token_input || d.cin <= 0 || d.cout <= 0 || (d.cout * es) % 16)
+          SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": bad embedding");
+        L.on = L.n * L.h * L.w * L.c; L.oh = 1; L.ow = 1; L.oc = d.cout;
+        L.n_tensors = 1;
+        L.tbytes[0] = (uint64_t)d.cin * d.cout * es;
+        L.host_resident = true;
+        break;
+      }
+      case SWAPNET_OP_RMSNORM:
+        if (d.cout != L.c || L.h != 1 || L.w != 1 || !(d.eps >= 0.f))
+          SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": bad rmsnorm");
+        L.on = L.n; L.oh = 1; L.ow = 1; L.oc = L.c;
+        L.n_tensors = 1;
+        L.tbytes[0] = (uint64_t)d.cout * es;
+        break;
+      case SWAPNET_OP_ATTENTION: {
+        if (!same_dims(d.src1) || !same_dims(d.src2) || L.h != 1 || L.w != 1 || d.cout != L.c || d.heads <= 0 ||
+            L.c % d.heads || d.max_seq <= 0 || !(d.theta > 0.f))
+          SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": bad attention");
+        L.on = L.n; L.oh = 1; L.ow = 1; L.oc = L.c;
+        L.flops = 4ull * L.n * (uint64_t)d.max_seq * L.c;
+        L.state_off = (int64_t)state_cur;
+        state_cur += 2 * align_up((uint64_t)d.max_seq * L.c * es);
+        m->has_attention = true;
+        break;
+      }
+      case SWAPNET_OP_ARGMAX:
+        L.on = L.n; L.oh = 1; L.ow = 1; L.oc = 1;
+        L.c1 = L.h * L.w * L.c;  // row length
+        break;
       default:
         SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": unknown op");
     }
-    if (d.op != SWAPNET_OP_CONCAT && d.src1 != SWAPNET_SRC_NONE)
-      SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": src1 only for concat");
+    if (d.op != SWAPNET_OP_CONCAT && d.op != SWAPNET_OP_ATTENTION && d.src1 != SWAPNET_SRC_NONE)
+      SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": src1 only for concat and attention");
+    if (d.op != SWAPNET_OP_ATTENTION && d.src2 != SWAPNET_SRC_NONE && d.src2 != 0)
+      SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": src2 only for attention");
     if (d.res != SWAPNET_SRC_NONE) {
       if (d.op != SWAPNET_OP_CONV2D && d.op != SWAPNET_OP_LINEAR)
         SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": residual only on conv/linear");
@@ -121,8 +170,10 @@ int analyse_model(const swapnet_model_desc* desc, Model* m) {
       if (R.on != L.on || R.oh != L.oh || R.ow != L.ow || R.oc != L.oc)
         SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": residual shape mismatch");
     }
-    if (d.act < SWAPNET_ACT_NONE || d.act > SWAPNET_ACT_LEAKY)
+    if (d.act < SWAPNET_ACT_NONE || d.act > SWAPNET_ACT_SWIGLU)
       SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": bad activation");
+    if (d.act == SWAPNET_ACT_SWIGLU && (d.op != SWAPNET_OP_LINEAR || d.res == SWAPNET_SRC_NONE))
+      SN_FAIL(SWAPNET_ERR_INVALID_ARG, "layer " + std::to_string(i) + ": SWIGLU needs a linear layer and a gate");
     if (d.t_ex_ns < 0) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "negative t_ex_ns");
     L.first_tensor = m->n_tensors;
     for (int t = 0; t < L.n_tensors; ++t) {
@@ -130,13 +181,14 @@ int analyse_model(const swapnet_model_desc* desc, Model* m) {
       m->weight_bytes += align_up(L.tbytes[t]);
     }
     m->n_tensors += L.n_tensors;
-    L.out_bytes = (uint64_t)L.on * L.oh * L.ow * L.oc * es;
+    L.out_bytes = (uint64_t)L.on * L.oh * L.ow * L.oc * (d.op == SWAPNET_OP_ARGMAX ? 4 : es);
   }
+  m->state_bytes = m->has_attention ? state_cur : 0;
   // liveness: last reader of every output
   for (int i = 0; i < nl; ++i) m->L[i].last_use = i;
   for (int j = 0; j < nl; ++j) {
     const swapnet_layer& d = m->L[j].d;
-    for (int s : {d.src0, d.src1, d.res})
+    for (int s : {d.src0, d.src1, d.res, d.op == SWAPNET_OP_ATTENTION ? d.src2 : -1})
       if (s >= 0) m->L[s].last_use = std::max(m->L[s].last_use, j);
   }
   // outputs go to the output buffer, in layer order
@@ -194,9 +246,10 @@ int make_units(const Model& m, const swapnet_options& opt, uint64_t slot, uint64
   for (int li = 0; li < (int)m.L.size(); ++li) {
     const Layer& L = m.L[li];
     uint64_t size = 0;
-    for (int t = 0; t < L.n_tensors; ++t) size += align_up(L.tbytes[t]);
+    for (int t = 0; t < L.n_tensors && !L.host_resident; ++t) size += align_up(L.tbytes[t]);
     if (size <= slot || (L.d.op != SWAPNET_OP_LINEAR && size <= region)) {
       Unit u{};
+      u.host = L.host_resident;
       u.layer = li; u.row0 = 0; u.rows = (L.d.op == SWAPNET_OP_LINEAR) ? L.d.cout : 0;
       u.depth = L.n_tensors; u.bytes = size; u.flops = L.flops;
       u.t_ex = unit_tex(m, opt, L, L.flops, u.rows);
@@ -211,7 +264,8 @@ int make_units(const Model& m, const swapnet_options& opt, uint64_t slot, uint64
       SN_FAIL(SWAPNET_ERR_INFEASIBLE, "layer " + std::to_string(li) + " (" + std::to_string(size) +
                                           " B) does not fit the arena of " + std::to_string(region) + " B");
     const uint64_t K = L.d.cin, N = L.d.cout;
-    auto piece_bytes = [&](uint64_t r) { return align_up(r * K * es) + align_up(r * es); };
+    const bool has_bias = L.n_tensors == 2;
+    auto piece_bytes = [&](uint64_t r) { return align_up(r * K * es) + (has_bias ? align_up(r * es) : 0); };
     uint64_t rmax = 0;
     for (uint64_t r = 128; r <= N + 127 && piece_bytes(r) <= slot; r += 128) rmax = r;
     if (rmax == 0)
@@ -221,13 +275,13 @@ int make_units(const Model& m, const swapnet_options& opt, uint64_t slot, uint64
     for (uint64_t r0 = 0; r0 < N; r0 += rr) {
       const uint64_t rows = std::min(rr, N - r0);
       Unit u{};
-      u.layer = li; u.row0 = (int)r0; u.rows = (int)rows; u.depth = 2;
+      u.layer = li; u.row0 = (int)r0; u.rows = (int)rows; u.depth = L.n_tensors;
       u.bytes = piece_bytes(rows);
       u.flops = 2ull * L.n * K * rows;
       u.t_ex = unit_tex(m, opt, L, u.flops, (int)rows);
-      u.nt = 2;
+      u.nt = L.n_tensors;
       u.tidx[0] = L.first_tensor; u.toff[0] = r0 * K * es; u.tlen[0] = rows * K * es;
-      u.tidx[1] = L.first_tensor + 1; u.toff[1] = r0 * es; u.tlen[1] = rows * es;
+      if (has_bias) { u.tidx[1] = L.first_tensor + 1; u.toff[1] = r0 * es; u.tlen[1] = rows * es; }
       out->push_back(u);
     }
   }
@@ -293,6 +347,7 @@ void finalize_blocks(swapnet_plan* p, const std::vector<uint32_t>& cuts) {
     uint64_t off = 0;
     for (int u = B.u0; u < B.u1; ++u) {
       Unit& U = p->units[u];
+      if (U.host) continue;  // read in host memory: no place in the slot
       for (int t = 0; t < U.nt; ++t) { U.slot_off[t] = off; off += align_up(U.tlen[t]); }
     }
     p->blocks.push_back(B);
@@ -317,7 +372,9 @@ static bool pair_ok(const swapnet_plan* p, uint64_t prev_bytes, uint64_t bytes) 
 namespace {
 
 struct State {
-  int64_t v[5];     // C, E, R_{k-1}, R_k (m = 2) or C, E, R_k, 0 (m = 1); bytes of the last block
+  // v[0] a: earliest start of the next copy (m = 2: max(C_k, R_{k-1});
+  //         m = 1: R_k); v[1] E_k; v[2] R_k; v[3] bytes of the last block
+  int64_t v[4];
   int nblocks;
   int prev_j;       // boundary of the previous state
   int prev_idx;     // index in the previous frontier
@@ -354,7 +411,7 @@ struct Search {
   }
 
   static bool le_all(const State& a, const State& b) {
-    for (int t = 0; t < 5; ++t)
+    for (int t = 0; t < 4; ++t)
       if (a.v[t] > b.v[t]) return false;
     return true;
   }
@@ -365,26 +422,26 @@ struct Search {
     const int is = (int)F.size() - 1;
     for (int t = 0; t < is; ++t)
       if (le_all(F[t], F[is]) && tie_le(j, t, is)) { F.pop_back(); return; }
-    std::vector<State> keep;
-    keep.reserve(F.size());
-    for (int t = 0; t < is; ++t)
-      if (!(le_all(F[is], F[t]) && tie_le(j, is, t))) keep.push_back(F[t]);
-    keep.push_back(F[is]);
-    F.swap(keep);
+    // drop the states the new one dominates (it stays last, at index w)
+    int w = 0;
+    for (int t = 0; t < is; ++t) {
+      if (le_all(F[is], F[t]) && tie_le(j, is, t)) continue;
+      if (w != t) F[w] = F[t];
+      ++w;
+    }
+    F[w] = F[is];
+    F.resize(w + 1);
   }
 
   State step(const State& s, const Block& B) const {
     State r{};
-    if (slots == 2) {
-      const int64_t C = std::max(s.v[0], s.v[2]) + B.t_in;
-      const int64_t E = std::max(s.v[1], C) + B.t_ex;
-      r.v[0] = C; r.v[1] = E; r.v[2] = s.v[3]; r.v[3] = E + B.t_out;
-    } else {
-      const int64_t C = std::max(s.v[0], s.v[2]) + B.t_in;
-      const int64_t E = std::max(s.v[1], C) + B.t_ex;
-      r.v[0] = C; r.v[1] = E; r.v[2] = E + B.t_out; r.v[3] = 0;
-    }
-    r.v[4] = slots == 2 ? (int64_t)B.bytes : 0;
+    const int64_t C = s.v[0] + B.t_in;
+    const int64_t E = std::max(s.v[1], C) + B.t_ex;
+    const int64_t R = E + B.t_out;
+    r.v[0] = slots == 2 ? std::max(C, s.v[2]) : std::max(C, R);
+    r.v[1] = E;
+    r.v[2] = R;
+    r.v[3] = slots == 2 ? (int64_t)B.bytes : 0;
     r.nblocks = s.nblocks + 1;
     return r;
   }
@@ -392,25 +449,92 @@ struct Search {
 
 }  // namespace
 
-static int search_pipeline(swapnet_plan* p, std::vector<uint32_t>* best_cuts) {
+// A feasible plan for an upper bound: consecutive units packed into blocks
+// of at most half the arena (any two such neighbours fit together).
+static int64_t greedy_upper_bound(const swapnet_plan* p) {
   const int U = (int)p->units.size();
+  const uint64_t cap = p->opt.slots == 2 ? p->region / 2 : p->region;
+  std::vector<Block> bl;
+  for (int j = 0; j < U;) {
+    uint64_t bytes = 0;
+    int j2 = j;
+    while (j2 < U && bytes + p->units[j2].bytes <= cap) bytes += p->units[j2++].bytes;
+    if (j2 == j) j2 = j + 1;  // one unit larger than the cap: a block of its own
+    Block B = make_block(p->units, j, j2, p->opt);
+    if (!pair_ok(p, bl.empty() ? 0 : bl.back().bytes, B.bytes)) return INT64_MAX;
+    bl.push_back(B);
+    j = j2;
+  }
+  return pipeline_ns(bl, p->opt.slots);
+}
+
+// Exact search over cut vectors: a Pareto front of pipeline states per unit
+// boundary, pruned by dominance and by a bound.  A state at boundary j that
+// next copies no earlier than a (and has executed up to E) finishes no
+// earlier than max(E + remaining t_ex, a + remaining t_in + t_ex of the last
+// unit), since copies and executions each form a chain; states whose bound
+// exceeds the best finish found (or a greedy plan's) cannot win.
+static int search_pipeline_capped(swapnet_plan* p, std::vector<uint32_t>* best_cuts, size_t cap,
+                                  int64_t ub_in, int64_t* best_ns, bool* exact) {
+  const int U = (int)p->units.size();
+  std::vector<int64_t> rem_ex(U + 1, 0), rem_in(U + 1, 0);
+  {
+    uint64_t bytes = 0, depth = 0;
+    for (int j = U - 1; j >= 0; --j) {
+      rem_ex[j] = rem_ex[j + 1] + p->units[j].t_ex;
+      bytes += p->units[j].bytes;
+      depth += p->units[j].depth;
+      rem_in[j] = (int64_t)mul_div_ceil(p->opt.alpha_as_per_byte, bytes, 1000000000ull) +
+                  (int64_t)(p->opt.beta_ns_per_tensor * depth);
+    }
+  }
+  const int64_t last_ex = U ? p->units[U - 1].t_ex : 0;
+  int64_t ub = std::min(ub_in, greedy_upper_bound(p));
+  auto bound = [&](const State& c, int j) -> int64_t {
+    if (j == U) return c.v[1];
+    return std::max(c.v[1] + rem_ex[j], c.v[0] + rem_in[j] + last_ex);
+  };
   Search S(p->units, p->opt, p->slot);
   S.front.assign(U + 1, {});
   State s0{};
   s0.prev_j = -1; s0.prev_idx = -1; s0.nblocks = 0;
   S.front[0].push_back(s0);
-  // frontier states of boundary j only get children once j is final
+  // frontier states of boundary j only get children once j is final; a
+  // frontier wider than kFrontCap keeps its kFrontCap states of smallest
+  // bound (the result is then the best plan found, not a proven optimum)
+  *exact = true;
   for (int j = 0; j < U; ++j) {
-    // rebuild the frontier list copy, since insert() on j' > j does not touch it
+    std::vector<State>& Fj = S.front[j];
+    if (Fj.size() > cap) {
+      std::vector<std::pair<std::pair<int64_t, int64_t>, size_t>> key(Fj.size());
+      for (size_t i = 0; i < Fj.size(); ++i) key[i] = {{bound(Fj[i], j), Fj[i].v[1]}, i};
+      std::nth_element(key.begin(), key.begin() + cap, key.end());
+      std::sort(key.begin(), key.begin() + cap, [](const auto& x, const auto& y) { return x.second < y.second; });
+      std::vector<State> kept;
+      kept.reserve(cap);
+      for (size_t i = 0; i < cap; ++i) kept.push_back(Fj[key[i].second]);
+      Fj.swap(kept);
+      *exact = false;
+    }
     for (int idx = 0; idx < (int)S.front[j].size(); ++idx) {
-      uint64_t bytes = 0;
-      const uint64_t prev = (uint64_t)S.front[j][idx].v[4];
+      if (bound(S.front[j][idx], j) > ub) continue;
+      const uint64_t prev = (uint64_t)S.front[j][idx].v[3];
+      Block B{};  // grown one unit at a time: units [j, j2)
+      B.u0 = j;
       for (int j2 = j + 1; j2 <= U; ++j2) {
-        bytes += p->units[j2 - 1].bytes;
-        if (!pair_ok(p, prev, bytes)) break;
-        Block B = make_block(p->units, j, j2, p->opt);
+        const Unit& un = p->units[j2 - 1];
+        B.u1 = j2;
+        B.bytes += un.bytes;
+        B.depth += un.depth;
+        B.t_ex += un.t_ex;
+        if (!pair_ok(p, prev, B.bytes)) break;
+        B.t_in = (int64_t)mul_div_ceil(p->opt.alpha_as_per_byte, B.bytes, 1000000000ull) +
+                 (int64_t)(p->opt.beta_ns_per_tensor * B.depth);
+        B.t_out = (int64_t)(p->opt.eta_ns_per_tensor * B.depth);
         State c = S.step(S.front[j][idx], B);
         c.prev_j = j; c.prev_idx = idx;
+        if (bound(c, j2) > ub) continue;
+        if (j2 == U) ub = std::min(ub, c.v[1]);
         S.insert(j2, c);
       }
     }
@@ -424,6 +548,29 @@ static int search_pipeline(swapnet_plan* p, std::vector<uint32_t>* best_cuts) {
       best = i;
   }
   *best_cuts = S.cuts_of(U, best);
+  *best_ns = F[best].v[1];
+  return SWAPNET_OK;
+}
+
+// A narrow beam first finds a good plan; its finish time then bounds the
+// full search, which prunes every state that cannot reach it.  States
+// whose bound equals it are kept, so ties are still broken exactly.
+static int search_pipeline(swapnet_plan* p, std::vector<uint32_t>* best_cuts) {
+  std::vector<uint32_t> beam_cuts;
+  int64_t beam_ns = INT64_MAX;
+  bool beam_exact = false;
+  int rc = search_pipeline_capped(p, &beam_cuts, 32, INT64_MAX, &beam_ns, &beam_exact);
+  if (rc) return rc;
+  if (beam_exact) {
+    p->exact = true;
+    *best_cuts = beam_cuts;
+    return SWAPNET_OK;
+  }
+  int64_t ns = 0;
+  bool exact = false;
+  rc = search_pipeline_capped(p, best_cuts, 4096, beam_ns, &ns, &exact);
+  if (rc) return rc;
+  p->exact = exact;
   return SWAPNET_OK;
 }
 
@@ -593,6 +740,8 @@ int swapnet_plan_info_get(const swapnet_plan* p, swapnet_plan_info* info) {
   r.plan_bytes = sizeof(swapnet_plan) + p->units.size() * sizeof(Unit) + p->blocks.size() * sizeof(Block) +
                  p->model.L.size() * sizeof(Layer) + p->cuts.size() * sizeof(uint32_t);
   r.predicted_ns = p->predicted;
+  r.state_bytes = p->model.state_bytes;
+  r.exact = p->exact ? 1 : 0;
   *info = r;
   return SWAPNET_OK;
 }

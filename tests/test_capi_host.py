@@ -112,9 +112,12 @@ def test_partition_eq4_objective_equals_oracle():
         assert plan.cuts() == ref["cuts"] and plan.info()["predicted_ns"] == ref["predicted_ns"]
 
 
-@pytest.mark.parametrize("name", ["mlp6", "resnet50", "vgg16", "yolov3"])
+@pytest.mark.parametrize("name", ["mlp6", "resnet50", "vgg16", "yolov3", "llm_small", "llm"])
 def test_units_workspace_match_oracle(name):
-    m = synth.arch.MODELS[name]()
+    if name == "llm_small":
+        m = synth.arch.llm(layers=2, d=256, heads=2, ffn=688, vocab=1000, tokens=64, max_seq=80)
+    else:
+        m = synth.arch.MODELS[name]()
     wb = P.weight_bytes(m)
     opt = capi.options()
     budget = wb * 3 // 10 // 256 * 256
