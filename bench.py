@@ -44,6 +44,10 @@ CONFIGS = {
              "6-layer MLP width 1024 fp32 batch 8, budget = 2 layers of weights + 2 activation buffers"),
     "vgg16_b1": ("vgg16", dict(batch=1), 0.25, "VGG-16-shaped CNN, fp16, batch 1, budget 25% of weight bytes"),
     "vgg16_b16": ("vgg16", dict(batch=16), 0.25, "VGG-16-shaped CNN, fp16, batch 16, budget 25% of weight bytes"),
+    "yolov3": ("yolov3", dict(batch=1), 0.30, "YOLOv3 (Darknet-53 + 3 heads), fp16, 1x3x416x416, budget 30%"),
+    "llm": ("llm", dict(tokens=512), None,
+            "LLaMA-7B-shaped decoder bf16 (32 layers, d 4096, 32 heads, FFN 11008, vocab 32000); "
+            "prefill 512 token ids + 32 greedy decode steps, batch 1; 4e9-byte weight arena"),
 }
 
 
@@ -159,9 +163,207 @@ def build_workload(name):
     return m, w, x, wb, budget, text
 
 
+def llm_host_weights(model, threads=16):
+    """The 7B weights generated in parallel straight into the packed buffer."""
+    import concurrent.futures as cf
+    import synth
+    from paper_2401_16757_gb300 import capi
+    jobs, sizes = [], []
+    for li, L in enumerate(model["layers"]):
+        for ti, (_, shp) in enumerate(synth.arch.tensor_shapes(L)):
+            jobs.append((li, ti, shp))
+            sizes.append(int(np.prod(shp)) * 2)
+    host = capi.HostWeights.allocate(sizes)
+
+    def fill(k):
+        li, ti, shp = jobs[k]
+        host.view(k)[:] = synth.gen.llm_tensor(model, li, ti, shp).view(np.uint8).reshape(-1)
+
+    with cf.ThreadPoolExecutor(threads) as ex:
+        list(ex.map(fill, range(len(jobs))))
+    return host
+
+
+def llm_cpu_sample(n_dec_sample=2):
+    """The float64 oracle on a bounded sample of the 7B workload: a model of
+    the same widths with ONE decoder layer runs the 512-token prefill and
+    n_dec_sample decode tokens; the embedding, layer and head parts are timed
+    separately and scaled to 32 layers and 32 decode tokens.  Returns
+    (seconds per whole inference, description)."""
+    import synth
+    from oracle import forward as F
+    m1 = synth.arch.llm(layers=1, tokens=512)
+    w = synth.gen.model_weights(m1)
+    ids = synth.gen.model_input(m1)
+    state = F.new_state()
+    nl = len(m1["layers"])
+
+    def parts(x):
+        acts, t = {}, []
+        for lo, hi in ((0, 1), (1, nl - 3), (nl - 3, nl)):
+            t0 = time.perf_counter()
+            F.forward_range(m1, w, acts, np.asarray(x), lo, hi, state)
+            t.append(time.perf_counter() - t0)
+        state["pos"] += int(np.asarray(x).shape[0])
+        return t, int(acts[nl - 1].reshape(-1)[-1])
+
+    tp, tok = parts(ids)
+    td = [0.0, 0.0, 0.0]
+    for _ in range(n_dec_sample):
+        t, tok = parts(np.array([[[[tok]]]], dtype=np.int32))
+        td = [a + b for a, b in zip(td, t)]
+    per_dec = [v / n_dec_sample for v in td]
+    total = (tp[0] + 32 * tp[1] + tp[2]) + 32 * (per_dec[0] + 32 * per_dec[1] + per_dec[2])
+    return total, ("float64 oracle, one 4096-wide decoder layer (+ embedding and LM head) over the 512-token "
+                   "prefill and %d decode tokens, scaled to 32 layers and 32 decode tokens" % n_dec_sample)
+
+
+def run_llm(args, rank, world):
+    """Config 5: prefill of 512 ids then 32 greedy decode steps per step."""
+    import torch
+    import synth
+    from oracle import plan as OP
+    from paper_2401_16757_gb300 import capi
+    text = CONFIGS["llm"][3]
+    t0 = time.perf_counter()
+    mp, md = synth.arch.llm(tokens=512), synth.arch.llm(tokens=1)
+    host = llm_host_weights(mp)
+    t_gen = time.perf_counter() - t0
+    stream = torch.cuda.current_stream()
+    sp = stream.cuda_stream
+    link_peak = measure_link_peak(stream)
+    alpha = int(round(1e18 / (link_peak * 1e9)))
+    budget = 4_000_000_000
+    variant = {"auto": capi.SWAP_AUTO, "memcpy": capi.SWAP_MEMCPY, "zerocopy": capi.SWAP_ZEROCOPY}[args.variant]
+    opt = capi.options(swap_variant=variant, alpha_as_per_byte=alpha, beta_ns_per_tensor=0)
+    dp, dd = capi.Desc(mp), capi.Desc(md)
+    t1 = time.perf_counter()
+    pp, pd = capi.Plan.partition(dp, budget, opt), capi.Plan.partition(dd, budget, opt)
+    t_plan = time.perf_counter() - t1
+    ip, idd = pp.info(), pd.info()
+    ep, ed = capi.Engine(pp, host), capi.Engine(pd, host)
+    rpp = capi.Plan.resident(dp)
+    arena = torch.empty(rpp.info()["arena_bytes"], dtype=torch.uint8, device="cuda")
+    rp = capi.Engine(rpp, host, d_arena=arena.data_ptr(), arena_bytes=arena.numel())
+    rd = capi.Engine(capi.Plan.resident(dd, capi.options(preloaded=1)), host, d_arena=arena.data_ptr(),
+                     arena_bytes=arena.numel())
+    state = torch.zeros(ip["state_bytes"], dtype=torch.uint8, device="cuda")
+    for e in (ep, ed, rp, rd):
+        e.bind_state(state.data_ptr(), ip["state_bytes"])
+    ids = synth.gen.model_input(mp).reshape(-1)
+    in_p = torch.from_numpy(ids.view(np.uint8).copy()).cuda()
+    out_p = torch.zeros(ip["output_bytes"], dtype=torch.uint8, device="cuda")
+    tok = torch.zeros(16, dtype=torch.uint8, device="cuda")
+    out_d = torch.zeros(idd["output_bytes"], dtype=torch.uint8, device="cuda")
+    offs_p, offs_d = pp.output_offsets(), pd.output_offsets()
+    n_dec = 32
+
+    def one(eng_p, eng_d, evs=None):
+        state[:256].zero_()
+        if evs: evs[0].record(stream)
+        eng_p.infer(in_p.data_ptr(), out_p.data_ptr(), sp)
+        if evs: evs[1].record(stream)
+        tok[:4].copy_(out_p[offs_p[1] + 511 * 4:offs_p[1] + 512 * 4])
+        for _ in range(n_dec):
+            eng_d.infer(tok.data_ptr(), out_d.data_ptr(), sp)
+            tok[:4].copy_(out_d[offs_d[1]:offs_d[1] + 4])
+        if evs: evs[2].record(stream)
+
+    def timed(eng_p, eng_d, steps):
+        res = []
+        for _ in range(steps):
+            evs = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+            one(eng_p, eng_d, evs)
+            torch.cuda.synchronize()
+            res.append((evs[0].elapsed_time(evs[1]), evs[1].elapsed_time(evs[2]) / n_dec))
+        return res
+
+    for _ in range(max(1, args.warmup)):
+        one(ep, ed)
+        one(rp, rd)
+    torch.cuda.synchronize()
+    for e in (ep, ed, rp, rd):
+        e.sync()
+    clocks = ClockSampler(int(os.environ.get("LOCAL_RANK", "0")))
+    clocks.start()
+    launches0 = ep.stats()["kernel_launches"] + ed.stats()["kernel_launches"]
+    sw = timed(ep, ed, args.steps)
+    launches = ep.stats()["kernel_launches"] + ed.stats()["kernel_launches"] - launches0
+    di = timed(rp, rd, args.steps)
+    clk = clocks.stop()
+    # greedy tokens agree between swapped and resident runs
+    one(ep, ed); torch.cuda.synchronize(); sw_tok = int(tok[:4].cpu().numpy().view(np.int32)[0])
+    one(rp, rd); torch.cuda.synchronize(); rs_tok = int(tok[:4].cpu().numpy().view(np.int32)[0])
+    pre_ms = statistics.mean(r[0] for r in sw)
+    dec_ms = statistics.mean(r[1] for r in sw)
+    pre_d = statistics.mean(r[0] for r in di)
+    dec_d = statistics.mean(r[1] for r in di)
+    step_ms = pre_ms + n_dec * dec_ms
+    dinf_ms = pre_d + n_dec * dec_d
+    swap_bytes_p = sum(b["bytes"] for b in pp.blocks())
+    swap_bytes_d = sum(b["bytes"] for b in pd.blocks())
+    bytes_step = swap_bytes_p + n_dec * swap_bytes_d
+    bound_ms = bytes_step / (link_peak * 1e9) * 1e3
+    line = {
+        "metric": METRIC, "value": world * 1000.0 / step_ms, "unit": "inferences/s (prefill 512 + 32 decode)",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": text, "budget_bytes": budget, "weight_bytes": ip["weight_bytes"],
+                   "prefill_blocks": ip["n_blocks"], "decode_blocks": idd["n_blocks"],
+                   "plans_exact": [ip["exact"], idd["exact"]], "l2": "inputs (13.2 GB of weights) larger than L2",
+                   "swap_variant": args.variant, "state_bytes": ip["state_bytes"]},
+        "prefill_ms": pre_ms, "decode_ms_per_token": dec_ms, "dinf_prefill_ms": pre_d,
+        "dinf_decode_ms_per_token": dec_d, "dinf_ms": dinf_ms, "ratio": step_ms / dinf_ms,
+        "greedy_token_swapped_equals_resident": sw_tok == rs_tok,
+        "link": {"achieved_gbs": bytes_step / (step_ms * 1e-3) / 1e9, "peak_gbs": link_peak,
+                 "peak_source": "pinned cudaMemcpy H2D 256 MiB", "bytes_per_step": bytes_step},
+        "step_roofline": {"bound": "host link", "bound_ms": bound_ms, "frac": bound_ms / step_ms},
+        "gpu_launches": launches, "clocks": clk,
+        "setup_s": {"weights": t_gen, "plans": t_plan},
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        tot, sample = llm_cpu_sample()
+        line["cpu_baseline"] = {"value": 1.0 / tot, "unit": "inferences/s", "cores": len(os.sched_getaffinity(0)),
+                                "kind": "oracle", "sample": sample}
+    if rank == 0:
+        print(json.dumps(line))
+
+
+def measure_link_peak(stream):
+    import torch
+    pk = torch.empty(256 << 20, dtype=torch.uint8, pin_memory=True)
+    dv = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    best = 1e9
+    for _ in range(5):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        dv.copy_(pk, non_blocking=True)
+        b.record(stream)
+        b.synchronize()
+        best = min(best, a.elapsed_time(b))
+    return (256 << 20) / (best / 1000.0) / 1e9
+
+
 def run_reference(args, rank, world):
     """The reference arm: the CPU oracle, timed as it stands on the host cores."""
     if rank != 0:
+        return
+    if args.config == "llm":
+        cores = len(os.sched_getaffinity(0))
+        llm_cpu_sample(1)
+        times = [llm_cpu_sample()[0] for _ in range(args.steps)]
+        ms = 1000.0 * sum(times) / len(times)
+        val = 1000.0 / ms
+        sample = llm_cpu_sample.__doc__.split("Returns")[0].strip()
+        print(json.dumps({
+            "impl": "reference", "metric": METRIC, "value": val, "unit": "inferences/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": CONFIGS["llm"][3], "budget_bytes": 4_000_000_000, "l2": "n/a (CPU)"},
+            "cpu_baseline": {"value": val, "unit": "inferences/s", "cores": cores, "kind": "oracle",
+                             "sample": " ".join(sample.split())},
+            "e2e": {"value": val, "unit": "inferences/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        }))
         return
     m, w, x, wb, budget, text = build_workload(args.config)
     from oracle import forward as F
@@ -203,6 +405,13 @@ def main():
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
         run_reference(args, rank, world)
+        return
+    if args.config == "llm":
+        import torch
+        torch.cuda.set_device(local)
+        import __graft_entry__
+        __graft_entry__.build()
+        run_llm(args, rank, world)
         return
 
     import torch

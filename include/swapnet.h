@@ -146,7 +146,10 @@ typedef struct swapnet_options {
   int32_t graphs;                /* 1 (default): each (input, output) binding of an
                                     engine is captured once as a CUDA graph and
                                     replayed; 0: launch eagerly every call      */
-  int32_t reserved[6];
+  int32_t preloaded;             /* resident plans only: the caller's arena already
+                                    holds this layout (loaded by another engine of
+                                    the same layers); swapnet_load skips the upload */
+  int32_t reserved[5];
 } swapnet_options;
 
 /* Fills the defaults: 2 slots, activations outside the budget, AUTO swap,

@@ -45,7 +45,7 @@ class Options(C.Structure):
     _fields_ = [("slots", C.c_int32), ("activations_in_budget", C.c_int32), ("swap_variant", C.c_int32),
                 ("objective", C.c_int32), ("alpha_as_per_byte", C.c_uint64), ("beta_ns_per_tensor", C.c_uint64),
                 ("gamma_as_per_flop", C.c_uint64), ("eta_ns_per_tensor", C.c_uint64), ("zc_ctas", C.c_int32),
-                ("graphs", C.c_int32), ("reserved", C.c_int32 * 6)]
+                ("graphs", C.c_int32), ("preloaded", C.c_int32), ("reserved", C.c_int32 * 5)]
 
 
 class PlanInfo(C.Structure):
@@ -333,6 +333,30 @@ class HostWeights:
     buffer, each tensor at a 256-byte aligned offset in layer order (the
     layout of the arena slots, so a block's tensors are one contiguous
     range)."""
+
+    @classmethod
+    def allocate(cls, nbytes_list):
+        """An uninitialised packed buffer for tensors of the given sizes;
+        fill tensor i through view(i)."""
+        self = cls.__new__(cls)
+        offs, cur = [], 0
+        for n in nbytes_list:
+            offs.append(cur)
+            cur += (n + 255) // 256 * 256
+        page = os.sysconf("SC_PAGE_SIZE")
+        raw = np.empty(cur + 2 * page, dtype=np.uint8)
+        start = (-raw.ctypes.data) % page
+        self._raw = raw
+        self.buf = raw[start:start + cur]
+        self._offs, self._sizes = offs, list(nbytes_list)
+        base = self.buf.ctypes.data
+        self.ptrs = (C.c_void_p * max(1, len(offs)))(*[base + o for o in offs])
+        self.n = len(offs)
+        self.nbytes = cur
+        return self
+
+    def view(self, i):
+        return self.buf[self._offs[i]:self._offs[i] + self._sizes[i]]
 
     def __init__(self, weights, buffer=None):
         """buffer: optional caller-provided uint8 array (e.g. already pinned)

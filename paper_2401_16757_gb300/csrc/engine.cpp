@@ -574,9 +574,11 @@ int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint
   }
   const int variant = plan->opt.swap_variant;
   if (plan->resident) {
-    for (size_t k = 0; k < e->blocks.size() && !rc; ++k) rc = swap_block(e, k, SWAPNET_SWAP_MEMCPY, e->copy);
-    if (rc) return rc;
-    CU(cudaStreamSynchronize(e->copy), "resident upload");
+    if (!(plan->opt.preloaded && d_arena)) {
+      for (size_t k = 0; k < e->blocks.size() && !rc; ++k) rc = swap_block(e, k, SWAPNET_SWAP_MEMCPY, e->copy);
+      if (rc) return rc;
+      CU(cudaStreamSynchronize(e->copy), "resident upload");
+    }
     e->weights_loaded = true;
   } else if (variant == SWAPNET_SWAP_AUTO) {
     rc = calibrate(e);

@@ -611,6 +611,7 @@ static int check_options(const swapnet_options& o) {
   if (o.swap_variant < 0 || o.swap_variant > 2) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad swap_variant");
   if (o.zc_ctas < 0 || o.zc_ctas > 4096) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad zc_ctas");
   if (o.graphs != 0 && o.graphs != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "graphs must be 0 or 1");
+  if (o.preloaded != 0 && o.preloaded != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "preloaded must be 0 or 1");
   return SWAPNET_OK;
 }
 
