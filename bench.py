@@ -284,6 +284,7 @@ def run_llm(args, rank, world):
     torch.cuda.synchronize()
     for e in (ep, ed, rp, rd):
         e.sync()
+    link_before = measure_link_peak(stream)
     clocks = ClockSampler(int(os.environ.get("LOCAL_RANK", "0")))
     clocks.start()
     launches0 = ep.stats()["kernel_launches"] + ed.stats()["kernel_launches"]
@@ -291,6 +292,7 @@ def run_llm(args, rank, world):
     launches = ep.stats()["kernel_launches"] + ed.stats()["kernel_launches"] - launches0
     di = timed(rp, rd, args.steps)
     clk = clocks.stop()
+    link_after = measure_link_peak(stream)
     # greedy tokens agree between swapped and resident runs
     one(ep, ed); torch.cuda.synchronize(); sw_tok = int(tok[:4].cpu().numpy().view(np.int32)[0])
     one(rp, rd); torch.cuda.synchronize(); rs_tok = int(tok[:4].cpu().numpy().view(np.int32)[0])
@@ -316,7 +318,10 @@ def run_llm(args, rank, world):
         "dinf_decode_ms_per_token": dec_d, "dinf_ms": dinf_ms, "ratio": step_ms / dinf_ms,
         "greedy_token_swapped_equals_resident": sw_tok == rs_tok,
         "link": {"achieved_gbs": bytes_step / (step_ms * 1e-3) / 1e9, "peak_gbs": link_peak,
-                 "peak_source": "pinned cudaMemcpy H2D 256 MiB", "bytes_per_step": bytes_step},
+                 "peak_source": "pinned cudaMemcpy H2D 256 MiB", "bytes_per_step": bytes_step,
+                 "peak_before_after_gbs": [link_before, link_after]},
+        "per_step": {"prefill_ms": [r[0] for r in sw], "decode_ms_per_token": [r[1] for r in sw],
+                     "dinf_prefill_ms": [r[0] for r in di], "dinf_decode_ms_per_token": [r[1] for r in di]},
         "step_roofline": {"bound": "host link", "bound_ms": bound_ms, "frac": bound_ms / step_ms},
         "gpu_launches": launches, "clocks": clk,
         "setup_s": {"weights": t_gen, "plans": t_plan},

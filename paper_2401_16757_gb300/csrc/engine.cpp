@@ -527,6 +527,9 @@ int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint
       SN_FAIL(SWAPNET_ERR_OOM, "arena allocation failed");
     }
     e->own_arena = true;
+    // touch every page now, so that the first inference does not pay for
+    // the driver backing fresh allocations
+    CU(cudaMemset(e->d_arena, 0, std::max<uint64_t>(arena_need, kAlign)), "arena first touch");
   }
   if (d_workspace || plan->model.ws_bytes == 0) {
     e->d_ws = static_cast<char*>(d_workspace);
@@ -537,6 +540,7 @@ int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint
       SN_FAIL(SWAPNET_ERR_OOM, "workspace allocation failed");
     }
     e->own_ws = true;
+    CU(cudaMemset(e->d_ws, 0, plan->model.ws_bytes), "workspace first touch");
   }
   if (injected(3)) SN_FAIL(SWAPNET_ERR_CUDA, "stream creation failed (injected)");
   int lo = 0, hi = 0;

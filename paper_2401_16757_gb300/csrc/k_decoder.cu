@@ -118,58 +118,123 @@ __global__ void __launch_bounds__(256) rope_append_kernel(T* __restrict__ q, con
 }
 
 // ------------------------------------------------------------ attention
-// Warp = one (query, head); each lane holds 4 of the 128 head dimensions.
-// Keys are visited in position order with an online softmax in fp32:
-// m (running max), l (running denominator), acc (running numerator).
+// CTA = one (query t, head h), 512 threads; the scores of all visible keys
+// live in shared memory, so the softmax is exact two-pass (max, then
+// exponentials and their sum) rather than online:
+//   phase 1: thread j computes key j's score (the whole 128-wide dot product
+//            from 16 independent 16-byte loads of its cache row);
+//   phase 2: block max, p_j = exp(s_j - max), block sum l in a fixed order;
+//   phase 3: thread (pair d, group g) accumulates p_j * v_j[2d..2d+1] over
+//            keys j = g, g + 8, ... (coalesced 4-byte loads along the row);
+//            the 8 groups are added in index order and divided by l.
+// Every key load of a phase is independent of the others, so a decode step
+// (one query, keys in HBM) is bound by a few memory round trips, not by a
+// chain of one round trip per key.
 constexpr int kDh = 128;
+constexpr int kAttThreads = 512;
+constexpr int kAttGroups = kAttThreads / (kDh / 2);
 
-template <typename T>
-__device__ __forceinline__ void load4(const T* p, float* f) {
-  const uint2 u = *reinterpret_cast<const uint2*>(p);
-  const T* e = reinterpret_cast<const T*>(&u);
+__device__ __forceinline__ float block_reduce(float v, float* red, bool is_max) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 #pragma unroll
-  for (int j = 0; j < 4; ++j) f[j] = to_f<T>(e[j]);
+  for (int off = 16; off > 0; off >>= 1) {
+    const float o = __shfl_xor_sync(0xffffffffu, v, off);
+    v = is_max ? fmaxf(v, o) : v + o;
+  }
+  __syncthreads();  // red is reused between calls
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  float r = red[0];
+  for (int w = 1; w < kAttThreads / 32; ++w) r = is_max ? fmaxf(r, red[w]) : r + red[w];
+  return r;
 }
 
 template <typename T>
-__global__ void __launch_bounds__(256) attention_kernel(const T* __restrict__ q, const T* __restrict__ kc,
-                                                        const T* __restrict__ vc, const int* __restrict__ pos_ptr,
-                                                        int T_, int heads, int width, int max_seq,
-                                                        T* __restrict__ out) {
+__global__ void __launch_bounds__(kAttThreads) attention_kernel(const T* __restrict__ q, const T* __restrict__ kc,
+                                                                const T* __restrict__ vc,
+                                                                const int* __restrict__ pos_ptr, int heads,
+                                                                int width, int max_seq, T* __restrict__ out) {
+  extern __shared__ float att_smem[];
+  float2* part = reinterpret_cast<float2*>(att_smem);          // kAttGroups x kDh/2 partial sums
+  float* red = att_smem + 2 * kAttGroups * (kDh / 2);          // kAttThreads / 32 partials
+  float* qs = red + kAttThreads / 32;                          // kDh query values
+  float* sc = qs + kDh;                                        // max_seq scores
   pdl_wait();
   pdl_launch_dependents();
-  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  if (warp >= T_ * heads) return;
-  const int t = warp / heads, h = warp % heads;
-  const int pos = *pos_ptr + t;
-  const int n = min(pos + 1, max_seq);
-  const int c0 = h * kDh + lane * 4;
-  float qv[4];
-  load4<T>(q + (int64_t)t * width + c0, qv);
+  const int h = blockIdx.x, t = blockIdx.y;
+  const int tid = threadIdx.x;
+  const int n = min(*pos_ptr + t + 1, max_seq);
+  const int64_t col = (int64_t)h * kDh;
+  if (tid < kDh) qs[tid] = to_f<T>(q[(int64_t)t * width + col + tid]);
+  __syncthreads();
   const float scale = rsqrtf((float)kDh);
-  float m = -INFINITY, l = 0.f, acc[4] = {0.f, 0.f, 0.f, 0.f};
-  for (int j = 0; j < n; ++j) {
-    float kv[4];
-    load4<T>(kc + (int64_t)j * width + c0, kv);
-    float s = qv[0] * kv[0] + qv[1] * kv[1] + qv[2] * kv[2] + qv[3] * kv[3];
+  float mx = -INFINITY;
+  for (int j = tid; j < n; j += kAttThreads) {
+    const uint4* kr = reinterpret_cast<const uint4*>(kc + (int64_t)j * width + col);
+    uint4 u[kDh / 8];
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+    for (int i = 0; i < kDh / 8; ++i) u[i] = kr[i];
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < kDh / 8; ++i) {
+      const T* e = reinterpret_cast<const T*>(&u[i]);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) s = fmaf(qs[i * 8 + k], to_f<T>(e[k]), s);
+    }
     s *= scale;
-    const float mn = fmaxf(m, s);
-    const float a = expf(m - mn);   // 0 on the first key (m = -inf)
-    const float p = expf(s - mn);
-    float vv[4];
-    load4<T>(vc + (int64_t)j * width + c0, vv);
-    l = l * a + p;
-#pragma unroll
-    for (int d = 0; d < 4; ++d) acc[d] = acc[d] * a + p * vv[d];
-    m = mn;
+    sc[j] = s;
+    mx = fmaxf(mx, s);
   }
-  const float inv = 1.0f / l;
-  T* o = out + (int64_t)t * width + c0;
+  mx = block_reduce(mx, red, true);
+  float l = 0.f;
+  for (int j = tid; j < n; j += kAttThreads) {
+    const float p = expf(sc[j] - mx);
+    sc[j] = p;
+    l += p;
+  }
+  l = block_reduce(l, red, false);  // the barriers inside also publish sc[]
+  const int d2 = tid % (kDh / 2), g = tid / (kDh / 2);
+  const T* vcol = vc + col + 2 * d2;
+  float a0 = 0.f, a1 = 0.f;
+  int j = g;
+#pragma unroll 1
+  for (; j + 3 * kAttGroups < n; j += 4 * kAttGroups) {
+    uint32_t w[4];
 #pragma unroll
-  for (int d = 0; d < 4; ++d) o[d] = from_f<T>(acc[d] * inv);
+    for (int i = 0; i < 4; ++i) w[i] = *reinterpret_cast<const uint32_t*>(vcol + (int64_t)(j + i * kAttGroups) * width);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const T* e = reinterpret_cast<const T*>(&w[i]);
+      const float p = sc[j + i * kAttGroups];
+      a0 = fmaf(p, to_f<T>(e[0]), a0);
+      a1 = fmaf(p, to_f<T>(e[1]), a1);
+    }
+  }
+  for (; j < n; j += kAttGroups) {
+    const uint32_t w = *reinterpret_cast<const uint32_t*>(vcol + (int64_t)j * width);
+    const T* e = reinterpret_cast<const T*>(&w);
+    const float p = sc[j];
+    a0 = fmaf(p, to_f<T>(e[0]), a0);
+    a1 = fmaf(p, to_f<T>(e[1]), a1);
+  }
+  part[g * (kDh / 2) + d2] = make_float2(a0, a1);
+  __syncthreads();
+  if (tid < kDh / 2) {
+    float o0 = 0.f, o1 = 0.f;
+    for (int gg = 0; gg < kAttGroups; ++gg) {
+      const float2 v = part[gg * (kDh / 2) + tid];
+      o0 += v.x;
+      o1 += v.y;
+    }
+    const float inv = 1.0f / l;
+    T* o = out + (int64_t)t * width + col + 2 * tid;
+    o[0] = from_f<T>(o0 * inv);
+    o[1] = from_f<T>(o1 * inv);
+  }
+}
+
+size_t attention_smem_bytes(int max_seq) {
+  return sizeof(float) * ((size_t)max_seq + kDh + kAttThreads / 32) + sizeof(float2) * kAttGroups * (kDh / 2);
 }
 
 // ------------------------------------------------------------ argmax
@@ -246,10 +311,15 @@ int launch_attention(int dtype, void* q, const void* k, const void* v, void* kc,
                              static_cast<T*>(vc), pos_ptr, width, kDh, theta, max_seq, err),
                   "rope launch");
     if (rc) return rc;
-    const int warps = tokens * heads;
-    return done(launch_pdl(attention_kernel<T>, dim3((warps * 32 + 255) / 256), dim3(256), 0, s,
+    const size_t smem = attention_smem_bytes(max_seq);
+    if (smem > 48 * 1024) {
+      cudaError_t e = cudaFuncSetAttribute(attention_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)smem);
+      if (e != cudaSuccess) return done(e, "attention shared memory");
+    }
+    return done(launch_pdl(attention_kernel<T>, dim3(heads, tokens), dim3(kAttThreads), smem, s,
                            static_cast<const T*>(q), static_cast<const T*>(kc), static_cast<const T*>(vc),
-                           pos_ptr, tokens, heads, width, max_seq, static_cast<T*>(out)),
+                           pos_ptr, heads, width, max_seq, static_cast<T*>(out)),
                 "attention launch");
   });
   return SWAPNET_OK;
