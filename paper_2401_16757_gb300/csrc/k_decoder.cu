@@ -118,7 +118,11 @@ __global__ void __launch_bounds__(256) rope_append_kernel(T* __restrict__ q, con
 }
 
 // ------------------------------------------------------------ attention
-// CTA = one (query t, head h), 512 threads; the scores of all visible keys
+// Two kernels with the same arithmetic definition; a call with fewer than
+// kRowsMinWarps (query, head) pairs (decode) takes the CTA kernel, longer
+// runs (prefill) the warp kernel.
+//
+// Short query runs: CTA = one (query t, head h), 512 threads; the scores of all visible keys
 // live in shared memory, so the softmax is exact two-pass (max, then
 // exponentials and their sum) rather than online:
 //   phase 1: thread j computes key j's score (the whole 128-wide dot product
@@ -133,6 +137,7 @@ __global__ void __launch_bounds__(256) rope_append_kernel(T* __restrict__ q, con
 constexpr int kDh = 128;
 constexpr int kAttThreads = 512;
 constexpr int kAttGroups = kAttThreads / (kDh / 2);
+constexpr int kRowsMinWarps = 1024;
 
 __device__ __forceinline__ float block_reduce(float v, float* red, bool is_max) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -233,6 +238,59 @@ __global__ void __launch_bounds__(kAttThreads) attention_kernel(const T* __restr
   }
 }
 
+// Long query runs (prefill): warp = one (query, head), each lane holding 4
+// of the 128 head dimensions; keys are visited in position order with an
+// online softmax in fp32 (m running max, l running denominator, acc running
+// numerator).  With hundreds of queries per head there are enough warps to
+// hide each warp's chain of one memory round trip per key.
+template <typename T>
+__device__ __forceinline__ void load4(const T* p, float* f) {
+  const uint2 u = *reinterpret_cast<const uint2*>(p);
+  const T* e = reinterpret_cast<const T*>(&u);
+#pragma unroll
+  for (int j = 0; j < 4; ++j) f[j] = to_f<T>(e[j]);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(256) attention_rows_kernel(const T* __restrict__ q, const T* __restrict__ kc,
+                                                             const T* __restrict__ vc,
+                                                             const int* __restrict__ pos_ptr, int T_, int heads,
+                                                             int width, int max_seq, T* __restrict__ out) {
+  pdl_wait();
+  pdl_launch_dependents();
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (warp >= T_ * heads) return;
+  const int t = warp / heads, h = warp % heads;
+  const int n = min(*pos_ptr + t + 1, max_seq);
+  const int c0 = h * kDh + lane * 4;
+  float qv[4];
+  load4<T>(q + (int64_t)t * width + c0, qv);
+  const float scale = rsqrtf((float)kDh);
+  float m = -INFINITY, l = 0.f, acc[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int j = 0; j < n; ++j) {
+    float kv[4];
+    load4<T>(kc + (int64_t)j * width + c0, kv);
+    float s = qv[0] * kv[0] + qv[1] * kv[1] + qv[2] * kv[2] + qv[3] * kv[3];
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+    s *= scale;
+    const float mn = fmaxf(m, s);
+    const float a = expf(m - mn);   // 0 on the first key (m = -inf)
+    const float p = expf(s - mn);
+    float vv[4];
+    load4<T>(vc + (int64_t)j * width + c0, vv);
+    l = l * a + p;
+#pragma unroll
+    for (int d = 0; d < 4; ++d) acc[d] = acc[d] * a + p * vv[d];
+    m = mn;
+  }
+  const float inv = 1.0f / l;
+  T* o = out + (int64_t)t * width + c0;
+#pragma unroll
+  for (int d = 0; d < 4; ++d) o[d] = from_f<T>(acc[d] * inv);
+}
+
 size_t attention_smem_bytes(int max_seq) {
   return sizeof(float) * ((size_t)max_seq + kDh + kAttThreads / 32) + sizeof(float2) * kAttGroups * (kDh / 2);
 }
@@ -311,6 +369,13 @@ int launch_attention(int dtype, void* q, const void* k, const void* v, void* kc,
                              static_cast<T*>(vc), pos_ptr, width, kDh, theta, max_seq, err),
                   "rope launch");
     if (rc) return rc;
+    if (tokens * heads >= kRowsMinWarps) {
+      const int warps = tokens * heads;
+      return done(launch_pdl(attention_rows_kernel<T>, dim3((warps * 32 + 255) / 256), dim3(256), 0, s,
+                             static_cast<const T*>(q), static_cast<const T*>(kc), static_cast<const T*>(vc),
+                             pos_ptr, tokens, heads, width, max_seq, static_cast<T*>(out)),
+                  "attention launch");
+    }
     const size_t smem = attention_smem_bytes(max_seq);
     if (smem > 48 * 1024) {
       cudaError_t e = cudaFuncSetAttribute(attention_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,

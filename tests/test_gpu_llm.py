@@ -14,22 +14,27 @@ pytestmark = pytest.mark.gpu
 
 SMALL = dict(layers=2, d=256, heads=2, ffn=688, vocab=1000, max_seq=80)
 
-# Relative-L2 bar per output tensor: 2e-3 for one decoder layer.  Deeper bf16
+# Relative-L2 bars.  Every layer, given the same stored inputs as the oracle
+# (local parity), is held to 2e-3 per output tensor.  End to end, bf16
 # chains saturate at the bf16 rounding noise: every stored bf16 tensor turns
 # an input discrepancy e into about sqrt(e * ulp) of flipped roundings, so
 # after a few chained rounding points GPU and oracle differ by about one bf16
 # ulp per element however exact each kernel is.  One ulp is between 2^-8 and
-# 2^-7 of the element it rounds, so the two-layer model is held to 2^-7.
+# 2^-7 of the element it rounds, so whole decoders are held to 2^-7 (the
+# small one-layer model happens to stay within 2e-3 and is held to that).
+LOCAL_TOL = 2e-3
 TOL = {1: 2e-3, 2: 2.0 ** -7}
+CHAIN_TOL = 2.0 ** -7
 
 
 class Decoder:
     """A prefill engine and a decode engine sharing weights and KV state."""
 
-    def __init__(self, prefill_tokens, budget_frac=0.5, resident=False, host=None, weights=None, layers=2):
+    def __init__(self, prefill_tokens, budget_frac=0.5, resident=False, host=None, weights=None, layers=2,
+                 **over):
         import torch
         self.torch = torch
-        cfg = dict(SMALL, layers=layers)
+        cfg = dict(SMALL, layers=layers, **over)
         self.mp = synth.arch.llm(tokens=prefill_tokens, **cfg)
         self.md = synth.arch.llm(tokens=1, **cfg)
         self.w = weights or synth.gen.model_weights(self.mp)
@@ -93,6 +98,89 @@ def test_llm_prefill_and_greedy_decode_teacher_forced(layers):
         _check_step(logits, toks, ref[0].reshape(1, -1), ref[1].reshape(-1), TOL[layers])
         tok = int(toks[0])
     assert int(dec.state[:4].cpu().numpy().view(np.int32)[0]) == 64 + 8
+
+
+WIDE = dict(layers=1, d=1024, heads=8, ffn=2752, max_seq=160)
+
+
+def test_llm_long_prefill_many_heads():
+    """128 queries x 8 heads: the prefill takes the warp-per-query attention
+    kernel, the decode steps after it the CTA-per-query kernel."""
+    dec = Decoder(prefill_tokens=128, **WIDE)
+    ids = synth.gen.model_input(dec.mp).reshape(-1)
+    st = F.new_state()
+    ref = F.forward(dec.mp, dec.w, ids.reshape(-1, 1, 1, 1), state=st)
+    logits, toks = dec.run(0, ids)
+    _check_step(logits, toks, ref[0].reshape(128, -1), ref[1].reshape(-1), CHAIN_TOL)
+    tok = int(toks[-1])
+    for step in range(4):
+        ref = F.forward(dec.md, dec.w, np.array([tok], dtype=np.int32).reshape(1, 1, 1, 1), state=st)
+        logits, toks = dec.run(1, np.array([tok], dtype=np.int32))
+        _check_step(logits, toks, ref[0].reshape(1, -1), ref[1].reshape(-1), CHAIN_TOL)
+        tok = int(toks[0])
+
+
+def test_llm_every_layer_local_parity():
+    """Each layer of a resident decoder whose every layer is a model output,
+    against the oracle layer run on the GPU's own stored inputs: prefill of
+    128 ids (warp-per-query attention) then two decode steps (CTA-per-query
+    attention), the oracle keeping its own KV cache built from the GPU's k
+    and v.  The q projection is rotated in place by the attention layer, so
+    attention takes the oracle's q computed from the GPU's normalised input."""
+    import torch
+    w = None
+    st_or = F.new_state()
+    state = None
+    for tokens in (128, 1, 1):
+        m = synth.arch.llm(tokens=tokens, vocab=SMALL["vocab"], **WIDE)
+        m = dict(m, outputs=list(range(len(m["layers"]))))
+        if w is None:
+            w = synth.gen.model_weights(m)
+            host = capi.HostWeights(w)
+            x = synth.gen.model_input(m)
+        else:
+            x = np.array([[[[next_tok]]]], dtype=np.int32)
+        plan = capi.Plan.resident(capi.Desc(m))
+        info = plan.info()
+        eng = capi.Engine(plan, host)
+        if state is None:
+            state = torch.zeros(info["state_bytes"], dtype=torch.uint8, device="cuda")
+        eng.bind_state(state.data_ptr(), info["state_bytes"])
+        din = torch.zeros(max(16, info["input_bytes"]), dtype=torch.uint8, device="cuda")
+        din[:x.nbytes].copy_(torch.from_numpy(x.view(np.uint8).reshape(-1)))
+        dout = torch.zeros(info["output_bytes"], dtype=torch.uint8, device="cuda")
+        eng.infer(din.data_ptr(), dout.data_ptr(), torch.cuda.current_stream().cuda_stream)
+        eng.sync()
+        hb = dout.cpu().numpy()
+        shapes = OP.out_shapes(m)
+        gpu = {}
+        for li, off in enumerate(plan.output_offsets()):
+            n = int(np.prod(shapes[li]))
+            if m["layers"][li]["op"] == "argmax":
+                gpu[li] = hb[off:off + 4 * n].view(np.int32).astype(np.float64).reshape(-1, 1, 1, 1)
+            else:
+                gpu[li] = F.decode(hb[off:off + 2 * n].view(np.uint16), "bf16").reshape(tokens, -1, 1, 1)
+        local = {}
+        for li, L in enumerate(m["layers"]):
+            acts = gpu
+            if L["op"] == "attention":
+                acts = dict(gpu)
+                acts[L["src"][0]] = local[L["src"][0]]
+            local[li] = F.run_layer(L, "bf16", w[li], acts, np.asarray(x), st_or, li)
+            att = [M for M in m["layers"] if M["op"] == "attention" and M["src"][0] == li]
+            if att:   # the stored q was rotated in place: compare with the oracle's rotated q
+                pos = np.arange(st_or["pos"], st_or["pos"] + tokens)
+                qr = F.round_as(F.rope(local[li].reshape(tokens, -1), pos, att[0]["heads"], att[0]["theta"]), "bf16")
+                e = rel_l2(gpu[li].ravel(), qr.ravel())
+                assert e <= LOCAL_TOL, (tokens, li, "rotated q", e)
+                continue
+            if L["op"] == "argmax":   # the GPU's logits decide: exact, ties to the lowest index
+                assert np.array_equal(gpu[li].ravel(), local[li].ravel()), li
+                continue
+            e = rel_l2(gpu[li].ravel(), local[li].ravel())
+            assert e <= LOCAL_TOL, (tokens, li, L["op"], e)
+        st_or["pos"] += tokens
+        next_tok = int(gpu[len(m["layers"]) - 1].ravel()[-1])
 
 
 def test_llm_swapped_equals_resident():
