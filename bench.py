@@ -148,19 +148,31 @@ def cpu_oracle_baseline(model, weights, x, budget_s=12.0, max_runs=5):
                       % (runs, cores)}
 
 
-def build_workload(name):
+def build_workload(name, weight_bytes_fn):
+    """The workload's structure, weights, input and budget.  weight_bytes_fn
+    gives the 256-byte-aligned weight bytes (the library's plan query on the
+    GPU leg; the oracle's count on the reference leg)."""
     import synth
-    from oracle import plan as OP
     arch, kw, frac, text = CONFIGS[name]
     m = synth.arch.MODELS[arch](**kw)
     w = synth.gen.model_weights(m)
     x = synth.gen.model_input(m)
-    wb = OP.weight_bytes(m)
+    wb = weight_bytes_fn(m)
     if frac is None:
         budget = 8_462_336
     else:
         budget = int(wb * frac) // 256 * 256
     return m, w, x, wb, budget, text
+
+
+def capi_weight_bytes(m):
+    from paper_2401_16757_gb300 import capi
+    return capi.Plan.resident(capi.Desc(m)).info()["weight_bytes"]
+
+
+def oracle_weight_bytes(m):
+    from oracle import plan as OP
+    return OP.weight_bytes(m)
 
 
 def llm_host_weights(model, threads=16):
@@ -222,7 +234,6 @@ def run_llm(args, rank, world):
     """Config 5: prefill of 512 ids then 32 greedy decode steps per step."""
     import torch
     import synth
-    from oracle import plan as OP
     from paper_2401_16757_gb300 import capi
     text = CONFIGS["llm"][3]
     t0 = time.perf_counter()
@@ -370,7 +381,7 @@ def run_reference(args, rank, world):
             "e2e": {"value": val, "unit": "inferences/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
         }))
         return
-    m, w, x, wb, budget, text = build_workload(args.config)
+    m, w, x, wb, budget, text = build_workload(args.config, oracle_weight_bytes)
     from oracle import forward as F
     for _ in range(max(0, min(args.warmup, 1))):
         F.forward(m, w, x)
@@ -430,7 +441,7 @@ def main():
     __graft_entry__.build()
     from paper_2401_16757_gb300 import capi
 
-    m, w, x, wb, budget, text = build_workload(args.config)
+    m, w, x, wb, budget, text = build_workload(args.config, capi_weight_bytes)
     d = capi.Desc(m)
     variant = {"auto": capi.SWAP_AUTO, "memcpy": capi.SWAP_MEMCPY, "zerocopy": capi.SWAP_ZEROCOPY}[args.variant]
     act_in = 1 if args.config == "mlp6" else 0

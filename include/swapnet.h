@@ -339,7 +339,8 @@ typedef enum swapnet_kernel_kind {
   SWAPNET_KERNEL_EMBED = 10,      /* zero-copy embedding gather               */
   SWAPNET_KERNEL_RMSNORM = 11,
   SWAPNET_KERNEL_ATTENTION = 12,  /* two launches: RoPE + cache append, attention */
-  SWAPNET_KERNEL_ARGMAX = 13
+  SWAPNET_KERNEL_ARGMAX = 13,
+  SWAPNET_KERNEL_TC_CONV_SMALL = 14 /* tcgen05 conv for C % 8 != 0 (RGB stems)  */
 } swapnet_kernel_kind;
 int swapnet_engine_unit_kernels(const swapnet_engine* eng, int32_t* kinds, uint32_t cap, uint32_t* n);
 

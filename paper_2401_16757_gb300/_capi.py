@@ -76,7 +76,7 @@ class EngineStats(C.Structure):
 
 KERNEL_KIND = {1: "tc_gemm", 2: "tc_conv", 3: "skinny_linear", 4: "direct_conv", 5: "maxpool", 6: "gap",
                7: "upsample2x", 8: "concat", 9: "tiled_linear", 10: "embed", 11: "rmsnorm", 12: "attention",
-               13: "argmax"}
+               13: "argmax", 14: "tc_conv_small"}
 
 
 class EngineBlock(C.Structure):

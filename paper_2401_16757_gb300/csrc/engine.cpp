@@ -327,12 +327,14 @@ static bool unit_gemm(const swapnet_engine* e, const Unit& U, const UnitExec& X,
   g->dtype = m.dtype;
   g->num_sms = e->num_sms;
   g->cluster_max = 16;
+  g->allow_persist = 1;
   g->W = X.w;
   g->e.bias = X.b;
   g->e.act = L.d.act;
   g->e.res_post = L.d.res_post;
   if (L.d.op == SWAPNET_OP_LINEAR) {
     g->M = L.n; g->N = U.rows; g->K = L.d.cin;
+    g->N_layer = L.d.cout;
     g->A = x; g->lda = L.d.cin; g->conv = 0;
     g->y = y + (int64_t)U.row0 * es; g->ldy = L.d.cout;
     g->e.res = r ? r + (int64_t)U.row0 * es : nullptr; g->e.ldr = L.d.cout;
@@ -357,11 +359,21 @@ static bool skinny_ok(const Model& m, const Layer& L) {
   return L.n <= 16 && ((uint64_t)L.d.cin * m.es) % 16 == 0;
 }
 
+// Rows above which a linear layer goes to the tensor cores: the SIMT GEMV
+// does 2 * rows FLOPs per weight byte, which outruns HBM only for a few rows
+// (fp32 FMA rate / HBM bandwidth ~ 6 FLOP/byte on this part).
+constexpr int kSkinnyMaxRows = 4;
+
 static bool wants_tc(const Model& m, const Layer& L) {
   if (m.dtype == SWAPNET_F32) return false;
-  if (L.d.op == SWAPNET_OP_LINEAR) return L.n > 16 && L.d.cin % 8 == 0;
+  if (L.d.op == SWAPNET_OP_LINEAR) return L.n > kSkinnyMaxRows && L.d.cin % 8 == 0;
   if (L.d.op == SWAPNET_OP_CONV2D) return L.d.cin % 8 == 0;
   return false;
+}
+
+static bool small_conv_ok(const Model& m, const Layer& L) {
+  return L.d.op == SWAPNET_OP_CONV2D && L.d.cin % 8 != 0 &&
+         tc_small_supported(m.dtype, L.d.kh * L.d.kw * L.d.cin);
 }
 
 static int prepare_units(swapnet_engine* e) {
@@ -377,7 +389,8 @@ static int prepare_units(swapnet_engine* e) {
         k = wants_tc(m, L) ? SWAPNET_KERNEL_TC_GEMM : skinny_ok(m, L) ? SWAPNET_KERNEL_SKINNY : SWAPNET_KERNEL_TILED;
         break;
       case SWAPNET_OP_CONV2D:
-        if (!wants_tc(m, L)) k = SWAPNET_KERNEL_DIRECT_CONV;
+        if (!wants_tc(m, L))
+          k = small_conv_ok(m, L) ? SWAPNET_KERNEL_TC_CONV_SMALL : SWAPNET_KERNEL_DIRECT_CONV;
         else if (L.d.kh == 1 && L.d.kw == 1 && L.d.stride == 1 && L.d.pad == 0) k = SWAPNET_KERNEL_TC_GEMM;
         else k = SWAPNET_KERNEL_TC_CONV;
         break;
@@ -459,6 +472,15 @@ static int run_unit(swapnet_engine* e, int u, const void* din, void* dout, cudaS
                                    s);
       }
       ep.res = r;
+      if (small_conv_ok(m, L)) {
+        TcSmallConv g;
+        g.dtype = m.dtype; g.x = x; g.W = X.w;
+        g.M = L.on * L.oh * L.ow; g.N = L.d.cout; g.K = L.d.kh * L.d.kw * L.d.cin;
+        g.H = L.h; g.Wd = L.w; g.C = L.d.cin; g.Ho = L.oh; g.Wo = L.ow;
+        g.kh = L.d.kh; g.kw = L.d.kw; g.stride = L.d.stride; g.pad = L.d.pad;
+        g.e = ep; g.y = y; g.ldy = L.d.cout; g.num_sms = e->num_sms;
+        return launch_tc_conv_small(g, e->err_word, s);
+      }
       return launch_conv_direct(m.dtype, x, L.n, L.h, L.w, L.d.cin, X.w, L.d.cout, L.d.kh, L.d.kw, L.d.stride,
                                 L.d.pad, L.oh, L.ow, ep, y, s);
     }

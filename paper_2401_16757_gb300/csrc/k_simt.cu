@@ -47,6 +47,14 @@ template <typename T> __device__ __forceinline__ void unpack16(const uint4& v, f
   for (int i = 0; i < Vec16<T>::N; ++i) f[i] = to_f<T>(e[i]);
 }
 
+template <typename T> __device__ __forceinline__ uint4 pack16(const float* f) {
+  uint4 v;
+  T* e = reinterpret_cast<T*>(&v);
+#pragma unroll
+  for (int i = 0; i < Vec16<T>::N; ++i) e[i] = from_f<T>(f[i]);
+  return v;
+}
+
 // ------------------------------------------------------------ skinny linear
 // One CTA (8 warps) computes COLS output features for all M rows.  Warp w
 // reduces the K range [w*Kw, (w+1)*Kw); inside a warp lane l takes the
@@ -327,6 +335,70 @@ __global__ void concat_kernel(const T* __restrict__ a, int ca, const T* __restri
   y[idx] = ch < ca ? a[p * ca + ch] : b[p * cb + (ch - ca)];
 }
 
+// Vectorised variants: a thread handles 16 bytes of channels (channels a
+// multiple of the vector width, rows 16-byte aligned).  Max is exact, so
+// the result equals the scalar kernels'.
+template <typename T>
+__global__ void maxpool_vec_kernel(const uint4* __restrict__ x, int n, int h, int w, int cv, int kh, int kw,
+                                   int stride, int pad, int oh, int ow, uint4* __restrict__ y) {
+  constexpr int V = Vec16<T>::N;
+  pdl_wait();
+  pdl_launch_dependents();
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t total = (int64_t)n * oh * ow * cv;
+  if (idx >= total) return;
+  const int ch = (int)(idx % cv);
+  const int64_t p = idx / cv;
+  const int ox = (int)(p % ow);
+  const int64_t q = p / ow;
+  const int oy = (int)(q % oh);
+  const int img = (int)(q / oh);
+  float m[V];
+#pragma unroll
+  for (int i = 0; i < V; ++i) m[i] = -INFINITY;
+  for (int r = 0; r < kh; ++r) {
+    const int iy = oy * stride + r - pad;
+    if (iy < 0 || iy >= h) continue;
+    for (int s = 0; s < kw; ++s) {
+      const int ix = ox * stride + s - pad;
+      if (ix < 0 || ix >= w) continue;
+      float f[V];
+      unpack16<T>(__ldg(x + (((int64_t)img * h + iy) * w + ix) * cv + ch), f);
+#pragma unroll
+      for (int i = 0; i < V; ++i) m[i] = fmaxf(m[i], f[i]);
+    }
+  }
+  y[idx] = pack16<T>(m);
+}
+
+__global__ void upsample2x_vec_kernel(const uint4* __restrict__ x, int n, int h, int w, int cv,
+                                      uint4* __restrict__ y) {
+  pdl_wait();
+  pdl_launch_dependents();
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t total = (int64_t)n * 2 * h * 2 * w * cv;
+  if (idx >= total) return;
+  const int ch = (int)(idx % cv);
+  const int64_t p = idx / cv;
+  const int ox = (int)(p % (2 * w));
+  const int64_t q = p / (2 * w);
+  const int oy = (int)(q % (2 * h));
+  const int img = (int)(q / (2 * h));
+  y[idx] = x[(((int64_t)img * h + oy / 2) * w + ox / 2) * cv + ch];
+}
+
+__global__ void concat_vec_kernel(const uint4* __restrict__ a, int ca, const uint4* __restrict__ b, int cb,
+                                  int64_t pixels, uint4* __restrict__ y) {
+  pdl_wait();
+  pdl_launch_dependents();
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int c = ca + cb;
+  if (idx >= pixels * c) return;
+  const int64_t p = idx / c;
+  const int ch = (int)(idx % c);
+  y[idx] = ch < ca ? a[p * ca + ch] : b[p * cb + (ch - ca)];
+}
+
 inline int grid1d(int64_t total, int block) { return (int)((total + block - 1) / block); }
 
 
@@ -389,6 +461,15 @@ int launch_conv_direct(int dtype, const void* x, int n, int h, int w, int cin, c
 
 int launch_maxpool(int dtype, const void* x, int n, int h, int w, int c, int kh, int kw, int stride, int pad,
                    int oh, int ow, void* y, cudaStream_t s) {
+  SN_DISPATCH(dtype, T, {
+    constexpr int V = Vec16<T>::N;
+    if (c % V == 0 && ((uintptr_t)x | (uintptr_t)y) % 16 == 0) {
+      const int64_t tv = (int64_t)n * oh * ow * (c / V);
+      launch_pdl(maxpool_vec_kernel<T>, dim3(grid1d(tv, 256)), dim3(256), 0, s, static_cast<const uint4*>(x), n, h,
+                 w, c / V, kh, kw, stride, pad, oh, ow, static_cast<uint4*>(y));
+      return last_launch();
+    }
+  });
   const int64_t total = (int64_t)n * oh * ow * c;
   SN_DISPATCH(dtype, T,
               launch_pdl(maxpool_kernel<T>, dim3(grid1d(total, 256)), dim3(256), 0, s, static_cast<const T*>(x), n, h,
@@ -404,6 +485,15 @@ int launch_gap(int dtype, const void* x, int n, int h, int w, int c, void* y, cu
 }
 
 int launch_upsample2x(int dtype, const void* x, int n, int h, int w, int c, void* y, cudaStream_t s) {
+  {
+    const int es = dtype == SWAPNET_F32 ? 4 : 2;
+    if ((c * es) % 16 == 0 && ((uintptr_t)x | (uintptr_t)y) % 16 == 0) {
+      const int cv = c * es / 16;
+      launch_pdl(upsample2x_vec_kernel, dim3(grid1d((int64_t)n * 4 * h * w * cv, 256)), dim3(256), 0, s,
+                 static_cast<const uint4*>(x), n, h, w, cv, static_cast<uint4*>(y));
+      return last_launch();
+    }
+  }
   const int64_t total = (int64_t)n * 4 * h * w * c;
   SN_DISPATCH(dtype, T,
               launch_pdl(upsample2x_kernel<T>, dim3(grid1d(total, 256)), dim3(256), 0, s, static_cast<const T*>(x), n,
@@ -413,6 +503,16 @@ int launch_upsample2x(int dtype, const void* x, int n, int h, int w, int c, void
 
 int launch_concat(int dtype, const void* a, int ca, const void* b, int cb, int64_t pixels, void* y,
                   cudaStream_t s) {
+  {
+    const int es = dtype == SWAPNET_F32 ? 4 : 2;
+    if ((ca * es) % 16 == 0 && (cb * es) % 16 == 0 && ((uintptr_t)a | (uintptr_t)b | (uintptr_t)y) % 16 == 0) {
+      const int av = ca * es / 16, bv = cb * es / 16;
+      launch_pdl(concat_vec_kernel, dim3(grid1d(pixels * (av + bv), 256)), dim3(256), 0, s,
+                 static_cast<const uint4*>(a), av, static_cast<const uint4*>(b), bv, pixels,
+                 static_cast<uint4*>(y));
+      return last_launch();
+    }
+  }
   const int64_t total = pixels * (ca + cb);
   SN_DISPATCH(dtype, T,
               launch_pdl(concat_kernel<T>, dim3(grid1d(total, 256)), dim3(256), 0, s, static_cast<const T*>(a), ca,

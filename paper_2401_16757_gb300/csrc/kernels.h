@@ -76,6 +76,10 @@ struct TcGemm {
   void* y;
   int64_t ldy;
   int num_sms;          // used by tc_prepare to size the grid
+  int allow_persist;    // 1: problems with a tile per SM take the persistent kernel
+  int N_layer;          // > 0: N of the whole layer this GEMM is a column piece
+                        // of; tiling and split-K follow it, so every piece sums
+                        // each output in the same order as the unsplit layer
   int cluster_max;      // > 0: split K across a thread-block cluster of at most
                         // this many CTAs (DSMEM reduction); 0: global scratch
   float* partial;       // split-K scratch (TcPlan::scratch_bytes), set per launch
@@ -91,10 +95,29 @@ struct TcPlan {
   int kb_per_split; // 64-wide k-blocks per split
   int64_t tiles;    // output tiles (split-K counters needed)
   uint64_t scratch_bytes;  // fp32 partials of all splits
+  int persist;      // persistent kernel (one CTA per SM looping over tiles)
   int ready;
 };
 int tc_prepare(const TcGemm& g, TcPlan* p);
 int launch_tc_gemm(const TcGemm& g, const TcPlan& p, int* dev_err, cudaStream_t s);
+int launch_tc_persist(const TcGemm& g, const TcPlan& p, int* dev_err, cudaStream_t s);
+
+// tcgen05 convolution for channel counts the gather cannot fetch in 16-byte
+// pieces (C % 8 != 0), K = kh*kw*C <= 192: weights built in shared memory,
+// im2col gathered element by element, persistent over output tiles.
+struct TcSmallConv {
+  int dtype;  // SWAPNET_F16 or SWAPNET_BF16
+  const void* x;  // NHWC input
+  const void* W;  // [N][kh][kw][C]
+  int M, N, K;    // M = n*Ho*Wo, N = cout, K = kh*kw*C
+  int H, Wd, C, Ho, Wo, kh, kw, stride, pad;
+  Epi e;
+  void* y;
+  int64_t ldy;
+  int num_sms;
+};
+bool tc_small_supported(int dtype, int K);
+int launch_tc_conv_small(const TcSmallConv& g, int* dev_err, cudaStream_t s);
 
 // Device error word of the tcgen05 kernels (bounded waits).
 int tc_error_word(int** ptr);

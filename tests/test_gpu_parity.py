@@ -53,8 +53,16 @@ def _check_model(m, budget_frac=0.5, slots=2, variant=capi.SWAP_AUTO):
     (3, 2, 32, 96, 23),     # Cin=32: K=288 not a multiple of 64; stride 2
     (1, 1, 64, 200, 17),    # pointwise: TMA A path, N not a multiple of 64
     (1, 2, 128, 256, 14),   # strided pointwise: gather path
-    (7, 2, 3, 64, 40),      # stem: direct conv (Cin=3)
-    (3, 1, 3, 16, 12),      # direct conv
+    (7, 2, 3, 64, 40),      # ResNet stem: small-channel tcgen05 conv, K=147 (3 k-blocks)
+    (3, 1, 3, 16, 12),      # small-channel conv, N=16
+    (3, 1, 3, 96, 37),      # small-channel conv, two 64-column slices, ragged M
+    (5, 1, 4, 32, 21),      # Cin=4, K=100 (2 k-blocks)
+    (3, 1, 3, 32, 224),     # 784 tiles: more tiles than resident CTAs (persistent loop)
+    (7, 1, 5, 40, 15),      # K=245 beyond the small-channel kernel: SIMT direct conv
+    (3, 1, 64, 64, 112),    # 196 x 1 tiles >= one per SM: persistent kernel, N tile 64, gather
+    (3, 1, 32, 128, 112),   # persistent, N tile 128, gather with k-blocks straddling taps
+    (1, 1, 64, 300, 112),   # persistent, N tile 256 (ragged), A by TMA
+    (3, 2, 64, 256, 224),   # persistent, N tile 256, strided gather
     (3, 1, 256, 256, 7),    # deep K, one M tile: split-K with last-CTA reduction
     (3, 1, 64, 24, 9),      # N below one 32-column chunk
 ])
@@ -80,14 +88,14 @@ def test_linear_layer(dtype, rows, k, n):
     _check_model(_model(layers, (rows, 1, 1, k), dtype))
 
 
-@pytest.mark.parametrize("dtype", ["f16", "f32"])
-def test_pool_upsample_concat(dtype):
+@pytest.mark.parametrize("dtype,ch", [("f16", 24), ("f32", 24), ("f16", 20), ("bf16", 8)])
+def test_pool_upsample_concat(dtype, ch):
     layers = [dict(op="maxpool", src=[-1], kh=3, kw=3, stride=2, pad=1),
               dict(op="maxpool", src=[0], kh=2, kw=2, stride=2, pad=0),
               dict(op="upsample2x", src=[1]),
               dict(op="concat", src=[2, 0]),
               dict(op="gap", src=[3])]
-    m = _model(layers, (2, 32, 32, 24), dtype, outputs=[3, 4])
+    m = _model(layers, (2, 32, 32, ch), dtype, outputs=[3, 4])   # 16-byte vectors unless ch=20 (f16)
     # no weights: swapped plan has nothing to swap; compare to the oracle
     w = synth.gen.model_weights(m)
     x = synth.gen.model_input(m)
