@@ -45,6 +45,8 @@ CONFIGS = {
     "vgg16_b1": ("vgg16", dict(batch=1), 0.25, "VGG-16-shaped CNN, fp16, batch 1, budget 25% of weight bytes"),
     "vgg16_b16": ("vgg16", dict(batch=16), 0.25, "VGG-16-shaped CNN, fp16, batch 16, budget 25% of weight bytes"),
     "yolov3": ("yolov3", dict(batch=1), 0.30, "YOLOv3 (Darknet-53 + 3 heads), fp16, 1x3x416x416, budget 30%"),
+    "multi": ("multi", {}, 0.30, "ResNet-50 + VGG-16 + YOLOv3 (fp16, batch 1), concurrent closed-loop request "
+              "streams, one arena of 30% of the summed weight bytes split by Eq. 1"),
     "llm": ("llm", dict(tokens=512), None,
             "LLaMA-7B-shaped decoder bf16 (32 layers, d 4096, 32 heads, FFN 11008, vocab 32000); "
             "prefill 512 token ids + 32 greedy decode steps, batch 1; 4e9-byte weight arena"),
@@ -345,6 +347,103 @@ def run_llm(args, rank, world):
         print(json.dumps(line))
 
 
+def run_multi(args, rank, world):
+    """Config 4: three models at batch 1, each with its own closed-loop request
+    stream on its own CUDA stream, sharing one arena split by Eq. 1
+    (swapnet_schedule); DInf is the same concurrent run with every model
+    resident."""
+    import torch
+    import synth
+    from paper_2401_16757_gb300 import capi
+    names = ("resnet50", "vgg16", "yolov3")
+    ms = [synth.arch.MODELS[n]() for n in names]
+    stream0 = torch.cuda.current_stream()
+    link_peak = measure_link_peak(stream0)
+    alpha = int(round(1e18 / (link_peak * 1e9)))
+    variant = {"auto": capi.SWAP_AUTO, "memcpy": capi.SWAP_MEMCPY, "zerocopy": capi.SWAP_ZEROCOPY}[args.variant]
+    opt = capi.options(swap_variant=variant, alpha_as_per_byte=alpha, beta_ns_per_tensor=0, eta_ns_per_tensor=0)
+    descs = [capi.Desc(m) for m in ms]
+    wbs = [capi_weight_bytes(m) for m in ms]
+    arena = int(sum(wbs) * 0.30) // 256 * 256
+    budgets, plans = capi.schedule(descs, [1.0, 1.0, 1.0], arena, opt)
+    hosts = [capi.HostWeights(synth.gen.model_weights(m)) for m in ms]
+    engs = [capi.Engine(p, h) for p, h in zip(plans, hosts)]
+    rengs = [capi.Engine(capi.Plan.resident(d), h) for d, h in zip(descs, hosts)]
+    infos = [p.info() for p in plans]
+    ins, outs = [], []
+    for m, inf in zip(ms, infos):
+        x = synth.gen.model_input(m)
+        d_in = torch.empty(max(16, inf["input_bytes"]), dtype=torch.uint8, device="cuda")
+        d_in[:inf["input_bytes"]].copy_(torch.from_numpy(x.view(np.uint8).reshape(-1)))
+        ins.append(d_in)
+        outs.append(torch.empty(inf["output_bytes"], dtype=torch.uint8, device="cuda"))
+    streams = [torch.cuda.Stream() for _ in ms]
+
+    def run(engines, steps):
+        ev = lambda: torch.cuda.Event(enable_timing=True)
+        evs = [[(ev(), ev()) for _ in range(steps)] for _ in engines]
+        start = ev()
+        start.record(stream0)
+        for s in streams:
+            s.wait_event(start)
+        for i in range(steps):
+            for k, e in enumerate(engines):
+                a, b = evs[k][i]
+                a.record(streams[k])
+                e.infer(ins[k].data_ptr(), outs[k].data_ptr(), streams[k].cuda_stream)
+                b.record(streams[k])
+        ends = []
+        for s in streams:
+            e_ = ev()
+            e_.record(s)
+            ends.append(e_)
+        torch.cuda.synchronize()
+        lat = [[a.elapsed_time(b) for a, b in evs[k]] for k in range(len(engines))]
+        wall = max(start.elapsed_time(e_) for e_ in ends)
+        return lat, wall
+
+    run(engs, args.warmup)
+    run(rengs, args.warmup)
+    for e in engs + rengs:
+        e.sync()
+    clocks = ClockSampler(int(os.environ.get("LOCAL_RANK", "0")))
+    clocks.start()
+    launches0 = sum(e.stats()["kernel_launches"] for e in engs)
+    lat_sw, wall_sw = run(engs, args.steps)
+    launches = sum(e.stats()["kernel_launches"] for e in engs) - launches0
+    lat_di, wall_di = run(rengs, args.steps)
+    clk = clocks.stop()
+    for e in engs:
+        e.sync()
+    n_req = len(ms) * args.steps
+    swap_bytes = sum(sum(b["bytes"] for b in p.blocks()) for p in plans)
+    hbm, tf_burst, tf_sust, peak_src = load_peaks()
+    flops = sum(sum(u["flops"] for u in p.units()) for p in plans)
+    bound_ms = max(flops / (tf_burst * 1e12), swap_bytes / (link_peak * 1e9)) * 1e3  # one request of each model
+    per_model = {}
+    for k, n in enumerate(names):
+        sw, di = statistics.mean(lat_sw[k]), statistics.mean(lat_di[k])
+        per_model[n] = {"budget_bytes": budgets[k], "weight_bytes": wbs[k], "n_blocks": infos[k]["n_blocks"],
+                        "ms_swapped": sw, "ms_dinf": di, "ratio": sw / di,
+                        "p50_swapped": statistics.median(lat_sw[k]), "p50_dinf": statistics.median(lat_di[k])}
+    line = {
+        "metric": METRIC, "value": n_req / (wall_sw * 1e-3), "unit": "inferences/s (3 models, concurrent)",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": wall_sw / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f16", "data": "synthetic",
+        "config": {"workload": CONFIGS["multi"][3], "arena_bytes": arena, "weight_bytes": sum(wbs),
+                   "l2": "no flush: 451.6 MB of weights stream through the arena every round"},
+        "per_model": per_model,
+        "dinf_ms_per_step": wall_di / args.steps, "throughput_ratio": wall_sw / wall_di,
+        "link": {"achieved_gbs": swap_bytes * args.steps / (wall_sw * 1e-3) / 1e9, "peak_gbs": link_peak,
+                 "peak_source": "pinned cudaMemcpy H2D 256 MiB", "bytes_per_step": swap_bytes},
+        "step_roofline": {"bound": "host link" if swap_bytes / (link_peak * 1e9) > flops / (tf_burst * 1e12)
+                          else "tensor", "bound_ms": bound_ms, "frac": bound_ms / (wall_sw / args.steps)},
+        "gpu_launches": launches, "clocks": clk,
+    }
+    if rank == 0:
+        print(json.dumps(line))
+
+
 def measure_link_peak(stream):
     import torch
     pk = torch.empty(256 << 20, dtype=torch.uint8, pin_memory=True)
@@ -363,6 +462,33 @@ def measure_link_peak(stream):
 def run_reference(args, rank, world):
     """The reference arm: the CPU oracle, timed as it stands on the host cores."""
     if rank != 0:
+        return
+    if args.config == "multi":
+        import synth
+        from oracle import forward as F
+        cores = len(os.sched_getaffinity(0))
+        work = []
+        for n in ("resnet50", "vgg16", "yolov3"):
+            m = synth.arch.MODELS[n]()
+            work.append((m, synth.gen.model_weights(m), synth.gen.model_input(m)))
+        times = []
+        for _ in range(args.steps):   # one request of each model per step
+            t0 = time.perf_counter()
+            for m, w, x in work:
+                F.forward(m, w, x)
+            times.append(time.perf_counter() - t0)
+        ms = 1000.0 * sum(times) / len(times)
+        val = 3000.0 / ms
+        print(json.dumps({
+            "impl": "reference", "metric": METRIC, "value": val, "unit": "inferences/s (3 models, concurrent)",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": CONFIGS["multi"][3], "l2": "n/a (CPU)"},
+            "cpu_baseline": {"value": val, "unit": "inferences/s", "cores": cores, "kind": "oracle",
+                             "sample": "one float64 inference of each of the three models per step, in sequence"},
+            "e2e": {"value": val, "unit": "inferences/s (3 models, concurrent)", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0},
+        }))
         return
     if args.config == "llm":
         cores = len(os.sched_getaffinity(0))
@@ -422,12 +548,12 @@ def main():
     if args.impl == "reference":
         run_reference(args, rank, world)
         return
-    if args.config == "llm":
+    if args.config in ("llm", "multi"):
         import torch
         torch.cuda.set_device(local)
         import __graft_entry__
         __graft_entry__.build()
-        run_llm(args, rank, world)
+        (run_llm if args.config == "llm" else run_multi)(args, rank, world)
         return
 
     import torch
