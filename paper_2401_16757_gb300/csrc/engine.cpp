@@ -451,7 +451,7 @@ static int run_unit(swapnet_engine* e, int u, const void* din, void* dout, cudaS
       if (X.use_tc) {
         TcGemm g;
         unit_gemm(e, U, X, x, r, y, &g);
-        if (!g.conv && g.A != X.tmA_for) {
+        if ((!g.conv || X.tc.tma_conv) && g.A != X.tmA_for) {
           int rc = tc_prepare(g, &X.tc);
           if (rc) return rc;
           X.tmA_for = g.A;

@@ -396,6 +396,48 @@ int make_tmap(CUtensorMap* m, int dtype, const void* base, uint64_t inner, uint6
   return SWAPNET_OK;
 }
 
+// 4-D map of an NHWC activation tensor for per-tap im2col loads: box of 64
+// channels x wt columns x ht rows of one image, every s-th column and row
+// (the conv stride), zero fill outside the image (the conv padding).
+int make_tmap_conv4d(CUtensorMap* m, int dtype, const void* base, int n, int h, int w, int c, int wt, int ht,
+                     int stride) {
+  auto fn = encode_fn();
+  if (!fn) SN_FAIL(SWAPNET_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+  if (((uintptr_t)base & 15) || (c * 2) % 16)
+    SN_FAIL(SWAPNET_ERR_MISALIGNED, "TMA conv operand must be 16-byte aligned");
+  const cuuint64_t dims[4] = {(cuuint64_t)c, (cuuint64_t)w, (cuuint64_t)h, (cuuint64_t)n};
+  const cuuint64_t strides[3] = {(cuuint64_t)c * 2, (cuuint64_t)w * c * 2, (cuuint64_t)h * w * c * 2};
+  const cuuint32_t box[4] = {(cuuint32_t)kBK, (cuuint32_t)(wt * stride), (cuuint32_t)(ht * stride), 1};
+  const cuuint32_t estr[4] = {1, (cuuint32_t)stride, (cuuint32_t)stride, 1};
+  const CUresult r = fn(m, dtype == SWAPNET_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16,
+                        4, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS)
+    SN_FAIL(SWAPNET_ERR_CUDA, "cuTensorMapEncodeTiled (conv) failed (" + std::to_string((int)r) + ")");
+  return SWAPNET_OK;
+}
+
+// Output patch (wt x ht pixels, wt * ht <= 128) for per-tap TMA loads that
+// wastes the fewest of the 128 MMA rows; returns the used fraction.
+double conv_patch(int ho, int wo, int stride, int* wt, int* ht) {
+  double best = 0.0;
+  *wt = *ht = 0;
+  for (int cand : {wo, 128, 64, 32, 16, 8, 4}) {
+    if (cand < 1 || cand > 128 || cand * stride > 256) continue;
+    const int w_ = cand, h_ = std::min(128 / w_, ho);
+    if (h_ < 1 || h_ * stride > 256) continue;
+    const double tiles = (double)((wo + w_ - 1) / w_) * ((ho + h_ - 1) / h_);
+    const double util = (double)ho * wo / (tiles * kBM);
+    if (util > best + 1e-9) {
+      best = util;
+      *wt = w_;
+      *ht = h_;
+    }
+  }
+  return best;
+}
+
 template <typename T, int BN, bool GATHER>
 int launch_inst(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) {
   static bool attr_done = false;  // per instantiation
@@ -511,16 +553,35 @@ int tc_prepare(const TcGemm& g, TcPlan* p) {
   if (g.allow_persist) {
     // at least one output tile per SM: the persistent kernel, no split
     const int pbn = Nd <= 64 ? 64 : (Nd <= 128 ? 128 : 256);
-    if (mtiles * ((Nd + pbn - 1) / pbn) >= sms) {
+    // convolutions whose taps are whole 64-channel k-blocks load A by 4-D TMA
+    // when a pixel patch fills the 128 MMA rows well enough
+    int wt = 0, ht = 0;
+    const bool tmac = g.conv && g.C % kBK == 0 && conv_patch(g.Ho, g.Wo, g.stride, &wt, &ht) >= 0.85;
+    const int64_t sp_tiles = tmac ? (int64_t)g.M / ((int64_t)g.Ho * g.Wo) * ((g.Wo + wt - 1) / wt) *
+                                        ((g.Ho + ht - 1) / ht)
+                                  : mtiles;
+    if (sp_tiles * ((Nd + pbn - 1) / pbn) >= sms) {
       p->persist = 1;
+      if (tmac) {
+        p->tma_conv = 1;
+        p->wt = wt;
+        p->ht = ht;
+        p->tiles_w = (g.Wo + wt - 1) / wt;
+        p->tiles_h = (g.Ho + ht - 1) / ht;
+      }
       p->bn = pbn;
       p->splits = 1;
       p->kb_per_split = (g.K + kBK - 1) / kBK;
-      p->tiles = mtiles * ((g.N + pbn - 1) / pbn);
+      p->tiles = sp_tiles * ((g.N + pbn - 1) / pbn);
       int rc = make_tmap(&p->tmB, g.dtype, g.W, (uint64_t)g.K, (uint64_t)g.N, (uint64_t)g.K * 2, (uint32_t)pbn);
       if (rc) return rc;
       if (!g.conv && g.A) {
         rc = make_tmap(&p->tmA, g.dtype, g.A, (uint64_t)g.K, (uint64_t)g.M, (uint64_t)g.lda * 2, (uint32_t)kBM);
+        if (rc) return rc;
+      }
+      if (tmac && g.A) {
+        const int n_img = (int)((int64_t)g.M / ((int64_t)g.Ho * g.Wo));
+        rc = make_tmap_conv4d(&p->tmA, g.dtype, g.A, n_img, g.H, g.Wd, g.C, wt, ht, g.stride);
         if (rc) return rc;
       }
       p->ready = 1;

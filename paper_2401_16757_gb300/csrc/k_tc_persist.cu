@@ -11,7 +11,13 @@
 //   warp 1       TMEM owner and MMA issuer (one elected lane)
 //   warps 2..5   epilogue: TMEM -> registers -> bias / residual / activation
 //                -> global, warp w reading TMEM lanes 32 * (w % 4) .. + 31
-//   warps 6..9   (convolutions) implicit im2col gather of A with cp.async
+//   warps 6..9   (convolutions without whole-tap TMA) implicit im2col gather of
+//                A with cp.async
+// A-operand modes: kAT2d (row-major A by 2-D TMA), kAGather (cp.async im2col
+// gather), kATap (convolution A by one 4-D TMA per k-block: the 64 channels
+// of one filter tap at a wt x ht patch of output pixels, the image border
+// and the stride handled by the copy engine's zero fill and element stride;
+// the output tile is then that patch, rows >= wt * ht unused).
 // A ring of shared-memory stages (full / empty mbarriers) feeds the MMAs,
 // continuous across tiles.  The accumulator is double-buffered in TMEM
 // (2 x BN columns, tfull / tempty mbarriers): the MMAs of the next tile run
@@ -46,12 +52,15 @@ template <int BN> struct PCfg {
   static constexpr int kSmem = kStageBytes + kBias + 256 + 1024;
 };
 
-template <bool GATHER> constexpr int persist_threads() { return GATHER ? 320 : 192; }
+constexpr int kAT2d = 0, kAGather = 1, kATap = 2;
 
-template <typename T, int BN, bool GATHER>
-__global__ void __launch_bounds__(persist_threads<GATHER>(), 1)
+template <int AMODE> constexpr int persist_threads() { return AMODE == kAGather ? 320 : 192; }
+
+template <typename T, int BN, int AMODE>
+__global__ void __launch_bounds__(persist_threads<AMODE>(), 1)
     tc_persist_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const TcArgs p) {
+  constexpr bool GATHER = AMODE == kAGather;
   using Cfg = PCfg<BN>;
   constexpr int kStages = Cfg::kStages;
   extern __shared__ uint8_t smem_raw[];
@@ -70,7 +79,12 @@ __global__ void __launch_bounds__(persist_threads<GATHER>(), 1)
   auto empty_bar = [&](int s) { return empty0 + 8u * s; };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int mt = (p.M + kPBM - 1) / kPBM, nt = (p.N + BN - 1) / BN;
+  // m-tiles: 128-row blocks of the output matrix, or pixel patches (kATap)
+  const int hw = p.Ho * p.Wo;
+  const int patches = p.tiles_w * p.tiles_h;
+  const int mt = AMODE == kATap ? (p.M / hw) * patches : (p.M + kPBM - 1) / kPBM;
+  const int nt = (p.N + BN - 1) / BN;
+  const uint32_t a_bytes = AMODE == kATap ? (uint32_t)(p.wt * p.ht * 128) : (AMODE == kAT2d ? kPA : 0);
   const int tiles = mt * nt;
   const int KB = (p.K + kPBK - 1) / kPBK;
   const int my_tiles = blockIdx.x < tiles ? (tiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
@@ -115,29 +129,40 @@ __global__ void __launch_bounds__(persist_threads<GATHER>(), 1)
         *m0 = (tile % mt) * kPBM;
         *n0 = (tile / mt) * BN;
       };
+      auto load_a = [&](int s, int g) {
+        const int tile = tile_of(g / KB);
+        const int k0 = (g % KB) * kPBK;
+        if (AMODE == kAT2d) {
+          tma_load_2d(smem_u32(sA + s * kPA), &tmA, full_bar(s), k0, (tile % mt) * kPBM);
+        } else if (AMODE == kATap) {
+          const int sp = tile % mt;
+          const int img = sp / patches, rem = sp - img * patches;
+          const int th = rem / p.tiles_w, tw = rem - th * p.tiles_w;
+          const int tap = k0 / p.C, c0 = k0 - tap * p.C;
+          const int ry = tap / p.kw, rx = tap - ry * p.kw;
+          tma_load_4d(smem_u32(sA + s * kPA), &tmA, full_bar(s), c0, tw * p.wt * p.stride - p.pad + rx,
+                      th * p.ht * p.stride - p.pad + ry, img);
+        }
+      };
       const int early = min(work, kStages);
       for (int g = 0; g < early; ++g) {
         int kx, m0, n0;
         coords(g, &kx, &m0, &n0);
-        mbar_arrive_expect_tx(full_bar(g), Cfg::kB + (GATHER ? 0 : kPA));
+        mbar_arrive_expect_tx(full_bar(g), Cfg::kB + a_bytes);
         tma_load_2d(smem_u32(sB + g * Cfg::kB), &tmB, full_bar(g), kx, n0);
       }
       pdl_wait();
       if (!GATHER)
-        for (int g = 0; g < early; ++g) {
-          int kx, m0, n0;
-          coords(g, &kx, &m0, &n0);
-          tma_load_2d(smem_u32(sA + g * kPA), &tmA, full_bar(g), kx, m0);
-        }
+        for (int g = 0; g < early; ++g) load_a(g, g);
       int g = early;
       for (; g < work; ++g) {
         const int s = g % kStages, r = g / kStages;
         if (!mbar_wait_bounded(empty_bar(s), (r & 1) ^ 1, abort_flag, p.err)) break;
         int kx, m0, n0;
         coords(g, &kx, &m0, &n0);
-        mbar_arrive_expect_tx(full_bar(s), Cfg::kB + (GATHER ? 0 : kPA));
+        mbar_arrive_expect_tx(full_bar(s), Cfg::kB + a_bytes);
         tma_load_2d(smem_u32(sB + s * Cfg::kB), &tmB, full_bar(s), kx, n0);
-        if (!GATHER) tma_load_2d(smem_u32(sA + s * kPA), &tmA, full_bar(s), kx, m0);
+        if (!GATHER) load_a(s, g);
       }
       if (g < work) {
         // aborted: let the loads already issued land before the CTA exits
@@ -188,7 +213,20 @@ __global__ void __launch_bounds__(persist_threads<GATHER>(), 1)
     for (int lt = 0; lt < my_tiles; ++lt) {
       const int buf = lt & 1, use = lt >> 1;
       const int tile = tile_of(lt);
-      const int m0 = (tile % mt) * kPBM, n0 = (tile / mt) * BN;
+      const int n0 = (tile / mt) * BN;
+      int m = -1;  // output row of this thread's TMEM lane, -1 when unused
+      if (AMODE == kATap) {
+        const int sp = tile % mt;
+        const int img = sp / patches, rem = sp - img * patches;
+        const int th = rem / p.tiles_w, tw = rem - th * p.tiles_w;
+        if (row < p.wt * p.ht) {
+          const int oy = th * p.ht + row / p.wt, ox = tw * p.wt + row % p.wt;
+          if (oy < p.Ho && ox < p.Wo) m = (img * p.Ho + oy) * p.Wo + ox;
+        }
+      } else {
+        m = (tile % mt) * kPBM + row;
+        if (m >= p.M) m = -1;
+      }
       // each warp stages its own copy of the tile's bias: no cross-warp barrier
       float* sb = sbias + (buf * 4 + q) * BN;
       const T* bias = static_cast<const T*>(p.e.bias);
@@ -197,14 +235,13 @@ __global__ void __launch_bounds__(persist_threads<GATHER>(), 1)
       const bool got = mbar_wait_bounded(tfull0 + 8u * buf, use & 1, abort_flag, p.err);
       if (!__all_sync(0xffffffffu, got)) break;  // tcgen05.ld is warp-collective
       tc_fence_after();
-      const int m = m0 + row;
       const bool vec_ok = ((p.ldy | n0) % 8 == 0) && (!p.e.res || ((p.e.ldr | n0) % 8 == 0));
 #pragma unroll 1
       for (int c0 = 0; c0 < BN; c0 += 32) {
         uint32_t r[32];
         tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN + c0), r);
         tmem_ld_wait();
-        if (m < p.M && n0 + c0 < p.N) {
+        if (m >= 0 && n0 + c0 < p.N) {
           float v[32];
 #pragma unroll
           for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
@@ -295,10 +332,10 @@ __global__ void __launch_bounds__(persist_threads<GATHER>(), 1)
   }
 }
 
-template <typename T, int BN, bool GATHER>
+template <typename T, int BN, int AMODE>
 int launch_persist_inst(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) {
   static bool attr_done = false;  // per instantiation
-  auto kern = tc_persist_kernel<T, BN, GATHER>;
+  auto kern = tc_persist_kernel<T, BN, AMODE>;
   if (!attr_done) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, PCfg<BN>::kSmem) != cudaSuccess)
       SN_FAIL(SWAPNET_ERR_CUDA, "cudaFuncSetAttribute failed");
@@ -311,12 +348,15 @@ int launch_persist_inst(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_
   a.H = g.H; a.Wd = g.Wd; a.C = g.C; a.Ho = g.Ho; a.Wo = g.Wo;
   a.kh = g.kh; a.kw = g.kw; a.stride = g.stride; a.pad = g.pad;
   a.e = g.e; a.y = g.y; a.ldy = g.ldy; a.err = err;
-  const int64_t tiles = (int64_t)((g.M + kPBM - 1) / kPBM) * ((g.N + BN - 1) / BN);
+  a.wt = pl.wt; a.ht = pl.ht; a.tiles_w = pl.tiles_w; a.tiles_h = pl.tiles_h;
+  const int64_t mt = AMODE == kATap ? (int64_t)g.M / ((int64_t)g.Ho * g.Wo) * pl.tiles_w * pl.tiles_h
+                                    : (g.M + kPBM - 1) / kPBM;
+  const int64_t tiles = mt * ((g.N + BN - 1) / BN);
   const int sms = g.num_sms > 0 ? g.num_sms : 148;
   cudaLaunchConfig_t cfg;
   std::memset(&cfg, 0, sizeof(cfg));
   cfg.gridDim = dim3((unsigned)std::min<int64_t>(tiles, sms));
-  cfg.blockDim = dim3(persist_threads<GATHER>());
+  cfg.blockDim = dim3(persist_threads<AMODE>());
   cfg.dynamicSmemBytes = PCfg<BN>::kSmem;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
@@ -329,13 +369,19 @@ int launch_persist_inst(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_
   return SWAPNET_OK;
 }
 
+template <typename T, int BN>
+int launch_persist_bn(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) {
+  if (!g.conv) return launch_persist_inst<T, BN, kAT2d>(g, pl, err, s);
+  if (pl.tma_conv) return launch_persist_inst<T, BN, kATap>(g, pl, err, s);
+  return launch_persist_inst<T, BN, kAGather>(g, pl, err, s);
+}
+
 template <typename T>
 int launch_persist_t(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) {
-  const bool ga = g.conv != 0;
   switch (pl.bn) {
-    case 64: return ga ? launch_persist_inst<T, 64, true>(g, pl, err, s) : launch_persist_inst<T, 64, false>(g, pl, err, s);
-    case 128: return ga ? launch_persist_inst<T, 128, true>(g, pl, err, s) : launch_persist_inst<T, 128, false>(g, pl, err, s);
-    case 256: return ga ? launch_persist_inst<T, 256, true>(g, pl, err, s) : launch_persist_inst<T, 256, false>(g, pl, err, s);
+    case 64: return launch_persist_bn<T, 64>(g, pl, err, s);
+    case 128: return launch_persist_bn<T, 128>(g, pl, err, s);
+    case 256: return launch_persist_bn<T, 256>(g, pl, err, s);
     default: SN_FAIL(SWAPNET_ERR_INVALID_ARG, "persistent GEMM: bad N tile");
   }
 }

@@ -96,6 +96,8 @@ struct TcPlan {
   int64_t tiles;    // output tiles (split-K counters needed)
   uint64_t scratch_bytes;  // fp32 partials of all splits
   int persist;      // persistent kernel (one CTA per SM looping over tiles)
+  int tma_conv;     // convolution A by 4-D TMA per filter tap (tmA is then 4-D)
+  int wt, ht, tiles_w, tiles_h;  // its output patch and patch counts per image
   int ready;
 };
 int tc_prepare(const TcGemm& g, TcPlan* p);

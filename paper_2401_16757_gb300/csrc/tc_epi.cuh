@@ -19,6 +19,9 @@ struct TcArgs {
   float* partial;    // [splits][M][N] fp32 partial sums (global split-K only)
   int* counters;     // per output tile, zero between launches (global split-K only)
   int cluster;       // 1: the splits of a tile form a cluster and reduce through DSMEM
+  // TMA im2col (persistent kernel): output tiles are wt x ht pixel patches of
+  // one image, tiles_w x tiles_h of them per image; rows >= wt * ht are unused
+  int wt, ht, tiles_w, tiles_h;
 };
 
 // ---- register-only epilogue helpers
