@@ -344,6 +344,19 @@ typedef enum swapnet_kernel_kind {
 } swapnet_kernel_kind;
 int swapnet_engine_unit_kernels(const swapnet_engine* eng, int32_t* kinds, uint32_t cap, uint32_t* n);
 
+/* How each tensor-core unit is tiled (introspection for measurement; the
+ * paper has no counterpart).  For unit i, tiling[i] gets: n_tile (N columns
+ * per output tile), splits (K splits; 1 = none), cluster (1: the splits of a
+ * tile reduce through a thread-block cluster), persistent (1: one CTA per SM
+ * loops over the tiles), tap_tma (1: convolution A loaded by one 4-D TMA per
+ * filter tap).  Units off the tensor cores get all zeros.  Same count
+ * protocol as swapnet_engine_unit_kernels. */
+typedef struct swapnet_unit_tiling {
+  int32_t n_tile, splits, cluster, persistent, tap_tma, reserved[3];
+} swapnet_unit_tiling;
+int swapnet_engine_unit_tiling(const swapnet_engine* eng, swapnet_unit_tiling* tiling, uint32_t cap,
+                               uint32_t* n);
+
 /* Device timing for measurement: while enabled, every swapnet_infer records
  * a CUDA event pair around each unit's kernel (on the inference stream) and
  * around each block's swap-in (on the copy stream).  The events add a small

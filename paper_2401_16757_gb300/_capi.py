@@ -79,6 +79,11 @@ KERNEL_KIND = {1: "tc_gemm", 2: "tc_conv", 3: "skinny_linear", 4: "direct_conv",
                13: "argmax", 14: "tc_conv_small"}
 
 
+class UnitTiling(C.Structure):
+    _fields_ = [("n_tile", C.c_int32), ("splits", C.c_int32), ("cluster", C.c_int32), ("persistent", C.c_int32),
+                ("tap_tma", C.c_int32), ("reserved", C.c_int32 * 3)]
+
+
 class EngineBlock(C.Structure):
     _fields_ = [("variant", C.c_int32), ("n_segments", C.c_int32), ("memcpy_us", C.c_float),
                 ("zerocopy_us", C.c_float)]
@@ -88,7 +93,7 @@ EXPORTS = ["swapnet_default_options", "swapnet_partition", "swapnet_plan_from_cu
            "swapnet_plan_info_get", "swapnet_plan_cuts", "swapnet_plan_units", "swapnet_plan_blocks",
            "swapnet_plan_output_offsets", "swapnet_plan_free", "swapnet_schedule", "swapnet_load",
            "swapnet_infer", "swapnet_infer_host", "swapnet_engine_sync", "swapnet_engine_blocks",
-           "swapnet_engine_free", "swapnet_engine_stats_get", "swapnet_engine_unit_kernels",
+           "swapnet_engine_free", "swapnet_engine_stats_get", "swapnet_engine_unit_kernels", "swapnet_engine_unit_tiling",
            "swapnet_engine_set_profiling", "swapnet_engine_last_times", "swapnet_engine_measure_units",
            "swapnet_engine_last_timeline",
            "swapnet_engine_bind_state", "swapnet_strerror", "swapnet_last_error", "swapnet_debug_fail_next", "swapnet_gemm_noalloc"]
@@ -136,6 +141,7 @@ def lib():
         "swapnet_engine_free": (None, [P]),
         "swapnet_engine_stats_get": (C.c_int, [P, C.POINTER(EngineStats)]),
         "swapnet_engine_unit_kernels": (C.c_int, [P, C.POINTER(C.c_int32), C.c_uint32, C.POINTER(C.c_uint32)]),
+        "swapnet_engine_unit_tiling": (C.c_int, [P, C.POINTER(UnitTiling), C.c_uint32, C.POINTER(C.c_uint32)]),
         "swapnet_engine_set_profiling": (C.c_int, [P, C.c_int]),
         "swapnet_engine_measure_units": (C.c_int, [P, C.c_int32, C.POINTER(C.c_float), C.c_uint32]),
         "swapnet_engine_last_timeline": (C.c_int, [P, C.POINTER(C.c_float), C.POINTER(C.c_float), C.c_uint32,
@@ -431,6 +437,13 @@ class Engine:
         arr = (C.c_int32 * max(1, n.value))()
         check(lib().swapnet_engine_unit_kernels(self.h, arr, n.value, None), "swapnet_engine_unit_kernels")
         return [KERNEL_KIND.get(k, str(k)) for k in arr[:n.value]]
+
+    def unit_tiling(self):
+        n = C.c_uint32()
+        check(lib().swapnet_engine_unit_tiling(self.h, None, 0, C.byref(n)), "swapnet_engine_unit_tiling")
+        arr = (UnitTiling * max(1, n.value))()
+        check(lib().swapnet_engine_unit_tiling(self.h, arr, n.value, None), "swapnet_engine_unit_tiling")
+        return [{f: getattr(u, f) for f, _ in UnitTiling._fields_ if f != "reserved"} for u in arr[:n.value]]
 
     def set_profiling(self, enable):
         check(lib().swapnet_engine_set_profiling(self.h, 1 if enable else 0), "swapnet_engine_set_profiling")

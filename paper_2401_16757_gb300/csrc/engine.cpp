@@ -417,6 +417,10 @@ static int prepare_units(swapnet_engine* e) {
         if (U.nt == 2) X.b = base + U.slot_off[1];
       }
       const Layer& L = m.L[U.layer];
+      if (small_conv_ok(m, L)) {
+        int rc = tc_small_prepare(m.dtype, L.d.kh * L.d.kw * L.d.cin);
+        if (rc) return rc;
+      }
       if (!wants_tc(m, L)) continue;
       X.use_tc = true;
       // A pointers in the workspace are fixed; the model input and outputs
@@ -856,6 +860,25 @@ int swapnet_engine_unit_kernels(const swapnet_engine* e, int32_t* kinds, uint32_
   if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
   if (n) *n = (uint32_t)e->unit_kind.size();
   for (uint32_t i = 0; kinds && i < cap && i < e->unit_kind.size(); ++i) kinds[i] = e->unit_kind[i];
+  return SWAPNET_OK;
+}
+
+int swapnet_engine_unit_tiling(const swapnet_engine* e, swapnet_unit_tiling* t, uint32_t cap, uint32_t* n) {
+  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+  if (n) *n = (uint32_t)e->ux.size();
+  for (uint32_t i = 0; t && i < cap && i < e->ux.size(); ++i) {
+    const UnitExec& X = e->ux[i];
+    swapnet_unit_tiling r;
+    std::memset(&r, 0, sizeof(r));
+    if (X.use_tc) {
+      r.n_tile = X.tc.bn;
+      r.splits = X.tc.splits;
+      r.cluster = X.tc.splits > 1 && X.tc.cluster;
+      r.persistent = X.tc.persist;
+      r.tap_tma = X.tc.tma_conv;
+    }
+    t[i] = r;
+  }
   return SWAPNET_OK;
 }
 

@@ -551,15 +551,17 @@ int tc_prepare(const TcGemm& g, TcPlan* p) {
   const int Nd = g.N_layer > 0 ? g.N_layer : g.N;  // decisions follow the whole layer
   const int64_t mtiles = (g.M + kBM - 1) / kBM;
   if (g.allow_persist) {
-    // at least one output tile per SM: the persistent kernel, no split
-    const int pbn = Nd <= 64 ? 64 : (Nd <= 128 ? 128 : 256);
-    // convolutions whose taps are whole 64-channel k-blocks load A by 4-D TMA
-    // when a pixel patch fills the 128 MMA rows well enough
+    // at least one output tile per SM: the persistent kernel, no split.
+    // Convolutions whose taps are whole 64-channel k-blocks load A by 4-D TMA
+    // when a pixel patch fills the 128 MMA rows well enough.
     int wt = 0, ht = 0;
-    const bool tmac = g.conv && g.C % kBK == 0 && conv_patch(g.Ho, g.Wo, g.stride, &wt, &ht) >= 0.85;
+    const bool tmac = g.conv && g.C % kBK == 0 && conv_patch(g.Ho, g.Wo, g.stride, &wt, &ht) >= 0.75;
     const int64_t sp_tiles = tmac ? (int64_t)g.M / ((int64_t)g.Ho * g.Wo) * ((g.Wo + wt - 1) / wt) *
                                         ((g.Ho + ht - 1) / ht)
                                   : mtiles;
+    // widest useful N tile; convolutions narrow it until every SM has a tile
+    int pbn = Nd <= 64 ? 64 : (Nd <= 128 ? 128 : 256);
+    while (g.conv && pbn > 64 && sp_tiles * ((Nd + pbn - 1) / pbn) < sms) pbn /= 2;
     if (sp_tiles * ((Nd + pbn - 1) / pbn) >= sms) {
       p->persist = 1;
       if (tmac) {

@@ -109,7 +109,7 @@ __device__ __forceinline__ void small_epilogue(const SmallArgs& p, uint32_t tmem
 }
 
 template <typename T>
-__global__ void __launch_bounds__(kSmThreads) tc_conv_small_kernel(const SmallArgs p) {
+__global__ void __launch_bounds__(kSmThreads, 4) tc_conv_small_kernel(const SmallArgs p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int nkb = p.nkb;
@@ -201,19 +201,23 @@ __global__ void __launch_bounds__(kSmThreads) tc_conv_small_kernel(const SmallAr
     const T* xw = X + (((int64_t)img * p.H + iy0) * p.Wd + ix0) * p.C;
     const uint32_t abase = smem_u32(sA + buf * nkb * kSmATile) + row_off;
     for (int kb = 0; kb < nkb; ++kb) {
-      T e[64];
+      uint32_t e2[32];  // packed pairs: 64 independent loads in flight
 #pragma unroll
-      for (int h = 0; h < 64; ++h) {  // 64 independent loads in flight
-        const int2 t = tab[kb * 64 + h];
-        const int iy = iy0 + (t.y >> 16), ix = ix0 + (t.y & 0xffff);
-        const bool valid = mv && (unsigned)iy < (unsigned)p.H && (unsigned)ix < (unsigned)p.Wd;
-        e[h] = valid ? __ldg(xw + t.x) : zero;
+      for (int h = 0; h < 64; h += 2) {
+        T e[2];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const int2 t = tab[kb * 64 + h + u];
+          const int iy = iy0 + (t.y >> 16), ix = ix0 + (t.y & 0xffff);
+          const bool valid = mv && (unsigned)iy < (unsigned)p.H && (unsigned)ix < (unsigned)p.Wd;
+          e[u] = valid ? __ldg(xw + t.x) : zero;
+        }
+        e2[h >> 1] = bits2<T>(e[0], e[1]);
       }
 #pragma unroll
       for (int j = 0; j < 8; ++j)
         st_shared_v4(abase + kb * kSmATile + (((uint32_t)j ^ sw) << 4),
-                     make_uint4(bits2<T>(e[8 * j], e[8 * j + 1]), bits2<T>(e[8 * j + 2], e[8 * j + 3]),
-                                bits2<T>(e[8 * j + 4], e[8 * j + 5]), bits2<T>(e[8 * j + 6], e[8 * j + 7])));
+                     make_uint4(e2[4 * j], e2[4 * j + 1], e2[4 * j + 2], e2[4 * j + 3]));
     }
     fence_proxy_async_smem();
     tc_fence_before();
@@ -260,25 +264,52 @@ __global__ void __launch_bounds__(kSmThreads) tc_conv_small_kernel(const SmallAr
   }
 }
 
+// CTAs per SM for a given k-block count, per element type; computed outside
+// stream capture (tc_small_prepare), where the occupancy query is allowed.
+template <typename T>
+int& small_occ(int nkb) {
+  static int occ[kSmMaxKB + 1] = {0, 0, 0, 0};
+  return occ[nkb];
+}
+
+template <typename T>
+int small_prepare_t(int nkb) {
+  auto kern = tc_conv_small_kernel<T>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, small_smem_bytes(kSmMaxKB)) !=
+      cudaSuccess)
+    SN_FAIL(SWAPNET_ERR_CUDA, "cudaFuncSetAttribute failed");
+  // several CTAs share an SM: ask for the whole carveout as shared memory
+  // (without a preference the occupancy query assumes room for one CTA)
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared) !=
+      cudaSuccess)
+    cudaGetLastError();
+  // CTAs per SM from the kernel's registers and shared memory
+  cudaFuncAttributes fa;
+  int dev = 0, regs_sm = 0, smem_sm = 0, reserved = 0, blocks_sm = 0;
+  if (cudaFuncGetAttributes(&fa, kern) != cudaSuccess || cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&regs_sm, cudaDevAttrMaxRegistersPerMultiprocessor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&blocks_sm, cudaDevAttrMaxBlocksPerMultiprocessor, dev) != cudaSuccess)
+    SN_FAIL(SWAPNET_ERR_CUDA, "small-channel conv: kernel attributes unavailable");
+  const int warp_regs = (fa.numRegs * 32 + 255) / 256 * 256;
+  const int by_regs = regs_sm / std::max(1, warp_regs * (kSmThreads / 32));
+  const int by_smem = smem_sm / std::max(1, small_smem_bytes(nkb) + (int)fa.sharedSizeBytes + reserved);
+  const int n = std::min(std::min(by_regs, by_smem), blocks_sm);
+  small_occ<T>(nkb) = std::max(1, std::min(n, 512 / (2 * kSmBN)));  // TMEM: 128 columns per CTA
+  return SWAPNET_OK;
+}
+
 template <typename T>
 int launch_small(const TcSmallConv& g, int* err, cudaStream_t s) {
-  static int occ = -1;  // CTAs per SM (per instantiation; the smem size depends on nkb)
-  static int occ_nkb = -1;
   auto kern = tc_conv_small_kernel<T>;
   const int nkb = (g.K + 63) / 64;
   const int smem = small_smem_bytes(nkb);
-  if (occ < 0 || occ_nkb != nkb) {
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, small_smem_bytes(kSmMaxKB)) !=
-        cudaSuccess)
-      SN_FAIL(SWAPNET_ERR_CUDA, "cudaFuncSetAttribute failed");
-    int n = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kern, kSmThreads, smem) != cudaSuccess) {
-      cudaGetLastError();
-      n = 1;
-    }
-    occ = std::max(1, std::min(n, 512 / (2 * kSmBN)));  // TMEM: 128 columns per CTA
-    occ_nkb = nkb;
+  if (small_occ<T>(nkb) == 0) {
+    const int rc = small_prepare_t<T>(nkb);
+    if (rc) return rc;
   }
+  const int occ = small_occ<T>(nkb);
   SmallArgs a;
   std::memset(&a, 0, sizeof(a));
   a.x = g.x; a.w = g.W;
@@ -310,6 +341,12 @@ int launch_small(const TcSmallConv& g, int* err, cudaStream_t s) {
 
 bool tc_small_supported(int dtype, int K) {
   return (dtype == SWAPNET_F16 || dtype == SWAPNET_BF16) && K >= 1 && K <= 64 * kSmMaxKB;
+}
+
+int tc_small_prepare(int dtype, int K) {
+  if (!tc_small_supported(dtype, K)) SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "small-channel conv: K out of range");
+  const int nkb = (K + 63) / 64;
+  return dtype == SWAPNET_BF16 ? small_prepare_t<__nv_bfloat16>(nkb) : small_prepare_t<__half>(nkb);
 }
 
 int launch_tc_conv_small(const TcSmallConv& g, int* err, cudaStream_t s) {

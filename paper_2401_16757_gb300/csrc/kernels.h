@@ -119,6 +119,7 @@ struct TcSmallConv {
   int num_sms;
 };
 bool tc_small_supported(int dtype, int K);
+int tc_small_prepare(int dtype, int K);  // once per shape class, outside stream capture
 int launch_tc_conv_small(const TcSmallConv& g, int* dev_err, cudaStream_t s);
 
 // Device error word of the tcgen05 kernels (bounded waits).
