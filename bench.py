@@ -57,16 +57,16 @@ CONFIGS = {
 # + dram__bytes_write.sum averaged over the launches of one swapped step of
 # the named workload), valid only for the kernel sources it was taken on.
 TRAFFIC = {
-    # (workload, kernel family): (sha1 prefix of the kernel sources, bytes per launch)
-    ("resnet50", "tc_gemm"): ("2b29561bcde9", 1419277),
-    ("resnet50", "tc_conv"): ("2b29561bcde9", 1804400),
+    ("resnet50", "tc_gemm"): ("672713681337", 1424281),
+    ("resnet50", "tc_conv"): ("672713681337", 1807171),
 }
 
 
 def kernel_sources_sha():
     import hashlib
     h = hashlib.sha1()
-    for f in ("k_tc.cu", "k_simt.cu", "device.cuh"):
+    for f in ("k_tc.cu", "k_tc_persist.cu", "k_tc_small.cu", "tc_epi.cuh", "k_simt.cu", "k_decoder.cu",
+              "device.cuh"):
         with open(os.path.join(ROOT, "paper_2401_16757_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:12]
@@ -459,6 +459,24 @@ def measure_link_peak(stream):
     return (256 << 20) / (best / 1000.0) / 1e9
 
 
+def run_profile_once(args):
+    """One resident inference of a single-model config (no timing)."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2401_16757_gb300 import capi
+    m, w, x, wb, budget, text = build_workload(args.config, capi_weight_bytes)
+    plan = capi.Plan.resident(capi.Desc(m))
+    info = plan.info()
+    eng = capi.Engine(plan, capi.HostWeights(w))
+    d_in = torch.empty(max(16, info["input_bytes"]), dtype=torch.uint8, device="cuda")
+    d_in[:info["input_bytes"]].copy_(torch.from_numpy(x.view(np.uint8).reshape(-1)))
+    d_out = torch.empty(info["output_bytes"], dtype=torch.uint8, device="cuda")
+    eng.infer(d_in.data_ptr(), d_out.data_ptr(), torch.cuda.current_stream().cuda_stream)
+    eng.sync()
+    print(json.dumps({"profile_once": args.config, "kernels": eng.unit_kernels(), "tiling": eng.unit_tiling()}))
+
+
 def run_reference(args, rank, world):
     """The reference arm: the CPU oracle, timed as it stands on the host cores."""
     if rank != 0:
@@ -539,6 +557,9 @@ def main():
     ap.add_argument("--config", default="resnet50", choices=sorted(CONFIGS))
     ap.add_argument("--variant", default="auto", choices=["auto", "memcpy", "zerocopy"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile-once", action="store_true",
+                    help="run one resident inference of --config through the C ABI and exit "
+                         "(a driver for profiler captures of its kernels); prints one JSON line")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -547,6 +568,9 @@ def main():
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
         run_reference(args, rank, world)
+        return
+    if args.profile_once:
+        run_profile_once(args)
         return
     if args.config in ("llm", "multi"):
         import torch
