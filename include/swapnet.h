@@ -149,7 +149,14 @@ typedef struct swapnet_options {
   int32_t preloaded;             /* resident plans only: the caller's arena already
                                     holds this layout (loaded by another engine of
                                     the same layers); swapnet_load skips the upload */
-  int32_t reserved[5];
+  int32_t branches;              /* 1 (default): a conv / linear layer whose inputs
+                                     were all produced before the previous layer runs
+                                     on a second stream beside the layers in between
+                                     (e.g. a ResNet projection shortcut), when it, its
+                                     last producer and its consumers share a block;
+                                     0: every layer in order on one stream.  Results
+                                     are identical either way. */
+  int32_t reserved[4];
 } swapnet_options;
 
 /* Fills the defaults: 2 slots, activations outside the budget, AUTO swap,

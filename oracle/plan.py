@@ -127,8 +127,11 @@ def layer_flops(model, li, shapes):
 def workspace(model):
     """Liveness-based placement of intermediate activations.
 
-    A non-output layer output lives over [i, last reader] (inclusive).  In
-    layer order each one takes the lowest 256-byte-aligned offset where it
+    A non-output layer output lives over [start, last reader] (inclusive),
+    start = i, except for a conv / linear layer whose producers all come
+    before i - 1: it may be computed beside the layers between its last
+    producer and itself, so it lives from one step after that producer.  In
+    layer order each output takes the lowest 256-byte-aligned offset where it
     overlaps no placed tensor whose live interval meets its own.  The lowest
     such offset is 0 or the end of one of those tensors (if an offset o > 0
     fits and o - 256 does not, some conflicting tensor ends in (o-256, o],
@@ -140,12 +143,13 @@ def workspace(model):
     shapes = out_shapes(model)
     es = ES[model["dtype"]]
     nl = len(model["layers"])
-    last = list(range(nl))
+    last, start = list(range(nl)), list(range(nl))
     for j, L in enumerate(model["layers"]):
-        refs = list(L["src"]) + ([L["res"]] if L.get("res") is not None else [])
+        refs = [i for i in list(L["src"]) + ([L["res"]] if L.get("res") is not None else []) if i >= 0]
         for i in refs:
-            if i >= 0:
-                last[i] = max(last[i], j)
+            last[i] = max(last[i], j)
+        if L["op"] in ("conv", "linear") and refs and max(refs) + 1 < j:
+            start[j] = max(refs) + 1
     outs = sorted(model["outputs"])
     placed = []  # (lo, hi, off, size)
     offs = {}
@@ -153,13 +157,13 @@ def workspace(model):
         if i in outs:
             continue
         size = align(math.prod(shapes[i]) * out_elem_bytes(model, i))
-        conflict = [p for p in placed if p[0] <= last[i] and i <= p[1]]
+        conflict = [p for p in placed if p[0] <= last[i] and start[i] <= p[1]]
         cands = sorted({0} | {p[2] + p[3] for p in conflict})
         for o in cands:
             if all(o + size <= p[2] or p[2] + p[3] <= o for p in conflict):
                 break
         offs[i] = o
-        placed.append((i, last[i], o, size))
+        placed.append((start[i], last[i], o, size))
     ws = max([p[2] + p[3] for p in placed], default=0)
     out_off, cur = {}, 0
     for i in outs:

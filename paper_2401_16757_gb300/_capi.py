@@ -46,7 +46,8 @@ class Options(C.Structure):
     _fields_ = [("slots", C.c_int32), ("activations_in_budget", C.c_int32), ("swap_variant", C.c_int32),
                 ("objective", C.c_int32), ("alpha_as_per_byte", C.c_uint64), ("beta_ns_per_tensor", C.c_uint64),
                 ("gamma_as_per_flop", C.c_uint64), ("eta_ns_per_tensor", C.c_uint64), ("zc_ctas", C.c_int32),
-                ("graphs", C.c_int32), ("preloaded", C.c_int32), ("reserved", C.c_int32 * 5)]
+                ("graphs", C.c_int32), ("preloaded", C.c_int32), ("branches", C.c_int32),
+                ("reserved", C.c_int32 * 4)]
 
 
 class PlanInfo(C.Structure):

@@ -112,6 +112,14 @@ struct swapnet_engine {
   // per (input, output, profiling) binding
   std::map<std::pair<std::pair<const void*, void*>, bool>, cudaGraphExec_t> graphs;
   char* d_state = nullptr;           // decoder state (position + KV caches), caller-owned
+  // concurrent branches: side units run on `side`, forked after their last
+  // producer's unit and joined before their first consumer's
+  cudaStream_t side = nullptr;
+  cudaEvent_t side_fork = nullptr;
+  std::vector<cudaEvent_t> side_done;        // per unit (side units only)
+  std::vector<std::vector<int>> side_after;  // per unit: side units forked after it
+  std::vector<std::vector<int>> side_wait;   // per unit: side units it waits for
+  std::vector<char> is_side;
   char* d_splitk = nullptr;          // split-K scratch: tile counters, then fp32 partials
   uint64_t splitk_bytes = 0;
   uint64_t splitk_counter_bytes = 0;
@@ -126,6 +134,11 @@ static int release(swapnet_engine* e) {
   for (cudaEvent_t ev : {e->slot_free[0], e->slot_free[1], e->ready[0], e->ready[1]})
     if (ev) cudaEventDestroy(ev);
   for (auto& kv : e->graphs) cudaGraphExecDestroy(kv.second);
+  if (e->side) cudaStreamSynchronize(e->side);
+  for (cudaEvent_t ev : e->side_done)
+    if (ev) cudaEventDestroy(ev);
+  if (e->side_fork) cudaEventDestroy(e->side_fork);
+  if (e->side) cudaStreamDestroy(e->side);
   if (e->fork) cudaEventDestroy(e->fork);
   if (e->join) cudaEventDestroy(e->join);
   if (e->cap) cudaStreamDestroy(e->cap);
@@ -376,6 +389,8 @@ static bool small_conv_ok(const Model& m, const Layer& L) {
          tc_small_supported(m.dtype, L.d.kh * L.d.kw * L.d.cin);
 }
 
+static int plan_side(swapnet_engine* e);
+
 static int prepare_units(swapnet_engine* e) {
   const swapnet_plan& p = e->plan;
   const Model& m = p.model;
@@ -584,6 +599,8 @@ int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint
   build_segments(e);
   rc = prepare_units(e);
   if (rc) return rc;
+  rc = plan_side(e);
+  if (rc) return rc;
   {
     uint64_t part = 0;
     int64_t tiles = 0;
@@ -636,6 +653,63 @@ namespace swapnet {
 // waits for the block that last used it in this inference, and the copy
 // stream joins `s` again at the end.  The same sequence is captured as a
 // graph, where the fork, the slot gating and the join become graph edges.
+// Units that may run on the side stream: a whole-layer conv / linear unit
+// whose layer may start early (Layer::start < layer), whose last producer's
+// unit is on the main stream in the same block, and whose consumers are all
+// in that block (they wait for it; the block's slot is released after them).
+static int plan_side(swapnet_engine* e) {
+  const swapnet_plan& p = e->plan;
+  const Model& m = p.model;
+  const int n = (int)p.units.size(), nl = (int)m.L.size();
+  e->is_side.assign(n, 0);
+  e->side_after.assign(n, {});
+  e->side_wait.assign(n, {});
+  e->side_done.assign(n, nullptr);
+  if (!p.opt.branches) return SWAPNET_OK;
+  std::vector<int> lfirst(nl, -1), llast(nl, -1), ublock(n, -1);
+  for (size_t b = 0; b < p.blocks.size(); ++b)
+    for (int u = p.blocks[b].u0; u < p.blocks[b].u1; ++u) ublock[u] = (int)b;
+  for (int u = 0; u < n; ++u) {
+    const int l = p.units[u].layer;
+    if (lfirst[l] < 0) lfirst[l] = u;
+    llast[l] = u;
+  }
+  auto reads = [&](const Layer& L, int l) {
+    const swapnet_layer& d = L.d;
+    return d.src0 == l || d.src1 == l || d.res == l || (d.op == SWAPNET_OP_ATTENTION && d.src2 == l);
+  };
+  for (int u = 0; u < n; ++u) {
+    const Unit& U = p.units[u];
+    const Layer& L = m.L[U.layer];
+    if (L.start >= U.layer || U.host || lfirst[U.layer] != u || llast[U.layer] != u) continue;
+    const UnitExec& X = e->ux[u];
+    if (X.use_tc && X.tc.splits > 1 && !X.tc.cluster) continue;  // global split-K scratch is shared
+    const int du = llast[L.start - 1];
+    if (du < 0 || ublock[du] != ublock[u] || e->is_side[du]) continue;
+    bool ok = true;
+    for (int s : {L.d.src0, L.d.src1, L.d.res})
+      if (s >= 0 && e->is_side[llast[s]]) ok = false;
+    std::vector<int> cons;
+    for (int v = u + 1; v < n && ok; ++v)
+      if (reads(m.L[p.units[v].layer], U.layer)) {
+        if (ublock[v] != ublock[u] || e->is_side[v]) ok = false;
+        cons.push_back(v);
+      }
+    if (!ok || cons.empty()) continue;
+    e->is_side[u] = 1;
+    e->side_after[du].push_back(u);
+    for (int v : cons) e->side_wait[v].push_back(u);
+    CU(cudaEventCreateWithFlags(&e->side_done[u], cudaEventDisableTiming), "event");
+  }
+  if (!e->side) {
+    int lo = 0, hi = 0;
+    CU(cudaDeviceGetStreamPriorityRange(&lo, &hi), "stream priority range");
+    CU(cudaStreamCreateWithPriority(&e->side, cudaStreamNonBlocking, lo), "side stream");
+    CU(cudaEventCreateWithFlags(&e->side_fork, cudaEventDisableTiming), "event");
+  }
+  return SWAPNET_OK;
+}
+
 static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t s, bool capturing = false) {
   const swapnet_plan& p = e->plan;
   const bool prof = e->profiling && !capturing;
@@ -657,10 +731,21 @@ static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t 
       CU(cudaStreamWaitEvent(s, e->ready[B.slot], 0), "wait ready");
     }
     for (int u = B.u0; u < B.u1; ++u) {
+      if (e->is_side[u]) continue;  // launched on the side stream after its producer
+      for (int w : e->side_wait[u]) CU(cudaStreamWaitEvent(s, e->side_done[w], 0), "wait side");
       if (prof) CU(cudaEventRecord(e->ev_unit[2 * u], s), "profile event");
       int rc = run_unit(e, u, din, dout, s);
       if (rc) return rc;
       if (prof) CU(cudaEventRecord(e->ev_unit[2 * u + 1], s), "profile event");
+      for (int w : e->side_after[u]) {
+        CU(cudaEventRecord(e->side_fork, s), "record side fork");
+        CU(cudaStreamWaitEvent(e->side, e->side_fork, 0), "wait side fork");
+        if (prof) CU(cudaEventRecord(e->ev_unit[2 * w], e->side), "profile event");
+        rc = run_unit(e, w, din, dout, e->side);
+        if (rc) return rc;
+        if (prof) CU(cudaEventRecord(e->ev_unit[2 * w + 1], e->side), "profile event");
+        CU(cudaEventRecord(e->side_done[w], e->side), "record side done");
+      }
     }
     if (!p.resident) CU(cudaEventRecord(e->slot_free[B.slot], s), "record slot free");
   }

@@ -39,6 +39,10 @@ struct Layer {
   int first_tensor;      // global index of the first parameter tensor
   uint64_t flops;
   int last_use;          // last layer reading this output (inclusive)
+  int start;             // first layer step at which this output may be written:
+                         // i, or (conv / linear whose producers all precede
+                         // i - 1) one step after its last producer, so the
+                         // engine may run it beside the layers in between
   int64_t ws_off;        // workspace offset, -1 when the output is a model output
   int64_t out_off;       // offset in the output buffer, -1 if not an output
   uint64_t out_bytes;    // raw bytes of the output tensor

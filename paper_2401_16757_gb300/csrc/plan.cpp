@@ -188,8 +188,15 @@ int analyse_model(const swapnet_model_desc* desc, Model* m) {
   for (int i = 0; i < nl; ++i) m->L[i].last_use = i;
   for (int j = 0; j < nl; ++j) {
     const swapnet_layer& d = m->L[j].d;
+    int last_producer = -1;
     for (int s : {d.src0, d.src1, d.res, d.op == SWAPNET_OP_ATTENTION ? d.src2 : -1})
-      if (s >= 0) m->L[s].last_use = std::max(m->L[s].last_use, j);
+      if (s >= 0) {
+        m->L[s].last_use = std::max(m->L[s].last_use, j);
+        last_producer = std::max(last_producer, s);
+      }
+    m->L[j].start = j;
+    const bool weighted = d.op == SWAPNET_OP_CONV2D || d.op == SWAPNET_OP_LINEAR;
+    if (weighted && last_producer >= 0 && last_producer + 1 < j) m->L[j].start = last_producer + 1;
   }
   // outputs go to the output buffer, in layer order
   uint64_t cur = 0;
@@ -211,7 +218,7 @@ int analyse_model(const swapnet_model_desc* desc, Model* m) {
     const uint64_t size = align_up(L.out_bytes);
     std::vector<const Placed*> conf;
     for (const Placed& p : placed)
-      if (p.lo <= L.last_use && i <= p.hi) conf.push_back(&p);
+      if (p.lo <= L.last_use && L.start <= p.hi) conf.push_back(&p);
     std::vector<uint64_t> cand{0};
     for (const Placed* p : conf) cand.push_back(p->off + p->size);
     std::sort(cand.begin(), cand.end());
@@ -223,7 +230,7 @@ int analyse_model(const swapnet_model_desc* desc, Model* m) {
       if (ok) { chosen = o; break; }
     }
     L.ws_off = (int64_t)chosen;
-    placed.push_back(Placed{i, L.last_use, chosen, size});
+    placed.push_back(Placed{L.start, L.last_use, chosen, size});
     ws = std::max(ws, chosen + size);
   }
   m->ws_bytes = ws;
@@ -612,6 +619,7 @@ static int check_options(const swapnet_options& o) {
   if (o.zc_ctas < 0 || o.zc_ctas > 4096) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad zc_ctas");
   if (o.graphs != 0 && o.graphs != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "graphs must be 0 or 1");
   if (o.preloaded != 0 && o.preloaded != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "preloaded must be 0 or 1");
+  if (o.branches != 0 && o.branches != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "branches must be 0 or 1");
   return SWAPNET_OK;
 }
 
@@ -656,6 +664,7 @@ void swapnet_default_options(swapnet_options* o) {
   o->eta_ns_per_tensor = 0;
   o->zc_ctas = 0;
   o->graphs = 1;
+  o->branches = 1;
 }
 
 int swapnet_partition(const swapnet_model_desc* desc, uint64_t budget, const swapnet_options* opt,

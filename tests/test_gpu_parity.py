@@ -279,3 +279,21 @@ def test_multi_dnn_schedule_concurrent():
         r.engine.sync()
         got = r.outputs_raw()
         assert all(a.tobytes() == b.tobytes() for a, b in zip(got, ref))
+
+
+@pytest.mark.parametrize("name", ["resnet50", "yolov3"])
+def test_concurrent_branches_bit_exact(name):
+    """Layers run beside their neighbours on the second stream (projection
+    shortcuts, detection-head branches) give the same bits as strictly
+    sequential execution, resident and swapped."""
+    m = synth.arch.MODELS[name]()
+    w = synth.gen.model_weights(m)
+    x = synth.gen.model_input(m)
+    d = capi.Desc(m)
+    host = capi.HostWeights(w)
+    seq = Runner(m, w, capi.Plan.resident(d, capi.options(branches=0)), host).run(x)
+    par = Runner(m, w, capi.Plan.resident(d, capi.options(branches=1)), host).run(x)
+    budget = int(OP.weight_bytes(m) * 0.4) // 256 * 256
+    sw = Runner(m, w, capi.Plan.partition(d, budget, capi.options(branches=1)), host).run(x)
+    for a, b, c in zip(seq, par, sw):
+        assert a.tobytes() == b.tobytes() == c.tobytes()

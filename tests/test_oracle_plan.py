@@ -132,20 +132,23 @@ def test_workspace_no_live_overlap_and_first_fit(name):
     es = P.ES[m["dtype"]]
     nl = len(m["layers"])
     last = list(range(nl))
+    first = list(range(nl))   # earliest step a layer may run: after its last producer
     for j, L in enumerate(m["layers"]):
-        for i in list(L["src"]) + ([L["res"]] if L.get("res") is not None else []):
-            if i >= 0:
-                last[i] = max(last[i], j)
+        refs = [i for i in list(L["src"]) + ([L["res"]] if L.get("res") is not None else []) if i >= 0]
+        for i in refs:
+            last[i] = max(last[i], j)
+        if L["op"] in ("conv", "linear") and refs:
+            first[j] = min(j, max(refs) + 1)
     size = {i: P.align(int(np.prod(shapes[i])) * es) for i in offs}
     items = sorted(offs)
     for a, b in itertools.combinations(items, 2):
-        live = a <= last[b] and b <= last[a]
+        live = first[a] <= last[b] and first[b] <= last[a]
         if live:
             assert offs[a] + size[a] <= offs[b] or offs[b] + size[b] <= offs[a]
     assert ws == max(offs[i] + size[i] for i in items)
     # first fit: no lower aligned offset was free when the tensor was placed
     for i in items:
-        earlier = [j for j in items if j < i and j <= last[i] and i <= last[j]]
+        earlier = [j for j in items if j < i and first[j] <= last[i] and first[i] <= last[j]]
         for o in range(0, offs[i], 256 * max(1, offs[i] // 256 // 64)):
             clash = any(not (o + size[i] <= offs[j] or offs[j] + size[j] <= o) for j in earlier)
             assert clash
