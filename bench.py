@@ -359,7 +359,9 @@ def run_multi(args, rank, world):
     ms = [synth.arch.MODELS[n]() for n in names]
     stream0 = torch.cuda.current_stream()
     link_peak = measure_link_peak(stream0)
-    alpha = int(round(1e18 / (link_peak * 1e9)))
+    # the three pipelines share one host link: each model's delay model takes
+    # its share of the measured bandwidth (--link-share 1 plans as if alone)
+    alpha = int(round(1e18 / (link_peak * 1e9 / args.link_share)))
     variant = {"auto": capi.SWAP_AUTO, "memcpy": capi.SWAP_MEMCPY, "zerocopy": capi.SWAP_ZEROCOPY}[args.variant]
     opt = capi.options(swap_variant=variant, alpha_as_per_byte=alpha, beta_ns_per_tensor=0, eta_ns_per_tensor=0)
     descs = [capi.Desc(m) for m in ms]
@@ -431,6 +433,7 @@ def run_multi(args, rank, world):
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": wall_sw / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f16", "data": "synthetic",
         "config": {"workload": CONFIGS["multi"][3], "arena_bytes": arena, "weight_bytes": sum(wbs),
+                   "link_share": args.link_share,
                    "l2": "no flush: 451.6 MB of weights stream through the arena every round"},
         "per_model": per_model,
         "dinf_ms_per_step": wall_di / args.steps, "throughput_ratio": wall_sw / wall_di,
@@ -457,6 +460,76 @@ def measure_link_peak(stream):
         b.synchronize()
         best = min(best, a.elapsed_time(b))
     return (256 << 20) / (best / 1000.0) / 1e9
+
+
+def run_ablation(args):
+    """Ablations of the partition (the shape of the paper's Sec. 8.4-8.5
+    studies) on one single-model config: the planner's plan against
+    equal-byte plans with the paper's block count ceil(2s/b) and the next
+    four counts, the Eq. 4 objective, strictly sequential layers, and each
+    swap variant forced.  Latency of each (ms, CUDA events, L2 flushed)."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2401_16757_gb300 import capi
+    m, w, x, wb, budget, text = build_workload(args.config, capi_weight_bytes)
+    act_in = 1 if args.config == "mlp6" else 0
+    host = capi.HostWeights(w)
+    d = capi.Desc(m)
+    plan0 = capi.Plan.partition(d, budget, capi.options(activations_in_budget=act_in))
+    eng0 = capi.Engine(plan0, host)
+    t_ex, alpha = capi.calibrate(m, plan0, eng0)
+    eng0.free()
+    dc = capi.Desc(m, t_ex_ns=t_ex)
+    base = dict(activations_in_budget=act_in, alpha_as_per_byte=alpha or 4_750_000, beta_ns_per_tensor=0,
+                eta_ns_per_tensor=0, swap_variant=capi.SWAP_MEMCPY)
+    stream = torch.cuda.current_stream()
+    flush = torch.empty(512 << 20, dtype=torch.uint8, device="cuda")
+    x8 = x.view(np.uint8).reshape(-1)
+
+    def latency(plan):
+        info = plan.info()
+        eng = capi.Engine(plan, host)
+        d_in = torch.empty(max(16, info["input_bytes"]), dtype=torch.uint8, device="cuda")
+        d_in[:x8.size].copy_(torch.from_numpy(x8))
+        d_out = torch.empty(info["output_bytes"], dtype=torch.uint8, device="cuda")
+        for _ in range(3):
+            eng.infer(d_in.data_ptr(), d_out.data_ptr(), stream.cuda_stream)
+        ts = []
+        for _ in range(args.steps):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            eng.infer(d_in.data_ptr(), d_out.data_ptr(), stream.cuda_stream)
+            b.record(stream)
+            b.synchronize()
+            ts.append(a.elapsed_time(b))
+        eng.sync()
+        eng.free()
+        return {"ms": statistics.median(ts), "n_blocks": info["n_blocks"], "predicted_ms": info["predicted_ns"] / 1e6}
+
+    def try_plan(make):
+        try:
+            return latency(make())
+        except capi.SwapnetError as ex:
+            return {"infeasible": str(ex)}
+
+    out = {"planner": try_plan(lambda: capi.Plan.partition(dc, budget, capi.options(**base)))}
+    units = capi.Plan.partition(dc, budget, capi.options(**base)).units()
+    ub = np.cumsum([u["bytes"] for u in units])
+    n_min = int(np.ceil(2.0 * wb / budget))
+    for n in range(n_min, n_min + 5):
+        cuts = sorted({int(np.searchsorted(ub, ub[-1] * k / n, side="left")) + 1 for k in range(1, n)})
+        cuts = [c for c in cuts if 0 < c < len(units)]
+        out["equal_bytes_n%d" % n] = try_plan(lambda: capi.Plan.from_cuts(dc, cuts, budget, capi.options(**base)))
+    if len(units) <= 24:
+        out["objective_eq4"] = try_plan(lambda: capi.Plan.partition(dc, budget, capi.options(**dict(base, objective=1))))
+    out["sequential_layers"] = try_plan(lambda: capi.Plan.partition(dc, budget, capi.options(**dict(base, branches=0))))
+    out["zero_copy_swap"] = try_plan(
+        lambda: capi.Plan.partition(dc, budget, capi.options(**dict(base, swap_variant=capi.SWAP_ZEROCOPY))))
+    out["resident_dinf"] = try_plan(lambda: capi.Plan.resident(d))
+    print(json.dumps({"ablation": args.config, "workload": text, "budget_bytes": budget, "weight_bytes": wb,
+                      "paper_block_count": n_min, "steps": args.steps, "results": out}))
 
 
 def run_profile_once(args):
@@ -557,6 +630,11 @@ def main():
     ap.add_argument("--config", default="resnet50", choices=sorted(CONFIGS))
     ap.add_argument("--variant", default="auto", choices=["auto", "memcpy", "zerocopy"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--link-share", type=float, default=1.0,
+                    help="multi: models sharing the host link in each model's delay model")
+    ap.add_argument("--ablation", action="store_true",
+                    help="partition ablations of --config (planner vs equal-byte plans, Eq. 4, sequential "
+                         "layers, zero-copy swap, DInf); prints one JSON line")
     ap.add_argument("--profile-once", action="store_true",
                     help="run one resident inference of --config through the C ABI and exit "
                          "(a driver for profiler captures of its kernels); prints one JSON line")
@@ -571,6 +649,9 @@ def main():
         return
     if args.profile_once:
         run_profile_once(args)
+        return
+    if args.ablation:
+        run_ablation(args)
         return
     if args.config in ("llm", "multi"):
         import torch

@@ -317,6 +317,73 @@ static int calibrate(swapnet_engine* e) {
   return rc;
 }
 
+static int capture(swapnet_engine* e, const void* din, void* dout, cudaGraphExec_t* out);
+
+// Second stage of the AUTO choice.  The first stage times each block's copy
+// alone; inside the pipeline a zero-copy swap shares the SMs with the layers
+// while a copy-engine swap does not, and their start-up latencies differ.
+// So whole inferences (CUDA graph replays on scratch input and output
+// buffers) are timed with the per-block choice, with every block on the copy
+// engine and with every block zero-copy, and the fastest assignment is kept.
+// Decoder models (which need a bound state) keep the per-block choice.
+static int calibrate_in_situ(swapnet_engine* e) {
+  const Model& m = e->plan.model;
+  if (m.has_attention || e->blocks.empty()) return SWAPNET_OK;
+  void* din = nullptr;
+  void* dout = nullptr;
+  if (cudaMalloc(&din, align_up(m.in_bytes)) != cudaSuccess ||
+      cudaMalloc(&dout, align_up(m.out_bytes)) != cudaSuccess) {
+    cudaGetLastError();
+    if (din) cudaFree(din);
+    return SWAPNET_OK;  // no room for scratch buffers: keep the per-block choice
+  }
+  cudaMemset(din, 0, align_up(m.in_bytes));
+  std::vector<std::vector<int>> cand(1);
+  for (const EngBlock& b : e->blocks) cand[0].push_back(b.variant);
+  cand.push_back(std::vector<int>(e->blocks.size(), SWAPNET_SWAP_MEMCPY));
+  bool zc_all = true;
+  for (const EngBlock& b : e->blocks) zc_all = zc_all && zerocopy_ok(b);
+  if (zc_all) cand.push_back(std::vector<int>(e->blocks.size(), SWAPNET_SWAP_ZEROCOPY));
+  cudaEvent_t a = nullptr, b = nullptr;
+  int rc = SWAPNET_OK;
+  if (cudaEventCreate(&a) != cudaSuccess || cudaEventCreate(&b) != cudaSuccess) rc = SWAPNET_ERR_CUDA;
+  float best = 1e30f;
+  size_t best_i = 0;
+  for (size_t c = 0; c < cand.size() && rc == SWAPNET_OK; ++c) {
+    for (size_t k = 0; k < e->blocks.size(); ++k) e->blocks[k].variant = cand[c][k];
+    cudaGraphExec_t ge = nullptr;
+    rc = capture(e, din, dout, &ge);
+    if (rc) break;
+    std::vector<float> t;
+    for (int rep = 0; rep < 7 && rc == SWAPNET_OK; ++rep) {
+      cudaEventRecord(a, e->cap);
+      if (cudaGraphLaunch(ge, e->cap) != cudaSuccess) rc = SWAPNET_ERR_CUDA;
+      cudaEventRecord(b, e->cap);
+      if (cudaEventSynchronize(b) != cudaSuccess) rc = SWAPNET_ERR_CUDA;
+      float ms = 0.f;
+      cudaEventElapsedTime(&ms, a, b);
+      if (rep >= 2) t.push_back(ms);  // two warm-up replays
+    }
+    cudaGraphExecDestroy(ge);
+    if (rc) break;
+    std::sort(t.begin(), t.end());
+    const float med = t[t.size() / 2];
+    if (med < best * 0.98f) {  // prefer the earlier candidate unless clearly faster
+      best = med;
+      best_i = c;
+    }
+  }
+  if (rc == SWAPNET_OK)
+    for (size_t k = 0; k < e->blocks.size(); ++k) e->blocks[k].variant = cand[best_i][k];
+  else
+    set_error("swap variant calibration failed");
+  if (a) cudaEventDestroy(a);
+  if (b) cudaEventDestroy(b);
+  cudaFree(din);
+  cudaFree(dout);
+  return rc;
+}
+
 static const char* act_ptr(const swapnet_engine* e, int src, const void* din, const void* dout) {
   if (src == SWAPNET_SRC_INPUT) return static_cast<const char*>(din);
   const Layer& L = e->plan.model.L[src];
@@ -629,6 +696,8 @@ int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint
     e->weights_loaded = true;
   } else if (variant == SWAPNET_SWAP_AUTO) {
     rc = calibrate(e);
+    if (rc) return rc;
+    rc = calibrate_in_situ(e);
     if (rc) return rc;
   } else {
     for (EngBlock& b : e->blocks) {
