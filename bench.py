@@ -309,6 +309,23 @@ def run_llm(args, rank, world):
     # greedy tokens agree between swapped and resident runs
     one(ep, ed); torch.cuda.synchronize(); sw_tok = int(tok[:4].cpu().numpy().view(np.int32)[0])
     one(rp, rd); torch.cuda.synchronize(); rs_tok = int(tok[:4].cpu().numpy().view(np.int32)[0])
+    # extension (not the paper's method): resident-prefix plans in the same budget
+    opt_rp = capi.options(swap_variant=variant, alpha_as_per_byte=alpha, beta_ns_per_tensor=0, resident_prefix=1)
+    pp_rp, pd_rp = capi.Plan.partition(dp, budget, opt_rp), capi.Plan.partition(dd, budget, opt_rp)
+    ep.free(); ed.free()
+    ep_rp, ed_rp = capi.Engine(pp_rp, host), capi.Engine(pd_rp, host)
+    for e_ in (ep_rp, ed_rp):
+        e_.bind_state(state.data_ptr(), ip["state_bytes"])
+    one(ep_rp, ed_rp)
+    torch.cuda.synchronize()
+    rp_t = timed(ep_rp, ed_rp, args.steps)
+    ext_rp = {"prefill_ms": statistics.mean(r[0] for r in rp_t),
+              "decode_ms_per_token": statistics.mean(r[1] for r in rp_t),
+              "prefix_units": [pp_rp.info()["prefix_units"], pd_rp.info()["prefix_units"]],
+              "prefix_bytes": [pp_rp.info()["prefix_bytes"], pd_rp.info()["prefix_bytes"]]}
+    ext_rp["ms_per_step"] = ext_rp["prefill_ms"] + n_dec * ext_rp["decode_ms_per_token"]
+    one(ep_rp, ed_rp); torch.cuda.synchronize()
+    ext_rp["greedy_token_equals_resident"] = int(tok[:4].cpu().numpy().view(np.int32)[0]) == rs_tok
     pre_ms = statistics.mean(r[0] for r in sw)
     dec_ms = statistics.mean(r[1] for r in sw)
     pre_d = statistics.mean(r[0] for r in di)
@@ -338,6 +355,7 @@ def run_llm(args, rank, world):
         "step_roofline": {"bound": "host link", "bound_ms": bound_ms, "frac": bound_ms / step_ms},
         "gpu_launches": launches, "clocks": clk,
         "setup_s": {"weights": t_gen, "plans": t_plan},
+        "extension_resident_prefix": ext_rp,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         tot, sample = llm_cpu_sample()
@@ -747,6 +765,20 @@ def main():
         eng0.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
     ms_uncal_list = timed(eng0, min(args.steps, 50))
     ms_uncal = sum(ms_uncal_list) / len(ms_uncal_list)
+    # ---- extension (not the paper's method): the first units stay resident
+    # in the arena between inferences, the rest swap through the region left
+    opt_rp = capi.options(slots=2, activations_in_budget=act_in, swap_variant=variant,
+                          alpha_as_per_byte=alpha or 4_750_000, beta_ns_per_tensor=0, eta_ns_per_tensor=0,
+                          resident_prefix=1)
+    plan_rp = capi.Plan.partition(dc, budget, opt_rp)
+    eng_rp = capi.Engine(plan_rp, host)
+    for _ in range(3):
+        eng_rp.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
+    ms_rp_list = timed(eng_rp, min(args.steps, 50))
+    ext_rp = {"ms": sum(ms_rp_list) / len(ms_rp_list), "prefix_units": plan_rp.info()["prefix_units"],
+              "prefix_bytes": plan_rp.info()["prefix_bytes"], "n_blocks": plan_rp.info()["n_blocks"],
+              "swapped_bytes_per_step": sum(b["bytes"] for b in plan_rp.blocks()[1 if plan_rp.info()["prefix_units"] else 0:])}
+    eng_rp.free()
 
     # ---- e2e: host buffers through swapnet_infer_host
     h_in = torch.empty(info["input_bytes"], dtype=torch.uint8, pin_memory=True)
@@ -840,6 +872,7 @@ def main():
             "dinf_ms": ms_dinf, "ratio": ms_swapped / ms_dinf,
             "predicted_ms": info["predicted_ns"] / 1e6,
             "uncalibrated_plan": {"cuts": plan0.cuts(), "ms": ms_uncal},
+            "extension_resident_prefix": ext_rp,
             "p50_ms": statistics.median(ms_list), "p99_ms": float(np.percentile(ms_list, 99)),
             "e2e": {"value": e2e_val, "unit": "inferences/s", "h2d_bytes_per_step": info["input_bytes"],
                     "d2h_bytes_per_step": info["output_bytes"]},

@@ -156,7 +156,17 @@ typedef struct swapnet_options {
                                      last producer and its consumers share a block;
                                      0: every layer in order on one stream.  Results
                                      are identical either way. */
-  int32_t reserved[4];
+  int32_t resident_prefix;       /* 0 (default, the paper's method): every block is
+                                     swapped in for every inference.  1 (an extension
+                                     the paper has no counterpart for): the planner may
+                                     keep the first units' weights in the arena across
+                                     inferences (uploaded once at load, never swapped)
+                                     and swap the rest through the remaining region;
+                                     the prefix length is chosen by the objective among
+                                     0, the longest prefix that leaves room for the
+                                     rest, and the longest within 1/4, 1/2, 3/4 of its
+                                     bytes.  Objective 0 only. */
+  int32_t reserved[3];
 } swapnet_options;
 
 /* Fills the defaults: 2 slots, activations outside the budget, AUTO swap,
@@ -185,6 +195,10 @@ typedef struct swapnet_plan_info {
   int32_t exact;           /* 1: the search proved the plan optimal; 0: its
                               frontier was capped and the plan is the best found */
   int32_t reserved;
+  uint32_t prefix_units;   /* resident_prefix: units kept in the arena (block 0) */
+  uint32_t reserved2;
+  uint64_t prefix_bytes;   /* their bytes at the bottom of the arena; the swap
+                              region follows them                             */
 } swapnet_plan_info;
 
 typedef struct swapnet_unit_info {
@@ -199,7 +213,8 @@ typedef struct swapnet_unit_info {
 
 typedef struct swapnet_block_info {
   uint32_t unit0, unit1; /* units [unit0, unit1)                             */
-  uint32_t slot;         /* block parity: which co-resident position it takes */
+  uint32_t slot;         /* block parity: which co-resident position it takes;
+                            UINT32_MAX for a resident prefix block           */
   uint32_t depth;
   uint64_t bytes;
   int64_t t_in_ns, t_ex_ns, t_out_ns;

@@ -248,16 +248,47 @@ def block_costs(us, cuts, coef):
     return res
 
 
-def pipeline_time(blocks, slots):
-    """Objective 0: completion time of the m-slot pipeline."""
+def pipeline_time(blocks, slots, prefix=False):
+    """Objective 0: completion time of the m-slot pipeline.  With prefix,
+    blocks[0] is a resident prefix (an extension, not the paper's method):
+    its layers start at t = 0 without a copy and it never frees room, so the
+    swapped blocks after it gate only on each other."""
     C = E = 0
     R = []
+    lo = 1 if prefix else 0
     for k, (_, t_in, t_ex, t_out) in enumerate(blocks):
-        gate = R[k - slots] if k - slots >= 0 else 0
+        if prefix and k == 0:
+            E = t_ex
+            R.append(0)
+            continue
+        gate = R[k - slots] if k - slots >= lo else 0
         C = max(C, gate) + t_in
         E = max(E, C) + t_ex
         R.append(E + t_out)
     return E
+
+
+def prefix_candidates(us, region, slots):
+    """Resident-prefix lengths tried: 0; the longest prefix r whose bytes
+    plus the smallest region the remaining units need (each unit, and with
+    two co-resident blocks each adjacent pair) fit the region; and the
+    longest prefixes within 1/4, 1/2 and 3/4 of that prefix's bytes."""
+    U = len(us)
+    pb = [0]
+    for u in us:
+        pb.append(pb[-1] + u["bytes"])
+
+    def need(r):
+        m = [u["bytes"] for u in us[r:]]
+        if slots == 2:
+            m += [us[i]["bytes"] + us[i + 1]["bytes"] for i in range(r, U - 1)]
+        return max(m, default=0)
+
+    rmax = max([r for r in range(1, U + 1) if align(pb[r]) + need(r) <= region], default=0)
+    cands = {0, rmax}
+    for q in (1, 2, 3):
+        cands.add(max(r for r in range(0, rmax + 1) if 4 * pb[r] <= q * pb[rmax]))
+    return sorted(cands), pb
 
 
 def eq4_objective(blocks):
@@ -296,11 +327,17 @@ def feasible(blocks, region, slots):
 
 
 def exhaustive_partition(model, budget, coef, slots=2, activations_in_budget=False,
-                         objective=0, t_ex_override=None):
+                         objective=0, t_ex_override=None, resident_prefix=False):
     """Best cut vector by brute force over all 2^(U-1) candidates.
 
-    Returns dict(n, cuts, predicted_ns, slot, arena, workspace, units) or
-    None when no partition is feasible."""
+    With resident_prefix (objective 0 only) the first r units may stay in the
+    arena across inferences, r among prefix_candidates(); for each r every
+    cut vector of the remaining units is tried in the region left beside the
+    prefix.  Ties: smaller objective, then shorter prefix, then fewer blocks,
+    then the lexicographically smallest cut vector.
+
+    Returns dict(n, cuts, predicted_ns, slot, arena, workspace, units,
+    prefix_units, prefix_bytes) or None when no partition is feasible."""
     a = arena_and_slot(model, budget, slots, activations_in_budget)
     if a is None:
         return None
@@ -310,20 +347,34 @@ def exhaustive_partition(model, budget, coef, slots=2, activations_in_budget=Fal
     if us is None:
         return None
     U = len(us)
+    if resident_prefix:
+        cands, pb = prefix_candidates(us, region, slots)
+    else:
+        cands, pb = [0], [0]
     best = None
-    for mask in range(1 << (U - 1)):
-        cuts = tuple(c for c in range(1, U) if mask >> (c - 1) & 1)
-        blocks = block_costs(us, cuts, coef)
-        if not feasible(blocks, region, slots):
-            continue
-        obj = pipeline_time(blocks, slots) if objective == 0 else eq4_objective(blocks)
-        key = (obj, len(blocks), cuts)
-        if best is None or key < best:
-            best = key
+    for r in cands:
+        reg = region - (align(pb[r]) if r else 0)
+        rest = U - r
+        masks = range(1 << (rest - 1)) if rest > 0 else [0]
+        for mask in masks:
+            inner = tuple(r + c for c in range(1, rest) if mask >> (c - 1) & 1)
+            cuts = ((r,) if 0 < r < U else ()) + inner
+            blocks = block_costs(us, cuts, coef)
+            swapped = blocks[1:] if r else blocks
+            if not feasible(swapped, reg, slots):
+                continue
+            if objective == 0:
+                obj = pipeline_time(blocks, slots, prefix=r > 0)
+            else:
+                obj = eq4_objective(blocks)
+            key = (obj, r, len(blocks), cuts)
+            if best is None or key < best:
+                best = key
     if best is None:
         return None
-    return dict(n=best[1], cuts=list(best[2]), predicted_ns=best[0], slot=slot, arena=arena,
-                workspace=ws, units=us)
+    r = best[1]
+    return dict(n=best[2], cuts=list(best[3]), predicted_ns=best[0], slot=slot, arena=arena,
+                workspace=ws, units=us, prefix_units=r, prefix_bytes=align(pb[r]) if r else 0)
 
 
 def evaluate_cuts(model, budget, coef, cuts, slots=2, activations_in_budget=False,

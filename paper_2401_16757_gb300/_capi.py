@@ -47,7 +47,7 @@ class Options(C.Structure):
                 ("objective", C.c_int32), ("alpha_as_per_byte", C.c_uint64), ("beta_ns_per_tensor", C.c_uint64),
                 ("gamma_as_per_flop", C.c_uint64), ("eta_ns_per_tensor", C.c_uint64), ("zc_ctas", C.c_int32),
                 ("graphs", C.c_int32), ("preloaded", C.c_int32), ("branches", C.c_int32),
-                ("reserved", C.c_int32 * 4)]
+                ("resident_prefix", C.c_int32), ("reserved", C.c_int32 * 3)]
 
 
 class PlanInfo(C.Structure):
@@ -56,7 +56,8 @@ class PlanInfo(C.Structure):
                 ("slot_bytes", C.c_uint64), ("workspace_bytes", C.c_uint64), ("input_bytes", C.c_uint64),
                 ("output_bytes", C.c_uint64), ("weight_bytes", C.c_uint64), ("plan_bytes", C.c_uint64),
                 ("predicted_ns", C.c_int64), ("state_bytes", C.c_uint64), ("exact", C.c_int32),
-                ("reserved", C.c_int32)]
+                ("reserved", C.c_int32), ("prefix_units", C.c_uint32), ("reserved2", C.c_uint32),
+                ("prefix_bytes", C.c_uint64)]
 
 
 class UnitInfo(C.Structure):

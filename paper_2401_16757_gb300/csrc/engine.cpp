@@ -295,6 +295,7 @@ static int calibrate(swapnet_engine* e) {
   int rc = SWAPNET_OK;
   for (size_t k = 0; k < e->blocks.size() && rc == SWAPNET_OK; ++k) {
     EngBlock& B = e->blocks[k];
+    if (e->plan.blocks[k].slot < 0) continue;  // resident prefix: never swapped
     float best[3] = {1e30f, 1e30f, 1e30f};
     for (int v : {SWAPNET_SWAP_MEMCPY, SWAPNET_SWAP_ZEROCOPY}) {
       if (v == SWAPNET_SWAP_ZEROCOPY && !zerocopy_ok(B)) continue;
@@ -342,7 +343,8 @@ static int calibrate_in_situ(swapnet_engine* e) {
   for (const EngBlock& b : e->blocks) cand[0].push_back(b.variant);
   cand.push_back(std::vector<int>(e->blocks.size(), SWAPNET_SWAP_MEMCPY));
   bool zc_all = true;
-  for (const EngBlock& b : e->blocks) zc_all = zc_all && zerocopy_ok(b);
+  for (size_t k = 0; k < e->blocks.size(); ++k)
+    zc_all = zc_all && (e->plan.blocks[k].slot < 0 || zerocopy_ok(e->blocks[k]));
   if (zc_all) cand.push_back(std::vector<int>(e->blocks.size(), SWAPNET_SWAP_ZEROCOPY));
   cudaEvent_t a = nullptr, b = nullptr;
   int rc = SWAPNET_OK;
@@ -608,8 +610,10 @@ int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint
     SN_FAIL(SWAPNET_ERR_INVALID_ARG, "expected " + std::to_string(plan->model.n_tensors) + " host tensors");
   if (((uintptr_t)d_arena | (uintptr_t)d_workspace) % kAlign)
     SN_FAIL(SWAPNET_ERR_MISALIGNED, "device buffers must be 256-byte aligned");
-  const uint64_t arena_need = plan->region;
+  const uint64_t arena_need = plan->prefix_bytes + plan->region;  // resident prefix, then the swap region
   if (d_arena && arena_bytes < arena_need) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "arena buffer too small");
+  for (const Block& B : plan->blocks)  // every block lies inside the arena
+    if (B.base + B.bytes > arena_need) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "plan places a block outside the arena");
   if (d_workspace && workspace_bytes < plan->model.ws_bytes)
     SN_FAIL(SWAPNET_ERR_INVALID_ARG, "workspace buffer too small");
   swapnet_engine* e = new (std::nothrow) swapnet_engine();
@@ -694,15 +698,23 @@ int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint
       CU(cudaStreamSynchronize(e->copy), "resident upload");
     }
     e->weights_loaded = true;
-  } else if (variant == SWAPNET_SWAP_AUTO) {
+  } else if (plan->prefix_units > 0 && !plan->blocks.empty() && plan->blocks[0].slot < 0) {
+    // resident prefix: uploaded once, then only the other blocks are swapped
+    rc = swap_block(e, 0, SWAPNET_SWAP_MEMCPY, e->copy);
+    if (rc) return rc;
+    CU(cudaStreamSynchronize(e->copy), "prefix upload");
+  }
+  if (!plan->resident && variant == SWAPNET_SWAP_AUTO) {
     rc = calibrate(e);
     if (rc) return rc;
     rc = calibrate_in_situ(e);
     if (rc) return rc;
-  } else {
-    for (EngBlock& b : e->blocks) {
+  } else if (!plan->resident) {
+    for (size_t k = 0; k < e->blocks.size(); ++k) {
+      EngBlock& b = e->blocks[k];
       b.variant = variant;
-      if (variant == SWAPNET_SWAP_ZEROCOPY && !zerocopy_ok(b)) SN_FAIL(SWAPNET_ERR_MISALIGNED, "zero-copy needs 16-byte aligned host tensors");
+      if (plan->blocks[k].slot >= 0 && variant == SWAPNET_SWAP_ZEROCOPY && !zerocopy_ok(b))
+        SN_FAIL(SWAPNET_ERR_MISALIGNED, "zero-copy needs 16-byte aligned host tensors");
     }
   }
   e->stats = swapnet_engine_stats{};
@@ -789,7 +801,8 @@ static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t 
   }
   for (size_t k = 0; k < p.blocks.size(); ++k) {
     const Block& B = p.blocks[k];
-    if (!p.resident) {
+    const bool swapped = !p.resident && B.slot >= 0;  // a resident prefix stays in the arena
+    if (swapped) {
       if (used[B.slot]) CU(cudaStreamWaitEvent(e->copy, e->slot_free[B.slot], 0), "wait slot");
       used[B.slot] = true;
       if (prof) CU(cudaEventRecord(e->ev_swap[2 * k], e->copy), "profile event");
@@ -816,7 +829,7 @@ static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t 
         CU(cudaEventRecord(e->side_done[w], e->side), "record side done");
       }
     }
-    if (!p.resident) CU(cudaEventRecord(e->slot_free[B.slot], s), "record slot free");
+    if (swapped) CU(cudaEventRecord(e->slot_free[B.slot], s), "record slot free");
   }
   if (p.model.has_attention) {
     if (!e->d_state) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "decoder state not bound (swapnet_engine_bind_state)");
@@ -835,8 +848,9 @@ static uint64_t launches_per_infer(const swapnet_engine* e) {
   uint64_t n = e->plan.units.size() + (e->plan.model.has_attention ? 1 : 0);
   for (int k : e->unit_kind) n += (k == SWAPNET_KERNEL_ATTENTION) ? 1 : 0;
   if (!e->plan.resident)
-    for (const EngBlock& b : e->blocks)
-      if (b.variant == SWAPNET_SWAP_ZEROCOPY) n += (b.segs.size() + 47) / 48;
+    for (size_t k = 0; k < e->blocks.size(); ++k)
+      if (e->plan.blocks[k].slot >= 0 && e->blocks[k].variant == SWAPNET_SWAP_ZEROCOPY)
+        n += (e->blocks[k].segs.size() + 47) / 48;
   return n;
 }
 
@@ -1061,7 +1075,8 @@ int swapnet_engine_last_times(swapnet_engine* e, float* unit_us, uint32_t nu, fl
   }
   for (uint32_t k = 0; swap_us && k < nb && k < e->plan.blocks.size(); ++k) {
     float ms = 0.f;
-    if (!e->plan.resident) CU(cudaEventElapsedTime(&ms, e->ev_swap[2 * k], e->ev_swap[2 * k + 1]), "elapsed");
+    if (!e->plan.resident && e->plan.blocks[k].slot >= 0)  // a resident prefix is never swapped
+      CU(cudaEventElapsedTime(&ms, e->ev_swap[2 * k], e->ev_swap[2 * k + 1]), "elapsed");
     swap_us[k] = ms * 1000.f;
   }
   return SWAPNET_OK;
@@ -1073,12 +1088,14 @@ int swapnet_engine_last_timeline(swapnet_engine* e, float* us0, float* us1, uint
   if (e->ev_unit.empty()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "profiling was never enabled");
   CU(cudaSetDevice(e->device), "cudaSetDevice");
   CU(cudaDeviceSynchronize(), "device synchronize");
-  const bool sw = !e->plan.resident && !e->ev_swap.empty();
-  cudaEvent_t origin = sw ? e->ev_swap[0] : e->ev_unit[0];
+  size_t k0 = 0;  // first swapped block (a resident prefix has no swap events)
+  while (k0 < e->plan.blocks.size() && e->plan.blocks[k0].slot < 0) ++k0;
+  const bool sw = !e->plan.resident && !e->ev_swap.empty() && k0 < e->plan.blocks.size();
+  cudaEvent_t origin = sw ? e->ev_swap[2 * k0] : e->ev_unit[0];
   float first = 0.f;
   if (sw) {  // the first kernel may start before the first swap event on another stream
     float d = 0.f;
-    CU(cudaEventElapsedTime(&d, e->ev_swap[0], e->ev_unit[0]), "elapsed");
+    CU(cudaEventElapsedTime(&d, e->ev_swap[2 * k0], e->ev_unit[0]), "elapsed");
     first = std::min(0.f, d);
   }
   auto rel = [&](cudaEvent_t ev, float* out) -> int {
@@ -1092,7 +1109,7 @@ int swapnet_engine_last_timeline(swapnet_engine* e, float* us0, float* us1, uint
     if (us1 && rel(e->ev_unit[2 * u + 1], &us1[u])) return SWAPNET_ERR_CUDA;
   }
   for (uint32_t k = 0; k < nb && k < e->plan.blocks.size(); ++k) {
-    if (!sw) {
+    if (!sw || e->plan.blocks[k].slot < 0) {
       if (ss0) ss0[k] = 0.f;
       if (ss1) ss1[k] = 0.f;
       continue;

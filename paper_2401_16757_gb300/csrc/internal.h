@@ -96,13 +96,15 @@ struct swapnet_plan {
   std::vector<uint32_t> cuts;
   int64_t predicted = 0;
   bool exact = true;  // the search proved the plan optimal for its objective
+  int prefix_units = 0;       // resident prefix: units [0, prefix_units) are block 0,
+  uint64_t prefix_bytes = 0;  // kept at arena offset 0; the swap region follows
 };
 
 namespace swapnet {
 int analyse_model(const swapnet_model_desc* desc, Model* m);
 int make_units(const Model& m, const swapnet_options& opt, uint64_t slot, uint64_t region, std::vector<Unit>* out);
 void finalize_blocks(swapnet_plan* p, const std::vector<uint32_t>& cuts);
-int64_t pipeline_ns(const std::vector<Block>& b, int slots);
+int64_t pipeline_ns(const std::vector<Block>& b, int slots, bool prefix = false);
 int64_t eq4_ns(const std::vector<Block>& b);
 uint64_t resident_latency_ns(const Model& m, const swapnet_options& opt);
 }  // namespace swapnet

@@ -305,11 +305,19 @@ static Block make_block(const std::vector<Unit>& us, int a, int b, const swapnet
   return B;
 }
 
-int64_t pipeline_ns(const std::vector<Block>& b, int slots) {
+// prefix: block 0 is the resident prefix (already in the arena: no copy,
+// never released); the swapped blocks after it gate only on each other.
+int64_t pipeline_ns(const std::vector<Block>& b, int slots, bool prefix) {
   int64_t C = 0, E = 0;
   std::vector<int64_t> R;
+  const int64_t lo = prefix ? 1 : 0;
   for (size_t k = 0; k < b.size(); ++k) {
-    const int64_t gate = ((int64_t)k - slots >= 0) ? R[k - slots] : 0;
+    if (prefix && k == 0) {
+      E = b[0].t_ex;
+      R.push_back(0);
+      continue;
+    }
+    const int64_t gate = ((int64_t)k - slots >= lo) ? R[k - slots] : 0;
     C = std::max(C, gate) + b[k].t_in;
     E = std::max(E, C) + b[k].t_ex;
     R.push_back(E + b[k].t_out);
@@ -343,13 +351,22 @@ void finalize_blocks(swapnet_plan* p, const std::vector<uint32_t>& cuts) {
   b.insert(b.end(), cuts.begin(), cuts.end());
   b.push_back((uint32_t)p->units.size());
   const int slots = p->resident ? 1 : p->opt.slots;
+  const bool prefix = !p->resident && p->prefix_units > 0;
   for (size_t k = 0; k + 1 < b.size(); ++k) {
     Block B = make_block(p->units, (int)b[k], (int)b[k + 1], p->opt);
-    B.slot = (int)(k % slots);
-    // two co-resident blocks (Eq. 3): even blocks from the bottom of the
-    // region, odd blocks against its top, so s_k + s_{k+1} <= region keeps
-    // consecutive blocks apart
-    B.base = (slots == 2 && (k % 2) == 1) ? p->region - B.bytes : 0;
+    if (prefix && k == 0) {  // resident prefix: bottom of the arena, never swapped
+      B.slot = -1;
+      B.base = 0;
+      B.t_in = 0;
+      B.t_out = 0;
+    } else {
+      const size_t s = prefix ? k - 1 : k;  // index among the swapped blocks
+      B.slot = (int)(s % slots);
+      // two co-resident blocks (Eq. 3): even blocks from the bottom of the
+      // region, odd blocks against its top, so s_k + s_{k+1} <= region keeps
+      // consecutive blocks apart
+      B.base = p->prefix_bytes + ((slots == 2 && (s % 2) == 1) ? p->region - B.bytes : 0);
+    }
     // slot layout: tensors in unit order, 256-byte aligned
     uint64_t off = 0;
     for (int u = B.u0; u < B.u1; ++u) {
@@ -364,7 +381,7 @@ void finalize_blocks(swapnet_plan* p, const std::vector<uint32_t>& cuts) {
     for (const Unit& u : p->units) t += u.t_ex;
     p->predicted = t;
   } else {
-    p->predicted = p->opt.objective == 0 ? pipeline_ns(p->blocks, p->opt.slots) : eq4_ns(p->blocks);
+    p->predicted = p->opt.objective == 0 ? pipeline_ns(p->blocks, p->opt.slots, prefix) : eq4_ns(p->blocks);
   }
 }
 
@@ -458,21 +475,27 @@ struct Search {
 
 // A feasible plan for an upper bound: consecutive units packed into blocks
 // of at most half the arena (any two such neighbours fit together).
-static int64_t greedy_upper_bound(const swapnet_plan* p) {
+static int64_t greedy_upper_bound(const swapnet_plan* p, int start, int64_t e0) {
   const int U = (int)p->units.size();
   const uint64_t cap = p->opt.slots == 2 ? p->region / 2 : p->region;
   std::vector<Block> bl;
-  for (int j = 0; j < U;) {
+  if (start > 0) {  // the resident prefix as block 0
+    Block P{};
+    P.t_ex = e0;
+    bl.push_back(P);
+  }
+  for (int j = start; j < U;) {
     uint64_t bytes = 0;
     int j2 = j;
     while (j2 < U && bytes + p->units[j2].bytes <= cap) bytes += p->units[j2++].bytes;
     if (j2 == j) j2 = j + 1;  // one unit larger than the cap: a block of its own
     Block B = make_block(p->units, j, j2, p->opt);
-    if (!pair_ok(p, bl.empty() ? 0 : bl.back().bytes, B.bytes)) return INT64_MAX;
+    const bool first = (int)bl.size() == (start > 0 ? 1 : 0);
+    if (!pair_ok(p, first ? 0 : bl.back().bytes, B.bytes)) return INT64_MAX;
     bl.push_back(B);
     j = j2;
   }
-  return pipeline_ns(bl, p->opt.slots);
+  return pipeline_ns(bl, p->opt.slots, start > 0);
 }
 
 // Exact search over cut vectors: a Pareto front of pipeline states per unit
@@ -482,7 +505,7 @@ static int64_t greedy_upper_bound(const swapnet_plan* p) {
 // unit), since copies and executions each form a chain; states whose bound
 // exceeds the best finish found (or a greedy plan's) cannot win.
 static int search_pipeline_capped(swapnet_plan* p, std::vector<uint32_t>* best_cuts, size_t cap,
-                                  int64_t ub_in, int64_t* best_ns, bool* exact) {
+                                  int64_t ub_in, int64_t* best_ns, bool* exact, int start, int64_t e0) {
   const int U = (int)p->units.size();
   std::vector<int64_t> rem_ex(U + 1, 0), rem_in(U + 1, 0);
   {
@@ -496,21 +519,25 @@ static int search_pipeline_capped(swapnet_plan* p, std::vector<uint32_t>* best_c
     }
   }
   const int64_t last_ex = U ? p->units[U - 1].t_ex : 0;
-  int64_t ub = std::min(ub_in, greedy_upper_bound(p));
+  int64_t ub = std::min(ub_in, greedy_upper_bound(p, start, e0));
   auto bound = [&](const State& c, int j) -> int64_t {
     if (j == U) return c.v[1];
     return std::max(c.v[1] + rem_ex[j], c.v[0] + rem_in[j] + last_ex);
   };
   Search S(p->units, p->opt, p->slot);
   S.front.assign(U + 1, {});
+  // initial state at boundary `start`: with a resident prefix, its layers
+  // execute from t = 0 (E = e0) while the first copy starts at t = 0, and
+  // no swapped block waits for the prefix to be released
   State s0{};
-  s0.prev_j = -1; s0.prev_idx = -1; s0.nblocks = 0;
-  S.front[0].push_back(s0);
+  s0.v[1] = e0;
+  s0.prev_j = -1; s0.prev_idx = -1; s0.nblocks = start > 0 ? 1 : 0;
+  S.front[start].push_back(s0);
   // frontier states of boundary j only get children once j is final; a
   // frontier wider than kFrontCap keeps its kFrontCap states of smallest
   // bound (the result is then the best plan found, not a proven optimum)
   *exact = true;
-  for (int j = 0; j < U; ++j) {
+  for (int j = start; j < U; ++j) {
     std::vector<State>& Fj = S.front[j];
     if (Fj.size() > cap) {
       std::vector<std::pair<std::pair<int64_t, int64_t>, size_t>> key(Fj.size());
@@ -554,7 +581,7 @@ static int search_pipeline_capped(swapnet_plan* p, std::vector<uint32_t>* best_c
                                      !S.tie_le(U, best, i)))
       best = i;
   }
-  *best_cuts = S.cuts_of(U, best);
+  *best_cuts = S.cuts_of(U, best);  // includes `start` (the first block's boundary)
   *best_ns = F[best].v[1];
   return SWAPNET_OK;
 }
@@ -562,22 +589,93 @@ static int search_pipeline_capped(swapnet_plan* p, std::vector<uint32_t>* best_c
 // A narrow beam first finds a good plan; its finish time then bounds the
 // full search, which prunes every state that cannot reach it.  States
 // whose bound equals it are kept, so ties are still broken exactly.
-static int search_pipeline(swapnet_plan* p, std::vector<uint32_t>* best_cuts) {
+static int search_pipeline(swapnet_plan* p, std::vector<uint32_t>* best_cuts, int64_t* best_ns = nullptr,
+                           int start = 0, int64_t e0 = 0) {
   std::vector<uint32_t> beam_cuts;
   int64_t beam_ns = INT64_MAX;
   bool beam_exact = false;
-  int rc = search_pipeline_capped(p, &beam_cuts, 32, INT64_MAX, &beam_ns, &beam_exact);
+  int rc = search_pipeline_capped(p, &beam_cuts, 32, INT64_MAX, &beam_ns, &beam_exact, start, e0);
   if (rc) return rc;
   if (beam_exact) {
     p->exact = true;
     *best_cuts = beam_cuts;
+    if (best_ns) *best_ns = beam_ns;
     return SWAPNET_OK;
   }
   int64_t ns = 0;
   bool exact = false;
-  rc = search_pipeline_capped(p, best_cuts, 4096, beam_ns, &ns, &exact);
+  rc = search_pipeline_capped(p, best_cuts, 4096, beam_ns, &ns, &exact, start, e0);
   if (rc) return rc;
   p->exact = exact;
+  if (best_ns) *best_ns = ns;
+  return SWAPNET_OK;
+}
+
+// Resident prefix (option resident_prefix): the candidate prefix lengths are
+// 0, the longest prefix that leaves a region every remaining unit (and with
+// two co-resident blocks every adjacent pair of remaining units) fits, and
+// the longest prefixes within 1/4, 1/2 and 3/4 of that one's bytes.  Each is
+// searched exactly; the smallest predicted time wins (ties: shorter prefix).
+static int search_with_prefix(swapnet_plan* p, std::vector<uint32_t>* best_cuts) {
+  const int U = (int)p->units.size();
+  const uint64_t region = p->region;
+  std::vector<uint64_t> pb(U + 1, 0);
+  std::vector<int64_t> pex(U + 1, 0);
+  for (int j = 0; j < U; ++j) {
+    pb[j + 1] = pb[j] + p->units[j].bytes;
+    pex[j + 1] = pex[j] + p->units[j].t_ex;
+  }
+  std::vector<uint64_t> need(U + 1, 0);  // smallest region units [r, U) need
+  for (int r = U - 1; r >= 0; --r) {
+    uint64_t m = std::max(need[r + 1], p->units[r].bytes);
+    if (p->opt.slots == 2 && r + 1 < U) m = std::max(m, p->units[r].bytes + p->units[r + 1].bytes);
+    need[r] = m;
+  }
+  int rmax = 0;
+  for (int r = 1; r <= U; ++r)
+    if (align_up(pb[r]) + need[r] <= region) rmax = r;
+  std::vector<int> cand{0};
+  for (int q = 1; q <= 3; ++q) {
+    int r = 0;
+    for (int j = 1; j <= rmax; ++j)
+      if (pb[j] * 4 <= pb[rmax] * (uint64_t)q) r = j;
+    cand.push_back(r);
+  }
+  cand.push_back(rmax);
+  std::sort(cand.begin(), cand.end());
+  cand.erase(std::unique(cand.begin(), cand.end()), cand.end());
+  int64_t best = INT64_MAX;
+  int best_r = -1;
+  bool best_exact = true;
+  std::vector<uint32_t> cuts;
+  for (int r : cand) {
+    p->prefix_units = r;
+    p->prefix_bytes = r > 0 ? align_up(pb[r]) : 0;
+    p->region = region - p->prefix_bytes;
+    std::vector<uint32_t> c;
+    int64_t ns = 0;
+    if (r == U) {  // everything fits: the prefix is the whole model
+      c = {};
+      ns = pex[U];
+      p->exact = true;
+    } else {
+      const int rc = search_pipeline(p, &c, &ns, r, pex[r]);
+      if (rc == SWAPNET_ERR_INFEASIBLE) continue;
+      if (rc) return rc;
+    }
+    if (ns < best) {
+      best = ns;
+      best_r = r;
+      best_exact = p->exact;
+      cuts = c;
+    }
+  }
+  if (best_r < 0) SN_FAIL(SWAPNET_ERR_INFEASIBLE, "no feasible partition");
+  p->prefix_units = best_r;
+  p->prefix_bytes = best_r > 0 ? align_up(pb[best_r]) : 0;
+  p->region = region - p->prefix_bytes;
+  p->exact = best_exact;
+  *best_cuts = cuts;
   return SWAPNET_OK;
 }
 
@@ -620,6 +718,10 @@ static int check_options(const swapnet_options& o) {
   if (o.graphs != 0 && o.graphs != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "graphs must be 0 or 1");
   if (o.preloaded != 0 && o.preloaded != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "preloaded must be 0 or 1");
   if (o.branches != 0 && o.branches != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "branches must be 0 or 1");
+  if (o.resident_prefix != 0 && o.resident_prefix != 1)
+    SN_FAIL(SWAPNET_ERR_INVALID_ARG, "resident_prefix must be 0 or 1");
+  if (o.resident_prefix && o.objective != 0)
+    SN_FAIL(SWAPNET_ERR_INVALID_ARG, "resident_prefix needs the pipeline objective (0)");
   return SWAPNET_OK;
 }
 
@@ -675,7 +777,9 @@ int swapnet_partition(const swapnet_model_desc* desc, uint64_t budget, const swa
     int rc = prepare(desc, budget, opt, &p);
     if (rc) return rc;
     std::vector<uint32_t> cuts;
-    rc = p->opt.objective == 0 ? search_pipeline(p.get(), &cuts) : search_exhaustive_eq4(p.get(), &cuts);
+    if (p->opt.objective != 0) rc = search_exhaustive_eq4(p.get(), &cuts);
+    else if (p->opt.resident_prefix) rc = search_with_prefix(p.get(), &cuts);
+    else rc = search_pipeline(p.get(), &cuts);
     if (rc) return rc;
     finalize_blocks(p.get(), cuts);
     *out = p.release();
@@ -752,6 +856,8 @@ int swapnet_plan_info_get(const swapnet_plan* p, swapnet_plan_info* info) {
   r.predicted_ns = p->predicted;
   r.state_bytes = p->model.state_bytes;
   r.exact = p->exact ? 1 : 0;
+  r.prefix_units = (uint32_t)p->prefix_units;
+  r.prefix_bytes = p->prefix_bytes;
   *info = r;
   return SWAPNET_OK;
 }

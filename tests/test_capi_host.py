@@ -96,6 +96,61 @@ def test_partition_equals_exhaustive_oracle(slots, act_in_budget):
     assert checked >= 10
 
 
+@pytest.mark.parametrize("slots", [1, 2])
+def test_resident_prefix_partition_equals_exhaustive_oracle(slots):
+    """The resident-prefix extension: prefix length and cuts identical to
+    the oracle's brute force over the same candidate prefixes."""
+    r = np.random.default_rng(300 + slots)
+    checked = with_prefix = 0
+    for trial in range(40):
+        m = _random_model(r, int(r.integers(2, 9)))
+        opt = capi.options(slots=slots, resident_prefix=1,
+                           alpha_as_per_byte=int(r.integers(1_000_000, 5_000_000)),
+                           beta_ns_per_tensor=int(r.integers(0, 3000)),
+                           gamma_as_per_flop=int(r.integers(100, 100_000)),
+                           eta_ns_per_tensor=int(r.integers(0, 500)))
+        wb = P.weight_bytes(m)
+        if wb == 0:
+            continue
+        budget = int(r.integers(max(1, wb // 4), wb * 2 + 1))
+        ref = P.exhaustive_partition(m, budget, _coef(opt), slots=slots, resident_prefix=True)
+        desc = capi.Desc(m)
+        if ref is None:
+            with pytest.raises(capi.SwapnetError) as ei:
+                capi.Plan.partition(desc, budget, opt)
+            assert ei.value.code == capi.ERR_INFEASIBLE
+            continue
+        plan = capi.Plan.partition(desc, budget, opt)
+        info = plan.info()
+        assert info["prefix_units"] == ref["prefix_units"], (trial, info["prefix_units"], ref["prefix_units"])
+        assert info["prefix_bytes"] == ref["prefix_bytes"]
+        assert plan.cuts() == ref["cuts"]
+        assert info["n_blocks"] == ref["n"]
+        assert info["predicted_ns"] == ref["predicted_ns"]
+        blocks = plan.blocks()
+        if ref["prefix_units"]:
+            with_prefix += 1
+            assert blocks[0]["slot"] == 0xFFFFFFFF and blocks[0]["offset"] == 0
+            assert blocks[0]["unit1"] == ref["prefix_units"]
+            for b in blocks[1:]:  # swapped blocks sit in the region beside the prefix
+                assert b["offset"] >= ref["prefix_bytes"]
+                assert b["offset"] + b["bytes"] <= info["arena_bytes"] // 256 * 256
+        checked += 1
+    assert checked >= 10 and with_prefix >= 3
+
+
+def test_resident_prefix_never_worse_than_swapping_everything():
+    for name in ("mlp6", "resnet50", "vgg16"):
+        m = synth.arch.MODELS[name]()
+        wb = P.weight_bytes(m)
+        budget = int(wb * 0.4) // 256 * 256 if name != "mlp6" else 8_462_336
+        act = 1 if name == "mlp6" else 0
+        a = capi.Plan.partition(capi.Desc(m), budget, capi.options(activations_in_budget=act)).info()
+        b = capi.Plan.partition(capi.Desc(m), budget,
+                                capi.options(activations_in_budget=act, resident_prefix=1)).info()
+        assert b["predicted_ns"] <= a["predicted_ns"]
+
+
 def test_partition_eq4_objective_equals_oracle():
     r = np.random.default_rng(5)
     for _ in range(20):

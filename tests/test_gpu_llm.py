@@ -197,6 +197,33 @@ def test_llm_swapped_equals_resident():
         tok = np.array([a[1][0]], dtype=np.int32)
 
 
+def test_llm_resident_prefix_equals_resident():
+    """Decoder engines whose first units stay resident between passes."""
+    import torch
+    sw = Decoder(prefill_tokens=32, budget_frac=0.5)
+    rs = Decoder(prefill_tokens=32, resident=True, host=sw.host, weights=sw.w)
+    # rebuild the swapped engines with resident_prefix plans sharing sw's state
+    for i, m in enumerate((sw.mp, sw.md)):
+        budget = int(OP.weight_bytes(sw.mp) * 0.5) // 256 * 256
+        plan = capi.Plan.partition(capi.Desc(m), budget, capi.options(resident_prefix=1))
+        assert plan.info()["prefix_units"] > 0
+        eng = capi.Engine(plan, sw.host)
+        eng.bind_state(sw.state.data_ptr(), sw.state_bytes)
+        info = plan.info()
+        din = torch.zeros(max(16, info["input_bytes"]), dtype=torch.uint8, device="cuda")
+        dout = torch.zeros(info["output_bytes"], dtype=torch.uint8, device="cuda")
+        sw.engines[i] = (plan, eng, info)
+        sw.bufs[i] = (din, dout, plan.output_offsets())
+    ids = synth.gen.model_input(sw.mp).reshape(-1)
+    a, b = sw.run(0, ids), rs.run(0, ids)
+    assert a[0].tobytes() == b[0].tobytes() and a[1].tobytes() == b[1].tobytes()
+    tok = np.array([a[1][-1]], dtype=np.int32)
+    for _ in range(4):
+        a, b = sw.run(1, tok), rs.run(1, tok)
+        assert a[0].tobytes() == b[0].tobytes()
+        tok = np.array([a[1][0]], dtype=np.int32)
+
+
 def test_llm_cache_bound_reported_not_faulted():
     dec = Decoder(prefill_tokens=64)
     ids = synth.gen.model_input(dec.mp).reshape(-1)

@@ -297,3 +297,24 @@ def test_concurrent_branches_bit_exact(name):
     sw = Runner(m, w, capi.Plan.partition(d, budget, capi.options(branches=1)), host).run(x)
     for a, b, c in zip(seq, par, sw):
         assert a.tobytes() == b.tobytes() == c.tobytes()
+
+
+@pytest.mark.parametrize("name", ["resnet50", "yolov3"])
+def test_resident_prefix_bit_exact_over_repeated_inferences(name):
+    """Resident-prefix plans (an extension: the first units stay in the arena
+    between inferences) give the resident plan's bits on every call, so the
+    prefix is not disturbed by the blocks swapped beside it."""
+    m = synth.arch.MODELS[name]()
+    w = synth.gen.model_weights(m)
+    d = capi.Desc(m)
+    host = capi.HostWeights(w)
+    budget = int(OP.weight_bytes(m) * 0.4) // 256 * 256
+    plan = capi.Plan.partition(d, budget, capi.options(resident_prefix=1))
+    info = plan.info()
+    assert info["prefix_units"] > 0 and info["n_blocks"] > 1
+    sw = Runner(m, w, plan, host)
+    rs = Runner(m, w, capi.Plan.resident(d), host)
+    for req in range(3):
+        x = synth.gen.model_input(m, request=req)
+        a, b = sw.run(x), rs.run(x)
+        assert all(p.tobytes() == q.tobytes() for p, q in zip(a, b)), req

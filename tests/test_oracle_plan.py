@@ -213,3 +213,32 @@ def test_rule_count_is_fewest_feasible_blocks():
         assert fewest == P.block_count_rule(s, budget) == 6 // per_block
         assert P.exhaustive_partition(m, budget, coef)["n"] >= fewest
     assert P.evaluate_cuts(m, s, coef, []) is not None   # one block fits when s <= b
+
+
+def test_pipeline_with_resident_prefix_hand_worked():
+    """Resident prefix (extension): block 0 runs from t = 0 without a copy
+    and never frees room, so block 2 may start copying as soon as block 1's
+    copy ends.  Worked by hand: prefix t_ex 5; blocks (t_in, t_ex) = (3, 2),
+    (4, 1), (2, 2); two slots.  Copies end at 3, 7, 9 (block 3 waits for
+    block 1's release at 7); executions end at 7, 8, 11."""
+    blocks = [(0, 0, 5, 0), (10, 3, 2, 0), (10, 4, 1, 0), (10, 2, 2, 0)]
+    assert P.pipeline_time(blocks, 2, prefix=True) == 11
+    # read as an ordinary first block the same numbers make block 2 wait for
+    # block 0's release at 5: a different (later) finish
+    assert P.pipeline_time(blocks, 2) == 13
+    # one slot: every copy waits for the previous swapped block's release
+    assert P.pipeline_time(blocks, 1, prefix=True) == max(5, 3) + 2 + 4 + 1 + 2 + 2
+
+
+def test_prefix_candidates_rule():
+    us = [dict(bytes=b) for b in (256, 512, 256, 1024, 512)]
+    cands, pb = P.prefix_candidates(us, region=2048, slots=2)
+    # the remaining units always include the pair 1024 + 512 = 1536 while
+    # unit 3 is swapped: r = 1 (256 bytes) fits (1792), r = 2 (768) does not
+    # (2304); r = 4 leaves 512 beside 2048 bytes of prefix: 2560 > 2048
+    assert cands == [0, 1]
+    assert pb == [0, 256, 768, 1024, 2048, 2560]
+    cands1, _ = P.prefix_candidates(us, region=2048, slots=1)
+    # one slot: the rest needs only its largest unit; r = 3 leaves 1024 beside
+    # 1024 bytes of prefix (exactly 2048), r = 4 would need 2048 + 512
+    assert max(cands1) == 3
