@@ -550,6 +550,68 @@ def run_ablation(args):
                       "paper_block_count": n_min, "steps": args.steps, "results": out}))
 
 
+def run_adapt_study(args):
+    """Dynamic-budget case study (the paper's Sec. 8 adaptation experiment,
+    on ResNet-50 here): plans for three budgets are made ahead; one engine
+    runs `steps` inferences per phase and switches plan between phases with
+    swapnet_engine_adapt.  Reports per phase the budget, blocks, latency,
+    the planning time and the switch time."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2401_16757_gb300 import capi
+    name = args.config if args.config in ("resnet50", "vgg16_b1", "yolov3") else "resnet50"
+    m, w, x, wb, _, text = build_workload(name, capi_weight_bytes)
+    host = capi.HostWeights(w)
+    d = capi.Desc(m)
+    fracs = (0.80, 0.60, 0.40)
+    # offline profiling once (Sec. 6.1), then the look-up table of plans
+    plan0 = capi.Plan.partition(d, int(wb * fracs[-1]) // 256 * 256, capi.options())
+    eng0 = capi.Engine(plan0, host)
+    t_ex, alpha = capi.calibrate(m, plan0, eng0)
+    eng0.free()
+    dc = capi.Desc(m, t_ex_ns=t_ex)
+    opt = capi.options(alpha_as_per_byte=alpha or 4_750_000, beta_ns_per_tensor=0, eta_ns_per_tensor=0)
+    plans, t_plan = [], []
+    for f in fracs:
+        t0 = time.perf_counter()
+        plans.append(capi.Plan.partition(dc, int(wb * f) // 256 * 256, opt))
+        t_plan.append((time.perf_counter() - t0) * 1e3)
+    stream = torch.cuda.current_stream()
+    flush = torch.empty(512 << 20, dtype=torch.uint8, device="cuda")
+    info = plans[0].info()
+    d_in = torch.empty(max(16, info["input_bytes"]), dtype=torch.uint8, device="cuda")
+    d_in[:info["input_bytes"]].copy_(torch.from_numpy(x.view(np.uint8).reshape(-1)))
+    d_out = torch.empty(info["output_bytes"], dtype=torch.uint8, device="cuda")
+    eng = capi.Engine(plans[0], host)
+    phases = []
+    for i, (f, p) in enumerate(zip(fracs, plans)):
+        t_sw = None
+        if i:
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            eng.adapt(p)
+            t_sw = (time.perf_counter() - t0) * 1e3
+        for _ in range(3):
+            eng.infer(d_in.data_ptr(), d_out.data_ptr(), stream.cuda_stream)
+        ts = []
+        for _ in range(args.steps):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            eng.infer(d_in.data_ptr(), d_out.data_ptr(), stream.cuda_stream)
+            b.record(stream)
+            b.synchronize()
+            ts.append(a.elapsed_time(b))
+        pi = p.info()
+        phases.append({"budget_frac": f, "budget_bytes": pi["budget_bytes"], "n_blocks": pi["n_blocks"],
+                       "cuts": p.cuts(), "ms": statistics.median(ts), "plan_ms": t_plan[i],
+                       "switch_ms": t_sw, "free_device_bytes": torch.cuda.mem_get_info()[0]})
+    eng.sync()
+    print(json.dumps({"adapt_study": name, "workload": text, "weight_bytes": wb, "steps": args.steps,
+                      "phases": phases}))
+
+
 def run_profile_once(args):
     """One resident inference of a single-model config (no timing)."""
     import torch
@@ -653,6 +715,8 @@ def main():
     ap.add_argument("--ablation", action="store_true",
                     help="partition ablations of --config (planner vs equal-byte plans, Eq. 4, sequential "
                          "layers, zero-copy swap, DInf); prints one JSON line")
+    ap.add_argument("--adapt-study", action="store_true",
+                    help="dynamic-budget case study: one engine switched between plans for 80/60/40 % budgets")
     ap.add_argument("--profile-once", action="store_true",
                     help="run one resident inference of --config through the C ABI and exit "
                          "(a driver for profiler captures of its kernels); prints one JSON line")
@@ -670,6 +734,9 @@ def main():
         return
     if args.ablation:
         run_ablation(args)
+        return
+    if args.adapt_study:
+        run_adapt_study(args)
         return
     if args.config in ("llm", "multi"):
         import torch

@@ -313,6 +313,21 @@ int swapnet_infer_host(swapnet_engine* eng, const void* h_input, void* h_output,
  * on a device error. */
 int swapnet_engine_sync(swapnet_engine* eng);
 
+/* Runtime budget adaptation (Sec. 6.2.2 "adaptively partition and exchange
+ * blocks"; the dynamic-budget case study of Sec. 8): switch a loaded engine,
+ * between inferences, to another plan of the same model, e.g. one of several
+ * plans made ahead with swapnet_partition for different budgets (the
+ * paper's look-up table of partitions).  Waits for the engine's work in
+ * flight; keeps the host registration, streams, workspace and bound decoder
+ * state; re-derives blocks, copy segments, unit pointers and descriptors
+ * (the paper's "repeat steps 2 and 3"); re-allocates an engine-owned arena
+ * at the new plan's size, releasing the old one first, so a smaller budget
+ * gives memory back.  A caller-provided arena stays and must hold the new
+ * plan.  The plan is copied; the caller may free it after the call.
+ * Errors: INVALID_ARG (a plan for another model, or resident <-> swapped),
+ * OOM, CUDA. */
+int swapnet_engine_adapt(swapnet_engine* eng, const swapnet_plan* plan);
+
 /* Decoder state of a model with ATTENTION layers: a device buffer of
  * state_bytes (plan info), caller-owned, 256-byte aligned.  Layout: an int32
  * position (tokens already cached) in the first 256 bytes, then for every

@@ -95,7 +95,7 @@ EXPORTS = ["swapnet_default_options", "swapnet_partition", "swapnet_plan_from_cu
            "swapnet_plan_info_get", "swapnet_plan_cuts", "swapnet_plan_units", "swapnet_plan_blocks",
            "swapnet_plan_output_offsets", "swapnet_plan_free", "swapnet_schedule", "swapnet_load",
            "swapnet_infer", "swapnet_infer_host", "swapnet_engine_sync", "swapnet_engine_blocks",
-           "swapnet_engine_free", "swapnet_engine_stats_get", "swapnet_engine_unit_kernels", "swapnet_engine_unit_tiling",
+           "swapnet_engine_free", "swapnet_engine_stats_get", "swapnet_engine_unit_kernels", "swapnet_engine_unit_tiling", "swapnet_engine_adapt",
            "swapnet_engine_set_profiling", "swapnet_engine_last_times", "swapnet_engine_measure_units",
            "swapnet_engine_last_timeline",
            "swapnet_engine_bind_state", "swapnet_strerror", "swapnet_last_error", "swapnet_debug_fail_next", "swapnet_gemm_noalloc"]
@@ -138,6 +138,7 @@ def lib():
         "swapnet_infer": (C.c_int, [P, P, P, P]),
         "swapnet_infer_host": (C.c_int, [P, P, P, P]),
         "swapnet_engine_sync": (C.c_int, [P]),
+        "swapnet_engine_adapt": (C.c_int, [P, P]),
         "swapnet_engine_bind_state": (C.c_int, [P, P, C.c_uint64]),
         "swapnet_engine_blocks": (C.c_int, [P, C.POINTER(EngineBlock), C.c_uint32, C.POINTER(C.c_uint32)]),
         "swapnet_engine_free": (None, [P]),
@@ -420,6 +421,10 @@ class Engine:
 
     def sync(self):
         check(lib().swapnet_engine_sync(self.h), "swapnet_engine_sync")
+
+    def adapt(self, plan):
+        """Switch to another plan of the same model (a new budget)."""
+        check(lib().swapnet_engine_adapt(self.h, plan.h), "swapnet_engine_adapt")
 
     def blocks(self):
         n = C.c_uint32()

@@ -88,6 +88,7 @@ struct swapnet_engine {
   int num_sms = 0;
   char* d_arena = nullptr;
   bool own_arena = false;
+  uint64_t arena_bytes = 0;
   char* d_ws = nullptr;
   bool own_ws = false;
   char* d_in_stage = nullptr;
@@ -599,76 +600,38 @@ static int run_unit(swapnet_engine* e, int u, const void* din, void* dout, cudaS
   }
 }
 
-}  // namespace swapnet
-
-extern "C" {
-
-int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint32_t n_tensors, void* d_arena,
-                 uint64_t arena_bytes, void* d_workspace, uint64_t workspace_bytes, swapnet_engine** out) {
-  if (!plan || !out || (n_tensors && !host_weights)) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
-  if ((int)n_tensors != plan->model.n_tensors)
-    SN_FAIL(SWAPNET_ERR_INVALID_ARG, "expected " + std::to_string(plan->model.n_tensors) + " host tensors");
-  if (((uintptr_t)d_arena | (uintptr_t)d_workspace) % kAlign)
-    SN_FAIL(SWAPNET_ERR_MISALIGNED, "device buffers must be 256-byte aligned");
+// Everything an engine derives from its plan: arena (allocated when the
+// engine owns it), copy segments, unit pointers and TMA descriptors, side
+// branches, split-K scratch, the resident upload or prefix upload, and the
+// swap variants.  Used by swapnet_load and again by swapnet_engine_adapt.
+static int bind_plan(swapnet_engine* e, void* d_arena_user, uint64_t arena_bytes_user, bool preloaded_arena) {
+  const swapnet_plan* plan = &e->plan;
   const uint64_t arena_need = plan->prefix_bytes + plan->region;  // resident prefix, then the swap region
-  if (d_arena && arena_bytes < arena_need) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "arena buffer too small");
+  if (d_arena_user && arena_bytes_user < arena_need) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "arena buffer too small");
   for (const Block& B : plan->blocks)  // every block lies inside the arena
     if (B.base + B.bytes > arena_need) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "plan places a block outside the arena");
-  if (d_workspace && workspace_bytes < plan->model.ws_bytes)
-    SN_FAIL(SWAPNET_ERR_INVALID_ARG, "workspace buffer too small");
-  swapnet_engine* e = new (std::nothrow) swapnet_engine();
-  if (!e) SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
-  std::unique_ptr<swapnet_engine, int (*)(swapnet_engine*)> guard(e, release);
-  try {
-    e->plan = *plan;
-  } catch (const std::bad_alloc&) {
-    SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
-  }
-  CU(cudaGetDevice(&e->device), "cudaGetDevice");
-  CU(cudaDeviceGetAttribute(&e->num_sms, cudaDevAttrMultiProcessorCount, e->device), "device attribute");
-  e->zc_ctas = plan->opt.zc_ctas > 0 ? plan->opt.zc_ctas : 32;
-  int rc = tc_error_word(&e->err_word);
-  if (rc) return rc;
-  // device memory
-  if (d_arena) {
-    e->d_arena = static_cast<char*>(d_arena);
-  } else {
+  if (d_arena_user) {
+    e->d_arena = static_cast<char*>(d_arena_user);
+    e->arena_bytes = arena_bytes_user;
+  } else if (!e->own_arena || e->arena_bytes != std::max<uint64_t>(arena_need, kAlign)) {
+    if (e->own_arena && e->d_arena) cudaFree(e->d_arena);  // a new budget: give the old arena back
+    e->d_arena = nullptr;
+    e->own_arena = false;
     if (injected(2)) SN_FAIL(SWAPNET_ERR_OOM, "arena allocation failed (injected)");
-    if (cudaMalloc(&e->d_arena, std::max<uint64_t>(arena_need, kAlign)) != cudaSuccess) {
+    const uint64_t bytes = std::max<uint64_t>(arena_need, kAlign);
+    if (cudaMalloc(&e->d_arena, bytes) != cudaSuccess) {
       cudaGetLastError();
+      e->d_arena = nullptr;
       SN_FAIL(SWAPNET_ERR_OOM, "arena allocation failed");
     }
     e->own_arena = true;
+    e->arena_bytes = bytes;
     // touch every page now, so that the first inference does not pay for
     // the driver backing fresh allocations
-    CU(cudaMemset(e->d_arena, 0, std::max<uint64_t>(arena_need, kAlign)), "arena first touch");
+    CU(cudaMemset(e->d_arena, 0, bytes), "arena first touch");
   }
-  if (d_workspace || plan->model.ws_bytes == 0) {
-    e->d_ws = static_cast<char*>(d_workspace);
-  } else {
-    if (injected(2)) SN_FAIL(SWAPNET_ERR_OOM, "workspace allocation failed (injected)");
-    if (cudaMalloc(&e->d_ws, plan->model.ws_bytes) != cudaSuccess) {
-      cudaGetLastError();
-      SN_FAIL(SWAPNET_ERR_OOM, "workspace allocation failed");
-    }
-    e->own_ws = true;
-    CU(cudaMemset(e->d_ws, 0, plan->model.ws_bytes), "workspace first touch");
-  }
-  if (injected(3)) SN_FAIL(SWAPNET_ERR_CUDA, "stream creation failed (injected)");
-  int lo = 0, hi = 0;
-  CU(cudaDeviceGetStreamPriorityRange(&lo, &hi), "stream priority range");
-  CU(cudaStreamCreateWithPriority(&e->copy, cudaStreamNonBlocking, hi), "copy stream");
-  for (int s = 0; s < 2; ++s) {
-    CU(cudaEventCreateWithFlags(&e->slot_free[s], cudaEventDisableTiming), "event");
-    CU(cudaEventCreateWithFlags(&e->ready[s], cudaEventDisableTiming), "event");
-  }
-  CU(cudaStreamCreateWithFlags(&e->cap, cudaStreamNonBlocking), "capture stream");
-  CU(cudaEventCreateWithFlags(&e->fork, cudaEventDisableTiming), "event");
-  CU(cudaEventCreateWithFlags(&e->join, cudaEventDisableTiming), "event");
-  rc = register_host(e, host_weights, n_tensors);
-  if (rc) return rc;
   build_segments(e);
-  rc = prepare_units(e);
+  int rc = prepare_units(e);
   if (rc) return rc;
   rc = plan_side(e);
   if (rc) return rc;
@@ -685,6 +648,7 @@ int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint
       e->splitk_bytes = e->splitk_counter_bytes + part;
       if (injected(2) || cudaMalloc(&e->d_splitk, e->splitk_bytes) != cudaSuccess) {
         cudaGetLastError();
+        e->d_splitk = nullptr;
         SN_FAIL(SWAPNET_ERR_OOM, "split-K scratch allocation failed");
       }
       CU(cudaMemset(e->d_splitk, 0, e->splitk_counter_bytes), "split-K counters");
@@ -692,7 +656,7 @@ int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint
   }
   const int variant = plan->opt.swap_variant;
   if (plan->resident) {
-    if (!(plan->opt.preloaded && d_arena)) {
+    if (!preloaded_arena) {
       for (size_t k = 0; k < e->blocks.size() && !rc; ++k) rc = swap_block(e, k, SWAPNET_SWAP_MEMCPY, e->copy);
       if (rc) return rc;
       CU(cudaStreamSynchronize(e->copy), "resident upload");
@@ -717,8 +681,114 @@ int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint
         SN_FAIL(SWAPNET_ERR_MISALIGNED, "zero-copy needs 16-byte aligned host tensors");
     }
   }
+  return SWAPNET_OK;
+}
+
+// Drop what bind_plan derived from the previous plan (the arena stays
+// allocated until bind_plan knows the new size).
+static void unbind_plan(swapnet_engine* e) {
+  for (auto& kv : e->graphs) cudaGraphExecDestroy(kv.second);
+  e->graphs.clear();
+  for (cudaEvent_t& ev : e->side_done)
+    if (ev) cudaEventDestroy(ev);
+  e->side_done.clear();
+  for (cudaEvent_t ev : e->ev_unit) cudaEventDestroy(ev);
+  for (cudaEvent_t ev : e->ev_swap) cudaEventDestroy(ev);
+  e->ev_unit.clear();
+  e->ev_swap.clear();
+  if (e->d_splitk) cudaFree(e->d_splitk);
+  e->d_splitk = nullptr;
+  e->splitk_bytes = e->splitk_counter_bytes = 0;
+  e->weights_loaded = false;
+}
+
+}  // namespace swapnet
+
+extern "C" {
+
+int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint32_t n_tensors, void* d_arena,
+                 uint64_t arena_bytes, void* d_workspace, uint64_t workspace_bytes, swapnet_engine** out) {
+  if (!plan || !out || (n_tensors && !host_weights)) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+  if ((int)n_tensors != plan->model.n_tensors)
+    SN_FAIL(SWAPNET_ERR_INVALID_ARG, "expected " + std::to_string(plan->model.n_tensors) + " host tensors");
+  if (((uintptr_t)d_arena | (uintptr_t)d_workspace) % kAlign)
+    SN_FAIL(SWAPNET_ERR_MISALIGNED, "device buffers must be 256-byte aligned");
+  if (d_workspace && workspace_bytes < plan->model.ws_bytes)
+    SN_FAIL(SWAPNET_ERR_INVALID_ARG, "workspace buffer too small");
+  swapnet_engine* e = new (std::nothrow) swapnet_engine();
+  if (!e) SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
+  std::unique_ptr<swapnet_engine, int (*)(swapnet_engine*)> guard(e, release);
+  try {
+    e->plan = *plan;
+  } catch (const std::bad_alloc&) {
+    SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
+  }
+  CU(cudaGetDevice(&e->device), "cudaGetDevice");
+  CU(cudaDeviceGetAttribute(&e->num_sms, cudaDevAttrMultiProcessorCount, e->device), "device attribute");
+  e->zc_ctas = plan->opt.zc_ctas > 0 ? plan->opt.zc_ctas : 32;
+  int rc = tc_error_word(&e->err_word);
+  if (rc) return rc;
+  if (d_workspace || plan->model.ws_bytes == 0) {
+    e->d_ws = static_cast<char*>(d_workspace);
+  } else {
+    if (injected(2)) SN_FAIL(SWAPNET_ERR_OOM, "workspace allocation failed (injected)");
+    if (cudaMalloc(&e->d_ws, plan->model.ws_bytes) != cudaSuccess) {
+      cudaGetLastError();
+      SN_FAIL(SWAPNET_ERR_OOM, "workspace allocation failed");
+    }
+    e->own_ws = true;
+    CU(cudaMemset(e->d_ws, 0, plan->model.ws_bytes), "workspace first touch");
+  }
+  if (injected(3)) SN_FAIL(SWAPNET_ERR_CUDA, "stream creation failed (injected)");
+  int lo = 0, hi = 0;
+  CU(cudaDeviceGetStreamPriorityRange(&lo, &hi), "stream priority range");
+  CU(cudaStreamCreateWithPriority(&e->copy, cudaStreamNonBlocking, hi), "copy stream");
+  for (int s = 0; s < 2; ++s) {
+    CU(cudaEventCreateWithFlags(&e->slot_free[s], cudaEventDisableTiming), "event");
+    CU(cudaEventCreateWithFlags(&e->ready[s], cudaEventDisableTiming), "event");
+  }
+  CU(cudaStreamCreateWithFlags(&e->cap, cudaStreamNonBlocking), "capture stream");
+  CU(cudaEventCreateWithFlags(&e->fork, cudaEventDisableTiming), "event");
+  CU(cudaEventCreateWithFlags(&e->join, cudaEventDisableTiming), "event");
+  rc = register_host(e, host_weights, n_tensors);
+  if (rc) return rc;
+  rc = bind_plan(e, d_arena, arena_bytes, plan->resident && plan->opt.preloaded && d_arena);
+  if (rc) return rc;
   e->stats = swapnet_engine_stats{};
   *out = guard.release();
+  return SWAPNET_OK;
+}
+
+int swapnet_engine_adapt(swapnet_engine* e, const swapnet_plan* plan) {
+  if (!e || !plan) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+  const Model& a = e->plan.model;
+  const Model& b = plan->model;
+  bool same = a.L.size() == b.L.size() && a.n_tensors == b.n_tensors && a.dtype == b.dtype &&
+              a.weight_bytes == b.weight_bytes && a.in_bytes == b.in_bytes && a.ws_bytes == b.ws_bytes;
+  for (size_t i = 0; same && i < a.L.size(); ++i)
+    same = std::memcmp(&a.L[i].d, &b.L[i].d, sizeof(swapnet_layer)) == 0 ||
+           (a.L[i].d.op == b.L[i].d.op && a.L[i].d.cin == b.L[i].d.cin && a.L[i].d.cout == b.L[i].d.cout &&
+            a.L[i].tbytes[0] == b.L[i].tbytes[0] && a.L[i].tbytes[1] == b.L[i].tbytes[1]);
+  if (!same) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "the plan is for a different model");
+  if (plan->resident != e->plan.resident) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "cannot switch between resident and swapped plans");
+  CU(cudaSetDevice(e->device), "cudaSetDevice");
+  CU(cudaStreamSynchronize(e->copy), "drain copies");
+  if (e->side) CU(cudaStreamSynchronize(e->side), "drain side stream");
+  CU(cudaDeviceSynchronize(), "drain inferences");
+  swapnet::unbind_plan(e);
+  try {
+    e->plan = *plan;
+  } catch (const std::bad_alloc&) {
+    SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
+  }
+  // an engine given a caller arena keeps it (the new plan must fit it)
+  int rc = swapnet::bind_plan(e, e->own_arena ? nullptr : e->d_arena, e->own_arena ? 0 : e->arena_bytes, false);
+  if (rc) return rc;
+  if (e->profiling) {
+    e->profiling = false;
+    rc = swapnet_engine_set_profiling(e, 1);
+    if (rc) return rc;
+  }
   return SWAPNET_OK;
 }
 

@@ -318,3 +318,33 @@ def test_resident_prefix_bit_exact_over_repeated_inferences(name):
         x = synth.gen.model_input(m, request=req)
         a, b = sw.run(x), rs.run(x)
         assert all(p.tobytes() == q.tobytes() for p, q in zip(a, b)), req
+
+
+def test_engine_adapts_to_new_budgets_between_inferences():
+    """Runtime budget adaptation: one engine switched through plans for
+    shrinking and growing budgets (made ahead, like the paper's look-up
+    table) gives the resident bits after every switch; a plan for another
+    model is refused."""
+    import torch
+    m = synth.arch.resnet50()
+    w = synth.gen.model_weights(m)
+    d = capi.Desc(m)
+    host = capi.HostWeights(w)
+    wb = OP.weight_bytes(m)
+    plans = {f: capi.Plan.partition(d, int(wb * f) // 256 * 256, capi.options()) for f in (0.8, 0.5, 0.3, 0.6)}
+    sw = Runner(m, w, plans[0.8], host)
+    rs = Runner(m, w, capi.Plan.resident(d), host)
+    free0 = torch.cuda.mem_get_info()[0]
+    for i, f in enumerate((0.8, 0.5, 0.3, 0.6)):
+        if i:
+            sw.engine.adapt(plans[f])
+        x = synth.gen.model_input(m, request=i)
+        a, b = sw.run(x), rs.run(x)
+        assert all(p.tobytes() == q.tobytes() for p, q in zip(a, b)), f
+        assert sw.engine.stats()["infer_calls"] >= 1
+    other = synth.arch.vgg16()
+    with pytest.raises(capi.SwapnetError) as ei:
+        sw.engine.adapt(capi.Plan.partition(capi.Desc(other), int(OP.weight_bytes(other) * 0.5), capi.options()))
+    assert ei.value.code == capi.ERR_INVALID_ARG
+    with pytest.raises(capi.SwapnetError):
+        sw.engine.adapt(capi.Plan.resident(d))
