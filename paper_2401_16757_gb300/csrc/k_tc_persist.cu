@@ -43,11 +43,15 @@ constexpr int kPBM = 128;
 constexpr int kPBK = 64;  // one 128-byte swizzle row of 16-bit elements
 constexpr int kPA = kPBM * kPBK * 2;
 
-template <int BN> struct PCfg {
-  static constexpr int kStages = BN == 256 ? 4 : (BN == 128 ? 6 : 8);
+// MS: 128-row sub-tiles per tile sharing each weight stage (1, or 2 for
+// N tiles of 64, where one 128x64 MMA per k16 step is too little work per
+// stage): a tile is then 256 x BN, two accumulators side by side in TMEM.
+template <int BN, int MS> struct PCfg {
+  static constexpr int kStages = BN == 256 ? 4 : (BN == 128 ? 6 : (MS == 2 ? 5 : 8));
   static constexpr int kLag = kStages - 2;  // gather: cp.async groups in flight per thread
   static constexpr int kB = BN * kPBK * 2;
-  static constexpr int kStageBytes = kStages * (kPA + kB);
+  static constexpr int kSA = MS * kPA;      // A bytes per stage
+  static constexpr int kStageBytes = kStages * (kSA + kB);
   static constexpr int kBias = 2 * 4 * BN * 4;  // [buffer][epilogue warp][BN] fp32
   static constexpr int kSmem = kStageBytes + kBias + 256 + 1024;
 };
@@ -56,17 +60,18 @@ constexpr int kAT2d = 0, kAGather = 1, kATap = 2;
 
 template <int AMODE> constexpr int persist_threads() { return AMODE == kAGather ? 320 : 192; }
 
-template <typename T, int BN, int AMODE>
+template <typename T, int BN, int AMODE, int MS>
 __global__ void __launch_bounds__(persist_threads<AMODE>(), 1)
     tc_persist_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const TcArgs p) {
   constexpr bool GATHER = AMODE == kAGather;
-  using Cfg = PCfg<BN>;
+  static_assert(MS == 1 || !GATHER, "the gather threads cover one 128-row sub-tile");
+  using Cfg = PCfg<BN, MS>;
   constexpr int kStages = Cfg::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
-  uint8_t* sB = smem + kStages * kPA;
+  uint8_t* sB = smem + kStages * Cfg::kSA;
   float* sbias = reinterpret_cast<float*>(smem + Cfg::kStageBytes);  // [2][4][BN]
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + Cfg::kStageBytes + Cfg::kBias);
   // bars: full[kStages], empty[kStages], tfull[2], tempty[2], drain
@@ -85,7 +90,8 @@ __global__ void __launch_bounds__(persist_threads<AMODE>(), 1)
   const int mt = AMODE == kATap ? (p.M / hw) * patches : (p.M + kPBM - 1) / kPBM;
   const int nt = (p.N + BN - 1) / BN;
   const uint32_t a_bytes = AMODE == kATap ? (uint32_t)(p.wt * p.ht * 128) : (AMODE == kAT2d ? kPA : 0);
-  const int tiles = mt * nt;
+  const int mtp = (mt + MS - 1) / MS;  // tiles along M (MS sub-tiles each)
+  const int tiles = mtp * nt;
   const int KB = (p.K + kPBK - 1) / kPBK;
   const int my_tiles = blockIdx.x < tiles ? (tiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
   const int work = my_tiles * KB;  // (tile, k-block) items of this CTA
@@ -106,7 +112,7 @@ __global__ void __launch_bounds__(persist_threads<AMODE>(), 1)
     fence_proxy_async_smem();
   }
   if (warp == 1) {
-    tmem_alloc(smem_u32(tmem_slot), 2 * BN);
+    tmem_alloc(smem_u32(tmem_slot), 2 * MS * BN);
     tmem_relinquish();
   }
   if (threadIdx.x == 0) {
@@ -126,29 +132,34 @@ __global__ void __launch_bounds__(persist_threads<AMODE>(), 1)
       auto coords = [&](int g, int* kx, int* m0, int* n0) {
         const int tile = tile_of(g / KB);
         *kx = (g % KB) * kPBK;
-        *m0 = (tile % mt) * kPBM;
-        *n0 = (tile / mt) * BN;
+        *m0 = (tile % mtp) * MS * kPBM;
+        *n0 = (tile / mtp) * BN;
       };
       auto load_a = [&](int s, int g) {
         const int tile = tile_of(g / KB);
         const int k0 = (g % KB) * kPBK;
-        if (AMODE == kAT2d) {
-          tma_load_2d(smem_u32(sA + s * kPA), &tmA, full_bar(s), k0, (tile % mt) * kPBM);
-        } else if (AMODE == kATap) {
-          const int sp = tile % mt;
-          const int img = sp / patches, rem = sp - img * patches;
-          const int th = rem / p.tiles_w, tw = rem - th * p.tiles_w;
-          const int tap = k0 / p.C, c0 = k0 - tap * p.C;
-          const int ry = tap / p.kw, rx = tap - ry * p.kw;
-          tma_load_4d(smem_u32(sA + s * kPA), &tmA, full_bar(s), c0, tw * p.wt * p.stride - p.pad + rx,
-                      th * p.ht * p.stride - p.pad + ry, img);
+#pragma unroll
+        for (int sub = 0; sub < MS; ++sub) {
+          // a sub-tile past the last one reads only out-of-range coordinates (zero fill)
+          const int idx = (tile % mtp) * MS + sub;
+          const uint32_t dst = smem_u32(sA + s * Cfg::kSA + sub * kPA);
+          if (AMODE == kAT2d) {
+            tma_load_2d(dst, &tmA, full_bar(s), k0, idx * kPBM);
+          } else if (AMODE == kATap) {
+            const int img = idx / patches, rem = idx - img * patches;
+            const int th = rem / p.tiles_w, tw = rem - th * p.tiles_w;
+            const int tap = k0 / p.C, c0 = k0 - tap * p.C;
+            const int ry = tap / p.kw, rx = tap - ry * p.kw;
+            tma_load_4d(dst, &tmA, full_bar(s), c0, tw * p.wt * p.stride - p.pad + rx,
+                        th * p.ht * p.stride - p.pad + ry, img);
+          }
         }
       };
       const int early = min(work, kStages);
       for (int g = 0; g < early; ++g) {
         int kx, m0, n0;
         coords(g, &kx, &m0, &n0);
-        mbar_arrive_expect_tx(full_bar(g), Cfg::kB + a_bytes);
+        mbar_arrive_expect_tx(full_bar(g), Cfg::kB + MS * a_bytes);
         tma_load_2d(smem_u32(sB + g * Cfg::kB), &tmB, full_bar(g), kx, n0);
       }
       pdl_wait();
@@ -160,7 +171,7 @@ __global__ void __launch_bounds__(persist_threads<AMODE>(), 1)
         if (!mbar_wait_bounded(empty_bar(s), (r & 1) ^ 1, abort_flag, p.err)) break;
         int kx, m0, n0;
         coords(g, &kx, &m0, &n0);
-        mbar_arrive_expect_tx(full_bar(s), Cfg::kB + a_bytes);
+        mbar_arrive_expect_tx(full_bar(s), Cfg::kB + MS * a_bytes);
         tma_load_2d(smem_u32(sB + s * Cfg::kB), &tmB, full_bar(s), kx, n0);
         if (!GATHER) load_a(s, g);
       }
@@ -184,7 +195,7 @@ __global__ void __launch_bounds__(persist_threads<AMODE>(), 1)
         const int buf = lt & 1, use = lt >> 1;
         if (!mbar_wait_bounded(tempty0 + 8u * buf, (use & 1) ^ 1, abort_flag, p.err)) break;
         tc_fence_after();
-        const uint32_t d = tmem + (uint32_t)(buf * BN);
+        const uint32_t d = tmem + (uint32_t)(buf * MS * BN);
         for (int kb = 0; kb < KB; ++kb, ++g) {
           const int s = g % kStages, r = g / kStages;
           if (!mbar_wait_bounded(full_bar(s), r & 1, abort_flag, p.err)) {
@@ -192,10 +203,14 @@ __global__ void __launch_bounds__(persist_threads<AMODE>(), 1)
             break;
           }
           tc_fence_after();
-          const uint64_t ad = smem_desc_sw128(smem_u32(sA + s * kPA));
           const uint64_t bd = smem_desc_sw128(smem_u32(sB + s * Cfg::kB));
 #pragma unroll
-          for (int k = 0; k < kPBK / 16; ++k) tc_mma_f16(d, ad + 2ull * k, bd + 2ull * k, idesc, (kb | k) != 0);
+          for (int sub = 0; sub < MS; ++sub) {
+            const uint64_t ad = smem_desc_sw128(smem_u32(sA + s * Cfg::kSA + sub * kPA));
+#pragma unroll
+            for (int k = 0; k < kPBK / 16; ++k)
+              tc_mma_f16(d + (uint32_t)(sub * BN), ad + 2ull * k, bd + 2ull * k, idesc, (kb | k) != 0);
+          }
           tc_commit(empty_bar(s));
         }
         if (ok) tc_commit(tfull0 + 8u * buf);
@@ -213,20 +228,7 @@ __global__ void __launch_bounds__(persist_threads<AMODE>(), 1)
     for (int lt = 0; lt < my_tiles; ++lt) {
       const int buf = lt & 1, use = lt >> 1;
       const int tile = tile_of(lt);
-      const int n0 = (tile / mt) * BN;
-      int m = -1;  // output row of this thread's TMEM lane, -1 when unused
-      if (AMODE == kATap) {
-        const int sp = tile % mt;
-        const int img = sp / patches, rem = sp - img * patches;
-        const int th = rem / p.tiles_w, tw = rem - th * p.tiles_w;
-        if (row < p.wt * p.ht) {
-          const int oy = th * p.ht + row / p.wt, ox = tw * p.wt + row % p.wt;
-          if (oy < p.Ho && ox < p.Wo) m = (img * p.Ho + oy) * p.Wo + ox;
-        }
-      } else {
-        m = (tile % mt) * kPBM + row;
-        if (m >= p.M) m = -1;
-      }
+      const int n0 = (tile / mtp) * BN;
       // each warp stages its own copy of the tile's bias: no cross-warp barrier
       float* sb = sbias + (buf * 4 + q) * BN;
       const T* bias = static_cast<const T*>(p.e.bias);
@@ -237,15 +239,33 @@ __global__ void __launch_bounds__(persist_threads<AMODE>(), 1)
       tc_fence_after();
       const bool vec_ok = ((p.ldy | n0) % 8 == 0) && (!p.e.res || ((p.e.ldr | n0) % 8 == 0));
 #pragma unroll 1
-      for (int c0 = 0; c0 < BN; c0 += 32) {
-        uint32_t r[32];
-        tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN + c0), r);
-        tmem_ld_wait();
-        if (m >= 0 && n0 + c0 < p.N) {
-          float v[32];
+      for (int sub = 0; sub < MS; ++sub) {
+        const int idx = (tile % mtp) * MS + sub;  // m-tile (or pixel patch) of this sub-tile
+        int m = -1;  // output row of this thread's TMEM lane, -1 when unused
+        if (idx < mt) {
+          if (AMODE == kATap) {
+            const int img = idx / patches, rem = idx - img * patches;
+            const int th = rem / p.tiles_w, tw = rem - th * p.tiles_w;
+            if (row < p.wt * p.ht) {
+              const int oy = th * p.ht + row / p.wt, ox = tw * p.wt + row % p.wt;
+              if (oy < p.Ho && ox < p.Wo) m = (img * p.Ho + oy) * p.Wo + ox;
+            }
+          } else {
+            m = idx * kPBM + row;
+            if (m >= p.M) m = -1;
+          }
+        }
+#pragma unroll 1
+        for (int c0 = 0; c0 < BN; c0 += 32) {
+          uint32_t r[32];
+          tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)((buf * MS + sub) * BN + c0), r);
+          tmem_ld_wait();
+          if (m >= 0 && n0 + c0 < p.N) {
+            float v[32];
 #pragma unroll
-          for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-          finish32<T>(v, sb + c0, p, m, n0 + c0, vec_ok);
+            for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+            finish32<T>(v, sb + c0, p, m, n0 + c0, vec_ok);
+          }
         }
       }
       tc_fence_before();
@@ -264,7 +284,7 @@ __global__ void __launch_bounds__(persist_threads<AMODE>(), 1)
     bool ok = true;
     for (int lt = 0; lt < my_tiles && ok; ++lt) {
       const int tile = tile_of(lt);
-      const int m = (tile % mt) * kPBM + t;
+      const int m = (tile % mtp) * kPBM + t;  // MS == 1 here
       const bool mvalid = m < p.M;
       int img = 0, oy = 0, ox = 0;
       if (mvalid) {
@@ -328,16 +348,16 @@ __global__ void __launch_bounds__(persist_threads<AMODE>(), 1)
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, 2 * BN);
+    tmem_dealloc(tmem, 2 * MS * BN);
   }
 }
 
-template <typename T, int BN, int AMODE>
+template <typename T, int BN, int AMODE, int MS>
 int launch_persist_inst(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) {
   static bool attr_done = false;  // per instantiation
-  auto kern = tc_persist_kernel<T, BN, AMODE>;
+  auto kern = tc_persist_kernel<T, BN, AMODE, MS>;
   if (!attr_done) {
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, PCfg<BN>::kSmem) != cudaSuccess)
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, PCfg<BN, MS>::kSmem) != cudaSuccess)
       SN_FAIL(SWAPNET_ERR_CUDA, "cudaFuncSetAttribute failed");
     attr_done = true;
   }
@@ -351,13 +371,13 @@ int launch_persist_inst(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_
   a.wt = pl.wt; a.ht = pl.ht; a.tiles_w = pl.tiles_w; a.tiles_h = pl.tiles_h;
   const int64_t mt = AMODE == kATap ? (int64_t)g.M / ((int64_t)g.Ho * g.Wo) * pl.tiles_w * pl.tiles_h
                                     : (g.M + kPBM - 1) / kPBM;
-  const int64_t tiles = mt * ((g.N + BN - 1) / BN);
+  const int64_t tiles = (mt + MS - 1) / MS * ((g.N + BN - 1) / BN);
   const int sms = g.num_sms > 0 ? g.num_sms : 148;
   cudaLaunchConfig_t cfg;
   std::memset(&cfg, 0, sizeof(cfg));
   cfg.gridDim = dim3((unsigned)std::min<int64_t>(tiles, sms));
   cfg.blockDim = dim3(persist_threads<AMODE>());
-  cfg.dynamicSmemBytes = PCfg<BN>::kSmem;
+  cfg.dynamicSmemBytes = PCfg<BN, MS>::kSmem;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -371,9 +391,14 @@ int launch_persist_inst(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_
 
 template <typename T, int BN>
 int launch_persist_bn(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) {
-  if (!g.conv) return launch_persist_inst<T, BN, kAT2d>(g, pl, err, s);
-  if (pl.tma_conv) return launch_persist_inst<T, BN, kATap>(g, pl, err, s);
-  return launch_persist_inst<T, BN, kAGather>(g, pl, err, s);
+  if (BN == 64 && pl.msub == 2) {
+    if (!g.conv) return launch_persist_inst<T, BN, kAT2d, 2>(g, pl, err, s);
+    if (pl.tma_conv) return launch_persist_inst<T, BN, kATap, 2>(g, pl, err, s);
+    SN_FAIL(SWAPNET_ERR_INVALID_ARG, "persistent GEMM: two sub-tiles need A by TMA");
+  }
+  if (!g.conv) return launch_persist_inst<T, BN, kAT2d, 1>(g, pl, err, s);
+  if (pl.tma_conv) return launch_persist_inst<T, BN, kATap, 1>(g, pl, err, s);
+  return launch_persist_inst<T, BN, kAGather, 1>(g, pl, err, s);
 }
 
 template <typename T>

@@ -97,6 +97,7 @@ struct TcPlan {
   uint64_t scratch_bytes;  // fp32 partials of all splits
   int persist;      // persistent kernel (one CTA per SM looping over tiles)
   int tma_conv;     // convolution A by 4-D TMA per filter tap (tmA is then 4-D)
+  int msub;         // persistent: 128-row sub-tiles per tile (2 for N tiles of 64 with A by TMA)
   int wt, ht, tiles_w, tiles_h;  // its output patch and patch counts per image
   int ready;
 };
