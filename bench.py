@@ -187,7 +187,7 @@ def llm_host_weights(model, threads=16):
         for ti, (_, shp) in enumerate(synth.arch.tensor_shapes(L)):
             jobs.append((li, ti, shp))
             sizes.append(int(np.prod(shp)) * 2)
-    host = capi.HostWeights.allocate(sizes)
+    host = capi.HostWeights.allocate(sizes, pinned=True)
 
     def fill(k):
         li, ti, shp = jobs[k]

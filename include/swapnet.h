@@ -366,7 +366,7 @@ int swapnet_engine_stats_get(const swapnet_engine* eng, swapnet_engine_stats* st
 typedef enum swapnet_kernel_kind {
   SWAPNET_KERNEL_TC_GEMM = 1,     /* tcgen05 GEMM, A and B by TMA             */
   SWAPNET_KERNEL_TC_CONV = 2,     /* tcgen05 implicit-GEMM conv (A gathered)  */
-  SWAPNET_KERNEL_SKINNY = 3,      /* SIMT linear, <= 16 rows                  */
+  SWAPNET_KERNEL_SKINNY = 3,      /* SIMT GEMV family: fp32 <= 16 rows, fp16/bf16 <= 4 rows */
   SWAPNET_KERNEL_DIRECT_CONV = 4, /* SIMT direct convolution                  */
   SWAPNET_KERNEL_MAXPOOL = 5,
   SWAPNET_KERNEL_GAP = 6,
@@ -458,6 +458,17 @@ void swapnet_engine_free(swapnet_engine* eng);
 #define SWAPNET_NOALLOC_SCRATCH_BYTES (4u << 20)
 int swapnet_gemm_noalloc(int32_t dtype, const void* A, const void* W, const void* bias, void* Y, int32_t M,
                          int32_t N, int32_t K, int32_t act, swapnet_stream stream);
+
+/* --------------------------------------------------------- host weights */
+/* Page-locked, device-mapped host memory for weight storage (the pinned
+ * host copy that Sec. 4.2's swap-in reads): allocated by the CUDA driver in
+ * large physically contiguous pieces, so the copy engines and the zero-copy
+ * kernel stream it at full link rate however large it is; swapnet_load uses
+ * it in place (no registration).  Caller-owned: release with
+ * swapnet_host_free after every engine using it is freed.
+ * Errors: INVALID_ARG (null out or zero bytes), OOM. */
+int swapnet_host_alloc(uint64_t bytes, void** out);
+int swapnet_host_free(void* p);
 
 /* ------------------------------------------------------------------- misc */
 const char* swapnet_strerror(int status);

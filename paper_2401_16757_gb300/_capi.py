@@ -95,7 +95,7 @@ EXPORTS = ["swapnet_default_options", "swapnet_partition", "swapnet_plan_from_cu
            "swapnet_plan_info_get", "swapnet_plan_cuts", "swapnet_plan_units", "swapnet_plan_blocks",
            "swapnet_plan_output_offsets", "swapnet_plan_free", "swapnet_schedule", "swapnet_load",
            "swapnet_infer", "swapnet_infer_host", "swapnet_engine_sync", "swapnet_engine_blocks",
-           "swapnet_engine_free", "swapnet_engine_stats_get", "swapnet_engine_unit_kernels", "swapnet_engine_unit_tiling", "swapnet_engine_adapt",
+           "swapnet_engine_free", "swapnet_engine_stats_get", "swapnet_engine_unit_kernels", "swapnet_engine_unit_tiling", "swapnet_engine_adapt", "swapnet_host_alloc", "swapnet_host_free",
            "swapnet_engine_set_profiling", "swapnet_engine_last_times", "swapnet_engine_measure_units",
            "swapnet_engine_last_timeline",
            "swapnet_engine_bind_state", "swapnet_strerror", "swapnet_last_error", "swapnet_debug_fail_next", "swapnet_gemm_noalloc"]
@@ -139,6 +139,8 @@ def lib():
         "swapnet_infer_host": (C.c_int, [P, P, P, P]),
         "swapnet_engine_sync": (C.c_int, [P]),
         "swapnet_engine_adapt": (C.c_int, [P, P]),
+        "swapnet_host_alloc": (C.c_int, [C.c_uint64, C.POINTER(P)]),
+        "swapnet_host_free": (C.c_int, [P]),
         "swapnet_engine_bind_state": (C.c_int, [P, P, C.c_uint64]),
         "swapnet_engine_blocks": (C.c_int, [P, C.POINTER(EngineBlock), C.c_uint32, C.POINTER(C.c_uint32)]),
         "swapnet_engine_free": (None, [P]),
@@ -358,15 +360,24 @@ class HostWeights:
     range)."""
 
     @classmethod
-    def allocate(cls, nbytes_list):
+    def allocate(cls, nbytes_list, pinned=False):
         """An uninitialised packed buffer for tensors of the given sizes;
-        fill tensor i through view(i)."""
+        fill tensor i through view(i).  pinned: page-locked by the CUDA
+        driver (swapnet_host_alloc) instead of anonymous memory the library
+        page-locks at load (use it for buffers of many GB)."""
         self = cls.__new__(cls)
         offs, cur = [], 0
         for n in nbytes_list:
             offs.append(cur)
             cur += (n + 255) // 256 * 256
-        self._raw, self.buf = _host_buffer(cur)
+        if pinned:
+            p = C.c_void_p()
+            check(lib().swapnet_host_alloc(max(cur, 1), C.byref(p)), "swapnet_host_alloc")
+            self._pinned = p.value
+            self._raw = (C.c_uint8 * max(cur, 1)).from_address(p.value)
+            self.buf = np.frombuffer(self._raw, dtype=np.uint8)[:cur]
+        else:
+            self._raw, self.buf = _host_buffer(cur)
         self._offs, self._sizes = offs, list(nbytes_list)
         base = self.buf.ctypes.data
         self.ptrs = (C.c_void_p * max(1, len(offs)))(*[base + o for o in offs])
@@ -376,6 +387,16 @@ class HostWeights:
 
     def view(self, i):
         return self.buf[self._offs[i]:self._offs[i] + self._sizes[i]]
+
+    def __del__(self):
+        p = getattr(self, "_pinned", None)
+        if p:
+            self.buf = self._raw = None
+            self._pinned = None
+            try:
+                lib().swapnet_host_free(C.c_void_p(p))
+            except Exception:
+                pass
 
     def __init__(self, weights, buffer=None):
         """buffer: optional caller-provided uint8 array (e.g. already pinned)

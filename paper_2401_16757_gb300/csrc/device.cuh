@@ -100,7 +100,7 @@ __device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
 // error word; returns false then.
 __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort,
                                                   int* err) {
-  for (int it = 0; it < 4096; ++it)
+  for (int it = 0; it < 16; ++it)
     if (mbar_test_wait(bar, parity)) return true;
   uint64_t t0 = 0;
   for (uint32_t it = 0;; ++it) {

@@ -1192,6 +1192,23 @@ int swapnet_engine_last_timeline(swapnet_engine* e, float* us0, float* us1, uint
 
 void swapnet_engine_free(swapnet_engine* e) { release(e); }
 
+int swapnet_host_alloc(uint64_t bytes, void** out) {
+  if (!out || bytes == 0) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null out or zero bytes");
+  *out = nullptr;
+  if (injected(1) || cudaHostAlloc(out, bytes, cudaHostAllocPortable | cudaHostAllocMapped) != cudaSuccess) {
+    cudaGetLastError();
+    *out = nullptr;
+    SN_FAIL(SWAPNET_ERR_OOM, "page-locked host allocation failed");
+  }
+  return SWAPNET_OK;
+}
+
+int swapnet_host_free(void* p) {
+  if (!p) return SWAPNET_OK;
+  CU(cudaFreeHost(p), "cudaFreeHost");
+  return SWAPNET_OK;
+}
+
 int swapnet_debug_fail_next(int what, int count) {
   if (what < 1 || what > 3 || count < 0) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad fault-injection request");
   g_fail_next[what] = count;

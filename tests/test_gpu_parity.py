@@ -350,3 +350,19 @@ def test_engine_adapts_to_new_budgets_between_inferences():
     assert ei.value.code == capi.ERR_INVALID_ARG
     with pytest.raises(capi.SwapnetError):
         sw.engine.adapt(capi.Plan.resident(d))
+
+
+def test_driver_pinned_host_weights():
+    """Weights packed in swapnet_host_alloc memory are used in place."""
+    m = synth.arch.resnet50()
+    w = synth.gen.model_weights(m)
+    flat = [np.ascontiguousarray(t) for lw in w for t in lw]
+    host = capi.HostWeights.allocate([t.nbytes for t in flat], pinned=True)
+    for i, t in enumerate(flat):
+        host.view(i)[:] = t.view(np.uint8).reshape(-1)
+    x = synth.gen.model_input(m)
+    d = capi.Desc(m)
+    budget = int(OP.weight_bytes(m) * 0.4) // 256 * 256
+    a = Runner(m, w, capi.Plan.partition(d, budget, capi.options()), host).run(x)
+    b = Runner(m, w, capi.Plan.resident(d), capi.HostWeights(w)).run(x)
+    assert all(p.tobytes() == q.tobytes() for p, q in zip(a, b))
