@@ -559,10 +559,12 @@ int tc_prepare(const TcGemm& g, TcPlan* p) {
     const int64_t sp_tiles = tmac ? (int64_t)g.M / ((int64_t)g.Ho * g.Wo) * ((g.Wo + wt - 1) / wt) *
                                         ((g.Ho + ht - 1) / ht)
                                   : mtiles;
-    // widest useful N tile; convolutions narrow it until every SM has a tile
-    int pbn = Nd <= 64 ? 64 : (Nd <= 128 ? 128 : 256);
-    while (g.conv && pbn > 64 && sp_tiles * ((Nd + pbn - 1) / pbn) < sms) pbn /= 2;
-    if (sp_tiles * ((Nd + pbn - 1) / pbn) >= sms) {
+    // the widest useful N tile.  Measured on this kernel, a pipeline stage
+    // costs about the same (~0.5 us) whatever the tile width, so the time is
+    // about waves x k-blocks and wider tiles mean fewer waves; a third of the
+    // SMs busy with one wide tile each still beats splitting K across them
+    const int pbn = Nd <= 64 ? 64 : (Nd <= 128 ? 128 : 256);
+    if (sp_tiles * ((Nd + pbn - 1) / pbn) * 3 >= sms) {
       p->persist = 1;
       if (tmac) {
         p->tma_conv = 1;
