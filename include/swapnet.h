@@ -166,7 +166,13 @@ typedef struct swapnet_options {
                                      0, the longest prefix that leaves room for the
                                      rest, and the longest within 1/4, 1/2, 3/4 of its
                                      bytes.  Objective 0 only. */
-  int32_t reserved[3];
+  int32_t split_cap;             /* 0 (default): the kernels choose how many ways to
+                                     split K for layers with fewer output tiles than
+                                     SMs; n > 0: at most n (1 = never split).  A
+                                     tuning knob; results differ in the last bits
+                                     between split counts (each count is
+                                     deterministic). */
+  int32_t reserved[2];
 } swapnet_options;
 
 /* Fills the defaults: 2 slots, activations outside the budget, AUTO swap,

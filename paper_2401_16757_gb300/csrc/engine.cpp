@@ -409,7 +409,7 @@ static bool unit_gemm(const swapnet_engine* e, const Unit& U, const UnitExec& X,
   std::memset(g, 0, sizeof(*g));
   g->dtype = m.dtype;
   g->num_sms = e->num_sms;
-  g->cluster_max = 16;
+  g->cluster_max = e->plan.opt.split_cap > 0 ? std::min(16, (int)e->plan.opt.split_cap) : 16;
   g->allow_persist = 1;
   g->W = X.w;
   g->e.bias = X.b;

@@ -606,6 +606,14 @@ int tc_prepare(const TcGemm& g, TcPlan* p) {
   const int64_t tiles = (int64_t)((g.M + kBM - 1) / kBM) * ((g.N + p->bn - 1) / p->bn);
   const int KB = (g.K + kBK - 1) / kBK;
   int64_t splits = tiles_d >= sms ? 1 : std::min<int64_t>(sms / tiles_d, std::max(1, KB / 2));
+  if (g.cluster_max > 0) {
+    // cluster split-K, from a sweep of every split count on the batch-1 CNN
+    // layers: the cluster reduction costs more than it saves below nine
+    // k-blocks; clusters above 8 CTAs, or more than ~96 CTAs in clusters,
+    // wait longer to be scheduled than the split saves
+    if (KB <= 8) splits = 1;
+    else splits = std::min<int64_t>(splits, std::min<int64_t>(8, std::max<int64_t>(1, 96 / tiles_d)));
+  }
   const int cap = g.cluster_max > 0 ? std::min(g.cluster_max, max_cluster(g.dtype, p->bn, g.conv != 0)) : 32;
   splits = std::max<int64_t>(1, std::min<int64_t>(splits, cap));
   p->cluster = g.cluster_max > 0 ? 1 : 0;

@@ -718,6 +718,7 @@ static int check_options(const swapnet_options& o) {
   if (o.graphs != 0 && o.graphs != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "graphs must be 0 or 1");
   if (o.preloaded != 0 && o.preloaded != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "preloaded must be 0 or 1");
   if (o.branches != 0 && o.branches != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "branches must be 0 or 1");
+  if (o.split_cap < 0 || o.split_cap > 64) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "split_cap must be in [0, 64]");
   if (o.resident_prefix != 0 && o.resident_prefix != 1)
     SN_FAIL(SWAPNET_ERR_INVALID_ARG, "resident_prefix must be 0 or 1");
   if (o.resident_prefix && o.objective != 0)
