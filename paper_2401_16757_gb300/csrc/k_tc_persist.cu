@@ -165,15 +165,64 @@ __global__ void __launch_bounds__(persist_threads<AMODE>(), 1)
       pdl_wait();
       if (!GATHER)
         for (int g = 0; g < early; ++g) load_a(g, g);
+      // steady state: coordinates advance incrementally (divisions only when
+      // a new tile starts), so the single producer thread keeps ahead
       int g = early;
-      for (; g < work; ++g) {
-        const int s = g % kStages, r = g / kStages;
-        if (!mbar_wait_bounded(empty_bar(s), (r & 1) ^ 1, abort_flag, p.err)) break;
-        int kx, m0, n0;
-        coords(g, &kx, &m0, &n0);
-        mbar_arrive_expect_tx(full_bar(s), Cfg::kB + MS * a_bytes);
-        tma_load_2d(smem_u32(sB + s * Cfg::kB), &tmB, full_bar(s), kx, n0);
-        if (!GATHER) load_a(s, g);
+      if (g < work) {
+        int lt = g / KB, kb = g % KB;
+        int s = g % kStages, par = ((g / kStages) & 1) ^ 1;
+        int n0 = 0, ay[MS], az[MS], aw[MS];
+        int c0 = 0, rx = 0, ry = 0;
+        auto start_tile = [&]() {
+          const int tile = tile_of(lt);
+          n0 = (tile / mtp) * BN;
+#pragma unroll
+          for (int sub = 0; sub < MS; ++sub) {
+            const int idx = (tile % mtp) * MS + sub;
+            if (AMODE == kATap) {
+              const int img = idx / patches, rem = idx - img * patches;
+              const int th = rem / p.tiles_w, tw = rem - th * p.tiles_w;
+              ay[sub] = tw * p.wt * p.stride - p.pad;
+              az[sub] = th * p.ht * p.stride - p.pad;
+              aw[sub] = img;
+            } else {
+              ay[sub] = idx * kPBM;
+              az[sub] = aw[sub] = 0;
+            }
+          }
+        };
+        start_tile();
+        if (AMODE == kATap) {  // position of k-block kb inside the filter
+          const int k0 = kb * kPBK, tap = k0 / p.C;
+          c0 = k0 - tap * p.C;
+          ry = tap / p.kw;
+          rx = tap - ry * p.kw;
+        }
+        for (; g < work; ++g) {
+          if (!mbar_wait_bounded(empty_bar(s), par, abort_flag, p.err)) break;
+          mbar_arrive_expect_tx(full_bar(s), Cfg::kB + MS * a_bytes);
+          tma_load_2d(smem_u32(sB + s * Cfg::kB), &tmB, full_bar(s), kb * kPBK, n0);
+          if (!GATHER) {
+#pragma unroll
+            for (int sub = 0; sub < MS; ++sub) {
+              const uint32_t dst = smem_u32(sA + s * Cfg::kSA + sub * kPA);
+              if (AMODE == kAT2d) tma_load_2d(dst, &tmA, full_bar(s), kb * kPBK, ay[sub]);
+              else tma_load_4d(dst, &tmA, full_bar(s), c0, ay[sub] + rx, az[sub] + ry, aw[sub]);
+            }
+          }
+          if (++s == kStages) { s = 0; par ^= 1; }
+          if (++kb == KB) {
+            kb = 0;
+            c0 = rx = ry = 0;
+            if (++lt < my_tiles) start_tile();
+          } else if (AMODE == kATap) {
+            c0 += kPBK;
+            if (c0 == p.C) {
+              c0 = 0;
+              if (++rx == p.kw) { rx = 0; ++ry; }
+            }
+          }
+        }
       }
       if (g < work) {
         // aborted: let the loads already issued land before the CTA exits
