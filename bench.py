@@ -57,8 +57,8 @@ CONFIGS = {
 # + dram__bytes_write.sum averaged over the launches of one swapped step of
 # the named workload), valid only for the kernel sources it was taken on.
 TRAFFIC = {
-    ("resnet50", "tc_gemm"): ("311c8f454e1f", 1423859),
-    ("resnet50", "tc_conv"): ("311c8f454e1f", 1807458),
+    ("resnet50", "tc_gemm"): ("5691132c07c4", 1418749),
+    ("resnet50", "tc_conv"): ("5691132c07c4", 1804449),
 }
 
 
@@ -87,15 +87,19 @@ class ClockSampler:
               "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
               "clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, index):
+    def __init__(self, index, interval_ms=100):
+        # polling nvidia-smi itself disturbs the host link (measured: a
+        # link-bound 7B decode pass went from 63 to 67-100 ms under 50 ms
+        # polling), so poll no faster than needed to see the clocks
         self.index = index
+        self.interval_ms = interval_ms
         self.proc = None
         self.lines = []
 
     def start(self):
         try:
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.FIELDS,
-                                          "--format=csv,noheader,nounits", "-lms", "50"],
+                                          "--format=csv,noheader,nounits", "-lms", str(self.interval_ms)],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
@@ -298,7 +302,7 @@ def run_llm(args, rank, world):
     for e in (ep, ed, rp, rd):
         e.sync()
     link_before = measure_link_peak(stream)
-    clocks = ClockSampler(int(os.environ.get("LOCAL_RANK", "0")))
+    clocks = ClockSampler(int(os.environ.get("LOCAL_RANK", "0")), interval_ms=500)
     clocks.start()
     launches0 = ep.stats()["kernel_launches"] + ed.stats()["kernel_launches"]
     sw = timed(ep, ed, args.steps)
