@@ -8,7 +8,9 @@
 // either a row-major activation matrix (linear layers, 1x1 stride-1 convs),
 // also staged by TMA, or the implicit im2col of an NHWC input for general
 // convolutions, gathered by four warps with cp.async (zero fill for padding)
-// into the same swizzled layout.  One CTA computes one 128 x BN tile:
+// into the same swizzled layout.  One CTA computes one 128 x BN tile (BN 64
+// or 128; 256 for linear layers of at most kFewRows rows, whose work is
+// streaming the weight matrix):
 //   warp 0      TMA producer (one elected lane)
 //   warp 1      TMEM allocation and MMA issue (one elected lane)
 //   warps 2..5  im2col gather (conv) and the epilogue (TMEM -> registers ->
@@ -38,13 +40,20 @@ constexpr int kBK = 64;  // 64 x 2 bytes = one 128-byte swizzle row
 constexpr int kThreads = 192;
 constexpr int kABytes = kBM * kBK * 2;
 
+// N tile 256 serves GEMMs of at most kFewRows rows (one partly filled M
+// tile) that stream a large weight matrix: their cluster split-K partials
+// are distributed by column, so the receive buffer holds kFewRows rows.
+constexpr int kFewRows = 16;
+
 template <int BN> struct Cfg {
   static constexpr int kStages = BN == 64 ? 6 : 4;
   static constexpr int kLag = kStages - 2;  // gather: cp.async groups in flight per thread
   static constexpr int kBBytes = BN * kBK * 2;
   static constexpr int kStageBytes = kStages * (kABytes + kBBytes);
-  // cluster split-K receive buffer: up to 16 splits x ceil(128/splits) rows
-  static constexpr int kRecvBytes = (kBM + 15) * (BN + 4) * 4;
+  // cluster split-K receive buffer.  BN 64/128 (row owners): up to 16 splits
+  // x ceil(128/splits) rows.  BN 256 (column owners): splits x kFewRows rows
+  // x (columns per owner + 4), at most kFewRows x (256 + 8 x 8) floats.
+  static constexpr int kRecvBytes = BN == 256 ? kFewRows * (BN + 64) * 4 : (kBM + 15) * (BN + 4) * 4;
   static constexpr int kBiasBytes = BN * 4;
   static constexpr int kSmem = kStageBytes + kRecvBytes + kBiasBytes + 256 + 1024;
 };
@@ -245,6 +254,35 @@ __global__ void __launch_bounds__(kThreads, 1)
           finish32<T>(v, sbias + c0, p, m, n0 + c0, vec_ok);
         }
       }
+    } else if (csplit && BN == 256) {
+      // cluster split-K over columns (at most kFewRows rows): columns
+      // [o * cpo, (o + 1) * cpo) of the tile belong to CTA o of the cluster;
+      // this split's partial goes to slot blockIdx.z of each owner
+      const int cpo = (((BN + splits - 1) / splits) + 3) & ~3;
+      const int rs = cpo + 4;  // row stride of a slot, floats
+      const bool mine = ok && m < p.M && row < kFewRows;
+      asm volatile("barrier.cluster.wait;" ::: "memory");  // every peer is running
+#pragma unroll 1
+      for (int c0 = 0; c0 < BN; c0 += 32) {
+        uint32_t r[32];
+        tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)c0, r);
+        tmem_ld_wait();
+        if (mine) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int c = c0 + 4 * j;
+            const uint32_t owner = (uint32_t)(c / cpo);
+            const int cl = c - (int)owner * cpo;
+            const uint32_t la = smem_u32(recv) + (uint32_t)((((int)blockIdx.z * kFewRows + row) * rs + cl) * 4);
+            uint32_t ra;
+            asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(la), "r"(owner));
+            asm volatile("st.shared::cluster.v4.f32 [%0], {%1,%2,%3,%4};" ::"r"(ra), "f"(__uint_as_float(r[4 * j])),
+                         "f"(__uint_as_float(r[4 * j + 1])), "f"(__uint_as_float(r[4 * j + 2])),
+                         "f"(__uint_as_float(r[4 * j + 3]))
+                         : "memory");
+          }
+        }
+      }
     } else if (csplit) {
       // cluster split-K: push this split's rows to the CTA that owns them
       // (owner of row w = w / rows_per_owner), slot = this split's index
@@ -339,20 +377,41 @@ __global__ void __launch_bounds__(kThreads, 1)
     // all pushes are visible after this barrier; each CTA reduces the rows
     // it owns from its own receive buffer, in split order 0..S-1
     asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
-    const int rpo = (kBM + splits - 1) / splits;
-    const int r0 = (int)blockIdx.z * rpo;
-    const int rows = max(0, min(min(rpo, kBM - r0), p.M - m0 - r0));
-    const int groups = rows * (BN / 4);
-    for (int g = threadIdx.x; g < groups; g += kThreads) {
-      const int rr = g / (BN / 4), c4 = g % (BN / 4);
-      const int n = n0 + 4 * c4;
-      const float* src = recv + rr * (BN + 4) + 4 * c4;
-      float4 acc = *reinterpret_cast<const float4*>(src);
-      for (int z = 1; z < splits; ++z) {
-        const float4 v = *reinterpret_cast<const float4*>(src + z * rpo * (BN + 4));
-        acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+    if constexpr (BN == 256) {
+      // this CTA owns columns [c_lo, c_hi) of the tile, every row
+      const int cpo = (((BN + splits - 1) / splits) + 3) & ~3;
+      const int rs = cpo + 4;
+      const int c_lo = (int)blockIdx.z * cpo, c_hi = min(BN, c_lo + cpo);
+      const int rows = max(0, min(kFewRows, p.M - m0));
+      const int w4 = max(0, c_hi - c_lo) / 4;
+      const int groups = rows * w4;
+      for (int g = threadIdx.x; g < groups; g += kThreads) {
+        const int rr = g / w4, c4 = g % w4;
+        const int n = n0 + c_lo + 4 * c4;
+        const float* src = recv + rr * rs + 4 * c4;
+        float4 acc = *reinterpret_cast<const float4*>(src);
+        for (int z = 1; z < splits; ++z) {
+          const float4 v = *reinterpret_cast<const float4*>(src + z * kFewRows * rs);
+          acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+        }
+        if (n < p.N) finish4<T>(acc, sbias + c_lo + 4 * c4, p, m0 + rr, n);
       }
-      if (n < p.N) finish4<T>(acc, sbias + 4 * c4, p, m0 + r0 + rr, n);
+    } else {
+      const int rpo = (kBM + splits - 1) / splits;
+      const int r0 = (int)blockIdx.z * rpo;
+      const int rows = max(0, min(min(rpo, kBM - r0), p.M - m0 - r0));
+      const int groups = rows * (BN / 4);
+      for (int g = threadIdx.x; g < groups; g += kThreads) {
+        const int rr = g / (BN / 4), c4 = g % (BN / 4);
+        const int n = n0 + 4 * c4;
+        const float* src = recv + rr * (BN + 4) + 4 * c4;
+        float4 acc = *reinterpret_cast<const float4*>(src);
+        for (int z = 1; z < splits; ++z) {
+          const float4 v = *reinterpret_cast<const float4*>(src + z * rpo * (BN + 4));
+          acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+        }
+        if (n < p.N) finish4<T>(acc, sbias + 4 * c4, p, m0 + r0 + rr, n);
+      }
     }
   }
   tc_fence_before();
@@ -530,8 +589,43 @@ int max_cluster_inst() {
   return best;
 }
 
+// Clusters of c CTAs of the N-tile-256 instance that the device runs at
+// once (cudaOccupancyMaxActiveClusters; cached per dtype and size).
+template <typename T>
+int active_clusters_inst(int c) {
+  static int cached[9] = {-1, -1, -1, -1, -1, -1, -1, -1, -1};
+  if (c < 1 || c > 8) return 0;
+  if (cached[c] >= 0) return cached[c];
+  auto kern = tc_gemm_kernel<T, 256, false>;
+  cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<256>::kSmem);
+  cudaLaunchConfig_t cfg;
+  std::memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = dim3(1, 1, c);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = Cfg<256>::kSmem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 1;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = c;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    n = 0;
+  }
+  cached[c] = n;
+  return n;
+}
+
+int active_clusters(int dtype, int c) {
+  return dtype == SWAPNET_BF16 ? active_clusters_inst<__nv_bfloat16>(c) : active_clusters_inst<__half>(c);
+}
+
 int max_cluster(int dtype, int bn, bool gather) {
   const bool bf = dtype == SWAPNET_BF16;
+  if (bn == 256) return bf ? max_cluster_inst<__nv_bfloat16, 256, false>() : max_cluster_inst<__half, 256, false>();
   if (bn == 64)
     return gather ? (bf ? max_cluster_inst<__nv_bfloat16, 64, true>() : max_cluster_inst<__half, 64, true>())
                   : (bf ? max_cluster_inst<__nv_bfloat16, 64, false>() : max_cluster_inst<__half, 64, false>());
@@ -595,6 +689,41 @@ int tc_prepare(const TcGemm& g, TcPlan* p) {
       return SWAPNET_OK;
     }
   }
+  const int KB = (g.K + kBK - 1) / kBK;
+  if (g.cluster_max > 0 && !g.conv && g.M <= kFewRows && KB >= 16) {
+    // a few rows against a large weight matrix: streaming the weights is the
+    // work.  A 128xNx16 MMA costs about the same for N = 64 and 256, so the
+    // widest tile moves 4x the weight bytes per MMA; K is split across a
+    // cluster (column-owner reduction).  The split count minimises
+    // waves x k-blocks per CTA, a wave being the clusters of that size the
+    // device co-schedules: clusters of 7-8 CTAs of this kernel do not all
+    // fit at once, and the second wave costs more than the wider split saves
+    p->bn = 256;
+    const int64_t tiles_d = (Nd + 255) / 256;
+    const int smax = std::max(1, std::min(std::min(8, KB / 8), std::min(g.cluster_max, max_cluster(g.dtype, 256, false))));
+    int64_t splits = 1, best = -1;
+    for (int c = 1; c <= smax; ++c) {
+      const int64_t act = c == 1 ? sms : active_clusters(g.dtype, c);
+      if (act < 1) continue;
+      const int64_t cost = (tiles_d + act - 1) / act * ((KB + c - 1) / c);
+      if (best < 0 || cost < best) {
+        best = cost;
+        splits = c;
+      }
+    }
+    p->cluster = 1;
+    p->kb_per_split = (KB + (int)splits - 1) / (int)splits;
+    p->splits = (KB + p->kb_per_split - 1) / p->kb_per_split;
+    p->tiles = (g.N + 255) / 256;
+    int rc = make_tmap(&p->tmB, g.dtype, g.W, (uint64_t)g.K, (uint64_t)g.N, (uint64_t)g.K * 2, 256u);
+    if (rc) return rc;
+    if (g.A) {
+      rc = make_tmap(&p->tmA, g.dtype, g.A, (uint64_t)g.K, (uint64_t)g.M, (uint64_t)g.lda * 2, (uint32_t)kBM);
+      if (rc) return rc;
+    }
+    p->ready = 1;
+    return SWAPNET_OK;
+  }
   if (Nd <= 64) {
     p->bn = 64;
   } else {
@@ -604,7 +733,6 @@ int tc_prepare(const TcGemm& g, TcPlan* p) {
   // deterministic split-K: enough CTAs to cover the SMs, >= 2 k-blocks each
   const int64_t tiles_d = (int64_t)((g.M + kBM - 1) / kBM) * ((Nd + p->bn - 1) / p->bn);
   const int64_t tiles = (int64_t)((g.M + kBM - 1) / kBM) * ((g.N + p->bn - 1) / p->bn);
-  const int KB = (g.K + kBK - 1) / kBK;
   int64_t splits = tiles_d >= sms ? 1 : std::min<int64_t>(sms / tiles_d, std::max(1, KB / 2));
   if (g.cluster_max > 0) {
     // cluster split-K, from a sweep of every split count on the batch-1 CNN
@@ -640,6 +768,7 @@ int launch_tc_gemm(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) 
     return bf ? launch_inst<__nv_bfloat16, 128, true>(g, pl, err, s) : launch_inst<__half, 128, true>(g, pl, err, s);
   }
   if (pl.bn == 64) return bf ? launch_inst<__nv_bfloat16, 64, false>(g, pl, err, s) : launch_inst<__half, 64, false>(g, pl, err, s);
+  if (pl.bn == 256) return bf ? launch_inst<__nv_bfloat16, 256, false>(g, pl, err, s) : launch_inst<__half, 256, false>(g, pl, err, s);
   return bf ? launch_inst<__nv_bfloat16, 128, false>(g, pl, err, s) : launch_inst<__half, 128, false>(g, pl, err, s);
 }
 

@@ -83,7 +83,8 @@ def test_conv_residual_epilogue(res_post, act):
 
 @pytest.mark.parametrize("dtype", ["f16", "bf16", "f32"])
 @pytest.mark.parametrize("rows,k,n", [(1, 2048, 1000), (16, 4096, 640), (8, 1024, 1024), (200, 512, 384),
-                                      (300, 256, 64), (129, 1024, 136), (40, 512, 130)])
+                                      (300, 256, 64), (129, 1024, 136), (40, 512, 130),
+                                      (16, 25088, 1000), (12, 2048, 520), (5, 1024, 296)])
 def test_linear_layer(dtype, rows, k, n):
     layers = [dict(op="linear", src=[-1], k=k, n=n, act="relu", res=None, res_post=False),
               dict(op="linear", src=[0], k=n, n=n, act="none", res=0, res_post=False)]
