@@ -57,8 +57,8 @@ CONFIGS = {
 # + dram__bytes_write.sum averaged over the launches of one swapped step of
 # the named workload), valid only for the kernel sources it was taken on.
 TRAFFIC = {
-    ("resnet50", "tc_gemm"): ("5691132c07c4", 1418749),
-    ("resnet50", "tc_conv"): ("5691132c07c4", 1804449),
+    ("resnet50", "tc_gemm"): ("487ed6861217", 1418604),
+    ("resnet50", "tc_conv"): ("487ed6861217", 1804570),
 }
 
 
@@ -174,6 +174,43 @@ def build_workload(name, weight_bytes_fn):
 def capi_weight_bytes(m):
     from paper_2401_16757_gb300 import capi
     return capi.Plan.resident(capi.Desc(m)).info()["weight_bytes"]
+
+
+def unit_algorithmic_bytes(m, units):
+    """Bytes each unit must move at least once: its parameters, its inputs
+    (every source and the residual) and its output, for a linear piece the
+    share of the output it writes.  CNN and MLP layer types only."""
+    es = {"f32": 4, "f16": 2, "bf16": 2}[m["dtype"]]
+    shapes = []
+
+    def shp(i):
+        return tuple(m["input"]) if i == -1 else shapes[i]
+
+    for L in m["layers"]:
+        n, h, w, c = shp(L["src"][0])
+        op = L["op"]
+        if op in ("conv", "maxpool"):
+            ho = (h + 2 * L["pad"] - L["kh"]) // L["stride"] + 1
+            wo = (w + 2 * L["pad"] - L["kw"]) // L["stride"] + 1
+            shapes.append((n, ho, wo, L["cout"] if op == "conv" else c))
+        elif op == "linear":
+            shapes.append((n, 1, 1, L["n"]))
+        elif op == "gap":
+            shapes.append((n, 1, 1, c))
+        elif op == "upsample2x":
+            shapes.append((n, 2 * h, 2 * w, c))
+        elif op == "concat":
+            shapes.append((n, h, w, c + shp(L["src"][1])[3]))
+        else:
+            return None
+    out = []
+    for u in units:
+        L = m["layers"][u["layer"]]
+        frac = u["rows"] / L["n"] if L["op"] == "linear" and u["rows"] else 1.0
+        srcs = list(L["src"]) + ([L["res"]] if L.get("res") is not None else [])
+        b = u["bytes"] + sum(int(np.prod(shp(s))) * es for s in srcs) + int(np.prod(shapes[u["layer"]])) * es * frac
+        out.append(int(b))
+    return out
 
 
 def oracle_weight_bytes(m):
@@ -895,17 +932,31 @@ def main():
     dom_flops = sum(units[i]["flops"] for i in dom_idx)
     dom_us = sum(acc_u[i] for i in dom_idx)
     hbm, tf_burst, tf_sust, peak_src = load_peaks()
-    achieved_tf = dom_flops / (dom_us * 1e-6) / 1e12 if dom_us > 0 else 0.0
-    roofline = {"bound": "tensor", "kernel": dom, "launches_per_step": len(dom_idx),
-                "achieved": achieved_tf, "peak": tf_burst, "unit": "TFLOP/s",
-                "frac": achieved_tf / tf_burst, "peak_source": peak_src + " bf16 burst",
-                "traffic": None, "kernel_sources_sha": kernel_sources_sha(), "share_of_kernel_time": dom_us / max(1e-9, acc_u.sum()),
-                "kernel_time_share": {k: round(v / max(1e-9, acc_u.sum()), 4) for k, v in share.items()}}
+    # the binding roof of the dominant kernel family: tensor FLOPs when its
+    # algorithmic FLOPs per byte reach the ridge point (peak FLOP/s over
+    # peak bytes/s), HBM bytes otherwise
+    ubytes = unit_algorithmic_bytes(m, units)
+    dom_bytes = sum(ubytes[i] for i in dom_idx) if ubytes else 0
+    ridge = tf_burst * 1e12 / (hbm * 1e9)
+    tensor_bound = dom_flops > 0 and (not dom_bytes or dom_flops / dom_bytes >= ridge)
+    if tensor_bound:
+        achieved = dom_flops / (dom_us * 1e-6) / 1e12 if dom_us > 0 else 0.0
+        roofline = {"bound": "tensor", "achieved": achieved, "peak": tf_burst, "unit": "TFLOP/s",
+                    "peak_source": peak_src + " bf16 burst"}
+    else:
+        achieved = dom_bytes / (dom_us * 1e-6) / 1e9 if dom_us > 0 else 0.0
+        roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                    "peak_source": peak_src + " copy"}
+    roofline.update({"kernel": dom, "launches_per_step": len(dom_idx), "frac": achieved / roofline["peak"],
+                     "algorithmic_flops_per_step": dom_flops, "algorithmic_bytes_per_step": dom_bytes,
+                     "algorithmic_bytes_per_launch": dom_bytes // max(1, len(dom_idx)),
+                     "flops_per_byte": dom_flops / dom_bytes if dom_bytes else None, "ridge_flops_per_byte": ridge,
+                     "traffic": None, "kernel_sources_sha": kernel_sources_sha(),
+                     "share_of_kernel_time": dom_us / max(1e-9, acc_u.sum()),
+                     "kernel_time_share": {k: round(v / max(1e-9, acc_u.sum()), 4) for k, v in share.items()}})
     tr = TRAFFIC.get((args.config, dom))
     if tr and tr[0] == roofline["kernel_sources_sha"]:
         roofline["traffic"] = tr[1]
-    if dom in ("skinny_linear", "maxpool", "gap", "upsample2x", "concat"):
-        roofline.update(bound="hbm", unit="GB/s", peak=hbm, peak_source=peak_src + " copy")
 
     # ---- host link: bytes per swap over swap time, against pinned memcpy peak
     swap_bytes = sum(b["bytes"] for b in blocks)
