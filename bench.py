@@ -22,6 +22,7 @@ GPU with no collective on the data path.
 """
 import argparse
 import json
+import mmap
 import os
 import statistics
 import subprocess
@@ -653,6 +654,106 @@ def run_adapt_study(args):
                       "phases": phases}))
 
 
+def run_storage(args):
+    """Storage tier (Sec. 4.2.1 direct block fetch): the weights of --config
+    are written to a file in --storage and every inference reads its
+    swapped blocks from there with O_DIRECT (staging ring, read stream,
+    copy into the slot).  The delay model is calibrated on the file engine
+    (its per-block read + copy cost becomes alpha), the plan made from it,
+    and the swapped inference timed against DInf (resident, host memory).
+    Prints one JSON line."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2401_16757_gb300 import capi
+    name = args.config if args.config in ("resnet50", "vgg16_b1", "vgg16_b16", "yolov3", "mlp6") else "resnet50"
+    m, w, x, wb, budget, text = build_workload(name, capi_weight_bytes)
+    d = capi.Desc(m)
+    host = capi.HostWeights(w)
+    path = os.path.join(args.storage, "%s_%d.swnw" % (name, os.getpid()))
+    t0 = time.perf_counter()
+    capi.WeightsFile.write(path, d, host)
+    t_write = time.perf_counter() - t0
+    try:
+        wf = capi.WeightsFile(path, allow_buffered=True)
+        file_bytes = os.path.getsize(path)
+        # the file read alone, O_DIRECT into a page-aligned buffer (64 MiB reads)
+        buf = mmap.mmap(-1, 64 << 20)
+        fd = os.open(path, os.O_RDONLY | (os.O_DIRECT if wf.info()["direct"] else 0))
+        best = 1e30
+        for _ in range(3):
+            t0, off = time.perf_counter(), 0
+            while off < file_bytes:
+                k = os.preadv(fd, [buf], off)
+                if k <= 0:
+                    break
+                off += k
+            best = min(best, time.perf_counter() - t0)
+        os.close(fd)
+        read_gbs = file_bytes / best / 1e9
+        act_in = 1 if name == "mlp6" else 0
+        opt0 = capi.options(slots=2, activations_in_budget=act_in)
+        plan0 = capi.Plan.partition(d, budget, opt0)
+        eng0 = capi.Engine(plan0, wf)
+        t_ex, alpha = capi.calibrate(m, plan0, eng0)
+        eng0.free()
+        opt = capi.options(slots=2, activations_in_budget=act_in, alpha_as_per_byte=alpha or 4_750_000,
+                           beta_ns_per_tensor=0, eta_ns_per_tensor=0)
+        plan = capi.Plan.partition(capi.Desc(m, t_ex_ns=t_ex), budget, opt)
+        info = plan.info()
+        eng = capi.Engine(plan, wf)
+        reng = capi.Engine(capi.Plan.resident(d), host)
+        stream = torch.cuda.current_stream()
+        flush = torch.empty(512 << 20, dtype=torch.uint8, device="cuda")
+        d_in = torch.empty(max(16, info["input_bytes"]), dtype=torch.uint8, device="cuda")
+        d_in[:info["input_bytes"]].copy_(torch.from_numpy(x.view(np.uint8).reshape(-1)))
+        d_out = torch.empty(info["output_bytes"], dtype=torch.uint8, device="cuda")
+        r_out = torch.empty_like(d_out)
+
+        def timed(e, out, steps):
+            for _ in range(args.warmup):
+                e.infer(d_in.data_ptr(), out.data_ptr(), stream.cuda_stream)
+            ts = []
+            for _ in range(steps):
+                flush.zero_()
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                e.infer(d_in.data_ptr(), out.data_ptr(), stream.cuda_stream)
+                b.record(stream)
+                b.synchronize()
+                ts.append(a.elapsed_time(b))
+            e.sync()
+            return ts
+
+        ts = timed(eng, d_out, args.steps)
+        tr = timed(reng, r_out, min(args.steps, 50))
+        exact = bool(torch.equal(d_out, r_out))
+        ms = sum(ts) / len(ts)
+        swapped = sum(b["bytes"] for b in plan.blocks())
+        hbm, tf_burst, _, peak_src = load_peaks()
+        flops = sum(u["flops"] for u in plan.units())
+        bound_ms = max(flops / (tf_burst * 1e12), swapped / (read_gbs * 1e9)) * 1e3
+        print(json.dumps({
+            "metric": "inferences_per_second", "value": 1000.0 / ms, "unit": "inferences/s", "n_gpus": 1,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "p50_ms": statistics.median(ts), "dinf_ms": sum(tr) / len(tr), "bit_exact_vs_resident": exact,
+            "predicted_ms": info["predicted_ns"] / 1e6, "n_blocks": info["n_blocks"],
+            "config": {"workload": text + "; swapped blocks read from a weights file for every inference",
+                       "storage_dir": args.storage, "l2": "512 MiB flush before every step"},
+            "storage": {"file_bytes": file_bytes, "direct_io": wf.info()["direct"], "write_s": t_write,
+                        "read_gbs_file_alone": read_gbs, "swapped_bytes_per_step": swapped,
+                        "alpha_as_per_byte": alpha,
+                        "block_read_copy_us": [round(b["memcpy_us"], 1) for b in eng.blocks()]},
+            "step_bound": {"ms": bound_ms, "what": "max(FLOPs / bf16 peak, swapped bytes / file read GB/s)",
+                           "frac": bound_ms / ms},
+        }))
+        eng.free()
+        reng.free()
+        wf.close()
+    finally:
+        os.unlink(path)
+
+
 def run_profile_once(args):
     """One resident inference of a single-model config (no timing)."""
     import torch
@@ -758,6 +859,9 @@ def main():
                          "layers, zero-copy swap, DInf); prints one JSON line")
     ap.add_argument("--adapt-study", action="store_true",
                     help="dynamic-budget case study: one engine switched between plans for 80/60/40 % budgets")
+    ap.add_argument("--storage", default=None, metavar="DIR",
+                    help="storage tier: write --config's weights to a file in DIR and read every swapped block "
+                         "from it with O_DIRECT; prints one JSON line")
     ap.add_argument("--profile-once", action="store_true",
                     help="run one resident inference of --config through the C ABI and exit "
                          "(a driver for profiler captures of its kernels); prints one JSON line")
@@ -778,6 +882,9 @@ def main():
         return
     if args.adapt_study:
         run_adapt_study(args)
+        return
+    if args.storage:
+        run_storage(args)
         return
     if args.config in ("llm", "multi"):
         import torch

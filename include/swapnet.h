@@ -42,7 +42,8 @@ typedef enum swapnet_status {
   SWAPNET_ERR_CUDA = -4,        /* a CUDA runtime/driver call failed       */
   SWAPNET_ERR_TIMEOUT = -5,     /* a bounded device-side wait gave up      */
   SWAPNET_ERR_MISALIGNED = -6,  /* a pointer or size breaks an alignment rule */
-  SWAPNET_ERR_UNSUPPORTED = -7  /* shape/dtype combination not implemented */
+  SWAPNET_ERR_UNSUPPORTED = -7, /* shape/dtype combination not implemented */
+  SWAPNET_ERR_IO = -8           /* a weights-file read or write failed      */
 } swapnet_status;
 
 /* ------------------------------------------------------------ descriptors */
@@ -298,6 +299,60 @@ int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint
                  void* d_arena, uint64_t arena_bytes, void* d_workspace, uint64_t workspace_bytes,
                  swapnet_engine** out_engine);
 
+/* ----------------------------------------------------------- storage tier
+ * Sec. 4.2.1 "Direct Block Fetch": the blocks live in external storage and
+ * are fetched with direct I/O (O_DIRECT, bypassing the page cache, so no
+ * second copy of a block sits in host memory) into a dedicated swap-in
+ * channel.  Here the channel is two page-locked staging buffers per engine:
+ * block k is read from the file into staging buffer k mod 2 by a host
+ * function on the engine's read stream, then copied by the copy engine into
+ * its arena slot, so the read of block k+1 overlaps the copy of block k and
+ * the execution of block k-1.
+ *
+ * Weights file layout (little-endian), written by swapnet_weights_file_write:
+ *   bytes 0..7     magic "SWNWGT01"
+ *   uint32         version = 1
+ *   uint32         n_tensors
+ *   uint64         data_offset (first tensor; a multiple of 4096)
+ *   n_tensors x {uint64 offset, uint64 bytes}: tensor t in layer order, as
+ *                  in swapnet_load's host_weights; offset a multiple of 4096
+ *   zero padding; the file length is a multiple of 4096.
+ */
+typedef struct swapnet_weights_file swapnet_weights_file;
+
+enum { SWAPNET_FILE_ALLOW_BUFFERED = 1 }; /* open flag: no O_DIRECT -> page cache */
+
+/* Write every parameter tensor of `desc` (n_tensors host pointers in layer
+ * order, tensor sizes from the descriptor) to `path` in the layout above,
+ * then fsync.  Errors: INVALID_ARG, IO (errno text in swapnet_last_error). */
+int swapnet_weights_file_write(const char* path, const swapnet_model_desc* desc, const void* const* host_weights,
+                               uint32_t n_tensors);
+
+/* Open and validate a weights file for reading with O_DIRECT.  Where the
+ * file system refuses O_DIRECT, fails with IO unless flags has
+ * SWAPNET_FILE_ALLOW_BUFFERED (then reads go through the page cache and
+ * swapnet_weights_file_info reports direct = 0).  Errors: INVALID_ARG (bad
+ * header), IO, OOM. */
+int swapnet_weights_file_open(const char* path, uint32_t flags, swapnet_weights_file** out);
+int swapnet_weights_file_info(const swapnet_weights_file* f, uint32_t* n_tensors, int32_t* direct);
+/* Host read of bytes [offset, offset + bytes) of tensor t into dst through
+ * the file's read path (an aligned bounce buffer).  Errors: INVALID_ARG
+ * (range outside the tensor), IO. */
+int swapnet_weights_file_read(swapnet_weights_file* f, uint32_t tensor, uint64_t offset, uint64_t bytes, void* dst);
+/* The file must outlive every engine loaded from it. */
+void swapnet_weights_file_close(swapnet_weights_file* f);
+
+/* As swapnet_load, with the parameters in a weights file instead of host
+ * memory: swapped blocks are fetched from the file for every inference
+ * (staging, read stream and host functions as above); a resident plan or a
+ * resident prefix is read once here.  Swap variant: copy engine (AUTO and
+ * ZEROCOPY are taken as MEMCPY).  Models with host-resident parameters
+ * (EMBED) are not supported.  A failed read inside an inference is reported
+ * by the next swapnet_engine_sync as IO.  Errors: as swapnet_load, plus IO,
+ * UNSUPPORTED. */
+int swapnet_load_file(const swapnet_plan* plan, swapnet_weights_file* file, void* d_arena, uint64_t arena_bytes,
+                      void* d_workspace, uint64_t workspace_bytes, swapnet_engine** out_engine);
+
 /* One inference, asynchronous on `stream` (Sec. 4.3, Sec. 6.2.2 with m
  * slots): block k is swapped into slot k mod m on the engine's copy stream
  * once the slot's previous block has finished executing, and its layers run
@@ -316,7 +371,7 @@ int swapnet_infer_host(swapnet_engine* eng, const void* h_input, void* h_output,
 
 /* Waits for the engine's streams; returns TIMEOUT if a kernel's bounded
  * wait gave up since the last call (the error word is then cleared), CUDA
- * on a device error. */
+ * on a device error, IO if a weights-file read failed (then cleared). */
 int swapnet_engine_sync(swapnet_engine* eng);
 
 /* Runtime budget adaptation (Sec. 6.2.2 "adaptively partition and exchange

@@ -14,8 +14,8 @@ import numpy as np
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libswapnet.so")
 
-OK, ERR_INVALID_ARG, ERR_INFEASIBLE, ERR_OOM, ERR_CUDA, ERR_TIMEOUT, ERR_MISALIGNED, ERR_UNSUPPORTED = \
-    0, -1, -2, -3, -4, -5, -6, -7
+OK, ERR_INVALID_ARG, ERR_INFEASIBLE, ERR_OOM, ERR_CUDA, ERR_TIMEOUT, ERR_MISALIGNED, ERR_UNSUPPORTED, ERR_IO = \
+    0, -1, -2, -3, -4, -5, -6, -7, -8
 F32, F16, BF16 = 0, 1, 2
 I32 = 3
 OP = {"linear": 1, "conv": 2, "maxpool": 3, "gap": 4, "upsample2x": 5, "concat": 6, "embed": 7, "rmsnorm": 8,
@@ -99,7 +99,9 @@ EXPORTS = ["swapnet_default_options", "swapnet_partition", "swapnet_plan_from_cu
            "swapnet_engine_free", "swapnet_engine_stats_get", "swapnet_engine_unit_kernels", "swapnet_engine_unit_tiling", "swapnet_engine_adapt", "swapnet_host_alloc", "swapnet_host_free",
            "swapnet_engine_set_profiling", "swapnet_engine_last_times", "swapnet_engine_measure_units",
            "swapnet_engine_last_timeline",
-           "swapnet_engine_bind_state", "swapnet_strerror", "swapnet_last_error", "swapnet_debug_fail_next", "swapnet_gemm_noalloc"]
+           "swapnet_engine_bind_state", "swapnet_strerror", "swapnet_last_error", "swapnet_debug_fail_next", "swapnet_gemm_noalloc",
+           "swapnet_weights_file_write", "swapnet_weights_file_open", "swapnet_weights_file_info",
+           "swapnet_weights_file_read", "swapnet_weights_file_close", "swapnet_load_file"]
 
 _lib = None
 
@@ -158,6 +160,12 @@ def lib():
         "swapnet_last_error": (C.c_char_p, []),
         "swapnet_debug_fail_next": (C.c_int, [C.c_int, C.c_int]),
         "swapnet_gemm_noalloc": (C.c_int, [C.c_int32, P, P, P, P, C.c_int32, C.c_int32, C.c_int32, C.c_int32, P]),
+        "swapnet_weights_file_write": (C.c_int, [C.c_char_p, C.POINTER(ModelDesc), C.POINTER(P), C.c_uint32]),
+        "swapnet_weights_file_open": (C.c_int, [C.c_char_p, C.c_uint32, C.POINTER(P)]),
+        "swapnet_weights_file_info": (C.c_int, [P, C.POINTER(C.c_uint32), C.POINTER(C.c_int32)]),
+        "swapnet_weights_file_read": (C.c_int, [P, C.c_uint32, C.c_uint64, C.c_uint64, P]),
+        "swapnet_weights_file_close": (None, [P]),
+        "swapnet_load_file": (C.c_int, [P, P, P, C.c_uint64, P, C.c_uint64, C.POINTER(P)]),
     }
     for name, (res, args) in sig.items():
         f = getattr(L, name)
@@ -422,12 +430,60 @@ class HostWeights:
         self.nbytes = cur
 
 
+class WeightsFile:
+    """A weights file of the storage tier (Sec. 4.2.1), opened for direct
+    I/O; the layout is documented in swapnet.h."""
+
+    ALLOW_BUFFERED = 1
+
+    @staticmethod
+    def write(path, desc, host):
+        """Write the tensors of `host` (HostWeights) for model `desc`."""
+        check(lib().swapnet_weights_file_write(os.fsencode(path), C.byref(desc.c), host.ptrs, host.n),
+              "swapnet_weights_file_write")
+
+    def __init__(self, path, allow_buffered=False):
+        h = C.c_void_p()
+        check(lib().swapnet_weights_file_open(os.fsencode(path), self.ALLOW_BUFFERED if allow_buffered else 0,
+                                              C.byref(h)), "swapnet_weights_file_open")
+        self.h = h
+        self.path = path
+
+    def info(self):
+        n, d = C.c_uint32(), C.c_int32()
+        check(lib().swapnet_weights_file_info(self.h, C.byref(n), C.byref(d)), "swapnet_weights_file_info")
+        return {"n_tensors": n.value, "direct": bool(d.value)}
+
+    def read(self, tensor, offset, nbytes):
+        out = np.empty(nbytes, dtype=np.uint8)
+        check(lib().swapnet_weights_file_read(self.h, tensor, offset, nbytes, C.c_void_p(out.ctypes.data)),
+              "swapnet_weights_file_read")
+        return out
+
+    def close(self):
+        if self.h and self.h.value:
+            lib().swapnet_weights_file_close(self.h)
+            self.h = C.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
 class Engine:
     def __init__(self, plan, host, d_arena=0, arena_bytes=0, d_ws=0, ws_bytes=0):
-        self.host = host  # keep the host buffer alive
+        """host: HostWeights (parameters in host memory) or WeightsFile
+        (parameters read from storage for every swap-in)."""
+        self.host = host  # keep the host buffer (or the open file) alive
         h = C.c_void_p()
-        check(lib().swapnet_load(plan.h, host.ptrs, host.n, C.c_void_p(d_arena or None), arena_bytes,
-                                 C.c_void_p(d_ws or None), ws_bytes, C.byref(h)), "swapnet_load")
+        if isinstance(host, WeightsFile):
+            check(lib().swapnet_load_file(plan.h, host.h, C.c_void_p(d_arena or None), arena_bytes,
+                                          C.c_void_p(d_ws or None), ws_bytes, C.byref(h)), "swapnet_load_file")
+        else:
+            check(lib().swapnet_load(plan.h, host.ptrs, host.n, C.c_void_p(d_arena or None), arena_bytes,
+                                     C.c_void_p(d_ws or None), ws_bytes, C.byref(h)), "swapnet_load")
         self.h = h
 
     def bind_state(self, d_state, nbytes):

@@ -1,10 +1,12 @@
-// Engine: binds a plan to host weights and device memory, and runs the
-// block pipeline (Sec. 4 swapping, Sec. 5 assembly by reference, Sec. 6.2.2
-// with m = slots blocks co-resident).
+// Engine: binds a plan to host weights (or a weights file, Sec. 4.2.1) and
+// device memory, and runs the block pipeline (Sec. 4 swapping, Sec. 5
+// assembly by reference, Sec. 6.2.2 with m = slots blocks co-resident).
 #include <cuda_runtime.h>
 #include <unistd.h>
 
 #include <algorithm>
+#include <atomic>
+#include <chrono>
 #include <cstring>
 #include <map>
 #include <memory>
@@ -124,6 +126,20 @@ struct swapnet_engine {
   char* d_splitk = nullptr;          // split-K scratch: tile counters, then fp32 partials
   uint64_t splitk_bytes = 0;
   uint64_t splitk_counter_bytes = 0;
+  // storage tier: blocks fetched from a weights file into staging buffer
+  // k mod 2 by a host function on `rd`, then copied into their slot
+  swapnet_weights_file* file = nullptr;
+  char* stage[2] = {nullptr, nullptr};  // page-locked, kFileAlign aligned
+  uint64_t stage_bytes = 0;
+  cudaStream_t rd = nullptr;
+  cudaEvent_t staged[2] = {nullptr, nullptr}, stage_free[2] = {nullptr, nullptr};
+  std::vector<std::vector<FileRun>> fruns;  // per block
+  struct ReadJob {
+    swapnet_engine* e;
+    int k;
+  };
+  std::vector<ReadJob> jobs;  // host-function arguments, one per block
+  std::atomic<int> io_errno{0};
 };
 
 namespace swapnet {
@@ -146,6 +162,14 @@ static int release(swapnet_engine* e) {
   for (cudaEvent_t ev : e->ev_unit) cudaEventDestroy(ev);
   for (cudaEvent_t ev : e->ev_swap) cudaEventDestroy(ev);
   if (e->copy) cudaStreamDestroy(e->copy);
+  if (e->rd) {
+    cudaStreamSynchronize(e->rd);
+    cudaStreamDestroy(e->rd);
+  }
+  for (cudaEvent_t ev : {e->staged[0], e->staged[1], e->stage_free[0], e->stage_free[1]})
+    if (ev) cudaEventDestroy(ev);
+  for (char* p : e->stage)
+    if (p) cudaFreeHost(p);
   if (e->own_arena && e->d_arena) cudaFree(e->d_arena);
   if (e->own_ws && e->d_ws) cudaFree(e->d_ws);
   if (e->d_splitk) cudaFree(e->d_splitk);
@@ -235,7 +259,166 @@ static int register_host(swapnet_engine* e, const void* const* hw, uint32_t nt) 
 
 static char* block_base(swapnet_engine* e, const Block& B) { return e->d_arena + B.base; }
 
-static void build_segments(swapnet_engine* e) {
+// Storage tier: each block's parameter pieces become aligned file runs
+// (pieces closer than kRunGap share a run), packed one after another in the
+// block's staging buffer, and copy segments from staging to the slot.
+// Grows the two staging buffers to the largest block.
+static int build_file_blocks(swapnet_engine* e) {
+  constexpr uint64_t kRunGap = 256 * 1024;
+  const swapnet_plan& p = e->plan;
+  const swapnet_weights_file* f = e->file;
+  e->blocks.assign(p.blocks.size(), EngBlock{});
+  e->fruns.assign(p.blocks.size(), {});
+  struct Piece {
+    uint64_t file_off, len, slot_off;
+  };
+  std::vector<std::vector<Piece>> pieces(p.blocks.size());
+  uint64_t need = kFileAlign;
+  for (size_t k = 0; k < p.blocks.size(); ++k) {
+    const Block& B = p.blocks[k];
+    std::vector<Piece>& pc = pieces[k];
+    for (int u = B.u0; u < B.u1; ++u) {
+      const Unit& U = p.units[u];
+      if (U.host) SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "host-resident parameters cannot be read from a weights file");
+      for (int t = 0; t < U.nt; ++t) {
+        if (U.tlen[t] == 0) continue;
+        const int ti = U.tidx[t];
+        if (U.toff[t] + U.tlen[t] > f->bytes[ti]) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "weights file tensor too short");
+        pc.push_back(Piece{f->off[ti] + U.toff[t], U.tlen[t], U.slot_off[t]});
+      }
+    }
+    std::sort(pc.begin(), pc.end(), [](const Piece& a, const Piece& b) { return a.file_off < b.file_off; });
+    std::vector<FileRun>& runs = e->fruns[k];
+    uint64_t staged = 0;
+    for (const Piece& q : pc) {
+      const uint64_t lo = q.file_off / kFileAlign * kFileAlign, hi = align_up(q.file_off + q.len, kFileAlign);
+      if (!runs.empty() && lo <= runs.back().file_off + runs.back().len + kRunGap) {
+        FileRun& r = runs.back();
+        const uint64_t end = std::max(r.file_off + r.len, hi);
+        staged += end - (r.file_off + r.len);
+        r.len = end - r.file_off;
+      } else {
+        runs.push_back(FileRun{lo, hi - lo, staged});
+        staged += hi - lo;
+      }
+    }
+    need = std::max(need, staged);
+  }
+  if (need > e->stage_bytes) {
+    for (char*& b : e->stage) {
+      if (b) cudaFreeHost(b);
+      b = nullptr;
+    }
+    e->stage_bytes = 0;
+    for (char*& b : e->stage) {
+      void* q = nullptr;
+      if (injected(1) || cudaHostAlloc(&q, need, cudaHostAllocPortable) != cudaSuccess) {
+        cudaGetLastError();
+        SN_FAIL(SWAPNET_ERR_OOM, "page-locked staging allocation failed");
+      }
+      b = static_cast<char*>(q);
+    }
+    e->stage_bytes = need;
+  }
+  for (size_t k = 0; k < p.blocks.size(); ++k) {
+    const std::vector<FileRun>& runs = e->fruns[k];
+    char* stage = e->stage[k % 2];
+    char* base = block_base(e, p.blocks[k]);
+    std::vector<Segment>& segs = e->blocks[k].segs;
+    size_t r = 0;
+    for (const Piece& q : pieces[k]) {
+      while (q.file_off >= runs[r].file_off + runs[r].len) ++r;  // pieces and runs are both sorted
+      Segment g{stage + runs[r].stage_off + (q.file_off - runs[r].file_off), base + q.slot_off, q.len};
+      if (!segs.empty()) {
+        Segment& b = segs.back();
+        if (g.src == b.src + b.bytes && g.dst == b.dst + b.bytes) {
+          b.bytes += g.bytes;
+          continue;
+        }
+      }
+      segs.push_back(g);
+    }
+  }
+  e->jobs.assign(p.blocks.size(), swapnet_engine::ReadJob{e, 0});
+  for (size_t k = 0; k < p.blocks.size(); ++k) e->jobs[k].k = (int)k;
+  return SWAPNET_OK;
+}
+
+// Host function on the read stream: fetch block k's runs into its staging
+// buffer.  Calls no CUDA API; a failure is kept for swapnet_engine_sync.
+static void CUDART_CB read_block_host(void* arg) {
+  const swapnet_engine::ReadJob* j = static_cast<const swapnet_engine::ReadJob*>(arg);
+  swapnet_engine* e = j->e;
+  const std::vector<FileRun>& runs = e->fruns[j->k];
+  const int err = file_read_runs(e->file, runs.data(), runs.size(), e->stage[j->k % 2]);
+  if (err) {
+    int none = 0;
+    e->io_errno.compare_exchange_strong(none, err);
+  }
+}
+
+// Synchronous fetch of block k (load-time uploads and calibration).
+static int fetch_block_sync(swapnet_engine* e, size_t k, float* read_us) {
+  const auto t0 = std::chrono::steady_clock::now();
+  const int err = file_read_runs(e->file, e->fruns[k].data(), e->fruns[k].size(), e->stage[k % 2]);
+  if (read_us)
+    *read_us = std::chrono::duration<float, std::micro>(std::chrono::steady_clock::now() - t0).count();
+  if (err) SN_FAIL(SWAPNET_ERR_IO, std::string("weights file read: ") + std::strerror(err));
+  return SWAPNET_OK;
+}
+
+static int swap_block(swapnet_engine* e, size_t k, int variant, cudaStream_t s);
+
+static int upload_file_block(swapnet_engine* e, size_t k, float* us) {
+  float read_us = 0.f;
+  int rc = fetch_block_sync(e, k, &read_us);
+  if (rc) return rc;
+  cudaEvent_t a = nullptr, b = nullptr;
+  if (us) {
+    CU(cudaEventCreate(&a), "event");
+    CU(cudaEventCreate(&b), "event");
+    cudaEventRecord(a, e->copy);
+  }
+  rc = swap_block(e, k, SWAPNET_SWAP_MEMCPY, e->copy);
+  if (us) cudaEventRecord(b, e->copy);
+  const cudaError_t se = cudaStreamSynchronize(e->copy);
+  if (us) {
+    float ms = 0.f;
+    cudaEventElapsedTime(&ms, a, b);
+    *us = read_us + ms * 1000.f;
+    cudaEventDestroy(a);
+    cudaEventDestroy(b);
+  }
+  if (rc) return rc;
+  if (se != cudaSuccess) {
+    cudaGetLastError();
+    SN_FAIL(SWAPNET_ERR_CUDA, "staging to arena copy failed");
+  }
+  return SWAPNET_OK;
+}
+
+// Per-block swap cost of a file engine, read plus copy, each block alone
+// (best of 3): the measured counterpart of t_in for the planner.
+static int calibrate_file(swapnet_engine* e) {
+  for (size_t k = 0; k < e->blocks.size(); ++k) {
+    EngBlock& B = e->blocks[k];
+    B.variant = SWAPNET_SWAP_MEMCPY;
+    B.zerocopy_us = 0.f;
+    if (e->plan.blocks[k].slot < 0) continue;
+    float best = 1e30f;
+    for (int rep = 0; rep < 3; ++rep) {
+      float us = 0.f;
+      int rc = upload_file_block(e, k, &us);
+      if (rc) return rc;
+      best = std::min(best, us);
+    }
+    B.memcpy_us = best;
+  }
+  return SWAPNET_OK;
+}
+
+static int build_segments(swapnet_engine* e) {
+  if (e->file) return build_file_blocks(e);
   const swapnet_plan& p = e->plan;
   e->blocks.assign(p.blocks.size(), EngBlock{});
   for (size_t k = 0; k < p.blocks.size(); ++k) {
@@ -261,6 +444,7 @@ static void build_segments(swapnet_engine* e) {
       }
     }
   }
+  return SWAPNET_OK;
 }
 
 static int swap_block(swapnet_engine* e, size_t k, int variant, cudaStream_t s) {
@@ -630,8 +814,9 @@ static int bind_plan(swapnet_engine* e, void* d_arena_user, uint64_t arena_bytes
     // the driver backing fresh allocations
     CU(cudaMemset(e->d_arena, 0, bytes), "arena first touch");
   }
-  build_segments(e);
-  int rc = prepare_units(e);
+  int rc = build_segments(e);
+  if (rc) return rc;
+  rc = prepare_units(e);
   if (rc) return rc;
   rc = plan_side(e);
   if (rc) return rc;
@@ -657,16 +842,21 @@ static int bind_plan(swapnet_engine* e, void* d_arena_user, uint64_t arena_bytes
   const int variant = plan->opt.swap_variant;
   if (plan->resident) {
     if (!preloaded_arena) {
-      for (size_t k = 0; k < e->blocks.size() && !rc; ++k) rc = swap_block(e, k, SWAPNET_SWAP_MEMCPY, e->copy);
+      for (size_t k = 0; k < e->blocks.size() && !rc; ++k)
+        rc = e->file ? upload_file_block(e, k, nullptr) : swap_block(e, k, SWAPNET_SWAP_MEMCPY, e->copy);
       if (rc) return rc;
       CU(cudaStreamSynchronize(e->copy), "resident upload");
     }
     e->weights_loaded = true;
   } else if (plan->prefix_units > 0 && !plan->blocks.empty() && plan->blocks[0].slot < 0) {
     // resident prefix: uploaded once, then only the other blocks are swapped
-    rc = swap_block(e, 0, SWAPNET_SWAP_MEMCPY, e->copy);
+    rc = e->file ? upload_file_block(e, 0, nullptr) : swap_block(e, 0, SWAPNET_SWAP_MEMCPY, e->copy);
     if (rc) return rc;
     CU(cudaStreamSynchronize(e->copy), "prefix upload");
+  }
+  if (e->file) {
+    if (!plan->resident) return calibrate_file(e);
+    return SWAPNET_OK;
   }
   if (!plan->resident && variant == SWAPNET_SWAP_AUTO) {
     rc = calibrate(e);
@@ -702,15 +892,14 @@ static void unbind_plan(swapnet_engine* e) {
   e->weights_loaded = false;
 }
 
-}  // namespace swapnet
-
-extern "C" {
-
-int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint32_t n_tensors, void* d_arena,
-                 uint64_t arena_bytes, void* d_workspace, uint64_t workspace_bytes, swapnet_engine** out) {
-  if (!plan || !out || (n_tensors && !host_weights)) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+// swapnet_load and swapnet_load_file: parameters from host memory
+// (host_weights) or from a weights file (file).
+static int load_engine(const swapnet_plan* plan, const void* const* host_weights, uint32_t n_tensors,
+                       swapnet_weights_file* file, void* d_arena, uint64_t arena_bytes, void* d_workspace,
+                       uint64_t workspace_bytes, swapnet_engine** out) {
   if ((int)n_tensors != plan->model.n_tensors)
-    SN_FAIL(SWAPNET_ERR_INVALID_ARG, "expected " + std::to_string(plan->model.n_tensors) + " host tensors");
+    SN_FAIL(SWAPNET_ERR_INVALID_ARG, "expected " + std::to_string(plan->model.n_tensors) + " tensors, got " +
+                                         std::to_string(n_tensors));
   if (((uintptr_t)d_arena | (uintptr_t)d_workspace) % kAlign)
     SN_FAIL(SWAPNET_ERR_MISALIGNED, "device buffers must be 256-byte aligned");
   if (d_workspace && workspace_bytes < plan->model.ws_bytes)
@@ -750,13 +939,40 @@ int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint
   CU(cudaStreamCreateWithFlags(&e->cap, cudaStreamNonBlocking), "capture stream");
   CU(cudaEventCreateWithFlags(&e->fork, cudaEventDisableTiming), "event");
   CU(cudaEventCreateWithFlags(&e->join, cudaEventDisableTiming), "event");
-  rc = register_host(e, host_weights, n_tensors);
-  if (rc) return rc;
+  if (file) {
+    e->file = file;
+    CU(cudaStreamCreateWithPriority(&e->rd, cudaStreamNonBlocking, hi), "read stream");
+    for (int s = 0; s < 2; ++s) {
+      CU(cudaEventCreateWithFlags(&e->staged[s], cudaEventDisableTiming), "event");
+      CU(cudaEventCreateWithFlags(&e->stage_free[s], cudaEventDisableTiming), "event");
+    }
+  } else {
+    rc = register_host(e, host_weights, n_tensors);
+    if (rc) return rc;
+  }
   rc = bind_plan(e, d_arena, arena_bytes, plan->resident && plan->opt.preloaded && d_arena);
   if (rc) return rc;
   e->stats = swapnet_engine_stats{};
   *out = guard.release();
   return SWAPNET_OK;
+}
+
+}  // namespace swapnet
+
+extern "C" {
+
+int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint32_t n_tensors, void* d_arena,
+                 uint64_t arena_bytes, void* d_workspace, uint64_t workspace_bytes, swapnet_engine** out) {
+  if (!plan || !out || (n_tensors && !host_weights)) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+  return swapnet::load_engine(plan, host_weights, n_tensors, nullptr, d_arena, arena_bytes, d_workspace,
+                              workspace_bytes, out);
+}
+
+int swapnet_load_file(const swapnet_plan* plan, swapnet_weights_file* file, void* d_arena, uint64_t arena_bytes,
+                      void* d_workspace, uint64_t workspace_bytes, swapnet_engine** out) {
+  if (!plan || !file || !out) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+  return swapnet::load_engine(plan, nullptr, file->n, file, d_arena, arena_bytes, d_workspace, workspace_bytes,
+                              out);
 }
 
 int swapnet_engine_adapt(swapnet_engine* e, const swapnet_plan* plan) {
@@ -865,19 +1081,38 @@ static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t 
   const swapnet_plan& p = e->plan;
   const bool prof = e->profiling && !capturing;
   bool used[2] = {false, false};
+  bool stage_used[2] = {false, false};
   if (!p.resident) {
     CU(cudaEventRecord(e->fork, s), "record fork");
     CU(cudaStreamWaitEvent(e->copy, e->fork, 0), "wait fork");
+    if (e->file) CU(cudaStreamWaitEvent(e->rd, e->fork, 0), "wait fork");
   }
   for (size_t k = 0; k < p.blocks.size(); ++k) {
     const Block& B = p.blocks[k];
     const bool swapped = !p.resident && B.slot >= 0;  // a resident prefix stays in the arena
     if (swapped) {
+      const int j = (int)(k % 2);  // staging buffer of a file engine
+      if (e->file) {
+        // fetch into staging j once the copies of its previous block are done;
+        // this overlaps the copy of the block before and the layers running
+        if (stage_used[j]) CU(cudaStreamWaitEvent(e->rd, e->stage_free[j], 0), "wait staging");
+        if (prof) CU(cudaEventRecord(e->ev_swap[2 * k], e->rd), "profile event");
+        CU(cudaLaunchHostFunc(e->rd, read_block_host, &e->jobs[k]), "read host function");
+        CU(cudaEventRecord(e->staged[j], e->rd), "record staged");
+      }
       if (used[B.slot]) CU(cudaStreamWaitEvent(e->copy, e->slot_free[B.slot], 0), "wait slot");
       used[B.slot] = true;
-      if (prof) CU(cudaEventRecord(e->ev_swap[2 * k], e->copy), "profile event");
+      if (e->file) {
+        CU(cudaStreamWaitEvent(e->copy, e->staged[j], 0), "wait staged");
+      } else if (prof) {
+        CU(cudaEventRecord(e->ev_swap[2 * k], e->copy), "profile event");
+      }
       int rc = swap_block(e, k, e->blocks[k].variant, e->copy);
       if (rc) return rc;
+      if (e->file) {
+        CU(cudaEventRecord(e->stage_free[j], e->copy), "record staging free");
+        stage_used[j] = true;
+      }
       if (prof) CU(cudaEventRecord(e->ev_swap[2 * k + 1], e->copy), "profile event");
       CU(cudaEventRecord(e->ready[B.slot], e->copy), "record ready");
       CU(cudaStreamWaitEvent(s, e->ready[B.slot], 0), "wait ready");
@@ -908,6 +1143,10 @@ static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t 
     if (rc) return rc;
   }
   if (!p.resident) {
+    if (e->file) {  // the read stream's last fetch is waited for by the copy stream
+      CU(cudaEventRecord(e->staged[0], e->rd), "record read join");
+      CU(cudaStreamWaitEvent(e->copy, e->staged[0], 0), "wait read join");
+    }
     CU(cudaEventRecord(e->join, e->copy), "record join");
     CU(cudaStreamWaitEvent(s, e->join, 0), "wait join");
   }
@@ -1002,8 +1241,11 @@ int swapnet_infer_host(swapnet_engine* e, const void* hin, void* hout, swapnet_s
 int swapnet_engine_sync(swapnet_engine* e) {
   if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
   CU(cudaSetDevice(e->device), "cudaSetDevice");
+  if (e->rd) CU(cudaStreamSynchronize(e->rd), "read stream");
   CU(cudaStreamSynchronize(e->copy), "copy stream");
   CU(cudaDeviceSynchronize(), "device synchronize");
+  if (const int io = e->io_errno.exchange(0))
+    SN_FAIL(SWAPNET_ERR_IO, std::string("weights file read during an inference: ") + std::strerror(io));
   int w = 0;
   CU(cudaMemcpy(&w, e->err_word, sizeof(int), cudaMemcpyDeviceToHost), "error word");
   if (w) {

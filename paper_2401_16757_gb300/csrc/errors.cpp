@@ -20,6 +20,7 @@ const char* swapnet_strerror(int status) {
     case SWAPNET_ERR_TIMEOUT: return "device-side wait timed out";
     case SWAPNET_ERR_MISALIGNED: return "misaligned pointer or size";
     case SWAPNET_ERR_UNSUPPORTED: return "unsupported shape or dtype";
+    case SWAPNET_ERR_IO: return "weights file I/O error";
     default: return "unknown status";
   }
 }

@@ -100,7 +100,26 @@ struct swapnet_plan {
   uint64_t prefix_bytes = 0;  // kept at arena offset 0; the swap region follows
 };
 
+// An open weights file (storage tier): descriptor, O_DIRECT or not, and the
+// validated offset and length of every tensor.
+struct swapnet_weights_file {
+  int fd = -1;
+  bool direct = false;
+  uint32_t n = 0;
+  uint64_t file_bytes = 0;
+  std::vector<uint64_t> off, bytes;
+};
+
 namespace swapnet {
+constexpr uint64_t kFileAlign = 4096;  // O_DIRECT offset / length / buffer alignment
+// One aligned read of a block's swap-in: file bytes [file_off, file_off +
+// len) into staging + stage_off.
+struct FileRun {
+  uint64_t file_off, len, stage_off;
+};
+// Reads every run; 0, or the errno of the first failure (EIO at end of file).
+int file_read_runs(const swapnet_weights_file* f, const FileRun* runs, size_t n, char* stage);
+
 int analyse_model(const swapnet_model_desc* desc, Model* m);
 int make_units(const Model& m, const swapnet_options& opt, uint64_t slot, uint64_t region, std::vector<Unit>* out);
 void finalize_blocks(swapnet_plan* p, const std::vector<uint32_t>& cuts);
