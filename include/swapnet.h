@@ -173,7 +173,23 @@ typedef struct swapnet_options {
                                      tuning knob; results differ in the last bits
                                      between split counts (each count is
                                      deterministic). */
-  int32_t reserved[2];
+  int32_t prefetch;              /* 0 (default): every inference is self-contained and
+                                     starts by swapping in its first block.  1: steady-
+                                     state back-to-back inferences (Sec. 4.3 pipeline
+                                     carried across inferences): each inference ends by
+                                     swapping the next inference's first block into its
+                                     place, overlapped with its own last layers, and the
+                                     next one starts with it present (the engine swaps it
+                                     in once at load).  The planner minimises that cyclic
+                                     schedule: first block ready at t = 0; its next copy
+                                     starts once the copy engine is free and the last
+                                     block sharing its place (the last even-indexed
+                                     block) has executed; with an even number of blocks
+                                     the last block and the first must fit the region
+                                     together.  Objective 0, two slots, no resident
+                                     prefix.  Consecutive inferences of one engine must
+                                     be issued on one stream (as for any engine). */
+  int32_t reserved[1];
 } swapnet_options;
 
 /* Fills the defaults: 2 slots, activations outside the budget, AUTO swap,

@@ -28,6 +28,17 @@ arena alone.  The objective is either
 Ties: smaller objective, then fewer blocks, then the lexicographically
 smallest cut vector.  A cut c means "a block boundary before unit c".
 
+Steady state with first-block prefetch (option prefetch, two slots; the
+Sec. 4.3 pipeline carried across back-to-back inferences): block 1 of the
+next inference (index 0 here) is copied at the end of the current one, so
+C_0 = 0 and E_0 = t_ex_0; that copy starts when the copy engine is done
+with block n-1 and the last block in block 0's place is released -- the
+blocks alternate between the two ends of the region, so that is block n-1
+when n is odd and block n-2 when n is even -- and the inference ends at
+    max(E_{n-1}, max(C_{n-1}, R_g) + t_in_0).
+With n even, block n-1 and the next block 0 are co-resident, so Eq. 3 also
+holds for that pair: s_{n-1} + s_0 <= arena.
+
 The search here enumerates all 2^(U-1) cut vectors, so it is only for small U.
 
 Model bookkeeping (sizes, FLOPs, output shapes, the activation workspace and
@@ -268,6 +279,36 @@ def pipeline_time(blocks, slots, prefix=False):
     return E
 
 
+def cyclic_time(blocks):
+    """Steady-state time of one inference with first-block prefetch (two
+    slots), blocks = [(bytes, t_in, t_ex, t_out), ...]."""
+    n = len(blocks)
+    C = [0] * n
+    E = [0] * n
+    R = [0] * n
+    for k, (_, t_in, t_ex, t_out) in enumerate(blocks):
+        if k == 0:
+            C[0] = 0                      # copied during the previous inference
+            E[0] = t_ex
+        else:
+            gate = R[k - 2] if k >= 2 else 0
+            C[k] = max(C[k - 1], gate) + t_in
+            E[k] = max(E[k - 1], C[k]) + t_ex
+        R[k] = E[k] + t_out
+    g = n - 1 if n % 2 == 1 else n - 2    # last block at the same end as block 0
+    next_copy_done = max(C[n - 1], R[g]) + blocks[0][1]
+    return max(E[n - 1], next_copy_done)
+
+
+def feasible_cyclic(blocks, region):
+    """Eq. 3 for two slots, plus the pair (block n-1, next block 0) when n is
+    even (they sit at opposite ends of the region at the same time)."""
+    if not feasible(blocks, region, 2):
+        return False
+    n = len(blocks)
+    return n % 2 == 1 or blocks[-1][0] + blocks[0][0] <= region
+
+
 def prefix_candidates(us, region, slots):
     """Resident-prefix lengths tried: 0; the longest prefix r whose bytes
     plus the smallest region the remaining units need (each unit, and with
@@ -327,7 +368,7 @@ def feasible(blocks, region, slots):
 
 
 def exhaustive_partition(model, budget, coef, slots=2, activations_in_budget=False,
-                         objective=0, t_ex_override=None, resident_prefix=False):
+                         objective=0, t_ex_override=None, resident_prefix=False, prefetch=False):
     """Best cut vector by brute force over all 2^(U-1) candidates.
 
     With resident_prefix (objective 0 only) the first r units may stay in the
@@ -335,6 +376,9 @@ def exhaustive_partition(model, budget, coef, slots=2, activations_in_budget=Fal
     cut vector of the remaining units is tried in the region left beside the
     prefix.  Ties: smaller objective, then shorter prefix, then fewer blocks,
     then the lexicographically smallest cut vector.
+
+    With prefetch (objective 0, two slots, no prefix) the objective is
+    cyclic_time() under feasible_cyclic().
 
     Returns dict(n, cuts, predicted_ns, slot, arena, workspace, units,
     prefix_units, prefix_bytes) or None when no partition is feasible."""
@@ -361,9 +405,13 @@ def exhaustive_partition(model, budget, coef, slots=2, activations_in_budget=Fal
             cuts = ((r,) if 0 < r < U else ()) + inner
             blocks = block_costs(us, cuts, coef)
             swapped = blocks[1:] if r else blocks
-            if not feasible(swapped, reg, slots):
+            if prefetch:
+                if not feasible_cyclic(blocks, reg):
+                    continue
+                obj = cyclic_time(blocks)
+            elif not feasible(swapped, reg, slots):
                 continue
-            if objective == 0:
+            elif objective == 0:
                 obj = pipeline_time(blocks, slots, prefix=r > 0)
             else:
                 obj = eq4_objective(blocks)

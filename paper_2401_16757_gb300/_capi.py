@@ -47,8 +47,8 @@ class Options(C.Structure):
                 ("objective", C.c_int32), ("alpha_as_per_byte", C.c_uint64), ("beta_ns_per_tensor", C.c_uint64),
                 ("gamma_as_per_flop", C.c_uint64), ("eta_ns_per_tensor", C.c_uint64), ("zc_ctas", C.c_int32),
                 ("graphs", C.c_int32), ("preloaded", C.c_int32), ("branches", C.c_int32),
-                ("resident_prefix", C.c_int32), ("split_cap", C.c_int32),
-                ("reserved", C.c_int32 * 2)]
+                ("resident_prefix", C.c_int32), ("split_cap", C.c_int32), ("prefetch", C.c_int32),
+                ("reserved", C.c_int32 * 1)]
 
 
 class PlanInfo(C.Structure):

@@ -788,6 +788,8 @@ static int run_unit(swapnet_engine* e, int u, const void* din, void* dout, cudaS
 // engine owns it), copy segments, unit pointers and TMA descriptors, side
 // branches, split-K scratch, the resident upload or prefix upload, and the
 // swap variants.  Used by swapnet_load and again by swapnet_engine_adapt.
+static bool prefetch_on(const swapnet_engine* e);
+
 static int bind_plan(swapnet_engine* e, void* d_arena_user, uint64_t arena_bytes_user, bool preloaded_arena) {
   const swapnet_plan* plan = &e->plan;
   const uint64_t arena_need = plan->prefix_bytes + plan->region;  // resident prefix, then the swap region
@@ -855,7 +857,11 @@ static int bind_plan(swapnet_engine* e, void* d_arena_user, uint64_t arena_bytes
     CU(cudaStreamSynchronize(e->copy), "prefix upload");
   }
   if (e->file) {
-    if (!plan->resident) return calibrate_file(e);
+    if (!plan->resident) {
+      rc = calibrate_file(e);
+      if (rc) return rc;
+      if (prefetch_on(e)) return upload_file_block(e, 0, nullptr);  // present for the first inference
+    }
     return SWAPNET_OK;
   }
   if (!plan->resident && variant == SWAPNET_SWAP_AUTO) {
@@ -870,6 +876,11 @@ static int bind_plan(swapnet_engine* e, void* d_arena_user, uint64_t arena_bytes
       if (plan->blocks[k].slot >= 0 && variant == SWAPNET_SWAP_ZEROCOPY && !zerocopy_ok(b))
         SN_FAIL(SWAPNET_ERR_MISALIGNED, "zero-copy needs 16-byte aligned host tensors");
     }
+  }
+  if (prefetch_on(e)) {  // the first block is present for the first inference
+    rc = swap_block(e, 0, e->blocks[0].variant, e->copy);
+    if (rc) return rc;
+    CU(cudaStreamSynchronize(e->copy), "first block upload");
   }
   return SWAPNET_OK;
 }
@@ -1077,9 +1088,16 @@ static int plan_side(swapnet_engine* e) {
   return SWAPNET_OK;
 }
 
+// First-block prefetch is on for swapped plans made with option prefetch
+// (the planner allows it only with two slots and no resident prefix).
+static bool prefetch_on(const swapnet_engine* e) {
+  return !e->plan.resident && e->plan.opt.prefetch && !e->plan.blocks.empty() && e->plan.blocks[0].slot == 0;
+}
+
 static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t s, bool capturing = false) {
   const swapnet_plan& p = e->plan;
   const bool prof = e->profiling && !capturing;
+  const bool pf = prefetch_on(e);
   bool used[2] = {false, false};
   bool stage_used[2] = {false, false};
   if (!p.resident) {
@@ -1087,35 +1105,49 @@ static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t 
     CU(cudaStreamWaitEvent(e->copy, e->fork, 0), "wait fork");
     if (e->file) CU(cudaStreamWaitEvent(e->rd, e->fork, 0), "wait fork");
   }
+  // swap block k in once its place is free (the last block released in its
+  // slot); gate_compute: the layers on `s` wait for it
+  auto swap_in = [&](size_t k, bool gate_compute) -> int {
+    const Block& B = p.blocks[k];
+    const int j = (int)(k % 2);  // staging buffer of a file engine
+    if (e->file) {
+      // fetch into staging j once the copies of its previous block are done;
+      // this overlaps the copy of the block before and the layers running
+      if (stage_used[j]) CU(cudaStreamWaitEvent(e->rd, e->stage_free[j], 0), "wait staging");
+      if (prof) CU(cudaEventRecord(e->ev_swap[2 * k], e->rd), "profile event");
+      CU(cudaLaunchHostFunc(e->rd, read_block_host, &e->jobs[k]), "read host function");
+      CU(cudaEventRecord(e->staged[j], e->rd), "record staged");
+    }
+    if (used[B.slot]) CU(cudaStreamWaitEvent(e->copy, e->slot_free[B.slot], 0), "wait slot");
+    used[B.slot] = true;
+    if (e->file) {
+      CU(cudaStreamWaitEvent(e->copy, e->staged[j], 0), "wait staged");
+    } else if (prof) {
+      CU(cudaEventRecord(e->ev_swap[2 * k], e->copy), "profile event");
+    }
+    int rc = swap_block(e, k, e->blocks[k].variant, e->copy);
+    if (rc) return rc;
+    if (e->file) {
+      CU(cudaEventRecord(e->stage_free[j], e->copy), "record staging free");
+      stage_used[j] = true;
+    }
+    if (prof) CU(cudaEventRecord(e->ev_swap[2 * k + 1], e->copy), "profile event");
+    if (gate_compute) {
+      CU(cudaEventRecord(e->ready[B.slot], e->copy), "record ready");
+      CU(cudaStreamWaitEvent(s, e->ready[B.slot], 0), "wait ready");
+    }
+    return SWAPNET_OK;
+  };
   for (size_t k = 0; k < p.blocks.size(); ++k) {
     const Block& B = p.blocks[k];
     const bool swapped = !p.resident && B.slot >= 0;  // a resident prefix stays in the arena
     if (swapped) {
-      const int j = (int)(k % 2);  // staging buffer of a file engine
-      if (e->file) {
-        // fetch into staging j once the copies of its previous block are done;
-        // this overlaps the copy of the block before and the layers running
-        if (stage_used[j]) CU(cudaStreamWaitEvent(e->rd, e->stage_free[j], 0), "wait staging");
-        if (prof) CU(cudaEventRecord(e->ev_swap[2 * k], e->rd), "profile event");
-        CU(cudaLaunchHostFunc(e->rd, read_block_host, &e->jobs[k]), "read host function");
-        CU(cudaEventRecord(e->staged[j], e->rd), "record staged");
+      if (pf && k == 0) {
+        used[B.slot] = true;  // swapped in at the end of the previous inference (or at load)
+      } else {
+        int rc = swap_in(k, true);
+        if (rc) return rc;
       }
-      if (used[B.slot]) CU(cudaStreamWaitEvent(e->copy, e->slot_free[B.slot], 0), "wait slot");
-      used[B.slot] = true;
-      if (e->file) {
-        CU(cudaStreamWaitEvent(e->copy, e->staged[j], 0), "wait staged");
-      } else if (prof) {
-        CU(cudaEventRecord(e->ev_swap[2 * k], e->copy), "profile event");
-      }
-      int rc = swap_block(e, k, e->blocks[k].variant, e->copy);
-      if (rc) return rc;
-      if (e->file) {
-        CU(cudaEventRecord(e->stage_free[j], e->copy), "record staging free");
-        stage_used[j] = true;
-      }
-      if (prof) CU(cudaEventRecord(e->ev_swap[2 * k + 1], e->copy), "profile event");
-      CU(cudaEventRecord(e->ready[B.slot], e->copy), "record ready");
-      CU(cudaStreamWaitEvent(s, e->ready[B.slot], 0), "wait ready");
     }
     for (int u = B.u0; u < B.u1; ++u) {
       if (e->is_side[u]) continue;  // launched on the side stream after its producer
@@ -1140,6 +1172,13 @@ static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t 
     if (!e->d_state) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "decoder state not bound (swapnet_engine_bind_state)");
     const Model& m = p.model;
     int rc = launch_advance(reinterpret_cast<int*>(e->d_state), m.in_n * m.in_h * m.in_w * m.in_c, s);
+    if (rc) return rc;
+  }
+  if (pf) {
+    // the next inference's first block, into its place once the last block
+    // placed there has executed; overlaps this inference's last layers (the
+    // plan keeps the last block clear of it)
+    int rc = swap_in(0, false);
     if (rc) return rc;
   }
   if (!p.resident) {
@@ -1400,7 +1439,9 @@ int swapnet_engine_last_timeline(swapnet_engine* e, float* us0, float* us1, uint
   if (e->ev_unit.empty()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "profiling was never enabled");
   CU(cudaSetDevice(e->device), "cudaSetDevice");
   CU(cudaDeviceSynchronize(), "device synchronize");
-  size_t k0 = 0;  // first swapped block (a resident prefix has no swap events)
+  // first block swapped at the start (a resident prefix has no swap events;
+  // with first-block prefetch block 0's swap comes at the end)
+  size_t k0 = swapnet::prefetch_on(e) ? 1 : 0;
   while (k0 < e->plan.blocks.size() && e->plan.blocks[k0].slot < 0) ++k0;
   const bool sw = !e->plan.resident && !e->ev_swap.empty() && k0 < e->plan.blocks.size();
   cudaEvent_t origin = sw ? e->ev_swap[2 * k0] : e->ev_unit[0];

@@ -124,6 +124,7 @@ int analyse_model(const swapnet_model_desc* desc, Model* m);
 int make_units(const Model& m, const swapnet_options& opt, uint64_t slot, uint64_t region, std::vector<Unit>* out);
 void finalize_blocks(swapnet_plan* p, const std::vector<uint32_t>& cuts);
 int64_t pipeline_ns(const std::vector<Block>& b, int slots, bool prefix = false);
+int64_t cyclic_ns(const std::vector<Block>& b);
 int64_t eq4_ns(const std::vector<Block>& b);
 uint64_t resident_latency_ns(const Model& m, const swapnet_options& opt);
 }  // namespace swapnet

@@ -325,6 +325,28 @@ int64_t pipeline_ns(const std::vector<Block>& b, int slots, bool prefix) {
   return E;
 }
 
+// Steady state of back-to-back inferences with first-block prefetch (two
+// slots): block 0 was copied during the previous inference, so C_0 = 0;
+// the copy of the next inference's block 0 follows the copy of block n-1
+// (one copy engine) once the last block placed with it (the last even
+// block) is released; the inference ends when that copy and the last
+// execution have both finished.
+int64_t cyclic_ns(const std::vector<Block>& b) {
+  if (b.empty()) return 0;
+  const size_t n = b.size();
+  std::vector<int64_t> R(n);
+  int64_t C = 0, E = b[0].t_ex;
+  R[0] = E + b[0].t_out;
+  for (size_t k = 1; k < n; ++k) {
+    const int64_t gate = k >= 2 ? R[k - 2] : 0;
+    C = std::max(C, gate) + b[k].t_in;
+    E = std::max(E, C) + b[k].t_ex;
+    R[k] = E + b[k].t_out;
+  }
+  const size_t g = (n % 2 == 1) ? n - 1 : n - 2;
+  return std::max(E, std::max(C, R[g]) + b[0].t_in);
+}
+
 int64_t eq4_ns(const std::vector<Block>& b) {
   const size_t n = b.size();
   int64_t total = 0, ov_prev = 0;
@@ -381,7 +403,9 @@ void finalize_blocks(swapnet_plan* p, const std::vector<uint32_t>& cuts) {
     for (const Unit& u : p->units) t += u.t_ex;
     p->predicted = t;
   } else {
-    p->predicted = p->opt.objective == 0 ? pipeline_ns(p->blocks, p->opt.slots, prefix) : eq4_ns(p->blocks);
+    p->predicted = p->opt.objective != 0 ? eq4_ns(p->blocks)
+                   : p->opt.prefetch    ? cyclic_ns(p->blocks)
+                                        : pipeline_ns(p->blocks, p->opt.slots, prefix);
   }
 }
 
@@ -397,8 +421,9 @@ namespace {
 
 struct State {
   // v[0] a: earliest start of the next copy (m = 2: max(C_k, R_{k-1});
-  //         m = 1: R_k); v[1] E_k; v[2] R_k; v[3] bytes of the last block
-  int64_t v[4];
+  //         m = 1: R_k); v[1] E_k; v[2] R_k; v[3] bytes of the last block;
+  // with first-block prefetch also v[4] bytes and v[5] t_in of block 0
+  int64_t v[6];
   int nblocks;
   int prev_j;       // boundary of the previous state
   int prev_idx;     // index in the previous frontier
@@ -409,6 +434,7 @@ struct Search {
   const swapnet_options& opt;
   uint64_t slot;
   int slots;
+  bool cyclic = false;  // first-block prefetch: the finish depends on the block count's parity
   std::vector<std::vector<State>> front;
 
   Search(const std::vector<Unit>& u, const swapnet_options& o, uint64_t s)
@@ -434,8 +460,9 @@ struct Search {
     return cuts_of(j, ia) <= cuts_of(j, ib);
   }
 
-  static bool le_all(const State& a, const State& b) {
-    for (int t = 0; t < 4; ++t)
+  bool le_all(const State& a, const State& b) const {
+    if (cyclic && (a.nblocks & 1) != (b.nblocks & 1)) return false;
+    for (int t = 0; t < (cyclic ? 6 : 4); ++t)
       if (a.v[t] > b.v[t]) return false;
     return true;
   }
@@ -466,6 +493,8 @@ struct Search {
     r.v[1] = E;
     r.v[2] = R;
     r.v[3] = slots == 2 ? (int64_t)B.bytes : 0;
+    r.v[4] = s.v[4];
+    r.v[5] = s.v[5];
     r.nblocks = s.nblocks + 1;
     return r;
   }
@@ -505,7 +534,8 @@ static int64_t greedy_upper_bound(const swapnet_plan* p, int start, int64_t e0) 
 // unit), since copies and executions each form a chain; states whose bound
 // exceeds the best finish found (or a greedy plan's) cannot win.
 static int search_pipeline_capped(swapnet_plan* p, std::vector<uint32_t>* best_cuts, size_t cap,
-                                  int64_t ub_in, int64_t* best_ns, bool* exact, int start, int64_t e0) {
+                                  int64_t ub_in, int64_t* best_ns, bool* exact, int start, int64_t e0,
+                                  bool cyclic = false, int head = 0) {
   const int U = (int)p->units.size();
   std::vector<int64_t> rem_ex(U + 1, 0), rem_in(U + 1, 0);
   {
@@ -519,20 +549,62 @@ static int search_pipeline_capped(swapnet_plan* p, std::vector<uint32_t>* best_c
     }
   }
   const int64_t last_ex = U ? p->units[U - 1].t_ex : 0;
-  int64_t ub = std::min(ub_in, greedy_upper_bound(p, start, e0));
+  int64_t ub = std::min(ub_in, cyclic ? INT64_MAX : greedy_upper_bound(p, start, e0));
   auto bound = [&](const State& c, int j) -> int64_t {
     if (j == U) return c.v[1];
     return std::max(c.v[1] + rem_ex[j], c.v[0] + rem_in[j] + last_ex);
   };
+  // finish of a complete state: E, or with first-block prefetch the later of
+  // E and the next block 0's copy (INT64_MAX where the last block and the
+  // next block 0 would overlap)
+  auto finish = [&](const State& c) -> int64_t {
+    if (!cyclic) return c.v[1];
+    if (c.nblocks % 2 == 1) return std::max(c.v[1], c.v[2] + c.v[5]);  // block n-1 shares its place
+    if ((uint64_t)(c.v[3] + c.v[4]) > p->region) return INT64_MAX;
+    return std::max(c.v[1], c.v[0] + c.v[5]);
+  };
   Search S(p->units, p->opt, p->slot);
+  S.cyclic = cyclic;
   S.front.assign(U + 1, {});
   // initial state at boundary `start`: with a resident prefix, its layers
   // execute from t = 0 (E = e0) while the first copy starts at t = 0, and
-  // no swapped block waits for the prefix to be released
-  State s0{};
-  s0.v[1] = e0;
-  s0.prev_j = -1; s0.prev_idx = -1; s0.nblocks = start > 0 ? 1 : 0;
-  S.front[start].push_back(s0);
+  // no swapped block waits for the prefix to be released.  With first-block
+  // prefetch, the first block [0, c1) (c1 = head, or every c1 whose block
+  // fits the region when head is 0) gives a state at boundary c1: block 0
+  // is present at t = 0, executes at once, and the copy engine is free for
+  // block 1; states of different first blocks compete in the same fronts
+  // (v[4], v[5] carry what the finish needs)
+  if (cyclic) {
+    Block B0{};
+    for (int c1 = 1; c1 <= U; ++c1) {
+      const Unit& un = p->units[c1 - 1];
+      B0.bytes += un.bytes;
+      B0.depth += un.depth;
+      B0.t_ex += un.t_ex;
+      if (B0.bytes > p->region) break;
+      if (head > 0 && c1 != head) continue;
+      State s0{};
+      s0.v[1] = B0.t_ex;
+      s0.v[2] = B0.t_ex + (int64_t)(p->opt.eta_ns_per_tensor * B0.depth);
+      s0.v[3] = (int64_t)B0.bytes;
+      s0.v[4] = (int64_t)B0.bytes;
+      s0.v[5] = (int64_t)mul_div_ceil(p->opt.alpha_as_per_byte, B0.bytes, 1000000000ull) +
+                (int64_t)(p->opt.beta_ns_per_tensor * B0.depth);
+      s0.prev_j = -1; s0.prev_idx = -1; s0.nblocks = 1;
+      if (c1 == U) {
+        ub = std::min(ub, finish(s0));
+        S.insert(U, s0);
+      } else {
+        S.insert(c1, s0);
+      }
+    }
+    start = 1;
+  } else {
+    State s0{};
+    s0.v[1] = e0;
+    s0.prev_j = -1; s0.prev_idx = -1; s0.nblocks = start > 0 ? 1 : 0;
+    S.front[start].push_back(s0);
+  }
   // frontier states of boundary j only get children once j is final; a
   // frontier wider than kFrontCap keeps its kFrontCap states of smallest
   // bound (the result is then the best plan found, not a proven optimum)
@@ -568,7 +640,11 @@ static int search_pipeline_capped(swapnet_plan* p, std::vector<uint32_t>* best_c
         State c = S.step(S.front[j][idx], B);
         c.prev_j = j; c.prev_idx = idx;
         if (bound(c, j2) > ub) continue;
-        if (j2 == U) ub = std::min(ub, c.v[1]);
+        if (j2 == U) {
+          const int64_t f = finish(c);
+          if (f == INT64_MAX) continue;
+          ub = std::min(ub, f);
+        }
         S.insert(j2, c);
       }
     }
@@ -577,12 +653,11 @@ static int search_pipeline_capped(swapnet_plan* p, std::vector<uint32_t>* best_c
   if (F.empty()) SN_FAIL(SWAPNET_ERR_INFEASIBLE, "no feasible partition");
   int best = 0;
   for (int i = 1; i < (int)F.size(); ++i) {
-    if (F[i].v[1] < F[best].v[1] || (F[i].v[1] == F[best].v[1] && S.tie_le(U, i, best) &&
-                                     !S.tie_le(U, best, i)))
-      best = i;
+    const int64_t fi = finish(F[i]), fb = finish(F[best]);
+    if (fi < fb || (fi == fb && S.tie_le(U, i, best) && !S.tie_le(U, best, i))) best = i;
   }
   *best_cuts = S.cuts_of(U, best);  // includes `start` (the first block's boundary)
-  *best_ns = F[best].v[1];
+  *best_ns = finish(F[best]);
   return SWAPNET_OK;
 }
 
@@ -590,11 +665,12 @@ static int search_pipeline_capped(swapnet_plan* p, std::vector<uint32_t>* best_c
 // full search, which prunes every state that cannot reach it.  States
 // whose bound equals it are kept, so ties are still broken exactly.
 static int search_pipeline(swapnet_plan* p, std::vector<uint32_t>* best_cuts, int64_t* best_ns = nullptr,
-                           int start = 0, int64_t e0 = 0) {
+                           int start = 0, int64_t e0 = 0, bool cyclic = false, int head = 0,
+                           int64_t ub = INT64_MAX) {
   std::vector<uint32_t> beam_cuts;
   int64_t beam_ns = INT64_MAX;
   bool beam_exact = false;
-  int rc = search_pipeline_capped(p, &beam_cuts, 32, INT64_MAX, &beam_ns, &beam_exact, start, e0);
+  int rc = search_pipeline_capped(p, &beam_cuts, 32, ub, &beam_ns, &beam_exact, start, e0, cyclic, head);
   if (rc) return rc;
   if (beam_exact) {
     p->exact = true;
@@ -604,7 +680,7 @@ static int search_pipeline(swapnet_plan* p, std::vector<uint32_t>* best_cuts, in
   }
   int64_t ns = 0;
   bool exact = false;
-  rc = search_pipeline_capped(p, best_cuts, 4096, beam_ns, &ns, &exact, start, e0);
+  rc = search_pipeline_capped(p, best_cuts, 4096, std::min(ub, beam_ns), &ns, &exact, start, e0, cyclic, head);
   if (rc) return rc;
   p->exact = exact;
   if (best_ns) *best_ns = ns;
@@ -679,6 +755,80 @@ static int search_with_prefix(swapnet_plan* p, std::vector<uint32_t>* best_cuts)
   return SWAPNET_OK;
 }
 
+// First-block prefetch (option prefetch): for each first block [0, c1)
+// an exact search of the rest, finishing with the next block 0's copy.  The
+// plan without prefetch, timed as a cyclic schedule (when its last and first
+// blocks may be co-resident), gives the first bound; the best finish so far
+// bounds each next search.  Ties: smaller time, fewer blocks,
+// lexicographically smaller cut vector.  When the region holds more than
+// max_heads first blocks, the max_heads smallest and the first block of the
+// plan without prefetch are tried (the plan then reports exact = 0); models
+// of more than 128 units (each search takes seconds) try only the latter.
+static int search_cyclic(swapnet_plan* p, std::vector<uint32_t>* best_cuts) {
+  const int U = (int)p->units.size();
+  const int max_heads = U > 128 ? 0 : 16;
+  std::vector<int> heads;
+  {
+    uint64_t bytes = 0;
+    for (int c1 = 1; c1 <= U; ++c1) {
+      bytes += p->units[c1 - 1].bytes;
+      if (bytes > p->region) break;
+      heads.push_back(c1);
+    }
+  }
+  int64_t best = INT64_MAX;
+  int best_n = 0;
+  bool found = false;
+  std::vector<uint32_t> cuts;
+  auto consider = [&](int64_t ns, const std::vector<uint32_t>& c) {
+    const int n = (int)c.size() + 1;
+    if (!found || ns < best || (ns == best && (n < best_n || (n == best_n && c < cuts)))) {
+      best = ns;
+      best_n = n;
+      cuts = c;
+      found = true;
+    }
+  };
+  std::vector<uint32_t> cold;
+  {
+    swapnet_options o = p->opt;
+    p->opt.prefetch = 0;
+    const int rc = search_pipeline(p, &cold);
+    p->opt = o;
+    if (rc && rc != SWAPNET_ERR_INFEASIBLE) return rc;
+    if (!rc) {
+      std::vector<uint32_t> bnd{0};
+      bnd.insert(bnd.end(), cold.begin(), cold.end());
+      bnd.push_back((uint32_t)U);
+      std::vector<Block> bl;
+      for (size_t k = 0; k + 1 < bnd.size(); ++k) bl.push_back(make_block(p->units, (int)bnd[k], (int)bnd[k + 1], p->opt));
+      const size_t n = bl.size();
+      if (n % 2 == 1 || bl[0].bytes + bl[n - 1].bytes <= p->region) consider(cyclic_ns(bl), cold);
+    }
+  }
+  bool all_exact = true;
+  if ((int)heads.size() > max_heads) {
+    const int c1 = cold.empty() ? U : (int)cold[0];
+    heads.resize(max_heads);
+    if (std::find(heads.begin(), heads.end(), c1) == heads.end()) heads.insert(heads.begin(), c1);
+    all_exact = false;
+  }
+  for (int c1 : heads) {
+    std::vector<uint32_t> c;
+    int64_t ns = 0;
+    p->exact = true;
+    const int rc = search_pipeline(p, &c, &ns, 0, 0, true, c1, found ? best : INT64_MAX);
+    if (rc == SWAPNET_ERR_INFEASIBLE) continue;
+    if (rc) return rc;
+    all_exact = all_exact && p->exact;
+    consider(ns, c);
+  }
+  if (!found) SN_FAIL(SWAPNET_ERR_INFEASIBLE, "no feasible partition");
+  p->exact = all_exact;
+  *best_cuts = cuts;
+  return SWAPNET_OK;
+}
+
 static int search_exhaustive_eq4(swapnet_plan* p, std::vector<uint32_t>* best_cuts) {
   const int U = (int)p->units.size();
   if (U > 24) SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "objective 1 (Eq. 4) search is exhaustive: at most 24 units");
@@ -723,6 +873,9 @@ static int check_options(const swapnet_options& o) {
     SN_FAIL(SWAPNET_ERR_INVALID_ARG, "resident_prefix must be 0 or 1");
   if (o.resident_prefix && o.objective != 0)
     SN_FAIL(SWAPNET_ERR_INVALID_ARG, "resident_prefix needs the pipeline objective (0)");
+  if (o.prefetch != 0 && o.prefetch != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "prefetch must be 0 or 1");
+  if (o.prefetch && (o.objective != 0 || o.slots != 2 || o.resident_prefix))
+    SN_FAIL(SWAPNET_ERR_INVALID_ARG, "prefetch needs objective 0, two slots and no resident prefix");
   return SWAPNET_OK;
 }
 
@@ -780,6 +933,7 @@ int swapnet_partition(const swapnet_model_desc* desc, uint64_t budget, const swa
     std::vector<uint32_t> cuts;
     if (p->opt.objective != 0) rc = search_exhaustive_eq4(p.get(), &cuts);
     else if (p->opt.resident_prefix) rc = search_with_prefix(p.get(), &cuts);
+    else if (p->opt.prefetch) rc = search_cyclic(p.get(), &cuts);
     else rc = search_pipeline(p.get(), &cuts);
     if (rc) return rc;
     finalize_blocks(p.get(), cuts);
@@ -807,6 +961,9 @@ int swapnet_plan_from_cuts(const swapnet_model_desc* desc, const uint32_t* cuts,
     for (size_t k = 0; k < p->blocks.size(); ++k)
       if (!pair_ok(p.get(), k ? p->blocks[k - 1].bytes : 0, p->blocks[k].bytes))
         SN_FAIL(SWAPNET_ERR_INFEASIBLE, "a block (or two adjacent blocks) exceeds the arena");
+    const size_t n = p->blocks.size();
+    if (p->opt.prefetch && n >= 2 && n % 2 == 0 && p->blocks[0].bytes + p->blocks[n - 1].bytes > p->region)
+      SN_FAIL(SWAPNET_ERR_INFEASIBLE, "the last block and the next inference's first block exceed the arena");
     *out = p.release();
     return SWAPNET_OK;
   } catch (const std::bad_alloc&) {

@@ -139,6 +139,65 @@ def test_resident_prefix_partition_equals_exhaustive_oracle(slots):
     assert checked >= 10 and with_prefix >= 3
 
 
+def test_prefetch_partition_equals_exhaustive_oracle():
+    """First-block prefetch: the cyclic objective, the wrap pair and the
+    cuts identical to the oracle's brute force."""
+    r = np.random.default_rng(404)
+    checked = 0
+    for trial in range(50):
+        m = _random_model(r, int(r.integers(2, 9)))
+        opt = capi.options(slots=2, prefetch=1,
+                           alpha_as_per_byte=int(r.integers(1_000_000, 5_000_000)),
+                           beta_ns_per_tensor=int(r.integers(0, 3000)),
+                           gamma_as_per_flop=int(r.integers(100, 100_000)),
+                           eta_ns_per_tensor=int(r.integers(0, 500)))
+        wb = P.weight_bytes(m)
+        if wb == 0:
+            continue
+        budget = int(r.integers(max(1, wb // 4), wb * 2 + 1))
+        ref = P.exhaustive_partition(m, budget, _coef(opt), slots=2, prefetch=True)
+        desc = capi.Desc(m)
+        if ref is None:
+            with pytest.raises(capi.SwapnetError) as ei:
+                capi.Plan.partition(desc, budget, opt)
+            assert ei.value.code == capi.ERR_INFEASIBLE
+            continue
+        plan = capi.Plan.partition(desc, budget, opt)
+        info = plan.info()
+        assert plan.cuts() == ref["cuts"], (trial, plan.cuts(), ref["cuts"])
+        assert info["n_blocks"] == ref["n"]
+        assert info["predicted_ns"] == ref["predicted_ns"]
+        # an explicit cut vector gets the same cyclic prediction
+        again = capi.Plan.from_cuts(desc, ref["cuts"], budget, opt)
+        assert again.info()["predicted_ns"] == ref["predicted_ns"]
+        checked += 1
+    assert checked >= 10
+
+
+def test_prefetch_options_and_wrap_pair_are_checked():
+    m = _random_model(np.random.default_rng(9), 5)
+    desc = capi.Desc(m)
+    wb = P.weight_bytes(m)
+    for bad in (dict(prefetch=2), dict(prefetch=1, slots=1), dict(prefetch=1, objective=1),
+                dict(prefetch=1, resident_prefix=1)):
+        with pytest.raises(capi.SwapnetError) as ei:
+            capi.Plan.partition(desc, wb, capi.options(**bad))
+        assert ei.value.code == capi.ERR_INVALID_ARG
+    # eight equal layers of x bytes in blocks of 3, 1, 1, 3 layers in a
+    # region of 4x: every adjacent pair fits (4x, 2x, 4x), the wrap pair
+    # (last, first) needs 6x
+    layers = [dict(op="linear", src=[i - 1], k=128, n=128, act="relu", res=None, res_post=False) for i in range(8)]
+    mm = dict(name="rand", model_id=78, dtype="f16", input=(2, 1, 1, 128), layers=layers, outputs=[7])
+    x = sum(P.align(b) for b in P.layer_tensor_bytes(mm, 0))
+    d = capi.Desc(mm)
+    plain = capi.Plan.from_cuts(d, [3, 4, 5], 4 * x, capi.options())
+    assert [b["bytes"] for b in plain.blocks()] == [3 * x, x, x, 3 * x]
+    with pytest.raises(capi.SwapnetError) as ei:
+        capi.Plan.from_cuts(d, [3, 4, 5], 4 * x, capi.options(prefetch=1))
+    assert ei.value.code == capi.ERR_INFEASIBLE
+    capi.Plan.from_cuts(d, [3, 4, 5], 6 * x, capi.options(prefetch=1))
+
+
 def test_resident_prefix_never_worse_than_swapping_everything():
     for name in ("mlp6", "resnet50", "vgg16"):
         m = synth.arch.MODELS[name]()

@@ -323,6 +323,38 @@ def test_resident_prefix_bit_exact_over_repeated_inferences(name):
         assert all(p.tobytes() == q.tobytes() for p, q in zip(a, b)), req
 
 
+@pytest.mark.parametrize("name,variant", [("resnet50", capi.SWAP_AUTO), ("yolov3", capi.SWAP_MEMCPY),
+                                          ("resnet50", capi.SWAP_ZEROCOPY)])
+def test_first_block_prefetch_bit_exact_over_repeated_inferences(name, variant):
+    """First-block prefetch: each inference swaps the next one's first block
+    in at its end; every call (the first one from the load-time upload) and
+    every call after a switch to another prefetch plan gives the resident
+    bits, on eager and graph launches alike."""
+    m = synth.arch.MODELS[name]()
+    w = synth.gen.model_weights(m)
+    d = capi.Desc(m)
+    host = capi.HostWeights(w)
+    wb = OP.weight_bytes(m)
+    opt = capi.options(prefetch=1, swap_variant=variant)
+    plan = capi.Plan.partition(d, int(wb * 0.4) // 256 * 256, opt)
+    assert plan.info()["n_blocks"] > 2
+    sw = Runner(m, w, plan, host)
+    rs = Runner(m, w, capi.Plan.resident(d), host)
+    for req in range(3):
+        x = synth.gen.model_input(m, request=req)
+        a, b = sw.run(x), rs.run(x)
+        assert all(p.tobytes() == q.tobytes() for p, q in zip(a, b)), req
+    sw.engine.set_profiling(True)  # eager launches
+    x = synth.gen.model_input(m, request=7)
+    assert all(p.tobytes() == q.tobytes() for p, q in zip(sw.run(x), rs.run(x)))
+    sw.engine.set_profiling(False)
+    sw.engine.adapt(capi.Plan.partition(d, int(wb * 0.3) // 256 * 256, opt))
+    for req in range(2):
+        x = synth.gen.model_input(m, request=10 + req)
+        a, b = sw.run(x), rs.run(x)
+        assert all(p.tobytes() == q.tobytes() for p, q in zip(a, b)), req
+
+
 def test_engine_adapts_to_new_budgets_between_inferences():
     """Runtime budget adaptation: one engine switched through plans for
     shrinking and growing budgets (made ahead, like the paper's look-up

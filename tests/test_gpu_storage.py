@@ -44,6 +44,15 @@ def test_swapped_from_file_equals_resident(name, kw, frac, tmp_path):
     check_close(m, fr.decode(got), oracle_outputs(m, w, x))
 
 
+def test_first_block_prefetch_from_file(tmp_path):
+    m, w, x, d, host, wf, budget, _ = _setup("resnet50", dict(batch=1), 0.40, tmp_path)
+    rs = Runner(m, w, capi.Plan.resident(d), host).run(x)
+    fr = Runner(m, w, capi.Plan.partition(d, budget, capi.options(prefetch=1)), wf)
+    for rep in range(3):
+        got = fr.run(x)
+        assert all(a.tobytes() == b.tobytes() for a, b in zip(got, rs)), rep
+
+
 def test_resident_plan_and_adaptation_from_file(tmp_path):
     m, w, x, d, host, wf, budget, _ = _setup("resnet50", dict(batch=1), 0.40, tmp_path)
     ref = Runner(m, w, capi.Plan.resident(d), host).run(x)

@@ -242,3 +242,47 @@ def test_prefix_candidates_rule():
     # one slot: the rest needs only its largest unit; r = 3 leaves 1024 beside
     # 1024 bytes of prefix (exactly 2048), r = 4 would need 2048 + 512
     assert max(cands1) == 3
+
+
+def test_cyclic_pipeline_hand_worked():
+    """First-block prefetch (steady state): blocks (t_in, t_ex) = (4, 2),
+    (3, 5), (2, 1), (1, 3), t_out = 0, two slots.  Block 0 is present at
+    t = 0 and ends at 2; copies of blocks 1-3 end at 3, 5 (block 2 waits
+    for block 0's release at 2: no wait), 9 (block 3 waits for block 1's
+    release at 8); executions end at 8, 9, 12.  Four blocks: the next
+    block 0 shares block 2's place, so its copy starts at max(9, 9) and
+    ends at 13, after the last execution: 13.  The same blocks run cold
+    (block 0 copied first) finish at 16."""
+    blocks = [(10, 4, 2, 0), (10, 3, 5, 0), (10, 2, 1, 0), (10, 1, 3, 0)]
+    assert P.cyclic_time(blocks) == 13
+    assert P.pipeline_time(blocks, 2) == 16
+    # three blocks: block 2 shares block 0's place; its release at 9 plus 4
+    assert P.cyclic_time(blocks[:3]) == 13
+    # one block: execute, then copy it in again for the next inference
+    assert P.cyclic_time(blocks[:1]) == 2 + 4
+
+
+def test_cyclic_pipeline_invariants():
+    r = np.random.default_rng(17)
+    for _ in range(300):
+        n = int(r.integers(1, 7))
+        blocks = [(int(r.integers(1, 100)), int(r.integers(0, 50)), int(r.integers(0, 50)), 0) for _ in range(n)]
+        t = P.cyclic_time(blocks)
+        # one copy engine and one execution stream: both chains fit in a period
+        assert t >= sum(b[1] for b in blocks) and t >= sum(b[2] for b in blocks)
+        # a first block that costs nothing to copy: the cold pipeline exactly
+        free0 = [(blocks[0][0], 0) + blocks[0][2:]] + blocks[1:]
+        assert P.cyclic_time(free0) == P.pipeline_time(free0, 2)
+        # prefetching never loses to running cold (the copy moves, it does not grow)
+        assert t <= P.pipeline_time(blocks, 2) + blocks[0][1]
+
+
+def test_cyclic_feasibility_adds_the_wrap_pair():
+    # even count: the last block and the next first block are co-resident
+    # (every adjacent pair fits; only the wrap pair 424 + 624 does not)
+    wrap_fails = [(624, 0, 0, 0), (400, 0, 0, 0), (600, 0, 0, 0), (424, 0, 0, 0)]
+    assert P.feasible(wrap_fails, 1024, 2) is True
+    assert P.feasible_cyclic(wrap_fails, 1024) is False
+    assert P.feasible_cyclic([(600, 0, 0, 0), (400, 0, 0, 0), (600, 0, 0, 0), (424, 0, 0, 0)], 1024) is True
+    # odd count: the last block sits where the first does; only Eq. 3 applies
+    assert P.feasible_cyclic([(600, 0, 0, 0), (400, 0, 0, 0), (600, 0, 0, 0)], 1024) is True
