@@ -333,15 +333,18 @@ def run_llm(args, rank, world):
             res.append((evs[0].elapsed_time(evs[1]), evs[1].elapsed_time(evs[2]) / n_dec))
         return res
 
+    # the link check and the clock sampler start before the warm-up: a fresh
+    # page-locked allocation right before the timed steps made the next
+    # prefill pass 5x slower (the host mappings are walked again)
+    link_before = measure_link_peak(stream)
+    clocks = ClockSampler(int(os.environ.get("LOCAL_RANK", "0")), interval_ms=500)
+    clocks.start()
     for _ in range(max(1, args.warmup)):
         one(ep, ed)
         one(rp, rd)
     torch.cuda.synchronize()
     for e in (ep, ed, rp, rd):
         e.sync()
-    link_before = measure_link_peak(stream)
-    clocks = ClockSampler(int(os.environ.get("LOCAL_RANK", "0")), interval_ms=500)
-    clocks.start()
     launches0 = ep.stats()["kernel_launches"] + ed.stats()["kernel_launches"]
     sw = timed(ep, ed, args.steps)
     launches = ep.stats()["kernel_launches"] + ed.stats()["kernel_launches"] - launches0
