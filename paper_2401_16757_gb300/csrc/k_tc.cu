@@ -58,9 +58,18 @@ template <int BN> struct Cfg {
   static constexpr int kSmem = kStageBytes + kRecvBytes + kBiasBytes + 256 + 1024;
 };
 
-template <typename T, int BN, bool GATHER>
+// A operand: kA2d (2-D TMA of a row-major matrix: linear layers, 1x1
+// stride-1 convs), kAGather (cp.async im2col gather by warps 2..5), kATap
+// (convs whose taps are whole 64-channel k-blocks: one 4-D TMA per k-block
+// of the tap's 64 channels over a wt x ht patch of output pixels, zero fill
+// for the padding; the CTA's 128 rows are that patch, rows >= wt * ht unused)
+constexpr int kA2d = 0, kAGather = 1, kATap = 2;
+
+template <typename T, int BN, int AMODE>
 __global__ void __launch_bounds__(kThreads, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const TcArgs p) {
+  constexpr bool GATHER = AMODE == kAGather;
+  constexpr bool TAP = AMODE == kATap;
   constexpr int kStages = Cfg<BN>::kStages;
   constexpr int kLag = Cfg<BN>::kLag;
   constexpr int kBBytes = Cfg<BN>::kBBytes;
@@ -80,7 +89,36 @@ __global__ void __launch_bounds__(kThreads, 1)
   auto empty_bar = [&](int s) { return empty0 + 8u * s; };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m0 = blockIdx.x * kBM, n0 = blockIdx.y * BN;
+  const int m0 = TAP ? 0 : blockIdx.x * kBM, n0 = blockIdx.y * BN;
+  // tap mode: this CTA's patch (image, patch row th, patch column tw)
+  int pimg = 0, pth = 0, ptw = 0;
+  if (TAP) {
+    const int patches = p.tiles_w * p.tiles_h;
+    pimg = blockIdx.x / patches;
+    const int rem = blockIdx.x - pimg * patches;
+    pth = rem / p.tiles_w;
+    ptw = rem - pth * p.tiles_w;
+  }
+  const uint32_t a_bytes = TAP ? (uint32_t)(p.wt * p.ht * 128) : (GATHER ? 0u : (uint32_t)kABytes);
+  // output row of tile row r (-1: no output)
+  auto row_m = [&](int r) -> int {
+    if (TAP) {
+      if (r >= p.wt * p.ht) return -1;
+      const int oy = pth * p.ht + r / p.wt, ox = ptw * p.wt + r % p.wt;
+      return (oy < p.Ho && ox < p.Wo) ? (pimg * p.Ho + oy) * p.Wo + ox : -1;
+    }
+    return m0 + r < p.M ? m0 + r : -1;
+  };
+  // A tile of k-block kb into stage buffer dst (TMA modes)
+  auto load_a = [&](uint32_t dst, uint32_t bar, int kb) {
+    if (TAP) {
+      const int k0 = kb * kBK, tap = k0 / p.C, c0 = k0 - tap * p.C;
+      const int ry = tap / p.kw, rx = tap - ry * p.kw;
+      tma_load_4d(dst, &tmA, bar, c0, ptw * p.wt * p.stride - p.pad + rx, pth * p.ht * p.stride - p.pad + ry, pimg);
+    } else {
+      tma_load_2d(dst, &tmA, bar, kb * kBK, m0);
+    }
+  };
   const int KB = (p.K + kBK - 1) / kBK;
   const int kb0 = blockIdx.z * p.kb_per_split;
   const int nk = min(KB, kb0 + p.kb_per_split) - kb0;  // >= 1 by construction
@@ -124,20 +162,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       // out before waiting for the previous kernel (they do not depend on it)
       const int early = min(nk, kStages);
       for (int i = 0; i < early; ++i) {
-        mbar_arrive_expect_tx(full_bar(i), kBBytes + (GATHER ? 0 : kABytes));
+        mbar_arrive_expect_tx(full_bar(i), kBBytes + a_bytes);
         tma_load_2d(smem_u32(sB + i * kBBytes), &tmB, full_bar(i), (kb0 + i) * kBK, n0);
       }
       pdl_wait();
       if (!GATHER)
-        for (int i = 0; i < early; ++i)
-          tma_load_2d(smem_u32(sA + i * kABytes), &tmA, full_bar(i), (kb0 + i) * kBK, m0);
+        for (int i = 0; i < early; ++i) load_a(smem_u32(sA + i * kABytes), full_bar(i), kb0 + i);
       int i = early;
       for (; i < nk; ++i) {
         const int s = i % kStages, r = i / kStages, kb = kb0 + i;
         if (!mbar_wait_bounded(empty_bar(s), (r & 1) ^ 1, abort_flag, p.err)) break;
-        mbar_arrive_expect_tx(full_bar(s), kBBytes + (GATHER ? 0 : kABytes));
+        mbar_arrive_expect_tx(full_bar(s), kBBytes + a_bytes);
         tma_load_2d(smem_u32(sB + s * kBBytes), &tmB, full_bar(s), kb * kBK, n0);
-        if (!GATHER) tma_load_2d(smem_u32(sA + s * kABytes), &tmA, full_bar(s), kb * kBK, m0);
+        if (!GATHER) load_a(smem_u32(sA + s * kABytes), full_bar(s), kb);
       }
       if (i < nk) {
         // aborted: let the loads already issued land before the CTA exits
@@ -237,7 +274,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---------------- epilogue
     const int q = warp & 3;
     const int row = q * 32 + lane;
-    const int m = m0 + row;
+    const int m = row_m(row);  // -1: this row has no output
     const bool ok = mbar_wait_bounded(accum_bar, 0, abort_flag, p.err);
     tc_fence_after();
     const bool vec_ok = ((p.ldy | n0) % 8 == 0) && (!p.e.res || ((p.e.ldr | n0) % 8 == 0));
@@ -247,7 +284,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t r[32];
         tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)c0, r);
         tmem_ld_wait();
-        if (m < p.M && n0 + c0 < p.N) {
+        if (m >= 0 && n0 + c0 < p.N) {
           float v[32];
 #pragma unroll
           for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
@@ -260,7 +297,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // this split's partial goes to slot blockIdx.z of each owner
       const int cpo = (((BN + splits - 1) / splits) + 3) & ~3;
       const int rs = cpo + 4;  // row stride of a slot, floats
-      const bool mine = ok && m < p.M && row < kFewRows;
+      const bool mine = ok && m >= 0 && row < kFewRows;
       asm volatile("barrier.cluster.wait;" ::: "memory");  // every peer is running
 #pragma unroll 1
       for (int c0 = 0; c0 < BN; c0 += 32) {
@@ -296,7 +333,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t r[32];
         tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)c0, r);
         tmem_ld_wait();
-        if (ok && m < p.M) {
+        if (ok && m >= 0) {
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
             uint32_t ra;
@@ -319,7 +356,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)c0, r);
         tmem_ld_wait();
         const int n = n0 + c0;
-        if (m < p.M && n < p.N) {
+        if (m >= 0 && n < p.N) {
           float* dst = part + (int64_t)m * p.N + n;
           if (pvec && n + 32 <= p.N) {
 #pragma unroll
@@ -349,7 +386,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll 1
         for (int c0 = 0; c0 < BN; c0 += 32) {
           const int n = n0 + c0;
-          if (m >= p.M || n >= p.N) continue;
+          if (m < 0 || n >= p.N) continue;
           float v[32];
 #pragma unroll
           for (int j = 0; j < 32; ++j) v[j] = 0.f;
@@ -399,18 +436,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else {
       const int rpo = (kBM + splits - 1) / splits;
       const int r0 = (int)blockIdx.z * rpo;
-      const int rows = max(0, min(min(rpo, kBM - r0), p.M - m0 - r0));
+      const int rows = TAP ? max(0, min(rpo, kBM - r0)) : max(0, min(min(rpo, kBM - r0), p.M - m0 - r0));
       const int groups = rows * (BN / 4);
       for (int g = threadIdx.x; g < groups; g += kThreads) {
         const int rr = g / (BN / 4), c4 = g % (BN / 4);
         const int n = n0 + 4 * c4;
+        const int mm = row_m(r0 + rr);
+        if (mm < 0) continue;
         const float* src = recv + rr * (BN + 4) + 4 * c4;
         float4 acc = *reinterpret_cast<const float4*>(src);
         for (int z = 1; z < splits; ++z) {
           const float4 v = *reinterpret_cast<const float4*>(src + z * rpo * (BN + 4));
           acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
         }
-        if (n < p.N) finish4<T>(acc, sbias + 4 * c4, p, m0 + r0 + rr, n);
+        if (n < p.N) finish4<T>(acc, sbias + 4 * c4, p, mm, n);
       }
     }
   }
@@ -497,10 +536,10 @@ double conv_patch(int ho, int wo, int stride, int* wt, int* ht) {
   return best;
 }
 
-template <typename T, int BN, bool GATHER>
+template <typename T, int BN, int AMODE>
 int launch_inst(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) {
   static bool attr_done = false;  // per instantiation
-  auto kern = tc_gemm_kernel<T, BN, GATHER>;
+  auto kern = tc_gemm_kernel<T, BN, AMODE>;
   if (!attr_done) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<BN>::kSmem) != cudaSuccess)
       SN_FAIL(SWAPNET_ERR_CUDA, "cudaFuncSetAttribute failed");
@@ -518,7 +557,11 @@ int launch_inst(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) {
   a.counters = g.counters;
   if (pl.splits > 1 && !pl.cluster && (!g.partial || !g.counters))
     SN_FAIL(SWAPNET_ERR_INVALID_ARG, "split-K needs scratch");
-  const dim3 grid((g.M + kBM - 1) / kBM, (g.N + BN - 1) / BN, pl.splits);
+  a.wt = pl.wt; a.ht = pl.ht; a.tiles_w = pl.tiles_w; a.tiles_h = pl.tiles_h;
+  const int64_t mtiles = AMODE == kATap ? (int64_t)g.M / ((int64_t)g.Ho * g.Wo) * pl.tiles_w * pl.tiles_h
+                                        : (g.M + kBM - 1) / kBM;
+  if (AMODE == kATap && (pl.splits > 1 && !pl.cluster)) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "tap mode needs cluster split-K");
+  const dim3 grid((unsigned)mtiles, (g.N + BN - 1) / BN, pl.splits);
   a.cluster = pl.cluster;
   const bool csplit = pl.splits > 1 && pl.cluster;
   if (csplit) {
@@ -557,11 +600,11 @@ int launch_inst(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) {
 
 // Largest cluster (along the split dimension) that the device can co-schedule
 // for this kernel instance: 16, 8, 4 or 2 (cached per instance).
-template <typename T, int BN, bool GATHER>
+template <typename T, int BN, int AMODE>
 int max_cluster_inst() {
   static int cached = -1;
   if (cached >= 0) return cached;
-  auto kern = tc_gemm_kernel<T, BN, GATHER>;
+  auto kern = tc_gemm_kernel<T, BN, AMODE>;
   cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<BN>::kSmem);
   cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   int best = 1;
@@ -596,7 +639,7 @@ int active_clusters_inst(int c) {
   static int cached[9] = {-1, -1, -1, -1, -1, -1, -1, -1, -1};
   if (c < 1 || c > 8) return 0;
   if (cached[c] >= 0) return cached[c];
-  auto kern = tc_gemm_kernel<T, 256, false>;
+  auto kern = tc_gemm_kernel<T, 256, kA2d>;
   cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<256>::kSmem);
   cudaLaunchConfig_t cfg;
   std::memset(&cfg, 0, sizeof(cfg));
@@ -625,12 +668,12 @@ int active_clusters(int dtype, int c) {
 
 int max_cluster(int dtype, int bn, bool gather) {
   const bool bf = dtype == SWAPNET_BF16;
-  if (bn == 256) return bf ? max_cluster_inst<__nv_bfloat16, 256, false>() : max_cluster_inst<__half, 256, false>();
+  if (bn == 256) return bf ? max_cluster_inst<__nv_bfloat16, 256, kA2d>() : max_cluster_inst<__half, 256, kA2d>();
   if (bn == 64)
-    return gather ? (bf ? max_cluster_inst<__nv_bfloat16, 64, true>() : max_cluster_inst<__half, 64, true>())
-                  : (bf ? max_cluster_inst<__nv_bfloat16, 64, false>() : max_cluster_inst<__half, 64, false>());
-  return gather ? (bf ? max_cluster_inst<__nv_bfloat16, 128, true>() : max_cluster_inst<__half, 128, true>())
-                : (bf ? max_cluster_inst<__nv_bfloat16, 128, false>() : max_cluster_inst<__half, 128, false>());
+    return gather ? (bf ? max_cluster_inst<__nv_bfloat16, 64, kAGather>() : max_cluster_inst<__half, 64, kAGather>())
+                  : (bf ? max_cluster_inst<__nv_bfloat16, 64, kA2d>() : max_cluster_inst<__half, 64, kA2d>());
+  return gather ? (bf ? max_cluster_inst<__nv_bfloat16, 128, kAGather>() : max_cluster_inst<__half, 128, kAGather>())
+                : (bf ? max_cluster_inst<__nv_bfloat16, 128, kA2d>() : max_cluster_inst<__half, 128, kA2d>());
 }
 
 }  // namespace
@@ -724,15 +767,34 @@ int tc_prepare(const TcGemm& g, TcPlan* p) {
     p->ready = 1;
     return SWAPNET_OK;
   }
+  // convolutions whose taps are whole 64-channel k-blocks: A by one 4-D TMA
+  // per tap over a pixel patch (as in the persistent kernel) instead of the
+  // cp.async gather, when the patches fill the 128 rows well enough or need
+  // no more CTAs than 128-row tiles would (these layers are latency-bound:
+  // unused MMA rows cost nothing, the gather's address work does); the CTA
+  // grid then runs over patches
+  int twt = 0, tht = 0;
+  bool tap = false;
+  int64_t mt = (int64_t)((g.M + kBM - 1) / kBM);
+  if (g.conv && g.cluster_max > 0 && g.C % kBK == 0) {
+    const double util = conv_patch(g.Ho, g.Wo, g.stride, &twt, &tht);
+    const int64_t patches = twt > 0 ? (int64_t)g.M / ((int64_t)g.Ho * g.Wo) * ((g.Wo + twt - 1) / twt) *
+                                          ((g.Ho + tht - 1) / tht)
+                                    : 0;
+    if (twt > 0 && (util >= 0.75 || patches <= mt)) {
+      tap = true;
+      mt = patches;
+    }
+  }
   if (Nd <= 64) {
     p->bn = 64;
   } else {
-    const int64_t tiles128 = (int64_t)((g.M + kBM - 1) / kBM) * ((Nd + 127) / 128);
+    const int64_t tiles128 = mt * ((Nd + 127) / 128);
     p->bn = tiles128 < sms ? 64 : 128;
   }
   // deterministic split-K: enough CTAs to cover the SMs, >= 2 k-blocks each
-  const int64_t tiles_d = (int64_t)((g.M + kBM - 1) / kBM) * ((Nd + p->bn - 1) / p->bn);
-  const int64_t tiles = (int64_t)((g.M + kBM - 1) / kBM) * ((g.N + p->bn - 1) / p->bn);
+  const int64_t tiles_d = mt * ((Nd + p->bn - 1) / p->bn);
+  const int64_t tiles = mt * ((g.N + p->bn - 1) / p->bn);
   int64_t splits = tiles_d >= sms ? 1 : std::min<int64_t>(sms / tiles_d, std::max(1, KB / 2));
   if (g.cluster_max > 0) {
     // cluster split-K, from a sweep of every split count on the batch-1 CNN
@@ -742,7 +804,7 @@ int tc_prepare(const TcGemm& g, TcPlan* p) {
     if (KB <= 8) splits = 1;
     else splits = std::min<int64_t>(splits, std::min<int64_t>(8, std::max<int64_t>(1, 96 / tiles_d)));
   }
-  const int cap = g.cluster_max > 0 ? std::min(g.cluster_max, max_cluster(g.dtype, p->bn, g.conv != 0)) : 32;
+  const int cap = g.cluster_max > 0 ? std::min(g.cluster_max, max_cluster(g.dtype, p->bn, g.conv && !tap)) : 32;
   splits = std::max<int64_t>(1, std::min<int64_t>(splits, cap));
   p->cluster = g.cluster_max > 0 ? 1 : 0;
   p->kb_per_split = (KB + (int)splits - 1) / (int)splits;
@@ -755,6 +817,18 @@ int tc_prepare(const TcGemm& g, TcPlan* p) {
     rc = make_tmap(&p->tmA, g.dtype, g.A, (uint64_t)g.K, (uint64_t)g.M, (uint64_t)g.lda * 2, (uint32_t)kBM);
     if (rc) return rc;
   }
+  if (tap) {
+    p->tma_conv = 1;
+    p->wt = twt;
+    p->ht = tht;
+    p->tiles_w = (g.Wo + twt - 1) / twt;
+    p->tiles_h = (g.Ho + tht - 1) / tht;
+    if (g.A) {
+      const int n_img = (int)((int64_t)g.M / ((int64_t)g.Ho * g.Wo));
+      rc = make_tmap_conv4d(&p->tmA, g.dtype, g.A, n_img, g.H, g.Wd, g.C, twt, tht, g.stride);
+      if (rc) return rc;
+    }
+  }
   p->ready = 1;
   return SWAPNET_OK;
 }
@@ -763,13 +837,17 @@ int launch_tc_gemm(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) 
   if (!pl.ready) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "tcgen05 GEMM not prepared");
   if (pl.persist) return launch_tc_persist(g, pl, err, s);
   const bool bf = g.dtype == SWAPNET_BF16;
-  if (g.conv) {
-    if (pl.bn == 64) return bf ? launch_inst<__nv_bfloat16, 64, true>(g, pl, err, s) : launch_inst<__half, 64, true>(g, pl, err, s);
-    return bf ? launch_inst<__nv_bfloat16, 128, true>(g, pl, err, s) : launch_inst<__half, 128, true>(g, pl, err, s);
+  if (g.conv && pl.tma_conv) {
+    if (pl.bn == 64) return bf ? launch_inst<__nv_bfloat16, 64, kATap>(g, pl, err, s) : launch_inst<__half, 64, kATap>(g, pl, err, s);
+    return bf ? launch_inst<__nv_bfloat16, 128, kATap>(g, pl, err, s) : launch_inst<__half, 128, kATap>(g, pl, err, s);
   }
-  if (pl.bn == 64) return bf ? launch_inst<__nv_bfloat16, 64, false>(g, pl, err, s) : launch_inst<__half, 64, false>(g, pl, err, s);
-  if (pl.bn == 256) return bf ? launch_inst<__nv_bfloat16, 256, false>(g, pl, err, s) : launch_inst<__half, 256, false>(g, pl, err, s);
-  return bf ? launch_inst<__nv_bfloat16, 128, false>(g, pl, err, s) : launch_inst<__half, 128, false>(g, pl, err, s);
+  if (g.conv) {
+    if (pl.bn == 64) return bf ? launch_inst<__nv_bfloat16, 64, kAGather>(g, pl, err, s) : launch_inst<__half, 64, kAGather>(g, pl, err, s);
+    return bf ? launch_inst<__nv_bfloat16, 128, kAGather>(g, pl, err, s) : launch_inst<__half, 128, kAGather>(g, pl, err, s);
+  }
+  if (pl.bn == 64) return bf ? launch_inst<__nv_bfloat16, 64, kA2d>(g, pl, err, s) : launch_inst<__half, 64, kA2d>(g, pl, err, s);
+  if (pl.bn == 256) return bf ? launch_inst<__nv_bfloat16, 256, kA2d>(g, pl, err, s) : launch_inst<__half, 256, kA2d>(g, pl, err, s);
+  return bf ? launch_inst<__nv_bfloat16, 128, kA2d>(g, pl, err, s) : launch_inst<__half, 128, kA2d>(g, pl, err, s);
 }
 
 // ------------------------------------------------------------ allocation-free GEMM

@@ -67,6 +67,14 @@ def _check_model(m, budget_frac=0.5, slots=2, variant=capi.SWAP_AUTO):
     (1, 1, 64, 48, 220),    # persistent 2-D TMA, two sub-tiles per tile, odd m-tile count, N 48
     (3, 1, 256, 256, 7),    # deep K, one M tile: split-K with last-CTA reduction
     (3, 1, 64, 24, 9),      # N below one 32-column chunk
+    (3, 1, 64, 128, 14),    # few tiles, taps of 64 channels: A by 4-D TMA over 14 x 9 pixel patches
+    (3, 2, 128, 128, 28),   # the same, strided
+    (1, 2, 256, 256, 28),   # strided pointwise by 4-D TMA
+    (3, 1, 64, 64, 26),     # 26 x 4 patches, last patch row ragged
+    (3, 1, 256, 256, 14),   # 4-D TMA A with cluster split-K (36 k-blocks)
+    (1, 2, 128, 256, 56),   # 28 x 4 patches
+    (3, 1, 512, 128, 7),    # 7 x 7 patch (49 of 128 rows), as many CTAs as 128-row tiles
+    (3, 2, 256, 64, 13),    # strided, 7 x 7 output, ragged against the 13-pixel input
 ])
 def test_conv_layer(dtype, k, stride, cin, cout, hw):
     m = _model([_conv(-1, cin, cout, k, stride)], (2, hw, hw, cin), dtype)
