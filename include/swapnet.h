@@ -496,6 +496,10 @@ int swapnet_engine_last_times(swapnet_engine* eng, float* unit_us, uint32_t n_un
 int swapnet_engine_last_timeline(swapnet_engine* eng, float* unit_start, float* unit_end, uint32_t n_units,
                                  float* swap_start, float* swap_end, uint32_t n_blocks);
 
+/* Waits for the device to finish the engine's work (inferences may still be
+ * queued on the caller's stream), then releases its streams, events,
+ * graphs, staging buffers and engine-owned device memory, and unregisters
+ * the host ranges it registered.  NULL is ignored. */
 void swapnet_engine_free(swapnet_engine* eng);
 
 /* ------------------------------------------------- allocation-free GEMM */

@@ -147,6 +147,9 @@ namespace swapnet {
 static int release(swapnet_engine* e) {
   if (!e) return SWAPNET_OK;
   cudaSetDevice(e->device);
+  // a graph replay may still be queued on the caller's stream, and the read
+  // host functions of a file engine dereference this engine
+  cudaDeviceSynchronize();
   if (e->copy) cudaStreamSynchronize(e->copy);
   for (cudaEvent_t ev : {e->slot_free[0], e->slot_free[1], e->ready[0], e->ready[1]})
     if (ev) cudaEventDestroy(ev);
