@@ -53,6 +53,19 @@ def test_first_block_prefetch_from_file(tmp_path):
         assert all(a.tobytes() == b.tobytes() for a, b in zip(got, rs)), rep
 
 
+def test_resident_prefix_from_file(tmp_path):
+    """A resident-prefix plan (an extension) from a weights file: the
+    prefix is read once at load, the rest for every inference."""
+    m, w, x, d, host, wf, budget, _ = _setup("resnet50", dict(batch=1), 0.40, tmp_path)
+    rs = Runner(m, w, capi.Plan.resident(d), host).run(x)
+    plan = capi.Plan.partition(d, budget, capi.options(resident_prefix=1))
+    assert plan.info()["prefix_units"] > 0
+    fr = Runner(m, w, plan, wf)
+    for rep in range(3):
+        got = fr.run(x)
+        assert all(a.tobytes() == b.tobytes() for a, b in zip(got, rs)), rep
+
+
 def test_resident_plan_and_adaptation_from_file(tmp_path):
     m, w, x, d, host, wf, budget, _ = _setup("resnet50", dict(batch=1), 0.40, tmp_path)
     ref = Runner(m, w, capi.Plan.resident(d), host).run(x)
