@@ -519,6 +519,10 @@ static int capture(swapnet_engine* e, const void* din, void* dout, cudaGraphExec
 // So whole inferences (CUDA graph replays on scratch input and output
 // buffers) are timed with the per-block choice, with every block on the copy
 // engine and with every block zero-copy, and the fastest assignment is kept.
+// Unless the options fix the zero-copy kernel's CTA count, every-block
+// zero-copy is also timed with 24 and 16 CTAs: fewer CTAs leave more SMs to
+// the layers while still keeping ahead of them (measured on ResNet-50 and
+// YOLOv3: 1-2 % faster inferences than 32).
 // Decoder models (which need a bound state) keep the per-block choice.
 static int calibrate_in_situ(swapnet_engine* e) {
   const Model& m = e->plan.model;
@@ -533,19 +537,30 @@ static int calibrate_in_situ(swapnet_engine* e) {
   }
   cudaMemset(din, 0, align_up(m.in_bytes));
   std::vector<std::vector<int>> cand(1);
+  std::vector<int> ctas(1, e->zc_ctas);  // zero-copy CTAs of each candidate
   for (const EngBlock& b : e->blocks) cand[0].push_back(b.variant);
   cand.push_back(std::vector<int>(e->blocks.size(), SWAPNET_SWAP_MEMCPY));
+  ctas.push_back(e->zc_ctas);
   bool zc_all = true;
   for (size_t k = 0; k < e->blocks.size(); ++k)
     zc_all = zc_all && (e->plan.blocks[k].slot < 0 || zerocopy_ok(e->blocks[k]));
-  if (zc_all) cand.push_back(std::vector<int>(e->blocks.size(), SWAPNET_SWAP_ZEROCOPY));
+  if (zc_all) {
+    std::vector<int> n_ctas{e->zc_ctas};
+    if (e->plan.opt.zc_ctas == 0) n_ctas = {e->zc_ctas, 24, 16};
+    for (int c : n_ctas) {
+      cand.push_back(std::vector<int>(e->blocks.size(), SWAPNET_SWAP_ZEROCOPY));
+      ctas.push_back(c);
+    }
+  }
   cudaEvent_t a = nullptr, b = nullptr;
   int rc = SWAPNET_OK;
   if (cudaEventCreate(&a) != cudaSuccess || cudaEventCreate(&b) != cudaSuccess) rc = SWAPNET_ERR_CUDA;
   float best = 1e30f;
   size_t best_i = 0;
+  const int zc0 = e->zc_ctas;
   for (size_t c = 0; c < cand.size() && rc == SWAPNET_OK; ++c) {
     for (size_t k = 0; k < e->blocks.size(); ++k) e->blocks[k].variant = cand[c][k];
+    e->zc_ctas = ctas[c];
     cudaGraphExec_t ge = nullptr;
     rc = capture(e, din, dout, &ge);
     if (rc) break;
@@ -568,10 +583,13 @@ static int calibrate_in_situ(swapnet_engine* e) {
       best_i = c;
     }
   }
-  if (rc == SWAPNET_OK)
+  if (rc == SWAPNET_OK) {
     for (size_t k = 0; k < e->blocks.size(); ++k) e->blocks[k].variant = cand[best_i][k];
-  else
+    e->zc_ctas = ctas[best_i];
+  } else {
+    e->zc_ctas = zc0;
     set_error("swap variant calibration failed");
+  }
   if (a) cudaEventDestroy(a);
   if (b) cudaEventDestroy(b);
   cudaFree(din);
@@ -800,6 +818,7 @@ static bool prefetch_on(const swapnet_engine* e);
 
 static int bind_plan(swapnet_engine* e, void* d_arena_user, uint64_t arena_bytes_user, bool preloaded_arena) {
   const swapnet_plan* plan = &e->plan;
+  e->zc_ctas = plan->opt.zc_ctas > 0 ? plan->opt.zc_ctas : 32;  // the AUTO choice may lower it
   const uint64_t arena_need = plan->prefix_bytes + plan->region;  // resident prefix, then the swap region
   if (d_arena_user && arena_bytes_user < arena_need) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "arena buffer too small");
   for (const Block& B : plan->blocks)  // every block lies inside the arena
