@@ -320,17 +320,24 @@ def schedule(descs, urgency, arena_bytes, opt=None):
     return list(budgets), [Plan(p) for p in plans]
 
 
-def calibrate(model, plan, engine, reps=20):
+def calibrate(model, plan, engine, reps=20, resident_ns=None):
     """Measured delay model (Sec. 6.1) from a loaded engine: per-layer t_ex
     in ns (sum of the layer's units) and alpha in attoseconds per byte from
-    the per-block copy times measured at load.  Returns (t_ex_ns list,
-    alpha_as_per_byte or None)."""
+    the per-block copy times measured at load.  Each unit is timed alone
+    (a graph of `reps` launches of it); resident_ns, the measured latency of
+    the same model with every weight resident, rescales the t_ex so that
+    they add up to it (the units run as one dependent chain there, with the
+    launch and cache effects that timing a unit alone leaves out).  Returns
+    (t_ex_ns list, alpha_as_per_byte or None)."""
     units = plan.units()
     us = engine.measure_units(len(units), reps)
     t_ex = [0] * len(model["layers"])
     for u, t in zip(units, us):
         t_ex[u["layer"]] += int(round(t * 1000.0))
     t_ex = [max(1, v) for v in t_ex]
+    if resident_ns:
+        f = resident_ns / float(sum(t_ex))
+        t_ex = [max(1, int(round(v * f))) for v in t_ex]
     alpha = None
     blocks = plan.blocks()
     eb = engine.blocks()
