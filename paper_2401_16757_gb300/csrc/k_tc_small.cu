@@ -62,13 +62,56 @@ __device__ __forceinline__ uint32_t bits2(T lo, T hi) {
   return (uint32_t)a | ((uint32_t)b << 16);
 }
 
-// Epilogue of one finished tile: thread t owns row t (TMEM lane t).
+// Epilogue of one finished tile: thread t owns row t (TMEM lane t).  With no
+// residual and 32 or 64 columns left in the slice, each warp passes its 32
+// rows through `stage` (4 KB per warp of the idle A buffer, 16-byte chunks
+// swizzled by row) so that every store instruction writes whole rows (four
+// of 128 bytes, or eight of 64) instead of one 16-byte piece of 32 rows.
 template <typename T>
 __device__ __forceinline__ void small_epilogue(const SmallArgs& p, uint32_t tmem_buf, const float* sbias, int tile,
-                                               int n0) {
-  const int tid = threadIdx.x, warp = tid >> 5;
+                                               int n0, uint32_t stage) {
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int m = tile * kSmBM + tid;
   const T* res = static_cast<const T*>(p.e.res);
+  const int ncols = p.N - n0 >= kSmBN ? kSmBN : (p.N - n0 == 32 ? 32 : 0);
+  if (!res && ncols && ((p.ldy | n0) % 8 == 0)) {
+    const uint32_t wst = stage + (uint32_t)(warp * 32 * 128);
+#pragma unroll 1
+    for (int c0 = 0; c0 < ncols; c0 += 32) {
+      uint32_t r[32];
+      tmem_ld_32x32b_x32(tmem_buf + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, r);
+      tmem_ld_wait();
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        uint32_t o[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int j = 8 * q + 2 * i;
+          const T lo = from_f<T>(epilogue(__uint_as_float(r[j]), sbias[c0 + j], 0.f, 0, p.e.act, p.e.res_post));
+          const T hi = from_f<T>(epilogue(__uint_as_float(r[j + 1]), sbias[c0 + j + 1], 0.f, 0, p.e.act, p.e.res_post));
+          o[i] = bits2<T>(lo, hi);
+        }
+        const uint32_t chunk = (uint32_t)(c0 / 8 + q);
+        st_shared_v4(wst + (uint32_t)lane * 128 + ((chunk ^ (uint32_t)(lane & 7)) << 4),
+                     make_uint4(o[0], o[1], o[2], o[3]));
+      }
+    }
+    __syncwarp();
+    const int m_base = tile * kSmBM + warp * 32;
+    const int cpr_log2 = ncols == kSmBN ? 3 : 2;  // 16-byte chunks per row: 8 or 4
+#pragma unroll 1
+    for (int i = 0; i < (1 << cpr_log2); ++i) {
+      const int row = (i << (5 - cpr_log2)) + (lane >> cpr_log2), chunk = lane & ((1 << cpr_log2) - 1);
+      uint4 v;
+      asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
+                   : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                   : "r"(wst + (uint32_t)row * 128 + (((uint32_t)chunk ^ (uint32_t)(row & 7)) << 4)));
+      if (m_base + row < p.M)
+        *reinterpret_cast<uint4*>(static_cast<T*>(p.y) + (int64_t)(m_base + row) * p.ldy + n0 + chunk * 8) = v;
+    }
+    __syncwarp();
+    return;
+  }
 #pragma unroll 1
   for (int c0 = 0; c0 < kSmBN; c0 += 32) {
     uint32_t r[32];
@@ -201,18 +244,28 @@ __global__ void __launch_bounds__(kSmThreads, 4) tc_conv_small_kernel(const Smal
     const T* xw = X + (((int64_t)img * p.H + iy0) * p.Wd + ix0) * p.C;
     const uint32_t abase = smem_u32(sA + buf * nkb * kSmATile) + row_off;
     for (int kb = 0; kb < nkb; ++kb) {
-      uint32_t e2[32];  // packed pairs: 64 independent loads in flight
+      uint32_t e2[32];  // packed pairs: up to 64 independent loads in flight
 #pragma unroll
-      for (int h = 0; h < 64; h += 2) {
-        T e[2];
+      for (int q = 0; q < 4; ++q) {
+        // 16 k per chunk; a chunk wholly past K (e.g. k 32..63 of a 27-deep
+        // RGB 3x3 stem) is zero without touching the table or the input
+        if (kb * 64 + q * 16 < p.K) {
 #pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          const int2 t = tab[kb * 64 + h + u];
-          const int iy = iy0 + (t.y >> 16), ix = ix0 + (t.y & 0xffff);
-          const bool valid = mv && (unsigned)iy < (unsigned)p.H && (unsigned)ix < (unsigned)p.Wd;
-          e[u] = valid ? __ldg(xw + t.x) : zero;
+          for (int h = q * 16; h < q * 16 + 16; h += 2) {
+            T e[2];
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+              const int2 t = tab[kb * 64 + h + u];
+              const int iy = iy0 + (t.y >> 16), ix = ix0 + (t.y & 0xffff);
+              const bool valid = mv && (unsigned)iy < (unsigned)p.H && (unsigned)ix < (unsigned)p.Wd;
+              e[u] = valid ? __ldg(xw + t.x) : zero;
+            }
+            e2[h >> 1] = bits2<T>(e[0], e[1]);
+          }
+        } else {
+#pragma unroll
+          for (int h = q * 16; h < q * 16 + 16; h += 2) e2[h >> 1] = 0u;
         }
-        e2[h >> 1] = bits2<T>(e[0], e[1]);
       }
 #pragma unroll
       for (int j = 0; j < 8; ++j)
@@ -239,7 +292,8 @@ __global__ void __launch_bounds__(kSmThreads, 4) tc_conv_small_kernel(const Smal
       const bool got = mbar_wait_bounded(bar0 + 8u * pb, ((it - 1) >> 1) & 1, abort_flag, p.err);
       if (__all_sync(0xffffffffu, got)) {  // tcgen05.ld is warp-collective
         tc_fence_after();
-        small_epilogue<T>(p, tmem + (uint32_t)(pb * kSmBN), sbias, tile - (int)gridDim.x, n0);
+        small_epilogue<T>(p, tmem + (uint32_t)(pb * kSmBN), sbias, tile - (int)gridDim.x, n0,
+                          smem_u32(sA + pb * nkb * kSmATile));
       }
       tc_fence_before();
     }
@@ -253,7 +307,8 @@ __global__ void __launch_bounds__(kSmThreads, 4) tc_conv_small_kernel(const Smal
     const bool got = mbar_wait_bounded(bar0 + 8u * pending, (last >> 1) & 1, ok ? abort_flag : &no_abort, p.err);
     if (__all_sync(0xffffffffu, got && ok)) {
       tc_fence_after();
-      small_epilogue<T>(p, tmem + (uint32_t)(pending * kSmBN), sbias, blockIdx.x + last * (int)gridDim.x, n0);
+      small_epilogue<T>(p, tmem + (uint32_t)(pending * kSmBN), sbias, blockIdx.x + last * (int)gridDim.x, n0,
+                        smem_u32(sA + pending * nkb * kSmATile));
     }
   }
   tc_fence_before();
