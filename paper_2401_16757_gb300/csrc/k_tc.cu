@@ -713,9 +713,16 @@ int tc_prepare(const TcGemm& g, TcPlan* p) {
       p->bn = pbn;
       p->splits = 1;
       p->kb_per_split = (g.K + kBK - 1) / kBK;
-      // N tiles of 64 with A by TMA: two 128-row sub-tiles per tile share each
-      // weight stage when that still leaves a tile per SM
-      p->msub = (pbn == 64 && (!g.conv || tmac) && (sp_tiles + 1) / 2 * ((Nd + 63) / 64) >= sms) ? 2 : 1;
+      // N tiles of 64 with A by TMA: four (else two) 128-row sub-tiles per
+      // tile share each weight stage when that still leaves a tile per SM.
+      // Their MMAs go to independent accumulators, which the tensor pipe
+      // overlaps: a single 128x64x16 MMA chain leaves it mostly idle
+      p->msub = 1;
+      if (pbn == 64 && (!g.conv || tmac)) {
+        const int64_t nt64 = (Nd + 63) / 64;
+        if ((sp_tiles + 3) / 4 * nt64 >= sms) p->msub = 4;
+        else if ((sp_tiles + 1) / 2 * nt64 >= sms) p->msub = 2;
+      }
       p->tiles = (sp_tiles + p->msub - 1) / p->msub * ((g.N + pbn - 1) / pbn);
       int rc = make_tmap(&p->tmB, g.dtype, g.W, (uint64_t)g.K, (uint64_t)g.N, (uint64_t)g.K * 2, (uint32_t)pbn);
       if (rc) return rc;

@@ -43,17 +43,20 @@ constexpr int kPBM = 128;
 constexpr int kPBK = 64;  // one 128-byte swizzle row of 16-bit elements
 constexpr int kPA = kPBM * kPBK * 2;
 
-// MS: 128-row sub-tiles per tile sharing each weight stage (1, or 2 for
-// N tiles of 64, where one 128x64 MMA per k16 step is too little work per
-// stage): a tile is then 256 x BN, two accumulators side by side in TMEM.
+// MS: 128-row sub-tiles per tile sharing each weight stage (1, or 2 or 4
+// for N tiles of 64, where one 128x64 MMA chain per k16 step is too little
+// work per stage): a tile is then MS*128 x BN, MS accumulators side by side
+// in TMEM (2 x MS x BN columns with the double buffer: 512 for MS = 4).
 template <int BN, int MS> struct PCfg {
-  static constexpr int kStages = BN == 256 ? 4 : (BN == 128 ? 6 : (MS == 2 ? 5 : 8));
+  static constexpr int kStages = BN == 256 ? 4 : (BN == 128 ? 6 : (MS == 4 ? 3 : (MS == 2 ? 5 : 8)));
   static constexpr int kLag = kStages - 2;  // gather: cp.async groups in flight per thread
   static constexpr int kB = BN * kPBK * 2;
   static constexpr int kSA = MS * kPA;      // A bytes per stage
   static constexpr int kStageBytes = kStages * (kSA + kB);
   static constexpr int kBias = 2 * 4 * BN * 4;  // [buffer][epilogue warp][BN] fp32
   static constexpr int kSmem = kStageBytes + kBias + 256 + 1024;
+  static_assert(kSmem <= 232448, "dynamic shared memory above the 227 KB per-CTA limit");
+  static_assert(2 * MS * BN <= 512, "TMEM holds 512 fp32 columns");
 };
 
 constexpr int kAT2d = 0, kAGather = 1, kATap = 2;
@@ -440,11 +443,19 @@ int launch_persist_inst(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_
 
 template <typename T, int BN>
 int launch_persist_bn(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) {
-  if (BN == 64 && pl.msub == 2) {
-    if (!g.conv) return launch_persist_inst<T, BN, kAT2d, 2>(g, pl, err, s);
-    if (pl.tma_conv) return launch_persist_inst<T, BN, kATap, 2>(g, pl, err, s);
-    SN_FAIL(SWAPNET_ERR_INVALID_ARG, "persistent GEMM: two sub-tiles need A by TMA");
+  if constexpr (BN == 64) {  // sub-tiles only with N tiles of 64
+    if (pl.msub == 4) {
+      if (!g.conv) return launch_persist_inst<T, BN, kAT2d, 4>(g, pl, err, s);
+      if (pl.tma_conv) return launch_persist_inst<T, BN, kATap, 4>(g, pl, err, s);
+      SN_FAIL(SWAPNET_ERR_INVALID_ARG, "persistent GEMM: four sub-tiles need A by TMA");
+    }
+    if (pl.msub == 2) {
+      if (!g.conv) return launch_persist_inst<T, BN, kAT2d, 2>(g, pl, err, s);
+      if (pl.tma_conv) return launch_persist_inst<T, BN, kATap, 2>(g, pl, err, s);
+      SN_FAIL(SWAPNET_ERR_INVALID_ARG, "persistent GEMM: two sub-tiles need A by TMA");
+    }
   }
+  if (pl.msub != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "persistent GEMM: sub-tiles need N tiles of 64");
   if (!g.conv) return launch_persist_inst<T, BN, kAT2d, 1>(g, pl, err, s);
   if (pl.tma_conv) return launch_persist_inst<T, BN, kATap, 1>(g, pl, err, s);
   return launch_persist_inst<T, BN, kAGather, 1>(g, pl, err, s);

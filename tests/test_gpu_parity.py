@@ -63,8 +63,10 @@ def _check_model(m, budget_frac=0.5, slots=2, variant=capi.SWAP_AUTO):
     (3, 1, 32, 128, 112),   # persistent, N tile 128, gather with k-blocks straddling taps
     (1, 1, 64, 300, 112),   # persistent, N tile 256 (ragged), A by TMA
     (3, 2, 64, 256, 224),   # persistent, N tile 256, strided gather
-    (3, 1, 64, 64, 224),    # persistent, N tile 64, two 128-row patches per tile (784 patches)
-    (1, 1, 64, 48, 220),    # persistent 2-D TMA, two sub-tiles per tile, odd m-tile count, N 48
+    (3, 1, 64, 64, 224),    # persistent, N tile 64, four 128-row patches per tile (784 patches)
+    (1, 1, 64, 48, 220),    # persistent 2-D TMA, four sub-tiles per tile, ragged m-tile count, N 48
+    (1, 1, 64, 48, 160),    # persistent 2-D TMA, two sub-tiles per tile (400 m-tiles)
+    (3, 1, 64, 64, 150),    # persistent 4-D TMA, two 32 x 4 patches per tile (380 patches, ragged edge)
     (3, 1, 256, 256, 7),    # deep K, one M tile: split-K with last-CTA reduction
     (3, 1, 64, 24, 9),      # N below one 32-column chunk
     (3, 1, 64, 128, 14),    # few tiles, taps of 64 channels: A by 4-D TMA over 14 x 9 pixel patches
