@@ -58,8 +58,8 @@ CONFIGS = {
 # + dram__bytes_write.sum averaged over the launches of one swapped step of
 # the named workload), valid only for the kernel sources it was taken on.
 TRAFFIC = {
-    ("resnet50", "tc_gemm"): ("8b7980fffdc9", 1418232),
-    ("resnet50", "tc_conv"): ("8b7980fffdc9", 1807714),
+    ("resnet50", "tc_gemm"): ("d6f3d49da751", 1418268),
+    ("resnet50", "tc_conv"): ("d6f3d49da751", 1808496),
 }
 
 
