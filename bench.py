@@ -63,6 +63,45 @@ TRAFFIC = {
 }
 
 
+class RankGroup:
+    """Replicas under torchrun: each rank runs its own engine on its own GPU
+    and nothing crosses ranks on the data path; the group only brackets the
+    timed region with barriers and takes the slowest rank's time.  One rank:
+    no process group, every call is a no-op."""
+
+    def __init__(self, world, local=0, backend="nccl"):
+        self.world = world
+        self.dist = None
+        self.backend = backend
+        if world > 1:
+            import torch
+            import torch.distributed as dist
+            if not dist.is_initialized():
+                if backend == "nccl":
+                    dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+                else:
+                    dist.init_process_group(backend)
+            self.dist = dist
+
+    def barrier(self):
+        if self.dist:
+            self.dist.barrier()
+
+    def max(self, x):
+        """The largest x over the ranks (x on this rank)."""
+        if not self.dist:
+            return float(x)
+        import torch
+        t = torch.tensor([float(x)], dtype=torch.float64, device="cuda" if self.backend == "nccl" else "cpu")
+        self.dist.all_reduce(t, op=self.dist.ReduceOp.MAX)
+        return float(t.item())
+
+    def close(self):
+        if self.dist:
+            self.dist.destroy_process_group()
+            self.dist = None
+
+
 def kernel_sources_sha():
     import hashlib
     h = hashlib.sha1()
@@ -274,7 +313,7 @@ def llm_cpu_sample(n_dec_sample=2):
                    "prefill and %d decode tokens, scaled to 32 layers and 32 decode tokens" % n_dec_sample)
 
 
-def run_llm(args, rank, world):
+def run_llm(args, rank, world, group):
     """Config 5: prefill of 512 ids then 32 greedy decode steps per step."""
     import torch
     import synth
@@ -346,7 +385,9 @@ def run_llm(args, rank, world):
     for e in (ep, ed, rp, rd):
         e.sync()
     launches0 = ep.stats()["kernel_launches"] + ed.stats()["kernel_launches"]
+    group.barrier()
     sw = timed(ep, ed, args.steps)
+    group.barrier()
     launches = ep.stats()["kernel_launches"] + ed.stats()["kernel_launches"] - launches0
     di = timed(rp, rd, args.steps)
     clk = clocks.stop()
@@ -375,7 +416,7 @@ def run_llm(args, rank, world):
     dec_ms = statistics.mean(r[1] for r in sw)
     pre_d = statistics.mean(r[0] for r in di)
     dec_d = statistics.mean(r[1] for r in di)
-    step_ms = pre_ms + n_dec * dec_ms
+    step_ms = group.max(pre_ms + n_dec * dec_ms)  # the slowest rank
     dinf_ms = pre_d + n_dec * dec_d
     swap_bytes_p = sum(b["bytes"] for b in pp.blocks())
     swap_bytes_d = sum(b["bytes"] for b in pd.blocks())
@@ -410,7 +451,7 @@ def run_llm(args, rank, world):
         print(json.dumps(line))
 
 
-def run_multi(args, rank, world):
+def run_multi(args, rank, world, group):
     """Config 4: three models at batch 1, each with its own closed-loop request
     stream on its own CUDA stream, sharing one arena split by Eq. 1
     (swapnet_schedule); DInf is the same concurrent run with every model
@@ -474,7 +515,10 @@ def run_multi(args, rank, world):
     clocks = ClockSampler(int(os.environ.get("LOCAL_RANK", "0")))
     clocks.start()
     launches0 = sum(e.stats()["kernel_launches"] for e in engs)
+    group.barrier()
     lat_sw, wall_sw = run(engs, args.steps)
+    group.barrier()
+    wall_sw = group.max(wall_sw)  # the slowest rank
     launches = sum(e.stats()["kernel_launches"] for e in engs) - launches0
     lat_di, wall_di = run(rengs, args.steps)
     clk = clocks.stop()
@@ -492,7 +536,7 @@ def run_multi(args, rank, world):
                         "ms_swapped": sw, "ms_dinf": di, "ratio": sw / di,
                         "p50_swapped": statistics.median(lat_sw[k]), "p50_dinf": statistics.median(lat_di[k])}
     line = {
-        "metric": METRIC, "value": n_req / (wall_sw * 1e-3), "unit": "inferences/s (3 models, concurrent)",
+        "metric": METRIC, "value": world * n_req / (wall_sw * 1e-3), "unit": "inferences/s (3 models, concurrent)",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": wall_sw / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f16", "data": "synthetic",
         "config": {"workload": CONFIGS["multi"][3], "arena_bytes": arena, "weight_bytes": sum(wbs),
@@ -892,17 +936,16 @@ def main():
     if args.config in ("llm", "multi"):
         import torch
         torch.cuda.set_device(local)
+        group = RankGroup(world, local)
         import __graft_entry__
         __graft_entry__.build()
-        (run_llm if args.config == "llm" else run_multi)(args, rank, world)
+        (run_llm if args.config == "llm" else run_multi)(args, rank, world, group)
+        group.close()
         return
 
     import torch
     torch.cuda.set_device(local)
-    dist = None
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    group = RankGroup(world, local)
 
     import __graft_entry__
     __graft_entry__.build()
@@ -974,8 +1017,7 @@ def main():
     # ---- timed region: swapped inference
     clocks = ClockSampler(local)
     clocks.start()
-    if dist:
-        dist.barrier()
+    group.barrier()
     torch.cuda.synchronize()
     launches0 = eng.stats()["kernel_launches"]
     t_wall0 = time.perf_counter()
@@ -984,15 +1026,10 @@ def main():
     torch.cuda.nvtx.range_pop()
     t_wall = time.perf_counter() - t_wall0
     launches = eng.stats()["kernel_launches"] - launches0
-    if dist:
-        dist.barrier()
+    group.barrier()
     eng.sync()
     ms_swapped = sum(ms_list) / len(ms_list)
-    total_ms = sum(ms_list)
-    if dist:
-        t = torch.tensor([total_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = group.max(sum(ms_list))  # the slowest rank
     value = world * args.steps / (total_ms / 1000.0)
 
     # ---- DInf: same kernels, weights resident
@@ -1164,8 +1201,7 @@ def main():
             "wall_s_timed": t_wall,
         }
         print(json.dumps(line))
-    if dist:
-        dist.destroy_process_group()
+    group.close()
 
 
 if __name__ == "__main__":

@@ -55,3 +55,41 @@ def test_reference_arm_prints_one_oracle_line():
     assert line["cpu_baseline"]["kind"] == "oracle"
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["d2h_bytes_per_step"] == 0
     assert line["value"] > 0 and line["unit"] == line["e2e"]["unit"]
+
+
+def _rank_group_worker(rank, port, out_dir):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE="2")
+    sys.path.insert(0, ROOT)
+    import bench as b
+    g = b.RankGroup(2, backend="gloo")
+    g.barrier()
+    slowest = g.max(10.0 + 5.0 * rank)  # this rank's "timed" milliseconds
+    g.barrier()
+    g.close()
+    with open(os.path.join(out_dir, "rank%d" % rank), "w") as fh:
+        fh.write(repr(slowest))
+
+
+def test_rank_group_takes_the_slowest_rank_over_gloo(tmp_path):
+    """Replicas (N > 1): two ranks on the CPU (gloo) bracket the timed region
+    with barriers and both see the slowest rank's time, from which bench.py
+    computes the whole-job throughput; one rank needs no process group."""
+    import socket
+    import torch.multiprocessing as mp
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        port = s.getsockname()[1]
+    mp.spawn(_rank_group_worker, args=(port, str(tmp_path)), nprocs=2, join=True)
+    got = [float(open(os.path.join(str(tmp_path), "rank%d" % r)).read()) for r in range(2)]
+    assert got == [15.0, 15.0]
+    single = bench.RankGroup(1)
+    assert single.max(3.5) == 3.5 and single.dist is None
+    single.barrier()
+    single.close()
+
+
+def test_reference_arm_other_ranks_exit_quietly():
+    env = dict(os.environ, RANK="1", WORLD_SIZE="2", LOCAL_RANK="1")
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--config", "mlp6",
+                        "--steps", "1", "--warmup", "0"], capture_output=True, text=True, timeout=600, env=env)
+    assert r.returncode == 0 and r.stdout.strip() == ""
