@@ -560,6 +560,15 @@ const char* swapnet_last_error(void);
  * 2 = device allocation, 3 = event/stream creation.  count 0 disarms. */
 int swapnet_debug_fail_next(int what, int count);
 
+/* Failure-detection check for tests: launches on `stream` one kernel whose
+ * bounded device wait (the wait every kernel of the library uses on its
+ * mbarriers) waits on an mbarrier that nothing completes, so it gives up
+ * after the wait limit (one second), records the timeout in the library's
+ * device error word and returns; no trap, no fault, the context stays
+ * usable.  Synchronises the stream, reads and clears the error word, and
+ * returns what swapnet_engine_sync would: SWAPNET_ERR_TIMEOUT. */
+int swapnet_debug_wait_timeout(swapnet_stream stream);
+
 #ifdef __cplusplus
 }
 #endif

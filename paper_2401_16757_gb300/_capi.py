@@ -101,7 +101,8 @@ EXPORTS = ["swapnet_default_options", "swapnet_partition", "swapnet_plan_from_cu
            "swapnet_engine_last_timeline",
            "swapnet_engine_bind_state", "swapnet_strerror", "swapnet_last_error", "swapnet_debug_fail_next", "swapnet_gemm_noalloc",
            "swapnet_weights_file_write", "swapnet_weights_file_open", "swapnet_weights_file_info",
-           "swapnet_weights_file_read", "swapnet_weights_file_close", "swapnet_load_file"]
+           "swapnet_weights_file_read", "swapnet_weights_file_close", "swapnet_load_file",
+           "swapnet_debug_wait_timeout"]
 
 _lib = None
 
@@ -166,6 +167,7 @@ def lib():
         "swapnet_weights_file_read": (C.c_int, [P, C.c_uint32, C.c_uint64, C.c_uint64, P]),
         "swapnet_weights_file_close": (None, [P]),
         "swapnet_load_file": (C.c_int, [P, P, P, C.c_uint64, P, C.c_uint64, C.POINTER(P)]),
+        "swapnet_debug_wait_timeout": (C.c_int, [P]),
     }
     for name, (res, args) in sig.items():
         f = getattr(L, name)

@@ -409,3 +409,26 @@ def test_driver_pinned_host_weights():
     a = Runner(m, w, capi.Plan.partition(d, budget, capi.options()), host).run(x)
     b = Runner(m, w, capi.Plan.resident(d), capi.HostWeights(w)).run(x)
     assert all(p.tobytes() == q.tobytes() for p, q in zip(a, b))
+
+
+def test_device_wait_timeout_is_reported_and_the_context_stays_usable():
+    """Failure detection on the GPU without a fault: a kernel's bounded wait
+    on an mbarrier that nothing completes gives up after its limit, the
+    library reports SWAPNET_ERR_TIMEOUT once, and inference afterwards gives
+    the resident bits again."""
+    import torch
+    m = synth.arch.resnet50()
+    w = synth.gen.model_weights(m)
+    x = synth.gen.model_input(m)
+    d = capi.Desc(m)
+    host = capi.HostWeights(w)
+    rs = Runner(m, w, capi.Plan.resident(d), host)
+    before = rs.run(x)
+    rc = capi.lib().swapnet_debug_wait_timeout(capi.C.c_void_p(torch.cuda.current_stream().cuda_stream))
+    assert rc == capi.ERR_TIMEOUT
+    assert capi.lib().swapnet_debug_wait_timeout(None) == capi.ERR_TIMEOUT  # the legacy stream too
+    budget = int(OP.weight_bytes(m) * 0.4) // 256 * 256
+    sw = Runner(m, w, capi.Plan.partition(d, budget, capi.options()), host)
+    for a, b in zip(sw.run(x), before):
+        assert a.tobytes() == b.tobytes()
+    rs.engine.sync()  # the error word was cleared: no stale timeout
