@@ -432,3 +432,24 @@ def test_device_wait_timeout_is_reported_and_the_context_stays_usable():
     for a, b in zip(sw.run(x), before):
         assert a.tobytes() == b.tobytes()
     rs.engine.sync()  # the error word was cleared: no stale timeout
+
+
+@pytest.mark.parametrize("what,code", [(1, capi.ERR_CUDA), (2, capi.ERR_OOM), (3, capi.ERR_CUDA)])
+def test_injected_load_failures_leave_nothing_behind(what, code):
+    """Host-side fault injection at load (registration, device allocation,
+    stream creation): swapnet_load fails with the matching status, releases
+    what it had set up, and the next load of the same weights works."""
+    m = synth.arch.resnet50()
+    w = synth.gen.model_weights(m)
+    x = synth.gen.model_input(m)
+    d = capi.Desc(m)
+    host = capi.HostWeights(w)
+    plan = capi.Plan.partition(d, int(OP.weight_bytes(m) * 0.4) // 256 * 256, capi.options())
+    assert capi.lib().swapnet_debug_fail_next(what, 1) == capi.OK
+    with pytest.raises(capi.SwapnetError) as ei:
+        capi.Engine(plan, host)
+    assert ei.value.code == code, str(ei.value)
+    assert capi.lib().swapnet_debug_fail_next(what, 0) == capi.OK
+    got = Runner(m, w, plan, host).run(x)
+    ref = Runner(m, w, capi.Plan.resident(d), host).run(x)
+    assert all(a.tobytes() == b.tobytes() for a, b in zip(got, ref))
