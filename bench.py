@@ -395,6 +395,32 @@ def run_llm(args, rank, world, group):
     # greedy tokens agree between swapped and resident runs
     one(ep, ed); torch.cuda.synchronize(); sw_tok = int(tok[:4].cpu().numpy().view(np.int32)[0])
     one(rp, rd); torch.cuda.synchronize(); rs_tok = int(tok[:4].cpu().numpy().view(np.int32)[0])
+    # e2e through swapnet_infer_host: the token ids from pinned host memory,
+    # every pass's output back to the host, and each greedy token taken from
+    # the host copy for the next decode pass
+    h_ids = torch.from_numpy(ids.view(np.uint8).copy()).pin_memory()
+    h_out_p = torch.empty(ip["output_bytes"], dtype=torch.uint8).pin_memory()
+    h_tok = torch.zeros(16, dtype=torch.uint8).pin_memory()
+    h_out_d = torch.empty(idd["output_bytes"], dtype=torch.uint8).pin_memory()
+
+    def one_host():
+        state[:256].zero_()
+        ep.infer_host(h_ids.data_ptr(), h_out_p.data_ptr(), sp)
+        stream.synchronize()
+        h_tok[:4].copy_(h_out_p[offs_p[1] + 511 * 4:offs_p[1] + 512 * 4])
+        for _ in range(n_dec):
+            ed.infer_host(h_tok.data_ptr(), h_out_d.data_ptr(), sp)
+            stream.synchronize()
+            h_tok[:4].copy_(h_out_d[offs_d[1]:offs_d[1] + 4])
+
+    one_host()
+    e2e_ms = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        one_host()
+        e2e_ms.append((time.perf_counter() - t0) * 1e3)
+    e2e_step_ms = group.max(statistics.mean(e2e_ms))
+    e2e_tok_equal = int(h_tok[:4].numpy().view(np.int32)[0]) == sw_tok
     # extension (not the paper's method): resident-prefix plans in the same budget
     opt_rp = capi.options(swap_variant=variant, alpha_as_per_byte=alpha, beta_ns_per_tensor=0, resident_prefix=1)
     pp_rp, pd_rp = capi.Plan.partition(dp, budget, opt_rp), capi.Plan.partition(dd, budget, opt_rp)
@@ -433,6 +459,10 @@ def run_llm(args, rank, world, group):
         "prefill_ms": pre_ms, "decode_ms_per_token": dec_ms, "dinf_prefill_ms": pre_d,
         "dinf_decode_ms_per_token": dec_d, "dinf_ms": dinf_ms, "ratio": step_ms / dinf_ms,
         "greedy_token_swapped_equals_resident": sw_tok == rs_tok,
+        "e2e": {"value": world * 1000.0 / e2e_step_ms, "unit": "inferences/s (prefill 512 + 32 decode)",
+                "h2d_bytes_per_step": ip["input_bytes"] + n_dec * idd["input_bytes"],
+                "d2h_bytes_per_step": ip["output_bytes"] + n_dec * idd["output_bytes"],
+                "greedy_token_equals_device_run": e2e_tok_equal},
         "link": {"achieved_gbs": bytes_step / (step_ms * 1e-3) / 1e9, "peak_gbs": link_peak,
                  "peak_source": "pinned cudaMemcpy H2D 256 MiB", "bytes_per_step": bytes_step,
                  "peak_before_after_gbs": [link_before, link_after]},
@@ -521,6 +551,28 @@ def run_multi(args, rank, world, group):
     wall_sw = group.max(wall_sw)  # the slowest rank
     launches = sum(e.stats()["kernel_launches"] for e in engs) - launches0
     lat_di, wall_di = run(rengs, args.steps)
+    # e2e through swapnet_infer_host: each request's input from pinned host
+    # memory and its output back, the three models concurrently on their
+    # streams; wall time of all requests
+    h_ins, h_outs = [], []
+    for m, inf in zip(ms, infos):
+        x8 = synth.gen.model_input(m).view(np.uint8).reshape(-1)
+        h_in = torch.empty(inf["input_bytes"], dtype=torch.uint8, pin_memory=True)
+        h_in.copy_(torch.from_numpy(x8[:inf["input_bytes"]]))
+        h_ins.append(h_in)
+        h_outs.append(torch.empty(inf["output_bytes"], dtype=torch.uint8, pin_memory=True))
+
+    def run_host(steps):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(steps):
+            for k, e in enumerate(engs):
+                e.infer_host(h_ins[k].data_ptr(), h_outs[k].data_ptr(), streams[k].cuda_stream)
+        torch.cuda.synchronize()
+        return (time.perf_counter() - t0) * 1e3
+
+    run_host(args.warmup)
+    wall_e2e = group.max(run_host(args.steps))
     clk = clocks.stop()
     for e in engs:
         e.sync()
@@ -544,6 +596,9 @@ def run_multi(args, rank, world, group):
                    "l2": "no flush: 451.6 MB of weights stream through the arena every round"},
         "per_model": per_model,
         "dinf_ms_per_step": wall_di / args.steps, "throughput_ratio": wall_sw / wall_di,
+        "e2e": {"value": world * n_req / (wall_e2e * 1e-3), "unit": "inferences/s (3 models, concurrent)",
+                "h2d_bytes_per_step": sum(i["input_bytes"] for i in infos),
+                "d2h_bytes_per_step": sum(i["output_bytes"] for i in infos)},
         "link": {"achieved_gbs": swap_bytes * args.steps / (wall_sw * 1e-3) / 1e9, "peak_gbs": link_peak,
                  "peak_source": "pinned cudaMemcpy H2D 256 MiB", "bytes_per_step": swap_bytes},
         "step_roofline": {"bound": "host link" if swap_bytes / (link_peak * 1e9) > flops / (tf_burst * 1e12)
