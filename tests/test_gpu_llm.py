@@ -35,6 +35,7 @@ class Decoder:
         import torch
         self.torch = torch
         cfg = dict(SMALL, layers=layers, **over)
+        self.vocab = cfg["vocab"]
         self.mp = synth.arch.llm(tokens=prefill_tokens, **cfg)
         self.md = synth.arch.llm(tokens=1, **cfg)
         self.w = weights or synth.gen.model_weights(self.mp)
@@ -65,7 +66,7 @@ class Decoder:
         eng.sync()
         host = dout.cpu().numpy()
         t = ids.size
-        v = SMALL["vocab"]
+        v = self.vocab
         logits = host[offs[0]:offs[0] + t * v * 2].view(np.uint16).reshape(t, v)
         tokens = host[offs[1]:offs[1] + t * 4].view(np.int32).copy()
         return logits, tokens
@@ -101,6 +102,44 @@ def test_llm_prefill_and_greedy_decode_teacher_forced(layers):
 
 
 WIDE = dict(layers=1, d=1024, heads=8, ffn=2752, max_seq=160)
+# the 7B workload's widths (one decoder layer of the 32): d 4096, 32 heads,
+# FFN 11008, vocabulary 32000, a 512-token prefill
+FULL = dict(layers=1, d=4096, heads=32, ffn=11008, vocab=32000, max_seq=544)
+
+
+def _weights_parallel(model):
+    """synth.gen.model_weights, one tensor per thread (the same seeded
+    streams; the generators release the GIL on large draws)."""
+    import concurrent.futures as cf
+    jobs = [(li, ti, shp) for li, L in enumerate(model["layers"])
+            for ti, (_, shp) in enumerate(synth.arch.tensor_shapes(L))]
+    with cf.ThreadPoolExecutor(max_workers=16) as ex:
+        out = list(ex.map(lambda j: synth.gen.llm_tensor(model, *j), jobs))
+    w = [[] for _ in model["layers"]]
+    for (li, _, _), t in zip(jobs, out):
+        w[li].append(t)
+    return w
+
+
+def test_llm_full_width_layer_prefill_512_and_decode():
+    """The bench's launch configuration at full width on one decoder layer
+    (the float64 oracle of all 32 layers would need 54 GB): 512-token
+    prefill and two greedy decode passes, swapped through a budget of half
+    the weight bytes, against the oracle teacher-forced."""
+    mp = synth.arch.llm(tokens=512, **dict(SMALL, **FULL))
+    dec = Decoder(prefill_tokens=512, budget_frac=0.5, weights=_weights_parallel(mp), **FULL)
+    ids = synth.gen.model_input(dec.mp).reshape(-1)
+    st = F.new_state()
+    ref = F.forward(dec.mp, dec.w, ids.reshape(-1, 1, 1, 1), state=st)
+    logits, toks = dec.run(0, ids)
+    _check_step(logits, toks, ref[0].reshape(512, -1), ref[1].reshape(-1), CHAIN_TOL)
+    tok = int(toks[-1])
+    for step in range(2):
+        ref = F.forward(dec.md, dec.w, np.array([tok], dtype=np.int32).reshape(1, 1, 1, 1), state=st)
+        logits, toks = dec.run(1, np.array([tok], dtype=np.int32))
+        _check_step(logits, toks, ref[0].reshape(1, -1), ref[1].reshape(-1), CHAIN_TOL)
+        tok = int(toks[0])
+    assert int(dec.state[:4].cpu().numpy().view(np.int32)[0]) == 512 + 2
 
 
 def test_llm_long_prefill_many_heads():
