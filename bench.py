@@ -54,6 +54,15 @@ CONFIGS = {
 }
 
 
+# swap variants by name (--variant); "direct" reads SIMT-only blocks in place
+VARIANTS = ("auto", "memcpy", "zerocopy", "direct")
+
+
+def variant_code(name):
+    from paper_2401_16757_gb300 import capi
+    return {"auto": capi.SWAP_AUTO, "memcpy": capi.SWAP_MEMCPY, "zerocopy": capi.SWAP_ZEROCOPY,
+            "direct": capi.SWAP_DIRECT}[name]
+
 # DRAM traffic per launch of a kernel family, from ncu (dram__bytes_read.sum
 # + dram__bytes_write.sum averaged over the launches of one swapped step of
 # the named workload), valid only for the kernel sources it was taken on.
@@ -328,7 +337,7 @@ def run_llm(args, rank, world, group):
     link_peak = measure_link_peak(stream)
     alpha = int(round(1e18 / (link_peak * 1e9)))
     budget = 4_000_000_000
-    variant = {"auto": capi.SWAP_AUTO, "memcpy": capi.SWAP_MEMCPY, "zerocopy": capi.SWAP_ZEROCOPY}[args.variant]
+    variant = variant_code(args.variant)
     opt = capi.options(swap_variant=variant, alpha_as_per_byte=alpha, beta_ns_per_tensor=0)
     dp, dd = capi.Desc(mp), capi.Desc(md)
     t1 = time.perf_counter()
@@ -496,7 +505,7 @@ def run_multi(args, rank, world, group):
     # the three pipelines share one host link: each model's delay model takes
     # its share of the measured bandwidth (--link-share 1 plans as if alone)
     alpha = int(round(1e18 / (link_peak * 1e9 / args.link_share)))
-    variant = {"auto": capi.SWAP_AUTO, "memcpy": capi.SWAP_MEMCPY, "zerocopy": capi.SWAP_ZEROCOPY}[args.variant]
+    variant = variant_code(args.variant)
     opt = capi.options(swap_variant=variant, alpha_as_per_byte=alpha, beta_ns_per_tensor=0, eta_ns_per_tensor=0)
     descs = [capi.Desc(m) for m in ms]
     wbs = [capi_weight_bytes(m) for m in ms]
@@ -952,7 +961,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="swapnet", choices=["swapnet", "reference"])
     ap.add_argument("--config", default="resnet50", choices=sorted(CONFIGS))
-    ap.add_argument("--variant", default="auto", choices=["auto", "memcpy", "zerocopy"])
+    ap.add_argument("--variant", default="auto", choices=VARIANTS)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--link-share", type=float, default=1.0,
                     help="multi: models sharing the host link in each model's delay model")
@@ -1008,7 +1017,7 @@ def main():
 
     m, w, x, wb, budget, text = build_workload(args.config, capi_weight_bytes)
     d = capi.Desc(m)
-    variant = {"auto": capi.SWAP_AUTO, "memcpy": capi.SWAP_MEMCPY, "zerocopy": capi.SWAP_ZEROCOPY}[args.variant]
+    variant = variant_code(args.variant)
     act_in = 1 if args.config == "mlp6" else 0
     opt0 = capi.options(slots=2, activations_in_budget=act_in, swap_variant=variant)
     host = capi.HostWeights(w)

@@ -128,7 +128,13 @@ typedef struct swapnet_model_desc {
 typedef enum swapnet_swap_variant {
   SWAPNET_SWAP_AUTO = 0,     /* pick per block by measured time at load        */
   SWAPNET_SWAP_MEMCPY = 1,   /* copy engine: cudaMemcpyAsync from pinned memory */
-  SWAPNET_SWAP_ZEROCOPY = 2  /* SM kernel reading mapped host memory           */
+  SWAPNET_SWAP_ZEROCOPY = 2, /* SM kernel reading mapped host memory           */
+  SWAPNET_SWAP_DIRECT = 3    /* no swap-in: the block's kernels read their
+                                parameters in mapped host memory themselves
+                                (copy-free dispatch, Sec. 4.2.2, taken to the
+                                kernels); for blocks whose units all run SIMT
+                                kernels (GEMV, norms, attention, pools), other
+                                blocks take MEMCPY.  Never chosen by AUTO.    */
 } swapnet_swap_variant;
 
 /* Options.  Delay coefficients follow Sec. 6.1: t_in = alpha*s + beta*d,
@@ -428,9 +434,11 @@ typedef struct swapnet_engine_block {
 
 int swapnet_engine_blocks(const swapnet_engine* eng, swapnet_engine_block* blocks, uint32_t cap,
                           uint32_t* n);
-/* Counters since load (kernel launches include the layer kernels and the
- * zero-copy swap kernels the engine launched; memcpy_calls counts copy-engine
- * transfers). */
+/* Counters of the inferences since load: kernel launches include the layer
+ * kernels and the zero-copy swap kernels; memcpy_calls counts copy-engine
+ * transfers and bytes_swapped the bytes moved into the arena (uploads at
+ * load time excluded; a block read in place, SWAPNET_SWAP_DIRECT, adds
+ * nothing). */
 typedef struct swapnet_engine_stats {
   uint64_t infer_calls;
   uint64_t kernel_launches;

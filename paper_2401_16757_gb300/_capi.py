@@ -23,7 +23,7 @@ OP = {"linear": 1, "conv": 2, "maxpool": 3, "gap": 4, "upsample2x": 5, "concat":
 ACT = {"none": 0, "relu": 1, "leaky": 2, "swiglu": 3}
 DTYPE = {"f32": F32, "f16": F16, "bf16": BF16, "i32": I32}
 LAYER_NO_BIAS = 1
-SWAP_AUTO, SWAP_MEMCPY, SWAP_ZEROCOPY = 0, 1, 2
+SWAP_AUTO, SWAP_MEMCPY, SWAP_ZEROCOPY, SWAP_DIRECT = 0, 1, 2, 3
 SRC_INPUT, SRC_NONE = -1, -2
 
 

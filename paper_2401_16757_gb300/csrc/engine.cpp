@@ -455,18 +455,32 @@ static int swap_block(swapnet_engine* e, size_t k, int variant, cudaStream_t s) 
   if (variant == SWAPNET_SWAP_ZEROCOPY) {
     std::vector<ZcSeg> z;
     z.reserve(b.segs.size());
-    for (const Segment& g : b.segs) {
-      z.push_back(ZcSeg{g.src, g.dst, g.bytes});
-      e->stats.bytes_swapped += g.bytes;
-    }
+    for (const Segment& g : b.segs) z.push_back(ZcSeg{g.src, g.dst, g.bytes});
     return launch_zerocopy(z.data(), (int)z.size(), e->zc_ctas, s);
   }
-  for (const Segment& g : b.segs) {
-    CU(cudaMemcpyAsync(g.dst, g.src, g.bytes, cudaMemcpyDefault, s), "swap-in copy");
-    e->stats.bytes_swapped += g.bytes;
-    e->stats.memcpy_calls += 1;
-  }
+  for (const Segment& g : b.segs) CU(cudaMemcpyAsync(g.dst, g.src, g.bytes, cudaMemcpyDefault, s), "swap-in copy");
   return SWAPNET_OK;
+}
+
+static bool wants_tc(const Model& m, const Layer& L);
+static bool small_conv_ok(const Model& m, const Layer& L);
+
+// A block runs without a swap-in (SWAPNET_SWAP_DIRECT) when every unit
+// with parameters runs a SIMT kernel, which takes plain 16-byte global loads
+// that reach mapped host memory as well as the arena; tensor-core units read
+// their weights by TMA from device memory and keep the swap.
+static bool direct_ok(const swapnet_engine* e, size_t k) {
+  const swapnet_plan& p = e->plan;
+  const Block& B = p.blocks[k];
+  for (int u = B.u0; u < B.u1; ++u) {
+    const Unit& U = p.units[u];
+    if (U.host) continue;
+    const Layer& L = p.model.L[U.layer];
+    if (U.nt > 0 && (wants_tc(p.model, L) || small_conv_ok(p.model, L))) return false;
+    for (int t = 0; t < U.nt; ++t)
+      if ((uintptr_t)(e->tensor_dev[U.tidx[t]] + U.toff[t]) & 15) return false;
+  }
+  return true;
 }
 
 static bool zerocopy_ok(const EngBlock& b) {
@@ -707,6 +721,10 @@ static int prepare_units(swapnet_engine* e) {
       UnitExec& X = e->ux[u];
       if (U.host) {
         X.w = e->tensor_dev[U.tidx[0]];  // device alias of the page-locked host table
+      } else if (e->blocks[&B - p.blocks.data()].variant == SWAPNET_SWAP_DIRECT) {
+        // read in place in page-locked host memory (device aliases)
+        if (U.nt >= 1) X.w = e->tensor_dev[U.tidx[0]] + U.toff[0];
+        if (U.nt == 2) X.b = e->tensor_dev[U.tidx[1]] + U.toff[1];
       } else {
         if (U.nt >= 1) X.w = base + U.slot_off[0];
         if (U.nt == 2) X.b = base + U.slot_off[1];
@@ -845,6 +863,9 @@ static int bind_plan(swapnet_engine* e, void* d_arena_user, uint64_t arena_bytes
   }
   int rc = build_segments(e);
   if (rc) return rc;
+  if (!plan->resident && !e->file && plan->opt.swap_variant == SWAPNET_SWAP_DIRECT)
+    for (size_t k = 0; k < e->blocks.size(); ++k)
+      if (plan->blocks[k].slot >= 0 && direct_ok(e, k)) e->blocks[k].variant = SWAPNET_SWAP_DIRECT;
   rc = prepare_units(e);
   if (rc) return rc;
   rc = plan_side(e);
@@ -899,6 +920,10 @@ static int bind_plan(swapnet_engine* e, void* d_arena_user, uint64_t arena_bytes
   } else if (!plan->resident) {
     for (size_t k = 0; k < e->blocks.size(); ++k) {
       EngBlock& b = e->blocks[k];
+      if (variant == SWAPNET_SWAP_DIRECT) {  // the blocks direct_ok refused are copied
+        if (b.variant != SWAPNET_SWAP_DIRECT) b.variant = SWAPNET_SWAP_MEMCPY;
+        continue;
+      }
       b.variant = variant;
       if (plan->blocks[k].slot >= 0 && variant == SWAPNET_SWAP_ZEROCOPY && !zerocopy_ok(b))
         SN_FAIL(SWAPNET_ERR_MISALIGNED, "zero-copy needs 16-byte aligned host tensors");
@@ -1117,8 +1142,15 @@ static int plan_side(swapnet_engine* e) {
 
 // First-block prefetch is on for swapped plans made with option prefetch
 // (the planner allows it only with two slots and no resident prefix).
+// Block k is copied into its slot for every inference (not resident, not
+// part of a resident prefix, not read in place in host memory).
+static bool swapped(const swapnet_engine* e, size_t k) {
+  return !e->plan.resident && e->plan.blocks[k].slot >= 0 &&
+         (k >= e->blocks.size() || e->blocks[k].variant != SWAPNET_SWAP_DIRECT);
+}
+
 static bool prefetch_on(const swapnet_engine* e) {
-  return !e->plan.resident && e->plan.opt.prefetch && !e->plan.blocks.empty() && e->plan.blocks[0].slot == 0;
+  return e->plan.opt.prefetch && !e->plan.blocks.empty() && e->plan.blocks[0].slot == 0 && swapped(e, 0);
 }
 
 static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t s, bool capturing = false) {
@@ -1167,8 +1199,8 @@ static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t 
   };
   for (size_t k = 0; k < p.blocks.size(); ++k) {
     const Block& B = p.blocks[k];
-    const bool swapped = !p.resident && B.slot >= 0;  // a resident prefix stays in the arena
-    if (swapped) {
+    const bool swap_k = swapped(e, k);  // a resident prefix stays in the arena
+    if (swap_k) {
       if (pf && k == 0) {
         used[B.slot] = true;  // swapped in at the end of the previous inference (or at load)
       } else {
@@ -1193,7 +1225,7 @@ static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t 
         CU(cudaEventRecord(e->side_done[w], e->side), "record side done");
       }
     }
-    if (swapped) CU(cudaEventRecord(e->slot_free[B.slot], s), "record slot free");
+    if (swap_k) CU(cudaEventRecord(e->slot_free[B.slot], s), "record slot free");
   }
   if (p.model.has_attention) {
     if (!e->d_state) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "decoder state not bound (swapnet_engine_bind_state)");
@@ -1282,6 +1314,11 @@ int swapnet_infer(swapnet_engine* e, const void* din, void* dout, swapnet_stream
   }
   e->stats.kernel_launches += launches_per_infer(e);
   e->stats.infer_calls += 1;
+  for (size_t k = 0; k < e->blocks.size(); ++k) {  // every swapped block once per inference
+    if (!swapped(e, k)) continue;
+    for (const Segment& g : e->blocks[k].segs) e->stats.bytes_swapped += g.bytes;
+    if (e->blocks[k].variant != SWAPNET_SWAP_ZEROCOPY) e->stats.memcpy_calls += e->blocks[k].segs.size();
+  }
   return SWAPNET_OK;
 }
 
@@ -1453,7 +1490,7 @@ int swapnet_engine_last_times(swapnet_engine* e, float* unit_us, uint32_t nu, fl
   }
   for (uint32_t k = 0; swap_us && k < nb && k < e->plan.blocks.size(); ++k) {
     float ms = 0.f;
-    if (!e->plan.resident && e->plan.blocks[k].slot >= 0)  // a resident prefix is never swapped
+    if (swapped(e, k))  // a resident prefix and a block read in host memory are never swapped
       CU(cudaEventElapsedTime(&ms, e->ev_swap[2 * k], e->ev_swap[2 * k + 1]), "elapsed");
     swap_us[k] = ms * 1000.f;
   }
@@ -1469,7 +1506,7 @@ int swapnet_engine_last_timeline(swapnet_engine* e, float* us0, float* us1, uint
   // first block swapped at the start (a resident prefix has no swap events;
   // with first-block prefetch block 0's swap comes at the end)
   size_t k0 = swapnet::prefetch_on(e) ? 1 : 0;
-  while (k0 < e->plan.blocks.size() && e->plan.blocks[k0].slot < 0) ++k0;
+  while (k0 < e->plan.blocks.size() && !swapnet::swapped(e, k0)) ++k0;
   const bool sw = !e->plan.resident && !e->ev_swap.empty() && k0 < e->plan.blocks.size();
   cudaEvent_t origin = sw ? e->ev_swap[2 * k0] : e->ev_unit[0];
   float first = 0.f;
@@ -1489,7 +1526,7 @@ int swapnet_engine_last_timeline(swapnet_engine* e, float* us0, float* us1, uint
     if (us1 && rel(e->ev_unit[2 * u + 1], &us1[u])) return SWAPNET_ERR_CUDA;
   }
   for (uint32_t k = 0; k < nb && k < e->plan.blocks.size(); ++k) {
-    if (!sw || e->plan.blocks[k].slot < 0) {
+    if (!sw || !swapnet::swapped(e, k)) {
       if (ss0) ss0[k] = 0.f;
       if (ss1) ss1[k] = 0.f;
       continue;

@@ -174,6 +174,23 @@ def test_prefetch_partition_equals_exhaustive_oracle():
     assert checked >= 10
 
 
+def test_swap_variant_range():
+    """AUTO, MEMCPY, ZEROCOPY and DIRECT are the variants a plan accepts; the
+    variant changes what the engine does, not the partition."""
+    m = _random_model(np.random.default_rng(4), 6)
+    desc = capi.Desc(m)
+    budget = P.weight_bytes(m) // 256 * 256
+    cuts = None
+    for v in (capi.SWAP_AUTO, capi.SWAP_MEMCPY, capi.SWAP_ZEROCOPY, capi.SWAP_DIRECT):
+        got = capi.Plan.partition(desc, budget, capi.options(swap_variant=v)).cuts()
+        assert cuts is None or got == cuts
+        cuts = got
+    for bad in (-1, 4):
+        with pytest.raises(capi.SwapnetError) as ei:
+            capi.Plan.partition(desc, budget, capi.options(swap_variant=bad))
+        assert ei.value.code == capi.ERR_INVALID_ARG
+
+
 def test_prefetch_options_and_wrap_pair_are_checked():
     m = _random_model(np.random.default_rng(9), 5)
     desc = capi.Desc(m)

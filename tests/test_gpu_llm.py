@@ -31,7 +31,7 @@ class Decoder:
     """A prefill engine and a decode engine sharing weights and KV state."""
 
     def __init__(self, prefill_tokens, budget_frac=0.5, resident=False, host=None, weights=None, layers=2,
-                 **over):
+                 opts=None, **over):
         import torch
         self.torch = torch
         cfg = dict(SMALL, layers=layers, **over)
@@ -44,7 +44,7 @@ class Decoder:
         self.engines, self.bufs = [], []
         for m in (self.mp, self.md):
             d = capi.Desc(m)
-            plan = capi.Plan.resident(d) if resident else capi.Plan.partition(d, budget, capi.options())
+            plan = capi.Plan.resident(d) if resident else capi.Plan.partition(d, budget, capi.options(**(opts or {})))
             eng = capi.Engine(plan, self.host)
             info = plan.info()
             din = torch.zeros(max(16, info["input_bytes"]), dtype=torch.uint8, device="cuda")
