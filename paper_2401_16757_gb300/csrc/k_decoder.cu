@@ -53,29 +53,94 @@ __global__ void __launch_bounds__(256) embed_kernel(const T* __restrict__ table,
 }
 
 // ------------------------------------------------------------ RMSNorm
-// One CTA per row; the sum of squares is reduced in a fixed order (lane
-// partials, warp butterfly, warps in index order).
+// One CTA per row; the sum of squares is reduced in a fixed order (each
+// thread's elements in index order, warp butterfly, warps in index order).
+// Rows of whole 16-byte chunks are read once into registers (up to
+// kNormKeep chunks per thread, the rest read again for the scaling pass).
+constexpr int kNormThreads = 256;
+constexpr int kNormKeep = 4;
+
+template <typename T> struct Chunk8 {
+  static_assert(sizeof(T) == 2, "16-bit element types");
+  __device__ static void unpack(const uint4& v, float* f) {
+    const T* e = reinterpret_cast<const T*>(&v);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) f[i] = to_f<T>(e[i]);
+  }
+  __device__ static uint4 pack(const float* f) {
+    uint4 v;
+    T* e = reinterpret_cast<T*>(&v);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) e[i] = from_f<T>(f[i]);
+    return v;
+  }
+};
+
 template <typename T>
-__global__ void __launch_bounds__(256) rmsnorm_kernel(const T* __restrict__ x, const T* __restrict__ g, int d,
-                                                      float eps, T* __restrict__ y) {
-  __shared__ float wsum[8];
+__global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const T* __restrict__ x, const T* __restrict__ g,
+                                                               int d, float eps, T* __restrict__ y, int vec) {
+  __shared__ float wsum[kNormThreads / 32];
   pdl_wait();
   pdl_launch_dependents();
   const T* xr = x + (int64_t)blockIdx.x * d;
+  T* yr = y + (int64_t)blockIdx.x * d;
+  const int t = threadIdx.x;
   float s = 0.f;
-  for (int i = threadIdx.x; i < d; i += blockDim.x) {
-    const float v = to_f<T>(xr[i]);
-    s = fmaf(v, v, s);
+  uint4 keep[kNormKeep];
+  const int nc = d / 8;
+  if (vec) {
+    const uint4* xv = reinterpret_cast<const uint4*>(xr);
+#pragma unroll
+    for (int j = 0; j < kNormKeep; ++j) {
+      const int c = t + j * kNormThreads;
+      keep[j] = c < nc ? xv[c] : make_uint4(0u, 0u, 0u, 0u);
+    }
+#pragma unroll
+    for (int j = 0; j < kNormKeep; ++j) {
+      float f[8];
+      Chunk8<T>::unpack(keep[j], f);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) s = fmaf(f[i], f[i], s);
+    }
+    for (int c = t + kNormKeep * kNormThreads; c < nc; c += kNormThreads) {
+      float f[8];
+      Chunk8<T>::unpack(xv[c], f);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) s = fmaf(f[i], f[i], s);
+    }
+  } else {
+    for (int i = t; i < d; i += kNormThreads) {
+      const float v = to_f<T>(xr[i]);
+      s = fmaf(v, v, s);
+    }
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-  if ((threadIdx.x & 31) == 0) wsum[threadIdx.x >> 5] = s;
+  if ((t & 31) == 0) wsum[t >> 5] = s;
   __syncthreads();
   float tot = 0.f;
-  for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += wsum[w];
+#pragma unroll
+  for (int w = 0; w < kNormThreads / 32; ++w) tot += wsum[w];
   const float r = 1.0f / sqrtf(tot / (float)d + eps);
-  T* yr = y + (int64_t)blockIdx.x * d;
-  for (int i = threadIdx.x; i < d; i += blockDim.x) yr[i] = from_f<T>(to_f<T>(xr[i]) * r * to_f<T>(g[i]));
+  if (vec) {
+    const uint4* xv = reinterpret_cast<const uint4*>(xr);
+    const uint4* gv = reinterpret_cast<const uint4*>(g);
+    uint4* yv = reinterpret_cast<uint4*>(yr);
+    auto scale = [&](int c, const uint4& xc) {
+      float f[8], gf[8], o[8];
+      Chunk8<T>::unpack(xc, f);
+      Chunk8<T>::unpack(gv[c], gf);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) o[i] = f[i] * r * gf[i];
+      yv[c] = Chunk8<T>::pack(o);
+    };
+#pragma unroll
+    for (int j = 0; j < kNormKeep; ++j)
+      if (t + j * kNormThreads < nc) scale(t + j * kNormThreads, keep[j]);
+    for (int c = t + kNormKeep * kNormThreads; c < nc; c += kNormThreads) scale(c, xv[c]);
+  } else {
+    for (int i = t; i < d; i += kNormThreads) yr[i] = from_f<T>(to_f<T>(xr[i]) * r * to_f<T>(g[i]));
+  }
 }
 
 // ------------------------------------------------------------ RoPE + cache
@@ -296,34 +361,82 @@ size_t attention_smem_bytes(int max_seq) {
 }
 
 // ------------------------------------------------------------ argmax
+// One CTA per row.  Each thread scans its elements in index order keeping
+// the first maximum; threads, then warps, are combined by (larger value,
+// then smaller index), an order-independent rule, so ties go to the
+// lowest index.  Rows of whole 16-byte chunks are read kArgBatch chunks
+// per thread at a time.
+constexpr int kArgThreads = 1024;
+constexpr int kArgBatch = 4;
+
+__device__ __forceinline__ void arg_take(float& best, int& bi, float ov, int oi) {
+  if (ov > best || (ov == best && oi < bi)) {
+    best = ov;
+    bi = oi;
+  }
+}
+
 template <typename T>
-__global__ void __launch_bounds__(256) argmax_kernel(const T* __restrict__ x, int n, int* __restrict__ out) {
-  __shared__ float sv[256];
-  __shared__ int si[256];
+__global__ void __launch_bounds__(kArgThreads) argmax_kernel(const T* __restrict__ x, int n, int* __restrict__ out,
+                                                             int vec) {
+  __shared__ float sv[kArgThreads / 32];
+  __shared__ int si[kArgThreads / 32];
   pdl_wait();
   pdl_launch_dependents();
   const T* row = x + (int64_t)blockIdx.x * n;
+  const int t = threadIdx.x;
   float best = -INFINITY;
   int bi = 0x7fffffff;
-  for (int j = threadIdx.x; j < n; j += blockDim.x) {
-    const float v = to_f<T>(row[j]);
-    if (v > best) { best = v; bi = j; }  // strictly greater: first index wins
-  }
-  sv[threadIdx.x] = best;
-  si[threadIdx.x] = bi;
-  __syncthreads();
-  for (int stride = blockDim.x / 2; stride > 0; stride >>= 1) {
-    if ((int)threadIdx.x < stride) {
-      const float ov = sv[threadIdx.x + stride];
-      const int oi = si[threadIdx.x + stride];
-      if (ov > sv[threadIdx.x] || (ov == sv[threadIdx.x] && oi < si[threadIdx.x])) {
-        sv[threadIdx.x] = ov;
-        si[threadIdx.x] = oi;
+  if (vec) {
+    const uint4* rv = reinterpret_cast<const uint4*>(row);
+    const int nc = n / 8;
+    for (int c0 = t; c0 < nc; c0 += kArgBatch * kArgThreads) {
+      uint4 v[kArgBatch];
+#pragma unroll
+      for (int u = 0; u < kArgBatch; ++u) {
+        const int c = c0 + u * kArgThreads;
+        v[u] = c < nc ? rv[c] : make_uint4(0u, 0u, 0u, 0u);
+      }
+#pragma unroll
+      for (int u = 0; u < kArgBatch; ++u) {
+        const int c = c0 + u * kArgThreads;
+        if (c < nc) {
+          float f[8];
+          Chunk8<T>::unpack(v[u], f);
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            if (f[i] > best) {  // strictly greater: the first index wins
+              best = f[i];
+              bi = c * 8 + i;
+            }
+        }
       }
     }
-    __syncthreads();
+  } else {
+    for (int j = t; j < n; j += kArgThreads) {
+      const float v = to_f<T>(row[j]);
+      if (v > best) {
+        best = v;
+        bi = j;
+      }
+    }
   }
-  if (threadIdx.x == 0) out[blockIdx.x] = si[0] == 0x7fffffff ? 0 : si[0];
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1)
+    arg_take(best, bi, __shfl_xor_sync(0xffffffffu, best, off), __shfl_xor_sync(0xffffffffu, bi, off));
+  if ((t & 31) == 0) {
+    sv[t >> 5] = best;
+    si[t >> 5] = bi;
+  }
+  __syncthreads();
+  if (t < 32) {
+    best = sv[t];
+    bi = si[t];
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1)
+      arg_take(best, bi, __shfl_xor_sync(0xffffffffu, best, off), __shfl_xor_sync(0xffffffffu, bi, off));
+    if (t == 0) out[blockIdx.x] = bi == 0x7fffffff ? 0 : bi;
+  }
 }
 
 __global__ void advance_kernel(int* pos_ptr, int n) {
@@ -352,9 +465,10 @@ int launch_embed(int dtype, const void* table, const int* ids, int tokens, int v
 }
 
 int launch_rmsnorm(int dtype, const void* x, const void* g, int rows, int d, float eps, void* y, cudaStream_t s) {
-  SN_DISPATCH16(dtype, T, return done(launch_pdl(rmsnorm_kernel<T>, dim3(rows), dim3(256), 0, s,
+  const int vec = d % 8 == 0 && (((uintptr_t)x | (uintptr_t)g | (uintptr_t)y) & 15) == 0;
+  SN_DISPATCH16(dtype, T, return done(launch_pdl(rmsnorm_kernel<T>, dim3(rows), dim3(kNormThreads), 0, s,
                                                  static_cast<const T*>(x), static_cast<const T*>(g), d, eps,
-                                                 static_cast<T*>(y)), "rmsnorm launch"));
+                                                 static_cast<T*>(y), vec), "rmsnorm launch"));
   return SWAPNET_OK;
 }
 
@@ -391,8 +505,9 @@ int launch_attention(int dtype, void* q, const void* k, const void* v, void* kc,
 }
 
 int launch_argmax(int dtype, const void* x, int rows, int n, int* out, cudaStream_t s) {
-  SN_DISPATCH16(dtype, T, return done(launch_pdl(argmax_kernel<T>, dim3(rows), dim3(256), 0, s,
-                                                 static_cast<const T*>(x), n, out), "argmax launch"));
+  const int vec = n % 8 == 0 && ((uintptr_t)x & 15) == 0;
+  SN_DISPATCH16(dtype, T, return done(launch_pdl(argmax_kernel<T>, dim3(rows), dim3(kArgThreads), 0, s,
+                                                 static_cast<const T*>(x), n, out, vec), "argmax launch"));
   return SWAPNET_OK;
 }
 

@@ -56,80 +56,70 @@ template <typename T> __device__ __forceinline__ uint4 pack16(const float* f) {
 }
 
 // ------------------------------------------------------------ skinny linear
-// One CTA (8 warps) computes COLS output features for all M rows.  Warp w
-// reduces the K range [w*Kw, (w+1)*Kw); inside a warp lane l takes the
-// 16-byte chunks l, l+32, ...; partial sums are combined by a butterfly and
-// then across warps in index order, so the result does not depend on
-// scheduling.
-constexpr int kSkCols = 2;
+// One warp per output feature, for all M rows: lane l reads the 16-byte
+// chunks l, l+32, ... of the feature's weight row, kSkBatch loads in flight
+// per lane, and keeps one fp32 partial sum per row in chunk order; a
+// butterfly combines the lanes, so the result does not depend on
+// scheduling.  The weights do not depend on the kernel before (they are in
+// place before this kernel is launched), so the first batch is requested
+// before the programmatic wait and overlaps that kernel's drain.
 constexpr int kSkWarps = 8;
+constexpr int kSkBatch = 8;
 
 template <typename T, int MT>
 __global__ void __launch_bounds__(kSkWarps * 32) linear_skinny_kernel(const T* __restrict__ x, int M, int K,
                                                                       const T* __restrict__ W, int N, Epi e,
                                                                       T* __restrict__ y, int64_t ldy) {
   constexpr int V = Vec16<T>::N;
-  __shared__ float red[kSkWarps][kSkCols][MT];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int o = blockIdx.x * kSkWarps + warp;
+  const int kchunks = K / V;  // K % V == 0 (checked on the host)
+  const T* wrow = W + (int64_t)min(o, N - 1) * K;
+  uint4 wv[kSkBatch];
+  auto load_batch = [&](int c0) {
+#pragma unroll
+    for (int u = 0; u < kSkBatch; ++u) {
+      const int ch = c0 + u * 32;
+      wv[u] = ch < kchunks ? ld_stream16(wrow + (int64_t)ch * V) : make_uint4(0u, 0u, 0u, 0u);
+    }
+  };
+  if (o < N) load_batch(lane);
   pdl_wait();
   pdl_launch_dependents();
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int o0 = blockIdx.x * kSkCols;
-  const int kchunks = K / V;                       // K % V == 0 (checked on the host)
-  const int per_warp = (kchunks + kSkWarps - 1) / kSkWarps;
-  const int c_begin = warp * per_warp;
-  const int c_end = min(kchunks, c_begin + per_warp);
-  float acc[kSkCols][MT];
+  if (o >= N) return;
+  float acc[MT];
 #pragma unroll
-  for (int c = 0; c < kSkCols; ++c)
+  for (int m = 0; m < MT; ++m) acc[m] = 0.f;
+  for (int c0 = lane; c0 < kchunks; c0 += 32 * kSkBatch) {
+    if (c0 != lane) load_batch(c0);
 #pragma unroll
-    for (int m = 0; m < MT; ++m) acc[c][m] = 0.f;
-
-  for (int ch = c_begin + lane; ch < c_end; ch += 32) {
-    const int k = ch * V;
-    float wv[kSkCols][V];
+    for (int u = 0; u < kSkBatch; ++u) {
+      const int ch = c0 + u * 32;
+      if (ch < kchunks) {
+        float wf[V];
+        unpack16<T>(wv[u], wf);
 #pragma unroll
-    for (int c = 0; c < kSkCols; ++c) {
-      if (o0 + c < N) {
-        unpack16<T>(ld_stream16(W + (int64_t)(o0 + c) * K + k), wv[c]);
-      } else {
+        for (int m = 0; m < MT; ++m) {
+          if (m < M) {
+            float xv[V];
+            unpack16<T>(__ldg(reinterpret_cast<const uint4*>(x + (int64_t)m * K + (int64_t)ch * V)), xv);
 #pragma unroll
-        for (int i = 0; i < V; ++i) wv[c][i] = 0.f;
-      }
-    }
-#pragma unroll
-    for (int m = 0; m < MT; ++m) {
-      if (m < M) {
-        float xv[V];
-        unpack16<T>(__ldg(reinterpret_cast<const uint4*>(x + (int64_t)m * K + k)), xv);
-#pragma unroll
-        for (int c = 0; c < kSkCols; ++c)
-#pragma unroll
-          for (int i = 0; i < V; ++i) acc[c][m] = fmaf(wv[c][i], xv[i], acc[c][m]);
+            for (int i = 0; i < V; ++i) acc[m] = fmaf(wf[i], xv[i], acc[m]);
+          }
+        }
       }
     }
   }
+  const float b = e.bias ? to_f<T>(reinterpret_cast<const T*>(e.bias)[o]) : 0.f;
 #pragma unroll
-  for (int c = 0; c < kSkCols; ++c)
+  for (int m = 0; m < MT; ++m) {
+    float v = acc[m];
 #pragma unroll
-    for (int m = 0; m < MT; ++m) {
-      float v = acc[c][m];
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-      if (lane == 0) red[warp][c][m] = v;
-    }
-  __syncthreads();
-  const int t = threadIdx.x;
-  if (t < kSkCols * MT) {
-    const int c = t / MT, m = t % MT;
-    const int o = o0 + c;
-    if (m < M && o < N) {
-      float s = 0.f;
-#pragma unroll
-      for (int w = 0; w < kSkWarps; ++w) s += red[w][c][m];
-      const float b = e.bias ? to_f<T>(reinterpret_cast<const T*>(e.bias)[o]) : 0.f;
+    for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+    if (lane == m && m < M) {
       float r = 0.f;
       if (e.res) r = to_f<T>(reinterpret_cast<const T*>(e.res)[(int64_t)m * e.ldr + o]);
-      y[(int64_t)m * ldy + o] = from_f<T>(epilogue(s, b, r, e.res != nullptr, e.act, e.res_post));
+      y[(int64_t)m * ldy + o] = from_f<T>(epilogue(v, b, r, e.res != nullptr, e.act, e.res_post));
     }
   }
 }
@@ -137,7 +127,7 @@ __global__ void __launch_bounds__(kSkWarps * 32) linear_skinny_kernel(const T* _
 template <typename T>
 int skinny_dispatch(const void* x, int M, int K, const void* W, int N, const Epi& e, void* y, int64_t ldy,
                     cudaStream_t s) {
-  const dim3 grid((N + kSkCols - 1) / kSkCols), block(kSkWarps * 32);
+  const dim3 grid((N + kSkWarps - 1) / kSkWarps), block(kSkWarps * 32);
   const T* xp = static_cast<const T*>(x);
   const T* wp = static_cast<const T*>(W);
   T* yp = static_cast<T*>(y);

@@ -273,3 +273,39 @@ def test_llm_cache_bound_reported_not_faulted():
     with pytest.raises(capi.SwapnetError) as ei:
         eng.sync()
     assert ei.value.code == capi.ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("vocab", [1000, 1003])
+def test_argmax_ties_go_to_the_lowest_index(vocab):
+    """A head whose second half of features repeats the first half gives
+    every logit a twin: the argmax is the first of the two (and an all-zero
+    head makes every logit equal: index 0).  1000 features take the
+    16-byte-chunk scan, 1003 the element scan."""
+    import torch
+    m = synth.arch.llm(layers=0, d=256, heads=2, ffn=688, vocab=vocab, tokens=4, max_seq=16)
+    w = synth.gen.model_weights(m)
+    head = len(m["layers"]) - 2
+    half = vocab // 2
+    W = w[head][0]
+    W[half:2 * half] = W[:half]
+    x = synth.gen.model_input(m)
+    for zero in (False, True):
+        if zero:
+            W[:] = 0
+        plan = capi.Plan.resident(capi.Desc(m))
+        info = plan.info()
+        eng = capi.Engine(plan, capi.HostWeights(w))
+        din = torch.zeros(max(16, info["input_bytes"]), dtype=torch.uint8, device="cuda")
+        din[:x.nbytes].copy_(torch.from_numpy(x.view(np.uint8).reshape(-1)))
+        dout = torch.zeros(info["output_bytes"], dtype=torch.uint8, device="cuda")
+        eng.infer(din.data_ptr(), dout.data_ptr(), torch.cuda.current_stream().cuda_stream)
+        eng.sync()
+        hb = dout.cpu().numpy()
+        offs = plan.output_offsets()
+        logits = F.decode(hb[offs[0]:offs[0] + 4 * vocab * 2].view(np.uint16), "bf16").reshape(4, vocab)
+        tok = hb[offs[1]:offs[1] + 16].view(np.int32)
+        for t in range(4):
+            assert tok[t] == int(np.argmax(logits[t])), (zero, t)
+            assert tok[t] == 0 if zero else tok[t] < half or tok[t] == 2 * half
+            if not zero and tok[t] < half:
+                assert logits[t, tok[t]] == logits[t, tok[t] + half]
