@@ -338,18 +338,18 @@ def run_llm(args, rank, world, group):
     alpha = int(round(1e18 / (link_peak * 1e9)))
     budget = 4_000_000_000
     variant = variant_code(args.variant)
-    opt = capi.options(swap_variant=variant, alpha_as_per_byte=alpha, beta_ns_per_tensor=0)
+    opt = capi.options(swap_variant=variant, alpha_as_per_byte=alpha, beta_ns_per_tensor=0, merge=args.merge)
     dp, dd = capi.Desc(mp), capi.Desc(md)
     t1 = time.perf_counter()
     pp, pd = capi.Plan.partition(dp, budget, opt), capi.Plan.partition(dd, budget, opt)
     t_plan = time.perf_counter() - t1
     ip, idd = pp.info(), pd.info()
     ep, ed = capi.Engine(pp, host), capi.Engine(pd, host)
-    rpp = capi.Plan.resident(dp)
+    rpp = capi.Plan.resident(dp, capi.options(merge=args.merge))
     arena = torch.empty(rpp.info()["arena_bytes"], dtype=torch.uint8, device="cuda")
     rp = capi.Engine(rpp, host, d_arena=arena.data_ptr(), arena_bytes=arena.numel())
-    rd = capi.Engine(capi.Plan.resident(dd, capi.options(preloaded=1)), host, d_arena=arena.data_ptr(),
-                     arena_bytes=arena.numel())
+    rd = capi.Engine(capi.Plan.resident(dd, capi.options(preloaded=1, merge=args.merge)), host,
+                     d_arena=arena.data_ptr(), arena_bytes=arena.numel())
     state = torch.zeros(ip["state_bytes"], dtype=torch.uint8, device="cuda")
     for e in (ep, ed, rp, rd):
         e.bind_state(state.data_ptr(), ip["state_bytes"])
@@ -431,7 +431,8 @@ def run_llm(args, rank, world, group):
     e2e_step_ms = group.max(statistics.mean(e2e_ms))
     e2e_tok_equal = int(h_tok[:4].numpy().view(np.int32)[0]) == sw_tok
     # extension (not the paper's method): resident-prefix plans in the same budget
-    opt_rp = capi.options(swap_variant=variant, alpha_as_per_byte=alpha, beta_ns_per_tensor=0, resident_prefix=1)
+    opt_rp = capi.options(swap_variant=variant, alpha_as_per_byte=alpha, beta_ns_per_tensor=0, resident_prefix=1,
+                          merge=args.merge)
     pp_rp, pd_rp = capi.Plan.partition(dp, budget, opt_rp), capi.Plan.partition(dd, budget, opt_rp)
     ep.free(); ed.free()
     ep_rp, ed_rp = capi.Engine(pp_rp, host), capi.Engine(pd_rp, host)
@@ -464,7 +465,8 @@ def run_llm(args, rank, world, group):
         "config": {"workload": text, "budget_bytes": budget, "weight_bytes": ip["weight_bytes"],
                    "prefill_blocks": ip["n_blocks"], "decode_blocks": idd["n_blocks"],
                    "plans_exact": [ip["exact"], idd["exact"]], "l2": "inputs (13.2 GB of weights) larger than L2",
-                   "swap_variant": args.variant, "state_bytes": ip["state_bytes"]},
+                   "swap_variant": args.variant, "merged_gemv_launches": args.merge,
+                   "state_bytes": ip["state_bytes"]},
         "prefill_ms": pre_ms, "decode_ms_per_token": dec_ms, "dinf_prefill_ms": pre_d,
         "dinf_decode_ms_per_token": dec_d, "dinf_ms": dinf_ms, "ratio": step_ms / dinf_ms,
         "greedy_token_swapped_equals_resident": sw_tok == rs_tok,
@@ -963,6 +965,8 @@ def main():
     ap.add_argument("--config", default="resnet50", choices=sorted(CONFIGS))
     ap.add_argument("--variant", default="auto", choices=VARIANTS)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--merge", type=int, default=1, choices=[0, 1],
+                    help="decoder: GEMV layers sharing an input in one launch (1) or one launch each (0)")
     ap.add_argument("--link-share", type=float, default=1.0,
                     help="multi: models sharing the host link in each model's delay model")
     ap.add_argument("--ablation", action="store_true",

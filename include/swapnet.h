@@ -195,6 +195,10 @@ typedef struct swapnet_options {
                                      together.  Objective 0, two slots, no resident
                                      prefix.  Consecutive inferences of one engine must
                                      be issued on one stream (as for any engine). */
+  int32_t merge;                 /* 1 (default): GEMV layers of one block that read
+                                     the same input (e.g. q, k, v; a SwiGLU gate and
+                                     up projection) run as one launch; 0: one launch
+                                     per layer.  Results are identical either way. */
   int32_t reserved[1];
 } swapnet_options;
 

@@ -123,6 +123,11 @@ struct swapnet_engine {
   std::vector<std::vector<int>> side_after;  // per unit: side units forked after it
   std::vector<std::vector<int>> side_wait;   // per unit: side units it waits for
   std::vector<char> is_side;
+  // merged GEMV launches: unit u launches itself and the merge_n[u] units
+  // after it (merge_pair: as a gate and its paired layer); merged_into[v]:
+  // v is launched by an earlier unit
+  std::vector<int> merge_n;
+  std::vector<char> merge_pair, merged_into;
   char* d_splitk = nullptr;          // split-K scratch: tile counters, then fp32 partials
   uint64_t splitk_bytes = 0;
   uint64_t splitk_counter_bytes = 0;
@@ -685,6 +690,87 @@ static bool small_conv_ok(const Model& m, const Layer& L) {
 
 static int plan_side(swapnet_engine* e);
 
+// A whole (unsplit) linear layer on the GEMV kernel, its weights in the arena
+// or read in place.
+static bool whole_skinny(const swapnet_engine* e, int u) {
+  const Unit& U = e->plan.units[u];
+  return e->unit_kind[u] == SWAPNET_KERNEL_SKINNY && !U.host && U.row0 == 0 &&
+         U.rows == e->plan.model.L[U.layer].d.cout;
+}
+
+// Merged GEMV launches (option merge): inside one block, consecutive whole
+// GEMV layers that read the same input with the same K and rows run as one
+// launch: up to kSkMaxSeg siblings none of which reads another's output
+// (e.g. the q, k, v projections), or a pair whose second layer takes the
+// first's output as its residual and nothing else of it (e.g. gate and up
+// of a SwiGLU feed-forward).  Results are bit-identical to separate
+// launches.
+static void plan_merges(swapnet_engine* e) {
+  const swapnet_plan& p = e->plan;
+  const Model& m = p.model;
+  const int n = (int)p.units.size();
+  e->merge_n.assign(n, 0);
+  e->merge_pair.assign(n, 0);
+  e->merged_into.assign(n, 0);
+  if (!p.opt.merge) return;
+  for (const Block& B : p.blocks) {
+    for (int u = B.u0; u < B.u1; ++u) {
+      if (!whole_skinny(e, u)) continue;
+      const Layer& L0 = m.L[p.units[u].layer];
+      auto same_input = [&](int v) {
+        const Layer& L = m.L[p.units[v].layer];
+        return v < B.u1 && whole_skinny(e, v) && L.d.src0 == L0.d.src0 && L.d.cin == L0.d.cin && L.n == L0.n;
+      };
+      if (same_input(u + 1)) {
+        const Layer& L1 = m.L[p.units[u + 1].layer];
+        if (L1.d.res == p.units[u].layer && L1.d.cout == L0.d.cout) {
+          e->merge_n[u] = 1;
+          e->merge_pair[u] = 1;
+          e->merged_into[u + 1] = 1;
+          ++u;
+          continue;
+        }
+      }
+      int k = 1;
+      for (; k < kSkMaxSeg && same_input(u + k); ++k) {
+        const Layer& L = m.L[p.units[u + k].layer];
+        bool reads_group = false;
+        for (int i = 0; i < k; ++i) {
+          const int li = p.units[u + i].layer;
+          reads_group = reads_group || L.d.res == li || L.d.src0 == li;
+        }
+        if (reads_group) break;
+      }
+      if (k == 1) continue;
+      e->merge_n[u] = k - 1;
+      for (int i = 1; i < k; ++i) e->merged_into[u + i] = 1;
+      u += k - 1;
+    }
+  }
+}
+
+// Launch unit u with the merge_n[u] units after it as one GEMV launch.
+static int run_group(swapnet_engine* e, int u, const void* din, void* dout, cudaStream_t s) {
+  const swapnet_plan& p = e->plan;
+  const Model& m = p.model;
+  const Layer& L0 = m.L[p.units[u].layer];
+  SkJob j{};
+  j.x = act_ptr(e, L0.d.src0, din, dout);
+  j.M = L0.n;
+  j.K = L0.d.cin;
+  j.nseg = 1 + e->merge_n[u];
+  j.pair = e->merge_pair[u];
+  for (int i = 0; i < j.nseg; ++i) {
+    const int v = u + i;
+    const Layer& L = m.L[p.units[v].layer];
+    const UnitExec& X = e->ux[v];
+    const char* r = L.d.res == SWAPNET_SRC_NONE ? nullptr : act_ptr(e, L.d.res, din, dout);
+    j.seg[i] = SkSeg{X.w, Epi{X.b, r, L.d.cout, L.d.act, L.d.res_post}, L.d.cout,
+                     out_ptr(e, p.units[v].layer, dout), L.d.cout};
+  }
+  return launch_linear_skinny_job(m.dtype, j, s);
+}
+
 static int prepare_units(swapnet_engine* e) {
   const swapnet_plan& p = e->plan;
   const Model& m = p.model;
@@ -749,6 +835,7 @@ static int prepare_units(swapnet_engine* e) {
       X.tmA_for = g.A;
     }
   }
+  plan_merges(e);
   return SWAPNET_OK;
 }
 
@@ -1112,6 +1199,7 @@ static int plan_side(swapnet_engine* e) {
     const Unit& U = p.units[u];
     const Layer& L = m.L[U.layer];
     if (L.start >= U.layer || U.host || lfirst[U.layer] != u || llast[U.layer] != u) continue;
+    if (e->merge_n[u] || e->merged_into[u]) continue;  // one launch with its siblings
     const UnitExec& X = e->ux[u];
     if (X.use_tc && X.tc.splits > 1 && !X.tc.cluster) continue;  // global split-K scratch is shared
     const int du = llast[L.start - 1];
@@ -1210,19 +1298,26 @@ static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t 
     }
     for (int u = B.u0; u < B.u1; ++u) {
       if (e->is_side[u]) continue;  // launched on the side stream after its producer
-      for (int w : e->side_wait[u]) CU(cudaStreamWaitEvent(s, e->side_done[w], 0), "wait side");
-      if (prof) CU(cudaEventRecord(e->ev_unit[2 * u], s), "profile event");
-      int rc = run_unit(e, u, din, dout, s);
+      if (e->merged_into[u]) continue;  // launched with an earlier unit
+      const int g1 = u + e->merge_n[u];  // last unit of this launch
+      for (int v = u; v <= g1; ++v)
+        for (int w : e->side_wait[v]) CU(cudaStreamWaitEvent(s, e->side_done[w], 0), "wait side");
+      if (prof)
+        for (int v = u; v <= g1; ++v) CU(cudaEventRecord(e->ev_unit[2 * v], s), "profile event");
+      int rc = g1 > u ? run_group(e, u, din, dout, s) : run_unit(e, u, din, dout, s);
       if (rc) return rc;
-      if (prof) CU(cudaEventRecord(e->ev_unit[2 * u + 1], s), "profile event");
-      for (int w : e->side_after[u]) {
-        CU(cudaEventRecord(e->side_fork, s), "record side fork");
-        CU(cudaStreamWaitEvent(e->side, e->side_fork, 0), "wait side fork");
-        if (prof) CU(cudaEventRecord(e->ev_unit[2 * w], e->side), "profile event");
-        rc = run_unit(e, w, din, dout, e->side);
-        if (rc) return rc;
-        if (prof) CU(cudaEventRecord(e->ev_unit[2 * w + 1], e->side), "profile event");
-        CU(cudaEventRecord(e->side_done[w], e->side), "record side done");
+      if (prof)
+        for (int v = u; v <= g1; ++v) CU(cudaEventRecord(e->ev_unit[2 * v + 1], s), "profile event");
+      for (int v = u; v <= g1; ++v) {
+        for (int w : e->side_after[v]) {
+          CU(cudaEventRecord(e->side_fork, s), "record side fork");
+          CU(cudaStreamWaitEvent(e->side, e->side_fork, 0), "wait side fork");
+          if (prof) CU(cudaEventRecord(e->ev_unit[2 * w], e->side), "profile event");
+          rc = run_unit(e, w, din, dout, e->side);
+          if (rc) return rc;
+          if (prof) CU(cudaEventRecord(e->ev_unit[2 * w + 1], e->side), "profile event");
+          CU(cudaEventRecord(e->side_done[w], e->side), "record side done");
+        }
       }
     }
     if (swap_k) CU(cudaEventRecord(e->slot_free[B.slot], s), "record slot free");
@@ -1254,6 +1349,7 @@ static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t 
 static uint64_t launches_per_infer(const swapnet_engine* e) {
   uint64_t n = e->plan.units.size() + (e->plan.model.has_attention ? 1 : 0);
   for (int k : e->unit_kind) n += (k == SWAPNET_KERNEL_ATTENTION) ? 1 : 0;
+  for (char c : e->merged_into) n -= c ? 1 : 0;
   if (!e->plan.resident)
     for (size_t k = 0; k < e->blocks.size(); ++k)
       if (e->plan.blocks[k].slot >= 0 && e->blocks[k].variant == SWAPNET_SWAP_ZEROCOPY)

@@ -63,19 +63,23 @@ template <typename T> __device__ __forceinline__ uint4 pack16(const float* f) {
 // scheduling.  The weights do not depend on the kernel before (they are in
 // place before this kernel is launched), so the first batch is requested
 // before the programmatic wait and overlaps that kernel's drain.
+//
+// One launch may serve several layers that read the same input (SkJob
+// segments, e.g. the q, k, v projections): the warps are dealt to the
+// segments' features in order.  In pair mode (a gate and the layer whose
+// epilogue takes the gate's output as its residual, e.g. SwiGLU) one warp
+// computes feature o of both: it stores the gate's rounded output and uses
+// that same rounded value as the second layer's residual.  Every feature is
+// computed by the same per-row routine as in a one-layer launch, so the
+// results are bit-identical to launching the layers one by one.
 constexpr int kSkWarps = 8;
 constexpr int kSkBatch = 8;
 
 template <typename T, int MT>
-__global__ void __launch_bounds__(kSkWarps * 32) linear_skinny_kernel(const T* __restrict__ x, int M, int K,
-                                                                      const T* __restrict__ W, int N, Epi e,
-                                                                      T* __restrict__ y, int64_t ldy) {
+__device__ __forceinline__ void sk_row(const T* __restrict__ x, int M, int K, const T* __restrict__ wrow, int lane,
+                                       uint4 (&wv)[kSkBatch], bool preloaded, float (&acc)[MT]) {
   constexpr int V = Vec16<T>::N;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int o = blockIdx.x * kSkWarps + warp;
   const int kchunks = K / V;  // K % V == 0 (checked on the host)
-  const T* wrow = W + (int64_t)min(o, N - 1) * K;
-  uint4 wv[kSkBatch];
   auto load_batch = [&](int c0) {
 #pragma unroll
     for (int u = 0; u < kSkBatch; ++u) {
@@ -83,15 +87,10 @@ __global__ void __launch_bounds__(kSkWarps * 32) linear_skinny_kernel(const T* _
       wv[u] = ch < kchunks ? ld_stream16(wrow + (int64_t)ch * V) : make_uint4(0u, 0u, 0u, 0u);
     }
   };
-  if (o < N) load_batch(lane);
-  pdl_wait();
-  pdl_launch_dependents();
-  if (o >= N) return;
-  float acc[MT];
 #pragma unroll
   for (int m = 0; m < MT; ++m) acc[m] = 0.f;
   for (int c0 = lane; c0 < kchunks; c0 += 32 * kSkBatch) {
-    if (c0 != lane) load_batch(c0);
+    if (c0 != lane || !preloaded) load_batch(c0);
 #pragma unroll
     for (int u = 0; u < kSkBatch; ++u) {
       const int ch = c0 + u * 32;
@@ -110,33 +109,81 @@ __global__ void __launch_bounds__(kSkWarps * 32) linear_skinny_kernel(const T* _
       }
     }
   }
-  const float b = e.bias ? to_f<T>(reinterpret_cast<const T*>(e.bias)[o]) : 0.f;
 #pragma unroll
   for (int m = 0; m < MT; ++m) {
-    float v = acc[m];
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-    if (lane == m && m < M) {
-      float r = 0.f;
-      if (e.res) r = to_f<T>(reinterpret_cast<const T*>(e.res)[(int64_t)m * e.ldr + o]);
-      y[(int64_t)m * ldy + o] = from_f<T>(epilogue(v, b, r, e.res != nullptr, e.act, e.res_post));
+    for (int off = 16; off > 0; off >>= 1) acc[m] += __shfl_xor_sync(0xffffffffu, acc[m], off);
+  }
+}
+
+template <typename T, int MT>
+__global__ void __launch_bounds__(kSkWarps * 32) linear_skinny_kernel(const SkJob j) {
+  constexpr int V = Vec16<T>::N;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  int o = blockIdx.x * kSkWarps + warp;
+  // this warp's segment (pair mode: both segments, feature o)
+  int si = 0;
+  if (!j.pair)
+    for (int i = 0; i + 1 < j.nseg && o >= j.seg[i].N; ++i) {
+      o -= j.seg[i].N;
+      si = i + 1;
+    }
+  SkSeg S = j.seg[0];
+#pragma unroll
+  for (int i = 1; i < kSkMaxSeg; ++i)
+    if (i == si) S = j.seg[i];
+  const bool active = o < S.N;
+  const T* x = static_cast<const T*>(j.x);
+  uint4 wv[kSkBatch];
+  if (active) {
+    const T* wrow = static_cast<const T*>(S.W) + (int64_t)o * j.K;
+#pragma unroll
+    for (int u = 0; u < kSkBatch; ++u) {
+      const int ch = lane + u * 32;
+      wv[u] = ch < j.K / V ? ld_stream16(wrow + (int64_t)ch * V) : make_uint4(0u, 0u, 0u, 0u);
+    }
+  }
+  pdl_wait();
+  pdl_launch_dependents();
+  if (!active) return;
+  float acc[MT];
+  float gate[MT];
+  const int passes = j.pair ? 2 : 1;
+  for (int p = 0; p < passes; ++p) {
+    if (p == 1) S = j.seg[1];
+    sk_row<T, MT>(x, j.M, j.K, static_cast<const T*>(S.W) + (int64_t)o * j.K, lane, wv, p == 0, acc);
+    const float b = S.e.bias ? to_f<T>(static_cast<const T*>(S.e.bias)[o]) : 0.f;
+#pragma unroll
+    for (int m = 0; m < MT; ++m) {
+      if (m < j.M) {
+        float r = 0.f;
+        bool has_r = S.e.res != nullptr;
+        if (p == 1) {
+          r = gate[m];
+          has_r = true;
+        } else if (has_r) {
+          r = to_f<T>(static_cast<const T*>(S.e.res)[(int64_t)m * S.e.ldr + o]);
+        }
+        const T out = from_f<T>(epilogue(acc[m], b, r, has_r, S.e.act, S.e.res_post));
+        gate[m] = to_f<T>(out);  // the stored value, as the paired layer would read it
+        if (lane == m) static_cast<T*>(S.y)[(int64_t)m * S.ldy + o] = out;
+      }
     }
   }
 }
 
-template <typename T>
-int skinny_dispatch(const void* x, int M, int K, const void* W, int N, const Epi& e, void* y, int64_t ldy,
-                    cudaStream_t s) {
-  const dim3 grid((N + kSkWarps - 1) / kSkWarps), block(kSkWarps * 32);
-  const T* xp = static_cast<const T*>(x);
-  const T* wp = static_cast<const T*>(W);
-  T* yp = static_cast<T*>(y);
-  if (M <= 1) launch_pdl(linear_skinny_kernel<T, 1>, grid, block, 0, s, xp, M, K, wp, N, e, yp, ldy);
-  else if (M <= 2) launch_pdl(linear_skinny_kernel<T, 2>, grid, block, 0, s, xp, M, K, wp, N, e, yp, ldy);
-  else if (M <= 4) launch_pdl(linear_skinny_kernel<T, 4>, grid, block, 0, s, xp, M, K, wp, N, e, yp, ldy);
-  else if (M <= 8) launch_pdl(linear_skinny_kernel<T, 8>, grid, block, 0, s, xp, M, K, wp, N, e, yp, ldy);
-  else launch_pdl(linear_skinny_kernel<T, 16>, grid, block, 0, s, xp, M, K, wp, N, e, yp, ldy);
-  return cudaGetLastError() == cudaSuccess ? SWAPNET_OK : SWAPNET_ERR_CUDA;
+template <typename T> int skinny_dispatch(const SkJob& j, cudaStream_t s) {
+  int rows = j.seg[0].N;
+  if (!j.pair)
+    for (int i = 1; i < j.nseg; ++i) rows += j.seg[i].N;
+  const dim3 grid((rows + kSkWarps - 1) / kSkWarps), block(kSkWarps * 32);
+  cudaError_t e;
+  if (j.M <= 1) e = launch_pdl(linear_skinny_kernel<T, 1>, grid, block, 0, s, j);
+  else if (j.M <= 2) e = launch_pdl(linear_skinny_kernel<T, 2>, grid, block, 0, s, j);
+  else if (j.M <= 4) e = launch_pdl(linear_skinny_kernel<T, 4>, grid, block, 0, s, j);
+  else if (j.M <= 8) e = launch_pdl(linear_skinny_kernel<T, 8>, grid, block, 0, s, j);
+  else e = launch_pdl(linear_skinny_kernel<T, 16>, grid, block, 0, s, j);
+  return e == cudaSuccess ? SWAPNET_OK : SWAPNET_ERR_CUDA;
 }
 
 // ------------------------------------------------------------ tiled linear
@@ -412,14 +459,29 @@ static int last_launch() {
   return SWAPNET_OK;
 }
 
+int launch_linear_skinny_job(int dtype, const SkJob& j, cudaStream_t s) {
+  const int es = dtype_size(dtype);
+  if (j.M < 1 || j.M > 16 || j.K < 1 || j.nseg < 1 || j.nseg > kSkMaxSeg || (j.pair && j.nseg != 2))
+    SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "skinny linear: M must be in [1, 16], 1 to 3 layers");
+  if ((j.K * es) % 16 || (uintptr_t)j.x % 16) SN_FAIL(SWAPNET_ERR_MISALIGNED, "skinny linear: rows must be 16-byte aligned");
+  for (int i = 0; i < j.nseg; ++i) {
+    if (j.seg[i].N < 1) SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "skinny linear: no output features");
+    if ((uintptr_t)j.seg[i].W % 16) SN_FAIL(SWAPNET_ERR_MISALIGNED, "skinny linear: rows must be 16-byte aligned");
+  }
+  if (j.pair && j.seg[0].N != j.seg[1].N) SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "skinny linear: paired layers differ in width");
+  SN_DISPATCH(dtype, T, return skinny_dispatch<T>(j, s));
+  return SWAPNET_OK;
+}
+
 int launch_linear_skinny(int dtype, const void* x, int M, int K, const void* W, int N, const Epi& e, void* y,
                          int64_t ldy, cudaStream_t s) {
-  const int es = dtype_size(dtype);
-  if (M < 1 || M > 16 || K < 1 || N < 1) SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "skinny linear: M must be in [1, 16]");
-  if ((K * es) % 16 || ((uintptr_t)x | (uintptr_t)W) % 16)
-    SN_FAIL(SWAPNET_ERR_MISALIGNED, "skinny linear: rows must be 16-byte aligned");
-  SN_DISPATCH(dtype, T, return skinny_dispatch<T>(x, M, K, W, N, e, y, ldy, s));
-  return SWAPNET_OK;
+  SkJob j{};
+  j.x = x;
+  j.M = M;
+  j.K = K;
+  j.nseg = 1;
+  j.seg[0] = SkSeg{W, e, N, y, ldy};
+  return launch_linear_skinny_job(dtype, j, s);
 }
 
 int launch_linear_tiled(int dtype, const void* x, int M, int K, const void* W, int N, const Epi& e, void* y,

@@ -22,6 +22,27 @@ struct Epi {
 int launch_linear_skinny(int dtype, const void* x, int M, int K, const void* W, int N, const Epi& e, void* y,
                          int64_t ldy, cudaStream_t s);
 
+// Several skinny linear layers reading the same x (M rows, K columns) in one
+// launch: segment i computes y_i[m, o] = epi_i(sum_k x[m,k] W_i[o,k]) for
+// o < N_i.  pair = 1 (two segments of equal N): segment 1's residual is
+// segment 0's stored output (its own res is ignored).  Bit-identical to
+// launching the segments one by one.
+constexpr int kSkMaxSeg = 3;
+struct SkSeg {
+  const void* W;
+  Epi e;
+  int N;
+  void* y;
+  int64_t ldy;
+};
+struct SkJob {
+  const void* x;
+  int M, K;
+  int nseg, pair;
+  SkSeg seg[kSkMaxSeg];
+};
+int launch_linear_skinny_job(int dtype, const SkJob& j, cudaStream_t s);
+
 // General tiled SIMT linear (any M, K, N): the fallback when neither the
 // tensor-core nor the skinny kernel applies.
 int launch_linear_tiled(int dtype, const void* x, int M, int K, const void* W, int N, const Epi& e, void* y,

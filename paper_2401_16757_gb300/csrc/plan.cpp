@@ -868,6 +868,7 @@ static int check_options(const swapnet_options& o) {
   if (o.graphs != 0 && o.graphs != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "graphs must be 0 or 1");
   if (o.preloaded != 0 && o.preloaded != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "preloaded must be 0 or 1");
   if (o.branches != 0 && o.branches != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "branches must be 0 or 1");
+  if (o.merge != 0 && o.merge != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "merge must be 0 or 1");
   if (o.split_cap < 0 || o.split_cap > 64) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "split_cap must be in [0, 64]");
   if (o.resident_prefix != 0 && o.resident_prefix != 1)
     SN_FAIL(SWAPNET_ERR_INVALID_ARG, "resident_prefix must be 0 or 1");
@@ -921,6 +922,7 @@ void swapnet_default_options(swapnet_options* o) {
   o->zc_ctas = 0;
   o->graphs = 1;
   o->branches = 1;
+  o->merge = 1;
 }
 
 int swapnet_partition(const swapnet_model_desc* desc, uint64_t budget, const swapnet_options* opt,

@@ -189,6 +189,11 @@ def test_swap_variant_range():
         with pytest.raises(capi.SwapnetError) as ei:
             capi.Plan.partition(desc, budget, capi.options(swap_variant=bad))
         assert ei.value.code == capi.ERR_INVALID_ARG
+    assert capi.options().merge == 1
+    for bad in (dict(merge=2), dict(merge=-1)):
+        with pytest.raises(capi.SwapnetError) as ei:
+            capi.Plan.partition(desc, budget, capi.options(**bad))
+        assert ei.value.code == capi.ERR_INVALID_ARG
 
 
 def test_prefetch_options_and_wrap_pair_are_checked():

@@ -44,7 +44,8 @@ class Decoder:
         self.engines, self.bufs = [], []
         for m in (self.mp, self.md):
             d = capi.Desc(m)
-            plan = capi.Plan.resident(d) if resident else capi.Plan.partition(d, budget, capi.options(**(opts or {})))
+            o = capi.options(**(opts or {}))
+            plan = capi.Plan.resident(d, o) if resident else capi.Plan.partition(d, budget, o)
             eng = capi.Engine(plan, self.host)
             info = plan.info()
             din = torch.zeros(max(16, info["input_bytes"]), dtype=torch.uint8, device="cuda")
@@ -309,3 +310,28 @@ def test_argmax_ties_go_to_the_lowest_index(vocab):
             assert tok[t] == 0 if zero else tok[t] < half or tok[t] == 2 * half
             if not zero and tok[t] < half:
                 assert logits[t, tok[t]] == logits[t, tok[t] + half]
+
+
+@pytest.mark.parametrize("resident", [True, False])
+def test_merged_gemv_launches_equal_separate_launches(resident):
+    """The decode pass launches q, k, v as one GEMV and gate, up as one
+    paired GEMV (option merge, the default): bit-identical to one launch per
+    layer, three launches fewer per decoder layer when the members share a
+    block."""
+    mg = Decoder(prefill_tokens=32, budget_frac=0.4, resident=resident)
+    sp = Decoder(prefill_tokens=32, budget_frac=0.4, resident=resident, host=mg.host, weights=mg.w,
+                 opts=dict(merge=0))
+    ids = synth.gen.model_input(mg.mp).reshape(-1)
+    a, b = mg.run(0, ids), sp.run(0, ids)
+    assert a[0].tobytes() == b[0].tobytes() and a[1].tobytes() == b[1].tobytes()
+    tok = np.array([a[1][-1]], dtype=np.int32)
+    l0 = [d.engines[1][1].stats()["kernel_launches"] for d in (mg, sp)]
+    for _ in range(4):
+        a, b = mg.run(1, tok), sp.run(1, tok)
+        assert a[0].tobytes() == b[0].tobytes() and a[1].tobytes() == b[1].tobytes()
+        tok = np.array([a[1][0]], dtype=np.int32)
+    per = [(d.engines[1][1].stats()["kernel_launches"] - x) // 4 for d, x in zip((mg, sp), l0)]
+    if resident:
+        assert per[1] - per[0] == 3 * SMALL["layers"]
+    else:
+        assert 0 <= per[1] - per[0] <= 3 * SMALL["layers"]
