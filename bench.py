@@ -873,10 +873,20 @@ def run_profile_once(args):
     import __graft_entry__
     __graft_entry__.build()
     from paper_2401_16757_gb300 import capi
-    m, w, x, wb, budget, text = build_workload(args.config, capi_weight_bytes)
+    if args.config == "llm":  # one decode pass of a decoder of the 7B widths with --profile-layers layers
+        import synth
+        m = synth.arch.llm(layers=args.profile_layers, tokens=1)
+        host = llm_host_weights(m)
+        x = np.array([7], dtype=np.int32)
+    else:
+        m, w, x, wb, budget, text = build_workload(args.config, capi_weight_bytes)
+        host = capi.HostWeights(w)
     plan = capi.Plan.resident(capi.Desc(m))
     info = plan.info()
-    eng = capi.Engine(plan, capi.HostWeights(w))
+    eng = capi.Engine(plan, host)
+    if info["state_bytes"]:
+        state = torch.zeros(info["state_bytes"], dtype=torch.uint8, device="cuda")
+        eng.bind_state(state.data_ptr(), info["state_bytes"])
     d_in = torch.empty(max(16, info["input_bytes"]), dtype=torch.uint8, device="cuda")
     d_in[:info["input_bytes"]].copy_(torch.from_numpy(x.view(np.uint8).reshape(-1)))
     d_out = torch.empty(info["output_bytes"], dtype=torch.uint8, device="cuda")
@@ -965,6 +975,8 @@ def main():
     ap.add_argument("--config", default="resnet50", choices=sorted(CONFIGS))
     ap.add_argument("--variant", default="auto", choices=VARIANTS)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile-layers", type=int, default=2,
+                    help="--profile-once --config llm: decoder layers of the profiled decode pass")
     ap.add_argument("--merge", type=int, default=1, choices=[0, 1],
                     help="decoder: GEMV layers sharing an input in one launch (1) or one launch each (0)")
     ap.add_argument("--link-share", type=float, default=1.0,
