@@ -198,7 +198,9 @@ typedef struct swapnet_options {
   int32_t merge;                 /* 1 (default): GEMV layers of one block that read
                                      the same input (e.g. q, k, v; a SwiGLU gate and
                                      up projection) run as one launch; 0: one launch
-                                     per layer.  Results are identical either way. */
+                                     per layer.  Results are identical either way;
+                                     profiling gives every layer of a merged launch
+                                     that launch's start and end. */
   int32_t reserved[1];
 } swapnet_options;
 
