@@ -65,10 +65,11 @@ def variant_code(name):
 
 # DRAM traffic per launch of a kernel family, from ncu (dram__bytes_read.sum
 # + dram__bytes_write.sum averaged over the launches of one swapped step of
-# the named workload), valid only for the kernel sources it was taken on.
+# the named workload), valid only for the tensor-core sources it was taken on
+# (traffic_sources_sha).
 TRAFFIC = {
-    ("resnet50", "tc_gemm"): ("179d5c9fa897", 1418599),
-    ("resnet50", "tc_conv"): ("179d5c9fa897", 1807876),
+    ("resnet50", "tc_gemm"): ("1bb9110c06be", 1418599),
+    ("resnet50", "tc_conv"): ("1bb9110c06be", 1807876),
 }
 
 
@@ -111,14 +112,25 @@ class RankGroup:
             self.dist = None
 
 
-def kernel_sources_sha():
+def sources_sha(files):
     import hashlib
     h = hashlib.sha1()
-    for f in ("k_tc.cu", "k_tc_persist.cu", "k_tc_small.cu", "tc_epi.cuh", "k_simt.cu", "k_decoder.cu",
-              "device.cuh"):
+    for f in files:
         with open(os.path.join(ROOT, "paper_2401_16757_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:12]
+
+
+def kernel_sources_sha():
+    """Tag of every layer-kernel source (names the sources a profile was taken on)."""
+    return sources_sha(("k_tc.cu", "k_tc_persist.cu", "k_tc_small.cu", "tc_epi.cuh", "k_simt.cu", "k_decoder.cu",
+                        "device.cuh"))
+
+
+def traffic_sources_sha():
+    """Tag of the sources the tensor-core GEMM family is compiled from: its
+    TRAFFIC figures stay valid while these are unchanged."""
+    return sources_sha(("k_tc.cu", "k_tc_persist.cu", "tc_epi.cuh", "device.cuh", "kernels.h", "internal.h"))
 
 
 def load_peaks():
@@ -1223,10 +1235,11 @@ def main():
                      "algorithmic_bytes_per_launch": dom_bytes // max(1, len(dom_idx)),
                      "flops_per_byte": dom_flops / dom_bytes if dom_bytes else None, "ridge_flops_per_byte": ridge,
                      "traffic": None, "kernel_sources_sha": kernel_sources_sha(),
+                     "traffic_sources_sha": traffic_sources_sha(),
                      "share_of_kernel_time": dom_us / max(1e-9, acc_u.sum()),
                      "kernel_time_share": {k: round(v / max(1e-9, acc_u.sum()), 4) for k, v in share.items()}})
     tr = TRAFFIC.get((args.config, dom))
-    if tr and tr[0] == roofline["kernel_sources_sha"]:
+    if tr and tr[0] == roofline["traffic_sources_sha"]:
         roofline["traffic"] = tr[1]
 
     # ---- host link: bytes per swap over swap time, against pinned memcpy peak
