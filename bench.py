@@ -712,6 +712,9 @@ def run_ablation(args):
     out["sequential_layers"] = try_plan(lambda: capi.Plan.partition(dc, budget, capi.options(**dict(base, branches=0))))
     out["zero_copy_swap"] = try_plan(
         lambda: capi.Plan.partition(dc, budget, capi.options(**dict(base, swap_variant=capi.SWAP_ZEROCOPY))))
+    # weights left pageable: each swap staged by the driver (the paper's w/o-uni-add)
+    out["pageable_staged_copy"] = try_plan(
+        lambda: capi.Plan.partition(dc, budget, capi.options(**dict(base, pageable=1))))
     out["resident_dinf"] = try_plan(lambda: capi.Plan.resident(d))
     print(json.dumps({"ablation": args.config, "workload": text, "budget_bytes": budget, "weight_bytes": wb,
                       "paper_block_count": n_min, "steps": args.steps, "results": out}))

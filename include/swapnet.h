@@ -201,6 +201,17 @@ typedef struct swapnet_options {
                                      per layer.  Results are identical either way;
                                      profiling gives every layer of a merged launch
                                      that launch's start and end. */
+  int32_t pageable;              /* 0 (default): the host weights are page-locked
+                                     (registered at load unless CUDA already pinned
+                                     them).  1 (the paper's w/o-uni-add ablation): they
+                                     stay in pageable memory and every swap-in is a
+                                     copy-engine copy the driver stages through its own
+                                     page-locked buffer; launches are eager (no graphs),
+                                     the swap variant is MEMCPY (AUTO resolves to it;
+                                     ZEROCOPY and DIRECT are refused), and models whose
+                                     layers read a table in host memory (EMBED) are
+                                     refused (UNSUPPORTED) at load.  Ignored by engines
+                                     loaded from a weights file. */
   int32_t reserved[1];
 } swapnet_options;
 
@@ -413,8 +424,8 @@ int swapnet_engine_sync(swapnet_engine* eng);
  * at the new plan's size, releasing the old one first, so a smaller budget
  * gives memory back.  A caller-provided arena stays and must hold the new
  * plan.  The plan is copied; the caller may free it after the call.
- * Errors: INVALID_ARG (a plan for another model, or resident <-> swapped),
- * OOM, CUDA. */
+ * Errors: INVALID_ARG (a plan for another model, resident <-> swapped, or
+ * a different `pageable` option), OOM, CUDA. */
 int swapnet_engine_adapt(swapnet_engine* eng, const swapnet_plan* plan);
 
 /* Decoder state of a model with ATTENTION layers: a device buffer of

@@ -48,7 +48,7 @@ class Options(C.Structure):
                 ("gamma_as_per_flop", C.c_uint64), ("eta_ns_per_tensor", C.c_uint64), ("zc_ctas", C.c_int32),
                 ("graphs", C.c_int32), ("preloaded", C.c_int32), ("branches", C.c_int32),
                 ("resident_prefix", C.c_int32), ("split_cap", C.c_int32), ("prefetch", C.c_int32),
-                ("merge", C.c_int32), ("reserved", C.c_int32 * 1)]
+                ("merge", C.c_int32), ("pageable", C.c_int32), ("reserved", C.c_int32 * 1)]
 
 
 class PlanInfo(C.Structure):

@@ -193,6 +193,16 @@ static int release(swapnet_engine* e) {
 // alias of every tensor.
 static int register_host(swapnet_engine* e, const void* const* hw, uint32_t nt) {
   const Model& m = e->plan.model;
+  if (e->plan.opt.pageable) {  // never registered: every copy is staged by the driver
+    for (const Unit& U : e->plan.units)
+      if (U.host) SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "pageable weights: a layer reads its table in host memory");
+    e->tensor_dev.assign(nt, nullptr);
+    for (uint32_t t = 0; t < nt; ++t) {
+      if (!hw[t]) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null host weight pointer");
+      e->tensor_dev[t] = static_cast<const char*>(hw[t]);
+    }
+    return SWAPNET_OK;
+  }
   const uintptr_t page = (uintptr_t)sysconf(_SC_PAGESIZE);
   struct R { uintptr_t lo, hi; };
   std::vector<R> rs;
@@ -976,7 +986,8 @@ static int bind_plan(swapnet_engine* e, void* d_arena_user, uint64_t arena_bytes
       CU(cudaMemset(e->d_splitk, 0, e->splitk_counter_bytes), "split-K counters");
     }
   }
-  const int variant = plan->opt.swap_variant;
+  const int variant = (plan->opt.pageable && plan->opt.swap_variant == SWAPNET_SWAP_AUTO) ? SWAPNET_SWAP_MEMCPY
+                                                                                        : plan->opt.swap_variant;
   if (plan->resident) {
     if (!preloaded_arena) {
       for (size_t k = 0; k < e->blocks.size() && !rc; ++k)
@@ -1137,6 +1148,8 @@ int swapnet_engine_adapt(swapnet_engine* e, const swapnet_plan* plan) {
             a.L[i].tbytes[0] == b.L[i].tbytes[0] && a.L[i].tbytes[1] == b.L[i].tbytes[1]);
   if (!same) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "the plan is for a different model");
   if (plan->resident != e->plan.resident) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "cannot switch between resident and swapped plans");
+  if (!e->file && plan->opt.pageable != e->plan.opt.pageable)
+    SN_FAIL(SWAPNET_ERR_INVALID_ARG, "cannot switch between pageable and page-locked host weights");
   CU(cudaSetDevice(e->device), "cudaSetDevice");
   CU(cudaStreamSynchronize(e->copy), "drain copies");
   if (e->side) CU(cudaStreamSynchronize(e->side), "drain side stream");
@@ -1390,7 +1403,8 @@ int swapnet_infer(swapnet_engine* e, const void* din, void* dout, swapnet_stream
   if (((uintptr_t)din | (uintptr_t)dout) & 15) SN_FAIL(SWAPNET_ERR_MISALIGNED, "input/output must be 16-byte aligned");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   CU(cudaSetDevice(e->device), "cudaSetDevice");
-  if (e->plan.opt.graphs && !e->profiling) {  // event timing needs eager launches
+  // event timing needs eager launches; stream capture takes no copy from pageable memory
+  if (e->plan.opt.graphs && !e->profiling && !(e->plan.opt.pageable && !e->file)) {
     const auto key = std::make_pair(std::make_pair(din, dout), false);
     auto it = e->graphs.find(key);
     if (it == e->graphs.end()) {

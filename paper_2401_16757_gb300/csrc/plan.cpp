@@ -869,6 +869,9 @@ static int check_options(const swapnet_options& o) {
   if (o.preloaded != 0 && o.preloaded != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "preloaded must be 0 or 1");
   if (o.branches != 0 && o.branches != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "branches must be 0 or 1");
   if (o.merge != 0 && o.merge != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "merge must be 0 or 1");
+  if (o.pageable != 0 && o.pageable != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "pageable must be 0 or 1");
+  if (o.pageable && (o.swap_variant == SWAPNET_SWAP_ZEROCOPY || o.swap_variant == SWAPNET_SWAP_DIRECT))
+    SN_FAIL(SWAPNET_ERR_INVALID_ARG, "pageable weights are copied by the copy engine only");
   if (o.split_cap < 0 || o.split_cap > 64) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "split_cap must be in [0, 64]");
   if (o.resident_prefix != 0 && o.resident_prefix != 1)
     SN_FAIL(SWAPNET_ERR_INVALID_ARG, "resident_prefix must be 0 or 1");

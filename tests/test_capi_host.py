@@ -189,8 +189,11 @@ def test_swap_variant_range():
         with pytest.raises(capi.SwapnetError) as ei:
             capi.Plan.partition(desc, budget, capi.options(swap_variant=bad))
         assert ei.value.code == capi.ERR_INVALID_ARG
-    assert capi.options().merge == 1
-    for bad in (dict(merge=2), dict(merge=-1)):
+    assert capi.options().merge == 1 and capi.options().pageable == 0
+    capi.Plan.partition(desc, budget, capi.options(pageable=1))
+    capi.Plan.partition(desc, budget, capi.options(pageable=1, swap_variant=capi.SWAP_MEMCPY))
+    for bad in (dict(merge=2), dict(merge=-1), dict(pageable=2), dict(pageable=1, swap_variant=capi.SWAP_ZEROCOPY),
+                dict(pageable=1, swap_variant=capi.SWAP_DIRECT)):
         with pytest.raises(capi.SwapnetError) as ei:
             capi.Plan.partition(desc, budget, capi.options(**bad))
         assert ei.value.code == capi.ERR_INVALID_ARG
