@@ -181,24 +181,34 @@ def _as2d(a):
     return a.reshape(a.shape[0], -1)
 
 
-def run_layer(layer, dtype, tensors, acts, x_in, state=None, li=None):
+def decode_params(tensors, dtype):
+    """A layer's parameter tensors as float64 (exact)."""
+    return [decode(t, dtype) for t in tensors]
+
+
+def run_layer(layer, dtype, tensors, acts, x_in, state=None, li=None, params=None):
     """Compute one layer (float64 in, rounded float64 out).
 
     tensors: the layer's storage arrays; acts: dict layer index -> NCHW
     float64 output; x_in: NCHW float64 model input (token ids for a token
-    model); state: KV caches and position for attention layers.
+    model); state: KV caches and position for attention layers; params:
+    decode_params(tensors) when the caller already has them (a layer run
+    several times is decoded once).
     """
     def get(i):
         return x_in if i == -1 else acts[i]
 
+    def param(i):
+        return params[i] if params is not None else decode(tensors[i], dtype)
+
     op = layer["op"]
     src = get(layer["src"][0])
     if op == "embed":
-        table = decode(tensors[0], dtype)
+        table = param(0)
         ids = np.asarray(src).reshape(-1).astype(np.int64)
         return table[ids].reshape(len(ids), -1, 1, 1)          # a copy: no rounding needed
     if op == "rmsnorm":
-        y = rmsnorm(_as2d(src), decode(tensors[0], dtype), layer["eps"])
+        y = rmsnorm(_as2d(src), param(0), layer["eps"])
         return round_as(y, dtype).reshape(src.shape)
     if op == "attention":
         q, k, v = (_as2d(get(i)) for i in layer["src"])
@@ -217,8 +227,8 @@ def run_layer(layer, dtype, tensors, acts, x_in, state=None, li=None):
         a = _as2d(src)
         return np.argmax(a, axis=1).astype(np.float64).reshape(-1, 1, 1, 1)
     if op in ("conv", "linear"):
-        w = decode(tensors[0], dtype)
-        b = decode(tensors[1], dtype) if len(tensors) > 1 else np.zeros(w.shape[0])
+        w = param(0)
+        b = param(1) if len(tensors) > 1 else np.zeros(w.shape[0])
         if op == "conv":
             y = conv2d(src, w, b, layer["stride"], layer["pad"])
         else:

@@ -43,6 +43,7 @@ class Runner:
         import torch
         self.torch = torch
         self.model = model
+        self.host_weights = weights
         self.plan = plan
         self.info = plan.info()
         self.host = host or capi.HostWeights(weights)
@@ -78,3 +79,21 @@ class Runner:
 
 def oracle_outputs(model, weights, x):
     return F.forward(model, weights, x)
+
+
+_ORACLE_CACHE = {}
+
+
+def oracle_cached(model, weights, x, request=0):
+    """oracle_outputs of a workload built by synth (seeded weights, input of
+    `request`), kept for the rest of the session: several tests compare
+    different engines of the same workload with the same oracle run."""
+    key = (model["name"], model["model_id"], tuple(model["input"]), request, x.tobytes()[:64], x.nbytes)
+    if key not in _ORACLE_CACHE:
+        _ORACLE_CACHE[key] = F.forward(model, weights, x)
+    return _ORACLE_CACHE[key]
+
+
+def check_oracle(runner, got_raw, x, request=0):
+    """The engine's raw outputs of input x against the (cached) oracle."""
+    check_close(runner.model, runner.decode(got_raw), oracle_cached(runner.model, runner.host_weights, x, request))

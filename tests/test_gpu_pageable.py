@@ -2,13 +2,14 @@
 w/o-uni-add ablation): the host tensors are never page-locked and every
 swap-in is a copy the driver stages through its own page-locked buffer.
 The arena receives the same bytes, so the outputs equal the resident run's
-bit for bit; the options that need page-locked memory are refused."""
+bit for bit (and the oracle's within the fp16 bar); the options that need
+page-locked memory are refused."""
 import pytest
 
 from oracle import plan as OP
 import synth
 from paper_2401_16757_gb300 import capi
-from helpers import Runner
+from helpers import Runner, check_oracle
 
 pytestmark = pytest.mark.gpu
 
@@ -26,6 +27,7 @@ def test_pageable_swaps_equal_resident():
     for _ in range(3):
         got = pg.run(x)
         assert all(a.tobytes() == b.tobytes() for a, b in zip(got, ref))
+    check_oracle(pg, got, x)
     # a page-locked plan cannot be switched to on this engine
     with pytest.raises(capi.SwapnetError) as ei:
         pg.engine.adapt(capi.Plan.partition(d, budget, capi.options()))

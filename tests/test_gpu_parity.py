@@ -3,10 +3,11 @@ the CPU oracle, and swapped against all-resident (bit-exact)."""
 import numpy as np
 import pytest
 
+from oracle import forward as F
 from oracle import plan as OP
 import synth
 from paper_2401_16757_gb300 import capi
-from helpers import Runner, check_close, oracle_outputs, rel_l2
+from helpers import Runner, check_close, check_oracle, oracle_cached, oracle_outputs, rel_l2
 
 pytestmark = pytest.mark.gpu
 
@@ -206,7 +207,7 @@ def test_calibrated_plan_is_exact_and_feasible():
     budget = int(OP.weight_bytes(m) * 0.4) // 256 * 256
     p0 = capi.Plan.partition(d, budget, capi.options())
     r0 = Runner(m, w, p0, host)
-    t_ex, alpha = capi.calibrate(m, p0, r0.engine)
+    t_ex, alpha = capi.calibrate(m, r0.engine)
     assert all(t > 0 for t in t_ex) and alpha and alpha > 0
     p1 = capi.Plan.partition(capi.Desc(m, t_ex_ns=t_ex), budget,
                              capi.options(alpha_as_per_byte=alpha, beta_ns_per_tensor=0))
@@ -265,7 +266,8 @@ def test_yolov3_config():
 def test_multi_dnn_schedule_concurrent():
     """Eq. 1 split of one arena (30 % of the summed weight bytes) over
     ResNet-50, VGG-16 and YOLOv3; the three engines run concurrently on their
-    own streams and each output equals its resident run bit for bit."""
+    own streams and each output equals its resident run bit for bit and the
+    oracle within the fp16 bar."""
     import torch
     ms = [synth.arch.resnet50(), synth.arch.vgg16(), synth.arch.yolov3()]
     total = sum(OP.weight_bytes(m) for m in ms)
@@ -288,10 +290,11 @@ def test_multi_dnn_schedule_concurrent():
         for r, s in zip(runners, streams):
             r.engine.infer(r.d_in.data_ptr(), r.d_out.data_ptr(), s.cuda_stream)
     torch.cuda.synchronize()
-    for r, ref in zip(runners, refs):
+    for r, ref, x in zip(runners, refs, xs):
         r.engine.sync()
         got = r.outputs_raw()
         assert all(a.tobytes() == b.tobytes() for a, b in zip(got, ref))
+        check_oracle(r, got, x)
 
 
 @pytest.mark.parametrize("name", ["resnet50", "yolov3"])
@@ -310,6 +313,7 @@ def test_concurrent_branches_bit_exact(name):
     sw = Runner(m, w, capi.Plan.partition(d, budget, capi.options(branches=1)), host).run(x)
     for a, b, c in zip(seq, par, sw):
         assert a.tobytes() == b.tobytes() == c.tobytes()
+    check_close(m, [F.decode(o, m["dtype"]) for o in sw], oracle_cached(m, w, x))
 
 
 @pytest.mark.parametrize("name", ["resnet50", "yolov3"])
@@ -331,6 +335,8 @@ def test_resident_prefix_bit_exact_over_repeated_inferences(name):
         x = synth.gen.model_input(m, request=req)
         a, b = sw.run(x), rs.run(x)
         assert all(p.tobytes() == q.tobytes() for p, q in zip(a, b)), req
+        if req == 0:
+            check_oracle(sw, a, x)
 
 
 @pytest.mark.parametrize("name,variant", [("resnet50", capi.SWAP_AUTO), ("yolov3", capi.SWAP_MEMCPY),
@@ -354,6 +360,8 @@ def test_first_block_prefetch_bit_exact_over_repeated_inferences(name, variant):
         x = synth.gen.model_input(m, request=req)
         a, b = sw.run(x), rs.run(x)
         assert all(p.tobytes() == q.tobytes() for p, q in zip(a, b)), req
+        if req == 0:
+            check_oracle(sw, a, x)
     sw.engine.set_profiling(True)  # eager launches
     x = synth.gen.model_input(m, request=7)
     assert all(p.tobytes() == q.tobytes() for p, q in zip(sw.run(x), rs.run(x)))
@@ -368,8 +376,8 @@ def test_first_block_prefetch_bit_exact_over_repeated_inferences(name, variant):
 def test_engine_adapts_to_new_budgets_between_inferences():
     """Runtime budget adaptation: one engine switched through plans for
     shrinking and growing budgets (made ahead, like the paper's look-up
-    table) gives the resident bits after every switch; a plan for another
-    model is refused."""
+    table) gives the resident bits after every switch, and the oracle's
+    outputs for each new request; a plan for another model is refused."""
     import torch
     m = synth.arch.resnet50()
     w = synth.gen.model_weights(m)
@@ -386,6 +394,7 @@ def test_engine_adapts_to_new_budgets_between_inferences():
         x = synth.gen.model_input(m, request=i)
         a, b = sw.run(x), rs.run(x)
         assert all(p.tobytes() == q.tobytes() for p, q in zip(a, b)), f
+        check_oracle(sw, a, x, request=i)
         assert sw.engine.stats()["infer_calls"] >= 1
     other = synth.arch.vgg16()
     with pytest.raises(capi.SwapnetError) as ei:

@@ -10,7 +10,7 @@ import pytest
 from oracle import plan as OP
 import synth
 from paper_2401_16757_gb300 import capi
-from helpers import Runner, check_close, oracle_outputs
+from helpers import Runner, check_close, check_oracle, oracle_outputs
 
 pytestmark = pytest.mark.gpu
 
@@ -51,6 +51,7 @@ def test_first_block_prefetch_from_file(tmp_path):
     for rep in range(3):
         got = fr.run(x)
         assert all(a.tobytes() == b.tobytes() for a, b in zip(got, rs)), rep
+    check_oracle(fr, got, x)
 
 
 def test_resident_prefix_from_file(tmp_path):
@@ -64,6 +65,7 @@ def test_resident_prefix_from_file(tmp_path):
     for rep in range(3):
         got = fr.run(x)
         assert all(a.tobytes() == b.tobytes() for a, b in zip(got, rs)), rep
+    check_oracle(fr, got, x)
 
 
 def test_resident_plan_and_adaptation_from_file(tmp_path):
@@ -76,6 +78,7 @@ def test_resident_plan_and_adaptation_from_file(tmp_path):
         r.engine.adapt(capi.Plan.partition(d, int(OP.weight_bytes(m) * frac) // 256 * 256, capi.options()))
         got = r.run(x)
         assert all(a.tobytes() == b.tobytes() for a, b in zip(got, ref))
+        check_oracle(r, got, x)
 
 
 def test_read_failure_inside_an_inference_is_reported(tmp_path):

@@ -122,6 +122,34 @@ def test_activations_and_residual_order():
     assert F.run_layer(layer, "f32", w, acts, x)[0, 0, 0, 0] == 1.0          # relu(-3) + 1
 
 
+def test_swiglu_branch_closed_forms():
+    """SwiGLU layer (Sec. 10 names LLaMA-7B; its FFN is down(silu(gate x) *
+    up x)): the layer with act swiglu is the up projection and its residual
+    operand is the stored gate output r, so y = silu(r) * (acc + b).  One
+    hand-worked case tells apart the plausible mistakes: acc = 1.5, b = 0.5,
+    r = -1 gives silu(-1) * 2 = -2 / (1 + e) = -0.5378828427399902; swapping
+    the gate and up roles would give silu(2) * (-1) = -1.7615941559557649,
+    dropping the bias silu(-1) * 1.5 = -0.4034121320549927."""
+    layer = dict(op="linear", src=[-1], k=1, n=1, act="swiglu", res=0, res_post=False)
+    w = [np.array([[1.0]], dtype=np.float32), np.array([0.5], dtype=np.float32)]
+    x = np.array([[[[1.5]]]])
+    got = F.run_layer(layer, "f32", w, {0: np.array([[[[-1.0]]]])}, x)[0, 0, 0, 0]
+    np.testing.assert_allclose(got, -0.5378828427399902, rtol=1e-7)
+    # a zero gate closes the branch whatever the up projection gives
+    assert F.run_layer(layer, "f32", w, {0: np.array([[[[0.0]]]])}, x)[0, 0, 0, 0] == 0.0
+    # a large negative gate closes it too; a large positive one passes
+    # r * (acc + b): silu(r) -> r as r grows
+    assert abs(F.run_layer(layer, "f32", w, {0: np.array([[[[-60.0]]]])}, x)[0, 0, 0, 0]) < 1e-20
+    np.testing.assert_allclose(F.run_layer(layer, "f32", w, {0: np.array([[[[40.0]]]])}, x)[0, 0, 0, 0],
+                               80.0, rtol=1e-7)
+    # the branch is elementwise over features: gate [0, -1] and acc + b [5, 2]
+    layer2 = dict(layer, k=2, n=2)
+    w2 = [np.array([[1.0, 0.0], [0.0, 1.0]], dtype=np.float32), np.array([0.5, 0.5], dtype=np.float32)]
+    x2 = np.array([[[[4.5]], [[1.5]]]])
+    got2 = F.run_layer(layer2, "f32", w2, {0: np.array([[[[0.0]], [[-1.0]]]])}, x2).reshape(-1)
+    np.testing.assert_allclose(got2, [0.0, -0.5378828427399902], rtol=1e-7, atol=0)
+
+
 def test_rounding_ties_and_values():
     # fp16: 1 + 2^-11 is a tie between 1 and 1 + 2^-10 -> even (1)
     assert F.round_as(1 + 2.0 ** -11, "f16") == 1.0

@@ -56,6 +56,34 @@ def test_eq1_selfdriving_budgets_consistent():
     assert all(abs(float(a) - b) < 1.0 for a, b in zip(A, budgets))
 
 
+def _one_linear(mid, n):
+    return dict(name="mlp6", model_id=mid, dtype="f32", input=(1, 1, 1, 256), outputs=[0],
+                layers=[dict(op="linear", src=[-1], k=256, n=n, act="none", res=None, res_post=False,
+                             bias=False)])
+
+
+def test_schedule_performance_scores_hand_worked():
+    """schedule(): PS_i = u_i * latency_i / M_i (Sec. 6.2.2 beside Eq. 1),
+    hand-worked.  Model A holds 256 x 256 fp32 weights (262144 B), model B
+    256 x 512 (524288 B); their DInf latencies are set to 1000 and 4000 ns;
+    the budget is M = 393216 B, half the 786432 B demanded (n = 2).
+      u = (1, 1): PS_A = 1000/262144, PS_B = 4000/524288 = 2 PS_A, so the
+        score shares are 1/3 and 2/3 and
+        A_A = (1/3)(1/2)M + (1/3)(1/2)M = 65536 + 65536 = 131072,
+        A_B = (2/3)(1/2)M + (2/3)(1/2)M = 262144.
+      u = (3, 1): score shares 3/5 and 2/5:
+        A_A = 65536 + 117964.8 -> 183296 after flooring to 256 bytes,
+        A_B = 131072 + 78643.2 -> 209664.
+    PS = u * M / latency would give A_A = 196608 for u = (1, 1), and
+    PS = u * latency (no division by the memory) 104857.6 -> 104704."""
+    ms = [_one_linear(81, 256), _one_linear(82, 512)]
+    assert [P.weight_bytes(m) for m in ms] == [262144, 524288]
+    coef = P.Coef(2_500_000, 0, 2000, 0)
+    ovr = [[1000], [4000]]
+    assert P.schedule(ms, [1, 1], 393216, coef, t_ex_overrides=ovr) == [131072, 262144]
+    assert P.schedule(ms, [3, 1], 393216, coef, t_ex_overrides=ovr) == [183296, 209664]
+
+
 def test_eq1_within_budget_returns_demands():
     assert P.eq1_split([3, 4], [1, 1], 10) == [3, 4]
 
