@@ -2,8 +2,12 @@
 
 A step is one swapped inference of the workload: every block's weights are
 swapped from pinned host memory into the two-slot device arena and every
-layer runs from the arena.  Default workload: the ResNet-50-shaped CNN at
-batch 1 with a device budget of 40 % of its weight bytes.
+layer runs from the arena.  Default workload: the LLaMA-7B-shaped bf16
+decoder (13.5 GB of weights) through a 4e9-byte weight arena, one step =
+the prefill of 512 token ids plus 32 greedy decode passes; every other
+workload (the MLP, ResNet-50, VGG-16 at batch 1 and 16, YOLOv3, the
+multi-DNN mix) is measured after it in the same call and reported under
+the line's `configs` key (--configs none skips them).
 
 Reported (one JSON line, rank 0):
   value        whole-job inferences/s (device-timed, inputs resident in HBM)
@@ -334,6 +338,42 @@ def llm_cpu_sample(n_dec_sample=2):
                    "prefill and %d decode tokens, scaled to 32 layers and 32 decode tokens" % n_dec_sample)
 
 
+def decoder_unit_bytes(model, units, positions):
+    """Algorithmic bytes of each unit of a decoder pass over `positions`
+    cached positions after it: parameters, every input read and the output
+    written, each once (the attention layer reads the cached keys and values
+    of all positions once)."""
+    es = 2
+    rows = model["input"][0]
+    width = {}
+    out = []
+    for u in units:
+        L = model["layers"][u["layer"]]
+        op = L["op"]
+        if op == "embed":
+            b = 2 * rows * L["d"] * es            # rows gathered from the host table, written
+            width[u["layer"]] = L["d"]
+        elif op == "rmsnorm":
+            b = u["bytes"] + 2 * rows * L["d"] * es
+            width[u["layer"]] = L["d"]
+        elif op == "linear":
+            frac = u["rows"] / L["n"] if u["rows"] else 1.0
+            # input rows, output rows, and the residual (or SwiGLU gate) rows
+            outs = 2 if L.get("res") is not None else 1
+            b = u["bytes"] + rows * L["k"] * es + outs * rows * L["n"] * es * frac
+            width[u["layer"]] = L["n"]
+        elif op == "attention":
+            d = width[L["src"][0]]
+            b = 4 * rows * d * es + 2 * positions * d * es   # q, k, v in, out; the whole cache read
+            width[u["layer"]] = d
+        elif op == "argmax":
+            b = rows * width[L["src"][0]] * es + rows * 4
+        else:
+            b = u["bytes"]
+        out.append(int(b))
+    return out
+
+
 def run_llm(args, rank, world, group):
     """Config 5: prefill of 512 ids then 32 greedy decode steps per step."""
     import torch
@@ -358,10 +398,10 @@ def run_llm(args, rank, world, group):
     ip, idd = pp.info(), pd.info()
     ep, ed = capi.Engine(pp, host), capi.Engine(pd, host)
     rpp = capi.Plan.resident(dp, capi.options(merge=args.merge))
+    rdp = capi.Plan.resident(dd, capi.options(preloaded=1, merge=args.merge))
     arena = torch.empty(rpp.info()["arena_bytes"], dtype=torch.uint8, device="cuda")
     rp = capi.Engine(rpp, host, d_arena=arena.data_ptr(), arena_bytes=arena.numel())
-    rd = capi.Engine(capi.Plan.resident(dd, capi.options(preloaded=1, merge=args.merge)), host,
-                     d_arena=arena.data_ptr(), arena_bytes=arena.numel())
+    rd = capi.Engine(rdp, host, d_arena=arena.data_ptr(), arena_bytes=arena.numel())
     state = torch.zeros(ip["state_bytes"], dtype=torch.uint8, device="cuda")
     for e in (ep, ed, rp, rd):
         e.bind_state(state.data_ptr(), ip["state_bytes"])
@@ -373,14 +413,16 @@ def run_llm(args, rank, world, group):
     offs_p, offs_d = pp.output_offsets(), pd.output_offsets()
     n_dec = 32
 
-    def one(eng_p, eng_d, evs=None):
+    def one(eng_p, eng_d, evs=None, after_pass=None):
         state[:256].zero_()
         if evs: evs[0].record(stream)
         eng_p.infer(in_p.data_ptr(), out_p.data_ptr(), sp)
+        if after_pass: after_pass(0)
         if evs: evs[1].record(stream)
         tok[:4].copy_(out_p[offs_p[1] + 511 * 4:offs_p[1] + 512 * 4])
         for _ in range(n_dec):
             eng_d.infer(tok.data_ptr(), out_d.data_ptr(), sp)
+            if after_pass: after_pass(1)
             tok[:4].copy_(out_d[offs_d[1]:offs_d[1] + 4])
         if evs: evs[2].record(stream)
 
@@ -416,6 +458,68 @@ def run_llm(args, rank, world, group):
     # greedy tokens agree between swapped and resident runs
     one(ep, ed); torch.cuda.synchronize(); sw_tok = int(tok[:4].cpu().numpy().view(np.int32)[0])
     one(rp, rd); torch.cuda.synchronize(); rs_tok = int(tok[:4].cpu().numpy().view(np.int32)[0])
+
+    # ---- the dominant kernel: one step with profiling on (eager launches,
+    # events around every unit kernel and every block's swap-in on the copy
+    # stream); per pass, per-block swap times and per-unit kernel times
+    units_p, units_d = pp.units(), pd.units()
+    kinds_p, kinds_d = ep.unit_kernels(), ed.unit_kernels()
+    blocks_p, blocks_d = pp.blocks(), pd.blocks()
+    var_p = [b["variant"] for b in ep.blocks()]
+    var_d = [b["variant"] for b in ed.blocks()]
+    prof = {"swap": [], "kern": {}}
+
+    def collect(which):
+        eng, units, blocks, kinds, var = ((ep, units_p, blocks_p, kinds_p, var_p) if which == 0
+                                          else (ed, units_d, blocks_d, kinds_d, var_d))
+        u_us, s_us = eng.last_times(len(units), len(blocks))
+        for b, t, v in zip(blocks, s_us, var):
+            prof["swap"].append((b["bytes"], t, v))
+        for k, t in zip(kinds, u_us):
+            prof["kern"][k] = prof["kern"].get(k, 0.0) + t
+
+    for e in (ep, ed):
+        e.set_profiling(True)
+    one(ep, ed, after_pass=collect)
+    torch.cuda.synchronize()
+    for e in (ep, ed):
+        e.set_profiling(False)
+    zc = [(b, t) for b, t, v in prof["swap"] if v == capi.SWAP_ZEROCOPY and t > 0]
+    swap_us_step = sum(t for _, t, _ in prof["swap"])
+    step_us = (statistics.mean(r[0] for r in sw) + n_dec * statistics.mean(r[1] for r in sw)) * 1e3
+    if zc:
+        zb, zt = sum(b for b, _ in zc), sum(t for _, t in zc)
+        zc_us_step = zt
+        ach = zb / (zt * 1e-6) / 1e9
+        roofline = {
+            "bound": "host_link", "kernel": "zerocopy_kernel", "achieved": ach, "peak": link_peak, "unit": "GB/s",
+            "frac": ach / link_peak,
+            "peak_source": "pinned cudaMemcpy H2D of 256 MiB measured in this run (MEASURED_PEAKS.json has no "
+                           "host-link figure)",
+            "launches_per_step": len(zc), "algorithmic_bytes_per_launch": zb // len(zc),
+            "us_per_launch": zt / len(zc), "us_per_step": zt, "step_us": step_us,
+            "timing": "CUDA events on the copy stream around each block's swap-in, one profiled step",
+            "share_of_step": zt / step_us,
+            "kernel_time_share_eager": {k: round(v / (zt + sum(prof["kern"].values())), 4)
+                                        for k, v in list(prof["kern"].items()) + [("zerocopy_kernel", zt)]},
+            "traffic": None}
+        tr = TRAFFIC.get(("llm", "zerocopy_kernel"))
+        if tr and tr[0] == sources_sha(("k_swap.cu",)):
+            roofline["traffic"] = int(tr[1] * (zb // len(zc)))
+            roofline["traffic_note"] = "ncu DRAM bytes per byte swapped on a smaller capture, times the bytes of a launch"
+    else:
+        roofline = None
+
+    # ---- the resident (DInf) kernels: every unit timed as a graph of 20
+    # back-to-back launches, grouped by kernel family, per decoder step
+    hbm, tf_burst, tf_sust, peak_src = load_peaks()
+    us_rp = np.array(rp.measure_units(len(rpp.units()), 20))
+    us_rd = np.array(rd.measure_units(len(rdp.units()), 20))
+    fam_p = kernel_rooflines(rp.unit_kernels(), rpp.units(), us_rp, decoder_unit_bytes(mp, rpp.units(), 512),
+                             hbm, tf_burst, peak_src)
+    fam_d = kernel_rooflines(rd.unit_kernels(), rdp.units(), us_rd, decoder_unit_bytes(md, rdp.units(), 528),
+                             hbm, tf_burst, peak_src)
+
     # e2e through swapnet_infer_host: the token ids from pinned host memory,
     # every pass's output back to the host, and each greedy token taken from
     # the host copy for the next decode pass
@@ -435,8 +539,9 @@ def run_llm(args, rank, world, group):
             h_tok[:4].copy_(h_out_d[offs_d[1]:offs_d[1] + 4])
 
     one_host()
+    e2e_steps = min(args.steps, 5)
     e2e_ms = []
-    for _ in range(args.steps):
+    for _ in range(e2e_steps):
         t0 = time.perf_counter()
         one_host()
         e2e_ms.append((time.perf_counter() - t0) * 1e3)
@@ -452,56 +557,63 @@ def run_llm(args, rank, world, group):
         e_.bind_state(state.data_ptr(), ip["state_bytes"])
     one(ep_rp, ed_rp)
     torch.cuda.synchronize()
-    rp_t = timed(ep_rp, ed_rp, args.steps)
+    rp_t = timed(ep_rp, ed_rp, min(args.steps, 3))
     ext_rp = {"prefill_ms": statistics.mean(r[0] for r in rp_t),
               "decode_ms_per_token": statistics.mean(r[1] for r in rp_t),
               "prefix_units": [pp_rp.info()["prefix_units"], pd_rp.info()["prefix_units"]],
-              "prefix_bytes": [pp_rp.info()["prefix_bytes"], pd_rp.info()["prefix_bytes"]]}
+              "prefix_bytes": [pp_rp.info()["prefix_bytes"], pd_rp.info()["prefix_bytes"]], "steps": len(rp_t)}
     ext_rp["ms_per_step"] = ext_rp["prefill_ms"] + n_dec * ext_rp["decode_ms_per_token"]
     one(ep_rp, ed_rp); torch.cuda.synchronize()
     ext_rp["greedy_token_equals_resident"] = int(tok[:4].cpu().numpy().view(np.int32)[0]) == rs_tok
+    ep_rp.free(); ed_rp.free()
     pre_ms = statistics.mean(r[0] for r in sw)
     dec_ms = statistics.mean(r[1] for r in sw)
     pre_d = statistics.mean(r[0] for r in di)
     dec_d = statistics.mean(r[1] for r in di)
     step_ms = group.max(pre_ms + n_dec * dec_ms)  # the slowest rank
     dinf_ms = pre_d + n_dec * dec_d
-    swap_bytes_p = sum(b["bytes"] for b in pp.blocks())
-    swap_bytes_d = sum(b["bytes"] for b in pd.blocks())
+    swap_bytes_p = sum(b["bytes"] for b in blocks_p)
+    swap_bytes_d = sum(b["bytes"] for b in blocks_d)
     bytes_step = swap_bytes_p + n_dec * swap_bytes_d
     bound_ms = bytes_step / (link_peak * 1e9) * 1e3
+    unit = "inferences/s (prefill 512 + 32 decode)"
     line = {
-        "metric": METRIC, "value": world * 1000.0 / step_ms, "unit": "inferences/s (prefill 512 + 32 decode)",
+        "metric": METRIC, "value": world * 1000.0 / step_ms, "unit": unit,
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": text, "budget_bytes": budget, "weight_bytes": ip["weight_bytes"],
                    "prefill_blocks": ip["n_blocks"], "decode_blocks": idd["n_blocks"],
                    "plans_exact": [ip["exact"], idd["exact"]], "l2": "inputs (13.2 GB of weights) larger than L2",
-                   "swap_variant": args.variant, "merged_gemv_launches": args.merge,
-                   "state_bytes": ip["state_bytes"]},
+                   "swap_variant": args.variant, "swap_variants_prefill": var_p, "swap_variants_decode": var_d,
+                   "merged_gemv_launches": args.merge, "state_bytes": ip["state_bytes"]},
         "prefill_ms": pre_ms, "decode_ms_per_token": dec_ms, "dinf_prefill_ms": pre_d,
         "dinf_decode_ms_per_token": dec_d, "dinf_ms": dinf_ms, "ratio": step_ms / dinf_ms,
         "greedy_token_swapped_equals_resident": sw_tok == rs_tok,
-        "e2e": {"value": world * 1000.0 / e2e_step_ms, "unit": "inferences/s (prefill 512 + 32 decode)",
+        "e2e": {"value": world * 1000.0 / e2e_step_ms, "unit": unit, "steps": e2e_steps,
                 "h2d_bytes_per_step": ip["input_bytes"] + n_dec * idd["input_bytes"],
                 "d2h_bytes_per_step": ip["output_bytes"] + n_dec * idd["output_bytes"],
                 "greedy_token_equals_device_run": e2e_tok_equal},
         "link": {"achieved_gbs": bytes_step / (step_ms * 1e-3) / 1e9, "peak_gbs": link_peak,
                  "peak_source": "pinned cudaMemcpy H2D 256 MiB", "bytes_per_step": bytes_step,
+                 "swap_busy_gbs": bytes_step / (swap_us_step * 1e-6) / 1e9 if swap_us_step > 0 else None,
                  "peak_before_after_gbs": [link_before, link_after]},
         "per_step": {"prefill_ms": [r[0] for r in sw], "decode_ms_per_token": [r[1] for r in sw],
                      "dinf_prefill_ms": [r[0] for r in di], "dinf_decode_ms_per_token": [r[1] for r in di]},
         "step_roofline": {"bound": "host link", "bound_ms": bound_ms, "frac": bound_ms / step_ms},
+        "roofline": roofline,
+        "kernel_rooflines": {"dinf_prefill_pass": fam_p, "dinf_decode_pass": fam_d,
+                             "timing": "unit graphs of 20 back-to-back launches (swapnet_engine_measure_units)"},
         "gpu_launches": launches, "clocks": clk,
         "setup_s": {"weights": t_gen, "plans": t_plan},
         "extension_resident_prefix": ext_rp,
     }
+    rp.free(); rd.free()
+    del arena
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         tot, sample = llm_cpu_sample()
-        line["cpu_baseline"] = {"value": 1.0 / tot, "unit": "inferences/s", "cores": len(os.sched_getaffinity(0)),
+        line["cpu_baseline"] = {"value": 1.0 / tot, "unit": unit, "cores": len(os.sched_getaffinity(0)),
                                 "kind": "oracle", "sample": sample}
-    if rank == 0:
-        print(json.dumps(line))
+    return line if rank == 0 else {}
 
 
 def run_multi(args, rank, world, group):
@@ -628,8 +740,9 @@ def run_multi(args, rank, world, group):
                           else "tensor", "bound_ms": bound_ms, "frac": bound_ms / (wall_sw / args.steps)},
         "gpu_launches": launches, "clocks": clk,
     }
-    if rank == 0:
-        print(json.dumps(line))
+    for e in engs + rengs:
+        e.free()
+    return line if rank == 0 else {}
 
 
 def measure_link_peak(stream):
@@ -663,7 +776,7 @@ def run_ablation(args):
     d = capi.Desc(m)
     plan0 = capi.Plan.partition(d, budget, capi.options(activations_in_budget=act_in))
     eng0 = capi.Engine(plan0, host)
-    t_ex, alpha = capi.calibrate(m, plan0, eng0)
+    t_ex, alpha = capi.calibrate(m, eng0)
     eng0.free()
     dc = capi.Desc(m, t_ex_ns=t_ex)
     base = dict(activations_in_budget=act_in, alpha_as_per_byte=alpha or 4_750_000, beta_ns_per_tensor=0,
@@ -738,7 +851,7 @@ def run_adapt_study(args):
     # offline profiling once (Sec. 6.1), then the look-up table of plans
     plan0 = capi.Plan.partition(d, int(wb * fracs[-1]) // 256 * 256, capi.options())
     eng0 = capi.Engine(plan0, host)
-    t_ex, alpha = capi.calibrate(m, plan0, eng0)
+    t_ex, alpha = capi.calibrate(m, eng0)
     eng0.free()
     dc = capi.Desc(m, t_ex_ns=t_ex)
     opt = capi.options(alpha_as_per_byte=alpha or 4_750_000, beta_ns_per_tensor=0, eta_ns_per_tensor=0)
@@ -823,7 +936,7 @@ def run_storage(args):
         opt0 = capi.options(slots=2, activations_in_budget=act_in)
         plan0 = capi.Plan.partition(d, budget, opt0)
         eng0 = capi.Engine(plan0, wf)
-        t_ex, alpha = capi.calibrate(m, plan0, eng0)
+        t_ex, alpha = capi.calibrate(m, eng0)
         eng0.free()
         opt = capi.options(slots=2, activations_in_budget=act_in, alpha_as_per_byte=alpha or 4_750_000,
                            beta_ns_per_tensor=0, eta_ns_per_tensor=0)
@@ -896,7 +1009,14 @@ def run_profile_once(args):
     else:
         m, w, x, wb, budget, text = build_workload(args.config, capi_weight_bytes)
         host = capi.HostWeights(w)
-    plan = capi.Plan.resident(capi.Desc(m))
+    if args.profile_swapped:
+        # one swapped pass through an arena of half the weight bytes, with
+        # the swap variant of --variant (the zero-copy kernel's captures)
+        wbytes = capi.Plan.resident(capi.Desc(m)).info()["weight_bytes"]
+        plan = capi.Plan.partition(capi.Desc(m), wbytes // 2 // 256 * 256,
+                                   capi.options(swap_variant=variant_code(args.variant)))
+    else:
+        plan = capi.Plan.resident(capi.Desc(m))
     info = plan.info()
     eng = capi.Engine(plan, host)
     if info["state_bytes"]:
@@ -907,7 +1027,9 @@ def run_profile_once(args):
     d_out = torch.empty(info["output_bytes"], dtype=torch.uint8, device="cuda")
     eng.infer(d_in.data_ptr(), d_out.data_ptr(), torch.cuda.current_stream().cuda_stream)
     eng.sync()
-    print(json.dumps({"profile_once": args.config, "kernels": eng.unit_kernels(), "tiling": eng.unit_tiling()}))
+    print(json.dumps({"profile_once": args.config, "kernels": eng.unit_kernels(), "tiling": eng.unit_tiling(),
+                      "blocks": [dict(b, bytes=pb["bytes"]) for b, pb in zip(eng.blocks(), plan.blocks())]
+                      if args.profile_swapped else None}))
 
 
 def run_reference(args, rank, world):
@@ -948,14 +1070,15 @@ def run_reference(args, rank, world):
         ms = 1000.0 * sum(times) / len(times)
         val = 1000.0 / ms
         sample = llm_cpu_sample.__doc__.split("Returns")[0].strip()
+        unit = "inferences/s (prefill 512 + 32 decode)"
         print(json.dumps({
-            "impl": "reference", "metric": METRIC, "value": val, "unit": "inferences/s", "n_gpus": world,
+            "impl": "reference", "metric": METRIC, "value": val, "unit": unit, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": CONFIGS["llm"][3], "budget_bytes": 4_000_000_000, "l2": "n/a (CPU)"},
-            "cpu_baseline": {"value": val, "unit": "inferences/s", "cores": cores, "kind": "oracle",
+            "cpu_baseline": {"value": val, "unit": unit, "cores": cores, "kind": "oracle",
                              "sample": " ".join(sample.split())},
-            "e2e": {"value": val, "unit": "inferences/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "e2e": {"value": val, "unit": unit, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
         }))
         return
     m, w, x, wb, budget, text = build_workload(args.config, oracle_weight_bytes)
@@ -987,7 +1110,10 @@ def main():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="swapnet", choices=["swapnet", "reference"])
-    ap.add_argument("--config", default="resnet50", choices=sorted(CONFIGS))
+    ap.add_argument("--config", default="llm", choices=sorted(CONFIGS))
+    ap.add_argument("--configs", default="mlp6,resnet50,vgg16_b1,vgg16_b16,yolov3,multi",
+                    help="other configs measured after the main line (N=1 only) and reported under its "
+                         "'configs' key; 'none' to skip")
     ap.add_argument("--variant", default="auto", choices=VARIANTS)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile-layers", type=int, default=2,
@@ -1004,6 +1130,9 @@ def main():
     ap.add_argument("--storage", default=None, metavar="DIR",
                     help="storage tier: write --config's weights to a file in DIR and read every swapped block "
                          "from it with O_DIRECT; prints one JSON line")
+    ap.add_argument("--profile-swapped", action="store_true",
+                    help="with --profile-once: one swapped pass (arena of half the weight bytes, --variant) "
+                         "instead of a resident one")
     ap.add_argument("--profile-once", action="store_true",
                     help="run one resident inference of --config through the C ABI and exit "
                          "(a driver for profiler captures of its kernels); prints one JSON line")
@@ -1028,28 +1157,67 @@ def main():
     if args.storage:
         run_storage(args)
         return
-    if args.config in ("llm", "multi"):
-        import torch
-        torch.cuda.set_device(local)
-        group = RankGroup(world, local)
-        import __graft_entry__
-        __graft_entry__.build()
-        (run_llm if args.config == "llm" else run_multi)(args, rank, world, group)
-        group.close()
-        return
-
     import torch
     torch.cuda.set_device(local)
     group = RankGroup(world, local)
-
     import __graft_entry__
     __graft_entry__.build()
-    from paper_2401_16757_gb300 import capi
+    if args.config == "llm":
+        line = run_llm(args, rank, world, group)
+    elif args.config == "multi":
+        line = run_multi(args, rank, world, group)
+    else:
+        line = run_cnn(args, rank, world, group, args.config)
+    extra = [c for c in args.configs.split(",") if c and c != "none" and c != args.config]
+    if extra and world == 1:
+        # every other config measured in the same call, after the main line's
+        # engines and buffers are released
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+        line["configs"] = {}
+        for c in extra:
+            sub = argparse.Namespace(**vars(args))
+            sub.config = c
+            sub.steps = min(args.steps, 30)
+            sub.warmup = 3
+            sub.no_cpu_baseline = True
+            t0 = time.perf_counter()
+            if c == "multi":
+                r = run_multi(sub, rank, world, group)
+            else:
+                r = run_cnn(sub, rank, world, group, c, compact=True)
+            r = compact_line(r)
+            r["wall_s"] = time.perf_counter() - t0
+            line["configs"][c] = r
+            torch.cuda.synchronize()
+            torch.cuda.empty_cache()
+    if rank == 0:
+        print(json.dumps(line))
+    group.close()
 
-    m, w, x, wb, budget, text = build_workload(args.config, capi_weight_bytes)
+
+def compact_line(r):
+    """The keys of a config's line kept under the main line's `configs`."""
+    keep = ("value", "unit", "ms_per_step", "p50_ms", "dinf_ms", "ratio", "dinf_ms_per_step", "throughput_ratio",
+            "per_model", "link", "step_roofline", "roofline", "strict_budget", "gpu_launches", "clocks", "steps",
+            "config", "e2e")
+    return {k: r[k] for k in keep if k in r}
+
+
+def run_cnn(args, rank, world, group, name, compact=False):
+    """One single-model config (the CNNs and the MLP): the plan is made on a
+    delay model calibrated on this GPU (Sec. 6.1), then swapped and
+    all-resident latency, e2e, link rate and rooflines; the strict budget
+    reading (activations inside the budget) for the CNNs; and unless compact
+    the uncalibrated plan, the extension and prefetch lines and the CPU
+    baseline.  Returns the line (rank 0)."""
+    import torch
+    from paper_2401_16757_gb300 import capi
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    m, w, x, wb, budget, text = build_workload(name, capi_weight_bytes)
     d = capi.Desc(m)
     variant = variant_code(args.variant)
-    act_in = 1 if args.config == "mlp6" else 0
+    act_in = 1 if name == "mlp6" else 0
     opt0 = capi.options(slots=2, activations_in_budget=act_in, swap_variant=variant)
     host = capi.HostWeights(w)
     rplan = capi.Plan.resident(d)
@@ -1061,40 +1229,33 @@ def main():
     d_in[:rinfo["input_bytes"]].copy_(torch.from_numpy(x.view(np.uint8).reshape(-1)))
     d_out = torch.empty(rinfo["output_bytes"], dtype=torch.uint8, device="cuda")
     flush = torch.empty(512 << 20, dtype=torch.uint8, device="cuda")
-    # offline profiling (Sec. 6.1): plan with default coefficients, measure
-    # every layer's execution delay (scaled to the resident latency measured
-    # here) and the link on this GPU, then plan again
-    for _ in range(3):
-        reng.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
-    rts = []
-    for _ in range(20):
-        flush.zero_()
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        reng.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
-        b.record(stream)
-        b.synchronize()
-        rts.append(a.elapsed_time(b))
-    plan0 = capi.Plan.partition(d, budget, opt0)
-    eng0 = capi.Engine(plan0, host)
-    t_ex, alpha = capi.calibrate(m, plan0, eng0, resident_ns=statistics.median(rts) * 1e6)
-    dc = capi.Desc(m, t_ex_ns=t_ex)
-    opt = capi.options(slots=2, activations_in_budget=act_in, swap_variant=variant,
-                       alpha_as_per_byte=alpha or 4_750_000, beta_ns_per_tensor=0, eta_ns_per_tensor=0)
-    plan = capi.Plan.partition(dc, budget, opt)
-    info = plan.info()
-    eng = capi.Engine(plan, host)
 
-    def timed(engine, steps, flush_l2=True):
+    def timed(engine, steps, flush_l2=True, out=None):
         evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
         for a, b in evs:
             if flush_l2:
                 flush.zero_()
             a.record(stream)
-            engine.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
+            engine.infer(d_in.data_ptr(), (out if out is not None else d_out).data_ptr(), sp)
             b.record(stream)
         torch.cuda.synchronize()
         return [a.elapsed_time(b) for a, b in evs]
+
+    # offline profiling (Sec. 6.1): plan with default coefficients, measure
+    # every layer's execution delay (scaled to the resident latency measured
+    # here) and the link on this GPU, then plan again
+    for _ in range(3):
+        reng.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
+    rts = timed(reng, 20)
+    plan0 = capi.Plan.partition(d, budget, opt0)
+    eng0 = capi.Engine(plan0, host)
+    t_ex, alpha = capi.calibrate(m, eng0, resident_ns=statistics.median(rts) * 1e6)
+    dc = capi.Desc(m, t_ex_ns=t_ex)
+    coef = dict(alpha_as_per_byte=alpha or 4_750_000, beta_ns_per_tensor=0, eta_ns_per_tensor=0)
+    opt = capi.options(slots=2, activations_in_budget=act_in, swap_variant=variant, **coef)
+    plan = capi.Plan.partition(dc, budget, opt)
+    info = plan.info()
+    eng = capi.Engine(plan, host)
 
     # cold: the engine's first inference (CUDA graph capture and
     # instantiation included), host wall time to its completion
@@ -1130,49 +1291,6 @@ def main():
     # ---- DInf: same kernels, weights resident
     ms_dinf_list = timed(reng, args.steps)
     ms_dinf = sum(ms_dinf_list) / len(ms_dinf_list)
-    # ---- the plan made with the default (uncalibrated) coefficients
-    for _ in range(3):
-        eng0.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
-    ms_uncal_list = timed(eng0, min(args.steps, 50))
-    ms_uncal = sum(ms_uncal_list) / len(ms_uncal_list)
-    # ---- extension (not the paper's method): the first units stay resident
-    # in the arena between inferences, the rest swap through the region left
-    opt_rp = capi.options(slots=2, activations_in_budget=act_in, swap_variant=variant,
-                          alpha_as_per_byte=alpha or 4_750_000, beta_ns_per_tensor=0, eta_ns_per_tensor=0,
-                          resident_prefix=1)
-    plan_rp = capi.Plan.partition(dc, budget, opt_rp)
-    eng_rp = capi.Engine(plan_rp, host)
-    for _ in range(3):
-        eng_rp.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
-    ms_rp_list = timed(eng_rp, min(args.steps, 50))
-    ext_rp = {"ms": sum(ms_rp_list) / len(ms_rp_list), "prefix_units": plan_rp.info()["prefix_units"],
-              "prefix_bytes": plan_rp.info()["prefix_bytes"], "n_blocks": plan_rp.info()["n_blocks"],
-              "swapped_bytes_per_step": sum(b["bytes"] for b in plan_rp.blocks()[1 if plan_rp.info()["prefix_units"] else 0:])}
-    eng_rp.free()
-    # ---- steady state with first-block prefetch: each inference swaps the
-    # next one's first block in at its end (the cyclic objective)
-    opt_pf = capi.options(slots=2, activations_in_budget=act_in, swap_variant=variant,
-                          alpha_as_per_byte=alpha or 4_750_000, beta_ns_per_tensor=0, eta_ns_per_tensor=0,
-                          prefetch=1)
-    plan_pf = capi.Plan.partition(dc, budget, opt_pf)
-    eng_pf = capi.Engine(plan_pf, host)
-    pf_out = torch.empty_like(d_out)
-    for _ in range(3):
-        eng_pf.infer(d_in.data_ptr(), pf_out.data_ptr(), sp)
-    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
-    for a, b in evs:
-        flush.zero_()
-        a.record(stream)
-        eng_pf.infer(d_in.data_ptr(), pf_out.data_ptr(), sp)
-        b.record(stream)
-    torch.cuda.synchronize()
-    ms_pf_list = [a.elapsed_time(b) for a, b in evs]
-    eng_pf.sync()
-    first_block_prefetch = {"ms": sum(ms_pf_list) / len(ms_pf_list), "p50_ms": statistics.median(ms_pf_list),
-                            "n_blocks": plan_pf.info()["n_blocks"], "cuts": plan_pf.cuts(),
-                            "predicted_ms": plan_pf.info()["predicted_ns"] / 1e6, "exact": plan_pf.info()["exact"],
-                            "bit_exact_vs_cold": bool(torch.equal(pf_out, d_out))}
-    eng_pf.free()
 
     # ---- e2e: host buffers through swapnet_infer_host
     h_in = torch.empty(info["input_bytes"], dtype=torch.uint8, pin_memory=True)
@@ -1193,111 +1311,187 @@ def main():
     e2e_val = 1000.0 / (sum(e2e_ms) / len(e2e_ms))
     clk = clocks.stop()
 
-    # ---- profiled pass: per-unit kernel and per-block swap times
+    line = {}
+    if not compact:
+        # ---- the plan made with the default (uncalibrated) coefficients
+        for _ in range(3):
+            eng0.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
+        ms_uncal_list = timed(eng0, min(args.steps, 50))
+        line["uncalibrated_plan"] = {"cuts": plan0.cuts(), "ms": sum(ms_uncal_list) / len(ms_uncal_list)}
+        # ---- extension (not the paper's method): the first units stay
+        # resident in the arena between inferences, the rest swap through
+        # the region left
+        plan_rp = capi.Plan.partition(dc, budget, capi.options(slots=2, activations_in_budget=act_in,
+                                                                swap_variant=variant, resident_prefix=1, **coef))
+        eng_rp = capi.Engine(plan_rp, host)
+        for _ in range(3):
+            eng_rp.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
+        ms_rp_list = timed(eng_rp, min(args.steps, 50))
+        ri = plan_rp.info()
+        line["extension_resident_prefix"] = {
+            "ms": sum(ms_rp_list) / len(ms_rp_list), "prefix_units": ri["prefix_units"],
+            "prefix_bytes": ri["prefix_bytes"], "n_blocks": ri["n_blocks"],
+            "swapped_bytes_per_step": sum(b["bytes"] for b in plan_rp.blocks()[1 if ri["prefix_units"] else 0:])}
+        eng_rp.free()
+        # ---- steady state with first-block prefetch: each inference swaps
+        # the next one's first block in at its end (the cyclic objective)
+        plan_pf = capi.Plan.partition(dc, budget, capi.options(slots=2, activations_in_budget=act_in,
+                                                                swap_variant=variant, prefetch=1, **coef))
+        eng_pf = capi.Engine(plan_pf, host)
+        pf_out = torch.empty_like(d_out)
+        for _ in range(3):
+            eng_pf.infer(d_in.data_ptr(), pf_out.data_ptr(), sp)
+        ms_pf_list = timed(eng_pf, args.steps, out=pf_out)
+        eng_pf.sync()
+        pi = plan_pf.info()
+        line["first_block_prefetch"] = {
+            "ms": sum(ms_pf_list) / len(ms_pf_list), "p50_ms": statistics.median(ms_pf_list),
+            "n_blocks": pi["n_blocks"], "cuts": plan_pf.cuts(), "predicted_ms": pi["predicted_ns"] / 1e6,
+            "exact": pi["exact"], "bit_exact_vs_cold": bool(torch.equal(pf_out, d_out))}
+        eng_pf.free()
+    eng0.free()
+
+    # ---- stricter budget reading: the activation workspace inside the
+    # budget as well (the same budget if a plan fits it, else the smallest
+    # budget in steps of 5 % of the weight bytes that does)
+    strict = None
+    if name != "mlp6":
+        opt_s = capi.options(slots=2, activations_in_budget=1, swap_variant=variant, **coef)
+        b_s, plan_s = budget, None
+        while plan_s is None and b_s <= wb + info["workspace_bytes"] + (1 << 20):
+            try:
+                plan_s = capi.Plan.partition(dc, b_s, opt_s)
+            except capi.SwapnetError as e_:
+                if e_.code != capi.ERR_INFEASIBLE:
+                    raise
+                b_s = (b_s + int(0.05 * wb)) // 256 * 256
+        if plan_s is not None:
+            eng_s = capi.Engine(plan_s, host)
+            for _ in range(3):
+                eng_s.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
+            ms_s = statistics.mean(timed(eng_s, args.steps))
+            si = plan_s.info()
+            strict = {"budget_bytes": b_s, "budget_frac_of_weights": b_s / wb, "arena_bytes": si["arena_bytes"],
+                      "workspace_bytes": si["workspace_bytes"],
+                      "arena_plus_workspace_bytes": si["arena_bytes"] + si["workspace_bytes"],
+                      "n_blocks": si["n_blocks"], "ms": ms_s, "ratio": ms_s / ms_dinf,
+                      "swapped_bytes_per_step": sum(b["bytes"] for b in plan_s.blocks())}
+            eng_s.free()
+
+    # ---- kernel rooflines: each unit's kernels timed as a CUDA graph of
+    # back-to-back launches (the dependent-launch overlap of a real
+    # inference, no events between launches), grouped by kernel family
     units = plan.units()
     blocks = plan.blocks()
     kinds = eng.unit_kernels()
-    eng.set_profiling(True)
-    prof_steps = min(20, args.steps)
-    acc_u = np.zeros(len(units))
-    acc_s = np.zeros(len(blocks))
-    for _ in range(prof_steps):
-        flush.zero_()
-        eng.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
-        u_us, s_us = eng.last_times(len(units), len(blocks))
-        acc_u += np.array(u_us)
-        acc_s += np.array(s_us)
-    eng.set_profiling(False)
-    acc_u /= prof_steps
-    acc_s /= prof_steps
-    share = {}
-    for k, t in zip(kinds, acc_u):
-        share[k] = share.get(k, 0.0) + t
-    dom = max(share, key=share.get)
-    dom_idx = [i for i, k in enumerate(kinds) if k == dom]
-    dom_flops = sum(units[i]["flops"] for i in dom_idx)
-    dom_us = sum(acc_u[i] for i in dom_idx)
+    unit_us = np.array(eng.measure_units(len(units), 20))
     hbm, tf_burst, tf_sust, peak_src = load_peaks()
-    # the binding roof of the dominant kernel family: tensor FLOPs when its
-    # algorithmic FLOPs per byte reach the ridge point (peak FLOP/s over
-    # peak bytes/s), HBM bytes otherwise
     ubytes = unit_algorithmic_bytes(m, units)
-    dom_bytes = sum(ubytes[i] for i in dom_idx) if ubytes else 0
-    ridge = tf_burst * 1e12 / (hbm * 1e9)
-    tensor_bound = dom_flops > 0 and (not dom_bytes or dom_flops / dom_bytes >= ridge)
-    if tensor_bound:
-        achieved = dom_flops / (dom_us * 1e-6) / 1e12 if dom_us > 0 else 0.0
-        roofline = {"bound": "tensor", "achieved": achieved, "peak": tf_burst, "unit": "TFLOP/s",
-                    "peak_source": peak_src + " bf16 burst"}
-    else:
-        achieved = dom_bytes / (dom_us * 1e-6) / 1e9 if dom_us > 0 else 0.0
-        roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                    "peak_source": peak_src + " copy"}
-    roofline.update({"kernel": dom, "launches_per_step": len(dom_idx), "frac": achieved / roofline["peak"],
-                     "algorithmic_flops_per_step": dom_flops, "algorithmic_bytes_per_step": dom_bytes,
-                     "algorithmic_bytes_per_launch": dom_bytes // max(1, len(dom_idx)),
-                     "flops_per_byte": dom_flops / dom_bytes if dom_bytes else None, "ridge_flops_per_byte": ridge,
+    fam = kernel_rooflines(kinds, units, unit_us, ubytes, hbm, tf_burst, peak_src)
+    dom = max(fam, key=lambda k: fam[k]["us_per_step"])
+    roofline = dict(fam[dom])
+    roofline.update({"kernel": dom, "timing": "unit graphs of 20 back-to-back launches (swapnet_engine_measure_units)",
+                     "family_us_per_step_vs_step_us": [roofline["us_per_step"], ms_swapped * 1e3],
                      "traffic": None, "kernel_sources_sha": kernel_sources_sha(),
                      "traffic_sources_sha": traffic_sources_sha(),
-                     "share_of_kernel_time": dom_us / max(1e-9, acc_u.sum()),
-                     "kernel_time_share": {k: round(v / max(1e-9, acc_u.sum()), 4) for k, v in share.items()}})
-    tr = TRAFFIC.get((args.config, dom))
+                     "kernel_time_share": {k: round(v["us_per_step"] / max(1e-9, unit_us.sum()), 4)
+                                           for k, v in fam.items()}})
+    tr = TRAFFIC.get((name, dom))
     if tr and tr[0] == roofline["traffic_sources_sha"]:
         roofline["traffic"] = tr[1]
 
-    # ---- host link: bytes per swap over swap time, against pinned memcpy peak
+    # ---- host link: one profiled pass per step (events around each swap on
+    # the copy stream), bytes per swap over swap time, against the pinned
+    # memcpy peak
+    eng.set_profiling(True)
+    acc_s = np.zeros(len(blocks))
+    prof_steps = min(10, args.steps)
+    for _ in range(prof_steps):
+        flush.zero_()
+        eng.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
+        acc_s += np.array(eng.last_times(len(units), len(blocks))[1])
+    eng.set_profiling(False)
+    acc_s /= prof_steps
     swap_bytes = sum(b["bytes"] for b in blocks)
     swap_us = float(acc_s.sum())
-    pk = torch.empty(256 << 20, dtype=torch.uint8, pin_memory=True)
-    dv = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
-    best = 1e9
-    for _ in range(5):
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        dv.copy_(pk, non_blocking=True)
-        b.record(stream)
-        b.synchronize()
-        best = min(best, a.elapsed_time(b))
-    link_peak = (256 << 20) / (best / 1000.0) / 1e9
+    link_peak = measure_link_peak(stream)
     link_gbs = swap_bytes / (swap_us * 1e-6) / 1e9 if swap_us > 0 else None
     # roofline of the whole step (slower of tensor FLOPs and swapped bytes over the link)
     flops = sum(u["flops"] for u in units)
     step_bound_ms = max(flops / (tf_burst * 1e12), swap_bytes / (link_peak * 1e9)) * 1e3
+    if strict is not None:
+        sb = max(flops / (tf_burst * 1e12), strict["swapped_bytes_per_step"] / (link_peak * 1e9)) * 1e3
+        strict["step_roofline"] = {"bound_ms": sb, "frac": sb / strict["ms"]}
 
     cpu = None
-    if rank == 0 and not args.no_cpu_baseline:
+    if rank == 0 and not args.no_cpu_baseline and not compact:
         cpu = cpu_oracle_baseline(m, w, x)
 
-    if rank == 0:
-        eb = eng.blocks()
-        line = {
-            "metric": METRIC, "value": value, "unit": "inferences/s", "n_gpus": world, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": ms_swapped, "higher_is_better": True, "scaling": "weak",
-            "vs_baseline": None, "dtype": "f32" if m["dtype"] == "f32" else m["dtype"], "data": "synthetic",
-            "config": {"workload": text, "budget_bytes": budget, "weight_bytes": wb,
-                       "n_blocks": info["n_blocks"], "cuts": plan.cuts(), "slot_bytes": info["slot_bytes"],
-                       "workspace_bytes": info["workspace_bytes"], "l2": "flushed (512 MiB write) before each step",
-                       "swap_variants": [b["variant"] for b in eb], "parallelism": "replicas" if world > 1 else "1 GPU"},
-            "dinf_ms": ms_dinf, "ratio": ms_swapped / ms_dinf,
-            "predicted_ms": info["predicted_ns"] / 1e6,
-            "uncalibrated_plan": {"cuts": plan0.cuts(), "ms": ms_uncal},
-            "extension_resident_prefix": ext_rp,
-            "first_block_prefetch": first_block_prefetch,
-            "p50_ms": statistics.median(ms_list), "p99_ms": float(np.percentile(ms_list, 99)),
-            "cold_first_inference_ms": cold_ms,
-            "e2e": {"value": e2e_val, "unit": "inferences/s", "h2d_bytes_per_step": info["input_bytes"],
-                    "d2h_bytes_per_step": info["output_bytes"]},
-            "link": {"achieved_gbs": link_gbs, "peak_gbs": link_peak, "peak_source": "pinned cudaMemcpy H2D 256 MiB",
-                     "frac": (link_gbs / link_peak) if link_gbs else None, "bytes_per_step": swap_bytes},
-            "step_roofline": {"bound_ms": step_bound_ms, "frac": step_bound_ms / ms_swapped},
-            "roofline": roofline,
-            "gpu_launches": launches,
-            "clocks": clk,
-            "cpu_baseline": cpu,
-            "wall_s_timed": t_wall,
-        }
-        print(json.dumps(line))
-    group.close()
+    if rank != 0:
+        return {}
+    eb = eng.blocks()
+    line.update({
+        "metric": METRIC, "value": value, "unit": "inferences/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_swapped, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32" if m["dtype"] == "f32" else m["dtype"], "data": "synthetic",
+        "config": {"workload": text, "budget_bytes": budget, "weight_bytes": wb,
+                   "n_blocks": info["n_blocks"], "cuts": plan.cuts(), "slot_bytes": info["slot_bytes"],
+                   "workspace_bytes": info["workspace_bytes"], "l2": "flushed (512 MiB write) before each step",
+                   "swap_variants": [b["variant"] for b in eb], "parallelism": "replicas" if world > 1 else "1 GPU"},
+        "dinf_ms": ms_dinf, "ratio": ms_swapped / ms_dinf,
+        "predicted_ms": info["predicted_ns"] / 1e6,
+        "p50_ms": statistics.median(ms_list), "p99_ms": float(np.percentile(ms_list, 99)),
+        "cold_first_inference_ms": cold_ms,
+        "e2e": {"value": e2e_val, "unit": "inferences/s", "h2d_bytes_per_step": info["input_bytes"],
+                "d2h_bytes_per_step": info["output_bytes"]},
+        "link": {"achieved_gbs": link_gbs, "peak_gbs": link_peak, "peak_source": "pinned cudaMemcpy H2D 256 MiB",
+                 "frac": (link_gbs / link_peak) if link_gbs else None, "bytes_per_step": swap_bytes},
+        "step_roofline": {"bound_ms": step_bound_ms, "frac": step_bound_ms / ms_swapped},
+        "strict_budget": strict,
+        "roofline": roofline,
+        "kernel_rooflines": fam,
+        "gpu_launches": launches,
+        "clocks": clk,
+        "cpu_baseline": cpu,
+        "wall_s_timed": t_wall,
+    })
+    eng.free()
+    reng.free()
+    return line
+
+
+def kernel_rooflines(kinds, units, unit_us, ubytes, hbm, tf_burst, peak_src):
+    """Per kernel family: launches, time per step, algorithmic FLOPs and bytes,
+    and the roof that binds it.  The binding roof is the tensor pipe when the
+    family's algorithmic FLOPs per byte reach the ridge point (peak FLOP/s
+    over peak bytes/s), HBM bandwidth otherwise.  ubytes: algorithmic bytes
+    per unit, or None where the workload's layer types have no count."""
+    ridge = tf_burst * 1e12 / (hbm * 1e9)
+    fam = {}
+    for i, k in enumerate(kinds):
+        f = fam.setdefault(k, {"launches_per_step": 0, "us_per_step": 0.0, "flops": 0, "bytes": 0})
+        f["launches_per_step"] += 1
+        f["us_per_step"] += float(unit_us[i])
+        f["flops"] += units[i]["flops"]
+        f["bytes"] += ubytes[i] if ubytes else 0
+    out = {}
+    for k, f in fam.items():
+        us = f["us_per_step"]
+        tensor = f["flops"] > 0 and (not f["bytes"] or f["flops"] / f["bytes"] >= ridge)
+        if tensor:
+            ach = f["flops"] / (us * 1e-6) / 1e12 if us > 0 else 0.0
+            r = {"bound": "tensor", "achieved": ach, "peak": tf_burst, "unit": "TFLOP/s",
+                 "peak_source": peak_src + " bf16 burst (fp16 has the same dense rate)"}
+        else:
+            ach = f["bytes"] / (us * 1e-6) / 1e9 if us > 0 else 0.0
+            r = {"bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s", "peak_source": peak_src + " copy"}
+        n = max(1, f["launches_per_step"])
+        r.update({"frac": ach / r["peak"], "launches_per_step": f["launches_per_step"], "us_per_step": us,
+                  "us_per_launch": us / n, "algorithmic_flops_per_launch": f["flops"] // n,
+                  "algorithmic_bytes_per_launch": f["bytes"] // n,
+                  "flops_per_byte": f["flops"] / f["bytes"] if f["bytes"] else None, "ridge_flops_per_byte": ridge})
+        out[k] = r
+    return out
 
 
 if __name__ == "__main__":

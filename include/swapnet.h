@@ -514,6 +514,27 @@ int swapnet_engine_set_profiling(swapnet_engine* eng, int enable);
 int swapnet_engine_measure_units(swapnet_engine* eng, int32_t reps, float* unit_us, uint32_t n_units);
 int swapnet_engine_last_times(swapnet_engine* eng, float* unit_us, uint32_t n_units, float* swap_us,
                               uint32_t n_blocks);
+
+/* The offline fit of the delay model on this device (Sec. 6.1: the paper
+ * profiles each device once and fits t_ex = gamma * f and t_in = alpha * s +
+ * beta * d by linear regression).  Here the execution delays are measured
+ * per layer instead of fitted per FLOP:
+ *   t_ex_ns[l] (n_layers entries, the model's layer count) = the summed
+ *     swapnet_engine_measure_units time of layer l's units (reps launches
+ *     each), at least 1 ns; when resident_ns > 0 (the measured latency of
+ *     the same model with every weight resident), every t_ex is scaled so
+ *     that they add up to it, since units timed alone miss the launch and
+ *     cache effects of the whole dependent chain;
+ *   alpha_as_per_byte = the copy-engine swap-in times measured at load
+ *     (SWAPNET_SWAP_AUTO engines) over those blocks' bytes, in attoseconds
+ *     per byte; 0 when the engine measured none.
+ * The results are meant for swapnet_layer.t_ex_ns and
+ * swapnet_options.alpha_as_per_byte of the next swapnet_partition (with
+ * beta_ns_per_tensor 0: the per-block times already contain it).
+ * Synchronous.  Errors: INVALID_ARG (n_layers other than the model's), OOM,
+ * CUDA. */
+int swapnet_engine_calibrate(swapnet_engine* eng, int32_t reps, int64_t resident_ns, int64_t* t_ex_ns,
+                             uint32_t n_layers, uint64_t* alpha_as_per_byte);
 /* Start and end of every unit kernel and block swap-in of the most recent
  * profiled inference, in microseconds after the first of those events
  * (arrays of n_units and n_blocks entries; swap entries are 0 for a
@@ -557,10 +578,19 @@ void swapnet_engine_free(swapnet_engine* eng);
  * different streams, or on the same device from several threads) race on
  * the array and must be serialised by the caller.
  *
+ * Ordering: the kernel starts only after the work queued before it on
+ * `stream` has completed (no programmatic early start), so A, W and bias may
+ * be the output of the previous call or kernel on the stream.
+ *
  * Set-up: the first call on a device looks up the array's device address
  * (cudaGetSymbolAddress) with that device current and caches it; make that
  * first call before any stream capture.
- * Errors: INVALID_ARG, MISALIGNED, UNSUPPORTED, CUDA. */
+ * Errors: INVALID_ARG, MISALIGNED, UNSUPPORTED, CUDA.  Device-side failures
+ * are not returned by this call, which does not wait for its kernel: if a
+ * bounded wait inside the kernel gives up (one second), Y is incomplete and
+ * the timeout is recorded in the library's device error word, which the
+ * next swapnet_engine_sync (of any engine on the device) reports as
+ * SWAPNET_ERR_TIMEOUT and clears. */
 #define SWAPNET_NOALLOC_SCRATCH_BYTES (4u << 20)
 int swapnet_gemm_noalloc(int32_t dtype, const void* A, const void* W, const void* bias, void* Y, int32_t M,
                          int32_t N, int32_t K, int32_t act, swapnet_stream stream);

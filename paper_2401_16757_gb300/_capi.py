@@ -98,7 +98,7 @@ EXPORTS = ["swapnet_default_options", "swapnet_partition", "swapnet_plan_from_cu
            "swapnet_infer", "swapnet_infer_host", "swapnet_engine_sync", "swapnet_engine_blocks",
            "swapnet_engine_free", "swapnet_engine_stats_get", "swapnet_engine_unit_kernels", "swapnet_engine_unit_tiling", "swapnet_engine_adapt", "swapnet_host_alloc", "swapnet_host_free",
            "swapnet_engine_set_profiling", "swapnet_engine_last_times", "swapnet_engine_measure_units",
-           "swapnet_engine_last_timeline",
+           "swapnet_engine_last_timeline", "swapnet_engine_calibrate",
            "swapnet_engine_bind_state", "swapnet_strerror", "swapnet_last_error", "swapnet_debug_fail_next", "swapnet_gemm_noalloc",
            "swapnet_weights_file_write", "swapnet_weights_file_open", "swapnet_weights_file_info",
            "swapnet_weights_file_read", "swapnet_weights_file_close", "swapnet_load_file",
@@ -157,6 +157,8 @@ def lib():
                                                    C.POINTER(C.c_float), C.POINTER(C.c_float), C.c_uint32]),
         "swapnet_engine_last_times": (C.c_int, [P, C.POINTER(C.c_float), C.c_uint32, C.POINTER(C.c_float),
                                                 C.c_uint32]),
+        "swapnet_engine_calibrate": (C.c_int, [P, C.c_int32, C.c_int64, C.POINTER(C.c_int64), C.c_uint32,
+                                               C.POINTER(C.c_uint64)]),
         "swapnet_strerror": (C.c_char_p, [C.c_int]),
         "swapnet_last_error": (C.c_char_p, []),
         "swapnet_debug_fail_next": (C.c_int, [C.c_int, C.c_int]),
@@ -322,32 +324,17 @@ def schedule(descs, urgency, arena_bytes, opt=None):
     return list(budgets), [Plan(p) for p in plans]
 
 
-def calibrate(model, plan, engine, reps=20, resident_ns=None):
-    """Measured delay model (Sec. 6.1) from a loaded engine: per-layer t_ex
-    in ns (sum of the layer's units) and alpha in attoseconds per byte from
-    the per-block copy times measured at load.  Each unit is timed alone
-    (a graph of `reps` launches of it); resident_ns, the measured latency of
-    the same model with every weight resident, rescales the t_ex so that
-    they add up to it (the units run as one dependent chain there, with the
-    launch and cache effects that timing a unit alone leaves out).  Returns
-    (t_ex_ns list, alpha_as_per_byte or None)."""
-    units = plan.units()
-    us = engine.measure_units(len(units), reps)
-    t_ex = [0] * len(model["layers"])
-    for u, t in zip(units, us):
-        t_ex[u["layer"]] += int(round(t * 1000.0))
-    t_ex = [max(1, v) for v in t_ex]
-    if resident_ns:
-        f = resident_ns / float(sum(t_ex))
-        t_ex = [max(1, int(round(v * f))) for v in t_ex]
-    alpha = None
-    blocks = plan.blocks()
-    eb = engine.blocks()
-    tot_b = sum(b["bytes"] for b, e in zip(blocks, eb) if e["memcpy_us"] > 0)
-    tot_us = sum(e["memcpy_us"] for e in eb if e["memcpy_us"] > 0)
-    if tot_b > 0 and tot_us > 0:
-        alpha = int(round(tot_us * 1e12 / tot_b))
-    return t_ex, alpha
+def calibrate(model, engine, reps=20, resident_ns=None):
+    """swapnet_engine_calibrate (Sec. 6.1 delay model measured on this GPU):
+    per-layer t_ex in ns and alpha in attoseconds per byte (None when the
+    engine measured no copy-engine swap).  resident_ns: the measured
+    all-resident latency the t_ex are scaled to, or None."""
+    n = len(model["layers"])
+    t_ex = (C.c_int64 * n)()
+    alpha = C.c_uint64()
+    check(lib().swapnet_engine_calibrate(engine.h, int(reps), int(resident_ns or 0), t_ex, n,
+                                         C.byref(alpha)), "swapnet_engine_calibrate")
+    return list(t_ex), (alpha.value or None)
 
 
 def gemm_noalloc(dtype, a_ptr, w_ptr, bias_ptr, y_ptr, M, N, K, act=0, stream=0):

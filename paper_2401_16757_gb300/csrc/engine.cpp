@@ -1532,6 +1532,41 @@ int swapnet_engine_measure_units(swapnet_engine* e, int32_t reps, float* unit_us
   return SWAPNET_OK;
 }
 
+int swapnet_engine_calibrate(swapnet_engine* e, int32_t reps, int64_t resident_ns, int64_t* t_ex_ns,
+                             uint32_t n_layers, uint64_t* alpha_as_per_byte) {
+  if (!e || !t_ex_ns || !alpha_as_per_byte || resident_ns < 0) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad argument");
+  const swapnet_plan& p = e->plan;
+  if (n_layers != p.model.L.size()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "t_ex_ns needs one entry per layer");
+  std::vector<float> us(p.units.size(), 0.f);
+  int rc = swapnet_engine_measure_units(e, reps, us.data(), (uint32_t)us.size());
+  if (rc) return rc;
+  // t_ex per layer: the sum of its units' launch times (a split linear
+  // layer's pieces run one after another)
+  std::vector<int64_t> t(n_layers, 0);
+  for (size_t u = 0; u < p.units.size(); ++u) t[p.units[u].layer] += (int64_t)llround((double)us[u] * 1000.0);
+  for (auto& v : t) v = std::max<int64_t>(1, v);
+  if (resident_ns > 0) {
+    // a unit timed alone runs faster than inside the dependent chain of a
+    // whole inference: scale the t_ex so they add up to the measured
+    // all-resident latency
+    double sum = 0.0;
+    for (int64_t v : t) sum += (double)v;
+    const double f = (double)resident_ns / sum;
+    for (auto& v : t) v = std::max<int64_t>(1, (int64_t)llround((double)v * f));
+  }
+  // alpha: the copy-engine time of every block measured at load over its bytes
+  double bytes = 0.0, copy_us = 0.0;
+  for (size_t k = 0; k < e->blocks.size() && k < p.blocks.size(); ++k) {
+    if (e->blocks[k].memcpy_us <= 0.f) continue;
+    bytes += (double)p.blocks[k].bytes;
+    copy_us += (double)e->blocks[k].memcpy_us;
+  }
+  const uint64_t alpha = (bytes > 0.0 && copy_us > 0.0) ? (uint64_t)llround(copy_us * 1e12 / bytes) : 0;
+  std::copy(t.begin(), t.end(), t_ex_ns);
+  *alpha_as_per_byte = alpha;
+  return SWAPNET_OK;
+}
+
 int swapnet_engine_bind_state(swapnet_engine* e, void* d_state, uint64_t bytes) {
   if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
   if (!e->plan.model.has_attention) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "the model has no decoder state");

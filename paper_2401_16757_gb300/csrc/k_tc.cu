@@ -538,12 +538,12 @@ double conv_patch(int ho, int wo, int stride, int* wt, int* ht) {
 
 template <typename T, int BN, int AMODE>
 int launch_inst(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) {
-  static bool attr_done = false;  // per instantiation
+  static std::atomic<uint64_t> attr_done{0};  // per instantiation, one bit per device
   auto kern = tc_gemm_kernel<T, BN, AMODE>;
-  if (!attr_done) {
+  if (attr_needed(attr_done)) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<BN>::kSmem) != cudaSuccess)
       SN_FAIL(SWAPNET_ERR_CUDA, "cudaFuncSetAttribute failed");
-    attr_done = true;
+    attr_set(attr_done);
   }
   TcArgs a;
   std::memset(&a, 0, sizeof(a));
@@ -565,11 +565,11 @@ int launch_inst(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) {
   a.cluster = pl.cluster;
   const bool csplit = pl.splits > 1 && pl.cluster;
   if (csplit) {
-    static bool np_done = false;  // per instantiation
-    if (!np_done) {
+    static std::atomic<uint64_t> np_done{0};  // per instantiation, one bit per device
+    if (attr_needed(np_done)) {
       if (cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)
         SN_FAIL(SWAPNET_ERR_CUDA, "non-portable cluster attribute failed");
-      np_done = true;
+      attr_set(np_done);
     }
   }
   cudaLaunchConfig_t cfg;
@@ -580,9 +580,11 @@ int launch_inst(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) {
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   int na = 0;
-  attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[na].val.programmaticStreamSerializationAllowed = 1;
-  ++na;
+  if (!g.no_pdl) {
+    attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+  }
   if (csplit) {
     attr[na].id = cudaLaunchAttributeClusterDimension;
     attr[na].val.clusterDim.x = 1;
@@ -938,6 +940,9 @@ extern "C" int swapnet_gemm_noalloc(int32_t dtype, const void* A, const void* W,
   g.e.bias = bias; g.e.res = nullptr; g.e.ldr = N; g.e.act = act; g.e.res_post = 0;
   g.y = Y; g.ldy = N;
   g.num_sms = d.sms;
+  // W and bias are caller memory that the previous work on the stream (an
+  // earlier call, say) may have written: no early start before it completes
+  g.no_pdl = 1;
   TcPlan pl;
   int rc = tc_prepare(g, &pl);
   if (rc) return rc;

@@ -406,12 +406,12 @@ __global__ void __launch_bounds__(persist_threads<AMODE>(), 1)
 
 template <typename T, int BN, int AMODE, int MS>
 int launch_persist_inst(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) {
-  static bool attr_done = false;  // per instantiation
+  static std::atomic<uint64_t> attr_done{0};  // per instantiation, one bit per device
   auto kern = tc_persist_kernel<T, BN, AMODE, MS>;
-  if (!attr_done) {
+  if (attr_needed(attr_done)) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, PCfg<BN, MS>::kSmem) != cudaSuccess)
       SN_FAIL(SWAPNET_ERR_CUDA, "cudaFuncSetAttribute failed");
-    attr_done = true;
+    attr_set(attr_done);
   }
   TcArgs a;
   std::memset(&a, 0, sizeof(a));
@@ -435,7 +435,7 @@ int launch_persist_inst(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = g.no_pdl ? 0 : 1;
   const cudaError_t le = cudaLaunchKernelEx(&cfg, kern, pl.tmA, pl.tmB, a);
   if (le != cudaSuccess) SN_FAIL(SWAPNET_ERR_CUDA, std::string("persistent GEMM launch: ") + cudaGetErrorString(le));
   return SWAPNET_OK;

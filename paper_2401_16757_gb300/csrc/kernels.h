@@ -4,9 +4,29 @@
 #pragma once
 #include <cuda.h>
 #include <cuda_runtime.h>
+#include <atomic>
 #include <cstdint>
 
 namespace swapnet {
+
+// Kernel attributes (dynamic shared memory size, cluster permissions) are
+// set per function and per device.  A launcher keeps one bit per device in
+// `done`: attr_needed() says whether the current device still lacks the
+// attribute, attr_set() records it once cudaFuncSetAttribute succeeded.
+// Two threads racing on a first launch may both set it, which is harmless.
+inline uint64_t device_bit() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    cudaGetLastError();
+    return 0;  // unknown device: always set the attribute
+  }
+  return 1ull << dev;
+}
+inline bool attr_needed(const std::atomic<uint64_t>& done) {
+  const uint64_t b = device_bit();
+  return b == 0 || (done.load(std::memory_order_acquire) & b) == 0;
+}
+inline void attr_set(std::atomic<uint64_t>& done) { done.fetch_or(device_bit(), std::memory_order_acq_rel); }
 
 // Epilogue operands shared by linear and conv layers.
 struct Epi {
@@ -105,6 +125,12 @@ struct TcGemm {
                         // this many CTAs (DSMEM reduction); 0: global scratch
   float* partial;       // split-K scratch (TcPlan::scratch_bytes), set per launch
   int* counters;        // split-K tile counters (TcPlan::tiles ints, zeroed once)
+  int no_pdl;           // 1: launch without programmatic dependent launch.  The
+                        // kernel reads its bias and issues its first weight
+                        // loads before waiting on the previous kernel, which
+                        // is safe only when nothing earlier on the stream
+                        // writes them (the engine's arena); callers whose W or
+                        // bias may come from the kernel just before set this.
 };
 // Pre-encoded descriptors of one GEMM (built once per layer at load time).
 struct TcPlan {

@@ -367,3 +367,41 @@ def test_partition_large_models_fast():
         plan = capi.Plan.partition(capi.Desc(m), wb * 4 // 10 // 256 * 256, capi.options())
         assert time.time() - t0 < 5.0
         assert plan.info()["n_blocks"] >= P.block_count_rule(wb, wb * 4 // 10 // 256 * 256)
+
+
+def test_calibrate_binding_only_marshals(monkeypatch):
+    """capi.calibrate passes its arguments to swapnet_engine_calibrate and
+    returns what the library wrote: the Sec. 6.1 arithmetic (summing unit
+    times per layer, the rescaling to the resident latency, alpha from the
+    copy times) lives behind the C ABI.  A fake library records the call."""
+    seen = {}
+
+    class FakeLib:
+        def swapnet_engine_calibrate(self, h, reps, resident_ns, t_ex, n, alpha):
+            seen.update(h=h, reps=reps, resident_ns=resident_ns, n=n)
+            for i in range(n):
+                t_ex[i] = 1000 + 7 * i
+            alpha._obj.value = 4_750_123
+            return 0
+
+    class FakeEngine:
+        h = "engine-handle"
+
+    m = synth.arch.mlp6()
+    monkeypatch.setattr(capi, "lib", lambda: FakeLib())
+    t_ex, alpha = capi.calibrate(m, FakeEngine(), reps=5, resident_ns=123456)
+    assert seen == dict(h="engine-handle", reps=5, resident_ns=123456, n=len(m["layers"]))
+    assert t_ex == [1000 + 7 * i for i in range(len(m["layers"]))] and alpha == 4_750_123
+
+    class ZeroAlpha(FakeLib):
+        def swapnet_engine_calibrate(self, h, reps, resident_ns, t_ex, n, alpha):
+            return 0
+
+    monkeypatch.setattr(capi, "lib", lambda: ZeroAlpha())
+    assert capi.calibrate(m, FakeEngine())[1] is None   # no copy-engine times measured
+
+
+def test_calibrate_rejects_a_null_engine():
+    t_ex = (capi.C.c_int64 * 3)()
+    alpha = capi.C.c_uint64()
+    assert capi.lib().swapnet_engine_calibrate(None, 5, 0, t_ex, 3, capi.C.byref(alpha)) == capi.ERR_INVALID_ARG
