@@ -449,7 +449,9 @@ def run_llm(args, rank, world, group):
         e.sync()
     launches0 = ep.stats()["kernel_launches"] + ed.stats()["kernel_launches"]
     group.barrier()
+    torch.cuda.nvtx.range_push("swapped_steps")  # ncu --nvtx --nvtx-include swapped_steps/
     sw = timed(ep, ed, args.steps)
+    torch.cuda.nvtx.range_pop()
     group.barrier()
     launches = ep.stats()["kernel_launches"] + ed.stats()["kernel_launches"] - launches0
     di = timed(rp, rd, args.steps)
@@ -511,10 +513,19 @@ def run_llm(args, rank, world, group):
         roofline = None
 
     # ---- the resident (DInf) kernels: every unit timed as a graph of 20
-    # back-to-back launches, grouped by kernel family, per decoder step
+    # back-to-back launches, grouped by kernel family, per decoder step.
+    # The units read the state's position: the prefill's units are timed at
+    # position 0, the decode pass's at 512 (the attention over 513 keys,
+    # near the middle of the 32 decode passes)
     hbm, tf_burst, tf_sust, peak_src = load_peaks()
+    torch.cuda.synchronize()
+    state[:256].zero_()
     us_rp = np.array(rp.measure_units(len(rpp.units()), 20))
+    state[:4].copy_(torch.tensor([512], dtype=torch.int32).view(torch.uint8))
     us_rd = np.array(rd.measure_units(len(rdp.units()), 20))
+    torch.cuda.synchronize()
+    rp.sync()
+    rd.sync()
     fam_p = kernel_rooflines(rp.unit_kernels(), rpp.units(), us_rp, decoder_unit_bytes(mp, rpp.units(), 512),
                              hbm, tf_burst, peak_src)
     fam_d = kernel_rooflines(rd.unit_kernels(), rdp.units(), us_rd, decoder_unit_bytes(md, rdp.units(), 528),
@@ -1001,11 +1012,11 @@ def run_profile_once(args):
     import __graft_entry__
     __graft_entry__.build()
     from paper_2401_16757_gb300 import capi
-    if args.config == "llm":  # one decode pass of a decoder of the 7B widths with --profile-layers layers
-        import synth
-        m = synth.arch.llm(layers=args.profile_layers, tokens=1)
+    if args.config == "llm":  # one pass of --profile-tokens ids through a decoder of the 7B widths
+        import synth                # with --profile-layers layers (1 token: a decode pass)
+        m = synth.arch.llm(layers=args.profile_layers, tokens=args.profile_tokens)
         host = llm_host_weights(m)
-        x = np.array([7], dtype=np.int32)
+        x = synth.gen.model_input(m).reshape(-1) if args.profile_tokens > 1 else np.array([7], dtype=np.int32)
     else:
         m, w, x, wb, budget, text = build_workload(args.config, capi_weight_bytes)
         host = capi.HostWeights(w)
@@ -1118,6 +1129,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--profile-layers", type=int, default=2,
                     help="--profile-once --config llm: decoder layers of the profiled decode pass")
+    ap.add_argument("--profile-tokens", type=int, default=1,
+                    help="--profile-once --config llm: token ids of the profiled pass (1: decode, 512: prefill)")
     ap.add_argument("--merge", type=int, default=1, choices=[0, 1],
                     help="decoder: GEMV layers sharing an input in one launch (1) or one launch each (0)")
     ap.add_argument("--link-share", type=float, default=1.0,
@@ -1182,11 +1195,14 @@ def main():
             sub.warmup = 3
             sub.no_cpu_baseline = True
             t0 = time.perf_counter()
-            if c == "multi":
-                r = run_multi(sub, rank, world, group)
-            else:
-                r = run_cnn(sub, rank, world, group, c, compact=True)
-            r = compact_line(r)
+            try:
+                if c == "multi":
+                    r = run_multi(sub, rank, world, group)
+                else:
+                    r = run_cnn(sub, rank, world, group, c, compact=True)
+                r = compact_line(r)
+            except Exception as ex:   # the main line is reported whatever happens here
+                r = {"error": "%s: %s" % (type(ex).__name__, ex)}
             r["wall_s"] = time.perf_counter() - t0
             line["configs"][c] = r
             torch.cuda.synchronize()

@@ -183,9 +183,10 @@ __global__ void __launch_bounds__(256) rope_append_kernel(T* __restrict__ q, con
 }
 
 // ------------------------------------------------------------ attention
-// Two kernels with the same arithmetic definition; a call with fewer than
-// kRowsMinWarps (query, head) pairs (decode) takes the CTA kernel, longer
-// runs (prefill) the warp kernel.
+// Runs of at least 64 queries (the prefill) take the tcgen05 kernel
+// (k_attn_tc.cu).  Shorter runs take one of two SIMT kernels with the same
+// arithmetic definition: fewer than kRowsMinWarps (query, head) pairs (a
+// decode step) the CTA kernel, more the warp kernel.
 //
 // Short query runs: CTA = one (query t, head h), 512 threads; the scores of all visible keys
 // live in shared memory, so the softmax is exact two-pass (max, then
@@ -483,6 +484,8 @@ int launch_attention(int dtype, void* q, const void* k, const void* v, void* kc,
                              static_cast<T*>(vc), pos_ptr, width, kDh, theta, max_seq, err),
                   "rope launch");
     if (rc) return rc;
+    if (attention_tc_supported(dtype, tokens, heads, width))  // prefill: both contractions on the tensor cores
+      return launch_attention_tc(dtype, q, kc, vc, pos_ptr, tokens, heads, width, max_seq, out, err, s);
     if (tokens * heads >= kRowsMinWarps) {
       const int warps = tokens * heads;
       return done(launch_pdl(attention_rows_kernel<T>, dim3((warps * 32 + 255) / 256), dim3(256), 0, s,

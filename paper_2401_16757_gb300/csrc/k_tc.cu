@@ -880,6 +880,24 @@ std::mutex g_noalloc_mu;
 NoAllocDevice g_noalloc_dev[64];
 }  // namespace
 
+int make_tmap_2d(CUtensorMap* m, int dtype, const void* base, uint64_t inner, uint64_t rows, uint64_t row_stride_bytes,
+                 uint32_t box_inner, uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (!fn) SN_FAIL(SWAPNET_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+  if (((uintptr_t)base & 15) || (row_stride_bytes & 15) || (box_inner * 2) % 16)
+    SN_FAIL(SWAPNET_ERR_MISALIGNED, "TMA operand must be 16-byte aligned with a 16-byte multiple row stride");
+  const cuuint64_t dims[2] = {inner, rows};
+  const cuuint64_t strides[1] = {row_stride_bytes};
+  const cuuint32_t box[2] = {box_inner, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  const CUresult r = fn(m, dtype == SWAPNET_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16,
+                        2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) SN_FAIL(SWAPNET_ERR_CUDA, "cuTensorMapEncodeTiled failed (" + std::to_string((int)r) + ")");
+  return SWAPNET_OK;
+}
+
 int tc_error_word(int** ptr) {
   void* p = nullptr;
   if (cudaGetSymbolAddress(&p, g_tc_err) != cudaSuccess) SN_FAIL(SWAPNET_ERR_CUDA, "cudaGetSymbolAddress failed");

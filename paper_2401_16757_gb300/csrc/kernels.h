@@ -173,4 +173,17 @@ int launch_tc_conv_small(const TcSmallConv& g, int* dev_err, cudaStream_t s);
 // Device error word of the tcgen05 kernels (bounded waits).
 int tc_error_word(int** ptr);
 
+// 2-D TMA map of a row-major fp16/bf16 matrix (inner x rows elements, row
+// stride in bytes), box of box_inner x box_rows elements, 128-byte swizzle,
+// zero fill outside the matrix.  box_inner * 2 bytes must be <= 128.
+int make_tmap_2d(CUtensorMap* m, int dtype, const void* base, uint64_t inner, uint64_t rows, uint64_t row_stride_bytes,
+                 uint32_t box_inner, uint32_t box_rows);
+
+// tcgen05 causal attention for long query runs (prefill): q [tokens][width]
+// (already rotated), key and value caches [max_seq][width], head width 128,
+// query t at position *pos_ptr + t attends to positions 0..*pos_ptr + t.
+bool attention_tc_supported(int dtype, int tokens, int heads, int width);
+int launch_attention_tc(int dtype, const void* q, const void* kc, const void* vc, const int* pos_ptr, int tokens,
+                        int heads, int width, int max_seq, void* out, int* err, cudaStream_t s);
+
 }  // namespace swapnet

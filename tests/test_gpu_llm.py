@@ -124,9 +124,9 @@ def _weights_parallel(model):
 
 def test_llm_full_width_layer_prefill_512_and_decode():
     """The bench's launch configuration at full width on one decoder layer
-    (the float64 oracle of all 32 layers would need 54 GB): 512-token
-    prefill and two greedy decode passes, swapped through a budget of half
-    the weight bytes, against the oracle teacher-forced."""
+    (the whole 32-layer model is tests/test_gpu_llm7b.py): 512-token prefill
+    and two greedy decode passes, swapped through a budget of half the
+    weight bytes, against the oracle teacher-forced."""
     mp = synth.arch.llm(tokens=512, **dict(SMALL, **FULL))
     dec = Decoder(prefill_tokens=512, budget_frac=0.5, weights=_weights_parallel(mp), **FULL)
     ids = synth.gen.model_input(dec.mp).reshape(-1)
@@ -144,7 +144,7 @@ def test_llm_full_width_layer_prefill_512_and_decode():
 
 
 def test_llm_long_prefill_many_heads():
-    """128 queries x 8 heads: the prefill takes the warp-per-query attention
+    """128 queries x 8 heads: the prefill takes the tensor-core attention
     kernel, the decode steps after it the CTA-per-query kernel."""
     dec = Decoder(prefill_tokens=128, **WIDE)
     ids = synth.gen.model_input(dec.mp).reshape(-1)
@@ -160,10 +160,35 @@ def test_llm_long_prefill_many_heads():
         tok = int(toks[0])
 
 
+@pytest.mark.parametrize("d,heads,chunk,max_seq", [
+    (512, 4, 150, 400),    # tensor-core prefill: 2 query tiles (ragged), up to 3 key tiles, second chunk at pos 150
+    (2560, 20, 60, 200),   # 60 queries x 20 heads: the SIMT warp-per-query kernel
+])
+def test_llm_prefill_in_chunks(d, heads, chunk, max_seq):
+    """A prefill engine called twice in a row: the second call's queries
+    start at the cache position the first left (pos0 > 0), so key tiles are
+    not aligned with query tiles and the causal mask cuts tiles in the
+    middle.  Both chunks and a decode step after them against the oracle
+    (its state carried along)."""
+    dec = Decoder(prefill_tokens=chunk, layers=1, d=d, heads=heads, max_seq=max_seq, ffn=688)
+    st = F.new_state()
+    tok = None
+    for c in range(2):
+        ids = synth.gen.model_input(dec.mp, request=c).reshape(-1)
+        ref = F.forward(dec.mp, dec.w, ids.reshape(-1, 1, 1, 1), state=st)
+        logits, toks = dec.run(0, ids)
+        _check_step(logits, toks, ref[0].reshape(chunk, -1), ref[1].reshape(-1), TOL[1])
+        tok = int(toks[-1])
+    ref = F.forward(dec.md, dec.w, np.array([tok], dtype=np.int32).reshape(1, 1, 1, 1), state=st)
+    logits, toks = dec.run(1, np.array([tok], dtype=np.int32))
+    _check_step(logits, toks, ref[0].reshape(1, -1), ref[1].reshape(-1), TOL[1])
+    assert int(dec.state[:4].cpu().numpy().view(np.int32)[0]) == 2 * chunk + 1
+
+
 def test_llm_every_layer_local_parity():
     """Each layer of a resident decoder whose every layer is a model output,
     against the oracle layer run on the GPU's own stored inputs: prefill of
-    128 ids (warp-per-query attention) then two decode steps (CTA-per-query
+    128 ids (tensor-core attention) then two decode steps (CTA-per-query
     attention), the oracle keeping its own KV cache built from the GPU's k
     and v.  The q projection is rotated in place by the attention layer, so
     attention takes the oracle's q computed from the GPU's normalised input."""
