@@ -169,7 +169,8 @@ def test_llm_prefill_in_chunks(d, heads, chunk, max_seq):
     start at the cache position the first left (pos0 > 0), so key tiles are
     not aligned with query tiles and the causal mask cuts tiles in the
     middle.  Both chunks and a decode step after them against the oracle
-    (its state carried along)."""
+    (its state carried along), end to end at the decoder bar (the per-layer
+    check of the same runs is test_llm_every_layer_local_parity)."""
     dec = Decoder(prefill_tokens=chunk, layers=1, d=d, heads=heads, max_seq=max_seq, ffn=688)
     st = F.new_state()
     tok = None
@@ -177,32 +178,39 @@ def test_llm_prefill_in_chunks(d, heads, chunk, max_seq):
         ids = synth.gen.model_input(dec.mp, request=c).reshape(-1)
         ref = F.forward(dec.mp, dec.w, ids.reshape(-1, 1, 1, 1), state=st)
         logits, toks = dec.run(0, ids)
-        _check_step(logits, toks, ref[0].reshape(chunk, -1), ref[1].reshape(-1), TOL[1])
+        _check_step(logits, toks, ref[0].reshape(chunk, -1), ref[1].reshape(-1), CHAIN_TOL)
         tok = int(toks[-1])
     ref = F.forward(dec.md, dec.w, np.array([tok], dtype=np.int32).reshape(1, 1, 1, 1), state=st)
     logits, toks = dec.run(1, np.array([tok], dtype=np.int32))
-    _check_step(logits, toks, ref[0].reshape(1, -1), ref[1].reshape(-1), TOL[1])
+    _check_step(logits, toks, ref[0].reshape(1, -1), ref[1].reshape(-1), CHAIN_TOL)
     assert int(dec.state[:4].cpu().numpy().view(np.int32)[0]) == 2 * chunk + 1
 
 
-def test_llm_every_layer_local_parity():
+@pytest.mark.parametrize("cfg,passes", [
+    (WIDE, (128, 1, 1)),                                               # tensor-core prefill, CTA decode
+    (dict(layers=1, d=512, heads=4, ffn=688, max_seq=400), (150, 150, 1)),   # second prefill at pos0 150
+    (dict(layers=1, d=2560, heads=20, ffn=688, max_seq=200), (60, 60, 1)),   # SIMT warp-per-query prefill
+])
+def test_llm_every_layer_local_parity(cfg, passes):
     """Each layer of a resident decoder whose every layer is a model output,
-    against the oracle layer run on the GPU's own stored inputs: prefill of
-    128 ids (tensor-core attention) then two decode steps (CTA-per-query
-    attention), the oracle keeping its own KV cache built from the GPU's k
-    and v.  The q projection is rotated in place by the attention layer, so
-    attention takes the oracle's q computed from the GPU's normalised input."""
+    against the oracle layer run on the GPU's own stored inputs, over
+    consecutive passes of the given token counts (a second prefill starts at
+    the position the first left), the oracle keeping its own KV cache built
+    from the GPU's k and v.  The q projection is rotated in place by the
+    attention layer, so attention takes the oracle's q computed from the
+    GPU's normalised input."""
     import torch
     w = None
     st_or = F.new_state()
     state = None
-    for tokens in (128, 1, 1):
-        m = synth.arch.llm(tokens=tokens, vocab=SMALL["vocab"], **WIDE)
+    for pi, tokens in enumerate(passes):
+        m = synth.arch.llm(tokens=tokens, vocab=SMALL["vocab"], **cfg)
         m = dict(m, outputs=list(range(len(m["layers"]))))
         if w is None:
             w = synth.gen.model_weights(m)
             host = capi.HostWeights(w)
-            x = synth.gen.model_input(m)
+        if tokens > 1:
+            x = synth.gen.model_input(m, request=pi)
         else:
             x = np.array([[[[next_tok]]]], dtype=np.int32)
         plan = capi.Plan.resident(capi.Desc(m))
