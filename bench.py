@@ -386,7 +386,8 @@ def run_llm(args, rank, world, group):
     t_gen = time.perf_counter() - t0
     stream = torch.cuda.current_stream()
     sp = stream.cuda_stream
-    link_peak = measure_link_peak(stream)
+    placement = {}
+    link_peak = measure_link_peak(stream, placement)
     alpha = int(round(1e18 / (link_peak * 1e9)))
     budget = 4_000_000_000
     variant = variant_code(args.variant)
@@ -486,8 +487,27 @@ def run_llm(args, rank, world, group):
     torch.cuda.synchronize()
     for e in (ep, ed):
         e.set_profiling(False)
-    zc = [(b, t) for b, t, v in prof["swap"] if v == capi.SWAP_ZEROCOPY and t > 0]
-    swap_us_step = sum(t for _, t, _ in prof["swap"])
+    # the swap kernel's own time inside the replayed graphs: one more step
+    # whose graphs carry an event-record node before and after every block's
+    # swap-in on the copy stream (the layer launches are those of the timed
+    # steps)
+    gswap = []
+
+    def collect_graph(which):
+        eng, blocks, var = (ep, blocks_p, var_p) if which == 0 else (ed, blocks_d, var_d)
+        for b, t, v in zip(blocks, eng.last_swap_times(len(blocks)), var):
+            gswap.append((b["bytes"], t, v))
+
+    for e in (ep, ed):
+        e.set_swap_timing(True)
+    one(ep, ed)
+    torch.cuda.synchronize()
+    one(ep, ed, after_pass=collect_graph)
+    torch.cuda.synchronize()
+    for e in (ep, ed):
+        e.set_swap_timing(False)
+    zc = [(b, t) for b, t, v in gswap if v == capi.SWAP_ZEROCOPY and t > 0]
+    swap_us_step = sum(t for _, t, _ in gswap)
     step_us = (statistics.mean(r[0] for r in sw) + n_dec * statistics.mean(r[1] for r in sw)) * 1e3
     if zc:
         zb, zt = sum(b for b, _ in zc), sum(t for _, t in zc)
@@ -500,8 +520,11 @@ def run_llm(args, rank, world, group):
                            "host-link figure)",
             "launches_per_step": len(zc), "algorithmic_bytes_per_launch": zb // len(zc),
             "us_per_launch": zt / len(zc), "us_per_step": zt, "step_us": step_us,
-            "timing": "CUDA events on the copy stream around each block's swap-in, one profiled step",
+            "timing": "CUDA events recorded inside the replayed inference graphs (event-record nodes on the copy "
+                      "stream around each block's swap-in), one step after the timed steps; step_us is the timed "
+                      "steps' mean",
             "share_of_step": zt / step_us,
+            "eager_profiled_us_per_step": sum(t for b, t, v in prof["swap"] if v == capi.SWAP_ZEROCOPY),
             "kernel_time_share_eager": {k: round(v / (zt + sum(prof["kern"].values())), 4)
                                         for k, v in list(prof["kern"].items()) + [("zerocopy_kernel", zt)]},
             "traffic": None}
@@ -607,7 +630,7 @@ def run_llm(args, rank, world, group):
         "link": {"achieved_gbs": bytes_step / (step_ms * 1e-3) / 1e9, "peak_gbs": link_peak,
                  "peak_source": "pinned cudaMemcpy H2D 256 MiB", "bytes_per_step": bytes_step,
                  "swap_busy_gbs": bytes_step / (swap_us_step * 1e-6) / 1e9 if swap_us_step > 0 else None,
-                 "peak_before_after_gbs": [link_before, link_after]},
+                 "peak_before_after_gbs": [link_before, link_after], "host_placement": placement},
         "per_step": {"prefill_ms": [r[0] for r in sw], "decode_ms_per_token": [r[1] for r in sw],
                      "dinf_prefill_ms": [r[0] for r in di], "dinf_decode_ms_per_token": [r[1] for r in di]},
         "step_roofline": {"bound": "host link", "bound_ms": bound_ms, "frac": bound_ms / step_ms},
@@ -756,7 +779,41 @@ def run_multi(args, rank, world, group):
     return line if rank == 0 else {}
 
 
-def measure_link_peak(stream):
+def host_placement(ptr):
+    """Where page-locked host memory sits relative to the GPU (a host-side
+    reading, no GPU setting): the online NUMA nodes, the GPU's node, and the
+    node of the page at `ptr` (move_pages query)."""
+    import ctypes
+    import platform
+    import torch
+
+    def rd(path):
+        try:
+            with open(path) as f:
+                return f.read().strip()
+        except OSError:
+            return None
+    out = {"numa_nodes_online": rd("/sys/devices/system/node/online")}
+    try:
+        p = torch.cuda.get_device_properties(torch.cuda.current_device())
+        bus = "%04x:%02x:%02x.0" % (p.pci_domain_id, p.pci_bus_id, p.pci_device_id)
+    except Exception:
+        bus = None
+    if bus:
+        out["gpu_pci"] = bus.lower()
+        node = rd("/sys/bus/pci/devices/%s/numa_node" % bus.lower())
+        out["gpu_numa_node"] = int(node) if node not in (None, "") else None
+    nr = {"aarch64": 239, "x86_64": 279}.get(platform.machine())
+    if nr is not None:
+        libc = ctypes.CDLL(None, use_errno=True)
+        pages = (ctypes.c_void_p * 1)(ptr & ~4095)
+        status = (ctypes.c_int * 1)(-99)
+        r = libc.syscall(ctypes.c_long(nr), 0, ctypes.c_ulong(1), pages, None, status, 0)
+        out["pinned_page_node"] = status[0] if r == 0 else None
+    return out
+
+
+def measure_link_peak(stream, placement=None):
     import torch
     pk = torch.empty(256 << 20, dtype=torch.uint8, pin_memory=True)
     dv = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
@@ -768,18 +825,25 @@ def measure_link_peak(stream):
         b.record(stream)
         b.synchronize()
         best = min(best, a.elapsed_time(b))
+    if placement is not None:
+        placement.update(host_placement(pk.data_ptr()))
     return (256 << 20) / (best / 1000.0) / 1e9
 
 
 def run_ablation(args):
+    import __graft_entry__
+    __graft_entry__.build()
+    print(json.dumps(ablation_line(args)))
+
+
+def ablation_line(args):
     """Ablations of the partition (the shape of the paper's Sec. 8.4-8.5
     studies) on one single-model config: the planner's plan against
     equal-byte plans with the paper's block count ceil(2s/b) and the next
     four counts, the Eq. 4 objective, strictly sequential layers, and each
-    swap variant forced.  Latency of each (ms, CUDA events, L2 flushed)."""
+    swap variant forced.  Latency of each (median ms, with the 10th and 90th
+    percentiles, CUDA events, L2 flushed)."""
     import torch
-    import __graft_entry__
-    __graft_entry__.build()
     from paper_2401_16757_gb300 import capi
     m, w, x, wb, budget, text = build_workload(args.config, capi_weight_bytes)
     act_in = 1 if args.config == "mlp6" else 0
@@ -815,7 +879,8 @@ def run_ablation(args):
             ts.append(a.elapsed_time(b))
         eng.sync()
         eng.free()
-        return {"ms": statistics.median(ts), "n_blocks": info["n_blocks"], "predicted_ms": info["predicted_ns"] / 1e6}
+        return {"ms": statistics.median(ts), "p10_p90_ms": [float(np.percentile(ts, 10)), float(np.percentile(ts, 90))],
+                "n_blocks": info["n_blocks"], "predicted_ms": info["predicted_ns"] / 1e6}
 
     def try_plan(make):
         try:
@@ -840,19 +905,24 @@ def run_ablation(args):
     out["pageable_staged_copy"] = try_plan(
         lambda: capi.Plan.partition(dc, budget, capi.options(**dict(base, pageable=1))))
     out["resident_dinf"] = try_plan(lambda: capi.Plan.resident(d))
-    print(json.dumps({"ablation": args.config, "workload": text, "budget_bytes": budget, "weight_bytes": wb,
-                      "paper_block_count": n_min, "steps": args.steps, "results": out}))
+    return {"ablation": args.config, "workload": text, "budget_bytes": budget, "weight_bytes": wb,
+            "paper_block_count": n_min, "steps": args.steps, "results": out}
 
 
 def run_adapt_study(args):
+    import __graft_entry__
+    __graft_entry__.build()
+    print(json.dumps(adapt_line(args)))
+
+
+def adapt_line(args):
     """Dynamic-budget case study (the paper's Sec. 8 adaptation experiment,
     on ResNet-50 here): plans for three budgets are made ahead; one engine
     runs `steps` inferences per phase and switches plan between phases with
-    swapnet_engine_adapt.  Reports per phase the budget, blocks, latency,
-    the planning time and the switch time."""
+    swapnet_engine_adapt.  Reports per phase the budget, blocks, latency
+    (median, 10th and 90th percentiles), the planning time and the switch
+    time."""
     import torch
-    import __graft_entry__
-    __graft_entry__.build()
     from paper_2401_16757_gb300 import capi
     name = args.config if args.config in ("resnet50", "vgg16_b1", "yolov3") else "resnet50"
     m, w, x, wb, _, text = build_workload(name, capi_weight_bytes)
@@ -899,11 +969,13 @@ def run_adapt_study(args):
             ts.append(a.elapsed_time(b))
         pi = p.info()
         phases.append({"budget_frac": f, "budget_bytes": pi["budget_bytes"], "n_blocks": pi["n_blocks"],
-                       "cuts": p.cuts(), "ms": statistics.median(ts), "plan_ms": t_plan[i],
+                       "cuts": p.cuts(), "ms": statistics.median(ts),
+                       "p10_p90_ms": [float(np.percentile(ts, 10)), float(np.percentile(ts, 90))],
+                       "plan_ms": t_plan[i],
                        "switch_ms": t_sw, "free_device_bytes": torch.cuda.mem_get_info()[0]})
     eng.sync()
-    print(json.dumps({"adapt_study": name, "workload": text, "weight_bytes": wb, "steps": args.steps,
-                      "phases": phases}))
+    eng.free()
+    return {"adapt_study": name, "workload": text, "weight_bytes": wb, "steps": args.steps, "phases": phases}
 
 
 def run_storage(args):
@@ -1205,6 +1277,21 @@ def main():
                 r = {"error": "%s: %s" % (type(ex).__name__, ex)}
             r["wall_s"] = time.perf_counter() - t0
             line["configs"][c] = r
+            torch.cuda.synchronize()
+            torch.cuda.empty_cache()
+        # the partition ablations and the runtime budget adaptation study on
+        # ResNet-50 (Sec. 8.4-8.5 and the adaptation experiment), same call
+        for key, fn in (("ablation", ablation_line), ("adapt_study", adapt_line)):
+            sub = argparse.Namespace(**vars(args))
+            sub.config = "resnet50"
+            sub.steps = min(args.steps, 30)
+            t0 = time.perf_counter()
+            try:
+                r = fn(sub)
+            except Exception as ex:
+                r = {"error": "%s: %s" % (type(ex).__name__, ex)}
+            r["wall_s"] = time.perf_counter() - t0
+            line[key] = r
             torch.cuda.synchronize()
             torch.cuda.empty_cache()
     if rank == 0:

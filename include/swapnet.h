@@ -515,6 +515,21 @@ int swapnet_engine_measure_units(swapnet_engine* eng, int32_t reps, float* unit_
 int swapnet_engine_last_times(swapnet_engine* eng, float* unit_us, uint32_t n_units, float* swap_us,
                               uint32_t n_blocks);
 
+/* Swap-in time of each block as it runs inside the inference graph that
+ * swapnet_infer replays (Sec. 4.2's t^in, measured in place rather than
+ * with the eager, event-instrumented launches of profiling).  With swap
+ * timing on, the engine captures (and caches) a graph variant that records
+ * an event on the copy stream right before and right after each block's
+ * swap-in; layer launches are unchanged, so the replay is the inference
+ * that swapnet_infer times, plus 2 event-record nodes per swapped block.
+ * swapnet_engine_last_swap_times waits for the most recent inference's last
+ * swap events and writes microseconds per block to swap_us[0..n_blocks)
+ * (0 for blocks that are not swapped: a resident prefix, blocks read in
+ * place, every block of a resident plan).
+ * Errors: INVALID_ARG (null engine or output, timing never enabled), CUDA. */
+int swapnet_engine_set_swap_timing(swapnet_engine* eng, int enable);
+int swapnet_engine_last_swap_times(swapnet_engine* eng, float* swap_us, uint32_t n_blocks);
+
 /* The offline fit of the delay model on this device (Sec. 6.1: the paper
  * profiles each device once and fits t_ex = gamma * f and t_in = alpha * s +
  * beta * d by linear regression).  Here the execution delays are measured

@@ -99,6 +99,7 @@ EXPORTS = ["swapnet_default_options", "swapnet_partition", "swapnet_plan_from_cu
            "swapnet_engine_free", "swapnet_engine_stats_get", "swapnet_engine_unit_kernels", "swapnet_engine_unit_tiling", "swapnet_engine_adapt", "swapnet_host_alloc", "swapnet_host_free",
            "swapnet_engine_set_profiling", "swapnet_engine_last_times", "swapnet_engine_measure_units",
            "swapnet_engine_last_timeline", "swapnet_engine_calibrate",
+           "swapnet_engine_set_swap_timing", "swapnet_engine_last_swap_times",
            "swapnet_engine_bind_state", "swapnet_strerror", "swapnet_last_error", "swapnet_debug_fail_next", "swapnet_gemm_noalloc",
            "swapnet_weights_file_write", "swapnet_weights_file_open", "swapnet_weights_file_info",
            "swapnet_weights_file_read", "swapnet_weights_file_close", "swapnet_load_file",
@@ -152,6 +153,8 @@ def lib():
         "swapnet_engine_unit_kernels": (C.c_int, [P, C.POINTER(C.c_int32), C.c_uint32, C.POINTER(C.c_uint32)]),
         "swapnet_engine_unit_tiling": (C.c_int, [P, C.POINTER(UnitTiling), C.c_uint32, C.POINTER(C.c_uint32)]),
         "swapnet_engine_set_profiling": (C.c_int, [P, C.c_int]),
+        "swapnet_engine_set_swap_timing": (C.c_int, [P, C.c_int]),
+        "swapnet_engine_last_swap_times": (C.c_int, [P, C.POINTER(C.c_float), C.c_uint32]),
         "swapnet_engine_measure_units": (C.c_int, [P, C.c_int32, C.POINTER(C.c_float), C.c_uint32]),
         "swapnet_engine_last_timeline": (C.c_int, [P, C.POINTER(C.c_float), C.POINTER(C.c_float), C.c_uint32,
                                                    C.POINTER(C.c_float), C.POINTER(C.c_float), C.c_uint32]),
@@ -528,6 +531,15 @@ class Engine:
 
     def set_profiling(self, enable):
         check(lib().swapnet_engine_set_profiling(self.h, 1 if enable else 0), "swapnet_engine_set_profiling")
+
+    def set_swap_timing(self, enable):
+        check(lib().swapnet_engine_set_swap_timing(self.h, 1 if enable else 0), "swapnet_engine_set_swap_timing")
+
+    def last_swap_times(self, n_blocks):
+        """Microseconds per block swap-in of the last inference, timed inside its graph."""
+        b = (C.c_float * max(1, n_blocks))()
+        check(lib().swapnet_engine_last_swap_times(self.h, b, n_blocks), "swapnet_engine_last_swap_times")
+        return list(b[:n_blocks])
 
     def measure_units(self, n_units, reps=20):
         u = (C.c_float * max(1, n_units))()

@@ -110,6 +110,10 @@ struct swapnet_engine {
   bool profiling = false;
   std::vector<cudaEvent_t> ev_unit;  // 2 per unit
   std::vector<cudaEvent_t> ev_swap;  // 2 per block
+  // swap timing inside the replayed graph: event-record nodes around each
+  // block's swap-in on the copy stream (swapnet_engine_set_swap_timing)
+  bool swap_timing = false;
+  std::vector<cudaEvent_t> ev_gswap;  // 2 per block
   cudaStream_t cap = nullptr;        // capture origin stream
   cudaEvent_t fork = nullptr, join = nullptr;
   // per (input, output, profiling) binding
@@ -169,6 +173,7 @@ static int release(swapnet_engine* e) {
   if (e->cap) cudaStreamDestroy(e->cap);
   for (cudaEvent_t ev : e->ev_unit) cudaEventDestroy(ev);
   for (cudaEvent_t ev : e->ev_swap) cudaEventDestroy(ev);
+  for (cudaEvent_t ev : e->ev_gswap) cudaEventDestroy(ev);
   if (e->copy) cudaStreamDestroy(e->copy);
   if (e->rd) {
     cudaStreamSynchronize(e->rd);
@@ -1285,8 +1290,13 @@ static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t 
     } else if (prof) {
       CU(cudaEventRecord(e->ev_swap[2 * k], e->copy), "profile event");
     }
+    // in a captured graph an event-record node (external event), eagerly a
+    // plain record: either way the copy stream's own time for this swap
+    const unsigned gflag = capturing ? cudaEventRecordExternal : cudaEventRecordDefault;
+    if (e->swap_timing) CU(cudaEventRecordWithFlags(e->ev_gswap[2 * k], e->copy, gflag), "swap timing event");
     int rc = swap_block(e, k, e->blocks[k].variant, e->copy);
     if (rc) return rc;
+    if (e->swap_timing) CU(cudaEventRecordWithFlags(e->ev_gswap[2 * k + 1], e->copy, gflag), "swap timing event");
     if (e->file) {
       CU(cudaEventRecord(e->stage_free[j], e->copy), "record staging free");
       stage_used[j] = true;
@@ -1405,7 +1415,7 @@ int swapnet_infer(swapnet_engine* e, const void* din, void* dout, swapnet_stream
   CU(cudaSetDevice(e->device), "cudaSetDevice");
   // event timing needs eager launches; stream capture takes no copy from pageable memory
   if (e->plan.opt.graphs && !e->profiling && !(e->plan.opt.pageable && !e->file)) {
-    const auto key = std::make_pair(std::make_pair(din, dout), false);
+    const auto key = std::make_pair(std::make_pair(din, dout), e->swap_timing);
     auto it = e->graphs.find(key);
     if (it == e->graphs.end()) {
       if (e->graphs.size() >= 8) {
@@ -1620,6 +1630,32 @@ int swapnet_engine_set_profiling(swapnet_engine* e, int enable) {
     for (cudaEvent_t& ev : e->ev_swap) CU(cudaEventCreate(&ev), "event");
   }
   e->profiling = enable != 0;
+  return SWAPNET_OK;
+}
+
+int swapnet_engine_set_swap_timing(swapnet_engine* e, int enable) {
+  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+  CU(cudaSetDevice(e->device), "cudaSetDevice");
+  if (enable && e->ev_gswap.empty()) {
+    e->ev_gswap.assign(2 * e->plan.blocks.size(), nullptr);
+    for (cudaEvent_t& ev : e->ev_gswap) CU(cudaEventCreate(&ev), "event");
+  }
+  e->swap_timing = enable != 0;
+  return SWAPNET_OK;
+}
+
+int swapnet_engine_last_swap_times(swapnet_engine* e, float* swap_us, uint32_t nb) {
+  if (!e || !swap_us) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+  if (e->ev_gswap.empty()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "swap timing was never enabled");
+  CU(cudaSetDevice(e->device), "cudaSetDevice");
+  for (uint32_t k = 0; k < nb && k < e->plan.blocks.size(); ++k) {
+    float ms = 0.f;
+    if (swapped(e, k)) {
+      CU(cudaEventSynchronize(e->ev_gswap[2 * k + 1]), "event synchronize");
+      CU(cudaEventElapsedTime(&ms, e->ev_gswap[2 * k], e->ev_gswap[2 * k + 1]), "elapsed");
+    }
+    swap_us[k] = ms * 1000.f;
+  }
   return SWAPNET_OK;
 }
 

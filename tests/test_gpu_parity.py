@@ -462,3 +462,45 @@ def test_injected_load_failures_leave_nothing_behind(what, code):
     got = Runner(m, w, plan, host).run(x)
     ref = Runner(m, w, capi.Plan.resident(d), host).run(x)
     assert all(a.tobytes() == b.tobytes() for a, b in zip(got, ref))
+
+
+@pytest.mark.parametrize("variant", [capi.SWAP_MEMCPY, capi.SWAP_ZEROCOPY])
+def test_swap_times_inside_the_replayed_graph(variant):
+    """Swap timing in the graph (event-record nodes around each block's
+    swap-in on the copy stream): the outputs stay the resident bits, every
+    swapped block reports a positive time that is at least its bytes over a
+    generous link ceiling, and the swaps of one inference add up to no more
+    than the inference's own time on its stream."""
+    import torch
+    m = synth.arch.MODELS["resnet50"]()
+    w = synth.gen.model_weights(m)
+    d = capi.Desc(m)
+    host = capi.HostWeights(w)
+    wb = OP.weight_bytes(m)
+    plan = capi.Plan.partition(d, int(wb * 0.4) // 256 * 256, capi.options(swap_variant=variant))
+    nb = plan.info()["n_blocks"]
+    sw = Runner(m, w, plan, host)
+    rs = Runner(m, w, capi.Plan.resident(d), host)
+    x = synth.gen.model_input(m, request=3)
+    ref = rs.run(x)
+    sw.engine.set_swap_timing(True)
+    for _ in range(2):
+        got = sw.run(x)
+        assert all(p.tobytes() == q.tobytes() for p, q in zip(got, ref))
+    s = torch.cuda.current_stream()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(s)
+    sw.engine.infer(sw.d_in.data_ptr(), sw.d_out.data_ptr(), s.cuda_stream)
+    b.record(s)
+    b.synchronize()
+    us = sw.engine.last_swap_times(nb)
+    blocks = plan.blocks()
+    for blk, t in zip(blocks, us):
+        if blk["bytes"]:
+            assert t > 0.0
+            assert blk["bytes"] / (t * 1e-6) < 1e12   # under 1 TB/s: a real copy was timed
+    assert sum(us) <= a.elapsed_time(b) * 1e3 * 1.01
+    sw.engine.set_swap_timing(False)
+    got = sw.run(x)
+    assert all(p.tobytes() == q.tobytes() for p, q in zip(got, ref))
+    sw.engine.sync()
