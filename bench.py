@@ -1104,6 +1104,8 @@ def run_profile_once(args):
     eng = capi.Engine(plan, host)
     if info["state_bytes"]:
         state = torch.zeros(info["state_bytes"], dtype=torch.uint8, device="cuda")
+        if args.profile_pos:
+            state[:4].copy_(torch.tensor([args.profile_pos], dtype=torch.int32).view(torch.uint8))
         eng.bind_state(state.data_ptr(), info["state_bytes"])
     d_in = torch.empty(max(16, info["input_bytes"]), dtype=torch.uint8, device="cuda")
     d_in[:info["input_bytes"]].copy_(torch.from_numpy(x.view(np.uint8).reshape(-1)))
@@ -1203,6 +1205,9 @@ def main():
                     help="--profile-once --config llm: decoder layers of the profiled decode pass")
     ap.add_argument("--profile-tokens", type=int, default=1,
                     help="--profile-once --config llm: token ids of the profiled pass (1: decode, 512: prefill)")
+    ap.add_argument("--profile-pos", type=int, default=0,
+                    help="--profile-once --config llm: cached positions before the profiled pass (the attention "
+                         "reads that many cache entries)")
     ap.add_argument("--merge", type=int, default=1, choices=[0, 1],
                     help="decoder: GEMV layers sharing an input in one launch (1) or one launch each (0)")
     ap.add_argument("--link-share", type=float, default=1.0,

@@ -134,7 +134,10 @@ typedef enum swapnet_swap_variant {
                                 (copy-free dispatch, Sec. 4.2.2, taken to the
                                 kernels); for blocks whose units all run SIMT
                                 kernels (GEMV, norms, attention, pools), other
-                                blocks take MEMCPY.  Never chosen by AUTO.    */
+                                blocks take ZEROCOPY (MEMCPY when a tensor is
+                                not 16-byte aligned), so copy-engine and SM
+                                reads of the host weights are not mixed.
+                                Never chosen by AUTO.                         */
 } swapnet_swap_variant;
 
 /* Options.  Delay coefficients follow Sec. 6.1: t_in = alpha*s + beta*d,
@@ -331,8 +334,13 @@ typedef struct CUstream_st* swapnet_stream; /* a cudaStream_t; NULL = legacy def
  * The plan is copied; it may be freed after this call.  Creates a copy
  * stream and per-slot events; resolves every layer's parameter address to
  * slot base + offset and builds its TMA descriptors once (the skeleton).
- * With SWAPNET_SWAP_AUTO it times both swap variants per block and keeps
- * the faster.  A resident plan copies all weights to the arena here.
+ * With SWAPNET_SWAP_AUTO it times both swap variants per block, then whole
+ * inferences with that per-block choice, with every block on the copy
+ * engine and with every block on the zero-copy kernel, and keeps the
+ * fastest; decoder models (attention layers, a bound state) take the
+ * zero-copy kernel for every block, so that the engines of one model never
+ * mix copy-engine and SM reads of their shared host weights.  A resident
+ * plan copies all weights to the arena here.
  * Errors: INVALID_ARG, MISALIGNED, OOM, CUDA, UNSUPPORTED. */
 int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint32_t n_tensors,
                  void* d_arena, uint64_t arena_bytes, void* d_workspace, uint64_t workspace_bytes,

@@ -71,6 +71,7 @@ struct UnitExec {
   TcGemm g{};
   TcPlan tc{};
   const void* tmA_for = nullptr;  // A pointer the TMA map was encoded for
+  bool in_place = false;          // parameters read in mapped host memory
 };
 
 struct HostRange {
@@ -557,10 +558,25 @@ static int capture(swapnet_engine* e, const void* din, void* dout, cudaGraphExec
 // zero-copy is also timed with 24 and 16 CTAs: fewer CTAs leave more SMs to
 // the layers while still keeping ahead of them (measured on ResNet-50 and
 // YOLOv3: 1-2 % faster inferences than 32).
-// Decoder models (which need a bound state) keep the per-block choice.
+// Decoder models (which need a bound state) are not timed whole: their
+// blocks all take the zero-copy kernel when every block allows it.  Their
+// prefill and decode engines read the same multi-GB host weights, and on
+// the GB300 machine copy-engine reads of a 13 GB page-locked region that SM
+// loads had just read ran about 9x below the link rate (a prefill pass of
+// the 7B decoder at 120 instead of 63 ms when one of its nine blocks took
+// the copy engine after decode passes on the zero-copy kernel), while SM
+// loads keep the link rate in every order.
 static int calibrate_in_situ(swapnet_engine* e) {
   const Model& m = e->plan.model;
-  if (m.has_attention || e->blocks.empty()) return SWAPNET_OK;
+  if (e->blocks.empty()) return SWAPNET_OK;
+  if (m.has_attention) {
+    bool zc_all = true;
+    for (size_t k = 0; k < e->blocks.size(); ++k)
+      zc_all = zc_all && (e->plan.blocks[k].slot < 0 || zerocopy_ok(e->blocks[k]));
+    if (zc_all)
+      for (EngBlock& b : e->blocks) b.variant = SWAPNET_SWAP_ZEROCOPY;
+    return SWAPNET_OK;
+  }
   void* din = nullptr;
   void* dout = nullptr;
   if (cudaMalloc(&din, align_up(m.in_bytes)) != cudaSuccess ||
@@ -783,6 +799,11 @@ static int run_group(swapnet_engine* e, int u, const void* din, void* dout, cuda
     j.seg[i] = SkSeg{X.w, Epi{X.b, r, L.d.cout, L.d.act, L.d.res_post}, L.d.cout,
                      out_ptr(e, p.units[v].layer, dout), L.d.cout};
   }
+  j.device_weights = 1;
+  for (int i = 0; i < j.nseg; ++i)
+    if (e->ux[u + i].in_place) j.device_weights = 0;
+  j.num_sms = e->num_sms;
+  j.err = e->err_word;
   return launch_linear_skinny_job(m.dtype, j, s);
 }
 
@@ -822,10 +843,12 @@ static int prepare_units(swapnet_engine* e) {
       UnitExec& X = e->ux[u];
       if (U.host) {
         X.w = e->tensor_dev[U.tidx[0]];  // device alias of the page-locked host table
+        X.in_place = true;
       } else if (e->blocks[&B - p.blocks.data()].variant == SWAPNET_SWAP_DIRECT) {
         // read in place in page-locked host memory (device aliases)
         if (U.nt >= 1) X.w = e->tensor_dev[U.tidx[0]] + U.toff[0];
         if (U.nt == 2) X.b = e->tensor_dev[U.tidx[1]] + U.toff[1];
+        X.in_place = true;
       } else {
         if (U.nt >= 1) X.w = base + U.slot_off[0];
         if (U.nt == 2) X.b = base + U.slot_off[1];
@@ -886,7 +909,7 @@ static int run_unit(swapnet_engine* e, int u, const void* din, void* dout, cudaS
         ep.res = r ? r + (int64_t)U.row0 * es : nullptr;
         if (skinny_ok(m, L))
           return launch_linear_skinny(m.dtype, x, L.n, L.d.cin, X.w, U.rows, ep, y + (int64_t)U.row0 * es,
-                                      L.d.cout, s);
+                                      L.d.cout, s, X.in_place ? 0 : 1, e->num_sms, e->err_word);
         return launch_linear_tiled(m.dtype, x, L.n, L.d.cin, X.w, U.rows, ep, y + (int64_t)U.row0 * es, L.d.cout,
                                    s);
       }
@@ -1023,8 +1046,13 @@ static int bind_plan(swapnet_engine* e, void* d_arena_user, uint64_t arena_bytes
   } else if (!plan->resident) {
     for (size_t k = 0; k < e->blocks.size(); ++k) {
       EngBlock& b = e->blocks[k];
-      if (variant == SWAPNET_SWAP_DIRECT) {  // the blocks direct_ok refused are copied
-        if (b.variant != SWAPNET_SWAP_DIRECT) b.variant = SWAPNET_SWAP_MEMCPY;
+      if (variant == SWAPNET_SWAP_DIRECT) {
+        // the blocks direct_ok refused are copied by SM loads too: on the
+        // GB300 machine, copy-engine reads of a large page-locked region right
+        // after SM loads had read it ran about 9x slower (24 instead of
+        // 210 GB/s over the 13.2 GB of the 7B decoder), while SM loads
+        // after SM loads keep the link rate
+        if (b.variant != SWAPNET_SWAP_DIRECT) b.variant = zerocopy_ok(b) ? SWAPNET_SWAP_ZEROCOPY : SWAPNET_SWAP_MEMCPY;
         continue;
       }
       b.variant = variant;

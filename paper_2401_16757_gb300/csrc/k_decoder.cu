@@ -2,6 +2,9 @@
 // table), RMSNorm, RoPE + KV-cache append, causal attention with an online
 // softmax, row argmax, and the device-side advance of the cache position.
 // bf16 / fp16 storage, fp32 arithmetic, fixed reduction orders.
+#include <cooperative_groups.h>
+
+#include <algorithm>
 #include <cstring>
 
 #include "device.cuh"
@@ -9,6 +12,8 @@
 #include "kernels.h"
 
 namespace swapnet {
+
+namespace cg = cooperative_groups;
 
 namespace {
 
@@ -188,24 +193,43 @@ __global__ void __launch_bounds__(256) rope_append_kernel(T* __restrict__ q, con
 // arithmetic definition: fewer than kRowsMinWarps (query, head) pairs (a
 // decode step) the CTA kernel, more the warp kernel.
 //
-// Short query runs: CTA = one (query t, head h), 512 threads; the scores of all visible keys
-// live in shared memory, so the softmax is exact two-pass (max, then
-// exponentials and their sum) rather than online:
-//   phase 1: thread j computes key j's score (the whole 128-wide dot product
-//            from 16 independent 16-byte loads of its cache row);
-//   phase 2: block max, p_j = exp(s_j - max), block sum l in a fixed order;
-//   phase 3: thread (pair d, group g) accumulates p_j * v_j[2d..2d+1] over
-//            keys j = g, g + 8, ... (coalesced 4-byte loads along the row);
-//            the 8 groups are added in index order and divided by l.
-// Every key load of a phase is independent of the others, so a decode step
-// (one query, keys in HBM) is bound by a few memory round trips, not by a
-// chain of one round trip per key.
+// Short query runs (a decode step): the visible keys of one (query t,
+// head h) are split into S consecutive chunks of `chunk` keys, one CTA per
+// chunk, and the S CTAs of a (t, h) form a thread-block cluster.  Each CTA
+// computes, over its chunk only (256 threads):
+//   phase 1: scores s_j = q . k_j / sqrt(128): 16 threads per key, one
+//            16-byte load each (8 head dims), summed over the 16 lanes in a
+//            fixed butterfly order; 16 keys per pass, the loads of four
+//            passes issued before their arithmetic;
+//   phase 2: the chunk's max m_c, p_j = exp(s_j - m_c) and l_c = sum p_j
+//            (block reductions in a fixed order);
+//   phase 3: a_c[d] = sum_j p_j v_j[d]: thread (key group g, 8-dim slice)
+//            over keys g, g + 16, ... with 16-byte loads, then the 16 groups
+//            added in index order.
+// After a cluster barrier the cluster's first CTA reads every chunk's
+// (m_c, l_c, a_c) through distributed shared memory and combines them in
+// chunk order: M = max m_c, L = sum l_c e^(m_c - M),
+// out[d] = sum a_c[d] e^(m_c - M) / L  (chunks past the visible keys hold
+// l_c = 0 and are skipped).  The result is that of one exact softmax over
+// all visible keys, with every sum in a fixed order.
 constexpr int kDh = 128;
-constexpr int kAttThreads = 512;
-constexpr int kAttGroups = kAttThreads / (kDh / 2);
+constexpr int kSpThreads = 256;
+constexpr int kSpMaxSplit = 8;      // portable cluster size
+constexpr int kSpKeysPerPass = kSpThreads / 16;
 constexpr int kRowsMinWarps = 1024;
 
-__device__ __forceinline__ float block_reduce(float v, float* red, bool is_max) {
+struct SplitPlan {
+  int split, chunk;
+};
+
+// Chunks of at least 64 keys (a multiple of 16), at most kSpMaxSplit of them.
+inline SplitPlan split_plan(int max_seq) {
+  int split = std::min(kSpMaxSplit, std::max(1, (max_seq + 63) / 64));
+  int chunk = ((max_seq + split - 1) / split + 15) / 16 * 16;
+  return SplitPlan{split, chunk};
+}
+
+__device__ __forceinline__ float sp_block_reduce(float v, float* red, bool is_max) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
@@ -216,92 +240,136 @@ __device__ __forceinline__ float block_reduce(float v, float* red, bool is_max) 
   if (lane == 0) red[warp] = v;
   __syncthreads();
   float r = red[0];
-  for (int w = 1; w < kAttThreads / 32; ++w) r = is_max ? fmaxf(r, red[w]) : r + red[w];
+  for (int w = 1; w < kSpThreads / 32; ++w) r = is_max ? fmaxf(r, red[w]) : r + red[w];
   return r;
 }
 
 template <typename T>
-__global__ void __launch_bounds__(kAttThreads) attention_kernel(const T* __restrict__ q, const T* __restrict__ kc,
-                                                                const T* __restrict__ vc,
-                                                                const int* __restrict__ pos_ptr, int heads,
-                                                                int width, int max_seq, T* __restrict__ out) {
-  extern __shared__ float att_smem[];
-  float2* part = reinterpret_cast<float2*>(att_smem);          // kAttGroups x kDh/2 partial sums
-  float* red = att_smem + 2 * kAttGroups * (kDh / 2);          // kAttThreads / 32 partials
-  float* qs = red + kAttThreads / 32;                          // kDh query values
-  float* sc = qs + kDh;                                        // max_seq scores
+__global__ void __launch_bounds__(kSpThreads) attention_split_kernel(const T* __restrict__ q,
+                                                                     const T* __restrict__ kc,
+                                                                     const T* __restrict__ vc,
+                                                                     const int* __restrict__ pos_ptr, int width,
+                                                                     int max_seq, int chunk, T* __restrict__ out) {
+  extern __shared__ float sp_smem[];
+  float* part = sp_smem;                         // 16 groups x kDh partial sums
+  float* acc = part + 16 * kDh;                  // kDh: this chunk's a_c
+  float* ml = acc + kDh;                         // m_c, l_c
+  float* red = ml + 2;                           // kSpThreads / 32 partials
+  float* sc = red + kSpThreads / 32;             // chunk scores
+  cg::cluster_group cluster = cg::this_cluster();
   pdl_wait();
   pdl_launch_dependents();
-  const int h = blockIdx.x, t = blockIdx.y;
+  const int c = (int)cluster.block_rank();
+  const int split = (int)cluster.num_blocks();
+  const int h = blockIdx.y, t = blockIdx.z;
   const int tid = threadIdx.x;
   const int n = min(*pos_ptr + t + 1, max_seq);
+  const int j0 = c * chunk, j1 = min(j0 + chunk, n);
   const int64_t col = (int64_t)h * kDh;
-  if (tid < kDh) qs[tid] = to_f<T>(q[(int64_t)t * width + col + tid]);
-  __syncthreads();
   const float scale = rsqrtf((float)kDh);
-  float mx = -INFINITY;
-  for (int j = tid; j < n; j += kAttThreads) {
-    const uint4* kr = reinterpret_cast<const uint4*>(kc + (int64_t)j * width + col);
-    uint4 u[kDh / 8];
+  float m_c = -INFINITY, l_c = 0.f;
+  if (j0 < j1) {
+    // phase 1: lane group of 16 per key, 8 dims per thread
+    const int sl = tid & 15, kq = tid >> 4;
+    float qv[8];
+    {
+      const uint4 u = *reinterpret_cast<const uint4*>(q + (int64_t)t * width + col + sl * 8);
+      const T* e = reinterpret_cast<const T*>(&u);
 #pragma unroll
-    for (int i = 0; i < kDh / 8; ++i) u[i] = kr[i];
-    float s = 0.f;
-#pragma unroll
-    for (int i = 0; i < kDh / 8; ++i) {
-      const T* e = reinterpret_cast<const T*>(&u[i]);
-#pragma unroll
-      for (int k = 0; k < 8; ++k) s = fmaf(qs[i * 8 + k], to_f<T>(e[k]), s);
+      for (int i = 0; i < 8; ++i) qv[i] = to_f<T>(e[i]);
     }
-    s *= scale;
-    sc[j] = s;
-    mx = fmaxf(mx, s);
-  }
-  mx = block_reduce(mx, red, true);
-  float l = 0.f;
-  for (int j = tid; j < n; j += kAttThreads) {
-    const float p = expf(sc[j] - mx);
-    sc[j] = p;
-    l += p;
-  }
-  l = block_reduce(l, red, false);  // the barriers inside also publish sc[]
-  const int d2 = tid % (kDh / 2), g = tid / (kDh / 2);
-  const T* vcol = vc + col + 2 * d2;
-  float a0 = 0.f, a1 = 0.f;
-  int j = g;
-#pragma unroll 1
-  for (; j + 3 * kAttGroups < n; j += 4 * kAttGroups) {
-    uint32_t w[4];
+    float mx = -INFINITY;
+    for (int jb = j0; jb < j1; jb += 4 * kSpKeysPerPass) {
+      uint4 ku[4];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) w[i] = *reinterpret_cast<const uint32_t*>(vcol + (int64_t)(j + i * kAttGroups) * width);
+      for (int r = 0; r < 4; ++r) {
+        const int j = jb + r * kSpKeysPerPass + kq;
+        ku[r] = j < j1 ? *reinterpret_cast<const uint4*>(kc + (int64_t)j * width + col + sl * 8)
+                       : make_uint4(0u, 0u, 0u, 0u);
+      }
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const T* e = reinterpret_cast<const T*>(&w[i]);
-      const float p = sc[j + i * kAttGroups];
-      a0 = fmaf(p, to_f<T>(e[0]), a0);
-      a1 = fmaf(p, to_f<T>(e[1]), a1);
+      for (int r = 0; r < 4; ++r) {
+        const int j = jb + r * kSpKeysPerPass + kq;
+        const T* e = reinterpret_cast<const T*>(&ku[r]);
+        float sdot = 0.f;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) sdot = fmaf(qv[i], to_f<T>(e[i]), sdot);
+#pragma unroll
+        for (int off = 8; off > 0; off >>= 1) sdot += __shfl_xor_sync(0xffffffffu, sdot, off);
+        sdot *= scale;
+        if (j < j1) {
+          if (sl == 0) sc[j - j0] = sdot;
+          mx = fmaxf(mx, sdot);
+        }
+      }
     }
-  }
-  for (; j < n; j += kAttGroups) {
-    const uint32_t w = *reinterpret_cast<const uint32_t*>(vcol + (int64_t)j * width);
-    const T* e = reinterpret_cast<const T*>(&w);
-    const float p = sc[j];
-    a0 = fmaf(p, to_f<T>(e[0]), a0);
-    a1 = fmaf(p, to_f<T>(e[1]), a1);
-  }
-  part[g * (kDh / 2) + d2] = make_float2(a0, a1);
-  __syncthreads();
-  if (tid < kDh / 2) {
-    float o0 = 0.f, o1 = 0.f;
-    for (int gg = 0; gg < kAttGroups; ++gg) {
-      const float2 v = part[gg * (kDh / 2) + tid];
-      o0 += v.x;
-      o1 += v.y;
+    // phase 2
+    m_c = sp_block_reduce(mx, red, true);
+    float l = 0.f;
+    for (int j = tid; j < j1 - j0; j += kSpThreads) {
+      const float pj = expf(sc[j] - m_c);
+      sc[j] = pj;
+      l += pj;
     }
-    const float inv = 1.0f / l;
-    T* o = out + (int64_t)t * width + col + 2 * tid;
-    o[0] = from_f<T>(o0 * inv);
-    o[1] = from_f<T>(o1 * inv);
+    l_c = sp_block_reduce(l, red, false);  // the barriers inside also publish sc[]
+    // phase 3: key group g = tid / 16, dims 8 * (tid % 16) .. + 7
+    const int g = tid >> 4;
+    float a[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) a[i] = 0.f;
+    const T* vcol = vc + col + sl * 8;
+    for (int jb = j0 + g; jb < j1; jb += 4 * 16) {
+      uint4 vu[4];
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        const int j = jb + r * 16;
+        vu[r] = j < j1 ? *reinterpret_cast<const uint4*>(vcol + (int64_t)j * width) : make_uint4(0u, 0u, 0u, 0u);
+      }
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        const int j = jb + r * 16;
+        if (j < j1) {
+          const float pj = sc[j - j0];
+          const T* e = reinterpret_cast<const T*>(&vu[r]);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) a[i] = fmaf(pj, to_f<T>(e[i]), a[i]);
+        }
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) part[g * kDh + sl * 8 + i] = a[i];
+    __syncthreads();
+    if (tid < kDh) {
+      float sum = 0.f;
+      for (int gg = 0; gg < 16; ++gg) sum += part[gg * kDh + tid];
+      acc[tid] = sum;
+    }
+  } else if (tid < kDh) {
+    acc[tid] = 0.f;
   }
+  if (tid == 0) {
+    ml[0] = m_c;
+    ml[1] = l_c;
+  }
+  cluster.sync();  // every chunk's (m_c, l_c, a_c) is visible to the cluster
+  if (c == 0 && tid < kDh) {
+    float M = -INFINITY;
+    for (int r = 0; r < split; ++r) {
+      const float* rml = cluster.map_shared_rank(ml, r);
+      if (rml[1] > 0.f) M = fmaxf(M, rml[0]);
+    }
+    float L = 0.f, o = 0.f;
+    for (int r = 0; r < split; ++r) {
+      const float* rml = cluster.map_shared_rank(ml, r);
+      if (rml[1] > 0.f) {
+        const float w = expf(rml[0] - M);
+        L += rml[1] * w;
+        o += cluster.map_shared_rank(acc, r)[tid] * w;
+      }
+    }
+    out[(int64_t)t * width + col + tid] = from_f<T>(o / L);
+  }
+  cluster.sync();  // the first CTA has read every chunk before any CTA exits
 }
 
 // Long query runs (prefill): warp = one (query, head), each lane holding 4
@@ -357,8 +425,8 @@ __global__ void __launch_bounds__(256) attention_rows_kernel(const T* __restrict
   for (int d = 0; d < 4; ++d) o[d] = from_f<T>(acc[d] * inv);
 }
 
-size_t attention_smem_bytes(int max_seq) {
-  return sizeof(float) * ((size_t)max_seq + kDh + kAttThreads / 32) + sizeof(float2) * kAttGroups * (kDh / 2);
+size_t attention_split_smem_bytes(int chunk) {
+  return sizeof(float) * (16 * kDh + kDh + 2 + kSpThreads / 32 + (size_t)chunk);
 }
 
 // ------------------------------------------------------------ argmax
@@ -493,15 +561,32 @@ int launch_attention(int dtype, void* q, const void* k, const void* v, void* kc,
                              pos_ptr, tokens, heads, width, max_seq, static_cast<T*>(out)),
                   "attention launch");
     }
-    const size_t smem = attention_smem_bytes(max_seq);
+    // decode: the visible keys split over a cluster of CTAs per (query, head)
+    const SplitPlan sp = split_plan(max_seq);
+    const size_t smem = attention_split_smem_bytes(sp.chunk);
     if (smem > 48 * 1024) {
-      cudaError_t e = cudaFuncSetAttribute(attention_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      cudaError_t e = cudaFuncSetAttribute(attention_split_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            (int)smem);
       if (e != cudaSuccess) return done(e, "attention shared memory");
     }
-    return done(launch_pdl(attention_kernel<T>, dim3(heads, tokens), dim3(kAttThreads), smem, s,
-                           static_cast<const T*>(q), static_cast<const T*>(kc), static_cast<const T*>(vc),
-                           pos_ptr, heads, width, max_seq, static_cast<T*>(out)),
+    cudaLaunchConfig_t cfg;
+    std::memset(&cfg, 0, sizeof(cfg));
+    cfg.gridDim = dim3(sp.split, heads, tokens);
+    cfg.blockDim = dim3(kSpThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = sp.split;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return done(cudaLaunchKernelEx(&cfg, attention_split_kernel<T>, static_cast<const T*>(q),
+                                   static_cast<const T*>(kc), static_cast<const T*>(vc), pos_ptr, width, max_seq,
+                                   sp.chunk, static_cast<T*>(out)),
                 "attention launch");
   });
   return SWAPNET_OK;

@@ -1,6 +1,8 @@
 // SIMT layer kernels: skinny linear (M <= 16, HBM-bound GEMV family),
 // direct convolution for channel counts the tensor-core path cannot tile,
 // pooling, upsampling and channel concatenation.  NHWC everywhere.
+#include <algorithm>
+#include <atomic>
 #include <cstdio>
 #include <cstring>
 
@@ -172,7 +174,229 @@ __global__ void __launch_bounds__(kSkWarps * 32) linear_skinny_kernel(const SkJo
   }
 }
 
+// ------------------------------------------------------------ streamed skinny linear
+// The same per-feature arithmetic as linear_skinny_kernel (lane l takes the
+// 16-byte chunks l, l + 32, ... of the weight row in order, one fp32 sum per
+// row of x, the same butterfly and epilogue), so its outputs are
+// bit-identical; only the way the weight rows reach the lanes differs.  For
+// weights in device memory each warp streams its rows into its own ring of
+// D shared-memory slots with bulk copies (cp.async.bulk, completion counted
+// on one mbarrier per slot), issued by lane 0 up to D rows ahead of the
+// row being summed, so each SM keeps D x row bytes per warp in flight
+// (about 100-200 KB) with a handful of registers.  x (M rows of K) is read
+// once per CTA into shared memory.  The first D rows of every warp are
+// requested before the programmatic wait (weights never depend on the
+// previous kernel), so the weight stream starts while that kernel drains.
+// One CTA per SM (grid = number of SMs, or fewer when there are fewer
+// features); warp g of the grid takes features g, g + G, ... (G = warps in
+// the grid); in pair mode a feature's two rows (gate, then its paired
+// layer) take two consecutive slots.  Every slot wait is bounded: on
+// timeout the warp records the error, stops, and waits (bounded) for the
+// copies it still has in flight before the CTA exits.
+constexpr int kStXMax = 64 * 1024;        // x staged in shared memory: at most this many bytes
+constexpr int kStSmem = 227 * 1024;       // dynamic shared memory of the streamed kernel's CTA
+constexpr int kStMaxWarps = 8;
+
+struct StLayout {
+  int warps, depth, slot_bytes, x_bytes, smem;
+};
+
+inline StLayout st_layout(int M, int K, int es, bool pair) {
+  StLayout L{0, 0, 0, 0, 0};
+  const int row = K * es;
+  L.x_bytes = (M * row + 127) / 128 * 128;
+  if (M * row > kStXMax) return L;
+  L.slot_bytes = (row + 127) / 128 * 128;
+  L.depth = row <= 8192 ? 4 : (row <= 16384 && !pair ? 3 : 2);
+  const int fixed = L.x_bytes + 256;  // + abort flag, alignment slack
+  const int per_warp = L.depth * (L.slot_bytes + 8);
+  L.warps = std::min(kStMaxWarps, (kStSmem - fixed) / per_warp);
+  L.smem = fixed + L.warps * per_warp;
+  return L;
+}
+
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               ::"r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
+}
+
+template <typename T, int MT>
+__global__ void __launch_bounds__(kStMaxWarps * 32, 1) linear_stream_kernel(const SkJob j, int depth, int slot_bytes,
+                                                                             int x_bytes) {
+  constexpr int V = Vec16<T>::N;
+  extern __shared__ __align__(128) uint8_t st_smem[];
+  const int warps = blockDim.x >> 5;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  T* xs = reinterpret_cast<T*>(st_smem);
+  uint8_t* ring = st_smem + x_bytes + (size_t)warp * depth * slot_bytes;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(st_smem + x_bytes + (size_t)warps * depth * slot_bytes) + warp * depth;
+  volatile int* abort_flag =
+      reinterpret_cast<volatile int*>(st_smem + x_bytes + (size_t)warps * depth * (slot_bytes + 8));
+  const int row_bytes = j.K * (int)sizeof(T);
+  const int kchunks = j.K / V;
+  const int rows_per_item = j.pair ? 2 : 1;
+  int features = j.seg[0].N;
+  if (!j.pair)
+    for (int i = 1; i < j.nseg; ++i) features += j.seg[i].N;
+  const int gw = blockIdx.x * warps + warp, G = gridDim.x * warps;
+  const int my_items = gw < features ? (features - 1 - gw) / G + 1 : 0;
+  const int my_rows = my_items * rows_per_item;
+  // weight row q of this warp's stream
+  auto row_ptr = [&](int q) -> const T* {
+    int o = gw + (q / rows_per_item) * G;
+    int si = j.pair ? (q % 2) : 0;
+    if (!j.pair)
+      for (int i = 0; i + 1 < j.nseg && o >= j.seg[i].N; ++i) {
+        o -= j.seg[i].N;
+        si = i + 1;
+      }
+    const T* W = static_cast<const T*>(j.seg[0].W);
+#pragma unroll
+    for (int i = 1; i < kSkMaxSeg; ++i)
+      if (i == si) W = static_cast<const T*>(j.seg[i].W);
+    return W + (int64_t)o * j.K;
+  };
+  auto issue = [&](int q) {
+    const int slot = q % depth;
+    const uint32_t bar = smem_u32(bars + slot);
+    mbar_arrive_expect_tx(bar, (uint32_t)row_bytes);
+    bulk_g2s(smem_u32(ring + (size_t)slot * slot_bytes), row_ptr(q), (uint32_t)row_bytes, bar);
+  };
+  if (lane == 0)
+    for (int i = 0; i < depth; ++i) mbar_init(smem_u32(bars + i), 1);
+  if (threadIdx.x == 0) *abort_flag = 0;
+  fence_barrier_init();
+  __syncthreads();
+  int issued = 0;
+  if (lane == 0)
+    for (; issued < depth && issued < my_rows; ++issued) issue(issued);
+  pdl_wait();
+  pdl_launch_dependents();
+  {  // x into shared memory, 16 bytes per access
+    const uint4* src = static_cast<const uint4*>(j.x);
+    uint4* dst = reinterpret_cast<uint4*>(xs);
+    const int n16 = j.M * row_bytes / 16;
+    for (int i = threadIdx.x; i < n16; i += blockDim.x) dst[i] = src[i];
+  }
+  __syncthreads();
+  int q = 0;
+  bool ok = true;
+  for (int it = 0; it < my_items && ok; ++it) {
+    const int o_global = gw + it * G;
+    int o = o_global, si = 0;
+    if (!j.pair)
+      for (int i = 0; i + 1 < j.nseg && o >= j.seg[i].N; ++i) {
+        o -= j.seg[i].N;
+        si = i + 1;
+      }
+    float gate[MT];
+    for (int p = 0; p < rows_per_item; ++p, ++q) {
+      SkSeg S = j.seg[0];
+#pragma unroll
+      for (int i = 1; i < kSkMaxSeg; ++i)
+        if (i == (j.pair ? p : si)) S = j.seg[i];
+      const int slot = q % depth;
+      if (!mbar_wait_bounded(smem_u32(bars + slot), (uint32_t)((q / depth) & 1), abort_flag, j.err)) {
+        ok = false;
+        break;
+      }
+      const uint4* wrow = reinterpret_cast<const uint4*>(ring + (size_t)slot * slot_bytes);
+      float acc[MT];
+#pragma unroll
+      for (int m = 0; m < MT; ++m) acc[m] = 0.f;
+      for (int ch = lane; ch < kchunks; ch += 32) {
+        float wf[V];
+        unpack16<T>(wrow[ch], wf);
+#pragma unroll
+        for (int m = 0; m < MT; ++m) {
+          if (m < j.M) {
+            float xv[V];
+            unpack16<T>(*reinterpret_cast<const uint4*>(xs + (int64_t)m * j.K + (int64_t)ch * V), xv);
+#pragma unroll
+            for (int i = 0; i < V; ++i) acc[m] = fmaf(wf[i], xv[i], acc[m]);
+          }
+        }
+      }
+#pragma unroll
+      for (int m = 0; m < MT; ++m) {
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) acc[m] += __shfl_xor_sync(0xffffffffu, acc[m], off);
+      }
+      // every lane has read the slot (its sums are complete): refill it
+      __syncwarp();
+      if (lane == 0 && issued < my_rows) {
+        fence_proxy_async_smem();
+        issue(issued);
+        ++issued;
+      }
+      const float b = S.e.bias ? to_f<T>(static_cast<const T*>(S.e.bias)[o]) : 0.f;
+#pragma unroll
+      for (int m = 0; m < MT; ++m) {
+        if (m < j.M) {
+          float r = 0.f;
+          bool has_r = S.e.res != nullptr;
+          if (p == 1) {
+            r = gate[m];
+            has_r = true;
+          } else if (has_r) {
+            r = to_f<T>(static_cast<const T*>(S.e.res)[(int64_t)m * S.e.ldr + o]);
+          }
+          const T out = from_f<T>(epilogue(acc[m], b, r, has_r, S.e.act, S.e.res_post));
+          gate[m] = to_f<T>(out);  // the stored value, as the paired layer reads it
+          if (lane == m) static_cast<T*>(S.y)[(int64_t)m * S.ldy + o] = out;
+        }
+      }
+    }
+  }
+  if (!ok && lane == 0) {
+    // copies still in flight land in this warp's slots: wait for them
+    // (bounded) before the CTA's shared memory goes away
+    volatile int drain = 0;
+    for (int r = q; r < issued; ++r)
+      mbar_wait_bounded(smem_u32(bars + r % depth), (uint32_t)((r / depth) & 1), &drain, nullptr);
+  }
+}
+
+template <typename T, int MT>
+int stream_launch(const SkJob& j, const StLayout& L, int grid, cudaStream_t s) {
+  static std::atomic<uint64_t> attr_done{0};  // per instantiation, one bit per device
+  auto kern = linear_stream_kernel<T, MT>;
+  if (attr_needed(attr_done)) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kStSmem) != cudaSuccess)
+      SN_FAIL(SWAPNET_ERR_CUDA, "cudaFuncSetAttribute failed");
+    attr_set(attr_done);
+  }
+  const cudaError_t e = launch_pdl(kern, dim3(grid), dim3(L.warps * 32), (size_t)L.smem, s, j, L.depth,
+                                   L.slot_bytes, L.x_bytes);
+  return e == cudaSuccess ? SWAPNET_OK : SWAPNET_ERR_CUDA;
+}
+
+template <typename T> int stream_dispatch(const SkJob& j, const StLayout& L, cudaStream_t s) {
+  int features = j.seg[0].N;
+  if (!j.pair)
+    for (int i = 1; i < j.nseg; ++i) features += j.seg[i].N;
+  const int grid = std::max(1, std::min(j.num_sms, (features + L.warps - 1) / L.warps));
+  if (j.M <= 1) return stream_launch<T, 1>(j, L, grid, s);
+  if (j.M <= 2) return stream_launch<T, 2>(j, L, grid, s);
+  if (j.M <= 4) return stream_launch<T, 4>(j, L, grid, s);
+  if (j.M <= 8) return stream_launch<T, 8>(j, L, grid, s);
+  return stream_launch<T, 16>(j, L, grid, s);
+}
+
+// Rows of x from which the streamed kernel is used.  Measured on the GB300
+// box: with 8 rows (the fp32 MLP, K = 1024) it took a layer from 11.9 to
+// 6.3 us, x being read once per CTA instead of once per warp; with one row
+// (the 7B decode projections) it was slower than the plain-load kernel
+// (20.6 against 12.2 us per launch): one CTA of 4-8 warps per SM sums its
+// rows one after another and cannot hide each row's shared-memory, reduction
+// and epilogue latency the way 32 resident warps with loads in flight do.
+constexpr int kStMinRows = 8;
+
 template <typename T> int skinny_dispatch(const SkJob& j, cudaStream_t s) {
+  if (j.device_weights && j.num_sms > 0 && j.M >= kStMinRows) {
+    const StLayout L = st_layout(j.M, j.K, (int)sizeof(T), j.pair != 0);
+    if (L.warps >= 1) return stream_dispatch<T>(j, L, s);
+  }
   int rows = j.seg[0].N;
   if (!j.pair)
     for (int i = 1; i < j.nseg; ++i) rows += j.seg[i].N;
@@ -474,13 +698,16 @@ int launch_linear_skinny_job(int dtype, const SkJob& j, cudaStream_t s) {
 }
 
 int launch_linear_skinny(int dtype, const void* x, int M, int K, const void* W, int N, const Epi& e, void* y,
-                         int64_t ldy, cudaStream_t s) {
+                         int64_t ldy, cudaStream_t s, int device_weights, int num_sms, int* err) {
   SkJob j{};
   j.x = x;
   j.M = M;
   j.K = K;
   j.nseg = 1;
   j.seg[0] = SkSeg{W, e, N, y, ldy};
+  j.device_weights = device_weights;
+  j.num_sms = num_sms;
+  j.err = err;
   return launch_linear_skinny_job(dtype, j, s);
 }
 

@@ -40,7 +40,8 @@ struct Epi {
 // y[m, col0 + o] (row stride ldy) = epi(sum_k x[m,k] W[o,k]) for o < N,
 // M <= 16.  fp32 / fp16 / bf16; fixed-order reduction (deterministic).
 int launch_linear_skinny(int dtype, const void* x, int M, int K, const void* W, int N, const Epi& e, void* y,
-                         int64_t ldy, cudaStream_t s);
+                         int64_t ldy, cudaStream_t s, int device_weights = 0, int num_sms = 0,
+                         int* err = nullptr);
 
 // Several skinny linear layers reading the same x (M rows, K columns) in one
 // launch: segment i computes y_i[m, o] = epi_i(sum_k x[m,k] W_i[o,k]) for
@@ -60,6 +61,12 @@ struct SkJob {
   int M, K;
   int nseg, pair;
   SkSeg seg[kSkMaxSeg];
+  // weights in device memory (an arena slot or a resident arena): the
+  // rows may be streamed into shared memory by bulk copies; 0 for weights
+  // read in place in mapped host memory (plain loads only)
+  int device_weights;
+  int num_sms;  // grid of the streamed kernel (0: plain-load kernel)
+  int* err;     // device error word for the streamed kernel's bounded waits
 };
 int launch_linear_skinny_job(int dtype, const SkJob& j, cudaStream_t s);
 

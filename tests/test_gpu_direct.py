@@ -53,7 +53,9 @@ def test_mlp_reads_every_block_in_place():
 
 def test_mixed_blocks_vgg16():
     """VGG-16 at batch 1 under a quarter of its weights: the convolution
-    blocks (tensor cores) are copied, the fully connected pieces (GEMV) are
+    blocks (tensor cores) are copied by the zero-copy kernel (so SM loads
+    and copy-engine reads of the host weights are not mixed), the fully
+    connected pieces (GEMV) are
     read in place; the swapped byte count is exactly that of the copied
     blocks."""
     m = synth.arch.vgg16(batch=1)
@@ -62,7 +64,7 @@ def test_mixed_blocks_vgg16():
     plan_blocks = sw.plan.blocks()
     kinds = sw.engine.unit_kernels()
     direct = [k for k, b in enumerate(blocks) if b["variant"] == capi.SWAP_DIRECT]
-    copied = [k for k, b in enumerate(blocks) if b["variant"] == capi.SWAP_MEMCPY]
+    copied = [k for k, b in enumerate(blocks) if b["variant"] == capi.SWAP_ZEROCOPY]
     assert direct and copied and len(direct) + len(copied) == len(blocks)
     for k in direct:
         pb = plan_blocks[k]
@@ -107,7 +109,7 @@ def test_adapt_between_direct_and_copied_plans():
 
 def test_decoder_decode_pass_reads_in_place():
     """The LLM-shaped decoder: the prefill engine (tensor-core GEMMs) copies
-    its blocks, the decode engine (GEMV, norms, attention) reads every block
+    its blocks with the zero-copy kernel, the decode engine (GEMV, norms, attention) reads every block
     in place; prefill and four greedy decode passes equal the resident run
     bit for bit."""
     sw = Decoder(prefill_tokens=32, budget_frac=0.4, opts=dict(swap_variant=capi.SWAP_DIRECT))
@@ -115,7 +117,7 @@ def test_decoder_decode_pass_reads_in_place():
     pre = sw.engines[0][1].blocks()
     dec = sw.engines[1][1].blocks()
     assert len(dec) > 1 and all(b["variant"] == capi.SWAP_DIRECT for b in dec)
-    assert any(b["variant"] == capi.SWAP_MEMCPY for b in pre)
+    assert any(b["variant"] == capi.SWAP_ZEROCOPY for b in pre)
     ids = synth.gen.model_input(sw.mp).reshape(-1)
     a, b = sw.run(0, ids), rs.run(0, ids)
     assert a[0].tobytes() == b[0].tobytes() and a[1].tobytes() == b[1].tobytes()
