@@ -74,6 +74,9 @@ def variant_code(name):
 TRAFFIC = {
     ("resnet50", "tc_gemm"): ("1bb9110c06be", 1418599),
     ("resnet50", "tc_conv"): ("1bb9110c06be", 1807876),
+    # zero-copy swap: bytes of a launch's output still in L2 when it ends
+    # (DRAM writes = block bytes - this, from an ncu capture of two smaller launches)
+    ("llm", "zerocopy_kernel"): ("d2d45db9fdff", 63_400_000),
 }
 
 
@@ -530,8 +533,10 @@ def run_llm(args, rank, world, group):
             "traffic": None}
         tr = TRAFFIC.get(("llm", "zerocopy_kernel"))
         if tr and tr[0] == sources_sha(("k_swap.cu",)):
-            roofline["traffic"] = int(tr[1] * (zb // len(zc)))
-            roofline["traffic_note"] = "ncu DRAM bytes per byte swapped on a smaller capture, times the bytes of a launch"
+            roofline["traffic"] = int(zb // len(zc) - tr[1])
+            roofline["traffic_note"] = ("ncu DRAM bytes of two smaller launches (224 and 315 MB blocks): reads ~0, "
+                                        "writes = block bytes minus ~63 MB still in L2 at the kernel's end; "
+                                        "applied to this line's mean launch")
     else:
         roofline = None
 

@@ -204,8 +204,9 @@ __global__ void __launch_bounds__(256) rope_append_kernel(T* __restrict__ q, con
 //   phase 2: the chunk's max m_c, p_j = exp(s_j - m_c) and l_c = sum p_j
 //            (block reductions in a fixed order);
 //   phase 3: a_c[d] = sum_j p_j v_j[d]: thread (key group g, 8-dim slice)
-//            over keys g, g + 16, ... with 16-byte loads, then the 16 groups
-//            added in index order.
+//            over keys g, g + 16, ... with 16-byte loads (the first eight of
+//            them issued before phase 1, so that they arrive during it),
+//            then the 16 groups added in index order.
 // After a cluster barrier the cluster's first CTA reads every chunk's
 // (m_c, l_c, a_c) through distributed shared memory and combines them in
 // chunk order: M = max m_c, L = sum l_c e^(m_c - M),
@@ -216,6 +217,7 @@ constexpr int kDh = 128;
 constexpr int kSpThreads = 256;
 constexpr int kSpMaxSplit = 8;      // portable cluster size
 constexpr int kSpKeysPerPass = kSpThreads / 16;
+constexpr int kSpVPre = 8;          // value rows per thread requested with the keys
 constexpr int kRowsMinWarps = 1024;
 
 struct SplitPlan {
@@ -269,8 +271,18 @@ __global__ void __launch_bounds__(kSpThreads) attention_split_kernel(const T* __
   const float scale = rsqrtf((float)kDh);
   float m_c = -INFINITY, l_c = 0.f;
   if (j0 < j1) {
-    // phase 1: lane group of 16 per key, 8 dims per thread
     const int sl = tid & 15, kq = tid >> 4;
+    // the first kSpVPre value rows this thread sums in phase 3 (keys
+    // kq, kq + 16, ... of the chunk), requested now so that they arrive
+    // while the scores and the softmax are computed
+    uint4 vpre[kSpVPre];
+#pragma unroll
+    for (int r = 0; r < kSpVPre; ++r) {
+      const int j = j0 + kq + r * 16;
+      vpre[r] = j < j1 ? *reinterpret_cast<const uint4*>(vc + (int64_t)j * width + col + sl * 8)
+                       : make_uint4(0u, 0u, 0u, 0u);
+    }
+    // phase 1: lane group of 16 per key, 8 dims per thread
     float qv[8];
     {
       const uint4 u = *reinterpret_cast<const uint4*>(q + (int64_t)t * width + col + sl * 8);
@@ -318,7 +330,17 @@ __global__ void __launch_bounds__(kSpThreads) attention_split_kernel(const T* __
 #pragma unroll
     for (int i = 0; i < 8; ++i) a[i] = 0.f;
     const T* vcol = vc + col + sl * 8;
-    for (int jb = j0 + g; jb < j1; jb += 4 * 16) {
+#pragma unroll
+    for (int r = 0; r < kSpVPre; ++r) {
+      const int j = j0 + g + r * 16;
+      if (j < j1) {
+        const float pj = sc[j - j0];
+        const T* e = reinterpret_cast<const T*>(&vpre[r]);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) a[i] = fmaf(pj, to_f<T>(e[i]), a[i]);
+      }
+    }
+    for (int jb = j0 + g + kSpVPre * 16; jb < j1; jb += 4 * 16) {
       uint4 vu[4];
 #pragma unroll
       for (int r = 0; r < 4; ++r) {

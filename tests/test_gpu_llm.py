@@ -368,3 +368,29 @@ def test_merged_gemv_launches_equal_separate_launches(resident):
         assert per[1] - per[0] == 3 * SMALL["layers"]
     else:
         assert 0 <= per[1] - per[0] <= 3 * SMALL["layers"]
+
+
+def test_llm_decode_to_the_end_of_the_cache_then_refused():
+    """Greedy decode passes until the KV cache is full: the last pass
+    attends over all max_seq positions, so the decode attention's last key
+    chunk ends exactly at the end of the cache; every pass against the
+    oracle (which consumes the GPU's token).  One pass more finds no place
+    in the cache: the device reports the position as out of range and
+    swapnet_engine_sync returns INVALID_ARG."""
+    max_seq = 40
+    dec = Decoder(prefill_tokens=32, layers=1, max_seq=max_seq)
+    ids = synth.gen.model_input(dec.mp).reshape(-1)
+    st = F.new_state()
+    ref = F.forward(dec.mp, dec.w, ids.reshape(-1, 1, 1, 1), state=st)
+    logits, toks = dec.run(0, ids)
+    _check_step(logits, toks, ref[0].reshape(32, -1), ref[1].reshape(-1), TOL[1])
+    tok = int(toks[-1])
+    for step in range(max_seq - 32):
+        ref = F.forward(dec.md, dec.w, np.array([tok], dtype=np.int32).reshape(1, 1, 1, 1), state=st)
+        logits, toks = dec.run(1, np.array([tok], dtype=np.int32))
+        _check_step(logits, toks, ref[0].reshape(1, -1), ref[1].reshape(-1), TOL[1])
+        tok = int(toks[0])
+    assert int(dec.state[:4].cpu().numpy().view(np.int32)[0]) == max_seq
+    with pytest.raises(capi.SwapnetError) as ei:
+        dec.run(1, np.array([tok], dtype=np.int32))
+    assert ei.value.code == capi.ERR_INVALID_ARG
