@@ -102,6 +102,28 @@ def test_linear_layer(dtype, rows, k, n):
     _check_model(_model(layers, (rows, 1, 1, k), dtype))
 
 
+@pytest.mark.parametrize("dtype", ["f16", "bf16"])
+@pytest.mark.parametrize("rows,k,n", [(1, 11008, 520), (3, 25088, 300), (4, 9000, 136), (2, 16384, 64)])
+def test_linear_long_rows(dtype, rows, k, n):
+    """GEMV rows of 9000 to 25088 elements (5 to 13 batches of loads per
+    lane, the longest the VGG-16 FC1 row): against the oracle, swapped equal
+    to resident bit for bit."""
+    layers = [dict(op="linear", src=[-1], k=k, n=n, act="relu", res=None, res_post=False)]
+    _check_model(_model(layers, (rows, 1, 1, k), dtype))
+
+
+@pytest.mark.parametrize("k", [4096, 11008])
+def test_swiglu_pair_long_rows(k):
+    """A SwiGLU gate and its paired layer (one merged launch, the gate's
+    stored output used as the pair's residual) at the 7B widths' K (4096)
+    and at the FFN width (11008), one row of bf16 input: against the
+    oracle, swapped (where the two layers may sit in different blocks and
+    run as separate launches) equal to resident bit for bit."""
+    layers = [dict(op="linear", src=[-1], k=k, n=192, act="none", res=None, res_post=False),
+              dict(op="linear", src=[-1], k=k, n=192, act="swiglu", res=0, res_post=False)]
+    _check_model(_model(layers, (1, 1, 1, k), "bf16"))
+
+
 @pytest.mark.parametrize("dtype,ch", [("f16", 24), ("f32", 24), ("f16", 20), ("bf16", 8)])
 def test_pool_upsample_concat(dtype, ch):
     layers = [dict(op="maxpool", src=[-1], kh=3, kw=3, stride=2, pad=1),
