@@ -313,13 +313,24 @@ def llm_cpu_sample(n_dec_sample=2):
     n_dec_sample decode tokens; the embedding, layer and head parts are timed
     separately and scaled to 32 layers and 32 decode tokens.  Returns
     (seconds per whole inference, description)."""
+    return llm_cpu_sampler()(n_dec_sample)
+
+
+def llm_cpu_sampler():
+    """The one-layer model and its weights of llm_cpu_sample, generated once
+    (untimed); returns the sample function, which runs on a fresh KV state
+    at every call."""
     import synth
     from oracle import forward as F
     m1 = synth.arch.llm(layers=1, tokens=512)
     w = synth.gen.model_weights(m1)
     ids = synth.gen.model_input(m1)
-    state = F.new_state()
     nl = len(m1["layers"])
+    return lambda n_dec_sample=2: _llm_cpu_run(F, m1, w, ids, nl, n_dec_sample)
+
+
+def _llm_cpu_run(F, m1, w, ids, nl, n_dec_sample):
+    state = F.new_state()
 
     def parts(x):
         acts, t = {}, []
@@ -1155,8 +1166,10 @@ def run_reference(args, rank, world):
         return
     if args.config == "llm":
         cores = len(os.sched_getaffinity(0))
-        llm_cpu_sample(1)
-        times = [llm_cpu_sample()[0] for _ in range(args.steps)]
+        sampler = llm_cpu_sampler()   # weights generated once, outside the timed samples
+        for _ in range(max(0, min(args.warmup, 1))):
+            sampler(1)
+        times = [sampler()[0] for _ in range(args.steps)]
         ms = 1000.0 * sum(times) / len(times)
         val = 1000.0 / ms
         sample = llm_cpu_sample.__doc__.split("Returns")[0].strip()
