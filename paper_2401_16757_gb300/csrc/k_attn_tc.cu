@@ -15,10 +15,10 @@
 //               written to shared memory as two bf16/fp16 parts p_hi + p_lo
 //               (p_lo = round(p - p_hi)), so the product with V keeps about
 //               16 significant bits of p instead of 8
-//   O_t = P V   tcgen05.mma, M 128 x N 64 x K 16 steps, twice (head dims
-//               0..63 and 64..127) for each part; V is the value tile as
-//               loaded by TMA, [keys][dims] with the dims contiguous, i.e. the
-//               B operand in MN-major layout; O_t in TMEM columns [128, 256)
+//   O_t = P V   tcgen05.mma, M 128 x N 128 x K 16 steps for each part; V
+//               is the value tile as loaded by TMA (two 64-dim boxes),
+//               [keys][dims] with the dims contiguous, i.e. the B operand in
+//               MN-major layout; O_t in TMEM columns [128, 256)
 //   O           the softmax warps keep the row's 128 outputs in registers:
 //               O = O * e^(m_old - m_new) + O_t
 // and at the end write O / l.  Warp 0 issues the TMA loads (key and value
@@ -57,8 +57,9 @@ constexpr uint32_t kTmemCols = 256;  // S: [0, 128), O_t: [128, 256)
 
 // Shared-memory descriptor of a B operand stored MN-major with the 128-byte
 // swizzle (the layout TMA gives a [K rows][64 N] box): 8-row K groups are
-// 1024 bytes apart (stride byte offset); the leading byte offset (between
-// 64-column N blocks) is not used by an N = 64 MMA.
+// 1024 bytes apart (stride byte offset); the two 64-column N blocks of the
+// value tile (the two TMA boxes) are kHalf bytes apart (leading byte
+// offset), so one N = 128 MMA covers all head dims.
 __device__ __forceinline__ uint64_t smem_desc_sw128_mn(uint32_t addr) {
   uint64_t d = 0;
   d |= (uint64_t)((addr & 0x3FFFFu) >> 4);
@@ -165,7 +166,7 @@ __global__ void __launch_bounds__(kAThreads, 1)
       // ---------------- MMA issuer
       constexpr int bf = std::is_same<T, __nv_bfloat16>::value ? 1 : 0;
       constexpr uint32_t idesc_s = idesc_f16(bf, kAQ, kAK);
-      constexpr uint32_t idesc_pv = idesc_f16(bf, kAQ, 64) | (1u << 16);  // B (values) MN-major
+      constexpr uint32_t idesc_pv = idesc_f16(bf, kAQ, kAD) | (1u << 16);  // B (values) MN-major, N = 128
       bool ok = mbar_wait_bounded(q_full, 0, abort_flag, p.err);
       for (int kt = 0; ok && kt < nkt; ++kt) {
         const int s = kt & 1;
@@ -183,15 +184,13 @@ __global__ void __launch_bounds__(kAThreads, 1)
         tc_fence_after();
         const uint32_t va = smem_u32(smem + kOffV + s * kTile);
 #pragma unroll
-        for (int half = 0; half < 2; ++half)
+        for (int part = 0; part < 2; ++part) {
+          const uint32_t pa = smem_u32(smem + (part ? kOffPl : kOffPh));
 #pragma unroll
-          for (int part = 0; part < 2; ++part) {
-            const uint32_t pa = smem_u32(smem + (part ? kOffPl : kOffPh));
-#pragma unroll
-            for (int ks = 0; ks < 8; ++ks)  // 16 keys per step
-              tc_mma_f16(tO + 64 * half, smem_desc_sw128(pa + (ks >> 2) * kHalf) + 2ull * (ks & 3),
-                         smem_desc_sw128_mn(va + half * kHalf + ks * 2048), idesc_pv, (part | ks) != 0);
-          }
+          for (int ks = 0; ks < 8; ++ks)  // 16 keys per step, all 128 head dims (both 64-wide halves)
+            tc_mma_f16(tO, smem_desc_sw128(pa + (ks >> 2) * kHalf) + 2ull * (ks & 3),
+                       smem_desc_sw128_mn(va + ks * 2048), idesc_pv, (part | ks) != 0);
+        }
         tc_commit(o_full);
         tc_commit(kv_empty(s));
       }
