@@ -145,7 +145,7 @@ def test_llm_full_width_layer_prefill_512_and_decode():
 
 def test_llm_long_prefill_many_heads():
     """128 queries x 8 heads: the prefill takes the tensor-core attention
-    kernel, the decode steps after it the CTA-per-query kernel."""
+    kernel, the decode steps after it the split-key cluster kernel."""
     dec = Decoder(prefill_tokens=128, **WIDE)
     ids = synth.gen.model_input(dec.mp).reshape(-1)
     st = F.new_state()
