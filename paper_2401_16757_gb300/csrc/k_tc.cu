@@ -275,12 +275,23 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int q = warp & 3;
     const int row = q * 32 + lane;
     const int m = row_m(row);  // -1: this row has no output
+    const bool vec_ok = ((p.ldy | n0) % 8 == 0) && (!p.e.res || ((p.e.ldr | n0) % 8 == 0));
+    // without a split, the residual of the first 32 columns is requested
+    // while the MMAs run, each later chunk's one chunk ahead of its use
+    const bool has_res = splits == 1 && p.e.res != nullptr;
+    uint4 rnext[4];
+    if (has_res) res_prefetch32<T>(rnext, p, m, n0, vec_ok);
     const bool ok = mbar_wait_bounded(accum_bar, 0, abort_flag, p.err);
     tc_fence_after();
-    const bool vec_ok = ((p.ldy | n0) % 8 == 0) && (!p.e.res || ((p.e.ldr | n0) % 8 == 0));
     if (ok && splits == 1) {
 #pragma unroll 1
       for (int c0 = 0; c0 < BN; c0 += 32) {
+        uint4 rcur[4];
+        if (has_res) {
+#pragma unroll
+          for (int i = 0; i < 4; ++i) rcur[i] = rnext[i];
+          if (c0 + 32 < BN) res_prefetch32<T>(rnext, p, m, n0 + c0 + 32, vec_ok);
+        }
         uint32_t r[32];
         tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)c0, r);
         tmem_ld_wait();
@@ -288,7 +299,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           float v[32];
 #pragma unroll
           for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-          finish32<T>(v, sbias + c0, p, m, n0 + c0, vec_ok);
+          if (has_res) finish32r<T>(v, sbias + c0, p, m, n0 + c0, vec_ok, rcur);
+          else finish32<T>(v, sbias + c0, p, m, n0 + c0, vec_ok);
         }
       }
     } else if (csplit && BN == 256) {
@@ -702,7 +714,12 @@ int tc_prepare(const TcGemm& g, TcPlan* p) {
     // costs about the same (~0.5 us) whatever the tile width, so the time is
     // about waves x k-blocks and wider tiles mean fewer waves; a third of the
     // SMs busy with one wide tile each still beats splitting K across them
-    const int pbn = Nd <= 64 ? 64 : (Nd <= 128 ? 128 : 256);
+    int pbn = Nd <= 64 ? 64 : (Nd <= 128 ? 128 : 256);
+    // with at most half as many 256-wide tiles as SMs, 128-wide tiles (twice
+    // the CTAs) were measured faster: the 512-token decoder projections
+    // 25.8 -> 23.4 us (q, k, v), 32.3 -> 26.7 us (o), 74.1 -> 57.1 us (down),
+    // VGG-16 b16's 14x14 convolutions 27.8 -> 25.1 us
+    if (pbn == 256 && sp_tiles * ((Nd + 255) / 256) * 2 <= sms) pbn = 128;
     if (sp_tiles * ((Nd + pbn - 1) / pbn) * 3 >= sms) {
       p->persist = 1;
       if (tmac) {

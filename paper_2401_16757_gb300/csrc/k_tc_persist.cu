@@ -286,14 +286,10 @@ __global__ void __launch_bounds__(persist_threads<AMODE>(), 1)
       const T* bias = static_cast<const T*>(p.e.bias);
       for (int j = lane; j < BN; j += 32) sb[j] = (bias && n0 + j < p.N) ? to_f<T>(bias[n0 + j]) : 0.f;
       __syncwarp();
-      const bool got = mbar_wait_bounded(tfull0 + 8u * buf, use & 1, abort_flag, p.err);
-      if (!__all_sync(0xffffffffu, got)) break;  // tcgen05.ld is warp-collective
-      tc_fence_after();
-      const bool vec_ok = ((p.ldy | n0) % 8 == 0) && (!p.e.res || ((p.e.ldr | n0) % 8 == 0));
-#pragma unroll 1
-      for (int sub = 0; sub < MS; ++sub) {
+      // output row of this thread's TMEM lane in sub-tile sub, -1 when unused
+      auto row_of = [&](int sub) {
         const int idx = (tile % mtp) * MS + sub;  // m-tile (or pixel patch) of this sub-tile
-        int m = -1;  // output row of this thread's TMEM lane, -1 when unused
+        int m = -1;
         if (idx < mt) {
           if (AMODE == kATap) {
             const int img = idx / patches, rem = idx - img * patches;
@@ -307,8 +303,31 @@ __global__ void __launch_bounds__(persist_threads<AMODE>(), 1)
             if (m >= p.M) m = -1;
           }
         }
+        return m;
+      };
+      const bool vec_ok = ((p.ldy | n0) % 8 == 0) && (!p.e.res || ((p.e.ldr | n0) % 8 == 0));
+      // with a residual, the residual of the first 32 columns is requested
+      // while the accumulator is still being computed, each later chunk's
+      // one chunk ahead of its use (layers without one keep the plain loop:
+      // the extra work slowed the short-K, N = 64 convolutions)
+      const bool has_res = p.e.res != nullptr;
+      uint4 rnext[4];
+      if (has_res) res_prefetch32<T>(rnext, p, row_of(0), n0, vec_ok);
+      const bool got = mbar_wait_bounded(tfull0 + 8u * buf, use & 1, abort_flag, p.err);
+      if (!__all_sync(0xffffffffu, got)) break;  // tcgen05.ld is warp-collective
+      tc_fence_after();
+#pragma unroll 1
+      for (int sub = 0; sub < MS; ++sub) {
+        const int m = row_of(sub);
 #pragma unroll 1
         for (int c0 = 0; c0 < BN; c0 += 32) {
+          uint4 rcur[4];
+          if (has_res) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) rcur[i] = rnext[i];
+            if (c0 + 32 < BN) res_prefetch32<T>(rnext, p, m, n0 + c0 + 32, vec_ok);
+            else if (sub + 1 < MS) res_prefetch32<T>(rnext, p, row_of(sub + 1), n0, vec_ok);
+          }
           uint32_t r[32];
           tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)((buf * MS + sub) * BN + c0), r);
           tmem_ld_wait();
@@ -316,7 +335,8 @@ __global__ void __launch_bounds__(persist_threads<AMODE>(), 1)
             float v[32];
 #pragma unroll
             for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-            finish32<T>(v, sb + c0, p, m, n0 + c0, vec_ok);
+            if (has_res) finish32r<T>(v, sb + c0, p, m, n0 + c0, vec_ok, rcur);
+            else finish32<T>(v, sb + c0, p, m, n0 + c0, vec_ok);
           }
         }
       }

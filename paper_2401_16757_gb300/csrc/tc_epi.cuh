@@ -47,6 +47,39 @@ template <> __device__ __forceinline__ float hi_f<__half>(uint32_t u) {
 template <> __device__ __forceinline__ float lo_f<__nv_bfloat16>(uint32_t u) { return __uint_as_float(u << 16); }
 template <> __device__ __forceinline__ float hi_f<__nv_bfloat16>(uint32_t u) { return __uint_as_float(u & 0xffff0000u); }
 
+// 8 consecutive outputs (16 bytes): acc -> bias, residual (the 8 stored
+// values r, when has_res), activation -> T.
+template <typename T>
+__device__ __forceinline__ void epi8r(const float (&a)[8], const float* sb, uint4 r, bool has_res, T* out, int act,
+                                      int res_post) {
+  const float4 b0 = *reinterpret_cast<const float4*>(sb);
+  const float4 b1 = *reinterpret_cast<const float4*>(sb + 4);
+  const float bf[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+  const uint32_t rw[4] = {r.x, r.y, r.z, r.w};
+  uint32_t o[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float v0 = epilogue(a[2 * i], bf[2 * i], lo_f<T>(rw[i]), has_res, act, res_post);
+    const float v1 = epilogue(a[2 * i + 1], bf[2 * i + 1], hi_f<T>(rw[i]), has_res, act, res_post);
+    o[i] = pack2<T>(v0, v1);
+  }
+  *reinterpret_cast<uint4*>(out) = make_uint4(o[0], o[1], o[2], o[3]);
+}
+
+// The residual of 32 columns [n, n+32) of row m as four 16-byte loads, for
+// the vector path of finish32 (zeros when there is no residual or the
+// vector path does not apply).  Issued a chunk ahead, so that the loads'
+// latency overlaps the accumulator reads and the arithmetic of the chunk
+// before.
+template <typename T>
+__device__ __forceinline__ void res_prefetch32(uint4 (&r)[4], const TcArgs& p, int m, int n, bool vec_ok) {
+  const T* res = static_cast<const T*>(p.e.res);
+  const bool ok = res && m >= 0 && vec_ok && n + 32 <= p.N;
+#pragma unroll
+  for (int q = 0; q < 4; ++q)
+    r[q] = ok ? *reinterpret_cast<const uint4*>(res + (int64_t)m * p.e.ldr + n + 8 * q) : make_uint4(0, 0, 0, 0);
+}
+
 // 8 consecutive outputs (16 bytes): acc -> bias, residual, activation -> T.
 template <typename T>
 __device__ __forceinline__ void epi8(const float (&a)[8], const float* sb, const T* res, T* out, int act,
@@ -90,6 +123,26 @@ __device__ __forceinline__ void finish32(const float (&v)[32], const float* sb, 
         y[n + j] = from_f<T>(epilogue(v[j], sb[j], rv, rrow != nullptr, p.e.act, p.e.res_post));
       }
     }
+  }
+}
+
+// finish32 with the residual already loaded by res_prefetch32 (same
+// arithmetic; the scalar path, for ragged or unaligned columns, loads it
+// itself).
+template <typename T>
+__device__ __forceinline__ void finish32r(const float (&v)[32], const float* sb, const TcArgs& p, int m, int n,
+                                          bool vec_ok, const uint4 (&r)[4]) {
+  if (vec_ok && n + 32 <= p.N) {
+    T* y = static_cast<T*>(p.y) + (int64_t)m * p.ldy;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      float a[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) a[j] = v[8 * q + j];
+      epi8r<T>(a, sb + 8 * q, r[q], p.e.res != nullptr, y + n + 8 * q, p.e.act, p.e.res_post);
+    }
+  } else {
+    finish32<T>(v, sb, p, m, n, vec_ok);
   }
 }
 
