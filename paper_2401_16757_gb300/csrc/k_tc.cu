@@ -277,8 +277,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int m = row_m(row);  // -1: this row has no output
     const bool vec_ok = ((p.ldy | n0) % 8 == 0) && (!p.e.res || ((p.e.ldr | n0) % 8 == 0));
     // without a split, the residual of the first 32 columns is requested
-    // while the MMAs run, each later chunk's one chunk ahead of its use
-    const bool has_res = splits == 1 && p.e.res != nullptr;
+    // while the MMAs run, each later chunk's one chunk ahead of its use (zeros
+    // for layers without one: one loop for both measured faster than two)
+    const bool has_res = splits == 1;
     uint4 rnext[4];
     if (has_res) res_prefetch32<T>(rnext, p, m, n0, vec_ok);
     const bool ok = mbar_wait_bounded(accum_bar, 0, abort_flag, p.err);
