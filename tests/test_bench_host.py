@@ -93,3 +93,22 @@ def test_reference_arm_other_ranks_exit_quietly():
     r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--config", "mlp6",
                         "--steps", "1", "--warmup", "0"], capture_output=True, text=True, timeout=600, env=env)
     assert r.returncode == 0 and r.stdout.strip() == ""
+
+
+def test_host_placement_reads_the_node_of_a_page():
+    """The link record's placement reading (a host-side query, no GPU
+    setting): the online NUMA nodes as the kernel lists them, and the node
+    of a touched page of ordinary memory, which must be one of them."""
+    import ctypes
+    buf = (ctypes.c_uint8 * (1 << 16))()
+    ctypes.memset(buf, 1, 1 << 16)
+    got = bench.host_placement(ctypes.addressof(buf))
+    online = got["numa_nodes_online"]
+    if online is None:
+        pytest.skip("no NUMA information on this host")
+    nodes = set()
+    for part in online.split(","):
+        lo, _, hi = part.partition("-")
+        nodes.update(range(int(lo), int(hi or lo) + 1))
+    if "pinned_page_node" in got and got["pinned_page_node"] is not None:
+        assert got["pinned_page_node"] in nodes
