@@ -1,6 +1,8 @@
 // Decoder-layer kernels: embedding gather (zero-copy from the host-resident
-// table), RMSNorm, RoPE + KV-cache append, causal attention with an online
-// softmax, row argmax, and the device-side advance of the cache position.
+// table), RMSNorm, RoPE + KV-cache append, causal attention for short query
+// runs (the decode step: keys split over a thread-block cluster) and for
+// long runs the tensor cores do not take (warp per query, online softmax),
+// row argmax, and the device-side advance of the cache position.
 // bf16 / fp16 storage, fp32 arithmetic, fixed reduction orders.
 #include <cooperative_groups.h>
 
