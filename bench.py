@@ -1535,18 +1535,48 @@ def run_cnn(args, rank, world, group, name, compact=False):
     if tr and tr[0] == roofline["traffic_sources_sha"]:
         roofline["traffic"] = tr[1]
 
-    # ---- host link: one profiled pass per step (events around each swap on
-    # the copy stream), bytes per swap over swap time, against the pinned
-    # memcpy peak
-    eng.set_profiling(True)
-    acc_s = np.zeros(len(blocks))
+    # ---- host link: each swap-in timed inside the replayed graph (event
+    # nodes on the copy stream only), bytes per swap over swap time, against
+    # the pinned memcpy peak
     prof_steps = min(10, args.steps)
+    eng.set_swap_timing(True)
+    for _ in range(2):
+        eng.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
+    acc_s = np.zeros(len(blocks))
     for _ in range(prof_steps):
         flush.zero_()
         eng.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
-        acc_s += np.array(eng.last_times(len(units), len(blocks))[1])
-    eng.set_profiling(False)
+        acc_s += np.array(eng.last_swap_times(len(blocks)))
+    eng.set_swap_timing(False)
     acc_s /= prof_steps
+    # ---- where the swapped time goes: the block timeline of the replayed
+    # graph (event nodes on both streams; those between blocks add a
+    # dependent launch at every block boundary, so this replay runs slower
+    # than the timed step and explains it rather than measures it)
+    eng.set_graph_timeline(True)
+    for _ in range(2):
+        eng.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
+    tls, replay_us = [], []
+    for _ in range(prof_steps):
+        flush.zero_()
+        a_, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a_.record(stream)
+        eng.infer(d_in.data_ptr(), d_out.data_ptr(), sp)
+        b_.record(stream)
+        b_.synchronize()
+        replay_us.append(a_.elapsed_time(b_) * 1e3)
+        tls.append(eng.last_graph_timeline(len(blocks)))
+    eng.set_graph_timeline(False)
+    tl = [[statistics.median(t[k][j] for t in tls) for j in range(4)] for k in range(len(blocks))]
+    # time the layers waited for a swap: a block's swap ending after the
+    # previous block's layers (the start of the inference for block 0)
+    waited = [max(0.0, b[1] - (tl[k - 1][3] if k else 0.0)) if b[1] >= 0 else 0.0 for k, b in enumerate(tl)]
+    line["graph_timeline"] = {
+        "replay_us": statistics.median(replay_us), "step_us": ms_swapped * 1e3,
+        "blocks_us": [[round(v, 1) for v in b] for b in tl],
+        "columns": ["swap start", "swap end", "layers start", "layers end"],
+        "layers_waited_for_swap_us": [round(v, 1) for v in waited],
+        "layers_us": round(sum(b[3] - b[2] for b in tl), 1)}
     swap_bytes = sum(b["bytes"] for b in blocks)
     swap_us = float(acc_s.sum())
     link_peak = measure_link_peak(stream)

@@ -538,6 +538,24 @@ int swapnet_engine_last_times(swapnet_engine* eng, float* unit_us, uint32_t n_un
 int swapnet_engine_set_swap_timing(swapnet_engine* eng, int enable);
 int swapnet_engine_last_swap_times(swapnet_engine* eng, float* swap_us, uint32_t n_blocks);
 
+/* The pipeline of Sec. 4.3 as it runs inside the replayed inference graph:
+ * with the timeline on, the engine captures (and caches) a graph variant
+ * that also records an event on the caller's stream at the start of the
+ * inference and right before and after each block's layers, besides the
+ * swap-in events above.  swapnet_engine_last_graph_timeline waits for the
+ * most recent inference's last block and writes 4 floats per block to
+ * t_us[4 * k .. 4 * k + 3], microseconds since the start of that inference:
+ * swap-in start, swap-in end (both -1 for blocks that are not swapped in
+ * during the inference: a resident prefix, blocks read in place, the first
+ * block under first-block prefetch, every block of a resident plan), start
+ * and end of the block's layers on the caller's stream.  The extra nodes
+ * sit between the last layer of one block and the first of the next, so
+ * they can add the cost of a dependent launch at each block boundary; the
+ * timeline explains a replay, swapnet_infer without it is the one to time.
+ * Errors: INVALID_ARG (null engine or output, timeline never enabled), CUDA. */
+int swapnet_engine_set_graph_timeline(swapnet_engine* eng, int enable);
+int swapnet_engine_last_graph_timeline(swapnet_engine* eng, float* t_us, uint32_t n_blocks);
+
 /* The offline fit of the delay model on this device (Sec. 6.1: the paper
  * profiles each device once and fits t_ex = gamma * f and t_in = alpha * s +
  * beta * d by linear regression).  Here the execution delays are measured

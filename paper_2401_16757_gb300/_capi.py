@@ -100,6 +100,7 @@ EXPORTS = ["swapnet_default_options", "swapnet_partition", "swapnet_plan_from_cu
            "swapnet_engine_set_profiling", "swapnet_engine_last_times", "swapnet_engine_measure_units",
            "swapnet_engine_last_timeline", "swapnet_engine_calibrate",
            "swapnet_engine_set_swap_timing", "swapnet_engine_last_swap_times",
+           "swapnet_engine_set_graph_timeline", "swapnet_engine_last_graph_timeline",
            "swapnet_engine_bind_state", "swapnet_strerror", "swapnet_last_error", "swapnet_debug_fail_next", "swapnet_gemm_noalloc",
            "swapnet_weights_file_write", "swapnet_weights_file_open", "swapnet_weights_file_info",
            "swapnet_weights_file_read", "swapnet_weights_file_close", "swapnet_load_file",
@@ -155,6 +156,8 @@ def lib():
         "swapnet_engine_set_profiling": (C.c_int, [P, C.c_int]),
         "swapnet_engine_set_swap_timing": (C.c_int, [P, C.c_int]),
         "swapnet_engine_last_swap_times": (C.c_int, [P, C.POINTER(C.c_float), C.c_uint32]),
+        "swapnet_engine_set_graph_timeline": (C.c_int, [P, C.c_int]),
+        "swapnet_engine_last_graph_timeline": (C.c_int, [P, C.POINTER(C.c_float), C.c_uint32]),
         "swapnet_engine_measure_units": (C.c_int, [P, C.c_int32, C.POINTER(C.c_float), C.c_uint32]),
         "swapnet_engine_last_timeline": (C.c_int, [P, C.POINTER(C.c_float), C.POINTER(C.c_float), C.c_uint32,
                                                    C.POINTER(C.c_float), C.POINTER(C.c_float), C.c_uint32]),
@@ -540,6 +543,18 @@ class Engine:
         b = (C.c_float * max(1, n_blocks))()
         check(lib().swapnet_engine_last_swap_times(self.h, b, n_blocks), "swapnet_engine_last_swap_times")
         return list(b[:n_blocks])
+
+    def set_graph_timeline(self, enable):
+        check(lib().swapnet_engine_set_graph_timeline(self.h, 1 if enable else 0),
+              "swapnet_engine_set_graph_timeline")
+
+    def last_graph_timeline(self, n_blocks):
+        """Per block (swap start, swap end, layers start, layers end) of the
+        last inference, microseconds since its start, timed inside its graph
+        (-1 for a swap that did not happen in that inference)."""
+        b = (C.c_float * max(4, 4 * n_blocks))()
+        check(lib().swapnet_engine_last_graph_timeline(self.h, b, n_blocks), "swapnet_engine_last_graph_timeline")
+        return [tuple(b[4 * k:4 * k + 4]) for k in range(n_blocks)]
 
     def measure_units(self, n_units, reps=20):
         u = (C.c_float * max(1, n_units))()

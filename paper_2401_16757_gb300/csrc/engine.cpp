@@ -115,10 +115,16 @@ struct swapnet_engine {
   // block's swap-in on the copy stream (swapnet_engine_set_swap_timing)
   bool swap_timing = false;
   std::vector<cudaEvent_t> ev_gswap;  // 2 per block
+  // block timeline inside the replayed graph (swapnet_engine_set_graph_timeline):
+  // also an event at the start of the inference on the caller's stream and
+  // around each block's layers
+  bool timeline = false;
+  std::vector<cudaEvent_t> ev_gexec;  // 2 per block
+  cudaEvent_t ev_g0 = nullptr;
   cudaStream_t cap = nullptr;        // capture origin stream
   cudaEvent_t fork = nullptr, join = nullptr;
   // per (input, output, profiling) binding
-  std::map<std::pair<std::pair<const void*, void*>, bool>, cudaGraphExec_t> graphs;
+  std::map<std::pair<std::pair<const void*, void*>, int>, cudaGraphExec_t> graphs;
   char* d_state = nullptr;           // decoder state (position + KV caches), caller-owned
   // concurrent branches: side units run on `side`, forked after their last
   // producer's unit and joined before their first consumer's
@@ -175,6 +181,8 @@ static int release(swapnet_engine* e) {
   for (cudaEvent_t ev : e->ev_unit) cudaEventDestroy(ev);
   for (cudaEvent_t ev : e->ev_swap) cudaEventDestroy(ev);
   for (cudaEvent_t ev : e->ev_gswap) cudaEventDestroy(ev);
+  for (cudaEvent_t ev : e->ev_gexec) cudaEventDestroy(ev);
+  if (e->ev_g0) cudaEventDestroy(e->ev_g0);
   if (e->copy) cudaStreamDestroy(e->copy);
   if (e->rd) {
     cudaStreamSynchronize(e->rd);
@@ -1293,6 +1301,11 @@ static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t 
   const bool pf = prefetch_on(e);
   bool used[2] = {false, false};
   bool stage_used[2] = {false, false};
+  // in a captured graph an event-record node (external event), eagerly a
+  // plain record
+  const unsigned gflag = capturing ? cudaEventRecordExternal : cudaEventRecordDefault;
+  const bool swap_ev = e->swap_timing || e->timeline;
+  if (e->timeline) CU(cudaEventRecordWithFlags(e->ev_g0, s, gflag), "timeline event");
   if (!p.resident) {
     CU(cudaEventRecord(e->fork, s), "record fork");
     CU(cudaStreamWaitEvent(e->copy, e->fork, 0), "wait fork");
@@ -1318,13 +1331,11 @@ static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t 
     } else if (prof) {
       CU(cudaEventRecord(e->ev_swap[2 * k], e->copy), "profile event");
     }
-    // in a captured graph an event-record node (external event), eagerly a
-    // plain record: either way the copy stream's own time for this swap
-    const unsigned gflag = capturing ? cudaEventRecordExternal : cudaEventRecordDefault;
-    if (e->swap_timing) CU(cudaEventRecordWithFlags(e->ev_gswap[2 * k], e->copy, gflag), "swap timing event");
+    // the copy stream's own time for this swap
+    if (swap_ev) CU(cudaEventRecordWithFlags(e->ev_gswap[2 * k], e->copy, gflag), "swap timing event");
     int rc = swap_block(e, k, e->blocks[k].variant, e->copy);
     if (rc) return rc;
-    if (e->swap_timing) CU(cudaEventRecordWithFlags(e->ev_gswap[2 * k + 1], e->copy, gflag), "swap timing event");
+    if (swap_ev) CU(cudaEventRecordWithFlags(e->ev_gswap[2 * k + 1], e->copy, gflag), "swap timing event");
     if (e->file) {
       CU(cudaEventRecord(e->stage_free[j], e->copy), "record staging free");
       stage_used[j] = true;
@@ -1347,6 +1358,7 @@ static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t 
         if (rc) return rc;
       }
     }
+    if (e->timeline) CU(cudaEventRecordWithFlags(e->ev_gexec[2 * k], s, gflag), "timeline event");
     for (int u = B.u0; u < B.u1; ++u) {
       if (e->is_side[u]) continue;  // launched on the side stream after its producer
       if (e->merged_into[u]) continue;  // launched with an earlier unit
@@ -1371,6 +1383,7 @@ static int enqueue(swapnet_engine* e, const void* din, void* dout, cudaStream_t 
         }
       }
     }
+    if (e->timeline) CU(cudaEventRecordWithFlags(e->ev_gexec[2 * k + 1], s, gflag), "timeline event");
     if (swap_k) CU(cudaEventRecord(e->slot_free[B.slot], s), "record slot free");
   }
   if (p.model.has_attention) {
@@ -1443,7 +1456,7 @@ int swapnet_infer(swapnet_engine* e, const void* din, void* dout, swapnet_stream
   CU(cudaSetDevice(e->device), "cudaSetDevice");
   // event timing needs eager launches; stream capture takes no copy from pageable memory
   if (e->plan.opt.graphs && !e->profiling && !(e->plan.opt.pageable && !e->file)) {
-    const auto key = std::make_pair(std::make_pair(din, dout), e->swap_timing);
+    const auto key = std::make_pair(std::make_pair(din, dout), (e->swap_timing ? 1 : 0) | (e->timeline ? 2 : 0));
     auto it = e->graphs.find(key);
     if (it == e->graphs.end()) {
       if (e->graphs.size() >= 8) {
@@ -1683,6 +1696,51 @@ int swapnet_engine_last_swap_times(swapnet_engine* e, float* swap_us, uint32_t n
       CU(cudaEventElapsedTime(&ms, e->ev_gswap[2 * k], e->ev_gswap[2 * k + 1]), "elapsed");
     }
     swap_us[k] = ms * 1000.f;
+  }
+  return SWAPNET_OK;
+}
+
+int swapnet_engine_set_graph_timeline(swapnet_engine* e, int enable) {
+  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+  CU(cudaSetDevice(e->device), "cudaSetDevice");
+  if (enable && e->ev_gswap.empty()) {
+    e->ev_gswap.assign(2 * e->plan.blocks.size(), nullptr);
+    for (cudaEvent_t& ev : e->ev_gswap) CU(cudaEventCreate(&ev), "event");
+  }
+  if (enable && e->ev_gexec.empty()) {
+    e->ev_gexec.assign(2 * e->plan.blocks.size(), nullptr);
+    for (cudaEvent_t& ev : e->ev_gexec) CU(cudaEventCreate(&ev), "event");
+    CU(cudaEventCreate(&e->ev_g0), "event");
+  }
+  e->timeline = enable != 0;
+  return SWAPNET_OK;
+}
+
+int swapnet_engine_last_graph_timeline(swapnet_engine* e, float* t_us, uint32_t nb) {
+  if (!e || !t_us) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+  if (e->ev_gexec.empty()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "the timeline was never enabled");
+  CU(cudaSetDevice(e->device), "cudaSetDevice");
+  const uint32_t n = std::min<uint32_t>(nb, (uint32_t)e->plan.blocks.size());
+  if (n) CU(cudaEventSynchronize(e->ev_gexec[2 * (n - 1) + 1]), "event synchronize");
+  auto since = [&](cudaEvent_t ev, float* out) -> int {
+    float ms = 0.f;
+    CU(cudaEventSynchronize(ev), "event synchronize");
+    CU(cudaEventElapsedTime(&ms, e->ev_g0, ev), "elapsed");
+    *out = ms * 1000.f;
+    return SWAPNET_OK;
+  };
+  for (uint32_t k = 0; k < n; ++k) {
+    float* o = t_us + 4 * k;
+    o[0] = o[1] = -1.f;
+    const bool pf_first = k == 0 && prefetch_on(e);
+    if (swapped(e, k) && !pf_first) {
+      int rc = since(e->ev_gswap[2 * k], o);
+      if (!rc) rc = since(e->ev_gswap[2 * k + 1], o + 1);
+      if (rc) return rc;
+    }
+    int rc = since(e->ev_gexec[2 * k], o + 2);
+    if (!rc) rc = since(e->ev_gexec[2 * k + 1], o + 3);
+    if (rc) return rc;
   }
   return SWAPNET_OK;
 }

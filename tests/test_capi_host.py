@@ -408,9 +408,12 @@ def test_calibrate_rejects_a_null_engine():
 
 
 def test_swap_timing_calls_reject_a_null_engine_or_output():
-    """The in-graph swap timing calls check their arguments before touching
-    a device (no GPU needed)."""
+    """The in-graph swap timing and timeline calls check their arguments
+    before touching a device (no GPU needed)."""
     us = (capi.C.c_float * 4)()
     assert capi.lib().swapnet_engine_set_swap_timing(None, 1) == capi.ERR_INVALID_ARG
     assert capi.lib().swapnet_engine_last_swap_times(None, us, 4) == capi.ERR_INVALID_ARG
+    assert b"null" in capi.lib().swapnet_last_error()
+    assert capi.lib().swapnet_engine_set_graph_timeline(None, 1) == capi.ERR_INVALID_ARG
+    assert capi.lib().swapnet_engine_last_graph_timeline(None, us, 1) == capi.ERR_INVALID_ARG
     assert b"null" in capi.lib().swapnet_last_error()

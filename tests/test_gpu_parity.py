@@ -526,3 +526,104 @@ def test_swap_times_inside_the_replayed_graph(variant):
     got = sw.run(x)
     assert all(p.tobytes() == q.tobytes() for p, q in zip(got, ref))
     sw.engine.sync()
+
+
+def _min_feasible_budget(d, opt, hi):
+    """Smallest multiple of 256 bytes the planner accepts (feasibility grows
+    with the budget)."""
+    lo = 0                       # infeasible
+    while hi - lo > 256:
+        mid = (lo + hi) // 2 // 256 * 256
+        mid = max(mid, lo + 256)
+        try:
+            capi.Plan.partition(d, mid, opt)
+            hi = mid
+        except capi.SwapnetError as e:
+            assert e.code == capi.ERR_INFEASIBLE
+            lo = mid
+    return hi
+
+
+def test_degenerate_budgets_bit_exact():
+    """The edge budgets run and equal resident bit for bit: the smallest
+    budget the planner accepts (256 bytes less is refused as infeasible), and
+    four times the weight bytes, where the paper's method still swaps every
+    block while a resident prefix keeps the whole model in one block that is
+    never swapped."""
+    layers = [_conv(-1, 16, 32, 3), _conv(0, 32, 64, 3, stride=2), _conv(1, 64, 64, 1, res=1),
+              dict(op="maxpool", src=[2], kh=2, kw=2, stride=2, pad=0),
+              dict(op="gap", src=[3]),
+              dict(op="linear", src=[4], k=64, n=40, act="none", res=None, res_post=False)]
+    m = _model(layers, (1, 24, 24, 16))
+    w = synth.gen.model_weights(m)
+    x = synth.gen.model_input(m)
+    d = capi.Desc(m)
+    host = capi.HostWeights(w)
+    wb = OP.weight_bytes(m)
+    base = Runner(m, w, capi.Plan.resident(d), host).run(x)[0].tobytes()
+    opt = capi.options()
+    lo = _min_feasible_budget(d, opt, 4 * wb // 256 * 256)
+    with pytest.raises(capi.SwapnetError) as ei:
+        capi.Plan.partition(d, lo - 256, opt)
+    assert ei.value.code == capi.ERR_INFEASIBLE
+    tight = Runner(m, w, capi.Plan.partition(d, lo, opt), host)
+    assert tight.info["n_blocks"] >= 3
+    assert tight.run(x)[0].tobytes() == base
+    big = 4 * wb // 256 * 256
+    sw = Runner(m, w, capi.Plan.partition(d, big, opt), host)
+    before = sw.engine.stats()["bytes_swapped"]
+    assert sw.run(x)[0].tobytes() == base
+    swapped = sw.engine.stats()["bytes_swapped"] - before    # every tensor, padding between them included
+    n_tensors = sum(len(t) for t in w)
+    assert wb - 256 * n_tensors < swapped <= wb, (swapped, wb)
+    pre = Runner(m, w, capi.Plan.partition(d, big, capi.options(resident_prefix=1)), host)
+    assert pre.info["n_blocks"] == 1 and pre.info["prefix_units"] == pre.info["n_units"]
+    before = pre.engine.stats()["bytes_swapped"]
+    for _ in range(2):
+        got = pre.run(x)
+        assert got[0].tobytes() == base
+    assert pre.engine.stats()["bytes_swapped"] == before
+    check_close(m, pre.decode(got), oracle_outputs(m, w, x))
+
+
+@pytest.mark.parametrize("variant", [capi.SWAP_MEMCPY, capi.SWAP_ZEROCOPY])
+def test_graph_timeline_follows_the_pipeline_order(variant):
+    """The block timeline of a replayed inference graph obeys the ordering
+    of the Sec. 4.3 pipeline: swaps one after another on the copy stream,
+    each block's layers after its own swap and after the previous block's
+    layers, a block's swap after the layers of the block that last held
+    its place (two blocks back); everything inside the inference's own time
+    on its stream.  The outputs stay the resident bits."""
+    import torch
+    m = synth.arch.MODELS["resnet50"]()
+    w = synth.gen.model_weights(m)
+    d = capi.Desc(m)
+    host = capi.HostWeights(w)
+    wb = OP.weight_bytes(m)
+    plan = capi.Plan.partition(d, int(wb * 0.4) // 256 * 256, capi.options(swap_variant=variant))
+    nb = plan.info()["n_blocks"]
+    assert nb >= 3
+    sw = Runner(m, w, plan, host)
+    ref = Runner(m, w, capi.Plan.resident(d), host).run(synth.gen.model_input(m))
+    sw.engine.set_graph_timeline(True)
+    got = sw.run(synth.gen.model_input(m))
+    assert all(p.tobytes() == q.tobytes() for p, q in zip(got, ref))
+    s = torch.cuda.current_stream()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(s)
+    sw.engine.infer(sw.d_in.data_ptr(), sw.d_out.data_ptr(), s.cuda_stream)
+    b.record(s)
+    b.synchronize()
+    tl = sw.engine.last_graph_timeline(nb)
+    eps = 1.0                                   # event resolution, microseconds
+    for k, (s0, s1, e0, e1) in enumerate(tl):
+        assert 0.0 <= s0 <= s1 + eps and s1 <= e0 + eps and e0 <= e1 + eps, (k, tl[k])
+        if k:
+            assert tl[k - 1][3] <= e0 + eps and tl[k - 1][1] <= s0 + eps, (k, tl[k - 1], tl[k])
+        if k >= 2:
+            assert tl[k - 2][3] <= s0 + eps, (k, tl[k - 2], tl[k])
+    assert tl[-1][3] <= a.elapsed_time(b) * 1e3 + eps
+    sw.engine.set_graph_timeline(False)
+    got = sw.run(synth.gen.model_input(m))
+    assert all(p.tobytes() == q.tobytes() for p, q in zip(got, ref))
+    sw.engine.sync()
