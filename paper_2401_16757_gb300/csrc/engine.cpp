@@ -1086,8 +1086,12 @@ static void unbind_plan(swapnet_engine* e) {
   e->side_done.clear();
   for (cudaEvent_t ev : e->ev_unit) cudaEventDestroy(ev);
   for (cudaEvent_t ev : e->ev_swap) cudaEventDestroy(ev);
+  for (cudaEvent_t ev : e->ev_gswap) cudaEventDestroy(ev);
+  for (cudaEvent_t ev : e->ev_gexec) cudaEventDestroy(ev);
   e->ev_unit.clear();
   e->ev_swap.clear();
+  e->ev_gswap.clear();
+  e->ev_gexec.clear();
   if (e->d_splitk) cudaFree(e->d_splitk);
   e->d_splitk = nullptr;
   e->splitk_bytes = e->splitk_counter_bytes = 0;
@@ -1201,15 +1205,18 @@ int swapnet_engine_adapt(swapnet_engine* e, const swapnet_plan* plan) {
   } catch (const std::bad_alloc&) {
     SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
   }
+  // per-unit and per-block events were sized for the old plan: they are
+  // made again for the new one after binding it (whose swap-variant
+  // calibration captures inferences without them)
+  const bool prof = e->profiling, st = e->swap_timing, tl = e->timeline;
+  e->profiling = e->swap_timing = e->timeline = false;
   // an engine given a caller arena keeps it (the new plan must fit it)
   int rc = swapnet::bind_plan(e, e->own_arena ? nullptr : e->d_arena, e->own_arena ? 0 : e->arena_bytes, false);
   if (rc) return rc;
-  if (e->profiling) {
-    e->profiling = false;
-    rc = swapnet_engine_set_profiling(e, 1);
-    if (rc) return rc;
-  }
-  return SWAPNET_OK;
+  if (prof) rc = swapnet_engine_set_profiling(e, 1);
+  if (!rc && st) rc = swapnet_engine_set_swap_timing(e, 1);
+  if (!rc && tl) rc = swapnet_engine_set_graph_timeline(e, 1);
+  return rc;
 }
 
 }  // extern "C"
@@ -1710,7 +1717,7 @@ int swapnet_engine_set_graph_timeline(swapnet_engine* e, int enable) {
   if (enable && e->ev_gexec.empty()) {
     e->ev_gexec.assign(2 * e->plan.blocks.size(), nullptr);
     for (cudaEvent_t& ev : e->ev_gexec) CU(cudaEventCreate(&ev), "event");
-    CU(cudaEventCreate(&e->ev_g0), "event");
+    if (!e->ev_g0) CU(cudaEventCreate(&e->ev_g0), "event");
   }
   e->timeline = enable != 0;
   return SWAPNET_OK;

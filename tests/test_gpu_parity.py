@@ -586,6 +586,17 @@ def test_degenerate_budgets_bit_exact():
     check_close(m, pre.decode(got), oracle_outputs(m, w, x))
 
 
+def _check_pipeline_order(tl, total_us):
+    eps = 1.0                                   # event resolution, microseconds
+    for k, (s0, s1, e0, e1) in enumerate(tl):
+        assert 0.0 <= s0 <= s1 + eps and s1 <= e0 + eps and e0 <= e1 + eps, (k, tl[k])
+        if k:
+            assert tl[k - 1][3] <= e0 + eps and tl[k - 1][1] <= s0 + eps, (k, tl[k - 1], tl[k])
+        if k >= 2:
+            assert tl[k - 2][3] <= s0 + eps, (k, tl[k - 2], tl[k])
+    assert tl[-1][3] <= total_us + eps
+
+
 @pytest.mark.parametrize("variant", [capi.SWAP_MEMCPY, capi.SWAP_ZEROCOPY])
 def test_graph_timeline_follows_the_pipeline_order(variant):
     """The block timeline of a replayed inference graph obeys the ordering
@@ -614,16 +625,46 @@ def test_graph_timeline_follows_the_pipeline_order(variant):
     sw.engine.infer(sw.d_in.data_ptr(), sw.d_out.data_ptr(), s.cuda_stream)
     b.record(s)
     b.synchronize()
-    tl = sw.engine.last_graph_timeline(nb)
-    eps = 1.0                                   # event resolution, microseconds
-    for k, (s0, s1, e0, e1) in enumerate(tl):
-        assert 0.0 <= s0 <= s1 + eps and s1 <= e0 + eps and e0 <= e1 + eps, (k, tl[k])
-        if k:
-            assert tl[k - 1][3] <= e0 + eps and tl[k - 1][1] <= s0 + eps, (k, tl[k - 1], tl[k])
-        if k >= 2:
-            assert tl[k - 2][3] <= s0 + eps, (k, tl[k - 2], tl[k])
-    assert tl[-1][3] <= a.elapsed_time(b) * 1e3 + eps
+    _check_pipeline_order(sw.engine.last_graph_timeline(nb), a.elapsed_time(b) * 1e3)
     sw.engine.set_graph_timeline(False)
     got = sw.run(synth.gen.model_input(m))
     assert all(p.tobytes() == q.tobytes() for p, q in zip(got, ref))
+    sw.engine.sync()
+
+
+def test_timing_follows_an_adapted_plan():
+    """Swap timing and the graph timeline stay on across
+    swapnet_engine_adapt to a plan with more blocks: every block of the new
+    plan is timed and the timeline keeps the pipeline order."""
+    import torch
+    m = synth.arch.MODELS["resnet50"]()
+    w = synth.gen.model_weights(m)
+    d = capi.Desc(m)
+    host = capi.HostWeights(w)
+    wb = OP.weight_bytes(m)
+    p_big = capi.Plan.partition(d, int(wb * 0.8) // 256 * 256, capi.options())
+    p_small = capi.Plan.partition(d, int(wb * 0.4) // 256 * 256, capi.options())
+    nb = p_small.info()["n_blocks"]
+    assert nb > p_big.info()["n_blocks"]
+    sw = Runner(m, w, p_big, host)
+    x = synth.gen.model_input(m)
+    ref = Runner(m, w, capi.Plan.resident(d), host).run(x)
+    sw.engine.set_swap_timing(True)
+    sw.engine.set_graph_timeline(True)
+    assert sw.run(x)[0].tobytes() == ref[0].tobytes()
+    sw.engine.adapt(p_small)
+    sw.plan = p_small
+    sw.offs = p_small.output_offsets()
+    s = torch.cuda.current_stream()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(s)
+    sw.engine.infer(sw.d_in.data_ptr(), sw.d_out.data_ptr(), s.cuda_stream)
+    b.record(s)
+    b.synchronize()
+    assert sw.outputs_raw()[0].tobytes() == ref[0].tobytes()
+    us = sw.engine.last_swap_times(nb)
+    assert all(t > 0.0 for t in us)
+    _check_pipeline_order(sw.engine.last_graph_timeline(nb), a.elapsed_time(b) * 1e3)
+    sw.engine.set_graph_timeline(False)
+    sw.engine.set_swap_timing(False)
     sw.engine.sync()
