@@ -614,11 +614,15 @@ int launch_inst(const TcGemm& g, const TcPlan& pl, int* err, cudaStream_t s) {
 
 
 // Largest cluster (along the split dimension) that the device can co-schedule
-// for this kernel instance: 16, 8, 4 or 2 (cached per instance).
+// for this kernel instance: 16, 8, 4 or 2 (cached per instance and device).
 template <typename T, int BN, int AMODE>
 int max_cluster_inst() {
-  static int cached = -1;
-  if (cached >= 0) return cached;
+  static std::atomic<int> cached[64];  // 0 until known
+  const int dev = device_index();
+  if (dev >= 0) {
+    const int c = cached[dev].load(std::memory_order_relaxed);
+    if (c > 0) return c;
+  }
   auto kern = tc_gemm_kernel<T, BN, AMODE>;
   cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<BN>::kSmem);
   cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
@@ -643,17 +647,21 @@ int max_cluster_inst() {
     }
     cudaGetLastError();
   }
-  cached = best;
+  if (dev >= 0) cached[dev].store(best, std::memory_order_relaxed);
   return best;
 }
 
 // Clusters of c CTAs of the N-tile-256 instance that the device runs at
-// once (cudaOccupancyMaxActiveClusters; cached per dtype and size).
+// once (cudaOccupancyMaxActiveClusters; cached per dtype, size and device).
 template <typename T>
 int active_clusters_inst(int c) {
-  static int cached[9] = {-1, -1, -1, -1, -1, -1, -1, -1, -1};
+  static std::atomic<int> cached[64][9];  // the count + 1, 0 until known
   if (c < 1 || c > 8) return 0;
-  if (cached[c] >= 0) return cached[c];
+  const int dev = device_index();
+  if (dev >= 0) {
+    const int v = cached[dev][c].load(std::memory_order_relaxed);
+    if (v > 0) return v - 1;
+  }
   auto kern = tc_gemm_kernel<T, 256, kA2d>;
   cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<256>::kSmem);
   cudaLaunchConfig_t cfg;
@@ -673,7 +681,7 @@ int active_clusters_inst(int c) {
     cudaGetLastError();
     n = 0;
   }
-  cached[c] = n;
+  if (dev >= 0) cached[dev][c].store(n + 1, std::memory_order_relaxed);
   return n;
 }
 

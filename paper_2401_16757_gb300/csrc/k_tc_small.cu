@@ -319,12 +319,15 @@ __global__ void __launch_bounds__(kSmThreads, 4) tc_conv_small_kernel(const Smal
   }
 }
 
-// CTAs per SM for a given k-block count, per element type; computed outside
-// stream capture (tc_small_prepare), where the occupancy query is allowed.
+// CTAs per SM for a given k-block count, per element type and device (0
+// until known); computed outside stream capture (tc_small_prepare), where
+// the occupancy query is allowed, together with the kernel's attributes on
+// that device.  An unknown device index shares the last slot.
 template <typename T>
-int& small_occ(int nkb) {
-  static int occ[kSmMaxKB + 1] = {0, 0, 0, 0};
-  return occ[nkb];
+std::atomic<int>& small_occ(int nkb) {
+  static std::atomic<int> occ[65][kSmMaxKB + 1];
+  const int dev = device_index();
+  return occ[dev >= 0 ? dev : 64][nkb];
 }
 
 template <typename T>
@@ -351,7 +354,7 @@ int small_prepare_t(int nkb) {
   const int by_regs = regs_sm / std::max(1, warp_regs * (kSmThreads / 32));
   const int by_smem = smem_sm / std::max(1, small_smem_bytes(nkb) + (int)fa.sharedSizeBytes + reserved);
   const int n = std::min(std::min(by_regs, by_smem), blocks_sm);
-  small_occ<T>(nkb) = std::max(1, std::min(n, 512 / (2 * kSmBN)));  // TMEM: 128 columns per CTA
+  small_occ<T>(nkb).store(std::max(1, std::min(n, 512 / (2 * kSmBN))));  // TMEM: 128 columns per CTA
   return SWAPNET_OK;
 }
 
@@ -360,11 +363,11 @@ int launch_small(const TcSmallConv& g, int* err, cudaStream_t s) {
   auto kern = tc_conv_small_kernel<T>;
   const int nkb = (g.K + 63) / 64;
   const int smem = small_smem_bytes(nkb);
-  if (small_occ<T>(nkb) == 0) {
+  if (small_occ<T>(nkb).load() == 0) {
     const int rc = small_prepare_t<T>(nkb);
     if (rc) return rc;
   }
-  const int occ = small_occ<T>(nkb);
+  const int occ = small_occ<T>(nkb).load();
   SmallArgs a;
   std::memset(&a, 0, sizeof(a));
   a.x = g.x; a.w = g.W;

@@ -22,6 +22,16 @@ inline uint64_t device_bit() {
   }
   return 1ull << dev;
 }
+// The current device's index for per-device caches (static arrays of 64),
+// or -1 when it is unknown or beyond them (then nothing is cached).
+inline int device_index() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    cudaGetLastError();
+    return -1;
+  }
+  return dev;
+}
 inline bool attr_needed(const std::atomic<uint64_t>& done) {
   const uint64_t b = device_bit();
   return b == 0 || (done.load(std::memory_order_acquire) & b) == 0;
