@@ -616,6 +616,36 @@ def run_llm(args, rank, world, group):
     one(ep_rp, ed_rp); torch.cuda.synchronize()
     ext_rp["greedy_token_equals_resident"] = int(tok[:4].cpu().numpy().view(np.int32)[0]) == rs_tok
     ep_rp.free(); ed_rp.free()
+    # extension (not the paper's method): the packed swap variant on the same
+    # plans (bf16 tensors packed losslessly at load, unpacked into the arena
+    # by an SM kernel, so fewer bytes cross the host link)
+    opt_pk = capi.options(swap_variant=capi.SWAP_PACKED, alpha_as_per_byte=alpha, beta_ns_per_tensor=0,
+                          merge=args.merge)
+    pp_pk, pd_pk = capi.Plan.partition(dp, budget, opt_pk), capi.Plan.partition(dd, budget, opt_pk)
+    t_pk = time.perf_counter()
+    ep_pk, ed_pk = capi.Engine(pp_pk, host), capi.Engine(pd_pk, host)
+    pack_s = time.perf_counter() - t_pk
+    for e_ in (ep_pk, ed_pk):
+        e_.bind_state(state.data_ptr(), ip["state_bytes"])
+    one(ep_pk, ed_pk)
+    torch.cuda.synchronize()
+    st0 = [ep_pk.stats(), ed_pk.stats()]
+    pk_t = timed(ep_pk, ed_pk, min(args.steps, 3))
+    st1 = [ep_pk.stats(), ed_pk.stats()]
+    pk_link = sum(b["link_bytes"] - a["link_bytes"] for a, b in zip(st0, st1)) / len(pk_t)
+    pk_swapped = sum(b["bytes_swapped"] - a["bytes_swapped"] for a, b in zip(st0, st1)) / len(pk_t)
+    ext_pk = {"prefill_ms": statistics.mean(r[0] for r in pk_t),
+              "decode_ms_per_token": statistics.mean(r[1] for r in pk_t), "steps": len(pk_t),
+              "load_s_with_packing": pack_s,
+              "link_bytes_per_step": pk_link, "bytes_swapped_per_step": pk_swapped,
+              "packed_fraction": pk_link / pk_swapped if pk_swapped else None,
+              "variants": [[b["variant"] for b in ep_pk.blocks()], [b["variant"] for b in ed_pk.blocks()]]}
+    ext_pk["ms_per_step"] = ext_pk["prefill_ms"] + n_dec * ext_pk["decode_ms_per_token"]
+    ext_pk["link_gbs"] = pk_link / (ext_pk["ms_per_step"] * 1e-3) / 1e9
+    ext_pk["link_frac"] = ext_pk["link_gbs"] / link_peak
+    one(ep_pk, ed_pk); torch.cuda.synchronize()
+    ext_pk["greedy_token_equals_resident"] = int(tok[:4].cpu().numpy().view(np.int32)[0]) == rs_tok
+    ep_pk.free(); ed_pk.free()
     pre_ms = statistics.mean(r[0] for r in sw)
     dec_ms = statistics.mean(r[1] for r in sw)
     pre_d = statistics.mean(r[0] for r in di)
@@ -656,6 +686,7 @@ def run_llm(args, rank, world, group):
         "gpu_launches": launches, "clocks": clk,
         "setup_s": {"weights": t_gen, "plans": t_plan},
         "extension_resident_prefix": ext_rp,
+        "extension_packed_swap": ext_pk,
     }
     rp.free(); rd.free()
     del arena

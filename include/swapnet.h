@@ -129,7 +129,7 @@ typedef enum swapnet_swap_variant {
   SWAPNET_SWAP_AUTO = 0,     /* pick per block by measured time at load        */
   SWAPNET_SWAP_MEMCPY = 1,   /* copy engine: cudaMemcpyAsync from pinned memory */
   SWAPNET_SWAP_ZEROCOPY = 2, /* SM kernel reading mapped host memory           */
-  SWAPNET_SWAP_DIRECT = 3    /* no swap-in: the block's kernels read their
+  SWAPNET_SWAP_DIRECT = 3,   /* no swap-in: the block's kernels read their
                                 parameters in mapped host memory themselves
                                 (copy-free dispatch, Sec. 4.2.2, taken to the
                                 kernels); for blocks whose units all run SIMT
@@ -138,6 +138,21 @@ typedef enum swapnet_swap_variant {
                                 not 16-byte aligned), so copy-engine and SM
                                 reads of the host weights are not mixed.
                                 Never chosen by AUTO.                         */
+  SWAPNET_SWAP_PACKED = 4    /* an extension the paper has no counterpart
+                                for: bf16 models only.  At load each swapped
+                                bf16 tensor whose size is a multiple of 8192
+                                bytes is packed losslessly (swapnet_pack_bf16)
+                                into engine-held page-locked memory, and an SM
+                                kernel reads the packed form over the host
+                                link and unpacks it into the arena, so fewer
+                                bytes cross the link for the same arena
+                                contents.  Pieces that do not pack, and blocks
+                                with none that do, take ZEROCOPY.  Packed
+                                images are shared by the engines over the same
+                                host tensors; the host weights must not change
+                                while one of those engines exists.  Not for
+                                pageable weights or weights files (a file
+                                engine ignores it).  Never chosen by AUTO.     */
 } swapnet_swap_variant;
 
 /* Options.  Delay coefficients follow Sec. 6.1: t_in = alpha*s + beta*d,
@@ -460,7 +475,7 @@ typedef struct swapnet_engine_block {
 int swapnet_engine_blocks(const swapnet_engine* eng, swapnet_engine_block* blocks, uint32_t cap,
                           uint32_t* n);
 /* Counters of the inferences since load: kernel launches include the layer
- * kernels and the zero-copy swap kernels; memcpy_calls counts copy-engine
+ * kernels and the swap kernels (zero-copy, unpack); memcpy_calls counts copy-engine
  * transfers and bytes_swapped the bytes moved into the arena (uploads at
  * load time excluded; a block read in place, SWAPNET_SWAP_DIRECT, adds
  * nothing). */
@@ -469,6 +484,9 @@ typedef struct swapnet_engine_stats {
   uint64_t kernel_launches;
   uint64_t memcpy_calls;
   uint64_t bytes_swapped;
+  uint64_t link_bytes;   /* bytes the swaps read over the host link: the
+                            packed form for SWAPNET_SWAP_PACKED blocks, the
+                            bytes swapped for the others */
 } swapnet_engine_stats;
 int swapnet_engine_stats_get(const swapnet_engine* eng, swapnet_engine_stats* stats);
 
@@ -646,6 +664,24 @@ int swapnet_gemm_noalloc(int32_t dtype, const void* A, const void* W, const void
  * Errors: INVALID_ARG (null out or zero bytes), OOM. */
 int swapnet_host_alloc(uint64_t bytes, void** out);
 int swapnet_host_free(void* p);
+
+/* The lossless packed form of n_elems bf16 values (SWAPNET_SWAP_PACKED; an
+ * extension the paper has no counterpart for).  Each value is split into
+ * its exponent and a sign-mantissa byte; the exponent is stored as a 4-bit
+ * code into a table of the tensor's 15 most frequent exponents, with up to
+ * 4 exceptions per chunk of 4096 values listed in the chunk's header and
+ * chunks with more stored unpacked.  Layout (little-endian): 16 table bytes,
+ * then one 6160-byte record per chunk (16-byte header: [0] exception count
+ * or 0xff for an unpacked chunk, [4,12) positions as uint16 (for 0xff: the
+ * overflow index as uint32 in [4,8)), [12,16) their exponents; then 2048
+ * bytes of codes, two per byte, low nibble first; then 4096 sign-mantissa
+ * bytes (w >> 8 & 0x80) | (w & 0x7f)), then the unpacked chunks, 8192 bytes
+ * each.  A value is rebuilt as ((s & 0x80) << 8) | (x << 7) | (s & 0x7f).
+ * With dst NULL only *used_bytes (the packed size) is written; otherwise
+ * dst (dst_bytes long, any alignment) receives the packed form.  Host only,
+ * multithreaded.  Errors: INVALID_ARG (null src or used_bytes, dst too
+ * small), UNSUPPORTED (n_elems not a positive multiple of 4096). */
+int swapnet_pack_bf16(const void* src, uint64_t n_elems, void* dst, uint64_t dst_bytes, uint64_t* used_bytes);
 
 /* ------------------------------------------------------------------- misc */
 const char* swapnet_strerror(int status);

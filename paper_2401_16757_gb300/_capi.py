@@ -23,7 +23,7 @@ OP = {"linear": 1, "conv": 2, "maxpool": 3, "gap": 4, "upsample2x": 5, "concat":
 ACT = {"none": 0, "relu": 1, "leaky": 2, "swiglu": 3}
 DTYPE = {"f32": F32, "f16": F16, "bf16": BF16, "i32": I32}
 LAYER_NO_BIAS = 1
-SWAP_AUTO, SWAP_MEMCPY, SWAP_ZEROCOPY, SWAP_DIRECT = 0, 1, 2, 3
+SWAP_AUTO, SWAP_MEMCPY, SWAP_ZEROCOPY, SWAP_DIRECT, SWAP_PACKED = 0, 1, 2, 3, 4
 SRC_INPUT, SRC_NONE = -1, -2
 
 
@@ -74,7 +74,7 @@ class BlockInfo(C.Structure):
 
 class EngineStats(C.Structure):
     _fields_ = [("infer_calls", C.c_uint64), ("kernel_launches", C.c_uint64), ("memcpy_calls", C.c_uint64),
-                ("bytes_swapped", C.c_uint64)]
+                ("bytes_swapped", C.c_uint64), ("link_bytes", C.c_uint64)]
 
 
 KERNEL_KIND = {1: "tc_gemm", 2: "tc_conv", 3: "skinny_linear", 4: "direct_conv", 5: "maxpool", 6: "gap",
@@ -104,7 +104,7 @@ EXPORTS = ["swapnet_default_options", "swapnet_partition", "swapnet_plan_from_cu
            "swapnet_engine_bind_state", "swapnet_strerror", "swapnet_last_error", "swapnet_debug_fail_next", "swapnet_gemm_noalloc",
            "swapnet_weights_file_write", "swapnet_weights_file_open", "swapnet_weights_file_info",
            "swapnet_weights_file_read", "swapnet_weights_file_close", "swapnet_load_file",
-           "swapnet_debug_wait_timeout"]
+           "swapnet_debug_wait_timeout", "swapnet_pack_bf16"]
 
 _lib = None
 
@@ -147,6 +147,7 @@ def lib():
         "swapnet_engine_adapt": (C.c_int, [P, P]),
         "swapnet_host_alloc": (C.c_int, [C.c_uint64, C.POINTER(P)]),
         "swapnet_host_free": (C.c_int, [P]),
+        "swapnet_pack_bf16": (C.c_int, [P, C.c_uint64, P, C.c_uint64, C.POINTER(C.c_uint64)]),
         "swapnet_engine_bind_state": (C.c_int, [P, P, C.c_uint64]),
         "swapnet_engine_blocks": (C.c_int, [P, C.POINTER(EngineBlock), C.c_uint32, C.POINTER(C.c_uint32)]),
         "swapnet_engine_free": (None, [P]),
@@ -341,6 +342,19 @@ def calibrate(model, engine, reps=20, resident_ns=None):
     check(lib().swapnet_engine_calibrate(engine.h, int(reps), int(resident_ns or 0), t_ex, n,
                                          C.byref(alpha)), "swapnet_engine_calibrate")
     return list(t_ex), (alpha.value or None)
+
+
+def pack_bf16(words):
+    """swapnet_pack_bf16 of a uint16 array (bf16 bit patterns): the packed
+    bytes as a uint8 array."""
+    words = np.ascontiguousarray(words, dtype=np.uint16)
+    used = C.c_uint64()
+    check(lib().swapnet_pack_bf16(C.c_void_p(words.ctypes.data), words.size, None, 0, C.byref(used)),
+          "swapnet_pack_bf16")
+    out = np.empty(used.value, dtype=np.uint8)
+    check(lib().swapnet_pack_bf16(C.c_void_p(words.ctypes.data), words.size, C.c_void_p(out.ctypes.data),
+                                  out.size, C.byref(used)), "swapnet_pack_bf16")
+    return out
 
 
 def gemm_noalloc(dtype, a_ptr, w_ptr, bias_ptr, y_ptr, M, N, K, act=0, stream=0):

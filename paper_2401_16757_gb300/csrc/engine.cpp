@@ -12,10 +12,12 @@
 #include <memory>
 #include <mutex>
 #include <new>
+#include <thread>
 #include <utility>
 
 #include "internal.h"
 #include "kernels.h"
+#include "pack.h"
 
 namespace swapnet {
 
@@ -81,6 +83,41 @@ struct HostRange {
   char* dev;
 };
 
+// The packed form of one host tensor (pack.h), made at load by the first
+// engine that swaps it with SWAPNET_SWAP_PACKED and shared by every engine
+// over the same host tensor (same address and size) until the last is freed.
+struct PackedImage {
+  uint8_t* host = nullptr;       // page-locked, mapped
+  const uint8_t* dev = nullptr;  // its device alias
+  uint64_t bytes = 0, chunks = 0, overflow_off = 0;
+  uint32_t table[4] = {0, 0, 0, 0};
+  std::vector<uint32_t> raw_before;  // overflow chunks before chunk c (chunks + 1 entries)
+  int refs = 0;
+};
+
+static std::mutex g_pk_mu;
+static std::map<std::pair<uintptr_t, uint64_t>, PackedImage*> g_pk;
+
+static void release_packed(PackedImage* im) {
+  std::lock_guard<std::mutex> lk(g_pk_mu);
+  if (--im->refs > 0) return;
+  for (auto it = g_pk.begin(); it != g_pk.end(); ++it)
+    if (it->second == im) {
+      g_pk.erase(it);
+      break;
+    }
+  if (im->host) cudaFreeHost(im->host);
+  delete im;
+}
+
+// Up to 1024 unpack jobs of a block launched together (first: their index
+// in the engine's device job array).
+struct PkLaunch {
+  size_t first;
+  int njobs;
+  uint32_t chunks;
+};
+
 }  // namespace swapnet
 
 using namespace swapnet;
@@ -98,6 +135,15 @@ struct swapnet_engine {
   char* d_out_stage = nullptr;
   std::vector<HostRange> ranges;
   std::vector<const char*> tensor_dev;  // device alias per tensor
+  std::vector<const char*> tensor_host;  // the caller's pointer per tensor
+  // packed swap variant: the packed image of each swapped tensor that packs
+  // (null otherwise), and per block the unpack launches, the segments that
+  // are not packed (zero-copy kernel) and the bytes read over the host link
+  std::vector<PackedImage*> packed;
+  PkJob* d_pkjobs = nullptr;
+  std::vector<std::vector<PkLaunch>> pk_launch;
+  std::vector<std::vector<Segment>> pk_rest;
+  std::vector<uint64_t> link_bytes;
   cudaStream_t copy = nullptr;
   cudaEvent_t slot_free[2] = {nullptr, nullptr};
   cudaEvent_t ready[2] = {nullptr, nullptr};
@@ -195,6 +241,9 @@ static int release(swapnet_engine* e) {
   if (e->own_arena && e->d_arena) cudaFree(e->d_arena);
   if (e->own_ws && e->d_ws) cudaFree(e->d_ws);
   if (e->d_splitk) cudaFree(e->d_splitk);
+  if (e->d_pkjobs) cudaFree(e->d_pkjobs);
+  for (PackedImage* im : e->packed)
+    if (im) release_packed(im);
   if (e->d_in_stage) cudaFree(e->d_in_stage);
   if (e->d_out_stage) cudaFree(e->d_out_stage);
   for (const HostRange& r : e->ranges)
@@ -276,6 +325,8 @@ static int register_host(swapnet_engine* e, const void* const* hw, uint32_t nt) 
     e->ranges.push_back(hr);
   }
   e->tensor_dev.assign(nt, nullptr);
+  e->tensor_host.assign(nt, nullptr);
+  for (uint32_t t = 0; t < nt; ++t) e->tensor_host[t] = static_cast<const char*>(hw[t]);
   for (uint32_t t = 0; t < nt; ++t) {
     if (m.tensor_raw[t] == 0) continue;
     void* dptr = nullptr;
@@ -450,6 +501,8 @@ static int calibrate_file(swapnet_engine* e) {
 }
 
 static int build_segments(swapnet_engine* e) {
+  e->link_bytes.assign(e->plan.blocks.size(), 0);
+  for (size_t k = 0; k < e->plan.blocks.size(); ++k) e->link_bytes[k] = e->plan.blocks[k].bytes;
   if (e->file) return build_file_blocks(e);
   const swapnet_plan& p = e->plan;
   e->blocks.assign(p.blocks.size(), EngBlock{});
@@ -479,8 +532,152 @@ static int build_segments(swapnet_engine* e) {
   return SWAPNET_OK;
 }
 
+static bool zerocopy_ok(const EngBlock& b);
+
+// The packed image of host tensor t: the one another engine made for the
+// same host tensor, or a new one packed from the caller's buffer now.
+static int acquire_packed(swapnet_engine* e, int t) {
+  const uint64_t raw = e->plan.model.tensor_raw[t];
+  const uintptr_t key = reinterpret_cast<uintptr_t>(e->tensor_host[t]);
+  std::lock_guard<std::mutex> lk(g_pk_mu);
+  auto it = g_pk.find({key, raw});
+  if (it != g_pk.end()) {
+    ++it->second->refs;
+    e->packed[t] = it->second;
+    return SWAPNET_OK;
+  }
+  const int threads = (int)std::min(32u, std::max(1u, std::thread::hardware_concurrency()));
+  const uint16_t* src = reinterpret_cast<const uint16_t*>(e->tensor_host[t]);
+  const uint64_t n = raw / 2;
+  PackInfo info;
+  try {
+    info = pack_prepare(src, n, threads);
+  } catch (const std::bad_alloc&) {
+    SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
+  }
+  std::unique_ptr<PackedImage> im(new (std::nothrow) PackedImage());
+  if (!im) SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
+  void* h = nullptr;
+  if (cudaHostAlloc(&h, info.bytes, cudaHostAllocMapped | cudaHostAllocPortable) != cudaSuccess) {
+    cudaGetLastError();
+    SN_FAIL(SWAPNET_ERR_OOM, "page-locked allocation of packed weights failed");
+  }
+  im->host = static_cast<uint8_t*>(h);
+  pack_write(src, n, info, im->host, threads);
+  void* d = nullptr;
+  if (cudaHostGetDevicePointer(&d, h, 0) != cudaSuccess || !d) {
+    cudaGetLastError();
+    cudaFreeHost(h);
+    SN_FAIL(SWAPNET_ERR_CUDA, "device alias of packed weights");
+  }
+  im->dev = static_cast<const uint8_t*>(d);
+  im->bytes = info.bytes;
+  im->chunks = n / kPkChunk;
+  im->overflow_off = kPkHeader + im->chunks * (uint64_t)kPkRecord;
+  std::memcpy(im->table, info.exp, 16);
+  im->raw_before.assign(im->chunks + 1, 0);
+  for (uint64_t c = 0; c < im->chunks; ++c)
+    im->raw_before[c + 1] = im->raw_before[c] + (info.overflow[c] != UINT32_MAX ? 1u : 0u);
+  im->refs = 1;
+  e->packed[t] = im.get();
+  g_pk[{key, raw}] = im.release();
+  return SWAPNET_OK;
+}
+
+// Packed swap variant: every piece of a bf16 tensor that starts and ends on
+// a chunk boundary is unpacked from its packed image; the other pieces
+// (other types, ragged tensors) are copied by the zero-copy kernel.  A
+// block with no packed piece takes the zero-copy kernel (the copy engine
+// when a piece is not 16-byte aligned).
+static int build_packed(swapnet_engine* e) {
+  const swapnet_plan& p = e->plan;
+  const Model& m = p.model;
+  e->packed.resize(m.n_tensors, nullptr);
+  e->pk_launch.assign(p.blocks.size(), {});
+  e->pk_rest.assign(p.blocks.size(), {});
+  std::vector<PkJob> jobs;
+  for (size_t k = 0; k < p.blocks.size(); ++k) {
+    const Block& B = p.blocks[k];
+    EngBlock& EB = e->blocks[k];
+    if (B.slot < 0) continue;  // a resident prefix is uploaded once
+    uint64_t link = 0;
+    std::vector<PkJob> bj;
+    for (int u = B.u0; u < B.u1; ++u) {
+      const Unit& U = p.units[u];
+      if (U.host) continue;
+      for (int t = 0; t < U.nt; ++t) {
+        if (U.tlen[t] == 0) continue;
+        const int ti = U.tidx[t];
+        char* dst = e->d_arena + B.base + U.slot_off[t];
+        const bool packs = m.dtype == SWAPNET_BF16 && m.tensor_raw[ti] % kPkChunkBytes == 0 &&
+                           U.toff[t] % kPkChunkBytes == 0 && U.tlen[t] % kPkChunkBytes == 0 &&
+                           ((uintptr_t)dst & 15) == 0;
+        if (!packs) {
+          e->pk_rest[k].push_back(Segment{e->tensor_dev[ti] + U.toff[t], dst, U.tlen[t]});
+          link += U.tlen[t];
+          continue;
+        }
+        if (!e->packed[ti]) {
+          int rc = acquire_packed(e, ti);
+          if (rc) return rc;
+        }
+        const PackedImage* im = e->packed[ti];
+        PkJob j;
+        std::memset(&j, 0, sizeof(j));
+        j.base = im->dev;
+        j.dst = reinterpret_cast<uint16_t*>(dst);
+        j.overflow_off = im->overflow_off;
+        j.c0 = (uint32_t)(U.toff[t] / kPkChunkBytes);
+        j.nchunks = (uint32_t)(U.tlen[t] / kPkChunkBytes);
+        std::memcpy(j.table, im->table, 16);
+        bj.push_back(j);
+        link += (uint64_t)j.nchunks * kPkRecord +
+                (uint64_t)(im->raw_before[j.c0 + j.nchunks] - im->raw_before[j.c0]) * kPkChunkBytes;
+      }
+    }
+    if (bj.empty()) {  // nothing packs: the block is copied as it is
+      e->pk_rest[k].clear();
+      EB.variant = zerocopy_ok(EB) ? SWAPNET_SWAP_ZEROCOPY : SWAPNET_SWAP_MEMCPY;
+      continue;
+    }
+    for (const Segment& g : e->pk_rest[k])
+      if (((uintptr_t)g.src | (uintptr_t)g.dst) & 15)
+        SN_FAIL(SWAPNET_ERR_MISALIGNED, "packed swaps: an unpacked piece is not 16-byte aligned");
+    for (size_t i = 0; i < bj.size(); i += 1024) {
+      PkLaunch L{jobs.size(), (int)std::min<size_t>(1024, bj.size() - i), 0};
+      for (int q = 0; q < L.njobs; ++q) {
+        PkJob j = bj[i + q];
+        j.first = L.chunks;
+        L.chunks += j.nchunks;
+        jobs.push_back(j);
+      }
+      e->pk_launch[k].push_back(L);
+    }
+    EB.variant = SWAPNET_SWAP_PACKED;
+    e->link_bytes[k] = link;
+  }
+  if (!jobs.empty()) {
+    if (cudaMalloc(&e->d_pkjobs, jobs.size() * sizeof(PkJob)) != cudaSuccess) {
+      cudaGetLastError();
+      e->d_pkjobs = nullptr;
+      SN_FAIL(SWAPNET_ERR_OOM, "unpack job table allocation failed");
+    }
+    CU(cudaMemcpy(e->d_pkjobs, jobs.data(), jobs.size() * sizeof(PkJob), cudaMemcpyHostToDevice), "unpack jobs");
+  }
+  return SWAPNET_OK;
+}
+
 static int swap_block(swapnet_engine* e, size_t k, int variant, cudaStream_t s) {
   const EngBlock& b = e->blocks[k];
+  if (variant == SWAPNET_SWAP_PACKED) {
+    for (const PkLaunch& L : e->pk_launch[k]) {
+      int rc = launch_unpack(e->d_pkjobs + L.first, L.njobs, L.chunks, e->zc_ctas, s);
+      if (rc) return rc;
+    }
+    std::vector<ZcSeg> z;
+    for (const Segment& g : e->pk_rest[k]) z.push_back(ZcSeg{g.src, g.dst, g.bytes});
+    return launch_zerocopy(z.data(), (int)z.size(), e->zc_ctas, s);
+  }
   if (variant == SWAPNET_SWAP_ZEROCOPY) {
     std::vector<ZcSeg> z;
     z.reserve(b.segs.size());
@@ -1051,6 +1248,10 @@ static int bind_plan(swapnet_engine* e, void* d_arena_user, uint64_t arena_bytes
     if (rc) return rc;
     rc = calibrate_in_situ(e);
     if (rc) return rc;
+  } else if (!plan->resident && variant == SWAPNET_SWAP_PACKED) {
+    for (EngBlock& b : e->blocks) b.variant = SWAPNET_SWAP_ZEROCOPY;  // until build_packed says otherwise
+    rc = build_packed(e);
+    if (rc) return rc;
   } else if (!plan->resident) {
     for (size_t k = 0; k < e->blocks.size(); ++k) {
       EngBlock& b = e->blocks[k];
@@ -1092,6 +1293,10 @@ static void unbind_plan(swapnet_engine* e) {
   e->ev_swap.clear();
   e->ev_gswap.clear();
   e->ev_gexec.clear();
+  if (e->d_pkjobs) cudaFree(e->d_pkjobs);
+  e->d_pkjobs = nullptr;
+  e->pk_launch.clear();
+  e->pk_rest.clear();
   if (e->d_splitk) cudaFree(e->d_splitk);
   e->d_splitk = nullptr;
   e->splitk_bytes = e->splitk_counter_bytes = 0;
@@ -1425,6 +1630,8 @@ static uint64_t launches_per_infer(const swapnet_engine* e) {
     for (size_t k = 0; k < e->blocks.size(); ++k)
       if (e->plan.blocks[k].slot >= 0 && e->blocks[k].variant == SWAPNET_SWAP_ZEROCOPY)
         n += (e->blocks[k].segs.size() + 47) / 48;
+      else if (e->plan.blocks[k].slot >= 0 && e->blocks[k].variant == SWAPNET_SWAP_PACKED)
+        n += e->pk_launch[k].size() + (e->pk_rest[k].size() + 47) / 48;
   return n;
 }
 
@@ -1485,7 +1692,8 @@ int swapnet_infer(swapnet_engine* e, const void* din, void* dout, swapnet_stream
   for (size_t k = 0; k < e->blocks.size(); ++k) {  // every swapped block once per inference
     if (!swapped(e, k)) continue;
     for (const Segment& g : e->blocks[k].segs) e->stats.bytes_swapped += g.bytes;
-    if (e->blocks[k].variant != SWAPNET_SWAP_ZEROCOPY) e->stats.memcpy_calls += e->blocks[k].segs.size();
+    e->stats.link_bytes += e->link_bytes[k];
+    if (e->blocks[k].variant == SWAPNET_SWAP_MEMCPY) e->stats.memcpy_calls += e->blocks[k].segs.size();
   }
   return SWAPNET_OK;
 }

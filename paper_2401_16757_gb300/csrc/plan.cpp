@@ -863,14 +863,15 @@ static int search_exhaustive_eq4(swapnet_plan* p, std::vector<uint32_t>* best_cu
 static int check_options(const swapnet_options& o) {
   if (o.slots != 1 && o.slots != 2) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "slots must be 1 or 2");
   if (o.objective != 0 && o.objective != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "objective must be 0 or 1");
-  if (o.swap_variant < 0 || o.swap_variant > 3) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad swap_variant");
+  if (o.swap_variant < 0 || o.swap_variant > 4) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad swap_variant");
   if (o.zc_ctas < 0 || o.zc_ctas > 4096) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad zc_ctas");
   if (o.graphs != 0 && o.graphs != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "graphs must be 0 or 1");
   if (o.preloaded != 0 && o.preloaded != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "preloaded must be 0 or 1");
   if (o.branches != 0 && o.branches != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "branches must be 0 or 1");
   if (o.merge != 0 && o.merge != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "merge must be 0 or 1");
   if (o.pageable != 0 && o.pageable != 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "pageable must be 0 or 1");
-  if (o.pageable && (o.swap_variant == SWAPNET_SWAP_ZEROCOPY || o.swap_variant == SWAPNET_SWAP_DIRECT))
+  if (o.pageable && (o.swap_variant == SWAPNET_SWAP_ZEROCOPY || o.swap_variant == SWAPNET_SWAP_DIRECT ||
+                     o.swap_variant == SWAPNET_SWAP_PACKED))
     SN_FAIL(SWAPNET_ERR_INVALID_ARG, "pageable weights are copied by the copy engine only");
   if (o.split_cap < 0 || o.split_cap > 64) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "split_cap must be in [0, 64]");
   if (o.resident_prefix != 0 && o.resident_prefix != 1)

@@ -19,7 +19,7 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 def _declared_functions():
     src = open(os.path.join(ROOT, "include", "swapnet.h")).read()
     src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
-    return sorted(set(re.findall(r"\b(swapnet_[a-z_]+)\s*\(", src)))
+    return sorted(set(re.findall(r"\b(swapnet_[a-z0-9_]+)\s*\(", src)))
 
 
 def test_library_exports_every_declared_symbol():
@@ -175,17 +175,22 @@ def test_prefetch_partition_equals_exhaustive_oracle():
 
 
 def test_swap_variant_range():
-    """AUTO, MEMCPY, ZEROCOPY and DIRECT are the variants a plan accepts; the
-    variant changes what the engine does, not the partition."""
+    """AUTO, MEMCPY, ZEROCOPY, DIRECT and PACKED are the variants a plan
+    accepts; the variant changes what the engine does, not the partition.
+    Pageable weights take the copy engine only."""
     m = _random_model(np.random.default_rng(4), 6)
     desc = capi.Desc(m)
     budget = P.weight_bytes(m) // 256 * 256
     cuts = None
-    for v in (capi.SWAP_AUTO, capi.SWAP_MEMCPY, capi.SWAP_ZEROCOPY, capi.SWAP_DIRECT):
+    for v in (capi.SWAP_AUTO, capi.SWAP_MEMCPY, capi.SWAP_ZEROCOPY, capi.SWAP_DIRECT, capi.SWAP_PACKED):
         got = capi.Plan.partition(desc, budget, capi.options(swap_variant=v)).cuts()
         assert cuts is None or got == cuts
         cuts = got
-    for bad in (-1, 4):
+    for v in (capi.SWAP_ZEROCOPY, capi.SWAP_DIRECT, capi.SWAP_PACKED):
+        with pytest.raises(capi.SwapnetError) as ei:
+            capi.Plan.partition(desc, budget, capi.options(swap_variant=v, pageable=1))
+        assert ei.value.code == capi.ERR_INVALID_ARG
+    for bad in (-1, 5):
         with pytest.raises(capi.SwapnetError) as ei:
             capi.Plan.partition(desc, budget, capi.options(swap_variant=bad))
         assert ei.value.code == capi.ERR_INVALID_ARG

@@ -423,3 +423,50 @@ def test_llm_decode_to_the_end_of_the_cache_then_refused():
     with pytest.raises(capi.SwapnetError) as ei:
         dec.run(1, np.array([tok], dtype=np.int32))
     assert ei.value.code == capi.ERR_INVALID_ARG
+
+
+def test_llm_packed_swaps_equal_resident():
+    """The packed swap variant (an extension: the bf16 tensors packed
+    losslessly at load and unpacked into the arena by an SM kernel): a
+    prefill and decode steps equal the resident run bit for bit and the
+    oracle at the decoder bar, the blocks that hold packable tensors take the
+    unpack kernel, and fewer bytes cross the host link than are swapped."""
+    sw = Decoder(prefill_tokens=32, budget_frac=0.4, opts=dict(swap_variant=capi.SWAP_PACKED))
+    rs = Decoder(prefill_tokens=32, resident=True, host=sw.host, weights=sw.w)
+    for _, eng, info in sw.engines:
+        assert info["n_blocks"] > 1
+        assert any(b["variant"] == capi.SWAP_PACKED for b in eng.blocks())
+    ids = synth.gen.model_input(sw.mp).reshape(-1)
+    st = F.new_state()
+    ref = F.forward(sw.mp, sw.w, ids.reshape(-1, 1, 1, 1), state=st)
+    a, b = sw.run(0, ids), rs.run(0, ids)
+    assert a[0].tobytes() == b[0].tobytes() and a[1].tobytes() == b[1].tobytes()
+    _check_step(a[0], a[1], ref[0].reshape(32, -1), ref[1].reshape(-1), CHAIN_TOL)
+    tok = np.array([a[1][-1]], dtype=np.int32)
+    for _ in range(4):
+        a, b = sw.run(1, tok), rs.run(1, tok)
+        assert a[0].tobytes() == b[0].tobytes() and a[1].tobytes() == b[1].tobytes()
+        tok = np.array([a[1][0]], dtype=np.int32)
+    for _, eng, _ in sw.engines:
+        s = eng.stats()
+        assert 0 < s["link_bytes"] < 0.85 * s["bytes_swapped"], s
+
+
+def test_packed_variant_falls_back_for_other_types():
+    """An fp16 CNN under the packed variant: nothing packs, every block takes
+    the zero-copy kernel, and the result is the resident one bit for bit."""
+    import torch
+    from helpers import Runner
+    m = synth.arch.MODELS["resnet50"]()
+    w = synth.gen.model_weights(m)
+    d = capi.Desc(m)
+    host = capi.HostWeights(w)
+    plan = capi.Plan.partition(d, int(OP.weight_bytes(m) * 0.4) // 256 * 256,
+                               capi.options(swap_variant=capi.SWAP_PACKED))
+    sw = Runner(m, w, plan, host)
+    assert all(b["variant"] == capi.SWAP_ZEROCOPY for b in sw.engine.blocks())
+    x = synth.gen.model_input(m)
+    assert sw.run(x)[0].tobytes() == Runner(m, w, capi.Plan.resident(d), host).run(x)[0].tobytes()
+    s = sw.engine.stats()
+    assert s["link_bytes"] == s["bytes_swapped"] or s["link_bytes"] >= 0.99 * s["bytes_swapped"]
+    torch.cuda.synchronize()

@@ -1,0 +1,106 @@
+"""The host packer of the packed swap variant (swapnet_pack_bf16): its
+output, read by a plain NumPy decoder of the documented layout, gives back
+every input word; chunks with more exceptions than a record holds go to the
+overflow area.  No GPU needed."""
+import numpy as np
+import pytest
+
+from paper_2401_16757_gb300 import capi
+
+CHUNK, RECORD = 4096, 6160
+
+
+def _bf16(x):
+    """float32 -> bf16 bit patterns (round to nearest even)."""
+    u = np.asarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    return ((u + 0x7FFF + ((u >> 16) & 1)) >> 16).astype(np.uint16)
+
+
+def _unpack(buf, n):
+    table = buf[:16]
+    chunks = n // CHUNK
+    rec = buf[16:16 + chunks * RECORD].reshape(chunks, RECORD)
+    overflow = buf[16 + chunks * RECORD:]
+    out = np.empty((chunks, CHUNK), dtype=np.uint16)
+    raw = 0
+    for c in range(chunks):
+        h = rec[c, :16]
+        if h[0] == 0xFF:
+            r = int(h[4:8].view(np.uint32)[0])
+            out[c] = overflow[r * 2 * CHUNK:(r + 1) * 2 * CHUNK].view(np.uint16)
+            raw += 1
+            continue
+        codes = rec[c, 16:16 + CHUNK // 2]
+        code = np.empty(CHUNK, dtype=np.uint8)
+        code[0::2] = codes & 15
+        code[1::2] = codes >> 4
+        sm = rec[c, 16 + CHUNK // 2:].astype(np.uint16)
+        x = table[np.minimum(code, 14)].astype(np.uint16)
+        k = int(h[0])
+        assert k <= 4
+        pos = h[4:12].view(np.uint16)[:k]
+        assert np.array_equal(np.flatnonzero(code == 15), pos)   # every escape listed, in order
+        x[pos] = h[12:12 + k]
+        out[c] = ((sm & 0x80) << 8) | (x << 7) | (sm & 0x7F)
+    assert overflow.size == raw * 2 * CHUNK
+    return out.reshape(-1), raw
+
+
+def test_round_trip_of_llm_shaped_weights():
+    """N(0, 0.02) weights (the decoder's initialisation): exact round trip,
+    about 6160 / 8192 of the bytes."""
+    r = np.random.default_rng(7)
+    w = _bf16(r.normal(0.0, 0.02, size=CHUNK * 37))
+    buf = capi.pack_bf16(w)
+    back, raw = _unpack(buf, w.size)
+    assert np.array_equal(back, w)
+    assert buf.size == 16 + 37 * RECORD + raw * 2 * CHUNK
+    assert raw <= 2
+    assert buf.size < 0.76 * w.nbytes
+
+
+def test_escapes_up_to_four_per_chunk_then_overflow():
+    """Exponents outside the table: zeros, huge values, infinities and NaN
+    (exponent 255), negative zero.  A chunk with 4 of them keeps them in its
+    header; one with 5 is stored unpacked."""
+    r = np.random.default_rng(8)
+    # fifteen exponents (108..122), the whole table, so only the planted
+    # values escape
+    n = CHUNK * 4
+    w = ((r.integers(0, 2, n) << 15) | (r.integers(108, 123, n) << 7) | r.integers(0, 128, n)).astype(np.uint16)
+    specials = np.array([0x0000, 0x8000, 0x7F80, 0x7FC1, 0x4700], dtype=np.uint16)
+    w[[5, 700, 4095]] = specials[:3]                       # chunk 0: 3 escapes
+    w[CHUNK + np.array([0, 1, 2, 4095])] = specials[1:]    # chunk 1: 4 escapes
+    w[2 * CHUNK + np.array([9, 99, 999, 2000, 3000])] = specials   # chunk 2: 5 -> overflow
+    buf = capi.pack_bf16(w)
+    back, raw = _unpack(buf, w.size)
+    assert np.array_equal(back, w)
+    assert raw == 1
+    rec = buf[16:].reshape(-1)[:4 * RECORD].reshape(4, RECORD)
+    assert list(rec[:, 0]) == [3, 4, 0xFF, 0]
+
+
+def test_one_exponent_and_every_exponent():
+    """A constant tensor (one table entry used) and a tensor holding all 256
+    exponents (most of them escapes: chunks overflow)."""
+    ones = np.full(CHUNK * 2, 0x3F80, dtype=np.uint16)
+    back, raw = _unpack(capi.pack_bf16(ones), ones.size)
+    assert np.array_equal(back, ones) and raw == 0
+    every = (np.arange(CHUNK * 3, dtype=np.uint32) * 0x9E37 % 65536).astype(np.uint16)
+    back, raw = _unpack(capi.pack_bf16(every), every.size)
+    assert np.array_equal(back, every) and raw == 3
+
+
+def test_argument_errors():
+    w = np.zeros(CHUNK, dtype=np.uint16)
+    used = capi.C.c_uint64()
+    lib = capi.lib()
+    assert lib.swapnet_pack_bf16(capi.C.c_void_p(w.ctypes.data), CHUNK + 8, None, 0,
+                                 capi.C.byref(used)) == capi.ERR_UNSUPPORTED
+    assert lib.swapnet_pack_bf16(capi.C.c_void_p(w.ctypes.data), 0, None, 0, capi.C.byref(used)) == \
+        capi.ERR_UNSUPPORTED
+    assert lib.swapnet_pack_bf16(None, CHUNK, None, 0, capi.C.byref(used)) == capi.ERR_INVALID_ARG
+    assert lib.swapnet_pack_bf16(capi.C.c_void_p(w.ctypes.data), CHUNK, None, 0, capi.C.byref(used)) == capi.OK
+    small = np.empty(used.value - 1, dtype=np.uint8)
+    assert lib.swapnet_pack_bf16(capi.C.c_void_p(w.ctypes.data), CHUNK, capi.C.c_void_p(small.ctypes.data),
+                                 small.size, capi.C.byref(used)) == capi.ERR_INVALID_ARG
