@@ -167,7 +167,9 @@ typedef struct swapnet_options {
   uint64_t beta_ns_per_tensor;
   uint64_t gamma_as_per_flop;
   uint64_t eta_ns_per_tensor;
-  int32_t zc_ctas;               /* CTAs of the zero-copy swap kernel, 0 = default */
+  int32_t zc_ctas;               /* CTAs of the zero-copy swap kernel (and of the
+                                    unpack kernel of SWAPNET_SWAP_PACKED), 0 =
+                                    default (32; one per SM for unpacking)     */
   int32_t graphs;                /* 1 (default): each (input, output) binding of an
                                     engine is captured once as a CUDA graph and
                                     replayed; 0: launch eagerly every call      */
@@ -667,16 +669,20 @@ int swapnet_host_free(void* p);
 
 /* The lossless packed form of n_elems bf16 values (SWAPNET_SWAP_PACKED; an
  * extension the paper has no counterpart for).  Each value is split into
- * its exponent and a sign-mantissa byte; the exponent is stored as a 4-bit
- * code into a table of the tensor's 15 most frequent exponents, with up to
- * 4 exceptions per chunk of 4096 values listed in the chunk's header and
- * chunks with more stored unpacked.  Layout (little-endian): 16 table bytes,
- * then one 6160-byte record per chunk (16-byte header: [0] exception count
- * or 0xff for an unpacked chunk, [4,12) positions as uint16 (for 0xff: the
- * overflow index as uint32 in [4,8)), [12,16) their exponents; then 2048
- * bytes of codes, two per byte, low nibble first; then 4096 sign-mantissa
- * bytes (w >> 8 & 0x80) | (w & 0x7f)), then the unpacked chunks, 8192 bytes
- * each.  A value is rebuilt as ((s & 0x80) << 8) | (x << 7) | (s & 0x7f).
+ * its exponent and a sign-mantissa byte; the exponent x is stored as the
+ * 4-bit code x - x0, where x0 .. x0 + 14 (x0 <= 240) is the window of 15
+ * consecutive exponents holding most of the tensor, code 15 marking an
+ * exception; up to 4 exceptions per chunk of 4096 values are listed in the
+ * chunk's header and chunks with more are stored unpacked.  Layout
+ * (little-endian): 16 bytes (x0, then zeros); a 16-byte header per chunk
+ * ([0] exception count or 0xff for an unpacked chunk, [4,12) positions as
+ * uint16 (for 0xff: the overflow index as uint32 in [4,8)), [12,16) their
+ * exponents); zeros up to a multiple of 128 bytes; a 6144-byte body per
+ * chunk (2048 bytes of codes, two per byte, low nibble first, then 4096
+ * sign-mantissa bytes (w >> 8 & 0x80) | (w & 0x7f); zeros for an unpacked
+ * chunk); then the unpacked chunks, 8192 bytes
+ * each.  A value is rebuilt as ((s & 0x80) << 8) | (x << 7) | (s & 0x7f)
+ * with x = x0 + code, or the listed exponent for code 15.
  * With dst NULL only *used_bytes (the packed size) is written; otherwise
  * dst (dst_bytes long, any alignment) receives the packed form.  Host only,
  * multithreaded.  Errors: INVALID_ARG (null src or used_bytes, dst too

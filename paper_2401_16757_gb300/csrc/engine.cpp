@@ -89,8 +89,8 @@ struct HostRange {
 struct PackedImage {
   uint8_t* host = nullptr;       // page-locked, mapped
   const uint8_t* dev = nullptr;  // its device alias
-  uint64_t bytes = 0, chunks = 0, overflow_off = 0;
-  uint32_t table[4] = {0, 0, 0, 0};
+  uint64_t bytes = 0, chunks = 0, body_off = 0, overflow_off = 0;
+  uint32_t x0 = 0;  // exponent window start
   std::vector<uint32_t> raw_before;  // overflow chunks before chunk c (chunks + 1 entries)
   int refs = 0;
 };
@@ -573,8 +573,9 @@ static int acquire_packed(swapnet_engine* e, int t) {
   im->dev = static_cast<const uint8_t*>(d);
   im->bytes = info.bytes;
   im->chunks = n / kPkChunk;
-  im->overflow_off = kPkHeader + im->chunks * (uint64_t)kPkRecord;
-  std::memcpy(im->table, info.exp, 16);
+  im->body_off = pk_body_off(im->chunks);
+  im->overflow_off = im->body_off + im->chunks * (uint64_t)kPkBody;
+  im->x0 = info.exp[0];
   im->raw_before.assign(im->chunks + 1, 0);
   for (uint64_t c = 0; c < im->chunks; ++c)
     im->raw_before[c + 1] = im->raw_before[c] + (info.overflow[c] != UINT32_MAX ? 1u : 0u);
@@ -626,12 +627,13 @@ static int build_packed(swapnet_engine* e) {
         std::memset(&j, 0, sizeof(j));
         j.base = im->dev;
         j.dst = reinterpret_cast<uint16_t*>(dst);
+        j.body_off = im->body_off;
         j.overflow_off = im->overflow_off;
         j.c0 = (uint32_t)(U.toff[t] / kPkChunkBytes);
         j.nchunks = (uint32_t)(U.tlen[t] / kPkChunkBytes);
-        std::memcpy(j.table, im->table, 16);
+        j.x0 = im->x0;
         bj.push_back(j);
-        link += (uint64_t)j.nchunks * kPkRecord +
+        link += (uint64_t)j.nchunks * (kPkBody + kPkHeader) +
                 (uint64_t)(im->raw_before[j.c0 + j.nchunks] - im->raw_before[j.c0]) * kPkChunkBytes;
       }
     }
@@ -671,7 +673,9 @@ static int swap_block(swapnet_engine* e, size_t k, int variant, cudaStream_t s) 
   const EngBlock& b = e->blocks[k];
   if (variant == SWAPNET_SWAP_PACKED) {
     for (const PkLaunch& L : e->pk_launch[k]) {
-      int rc = launch_unpack(e->d_pkjobs + L.first, L.njobs, L.chunks, e->zc_ctas, s);
+      // one CTA per SM unless the options fix the swap kernels' CTA count
+      const int ctas = e->plan.opt.zc_ctas > 0 ? e->plan.opt.zc_ctas : e->num_sms;
+      int rc = launch_unpack(e->d_pkjobs + L.first, L.njobs, L.chunks, ctas, s);
       if (rc) return rc;
     }
     std::vector<ZcSeg> z;

@@ -1,10 +1,15 @@
 // Unpacking swap-in kernel of the packed swap variant (layout in pack.h):
-// one warp per chunk record, read straight from page-locked, mapped host
-// memory with 16-byte loads (all of a record's loads issued before any is
-// used, so one link round trip per record), decoded in registers and
-// written to the arena with 16-byte stores.  Lane l of a warp decodes
-// elements d * 1024 + 32 l .. + 32 of its chunk for d = 0..3: 16 bytes of
-// codes and 32 bytes of sign-mantissa bytes each, 64 bytes of output.
+// one warp per chunk, its header and body read straight from page-locked,
+// mapped host memory (every load issued before any is used, so one link
+// round trip per chunk; the body in whole 128-byte lines), decoded in
+// registers and written to the arena with 16-byte stores.  Lane l takes elements 512 g + 16 l .. + 16 of its
+// chunk for g = 0..7, so each warp-wide load reads one contiguous range:
+// 8 bytes of codes (256 bytes a warp) and 16 sign-mantissa bytes (512).
+// Four elements are decoded at once as byte lanes of 32-bit words: the
+// exponents are x0 + code (no carry between bytes, since x0 + 15 <= 255),
+// then the high and low bytes of the four bf16 values are assembled with
+// masks and interleaved with byte permutes.  An escaped element (code 15)
+// gets the exponent its record header lists, patched before the store.
 #include <cstring>
 
 #include "internal.h"
@@ -15,7 +20,6 @@ namespace swapnet {
 
 namespace {
 
-constexpr int kUpThreads = 512;
 constexpr int kUpMaxJobs = 1024;
 
 __device__ __forceinline__ uint4 ld_host16(const void* p) {
@@ -26,31 +30,30 @@ __device__ __forceinline__ uint4 ld_host16(const void* p) {
   return r;
 }
 
-__device__ __forceinline__ uint32_t word_of(const uint4& v, int i) {
-  return i == 0 ? v.x : i == 1 ? v.y : i == 2 ? v.z : v.w;
+__device__ __forceinline__ uint2 ld_host8(const void* p) {
+  uint2 r;
+  asm volatile("ld.global.nc.L1::no_allocate.v2.u32 {%0,%1}, [%2];" : "=r"(r.x), "=r"(r.y) : "l"(p));
+  return r;
 }
 
-// exponent of code c (< 15) from the 16 table bytes in t
-__device__ __forceinline__ uint32_t table_exp(uint32_t c, const uint4& t) {
-  const uint32_t lo = __byte_perm(t.x, t.y, c & 7u);
-  const uint32_t hi = __byte_perm(t.z, t.w, c & 7u);
-  return (c < 8u ? lo : hi) & 0xffu;
+// four 4-bit codes (16 bits, element i in bits 4i..4i+3) -> one per byte
+__device__ __forceinline__ uint32_t spread4(uint32_t sel) {
+  uint32_t t = (sel | (sel << 8)) & 0x00ff00ffu;
+  return (t | (t << 4)) & 0x0f0f0f0fu;
 }
 
-// exponent of the escaped element at position pos of the chunk (the header
-// lists k <= 4 positions in hdr.y, hdr.z and their exponents in hdr.w)
-__device__ __forceinline__ uint32_t escape_exp(uint32_t pos, uint32_t k, const uint4& hdr) {
-  uint32_t x = 0;
-#pragma unroll
-  for (uint32_t i = 0; i < (uint32_t)kPkMaxEsc; ++i) {
-    const uint32_t p = ((i < 2 ? hdr.y : hdr.z) >> ((i & 1) * 16)) & 0xffffu;
-    if (i < k && p == pos) x = (hdr.w >> (i * 8)) & 0xffu;
-  }
-  return x;
+// four elements: codes (16 bits) and sign-mantissa bytes -> two words of
+// two bf16 values each
+__device__ __forceinline__ void decode4(uint32_t sel, uint32_t sm, uint32_t x0x4, uint32_t& w0, uint32_t& w1) {
+  const uint32_t x = spread4(sel) + x0x4;  // exponents, one per byte
+  const uint32_t hi = (sm & 0x80808080u) | ((x >> 1) & 0x7f7f7f7fu);
+  const uint32_t lo = ((x << 7) & 0x80808080u) | (sm & 0x7f7f7f7fu);
+  w0 = __byte_perm(lo, hi, 0x5140);
+  w1 = __byte_perm(lo, hi, 0x7362);
 }
 
-__global__ void __launch_bounds__(kUpThreads) unpack_kernel(const PkJob* __restrict__ jobs, int njobs,
-                                                            uint32_t total) {
+__global__ void __launch_bounds__(kUnpackThreads, 1) unpack_kernel(const PkJob* __restrict__ jobs, int njobs,
+                                                                uint32_t total) {
   __shared__ uint32_t s_first[kUpMaxJobs];
   for (int j = threadIdx.x; j < njobs; j += blockDim.x) s_first[j] = jobs[j].first;
   __syncthreads();
@@ -66,16 +69,17 @@ __global__ void __launch_bounds__(kUpThreads) unpack_kernel(const PkJob* __restr
     const PkJob* J = jobs + lo;
     const uint32_t rel = g - J->first;
     const uint8_t* base = J->base;
-    const uint8_t* rec = base + kPkHeader + (uint64_t)(J->c0 + rel) * kPkRecord;
+    const uint64_t c = J->c0 + rel;
+    const uint8_t* body = base + J->body_off + c * kPkBody;
     uint4* out = reinterpret_cast<uint4*>(J->dst + (uint64_t)rel * kPkChunk);
-    const uint4 t = make_uint4(J->table[0], J->table[1], J->table[2], J->table[3]);
-    const uint4 hdr = ld_host16(rec);
-    uint4 cd[4], s0[4], s1[4];
+    const uint32_t x0x4 = J->x0 * 0x01010101u;
+    const uint4 hdr = ld_host16(base + 16 + kPkHeader * c);
+    uint2 cd[8];
+    uint4 sm[8];
 #pragma unroll
-    for (int d = 0; d < 4; ++d) {
-      cd[d] = ld_host16(rec + 16 + d * 512 + lane * 16);
-      s0[d] = ld_host16(rec + 16 + kPkChunk / 2 + d * 1024 + lane * 32);
-      s1[d] = ld_host16(rec + 16 + kPkChunk / 2 + d * 1024 + lane * 32 + 16);
+    for (int q = 0; q < 8; ++q) {
+      cd[q] = ld_host8(body + q * 256 + lane * 8);
+      sm[q] = ld_host16(body + kPkChunk / 2 + q * 512 + lane * 16);
     }
     const uint32_t k = hdr.x & 0xffu;
     if (k == (uint32_t)kPkRaw) {  // stored unpacked in the overflow area
@@ -88,20 +92,28 @@ __global__ void __launch_bounds__(kUpThreads) unpack_kernel(const PkJob* __restr
       continue;
     }
 #pragma unroll
-    for (int d = 0; d < 4; ++d) {
-      const uint32_t e0 = d * 1024 + lane * 32;  // first element of this group
-      uint32_t w[16];
+    for (int q = 0; q < 8; ++q) {
+      uint32_t w[8];  // elements 2i, 2i + 1 of this lane's 16
+      decode4(cd[q].x & 0xffffu, sm[q].x, x0x4, w[0], w[1]);
+      decode4(cd[q].x >> 16, sm[q].y, x0x4, w[2], w[3]);
+      decode4(cd[q].y & 0xffffu, sm[q].z, x0x4, w[4], w[5]);
+      decode4(cd[q].y >> 16, sm[q].w, x0x4, w[6], w[7]);
+      const uint32_t e0 = q * 512 + lane * 16;  // this lane's first element
 #pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        const uint32_t c = (word_of(cd[d], j >> 3) >> ((j & 7) * 4)) & 0xfu;
-        const uint32_t s = (word_of(j < 16 ? s0[d] : s1[d], (j & 15) >> 2) >> ((j & 3) * 8)) & 0xffu;
-        const uint32_t x = c < 15u ? table_exp(c, t) : escape_exp(e0 + j, k, hdr);
-        const uint32_t v = ((s & 0x80u) << 8) | (x << 7) | (s & 0x7fu);
-        if (j & 1) w[j >> 1] |= v << 16;
-        else w[j >> 1] = v;
+      for (uint32_t i = 0; i < (uint32_t)kPkMaxEsc; ++i) {  // k is the same for the whole warp
+        const uint32_t pos = ((i < 2 ? hdr.y : hdr.z) >> ((i & 1) * 16)) & 0xffffu;
+        if (i < k && pos - e0 < 16u) {
+          const uint32_t j = pos - e0, sh = (j & 1) * 16;
+          const uint32_t m = 0x7f80u << sh, v = ((hdr.w >> (i * 8)) & 0xffu) << (7 + sh);
+#pragma unroll
+          for (int t = 0; t < 8; ++t) {  // masks, not an indexed store: w stays in registers
+            const uint32_t mt = (j >> 1) == (uint32_t)t ? m : 0u;
+            w[t] = (w[t] & ~mt) | (v & mt);
+          }
+        }
       }
-#pragma unroll
-      for (int q = 0; q < 4; ++q) out[e0 / 8 + q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
+      out[e0 / 8] = make_uint4(w[0], w[1], w[2], w[3]);
+      out[e0 / 8 + 1] = make_uint4(w[4], w[5], w[6], w[7]);
     }
   }
 }
@@ -112,7 +124,7 @@ int launch_unpack(const PkJob* jobs, int njobs, uint32_t total, int ctas, cudaSt
   if (njobs <= 0 || total == 0) return SWAPNET_OK;
   if (njobs > kUpMaxJobs) SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "unpack: too many jobs in one launch");
   if (ctas <= 0) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "unpack: ctas must be positive");
-  unpack_kernel<<<ctas, kUpThreads, 0, s>>>(jobs, njobs, total);
+  unpack_kernel<<<ctas, kUnpackThreads, 0, s>>>(jobs, njobs, total);
   const cudaError_t err = cudaGetLastError();
   if (err != cudaSuccess) SN_FAIL(SWAPNET_ERR_CUDA, std::string("unpack launch: ") + cudaGetErrorString(err));
   return SWAPNET_OK;

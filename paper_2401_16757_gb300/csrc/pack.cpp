@@ -49,16 +49,24 @@ PackInfo pack_prepare(const uint16_t* src, uint64_t n, int threads) {
   std::array<uint64_t, 256> hist{};
   for (const auto& h : part)
     for (int x = 0; x < 256; ++x) hist[x] += h[x];
-  // the 15 most frequent exponents (ties: the smaller exponent first)
-  std::array<int, 256> order;
-  for (int x = 0; x < 256; ++x) order[x] = x;
-  std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return hist[a] > hist[b]; });
+  // the window of 15 consecutive exponents x0 .. x0 + 14 that holds the
+  // most elements (the smallest x0 among equals; x0 <= 240, so that x0 + 15
+  // still fits a byte)
+  int x0 = 0;
+  uint64_t best = 0, run = 0;
+  for (int x = 0; x < 15; ++x) run += hist[x];
+  best = run;
+  for (int b = 1; b <= 240; ++b) {
+    run += hist[b + 14] - hist[b - 1];
+    if (run > best) {
+      best = run;
+      x0 = b;
+    }
+  }
   std::memset(info.code, 15, sizeof(info.code));
   std::memset(info.exp, 0, sizeof(info.exp));
-  for (int c = 0; c < 15; ++c) {
-    info.exp[c] = (uint8_t)order[c];
-    if (hist[order[c]]) info.code[order[c]] = (uint8_t)c;
-  }
+  info.exp[0] = (uint8_t)x0;
+  for (int c = 0; c < 15; ++c) info.code[x0 + c] = (uint8_t)c;
   // chunks with more escapes than a record holds go to the overflow area
   std::vector<uint8_t> raw(chunks, 0);
   parallel_for(chunks, threads, [&](uint64_t lo, uint64_t hi) {
@@ -73,29 +81,32 @@ PackInfo pack_prepare(const uint16_t* src, uint64_t n, int threads) {
   uint32_t r = 0;
   for (uint64_t c = 0; c < chunks; ++c)
     if (raw[c]) info.overflow[c] = r++;
-  info.bytes = kPkHeader + chunks * (uint64_t)kPkRecord + r * kPkChunkBytes;
+  info.bytes = pk_body_off(chunks) + chunks * (uint64_t)kPkBody + r * kPkChunkBytes;
   return info;
 }
 
 void pack_write(const uint16_t* src, uint64_t n, const PackInfo& info, uint8_t* dst, int threads) {
   const uint64_t chunks = n / kPkChunk;
+  const uint64_t body_off = pk_body_off(chunks);
+  std::memset(dst, 0, body_off);
   std::memcpy(dst, info.exp, 16);
-  uint8_t* records = dst + kPkHeader;
-  uint8_t* overflow = records + chunks * (uint64_t)kPkRecord;
+  uint8_t* bodies = dst + body_off;
+  uint8_t* overflow = bodies + chunks * (uint64_t)kPkBody;
   parallel_for(chunks, threads, [&](uint64_t lo, uint64_t hi) {
     for (uint64_t c = lo; c < hi; ++c) {
       const uint16_t* w = src + c * kPkChunk;
-      uint8_t* rec = records + c * (uint64_t)kPkRecord;
-      std::memset(rec, 0, kPkRecord);
+      uint8_t* hdr = dst + 16 + kPkHeader * c;
+      uint8_t* body = bodies + c * (uint64_t)kPkBody;
+      std::memset(body, 0, kPkBody);
       if (info.overflow[c] != UINT32_MAX) {
         const uint32_t r = info.overflow[c];
-        rec[0] = (uint8_t)kPkRaw;
-        std::memcpy(rec + 4, &r, 4);
+        hdr[0] = (uint8_t)kPkRaw;
+        std::memcpy(hdr + 4, &r, 4);
         std::memcpy(overflow + (uint64_t)r * kPkChunkBytes, w, kPkChunkBytes);
         continue;
       }
-      uint8_t* codes = rec + 16;
-      uint8_t* sm = rec + 16 + kPkChunk / 2;
+      uint8_t* codes = body;
+      uint8_t* sm = body + kPkChunk / 2;
       int k = 0;
       for (int e = 0; e < kPkChunk; ++e) {
         const uint32_t x = exponent(w[e]);
@@ -104,12 +115,12 @@ void pack_write(const uint16_t* src, uint64_t n, const PackInfo& info, uint8_t* 
         sm[e] = (uint8_t)(((w[e] >> 8) & 0x80u) | (w[e] & 0x7fu));
         if (cd == 15) {  // at most kPkMaxEsc here (pack_prepare sent the rest to the overflow area)
           const uint16_t pos = (uint16_t)e;
-          std::memcpy(rec + 4 + 2 * k, &pos, 2);
-          rec[12 + k] = (uint8_t)x;
+          std::memcpy(hdr + 4 + 2 * k, &pos, 2);
+          hdr[12 + k] = (uint8_t)x;
           ++k;
         }
       }
-      rec[0] = (uint8_t)k;
+      hdr[0] = (uint8_t)k;
     }
   });
 }

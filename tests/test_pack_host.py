@@ -7,7 +7,7 @@ import pytest
 
 from paper_2401_16757_gb300 import capi
 
-CHUNK, RECORD = 4096, 6160
+CHUNK, BODY = 4096, 6144
 
 
 def _bf16(x):
@@ -16,26 +16,35 @@ def _bf16(x):
     return ((u + 0x7FFF + ((u >> 16) & 1)) >> 16).astype(np.uint16)
 
 
+def _body_off(chunks):
+    return (16 + 16 * chunks + 127) // 128 * 128
+
+
 def _unpack(buf, n):
-    table = buf[:16]
+    x0 = int(buf[0])
+    assert x0 <= 240 and not buf[1:16].any()
     chunks = n // CHUNK
-    rec = buf[16:16 + chunks * RECORD].reshape(chunks, RECORD)
-    overflow = buf[16 + chunks * RECORD:]
+    hdrs = buf[16:16 + 16 * chunks].reshape(chunks, 16)
+    off = _body_off(chunks)
+    assert not buf[16 + 16 * chunks:off].any()
+    bodies = buf[off:off + chunks * BODY].reshape(chunks, BODY)
+    overflow = buf[off + chunks * BODY:]
     out = np.empty((chunks, CHUNK), dtype=np.uint16)
     raw = 0
     for c in range(chunks):
-        h = rec[c, :16]
+        h = hdrs[c]
         if h[0] == 0xFF:
             r = int(h[4:8].view(np.uint32)[0])
             out[c] = overflow[r * 2 * CHUNK:(r + 1) * 2 * CHUNK].view(np.uint16)
+            assert not bodies[c].any()
             raw += 1
             continue
-        codes = rec[c, 16:16 + CHUNK // 2]
+        codes = bodies[c, :CHUNK // 2]
         code = np.empty(CHUNK, dtype=np.uint8)
         code[0::2] = codes & 15
         code[1::2] = codes >> 4
-        sm = rec[c, 16 + CHUNK // 2:].astype(np.uint16)
-        x = table[np.minimum(code, 14)].astype(np.uint16)
+        sm = bodies[c, CHUNK // 2:].astype(np.uint16)
+        x = (x0 + code).astype(np.uint16)
         k = int(h[0])
         assert k <= 4
         pos = h[4:12].view(np.uint16)[:k]
@@ -48,13 +57,13 @@ def _unpack(buf, n):
 
 def test_round_trip_of_llm_shaped_weights():
     """N(0, 0.02) weights (the decoder's initialisation): exact round trip,
-    about 6160 / 8192 of the bytes."""
+    about (6144 + 16) / 8192 of the bytes."""
     r = np.random.default_rng(7)
     w = _bf16(r.normal(0.0, 0.02, size=CHUNK * 37))
     buf = capi.pack_bf16(w)
     back, raw = _unpack(buf, w.size)
     assert np.array_equal(back, w)
-    assert buf.size == 16 + 37 * RECORD + raw * 2 * CHUNK
+    assert buf.size == _body_off(37) + 37 * BODY + raw * 2 * CHUNK
     assert raw <= 2
     assert buf.size < 0.76 * w.nbytes
 
@@ -64,7 +73,7 @@ def test_escapes_up_to_four_per_chunk_then_overflow():
     (exponent 255), negative zero.  A chunk with 4 of them keeps them in its
     header; one with 5 is stored unpacked."""
     r = np.random.default_rng(8)
-    # fifteen exponents (108..122), the whole table, so only the planted
+    # fifteen exponents (108..122), the whole window, so only the planted
     # values escape
     n = CHUNK * 4
     w = ((r.integers(0, 2, n) << 15) | (r.integers(108, 123, n) << 7) | r.integers(0, 128, n)).astype(np.uint16)
@@ -76,13 +85,12 @@ def test_escapes_up_to_four_per_chunk_then_overflow():
     back, raw = _unpack(buf, w.size)
     assert np.array_equal(back, w)
     assert raw == 1
-    rec = buf[16:].reshape(-1)[:4 * RECORD].reshape(4, RECORD)
-    assert list(rec[:, 0]) == [3, 4, 0xFF, 0]
+    assert list(buf[16:16 + 4 * 16].reshape(4, 16)[:, 0]) == [3, 4, 0xFF, 0]
 
 
 def test_one_exponent_and_every_exponent():
-    """A constant tensor (one table entry used) and a tensor holding all 256
-    exponents (most of them escapes: chunks overflow)."""
+    """A constant tensor (one exponent of the window used) and a tensor
+    holding all 256 exponents (most of them escapes: chunks overflow)."""
     ones = np.full(CHUNK * 2, 0x3F80, dtype=np.uint16)
     back, raw = _unpack(capi.pack_bf16(ones), ones.size)
     assert np.array_equal(back, ones) and raw == 0
@@ -104,3 +112,20 @@ def test_argument_errors():
     small = np.empty(used.value - 1, dtype=np.uint8)
     assert lib.swapnet_pack_bf16(capi.C.c_void_p(w.ctypes.data), CHUNK, capi.C.c_void_p(small.ctypes.data),
                                  small.size, capi.C.byref(used)) == capi.ERR_INVALID_ARG
+
+
+def test_window_at_the_ends_of_the_exponent_range():
+    """Exponents 241..255 only: the window starts at 240 (x0 + 15 must fit a
+    byte), so exponent 255 escapes; exponents 0..14: the window starts at 0."""
+    r = np.random.default_rng(9)
+    n = CHUNK * 2
+    top = ((r.integers(241, 256, n) << 7) | r.integers(0, 128, n)).astype(np.uint16)
+    buf = capi.pack_bf16(top)
+    assert buf[0] == 240
+    back, _ = _unpack(buf, n)
+    assert np.array_equal(back, top)
+    low = ((r.integers(0, 2, n) << 15) | (r.integers(0, 15, n) << 7) | r.integers(0, 128, n)).astype(np.uint16)
+    buf = capi.pack_bf16(low)
+    assert buf[0] == 0
+    back, raw = _unpack(buf, n)
+    assert np.array_equal(back, low) and raw == 0
