@@ -59,13 +59,13 @@ CONFIGS = {
 
 
 # swap variants by name (--variant); "direct" reads SIMT-only blocks in place
-VARIANTS = ("auto", "memcpy", "zerocopy", "direct")
+VARIANTS = ("auto", "memcpy", "zerocopy", "direct", "packed")
 
 
 def variant_code(name):
     from paper_2401_16757_gb300 import capi
     return {"auto": capi.SWAP_AUTO, "memcpy": capi.SWAP_MEMCPY, "zerocopy": capi.SWAP_ZEROCOPY,
-            "direct": capi.SWAP_DIRECT}[name]
+            "direct": capi.SWAP_DIRECT, "packed": capi.SWAP_PACKED}[name]
 
 # DRAM traffic per launch of a kernel family, from ncu (dram__bytes_read.sum
 # + dram__bytes_write.sum averaged over the launches of one swapped step of
