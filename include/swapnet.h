@@ -686,7 +686,8 @@ int swapnet_host_free(void* p);
  * With dst NULL only *used_bytes (the packed size) is written; otherwise
  * dst (dst_bytes long, any alignment) receives the packed form.  Host only,
  * multithreaded.  Errors: INVALID_ARG (null src or used_bytes, dst too
- * small), UNSUPPORTED (n_elems not a positive multiple of 4096). */
+ * small), UNSUPPORTED (n_elems not a positive multiple of 4096), OOM (host
+ * memory or threads). */
 int swapnet_pack_bf16(const void* src, uint64_t n_elems, void* dst, uint64_t dst_bytes, uint64_t* used_bytes);
 
 /* ------------------------------------------------------------------- misc */

@@ -552,8 +552,8 @@ static int acquire_packed(swapnet_engine* e, int t) {
   PackInfo info;
   try {
     info = pack_prepare(src, n, threads);
-  } catch (const std::bad_alloc&) {
-    SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
+  } catch (...) {  // allocation or thread creation
+    SN_FAIL(SWAPNET_ERR_OOM, "packing: host resources exhausted");
   }
   std::unique_ptr<PackedImage> im(new (std::nothrow) PackedImage());
   if (!im) SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
@@ -563,7 +563,12 @@ static int acquire_packed(swapnet_engine* e, int t) {
     SN_FAIL(SWAPNET_ERR_OOM, "page-locked allocation of packed weights failed");
   }
   im->host = static_cast<uint8_t*>(h);
-  pack_write(src, n, info, im->host, threads);
+  try {
+    pack_write(src, n, info, im->host, threads);
+  } catch (...) {
+    cudaFreeHost(h);
+    SN_FAIL(SWAPNET_ERR_OOM, "packing: host resources exhausted");
+  }
   void* d = nullptr;
   if (cudaHostGetDevicePointer(&d, h, 0) != cudaSuccess || !d) {
     cudaGetLastError();

@@ -133,10 +133,14 @@ extern "C" int swapnet_pack_bf16(const void* src, uint64_t n_elems, void* dst, u
   if (n_elems == 0 || n_elems % swapnet::kPkChunk)
     SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "packing: the element count must be a positive multiple of 4096");
   const int threads = (int)std::min(32u, std::max(1u, std::thread::hardware_concurrency()));
-  const swapnet::PackInfo info = swapnet::pack_prepare(static_cast<const uint16_t*>(src), n_elems, threads);
-  *used_bytes = info.bytes;
-  if (!dst) return SWAPNET_OK;
-  if (dst_bytes < info.bytes) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "packing: destination too small");
-  swapnet::pack_write(static_cast<const uint16_t*>(src), n_elems, info, static_cast<uint8_t*>(dst), threads);
+  try {
+    const swapnet::PackInfo info = swapnet::pack_prepare(static_cast<const uint16_t*>(src), n_elems, threads);
+    *used_bytes = info.bytes;
+    if (!dst) return SWAPNET_OK;
+    if (dst_bytes < info.bytes) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "packing: destination too small");
+    swapnet::pack_write(static_cast<const uint16_t*>(src), n_elems, info, static_cast<uint8_t*>(dst), threads);
+  } catch (...) {  // allocation or thread creation
+    SN_FAIL(SWAPNET_ERR_OOM, "packing: host resources exhausted");
+  }
   return SWAPNET_OK;
 }
