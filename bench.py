@@ -645,7 +645,27 @@ def run_llm(args, rank, world, group):
     ext_pk["link_frac"] = ext_pk["link_gbs"] / link_peak
     one(ep_pk, ed_pk); torch.cuda.synchronize()
     ext_pk["greedy_token_equals_resident"] = int(tok[:4].cpu().numpy().view(np.int32)[0]) == rs_tok
+    # both extensions together: a resident prefix, the rest swapped packed
+    # (the packed images are shared with the engines above)
+    opt_pp = capi.options(swap_variant=capi.SWAP_PACKED, alpha_as_per_byte=alpha, beta_ns_per_tensor=0,
+                          resident_prefix=1, merge=args.merge)
+    ep_pp, ed_pp = capi.Engine(capi.Plan.partition(dp, budget, opt_pp), host), \
+        capi.Engine(capi.Plan.partition(dd, budget, opt_pp), host)
     ep_pk.free(); ed_pk.free()
+    for e_ in (ep_pp, ed_pp):
+        e_.bind_state(state.data_ptr(), ip["state_bytes"])
+    one(ep_pp, ed_pp)
+    torch.cuda.synchronize()
+    pp_t = timed(ep_pp, ed_pp, min(args.steps, 3))
+    ext_pk["with_resident_prefix"] = {"prefill_ms": statistics.mean(r[0] for r in pp_t),
+                                      "decode_ms_per_token": statistics.mean(r[1] for r in pp_t),
+                                      "steps": len(pp_t)}
+    ext_pk["with_resident_prefix"]["ms_per_step"] = (ext_pk["with_resident_prefix"]["prefill_ms"] +
+                                                     n_dec * ext_pk["with_resident_prefix"]["decode_ms_per_token"])
+    one(ep_pp, ed_pp); torch.cuda.synchronize()
+    ext_pk["with_resident_prefix"]["greedy_token_equals_resident"] = \
+        int(tok[:4].cpu().numpy().view(np.int32)[0]) == rs_tok
+    ep_pp.free(); ed_pp.free()
     pre_ms = statistics.mean(r[0] for r in sw)
     dec_ms = statistics.mean(r[1] for r in sw)
     pre_d = statistics.mean(r[0] for r in di)

@@ -425,13 +425,18 @@ def test_llm_decode_to_the_end_of_the_cache_then_refused():
     assert ei.value.code == capi.ERR_INVALID_ARG
 
 
-def test_llm_packed_swaps_equal_resident():
+@pytest.mark.parametrize("prefix", [0, 1])
+def test_llm_packed_swaps_equal_resident(prefix):
     """The packed swap variant (an extension: the bf16 tensors packed
-    losslessly at load and unpacked into the arena by an SM kernel): a
-    prefill and decode steps equal the resident run bit for bit and the
-    oracle at the decoder bar, the blocks that hold packable tensors take the
-    unpack kernel, and fewer bytes cross the host link than are swapped."""
-    sw = Decoder(prefill_tokens=32, budget_frac=0.4, opts=dict(swap_variant=capi.SWAP_PACKED))
+    losslessly at load and unpacked into the arena by an SM kernel), alone
+    and with a resident prefix: a prefill and decode steps equal the
+    resident run bit for bit and the oracle at the decoder bar, the blocks
+    that hold packable tensors take the unpack kernel, and fewer bytes cross
+    the host link than are swapped."""
+    sw = Decoder(prefill_tokens=32, budget_frac=0.6 if prefix else 0.4,
+                 opts=dict(swap_variant=capi.SWAP_PACKED, resident_prefix=prefix))
+    if prefix:
+        assert all(info["prefix_units"] > 0 for _, _, info in sw.engines)
     rs = Decoder(prefill_tokens=32, resident=True, host=sw.host, weights=sw.w)
     for _, eng, info in sw.engines:
         assert info["n_blocks"] > 1
