@@ -11,7 +11,8 @@
  *
  * Conventions for every call:
  *   - Status: int, SWAPNET_OK (0) on success, a negative swapnet_status
- *     otherwise.  No C++ exception crosses this boundary.  Output handles
+ *     otherwise.  No C++ exception crosses this boundary (a failed host
+ *     allocation is SWAPNET_ERR_OOM, any other one SWAPNET_ERR_INTERNAL).  Output handles
  *     and output arrays are written only on success.  swapnet_last_error()
  *     returns a message for the calling thread's most recent failure.
  *   - Ownership: plans and engines are opaque, library-owned and freed with
@@ -43,7 +44,9 @@ typedef enum swapnet_status {
   SWAPNET_ERR_TIMEOUT = -5,     /* a bounded device-side wait gave up      */
   SWAPNET_ERR_MISALIGNED = -6,  /* a pointer or size breaks an alignment rule */
   SWAPNET_ERR_UNSUPPORTED = -7, /* shape/dtype combination not implemented */
-  SWAPNET_ERR_IO = -8           /* a weights-file read or write failed      */
+  SWAPNET_ERR_IO = -8,          /* a weights-file read or write failed      */
+  SWAPNET_ERR_INTERNAL = -9     /* an unexpected host-side exception, caught
+                                   before it could cross the C ABI          */
 } swapnet_status;
 
 /* ------------------------------------------------------------ descriptors */

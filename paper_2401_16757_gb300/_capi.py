@@ -14,8 +14,8 @@ import numpy as np
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libswapnet.so")
 
-OK, ERR_INVALID_ARG, ERR_INFEASIBLE, ERR_OOM, ERR_CUDA, ERR_TIMEOUT, ERR_MISALIGNED, ERR_UNSUPPORTED, ERR_IO = \
-    0, -1, -2, -3, -4, -5, -6, -7, -8
+OK, ERR_INVALID_ARG, ERR_INFEASIBLE, ERR_OOM, ERR_CUDA, ERR_TIMEOUT, ERR_MISALIGNED, ERR_UNSUPPORTED, ERR_IO, \
+    ERR_INTERNAL = 0, -1, -2, -3, -4, -5, -6, -7, -8, -9
 F32, F16, BF16 = 0, 1, 2
 I32 = 3
 OP = {"linear": 1, "conv": 2, "maxpool": 3, "gap": 4, "upsample2x": 5, "concat": 6, "embed": 7, "rmsnorm": 8,

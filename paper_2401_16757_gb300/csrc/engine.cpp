@@ -1383,54 +1383,60 @@ extern "C" {
 
 int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint32_t n_tensors, void* d_arena,
                  uint64_t arena_bytes, void* d_workspace, uint64_t workspace_bytes, swapnet_engine** out) {
-  if (!plan || !out || (n_tensors && !host_weights)) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
-  return swapnet::load_engine(plan, host_weights, n_tensors, nullptr, d_arena, arena_bytes, d_workspace,
-                              workspace_bytes, out);
+  return swapnet::guard_abi([&]() -> int {
+    if (!plan || !out || (n_tensors && !host_weights)) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+    return swapnet::load_engine(plan, host_weights, n_tensors, nullptr, d_arena, arena_bytes, d_workspace,
+                                workspace_bytes, out);
+  });
 }
 
 int swapnet_load_file(const swapnet_plan* plan, swapnet_weights_file* file, void* d_arena, uint64_t arena_bytes,
                       void* d_workspace, uint64_t workspace_bytes, swapnet_engine** out) {
-  if (!plan || !file || !out) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
-  return swapnet::load_engine(plan, nullptr, file->n, file, d_arena, arena_bytes, d_workspace, workspace_bytes,
-                              out);
+  return swapnet::guard_abi([&]() -> int {
+    if (!plan || !file || !out) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+    return swapnet::load_engine(plan, nullptr, file->n, file, d_arena, arena_bytes, d_workspace, workspace_bytes,
+                                out);
+  });
 }
 
 int swapnet_engine_adapt(swapnet_engine* e, const swapnet_plan* plan) {
-  if (!e || !plan) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
-  const Model& a = e->plan.model;
-  const Model& b = plan->model;
-  bool same = a.L.size() == b.L.size() && a.n_tensors == b.n_tensors && a.dtype == b.dtype &&
-              a.weight_bytes == b.weight_bytes && a.in_bytes == b.in_bytes && a.ws_bytes == b.ws_bytes;
-  for (size_t i = 0; same && i < a.L.size(); ++i)
-    same = std::memcmp(&a.L[i].d, &b.L[i].d, sizeof(swapnet_layer)) == 0 ||
-           (a.L[i].d.op == b.L[i].d.op && a.L[i].d.cin == b.L[i].d.cin && a.L[i].d.cout == b.L[i].d.cout &&
-            a.L[i].tbytes[0] == b.L[i].tbytes[0] && a.L[i].tbytes[1] == b.L[i].tbytes[1]);
-  if (!same) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "the plan is for a different model");
-  if (plan->resident != e->plan.resident) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "cannot switch between resident and swapped plans");
-  if (!e->file && plan->opt.pageable != e->plan.opt.pageable)
-    SN_FAIL(SWAPNET_ERR_INVALID_ARG, "cannot switch between pageable and page-locked host weights");
-  CU(cudaSetDevice(e->device), "cudaSetDevice");
-  CU(cudaStreamSynchronize(e->copy), "drain copies");
-  if (e->side) CU(cudaStreamSynchronize(e->side), "drain side stream");
-  CU(cudaDeviceSynchronize(), "drain inferences");
-  swapnet::unbind_plan(e);
-  try {
-    e->plan = *plan;
-  } catch (const std::bad_alloc&) {
-    SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
-  }
-  // per-unit and per-block events were sized for the old plan: they are
-  // made again for the new one after binding it (whose swap-variant
-  // calibration captures inferences without them)
-  const bool prof = e->profiling, st = e->swap_timing, tl = e->timeline;
-  e->profiling = e->swap_timing = e->timeline = false;
-  // an engine given a caller arena keeps it (the new plan must fit it)
-  int rc = swapnet::bind_plan(e, e->own_arena ? nullptr : e->d_arena, e->own_arena ? 0 : e->arena_bytes, false);
-  if (rc) return rc;
-  if (prof) rc = swapnet_engine_set_profiling(e, 1);
-  if (!rc && st) rc = swapnet_engine_set_swap_timing(e, 1);
-  if (!rc && tl) rc = swapnet_engine_set_graph_timeline(e, 1);
-  return rc;
+  return swapnet::guard_abi([&]() -> int {
+    if (!e || !plan) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+    const Model& a = e->plan.model;
+    const Model& b = plan->model;
+    bool same = a.L.size() == b.L.size() && a.n_tensors == b.n_tensors && a.dtype == b.dtype &&
+                a.weight_bytes == b.weight_bytes && a.in_bytes == b.in_bytes && a.ws_bytes == b.ws_bytes;
+    for (size_t i = 0; same && i < a.L.size(); ++i)
+      same = std::memcmp(&a.L[i].d, &b.L[i].d, sizeof(swapnet_layer)) == 0 ||
+             (a.L[i].d.op == b.L[i].d.op && a.L[i].d.cin == b.L[i].d.cin && a.L[i].d.cout == b.L[i].d.cout &&
+              a.L[i].tbytes[0] == b.L[i].tbytes[0] && a.L[i].tbytes[1] == b.L[i].tbytes[1]);
+    if (!same) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "the plan is for a different model");
+    if (plan->resident != e->plan.resident) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "cannot switch between resident and swapped plans");
+    if (!e->file && plan->opt.pageable != e->plan.opt.pageable)
+      SN_FAIL(SWAPNET_ERR_INVALID_ARG, "cannot switch between pageable and page-locked host weights");
+    CU(cudaSetDevice(e->device), "cudaSetDevice");
+    CU(cudaStreamSynchronize(e->copy), "drain copies");
+    if (e->side) CU(cudaStreamSynchronize(e->side), "drain side stream");
+    CU(cudaDeviceSynchronize(), "drain inferences");
+    swapnet::unbind_plan(e);
+    try {
+      e->plan = *plan;
+    } catch (const std::bad_alloc&) {
+      SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
+    }
+    // per-unit and per-block events were sized for the old plan: they are
+    // made again for the new one after binding it (whose swap-variant
+    // calibration captures inferences without them)
+    const bool prof = e->profiling, st = e->swap_timing, tl = e->timeline;
+    e->profiling = e->swap_timing = e->timeline = false;
+    // an engine given a caller arena keeps it (the new plan must fit it)
+    int rc = swapnet::bind_plan(e, e->own_arena ? nullptr : e->d_arena, e->own_arena ? 0 : e->arena_bytes, false);
+    if (rc) return rc;
+    if (prof) rc = swapnet_engine_set_profiling(e, 1);
+    if (!rc && st) rc = swapnet_engine_set_swap_timing(e, 1);
+    if (!rc && tl) rc = swapnet_engine_set_graph_timeline(e, 1);
+    return rc;
+  });
 }
 
 }  // extern "C"
@@ -1673,384 +1679,424 @@ static int capture(swapnet_engine* e, const void* din, void* dout, cudaGraphExec
 extern "C" {
 
 int swapnet_infer(swapnet_engine* e, const void* din, void* dout, swapnet_stream stream) {
-  if (!e || !din || !dout) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
-  if (((uintptr_t)din | (uintptr_t)dout) & 15) SN_FAIL(SWAPNET_ERR_MISALIGNED, "input/output must be 16-byte aligned");
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  CU(cudaSetDevice(e->device), "cudaSetDevice");
-  // event timing needs eager launches; stream capture takes no copy from pageable memory
-  if (e->plan.opt.graphs && !e->profiling && !(e->plan.opt.pageable && !e->file)) {
-    const auto key = std::make_pair(std::make_pair(din, dout), (e->swap_timing ? 1 : 0) | (e->timeline ? 2 : 0));
-    auto it = e->graphs.find(key);
-    if (it == e->graphs.end()) {
-      if (e->graphs.size() >= 8) {
-        for (auto& kv : e->graphs) cudaGraphExecDestroy(kv.second);
-        e->graphs.clear();
+  return swapnet::guard_abi([&]() -> int {
+    if (!e || !din || !dout) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+    if (((uintptr_t)din | (uintptr_t)dout) & 15) SN_FAIL(SWAPNET_ERR_MISALIGNED, "input/output must be 16-byte aligned");
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    CU(cudaSetDevice(e->device), "cudaSetDevice");
+    // event timing needs eager launches; stream capture takes no copy from pageable memory
+    if (e->plan.opt.graphs && !e->profiling && !(e->plan.opt.pageable && !e->file)) {
+      const auto key = std::make_pair(std::make_pair(din, dout), (e->swap_timing ? 1 : 0) | (e->timeline ? 2 : 0));
+      auto it = e->graphs.find(key);
+      if (it == e->graphs.end()) {
+        if (e->graphs.size() >= 8) {
+          for (auto& kv : e->graphs) cudaGraphExecDestroy(kv.second);
+          e->graphs.clear();
+        }
+        cudaGraphExec_t ge = nullptr;
+        int rc = capture(e, din, dout, &ge);
+        if (rc) return rc;
+        it = e->graphs.emplace(key, ge).first;
       }
-      cudaGraphExec_t ge = nullptr;
-      int rc = capture(e, din, dout, &ge);
+      CU(cudaGraphLaunch(it->second, s), "graph launch");
+    } else {
+      int rc = enqueue(e, din, dout, s);
       if (rc) return rc;
-      it = e->graphs.emplace(key, ge).first;
     }
-    CU(cudaGraphLaunch(it->second, s), "graph launch");
-  } else {
-    int rc = enqueue(e, din, dout, s);
-    if (rc) return rc;
-  }
-  e->stats.kernel_launches += launches_per_infer(e);
-  e->stats.infer_calls += 1;
-  for (size_t k = 0; k < e->blocks.size(); ++k) {  // every swapped block once per inference
-    if (!swapped(e, k)) continue;
-    for (const Segment& g : e->blocks[k].segs) e->stats.bytes_swapped += g.bytes;
-    e->stats.link_bytes += e->link_bytes[k];
-    if (e->blocks[k].variant == SWAPNET_SWAP_MEMCPY) e->stats.memcpy_calls += e->blocks[k].segs.size();
-  }
-  return SWAPNET_OK;
+    e->stats.kernel_launches += launches_per_infer(e);
+    e->stats.infer_calls += 1;
+    for (size_t k = 0; k < e->blocks.size(); ++k) {  // every swapped block once per inference
+      if (!swapped(e, k)) continue;
+      for (const Segment& g : e->blocks[k].segs) e->stats.bytes_swapped += g.bytes;
+      e->stats.link_bytes += e->link_bytes[k];
+      if (e->blocks[k].variant == SWAPNET_SWAP_MEMCPY) e->stats.memcpy_calls += e->blocks[k].segs.size();
+    }
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_infer_host(swapnet_engine* e, const void* hin, void* hout, swapnet_stream stream) {
-  if (!e || !hin || !hout) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  CU(cudaSetDevice(e->device), "cudaSetDevice");
-  const Model& m = e->plan.model;
-  if (!e->d_in_stage) {
-    if (cudaMalloc(&e->d_in_stage, align_up(m.in_bytes)) != cudaSuccess ||
-        cudaMalloc(&e->d_out_stage, align_up(m.out_bytes)) != cudaSuccess) {
-      cudaGetLastError();
-      SN_FAIL(SWAPNET_ERR_OOM, "staging allocation failed");
+  return swapnet::guard_abi([&]() -> int {
+    if (!e || !hin || !hout) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    CU(cudaSetDevice(e->device), "cudaSetDevice");
+    const Model& m = e->plan.model;
+    if (!e->d_in_stage) {
+      if (cudaMalloc(&e->d_in_stage, align_up(m.in_bytes)) != cudaSuccess ||
+          cudaMalloc(&e->d_out_stage, align_up(m.out_bytes)) != cudaSuccess) {
+        cudaGetLastError();
+        SN_FAIL(SWAPNET_ERR_OOM, "staging allocation failed");
+      }
     }
-  }
-  CU(cudaMemcpyAsync(e->d_in_stage, hin, m.in_bytes, cudaMemcpyHostToDevice, s), "input copy");
-  int rc = swapnet_infer(e, e->d_in_stage, e->d_out_stage, stream);
-  if (rc) return rc;
-  CU(cudaMemcpyAsync(hout, e->d_out_stage, m.out_bytes, cudaMemcpyDeviceToHost, s), "output copy");
-  return SWAPNET_OK;
+    CU(cudaMemcpyAsync(e->d_in_stage, hin, m.in_bytes, cudaMemcpyHostToDevice, s), "input copy");
+    int rc = swapnet_infer(e, e->d_in_stage, e->d_out_stage, stream);
+    if (rc) return rc;
+    CU(cudaMemcpyAsync(hout, e->d_out_stage, m.out_bytes, cudaMemcpyDeviceToHost, s), "output copy");
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_engine_sync(swapnet_engine* e) {
-  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
-  CU(cudaSetDevice(e->device), "cudaSetDevice");
-  if (e->rd) CU(cudaStreamSynchronize(e->rd), "read stream");
-  CU(cudaStreamSynchronize(e->copy), "copy stream");
-  CU(cudaDeviceSynchronize(), "device synchronize");
-  if (const int io = e->io_errno.exchange(0))
-    SN_FAIL(SWAPNET_ERR_IO, std::string("weights file read during an inference: ") + std::strerror(io));
-  int w = 0;
-  CU(cudaMemcpy(&w, e->err_word, sizeof(int), cudaMemcpyDeviceToHost), "error word");
-  if (w) {
-    const int zero = 0;
-    cudaMemcpy(e->err_word, &zero, sizeof(int), cudaMemcpyHostToDevice);
-    if (e->d_splitk) cudaMemset(e->d_splitk, 0, e->splitk_counter_bytes);  // an aborted kernel may leave counts
-    if (w == 2) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "a token id or a cache position was out of range");
-    SN_FAIL(SWAPNET_ERR_TIMEOUT, "a device-side wait gave up");
-  }
-  return SWAPNET_OK;
+  return swapnet::guard_abi([&]() -> int {
+    if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+    CU(cudaSetDevice(e->device), "cudaSetDevice");
+    if (e->rd) CU(cudaStreamSynchronize(e->rd), "read stream");
+    CU(cudaStreamSynchronize(e->copy), "copy stream");
+    CU(cudaDeviceSynchronize(), "device synchronize");
+    if (const int io = e->io_errno.exchange(0))
+      SN_FAIL(SWAPNET_ERR_IO, std::string("weights file read during an inference: ") + std::strerror(io));
+    int w = 0;
+    CU(cudaMemcpy(&w, e->err_word, sizeof(int), cudaMemcpyDeviceToHost), "error word");
+    if (w) {
+      const int zero = 0;
+      cudaMemcpy(e->err_word, &zero, sizeof(int), cudaMemcpyHostToDevice);
+      if (e->d_splitk) cudaMemset(e->d_splitk, 0, e->splitk_counter_bytes);  // an aborted kernel may leave counts
+      if (w == 2) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "a token id or a cache position was out of range");
+      SN_FAIL(SWAPNET_ERR_TIMEOUT, "a device-side wait gave up");
+    }
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_engine_blocks(const swapnet_engine* e, swapnet_engine_block* b, uint32_t cap, uint32_t* n) {
-  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
-  if (n) *n = (uint32_t)e->blocks.size();
-  for (uint32_t i = 0; b && i < cap && i < e->blocks.size(); ++i) {
-    const EngBlock& B = e->blocks[i];
-    b[i] = swapnet_engine_block{B.variant, (int32_t)B.segs.size(), B.memcpy_us, B.zerocopy_us};
-  }
-  return SWAPNET_OK;
+  return swapnet::guard_abi([&]() -> int {
+    if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+    if (n) *n = (uint32_t)e->blocks.size();
+    for (uint32_t i = 0; b && i < cap && i < e->blocks.size(); ++i) {
+      const EngBlock& B = e->blocks[i];
+      b[i] = swapnet_engine_block{B.variant, (int32_t)B.segs.size(), B.memcpy_us, B.zerocopy_us};
+    }
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_engine_measure_units(swapnet_engine* e, int32_t reps, float* unit_us, uint32_t n_units) {
-  if (!e || !unit_us || reps < 1 || reps > 10000) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad argument");
-  CU(cudaSetDevice(e->device), "cudaSetDevice");
-  const Model& m = e->plan.model;
-  if (!e->d_in_stage) {
-    if (cudaMalloc(&e->d_in_stage, align_up(m.in_bytes)) != cudaSuccess ||
-        cudaMalloc(&e->d_out_stage, align_up(m.out_bytes)) != cudaSuccess) {
-      cudaGetLastError();
-      SN_FAIL(SWAPNET_ERR_OOM, "staging allocation failed");
+  return swapnet::guard_abi([&]() -> int {
+    if (!e || !unit_us || reps < 1 || reps > 10000) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad argument");
+    CU(cudaSetDevice(e->device), "cudaSetDevice");
+    const Model& m = e->plan.model;
+    if (!e->d_in_stage) {
+      if (cudaMalloc(&e->d_in_stage, align_up(m.in_bytes)) != cudaSuccess ||
+          cudaMalloc(&e->d_out_stage, align_up(m.out_bytes)) != cudaSuccess) {
+        cudaGetLastError();
+        SN_FAIL(SWAPNET_ERR_OOM, "staging allocation failed");
+      }
+      CU(cudaMemset(e->d_in_stage, 0, align_up(m.in_bytes)), "clear staging");
     }
-    CU(cudaMemset(e->d_in_stage, 0, align_up(m.in_bytes)), "clear staging");
-  }
-  cudaEvent_t a, b;
-  CU(cudaEventCreate(&a), "event");
-  CU(cudaEventCreate(&b), "event");
-  int rc = SWAPNET_OK;
-  const bool prof = e->profiling;
-  e->profiling = false;
-  for (uint32_t u = 0; u < n_units && u < e->plan.units.size() && rc == SWAPNET_OK; ++u) {
-    cudaGraph_t g = nullptr;
-    cudaGraphExec_t ge = nullptr;
-    if (cudaStreamBeginCapture(e->cap, cudaStreamCaptureModeThreadLocal) != cudaSuccess) { rc = SWAPNET_ERR_CUDA; break; }
-    for (int r = 0; r < reps && rc == SWAPNET_OK; ++r) rc = run_unit(e, (int)u, e->d_in_stage, e->d_out_stage, e->cap);
-    const cudaError_t ce = cudaStreamEndCapture(e->cap, &g);
-    if (rc || ce != cudaSuccess || cudaGraphInstantiate(&ge, g, 0) != cudaSuccess) {
-      if (g) cudaGraphDestroy(g);
-      cudaGetLastError();
-      rc = rc ? rc : SWAPNET_ERR_CUDA;
-      break;
+    cudaEvent_t a, b;
+    CU(cudaEventCreate(&a), "event");
+    CU(cudaEventCreate(&b), "event");
+    int rc = SWAPNET_OK;
+    const bool prof = e->profiling;
+    e->profiling = false;
+    for (uint32_t u = 0; u < n_units && u < e->plan.units.size() && rc == SWAPNET_OK; ++u) {
+      cudaGraph_t g = nullptr;
+      cudaGraphExec_t ge = nullptr;
+      if (cudaStreamBeginCapture(e->cap, cudaStreamCaptureModeThreadLocal) != cudaSuccess) { rc = SWAPNET_ERR_CUDA; break; }
+      for (int r = 0; r < reps && rc == SWAPNET_OK; ++r) rc = run_unit(e, (int)u, e->d_in_stage, e->d_out_stage, e->cap);
+      const cudaError_t ce = cudaStreamEndCapture(e->cap, &g);
+      if (rc || ce != cudaSuccess || cudaGraphInstantiate(&ge, g, 0) != cudaSuccess) {
+        if (g) cudaGraphDestroy(g);
+        cudaGetLastError();
+        rc = rc ? rc : SWAPNET_ERR_CUDA;
+        break;
+      }
+      cudaGraphDestroy(g);
+      float best = 1e30f;
+      for (int t = 0; t < 3; ++t) {
+        cudaEventRecord(a, e->cap);
+        cudaGraphLaunch(ge, e->cap);
+        cudaEventRecord(b, e->cap);
+        if (cudaEventSynchronize(b) != cudaSuccess) { rc = SWAPNET_ERR_CUDA; break; }
+        float ms = 0.f;
+        cudaEventElapsedTime(&ms, a, b);
+        if (t > 0) best = std::min(best, ms);  // the first replay warms caches
+      }
+      cudaGraphExecDestroy(ge);
+      unit_us[u] = best * 1000.f / (float)reps;
     }
-    cudaGraphDestroy(g);
-    float best = 1e30f;
-    for (int t = 0; t < 3; ++t) {
-      cudaEventRecord(a, e->cap);
-      cudaGraphLaunch(ge, e->cap);
-      cudaEventRecord(b, e->cap);
-      if (cudaEventSynchronize(b) != cudaSuccess) { rc = SWAPNET_ERR_CUDA; break; }
-      float ms = 0.f;
-      cudaEventElapsedTime(&ms, a, b);
-      if (t > 0) best = std::min(best, ms);  // the first replay warms caches
-    }
-    cudaGraphExecDestroy(ge);
-    unit_us[u] = best * 1000.f / (float)reps;
-  }
-  e->profiling = prof;
-  cudaEventDestroy(a);
-  cudaEventDestroy(b);
-  if (rc) SN_FAIL(rc, "unit measurement failed");
-  return SWAPNET_OK;
+    e->profiling = prof;
+    cudaEventDestroy(a);
+    cudaEventDestroy(b);
+    if (rc) SN_FAIL(rc, "unit measurement failed");
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_engine_calibrate(swapnet_engine* e, int32_t reps, int64_t resident_ns, int64_t* t_ex_ns,
                              uint32_t n_layers, uint64_t* alpha_as_per_byte) {
-  if (!e || !t_ex_ns || !alpha_as_per_byte || resident_ns < 0) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad argument");
-  const swapnet_plan& p = e->plan;
-  if (n_layers != p.model.L.size()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "t_ex_ns needs one entry per layer");
-  std::vector<float> us(p.units.size(), 0.f);
-  int rc = swapnet_engine_measure_units(e, reps, us.data(), (uint32_t)us.size());
-  if (rc) return rc;
-  // t_ex per layer: the sum of its units' launch times (a split linear
-  // layer's pieces run one after another)
-  std::vector<int64_t> t(n_layers, 0);
-  for (size_t u = 0; u < p.units.size(); ++u) t[p.units[u].layer] += (int64_t)llround((double)us[u] * 1000.0);
-  for (auto& v : t) v = std::max<int64_t>(1, v);
-  if (resident_ns > 0) {
-    // a unit timed alone runs faster than inside the dependent chain of a
-    // whole inference: scale the t_ex so they add up to the measured
-    // all-resident latency
-    double sum = 0.0;
-    for (int64_t v : t) sum += (double)v;
-    const double f = (double)resident_ns / sum;
-    for (auto& v : t) v = std::max<int64_t>(1, (int64_t)llround((double)v * f));
-  }
-  // alpha: the copy-engine time of every block measured at load over its bytes
-  double bytes = 0.0, copy_us = 0.0;
-  for (size_t k = 0; k < e->blocks.size() && k < p.blocks.size(); ++k) {
-    if (e->blocks[k].memcpy_us <= 0.f) continue;
-    bytes += (double)p.blocks[k].bytes;
-    copy_us += (double)e->blocks[k].memcpy_us;
-  }
-  const uint64_t alpha = (bytes > 0.0 && copy_us > 0.0) ? (uint64_t)llround(copy_us * 1e12 / bytes) : 0;
-  std::copy(t.begin(), t.end(), t_ex_ns);
-  *alpha_as_per_byte = alpha;
-  return SWAPNET_OK;
+  return swapnet::guard_abi([&]() -> int {
+    if (!e || !t_ex_ns || !alpha_as_per_byte || resident_ns < 0) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad argument");
+    const swapnet_plan& p = e->plan;
+    if (n_layers != p.model.L.size()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "t_ex_ns needs one entry per layer");
+    std::vector<float> us(p.units.size(), 0.f);
+    int rc = swapnet_engine_measure_units(e, reps, us.data(), (uint32_t)us.size());
+    if (rc) return rc;
+    // t_ex per layer: the sum of its units' launch times (a split linear
+    // layer's pieces run one after another)
+    std::vector<int64_t> t(n_layers, 0);
+    for (size_t u = 0; u < p.units.size(); ++u) t[p.units[u].layer] += (int64_t)llround((double)us[u] * 1000.0);
+    for (auto& v : t) v = std::max<int64_t>(1, v);
+    if (resident_ns > 0) {
+      // a unit timed alone runs faster than inside the dependent chain of a
+      // whole inference: scale the t_ex so they add up to the measured
+      // all-resident latency
+      double sum = 0.0;
+      for (int64_t v : t) sum += (double)v;
+      const double f = (double)resident_ns / sum;
+      for (auto& v : t) v = std::max<int64_t>(1, (int64_t)llround((double)v * f));
+    }
+    // alpha: the copy-engine time of every block measured at load over its bytes
+    double bytes = 0.0, copy_us = 0.0;
+    for (size_t k = 0; k < e->blocks.size() && k < p.blocks.size(); ++k) {
+      if (e->blocks[k].memcpy_us <= 0.f) continue;
+      bytes += (double)p.blocks[k].bytes;
+      copy_us += (double)e->blocks[k].memcpy_us;
+    }
+    const uint64_t alpha = (bytes > 0.0 && copy_us > 0.0) ? (uint64_t)llround(copy_us * 1e12 / bytes) : 0;
+    std::copy(t.begin(), t.end(), t_ex_ns);
+    *alpha_as_per_byte = alpha;
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_engine_bind_state(swapnet_engine* e, void* d_state, uint64_t bytes) {
-  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
-  if (!e->plan.model.has_attention) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "the model has no decoder state");
-  if (!d_state || bytes < e->plan.model.state_bytes) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "state buffer too small");
-  if ((uintptr_t)d_state % kAlign) SN_FAIL(SWAPNET_ERR_MISALIGNED, "state buffer must be 256-byte aligned");
-  e->d_state = static_cast<char*>(d_state);
-  for (auto& kv : e->graphs) cudaGraphExecDestroy(kv.second);  // captured with the old state
-  e->graphs.clear();
-  return SWAPNET_OK;
+  return swapnet::guard_abi([&]() -> int {
+    if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+    if (!e->plan.model.has_attention) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "the model has no decoder state");
+    if (!d_state || bytes < e->plan.model.state_bytes) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "state buffer too small");
+    if ((uintptr_t)d_state % kAlign) SN_FAIL(SWAPNET_ERR_MISALIGNED, "state buffer must be 256-byte aligned");
+    e->d_state = static_cast<char*>(d_state);
+    for (auto& kv : e->graphs) cudaGraphExecDestroy(kv.second);  // captured with the old state
+    e->graphs.clear();
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_engine_stats_get(const swapnet_engine* e, swapnet_engine_stats* st) {
-  if (!e || !st) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
-  *st = e->stats;
-  return SWAPNET_OK;
+  return swapnet::guard_abi([&]() -> int {
+    if (!e || !st) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+    *st = e->stats;
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_engine_unit_kernels(const swapnet_engine* e, int32_t* kinds, uint32_t cap, uint32_t* n) {
-  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
-  if (n) *n = (uint32_t)e->unit_kind.size();
-  for (uint32_t i = 0; kinds && i < cap && i < e->unit_kind.size(); ++i) kinds[i] = e->unit_kind[i];
-  return SWAPNET_OK;
+  return swapnet::guard_abi([&]() -> int {
+    if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+    if (n) *n = (uint32_t)e->unit_kind.size();
+    for (uint32_t i = 0; kinds && i < cap && i < e->unit_kind.size(); ++i) kinds[i] = e->unit_kind[i];
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_engine_unit_tiling(const swapnet_engine* e, swapnet_unit_tiling* t, uint32_t cap, uint32_t* n) {
-  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
-  if (n) *n = (uint32_t)e->ux.size();
-  for (uint32_t i = 0; t && i < cap && i < e->ux.size(); ++i) {
-    const UnitExec& X = e->ux[i];
-    swapnet_unit_tiling r;
-    std::memset(&r, 0, sizeof(r));
-    if (X.use_tc) {
-      r.n_tile = X.tc.bn;
-      r.splits = X.tc.splits;
-      r.cluster = X.tc.splits > 1 && X.tc.cluster;
-      r.persistent = X.tc.persist;
-      r.tap_tma = X.tc.tma_conv;
+  return swapnet::guard_abi([&]() -> int {
+    if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+    if (n) *n = (uint32_t)e->ux.size();
+    for (uint32_t i = 0; t && i < cap && i < e->ux.size(); ++i) {
+      const UnitExec& X = e->ux[i];
+      swapnet_unit_tiling r;
+      std::memset(&r, 0, sizeof(r));
+      if (X.use_tc) {
+        r.n_tile = X.tc.bn;
+        r.splits = X.tc.splits;
+        r.cluster = X.tc.splits > 1 && X.tc.cluster;
+        r.persistent = X.tc.persist;
+        r.tap_tma = X.tc.tma_conv;
+      }
+      t[i] = r;
     }
-    t[i] = r;
-  }
-  return SWAPNET_OK;
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_engine_set_profiling(swapnet_engine* e, int enable) {
-  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
-  CU(cudaSetDevice(e->device), "cudaSetDevice");
-  if (enable && e->ev_unit.empty()) {
-    e->ev_unit.assign(2 * e->plan.units.size(), nullptr);
-    e->ev_swap.assign(2 * e->plan.blocks.size(), nullptr);
-    for (cudaEvent_t& ev : e->ev_unit) CU(cudaEventCreate(&ev), "event");
-    for (cudaEvent_t& ev : e->ev_swap) CU(cudaEventCreate(&ev), "event");
-  }
-  e->profiling = enable != 0;
-  return SWAPNET_OK;
+  return swapnet::guard_abi([&]() -> int {
+    if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+    CU(cudaSetDevice(e->device), "cudaSetDevice");
+    if (enable && e->ev_unit.empty()) {
+      e->ev_unit.assign(2 * e->plan.units.size(), nullptr);
+      e->ev_swap.assign(2 * e->plan.blocks.size(), nullptr);
+      for (cudaEvent_t& ev : e->ev_unit) CU(cudaEventCreate(&ev), "event");
+      for (cudaEvent_t& ev : e->ev_swap) CU(cudaEventCreate(&ev), "event");
+    }
+    e->profiling = enable != 0;
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_engine_set_swap_timing(swapnet_engine* e, int enable) {
-  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
-  CU(cudaSetDevice(e->device), "cudaSetDevice");
-  if (enable && e->ev_gswap.empty()) {
-    e->ev_gswap.assign(2 * e->plan.blocks.size(), nullptr);
-    for (cudaEvent_t& ev : e->ev_gswap) CU(cudaEventCreate(&ev), "event");
-  }
-  e->swap_timing = enable != 0;
-  return SWAPNET_OK;
+  return swapnet::guard_abi([&]() -> int {
+    if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+    CU(cudaSetDevice(e->device), "cudaSetDevice");
+    if (enable && e->ev_gswap.empty()) {
+      e->ev_gswap.assign(2 * e->plan.blocks.size(), nullptr);
+      for (cudaEvent_t& ev : e->ev_gswap) CU(cudaEventCreate(&ev), "event");
+    }
+    e->swap_timing = enable != 0;
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_engine_last_swap_times(swapnet_engine* e, float* swap_us, uint32_t nb) {
-  if (!e || !swap_us) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
-  if (e->ev_gswap.empty()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "swap timing was never enabled");
-  CU(cudaSetDevice(e->device), "cudaSetDevice");
-  for (uint32_t k = 0; k < nb && k < e->plan.blocks.size(); ++k) {
-    float ms = 0.f;
-    if (swapped(e, k)) {
-      CU(cudaEventSynchronize(e->ev_gswap[2 * k + 1]), "event synchronize");
-      CU(cudaEventElapsedTime(&ms, e->ev_gswap[2 * k], e->ev_gswap[2 * k + 1]), "elapsed");
+  return swapnet::guard_abi([&]() -> int {
+    if (!e || !swap_us) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+    if (e->ev_gswap.empty()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "swap timing was never enabled");
+    CU(cudaSetDevice(e->device), "cudaSetDevice");
+    for (uint32_t k = 0; k < nb && k < e->plan.blocks.size(); ++k) {
+      float ms = 0.f;
+      if (swapped(e, k)) {
+        CU(cudaEventSynchronize(e->ev_gswap[2 * k + 1]), "event synchronize");
+        CU(cudaEventElapsedTime(&ms, e->ev_gswap[2 * k], e->ev_gswap[2 * k + 1]), "elapsed");
+      }
+      swap_us[k] = ms * 1000.f;
     }
-    swap_us[k] = ms * 1000.f;
-  }
-  return SWAPNET_OK;
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_engine_set_graph_timeline(swapnet_engine* e, int enable) {
-  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
-  CU(cudaSetDevice(e->device), "cudaSetDevice");
-  if (enable && e->ev_gswap.empty()) {
-    e->ev_gswap.assign(2 * e->plan.blocks.size(), nullptr);
-    for (cudaEvent_t& ev : e->ev_gswap) CU(cudaEventCreate(&ev), "event");
-  }
-  if (enable && e->ev_gexec.empty()) {
-    e->ev_gexec.assign(2 * e->plan.blocks.size(), nullptr);
-    for (cudaEvent_t& ev : e->ev_gexec) CU(cudaEventCreate(&ev), "event");
-    if (!e->ev_g0) CU(cudaEventCreate(&e->ev_g0), "event");
-  }
-  e->timeline = enable != 0;
-  return SWAPNET_OK;
+  return swapnet::guard_abi([&]() -> int {
+    if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+    CU(cudaSetDevice(e->device), "cudaSetDevice");
+    if (enable && e->ev_gswap.empty()) {
+      e->ev_gswap.assign(2 * e->plan.blocks.size(), nullptr);
+      for (cudaEvent_t& ev : e->ev_gswap) CU(cudaEventCreate(&ev), "event");
+    }
+    if (enable && e->ev_gexec.empty()) {
+      e->ev_gexec.assign(2 * e->plan.blocks.size(), nullptr);
+      for (cudaEvent_t& ev : e->ev_gexec) CU(cudaEventCreate(&ev), "event");
+      if (!e->ev_g0) CU(cudaEventCreate(&e->ev_g0), "event");
+    }
+    e->timeline = enable != 0;
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_engine_last_graph_timeline(swapnet_engine* e, float* t_us, uint32_t nb) {
-  if (!e || !t_us) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
-  if (e->ev_gexec.empty()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "the timeline was never enabled");
-  CU(cudaSetDevice(e->device), "cudaSetDevice");
-  const uint32_t n = std::min<uint32_t>(nb, (uint32_t)e->plan.blocks.size());
-  if (n) CU(cudaEventSynchronize(e->ev_gexec[2 * (n - 1) + 1]), "event synchronize");
-  auto since = [&](cudaEvent_t ev, float* out) -> int {
-    float ms = 0.f;
-    CU(cudaEventSynchronize(ev), "event synchronize");
-    CU(cudaEventElapsedTime(&ms, e->ev_g0, ev), "elapsed");
-    *out = ms * 1000.f;
-    return SWAPNET_OK;
-  };
-  for (uint32_t k = 0; k < n; ++k) {
-    float* o = t_us + 4 * k;
-    o[0] = o[1] = -1.f;
-    const bool pf_first = k == 0 && prefetch_on(e);
-    if (swapped(e, k) && !pf_first) {
-      int rc = since(e->ev_gswap[2 * k], o);
-      if (!rc) rc = since(e->ev_gswap[2 * k + 1], o + 1);
+  return swapnet::guard_abi([&]() -> int {
+    if (!e || !t_us) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+    if (e->ev_gexec.empty()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "the timeline was never enabled");
+    CU(cudaSetDevice(e->device), "cudaSetDevice");
+    const uint32_t n = std::min<uint32_t>(nb, (uint32_t)e->plan.blocks.size());
+    if (n) CU(cudaEventSynchronize(e->ev_gexec[2 * (n - 1) + 1]), "event synchronize");
+    auto since = [&](cudaEvent_t ev, float* out) -> int {
+      float ms = 0.f;
+      CU(cudaEventSynchronize(ev), "event synchronize");
+      CU(cudaEventElapsedTime(&ms, e->ev_g0, ev), "elapsed");
+      *out = ms * 1000.f;
+      return SWAPNET_OK;
+    };
+    for (uint32_t k = 0; k < n; ++k) {
+      float* o = t_us + 4 * k;
+      o[0] = o[1] = -1.f;
+      const bool pf_first = k == 0 && prefetch_on(e);
+      if (swapped(e, k) && !pf_first) {
+        int rc = since(e->ev_gswap[2 * k], o);
+        if (!rc) rc = since(e->ev_gswap[2 * k + 1], o + 1);
+        if (rc) return rc;
+      }
+      int rc = since(e->ev_gexec[2 * k], o + 2);
+      if (!rc) rc = since(e->ev_gexec[2 * k + 1], o + 3);
       if (rc) return rc;
     }
-    int rc = since(e->ev_gexec[2 * k], o + 2);
-    if (!rc) rc = since(e->ev_gexec[2 * k + 1], o + 3);
-    if (rc) return rc;
-  }
-  return SWAPNET_OK;
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_engine_last_times(swapnet_engine* e, float* unit_us, uint32_t nu, float* swap_us, uint32_t nb) {
-  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
-  if (e->ev_unit.empty()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "profiling was never enabled");
-  CU(cudaSetDevice(e->device), "cudaSetDevice");
-  CU(cudaDeviceSynchronize(), "device synchronize");
-  for (uint32_t u = 0; unit_us && u < nu && u < e->plan.units.size(); ++u) {
-    float ms = 0.f;
-    CU(cudaEventElapsedTime(&ms, e->ev_unit[2 * u], e->ev_unit[2 * u + 1]), "elapsed");
-    unit_us[u] = ms * 1000.f;
-  }
-  for (uint32_t k = 0; swap_us && k < nb && k < e->plan.blocks.size(); ++k) {
-    float ms = 0.f;
-    if (swapped(e, k))  // a resident prefix and a block read in host memory are never swapped
-      CU(cudaEventElapsedTime(&ms, e->ev_swap[2 * k], e->ev_swap[2 * k + 1]), "elapsed");
-    swap_us[k] = ms * 1000.f;
-  }
-  return SWAPNET_OK;
+  return swapnet::guard_abi([&]() -> int {
+    if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+    if (e->ev_unit.empty()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "profiling was never enabled");
+    CU(cudaSetDevice(e->device), "cudaSetDevice");
+    CU(cudaDeviceSynchronize(), "device synchronize");
+    for (uint32_t u = 0; unit_us && u < nu && u < e->plan.units.size(); ++u) {
+      float ms = 0.f;
+      CU(cudaEventElapsedTime(&ms, e->ev_unit[2 * u], e->ev_unit[2 * u + 1]), "elapsed");
+      unit_us[u] = ms * 1000.f;
+    }
+    for (uint32_t k = 0; swap_us && k < nb && k < e->plan.blocks.size(); ++k) {
+      float ms = 0.f;
+      if (swapped(e, k))  // a resident prefix and a block read in host memory are never swapped
+        CU(cudaEventElapsedTime(&ms, e->ev_swap[2 * k], e->ev_swap[2 * k + 1]), "elapsed");
+      swap_us[k] = ms * 1000.f;
+    }
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_engine_last_timeline(swapnet_engine* e, float* us0, float* us1, uint32_t nu, float* ss0, float* ss1,
                                  uint32_t nb) {
-  if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
-  if (e->ev_unit.empty()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "profiling was never enabled");
-  CU(cudaSetDevice(e->device), "cudaSetDevice");
-  CU(cudaDeviceSynchronize(), "device synchronize");
-  // first block swapped at the start (a resident prefix has no swap events;
-  // with first-block prefetch block 0's swap comes at the end)
-  size_t k0 = swapnet::prefetch_on(e) ? 1 : 0;
-  while (k0 < e->plan.blocks.size() && !swapnet::swapped(e, k0)) ++k0;
-  const bool sw = !e->plan.resident && !e->ev_swap.empty() && k0 < e->plan.blocks.size();
-  cudaEvent_t origin = sw ? e->ev_swap[2 * k0] : e->ev_unit[0];
-  float first = 0.f;
-  if (sw) {  // the first kernel may start before the first swap event on another stream
-    float d = 0.f;
-    CU(cudaEventElapsedTime(&d, e->ev_swap[2 * k0], e->ev_unit[0]), "elapsed");
-    first = std::min(0.f, d);
-  }
-  auto rel = [&](cudaEvent_t ev, float* out) -> int {
-    float ms = 0.f;
-    CU(cudaEventElapsedTime(&ms, origin, ev), "elapsed");
-    *out = (ms - first) * 1000.f;
-    return SWAPNET_OK;
-  };
-  for (uint32_t u = 0; u < nu && u < e->plan.units.size(); ++u) {
-    if (us0 && rel(e->ev_unit[2 * u], &us0[u])) return SWAPNET_ERR_CUDA;
-    if (us1 && rel(e->ev_unit[2 * u + 1], &us1[u])) return SWAPNET_ERR_CUDA;
-  }
-  for (uint32_t k = 0; k < nb && k < e->plan.blocks.size(); ++k) {
-    if (!sw || !swapnet::swapped(e, k)) {
-      if (ss0) ss0[k] = 0.f;
-      if (ss1) ss1[k] = 0.f;
-      continue;
+  return swapnet::guard_abi([&]() -> int {
+    if (!e) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null engine");
+    if (e->ev_unit.empty()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "profiling was never enabled");
+    CU(cudaSetDevice(e->device), "cudaSetDevice");
+    CU(cudaDeviceSynchronize(), "device synchronize");
+    // first block swapped at the start (a resident prefix has no swap events;
+    // with first-block prefetch block 0's swap comes at the end)
+    size_t k0 = swapnet::prefetch_on(e) ? 1 : 0;
+    while (k0 < e->plan.blocks.size() && !swapnet::swapped(e, k0)) ++k0;
+    const bool sw = !e->plan.resident && !e->ev_swap.empty() && k0 < e->plan.blocks.size();
+    cudaEvent_t origin = sw ? e->ev_swap[2 * k0] : e->ev_unit[0];
+    float first = 0.f;
+    if (sw) {  // the first kernel may start before the first swap event on another stream
+      float d = 0.f;
+      CU(cudaEventElapsedTime(&d, e->ev_swap[2 * k0], e->ev_unit[0]), "elapsed");
+      first = std::min(0.f, d);
     }
-    if (ss0 && rel(e->ev_swap[2 * k], &ss0[k])) return SWAPNET_ERR_CUDA;
-    if (ss1 && rel(e->ev_swap[2 * k + 1], &ss1[k])) return SWAPNET_ERR_CUDA;
-  }
-  return SWAPNET_OK;
+    auto rel = [&](cudaEvent_t ev, float* out) -> int {
+      float ms = 0.f;
+      CU(cudaEventElapsedTime(&ms, origin, ev), "elapsed");
+      *out = (ms - first) * 1000.f;
+      return SWAPNET_OK;
+    };
+    for (uint32_t u = 0; u < nu && u < e->plan.units.size(); ++u) {
+      if (us0 && rel(e->ev_unit[2 * u], &us0[u])) return SWAPNET_ERR_CUDA;
+      if (us1 && rel(e->ev_unit[2 * u + 1], &us1[u])) return SWAPNET_ERR_CUDA;
+    }
+    for (uint32_t k = 0; k < nb && k < e->plan.blocks.size(); ++k) {
+      if (!sw || !swapnet::swapped(e, k)) {
+        if (ss0) ss0[k] = 0.f;
+        if (ss1) ss1[k] = 0.f;
+        continue;
+      }
+      if (ss0 && rel(e->ev_swap[2 * k], &ss0[k])) return SWAPNET_ERR_CUDA;
+      if (ss1 && rel(e->ev_swap[2 * k + 1], &ss1[k])) return SWAPNET_ERR_CUDA;
+    }
+    return SWAPNET_OK;
+  });
 }
 
 void swapnet_engine_free(swapnet_engine* e) { release(e); }
 
 int swapnet_host_alloc(uint64_t bytes, void** out) {
-  if (!out || bytes == 0) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null out or zero bytes");
-  *out = nullptr;
-  if (injected(1) || cudaHostAlloc(out, bytes, cudaHostAllocPortable | cudaHostAllocMapped) != cudaSuccess) {
-    cudaGetLastError();
+  return swapnet::guard_abi([&]() -> int {
+    if (!out || bytes == 0) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null out or zero bytes");
     *out = nullptr;
-    SN_FAIL(SWAPNET_ERR_OOM, "page-locked host allocation failed");
-  }
-  return SWAPNET_OK;
+    if (injected(1) || cudaHostAlloc(out, bytes, cudaHostAllocPortable | cudaHostAllocMapped) != cudaSuccess) {
+      cudaGetLastError();
+      *out = nullptr;
+      SN_FAIL(SWAPNET_ERR_OOM, "page-locked host allocation failed");
+    }
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_host_free(void* p) {
-  if (!p) return SWAPNET_OK;
-  CU(cudaFreeHost(p), "cudaFreeHost");
-  return SWAPNET_OK;
+  return swapnet::guard_abi([&]() -> int {
+    if (!p) return SWAPNET_OK;
+    CU(cudaFreeHost(p), "cudaFreeHost");
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_debug_fail_next(int what, int count) {
-  if (what < 1 || what > 3 || count < 0) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad fault-injection request");
-  g_fail_next[what] = count;
-  return SWAPNET_OK;
+  return swapnet::guard_abi([&]() -> int {
+    if (what < 1 || what > 3 || count < 0) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad fault-injection request");
+    g_fail_next[what] = count;
+    return SWAPNET_OK;
+  });
 }
 
 }  // extern "C"

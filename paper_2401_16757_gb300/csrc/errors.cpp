@@ -5,7 +5,13 @@
 
 namespace swapnet {
 static thread_local std::string t_last_error;
-void set_error(const std::string& msg) { t_last_error = msg; }
+void set_error(const std::string& msg) {
+  try {
+    t_last_error = msg;
+  } catch (...) {  // no room for the message: leave it empty rather than throw
+    t_last_error.clear();
+  }
+}
 }  // namespace swapnet
 
 extern "C" {
@@ -21,6 +27,7 @@ const char* swapnet_strerror(int status) {
     case SWAPNET_ERR_MISALIGNED: return "misaligned pointer or size";
     case SWAPNET_ERR_UNSUPPORTED: return "unsupported shape or dtype";
     case SWAPNET_ERR_IO: return "weights file I/O error";
+    case SWAPNET_ERR_INTERNAL: return "unexpected host-side error";
     default: return "unknown status";
   }
 }

@@ -1,6 +1,8 @@
 // Internal structures shared by the host-side translation units of libswapnet.
 #pragma once
 #include <cstdint>
+#include <exception>
+#include <new>
 #include <string>
 #include <vector>
 
@@ -25,6 +27,25 @@ struct Status {
     ::swapnet::set_error(msg); \
     return (code);           \
   } while (0)
+
+// Runs the body of a C entry point so that no C++ exception crosses the C
+// ABI: a failed host allocation becomes SWAPNET_ERR_OOM, anything else
+// SWAPNET_ERR_INTERNAL, with the message in swapnet_last_error().
+template <typename F>
+inline int guard_abi(F&& body) noexcept {
+  try {
+    return body();
+  } catch (const std::bad_alloc&) {
+    set_error("host allocation failed");
+    return SWAPNET_ERR_OOM;
+  } catch (const std::exception& ex) {
+    set_error(ex.what());
+    return SWAPNET_ERR_INTERNAL;
+  } catch (...) {
+    set_error("unexpected host-side exception");
+    return SWAPNET_ERR_INTERNAL;
+  }
+}
 
 int dtype_size(int dtype);
 

@@ -30,20 +30,22 @@ __global__ void wait_timeout_probe_kernel(int* err) {
 }  // namespace swapnet
 
 extern "C" int swapnet_debug_wait_timeout(swapnet_stream stream) {
-  using namespace swapnet;
-  int* err = nullptr;
-  int rc = tc_error_word(&err);
-  if (rc) return rc;
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  wait_timeout_probe_kernel<<<1, 32, 0, s>>>(err);
-  int w = 0;
-  const int zero = 0;
-  cudaError_t ce = cudaGetLastError();
-  if (ce == cudaSuccess) ce = cudaStreamSynchronize(s);
-  if (ce == cudaSuccess) ce = cudaMemcpy(&w, err, sizeof(int), cudaMemcpyDeviceToHost);
-  if (ce == cudaSuccess) ce = cudaMemcpy(err, &zero, sizeof(int), cudaMemcpyHostToDevice);
-  if (ce != cudaSuccess) SN_FAIL(SWAPNET_ERR_CUDA, std::string("timeout probe: ") + cudaGetErrorString(ce));
-  if (w == kDevErrTimeout) SN_FAIL(SWAPNET_ERR_TIMEOUT, "a device-side wait gave up (probe)");
-  if (w) SN_FAIL(SWAPNET_ERR_CUDA, "unexpected error word from the probe");
-  return SWAPNET_OK;
+  return swapnet::guard_abi([&]() -> int {
+    using namespace swapnet;
+    int* err = nullptr;
+    int rc = tc_error_word(&err);
+    if (rc) return rc;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    wait_timeout_probe_kernel<<<1, 32, 0, s>>>(err);
+    int w = 0;
+    const int zero = 0;
+    cudaError_t ce = cudaGetLastError();
+    if (ce == cudaSuccess) ce = cudaStreamSynchronize(s);
+    if (ce == cudaSuccess) ce = cudaMemcpy(&w, err, sizeof(int), cudaMemcpyDeviceToHost);
+    if (ce == cudaSuccess) ce = cudaMemcpy(err, &zero, sizeof(int), cudaMemcpyHostToDevice);
+    if (ce != cudaSuccess) SN_FAIL(SWAPNET_ERR_CUDA, std::string("timeout probe: ") + cudaGetErrorString(ce));
+    if (w == kDevErrTimeout) SN_FAIL(SWAPNET_ERR_TIMEOUT, "a device-side wait gave up (probe)");
+    if (w) SN_FAIL(SWAPNET_ERR_CUDA, "unexpected error word from the probe");
+    return SWAPNET_OK;
+  });
 }

@@ -935,74 +935,76 @@ int tc_error_word(int** ptr) {
 
 extern "C" int swapnet_gemm_noalloc(int32_t dtype, const void* A, const void* W, const void* bias, void* Y,
                                     int32_t M, int32_t N, int32_t K, int32_t act, swapnet_stream stream) {
-  using namespace swapnet;
-  if (dtype != SWAPNET_F16 && dtype != SWAPNET_BF16) SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "fp16 or bf16 only");
-  if (!A || !W || !bias || !Y || M < 1 || N < 1 || K < 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null pointer or empty shape");
-  if (act < SWAPNET_ACT_NONE || act > SWAPNET_ACT_LEAKY) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad activation");
-  if (K % 8) SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "K must be a multiple of 8");
-  if (((uintptr_t)A | (uintptr_t)W | (uintptr_t)bias | (uintptr_t)Y) & 15)
-    SN_FAIL(SWAPNET_ERR_MISALIGNED, "pointers must be 16-byte aligned");
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
-    cudaGetLastError();
-    SN_FAIL(SWAPNET_ERR_CUDA, "no current CUDA device");
-  }
-  NoAllocDevice d;
-  {
-    std::lock_guard<std::mutex> lk(g_noalloc_mu);
-    NoAllocDevice& c = g_noalloc_dev[dev];
-    if (!c.scratch) {  // once per device, with that device current
-      void* p = nullptr;
-      cudaError_t r = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-      if (r != cudaSuccess || !p) {
-        cudaGetLastError();
-        SN_FAIL(SWAPNET_ERR_CUDA, std::string("cudaGetSymbolAddress(scratch): ") + cudaGetErrorString(r));
-      }
-      void* e = nullptr;
-      r = cudaGetSymbolAddress(&e, g_tc_err);
-      if (r != cudaSuccess || !e) {
-        cudaGetLastError();
-        SN_FAIL(SWAPNET_ERR_CUDA, std::string("cudaGetSymbolAddress(error word): ") + cudaGetErrorString(r));
-      }
-      int sms = 0;
-      if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
-        cudaGetLastError();
-        SN_FAIL(SWAPNET_ERR_CUDA, "device attribute query failed");
-      }
-      c.scratch = static_cast<unsigned char*>(p);
-      c.err = static_cast<int*>(e);
-      c.sms = sms;
-    }
-    d = c;
-  }
-  TcGemm g;
-  std::memset(&g, 0, sizeof(g));
-  g.dtype = dtype;
-  g.M = M; g.N = N; g.K = K;
-  g.W = W;
-  g.A = A; g.lda = K; g.conv = 0;
-  g.e.bias = bias; g.e.res = nullptr; g.e.ldr = N; g.e.act = act; g.e.res_post = 0;
-  g.y = Y; g.ldy = N;
-  g.num_sms = d.sms;
-  // W and bias are caller memory that the previous work on the stream (an
-  // earlier call, say) may have written: no early start before it completes
-  g.no_pdl = 1;
-  TcPlan pl;
-  int rc = tc_prepare(g, &pl);
-  if (rc) return rc;
-  if (pl.splits > 1) {  // cluster_max == 0: global split-K scratch
-    const uint64_t counters = (uint64_t)pl.tiles * sizeof(int);
-    if (counters > kNoAllocCounterBytes || kNoAllocCounterBytes + pl.scratch_bytes > kNoAllocBytes)
-      SN_FAIL(SWAPNET_ERR_INVALID_ARG, "problem needs " + std::to_string(kNoAllocCounterBytes + pl.scratch_bytes) +
-                                           " bytes of split-K scratch; the static scratch holds " +
-                                           std::to_string(kNoAllocBytes));
-    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    if (cudaMemsetAsync(d.scratch, 0, counters, s) != cudaSuccess) {
+  return swapnet::guard_abi([&]() -> int {
+    using namespace swapnet;
+    if (dtype != SWAPNET_F16 && dtype != SWAPNET_BF16) SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "fp16 or bf16 only");
+    if (!A || !W || !bias || !Y || M < 1 || N < 1 || K < 1) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null pointer or empty shape");
+    if (act < SWAPNET_ACT_NONE || act > SWAPNET_ACT_LEAKY) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad activation");
+    if (K % 8) SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "K must be a multiple of 8");
+    if (((uintptr_t)A | (uintptr_t)W | (uintptr_t)bias | (uintptr_t)Y) & 15)
+      SN_FAIL(SWAPNET_ERR_MISALIGNED, "pointers must be 16-byte aligned");
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
       cudaGetLastError();
-      SN_FAIL(SWAPNET_ERR_CUDA, "clearing the split-K counters failed");
+      SN_FAIL(SWAPNET_ERR_CUDA, "no current CUDA device");
     }
-    g.counters = reinterpret_cast<int*>(d.scratch);
-    g.partial = reinterpret_cast<float*>(d.scratch + kNoAllocCounterBytes);
-  }
-  return launch_tc_gemm(g, pl, d.err, reinterpret_cast<cudaStream_t>(stream));
+    NoAllocDevice d;
+    {
+      std::lock_guard<std::mutex> lk(g_noalloc_mu);
+      NoAllocDevice& c = g_noalloc_dev[dev];
+      if (!c.scratch) {  // once per device, with that device current
+        void* p = nullptr;
+        cudaError_t r = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (r != cudaSuccess || !p) {
+          cudaGetLastError();
+          SN_FAIL(SWAPNET_ERR_CUDA, std::string("cudaGetSymbolAddress(scratch): ") + cudaGetErrorString(r));
+        }
+        void* e = nullptr;
+        r = cudaGetSymbolAddress(&e, g_tc_err);
+        if (r != cudaSuccess || !e) {
+          cudaGetLastError();
+          SN_FAIL(SWAPNET_ERR_CUDA, std::string("cudaGetSymbolAddress(error word): ") + cudaGetErrorString(r));
+        }
+        int sms = 0;
+        if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+          cudaGetLastError();
+          SN_FAIL(SWAPNET_ERR_CUDA, "device attribute query failed");
+        }
+        c.scratch = static_cast<unsigned char*>(p);
+        c.err = static_cast<int*>(e);
+        c.sms = sms;
+      }
+      d = c;
+    }
+    TcGemm g;
+    std::memset(&g, 0, sizeof(g));
+    g.dtype = dtype;
+    g.M = M; g.N = N; g.K = K;
+    g.W = W;
+    g.A = A; g.lda = K; g.conv = 0;
+    g.e.bias = bias; g.e.res = nullptr; g.e.ldr = N; g.e.act = act; g.e.res_post = 0;
+    g.y = Y; g.ldy = N;
+    g.num_sms = d.sms;
+    // W and bias are caller memory that the previous work on the stream (an
+    // earlier call, say) may have written: no early start before it completes
+    g.no_pdl = 1;
+    TcPlan pl;
+    int rc = tc_prepare(g, &pl);
+    if (rc) return rc;
+    if (pl.splits > 1) {  // cluster_max == 0: global split-K scratch
+      const uint64_t counters = (uint64_t)pl.tiles * sizeof(int);
+      if (counters > kNoAllocCounterBytes || kNoAllocCounterBytes + pl.scratch_bytes > kNoAllocBytes)
+        SN_FAIL(SWAPNET_ERR_INVALID_ARG, "problem needs " + std::to_string(kNoAllocCounterBytes + pl.scratch_bytes) +
+                                             " bytes of split-K scratch; the static scratch holds " +
+                                             std::to_string(kNoAllocBytes));
+      cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+      if (cudaMemsetAsync(d.scratch, 0, counters, s) != cudaSuccess) {
+        cudaGetLastError();
+        SN_FAIL(SWAPNET_ERR_CUDA, "clearing the split-K counters failed");
+      }
+      g.counters = reinterpret_cast<int*>(d.scratch);
+      g.partial = reinterpret_cast<float*>(d.scratch + kNoAllocCounterBytes);
+    }
+    return launch_tc_gemm(g, pl, d.err, reinterpret_cast<cudaStream_t>(stream));
+  });
 }

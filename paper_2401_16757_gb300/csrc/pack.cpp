@@ -129,18 +129,20 @@ void pack_write(const uint16_t* src, uint64_t n, const PackInfo& info, uint8_t* 
 
 extern "C" int swapnet_pack_bf16(const void* src, uint64_t n_elems, void* dst, uint64_t dst_bytes,
                                  uint64_t* used_bytes) {
-  if (!src || !used_bytes) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
-  if (n_elems == 0 || n_elems % swapnet::kPkChunk)
-    SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "packing: the element count must be a positive multiple of 4096");
-  const int threads = (int)std::min(32u, std::max(1u, std::thread::hardware_concurrency()));
-  try {
-    const swapnet::PackInfo info = swapnet::pack_prepare(static_cast<const uint16_t*>(src), n_elems, threads);
-    *used_bytes = info.bytes;
-    if (!dst) return SWAPNET_OK;
-    if (dst_bytes < info.bytes) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "packing: destination too small");
-    swapnet::pack_write(static_cast<const uint16_t*>(src), n_elems, info, static_cast<uint8_t*>(dst), threads);
-  } catch (...) {  // allocation or thread creation
-    SN_FAIL(SWAPNET_ERR_OOM, "packing: host resources exhausted");
-  }
-  return SWAPNET_OK;
+  return swapnet::guard_abi([&]() -> int {
+    if (!src || !used_bytes) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+    if (n_elems == 0 || n_elems % swapnet::kPkChunk)
+      SN_FAIL(SWAPNET_ERR_UNSUPPORTED, "packing: the element count must be a positive multiple of 4096");
+    const int threads = (int)std::min(32u, std::max(1u, std::thread::hardware_concurrency()));
+    try {
+      const swapnet::PackInfo info = swapnet::pack_prepare(static_cast<const uint16_t*>(src), n_elems, threads);
+      *used_bytes = info.bytes;
+      if (!dst) return SWAPNET_OK;
+      if (dst_bytes < info.bytes) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "packing: destination too small");
+      swapnet::pack_write(static_cast<const uint16_t*>(src), n_elems, info, static_cast<uint8_t*>(dst), threads);
+    } catch (...) {  // allocation or thread creation
+      SN_FAIL(SWAPNET_ERR_OOM, "packing: host resources exhausted");
+    }
+    return SWAPNET_OK;
+  });
 }

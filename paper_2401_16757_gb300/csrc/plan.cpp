@@ -931,185 +931,203 @@ void swapnet_default_options(swapnet_options* o) {
 
 int swapnet_partition(const swapnet_model_desc* desc, uint64_t budget, const swapnet_options* opt,
                       swapnet_plan** out) {
-  if (!out) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null out_plan");
-  try {
-    std::unique_ptr<swapnet_plan> p;
-    int rc = prepare(desc, budget, opt, &p);
-    if (rc) return rc;
-    std::vector<uint32_t> cuts;
-    if (p->opt.objective != 0) rc = search_exhaustive_eq4(p.get(), &cuts);
-    else if (p->opt.resident_prefix) rc = search_with_prefix(p.get(), &cuts);
-    else if (p->opt.prefetch) rc = search_cyclic(p.get(), &cuts);
-    else rc = search_pipeline(p.get(), &cuts);
-    if (rc) return rc;
-    finalize_blocks(p.get(), cuts);
-    *out = p.release();
-    return SWAPNET_OK;
-  } catch (const std::bad_alloc&) {
-    SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
-  }
+  return swapnet::guard_abi([&]() -> int {
+    if (!out) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null out_plan");
+    try {
+      std::unique_ptr<swapnet_plan> p;
+      int rc = prepare(desc, budget, opt, &p);
+      if (rc) return rc;
+      std::vector<uint32_t> cuts;
+      if (p->opt.objective != 0) rc = search_exhaustive_eq4(p.get(), &cuts);
+      else if (p->opt.resident_prefix) rc = search_with_prefix(p.get(), &cuts);
+      else if (p->opt.prefetch) rc = search_cyclic(p.get(), &cuts);
+      else rc = search_pipeline(p.get(), &cuts);
+      if (rc) return rc;
+      finalize_blocks(p.get(), cuts);
+      *out = p.release();
+      return SWAPNET_OK;
+    } catch (const std::bad_alloc&) {
+      SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
+    }
+  });
 }
 
 int swapnet_plan_from_cuts(const swapnet_model_desc* desc, const uint32_t* cuts, uint32_t n_cuts,
                            uint64_t budget, const swapnet_options* opt, swapnet_plan** out) {
-  if (!out || (n_cuts && !cuts)) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
-  try {
-    std::unique_ptr<swapnet_plan> p;
-    int rc = prepare(desc, budget, opt, &p);
-    if (rc) return rc;
-    std::vector<uint32_t> c(cuts, cuts + n_cuts);
-    uint32_t prev = 0;
-    for (uint32_t v : c) {
-      if (v <= prev || v >= p->units.size()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "cuts must increase within [1, n_units)");
-      prev = v;
+  return swapnet::guard_abi([&]() -> int {
+    if (!out || (n_cuts && !cuts)) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+    try {
+      std::unique_ptr<swapnet_plan> p;
+      int rc = prepare(desc, budget, opt, &p);
+      if (rc) return rc;
+      std::vector<uint32_t> c(cuts, cuts + n_cuts);
+      uint32_t prev = 0;
+      for (uint32_t v : c) {
+        if (v <= prev || v >= p->units.size()) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "cuts must increase within [1, n_units)");
+        prev = v;
+      }
+      finalize_blocks(p.get(), c);
+      for (size_t k = 0; k < p->blocks.size(); ++k)
+        if (!pair_ok(p.get(), k ? p->blocks[k - 1].bytes : 0, p->blocks[k].bytes))
+          SN_FAIL(SWAPNET_ERR_INFEASIBLE, "a block (or two adjacent blocks) exceeds the arena");
+      const size_t n = p->blocks.size();
+      if (p->opt.prefetch && n >= 2 && n % 2 == 0 && p->blocks[0].bytes + p->blocks[n - 1].bytes > p->region)
+        SN_FAIL(SWAPNET_ERR_INFEASIBLE, "the last block and the next inference's first block exceed the arena");
+      *out = p.release();
+      return SWAPNET_OK;
+    } catch (const std::bad_alloc&) {
+      SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
     }
-    finalize_blocks(p.get(), c);
-    for (size_t k = 0; k < p->blocks.size(); ++k)
-      if (!pair_ok(p.get(), k ? p->blocks[k - 1].bytes : 0, p->blocks[k].bytes))
-        SN_FAIL(SWAPNET_ERR_INFEASIBLE, "a block (or two adjacent blocks) exceeds the arena");
-    const size_t n = p->blocks.size();
-    if (p->opt.prefetch && n >= 2 && n % 2 == 0 && p->blocks[0].bytes + p->blocks[n - 1].bytes > p->region)
-      SN_FAIL(SWAPNET_ERR_INFEASIBLE, "the last block and the next inference's first block exceed the arena");
-    *out = p.release();
-    return SWAPNET_OK;
-  } catch (const std::bad_alloc&) {
-    SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
-  }
+  });
 }
 
 int swapnet_plan_resident(const swapnet_model_desc* desc, const swapnet_options* opt, swapnet_plan** out) {
-  if (!out) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null out_plan");
-  try {
-    std::unique_ptr<swapnet_plan> p(new swapnet_plan());
-    if (opt) p->opt = *opt; else swapnet_default_options(&p->opt);
-    int rc = check_options(p->opt);
-    if (rc) return rc;
-    rc = analyse_model(desc, &p->model);
-    if (rc) return rc;
-    p->resident = true;
-    p->arena = p->model.weight_bytes;
-    p->region = p->arena;
-    p->slot = p->arena;
-    p->budget = p->arena;
-    rc = make_units(p->model, p->opt, ~0ull, ~0ull, &p->units);
-    if (rc) return rc;
-    finalize_blocks(p.get(), {});
-    *out = p.release();
-    return SWAPNET_OK;
-  } catch (const std::bad_alloc&) {
-    SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
-  }
+  return swapnet::guard_abi([&]() -> int {
+    if (!out) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null out_plan");
+    try {
+      std::unique_ptr<swapnet_plan> p(new swapnet_plan());
+      if (opt) p->opt = *opt; else swapnet_default_options(&p->opt);
+      int rc = check_options(p->opt);
+      if (rc) return rc;
+      rc = analyse_model(desc, &p->model);
+      if (rc) return rc;
+      p->resident = true;
+      p->arena = p->model.weight_bytes;
+      p->region = p->arena;
+      p->slot = p->arena;
+      p->budget = p->arena;
+      rc = make_units(p->model, p->opt, ~0ull, ~0ull, &p->units);
+      if (rc) return rc;
+      finalize_blocks(p.get(), {});
+      *out = p.release();
+      return SWAPNET_OK;
+    } catch (const std::bad_alloc&) {
+      SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
+    }
+  });
 }
 
 int swapnet_plan_info_get(const swapnet_plan* p, swapnet_plan_info* info) {
-  if (!p || !info) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
-  swapnet_plan_info r{};
-  r.n_blocks = (uint32_t)p->blocks.size();
-  r.n_units = (uint32_t)p->units.size();
-  r.slots = p->resident ? 0 : (uint32_t)p->opt.slots;
-  r.n_layers = (uint32_t)p->model.L.size();
-  r.budget_bytes = p->budget;
-  r.arena_bytes = p->arena;
-  r.slot_bytes = p->slot;
-  r.workspace_bytes = p->model.ws_bytes;
-  r.input_bytes = p->model.in_bytes;
-  r.output_bytes = p->model.out_bytes;
-  r.weight_bytes = p->model.weight_bytes;
-  r.plan_bytes = sizeof(swapnet_plan) + p->units.size() * sizeof(Unit) + p->blocks.size() * sizeof(Block) +
-                 p->model.L.size() * sizeof(Layer) + p->cuts.size() * sizeof(uint32_t);
-  r.predicted_ns = p->predicted;
-  r.state_bytes = p->model.state_bytes;
-  r.exact = p->exact ? 1 : 0;
-  r.prefix_units = (uint32_t)p->prefix_units;
-  r.prefix_bytes = p->prefix_bytes;
-  *info = r;
-  return SWAPNET_OK;
+  return swapnet::guard_abi([&]() -> int {
+    if (!p || !info) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+    swapnet_plan_info r{};
+    r.n_blocks = (uint32_t)p->blocks.size();
+    r.n_units = (uint32_t)p->units.size();
+    r.slots = p->resident ? 0 : (uint32_t)p->opt.slots;
+    r.n_layers = (uint32_t)p->model.L.size();
+    r.budget_bytes = p->budget;
+    r.arena_bytes = p->arena;
+    r.slot_bytes = p->slot;
+    r.workspace_bytes = p->model.ws_bytes;
+    r.input_bytes = p->model.in_bytes;
+    r.output_bytes = p->model.out_bytes;
+    r.weight_bytes = p->model.weight_bytes;
+    r.plan_bytes = sizeof(swapnet_plan) + p->units.size() * sizeof(Unit) + p->blocks.size() * sizeof(Block) +
+                   p->model.L.size() * sizeof(Layer) + p->cuts.size() * sizeof(uint32_t);
+    r.predicted_ns = p->predicted;
+    r.state_bytes = p->model.state_bytes;
+    r.exact = p->exact ? 1 : 0;
+    r.prefix_units = (uint32_t)p->prefix_units;
+    r.prefix_bytes = p->prefix_bytes;
+    *info = r;
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_plan_cuts(const swapnet_plan* p, uint32_t* cuts, uint32_t cap, uint32_t* n) {
-  if (!p) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null plan");
-  if (n) *n = (uint32_t)p->cuts.size();
-  for (uint32_t i = 0; cuts && i < cap && i < p->cuts.size(); ++i) cuts[i] = p->cuts[i];
-  return SWAPNET_OK;
+  return swapnet::guard_abi([&]() -> int {
+    if (!p) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null plan");
+    if (n) *n = (uint32_t)p->cuts.size();
+    for (uint32_t i = 0; cuts && i < cap && i < p->cuts.size(); ++i) cuts[i] = p->cuts[i];
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_plan_units(const swapnet_plan* p, swapnet_unit_info* u, uint32_t cap, uint32_t* n) {
-  if (!p) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null plan");
-  if (n) *n = (uint32_t)p->units.size();
-  for (uint32_t i = 0; u && i < cap && i < p->units.size(); ++i) {
-    const Unit& U = p->units[i];
-    u[i] = swapnet_unit_info{U.layer, U.row0, U.rows, U.depth, U.bytes, U.flops, U.t_ex};
-  }
-  return SWAPNET_OK;
+  return swapnet::guard_abi([&]() -> int {
+    if (!p) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null plan");
+    if (n) *n = (uint32_t)p->units.size();
+    for (uint32_t i = 0; u && i < cap && i < p->units.size(); ++i) {
+      const Unit& U = p->units[i];
+      u[i] = swapnet_unit_info{U.layer, U.row0, U.rows, U.depth, U.bytes, U.flops, U.t_ex};
+    }
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_plan_blocks(const swapnet_plan* p, swapnet_block_info* b, uint32_t cap, uint32_t* n) {
-  if (!p) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null plan");
-  if (n) *n = (uint32_t)p->blocks.size();
-  for (uint32_t i = 0; b && i < cap && i < p->blocks.size(); ++i) {
-    const Block& B = p->blocks[i];
-    b[i] = swapnet_block_info{(uint32_t)B.u0, (uint32_t)B.u1, (uint32_t)B.slot, (uint32_t)B.depth, B.bytes,
-                              B.t_in, B.t_ex, B.t_out, B.base};
-  }
-  return SWAPNET_OK;
+  return swapnet::guard_abi([&]() -> int {
+    if (!p) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null plan");
+    if (n) *n = (uint32_t)p->blocks.size();
+    for (uint32_t i = 0; b && i < cap && i < p->blocks.size(); ++i) {
+      const Block& B = p->blocks[i];
+      b[i] = swapnet_block_info{(uint32_t)B.u0, (uint32_t)B.u1, (uint32_t)B.slot, (uint32_t)B.depth, B.bytes,
+                                B.t_in, B.t_ex, B.t_out, B.base};
+    }
+    return SWAPNET_OK;
+  });
 }
 
 int swapnet_plan_output_offsets(const swapnet_plan* p, uint64_t* offs, uint32_t cap, uint32_t* n) {
-  if (!p) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null plan");
-  uint32_t k = 0;
-  for (const Layer& L : p->model.L) {
-    if (L.out_off < 0) continue;
-    if (offs && k < cap) offs[k] = (uint64_t)L.out_off;
-    ++k;
-  }
-  if (n) *n = k;
-  return SWAPNET_OK;
+  return swapnet::guard_abi([&]() -> int {
+    if (!p) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null plan");
+    uint32_t k = 0;
+    for (const Layer& L : p->model.L) {
+      if (L.out_off < 0) continue;
+      if (offs && k < cap) offs[k] = (uint64_t)L.out_off;
+      ++k;
+    }
+    if (n) *n = k;
+    return SWAPNET_OK;
+  });
 }
 
 void swapnet_plan_free(swapnet_plan* p) { delete p; }
 
 int swapnet_schedule(const swapnet_model_desc* const* models, const float* urgency, uint32_t n,
                      uint64_t M, const swapnet_options* opt, uint64_t* budgets_out, swapnet_plan** plans_out) {
-  if (!models || !urgency || n == 0 || !plans_out) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
-  try {
-    swapnet_options o;
-    if (opt) o = *opt; else swapnet_default_options(&o);
-    std::vector<Model> ms(n);
-    std::vector<long double> demand(n), ps(n);
-    long double sumM = 0, sumPS = 0;
-    for (uint32_t i = 0; i < n; ++i) {
-      int rc = analyse_model(models[i], &ms[i]);
-      if (rc) return rc;
-      if (!(urgency[i] >= 0.0f) || !std::isfinite(urgency[i])) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad urgency");
-      demand[i] = (long double)ms[i].weight_bytes;
-      const long double lat = (long double)resident_latency_ns(ms[i], o);
-      ps[i] = (long double)urgency[i] * lat / demand[i];
-      sumM += demand[i];
-      sumPS += ps[i];
-    }
-    std::vector<uint64_t> budgets(n);
-    for (uint32_t i = 0; i < n; ++i) {
-      if (sumM <= (long double)M) { budgets[i] = ms[i].weight_bytes; continue; }
-      long double a = demand[i] / sumM * (1.0L - 1.0L / n) * (long double)M;
-      if (sumPS > 0) a += ps[i] / sumPS * (1.0L / n) * (long double)M;
-      budgets[i] = (uint64_t)floorl(a) / kAlign * kAlign;
-    }
-    std::vector<swapnet_plan*> plans(n, nullptr);
-    for (uint32_t i = 0; i < n; ++i) {
-      int rc = swapnet_partition(models[i], budgets[i], &o, &plans[i]);
-      if (rc) {
-        for (swapnet_plan* q : plans) delete q;
-        return rc;
+  return swapnet::guard_abi([&]() -> int {
+    if (!models || !urgency || n == 0 || !plans_out) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "null argument");
+    try {
+      swapnet_options o;
+      if (opt) o = *opt; else swapnet_default_options(&o);
+      std::vector<Model> ms(n);
+      std::vector<long double> demand(n), ps(n);
+      long double sumM = 0, sumPS = 0;
+      for (uint32_t i = 0; i < n; ++i) {
+        int rc = analyse_model(models[i], &ms[i]);
+        if (rc) return rc;
+        if (!(urgency[i] >= 0.0f) || !std::isfinite(urgency[i])) SN_FAIL(SWAPNET_ERR_INVALID_ARG, "bad urgency");
+        demand[i] = (long double)ms[i].weight_bytes;
+        const long double lat = (long double)resident_latency_ns(ms[i], o);
+        ps[i] = (long double)urgency[i] * lat / demand[i];
+        sumM += demand[i];
+        sumPS += ps[i];
       }
+      std::vector<uint64_t> budgets(n);
+      for (uint32_t i = 0; i < n; ++i) {
+        if (sumM <= (long double)M) { budgets[i] = ms[i].weight_bytes; continue; }
+        long double a = demand[i] / sumM * (1.0L - 1.0L / n) * (long double)M;
+        if (sumPS > 0) a += ps[i] / sumPS * (1.0L / n) * (long double)M;
+        budgets[i] = (uint64_t)floorl(a) / kAlign * kAlign;
+      }
+      std::vector<swapnet_plan*> plans(n, nullptr);
+      for (uint32_t i = 0; i < n; ++i) {
+        int rc = swapnet_partition(models[i], budgets[i], &o, &plans[i]);
+        if (rc) {
+          for (swapnet_plan* q : plans) delete q;
+          return rc;
+        }
+      }
+      for (uint32_t i = 0; i < n; ++i) {
+        plans_out[i] = plans[i];
+        if (budgets_out) budgets_out[i] = budgets[i];
+      }
+      return SWAPNET_OK;
+    } catch (const std::bad_alloc&) {
+      SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
     }
-    for (uint32_t i = 0; i < n; ++i) {
-      plans_out[i] = plans[i];
-      if (budgets_out) budgets_out[i] = budgets[i];
-    }
-    return SWAPNET_OK;
-  } catch (const std::bad_alloc&) {
-    SN_FAIL(SWAPNET_ERR_OOM, "host allocation failed");
-  }
+  });
 }
 
 }  // extern "C"

@@ -422,3 +422,13 @@ def test_swap_timing_calls_reject_a_null_engine_or_output():
     assert capi.lib().swapnet_engine_set_graph_timeline(None, 1) == capi.ERR_INVALID_ARG
     assert capi.lib().swapnet_engine_last_graph_timeline(None, us, 1) == capi.ERR_INVALID_ARG
     assert b"null" in capi.lib().swapnet_last_error()
+
+
+def test_status_strings_cover_every_code():
+    """Every status code has its own message (no code falls to 'unknown')."""
+    codes = [capi.OK, capi.ERR_INVALID_ARG, capi.ERR_INFEASIBLE, capi.ERR_OOM, capi.ERR_CUDA, capi.ERR_TIMEOUT,
+             capi.ERR_MISALIGNED, capi.ERR_UNSUPPORTED, capi.ERR_IO, capi.ERR_INTERNAL]
+    msgs = [capi.lib().swapnet_strerror(c) for c in codes]
+    assert len(set(msgs)) == len(codes)
+    assert capi.lib().swapnet_strerror(-100) == b"unknown status"
+    assert all(m != b"unknown status" for m in msgs)
