@@ -587,11 +587,20 @@ def test_degenerate_budgets_bit_exact():
 
 
 def _check_pipeline_order(tl, total_us):
+    """Swaps (those of this inference: start >= 0) one after another, each
+    block's layers after its own swap and the previous block's layers, a
+    swap after the layers of the block two back."""
     eps = 1.0                                   # event resolution, microseconds
     for k, (s0, s1, e0, e1) in enumerate(tl):
-        assert 0.0 <= s0 <= s1 + eps and s1 <= e0 + eps and e0 <= e1 + eps, (k, tl[k])
+        assert 0.0 <= e0 <= e1 + eps, (k, tl[k])
         if k:
-            assert tl[k - 1][3] <= e0 + eps and tl[k - 1][1] <= s0 + eps, (k, tl[k - 1], tl[k])
+            assert tl[k - 1][3] <= e0 + eps, (k, tl[k - 1], tl[k])
+        if s0 < 0:                              # not swapped in during this inference
+            assert s1 < 0
+            continue
+        assert s0 <= s1 + eps and s1 <= e0 + eps, (k, tl[k])
+        if k and tl[k - 1][1] >= 0:
+            assert tl[k - 1][1] <= s0 + eps, (k, tl[k - 1], tl[k])
         if k >= 2:
             assert tl[k - 2][3] <= s0 + eps, (k, tl[k - 2], tl[k])
     assert tl[-1][3] <= total_us + eps
@@ -667,4 +676,37 @@ def test_timing_follows_an_adapted_plan():
     _check_pipeline_order(sw.engine.last_graph_timeline(nb), a.elapsed_time(b) * 1e3)
     sw.engine.set_graph_timeline(False)
     sw.engine.set_swap_timing(False)
+    sw.engine.sync()
+
+
+def test_graph_timeline_with_first_block_prefetch():
+    """First-block prefetch: the first block was swapped in by the previous
+    inference, so the timeline reports no swap for it in this one (-1), and
+    the other blocks keep the pipeline order; outputs stay the resident bits
+    over back-to-back inferences."""
+    import torch
+    m = synth.arch.MODELS["resnet50"]()
+    w = synth.gen.model_weights(m)
+    d = capi.Desc(m)
+    host = capi.HostWeights(w)
+    plan = capi.Plan.partition(d, int(OP.weight_bytes(m) * 0.4) // 256 * 256, capi.options(prefetch=1))
+    nb = plan.info()["n_blocks"]
+    sw = Runner(m, w, plan, host)
+    x = synth.gen.model_input(m)
+    ref = Runner(m, w, capi.Plan.resident(d), host).run(x)
+    sw.engine.set_graph_timeline(True)
+    for _ in range(2):
+        assert sw.run(x)[0].tobytes() == ref[0].tobytes()
+    s = torch.cuda.current_stream()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(s)
+    sw.engine.infer(sw.d_in.data_ptr(), sw.d_out.data_ptr(), s.cuda_stream)
+    b.record(s)
+    b.synchronize()
+    tl = sw.engine.last_graph_timeline(nb)
+    assert tl[0][0] < 0 and tl[0][1] < 0
+    assert all(t[0] >= 0 for t in tl[1:])
+    _check_pipeline_order(tl, a.elapsed_time(b) * 1e3)
+    sw.engine.set_graph_timeline(False)
+    assert sw.outputs_raw()[0].tobytes() == ref[0].tobytes()
     sw.engine.sync()
