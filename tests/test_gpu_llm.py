@@ -475,3 +475,28 @@ def test_packed_variant_falls_back_for_other_types():
     s = sw.engine.stats()
     assert s["link_bytes"] == s["bytes_swapped"] or s["link_bytes"] >= 0.99 * s["bytes_swapped"]
     torch.cuda.synchronize()
+
+
+def test_packed_engine_adapts_between_budgets():
+    """A packed-swap decoder engine switched between two budgets with
+    swapnet_engine_adapt keeps its packed images (no new packing) and equals
+    the resident run bit for bit under both plans."""
+    sw = Decoder(prefill_tokens=16, budget_frac=0.7, layers=2, opts=dict(swap_variant=capi.SWAP_PACKED))
+    rs = Decoder(prefill_tokens=16, resident=True, host=sw.host, weights=sw.w, layers=2)
+    ids = synth.gen.model_input(sw.mp).reshape(-1)
+    base = rs.run(0, ids)
+    a = sw.run(0, ids)
+    assert a[0].tobytes() == base[0].tobytes()
+    plan, eng, info = sw.engines[0]
+    small = capi.Plan.partition(capi.Desc(sw.mp), int(OP.weight_bytes(sw.mp) * 0.35) // 256 * 256,
+                                capi.options(swap_variant=capi.SWAP_PACKED))
+    assert small.info()["n_blocks"] > info["n_blocks"]
+    eng.adapt(small)
+    sw.engines[0] = (small, eng, small.info())
+    sw.bufs[0] = (sw.bufs[0][0], sw.bufs[0][1], small.output_offsets())
+    assert any(b["variant"] == capi.SWAP_PACKED for b in eng.blocks())
+    rs.state.zero_()
+    sw.state.zero_()
+    b = sw.run(0, ids)
+    c = rs.run(0, ids)
+    assert b[0].tobytes() == c[0].tobytes() == base[0].tobytes()
