@@ -129,3 +129,22 @@ def test_window_at_the_ends_of_the_exponent_range():
     assert buf[0] == 0
     back, raw = _unpack(buf, n)
     assert np.array_equal(back, low) and raw == 0
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_round_trip_of_mixed_distributions(seed):
+    """Random mixtures: scaled normals of several widths, exact zeros,
+    subnormals, infinities and NaNs, in random proportions and positions;
+    every word comes back and the size matches the layout."""
+    r = np.random.default_rng(100 + seed)
+    chunks = int(r.integers(1, 9))
+    n = CHUNK * chunks
+    sigma = 10.0 ** r.uniform(-4, 1)
+    w = _bf16(r.normal(0.0, sigma, n))
+    for pattern, frac in ((0x0000, 1e-3), (0x8000, 1e-4), (0x0001, 1e-4), (0x7F80, 1e-5), (0x7FC1, 1e-5)):
+        pick = r.random(n) < frac * 10 ** r.uniform(-1, 1)
+        w[pick] = pattern
+    buf = capi.pack_bf16(w)
+    back, raw = _unpack(buf, n)
+    assert np.array_equal(back, w)
+    assert buf.size == _body_off(chunks) + chunks * BODY + raw * 2 * CHUNK
