@@ -359,9 +359,12 @@ typedef struct CUstream_st* swapnet_stream; /* a cudaStream_t; NULL = legacy def
  * engine and with every block on the zero-copy kernel, and keeps the
  * fastest; decoder models (attention layers, a bound state) take the
  * zero-copy kernel for every block, so that the engines of one model never
- * mix copy-engine and SM reads of their shared host weights.  A resident
- * plan copies all weights to the arena here.
- * Errors: INVALID_ARG, MISALIGNED, OOM, CUDA, UNSUPPORTED. */
+ * mix copy-engine and SM reads of their shared host weights.  With
+ * SWAPNET_SWAP_PACKED it packs every swapped bf16 tensor that packs (or
+ * takes the packed image another engine made of the same host tensor) and
+ * keeps a device table of the unpack jobs of each block.  A resident plan
+ * copies all weights to the arena here.
+ * Errors: INVALID_ARG, MISALIGNED, OOM, CUDA, UNSUPPORTED, INTERNAL. */
 int swapnet_load(const swapnet_plan* plan, const void* const* host_weights, uint32_t n_tensors,
                  void* d_arena, uint64_t arena_bytes, void* d_workspace, uint64_t workspace_bytes,
                  swapnet_engine** out_engine);
